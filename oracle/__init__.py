@@ -1,0 +1,271 @@
+"""CPU oracle for the FQT quantized backward pass (arXiv 2010.14298).
+
+TEST INFRASTRUCTURE ONLY.  Only the test suite, ``__graft_entry__.smoke()``
+and the CPU-baseline / reference leg of ``bench.py`` may import this package.
+The CUDA library never calls it, and it shares no code with that library:
+the arithmetic lives in ``fqt_oracle.c`` (plain C, one IEEE rounding per
+operation, no FMA contraction) and in the plain loops here.
+
+Every function cites the passage of the paper it restates:
+
+* ``quantize_grad``  -- PTQ (Sec. 3.3), PSQ (Sec. 4.1), BHQ (Sec. 4.2, App. D.4)
+* ``quantize_fwd``   -- deterministic 8-bit PTQ of X and W (Sec. 2.1, App. E)
+* ``dequant``        -- Eq. 9: Q(dH) = S^-1 (codes + z' 1^T)
+* ``grad_x``/``grad_w`` -- Eq. 6 with the bifurcation of App. E
+* ``int_gemm``       -- the exact integer contraction the low-bit kernels do
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "fqt_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libfqt_oracle.so")
+_lib = None
+_lock = threading.Lock()
+
+PTQ, PSQ, BHQ = 0, 1, 2
+STREAM_B2, STREAM_B1 = 0, 1
+
+
+def build(force: bool = False) -> str:
+    """Compile fqt_oracle.c into oracle/_build/libfqt_oracle.so with gcc."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math",
+           "-fPIC", "-shared", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        i64, u64, u32, i32 = (ctypes.c_int64, ctypes.c_uint64, ctypes.c_uint32,
+                              ctypes.c_int)
+        lib.orc_philox4x32_10.argtypes = [P, P, P]
+        lib.orc_philox4x32_10.restype = None
+        lib.orc_u16.argtypes = [u64, u32, u64]
+        lib.orc_u16.restype = u32
+        lib.orc_sr.argtypes = [ctypes.c_float, u32, u32]
+        lib.orc_sr.restype = u32
+        lib.orc_sr_moments.argtypes = [ctypes.c_float, u32, P, P]
+        lib.orc_sr_moments.restype = None
+        lib.orc_range.argtypes = [P, i64, P, P]
+        lib.orc_range.restype = i64
+        lib.orc_quantize_grad.argtypes = [P, i64, i64, i32, i32, i32, u64, u32,
+                                          P, P, P, P, P]
+        lib.orc_quantize_grad.restype = i64
+        lib.orc_quant_det.argtypes = [P, i64, i64, i32, P, P, P]
+        lib.orc_quant_det.restype = i64
+        lib.orc_householder.argtypes = [i32, i32, P]
+        lib.orc_householder.restype = None
+        lib.orc_bhq_scales.argtypes = [ctypes.c_double, ctypes.c_double, i32,
+                                       u32, P, P]
+        lib.orc_bhq_scales.restype = None
+        lib.orc_dequant.argtypes = [P, i64, i64, i32, i32, P, P, P, P]
+        lib.orc_dequant.restype = None
+        lib.orc_dequant_f64.argtypes = [P, i64, i64, i32, i32, P, P, P, P]
+        lib.orc_dequant_f64.restype = None
+        lib.orc_int_gemm.argtypes = [P, i32, P, i32, i64, i64, i64, i32, i32, P]
+        lib.orc_int_gemm.restype = None
+        lib.orc_matmul_f64.argtypes = [P, i32, P, i64, i64, i64, P]
+        lib.orc_matmul_f64.restype = None
+        _lib = lib
+        return lib
+
+
+def _ptr(a: np.ndarray):
+    return ctypes.c_void_p(a.ctypes.data) if a is not None else None
+
+
+def _f32(x) -> np.ndarray:
+    """fp32 C-contiguous copy of x (bf16 sources arrive already widened)."""
+    return np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+# --------------------------------------------------------------------------
+# Random numbers and stochastic rounding (Sec. 3.3 / App. D)
+# --------------------------------------------------------------------------
+def philox4x32_10(ctr, key) -> tuple:
+    """One Philox4x32-10 block (Salmon et al., SC'11)."""
+    lib = _load()
+    c = np.asarray(ctr, dtype=np.uint32)
+    k = np.asarray(key, dtype=np.uint32)
+    out = np.zeros(4, dtype=np.uint32)
+    lib.orc_philox4x32_10(_ptr(c), _ptr(k), _ptr(out))
+    return tuple(int(x) for x in out)
+
+
+def u16(seed: int, stream: int, idx: int) -> int:
+    return int(_load().orc_u16(seed, stream, idx))
+
+
+def sr(v: float, u: int, B: int) -> int:
+    """SR(v) for one fixed uniform u (Sec. 3.3)."""
+    return int(_load().orc_sr(float(v), int(u), int(B)))
+
+
+def sr_moments(v: float, B: int) -> tuple:
+    """Exact mean / variance of SR(v) by enumeration of every 16-bit uniform."""
+    lib = _load()
+    m = np.zeros(1)
+    var = np.zeros(1)
+    lib.orc_sr_moments(float(v), int(B), _ptr(m), _ptr(var))
+    return float(m[0]), float(var[0])
+
+
+# --------------------------------------------------------------------------
+# Quantizers
+# --------------------------------------------------------------------------
+def quantize_grad(dH, kind: int, bits: int, block: int = 0, seed: int = 0,
+                  stream: int = STREAM_B2, want_v: bool = False) -> dict:
+    """Gradient quantizer Q_b: PTQ (Sec. 3.3), PSQ (Sec. 4.1), BHQ (Sec. 4.2).
+
+    Returns codes (uint8, N x C), inv_s and zero (1 entry for PTQ, N otherwise),
+    lead (BHQ: lead row of each block) and, with want_v, the pre-rounding
+    values v that SR acts on.
+    """
+    h = _f32(dH)
+    n, c = h.shape
+    if kind == BHQ and block < 1:
+        raise OracleError("BHQ needs block >= 1")
+    codes = np.zeros((n, c), dtype=np.uint8)
+    m = 1 if kind == PTQ else n
+    inv_s = np.zeros(m, dtype=np.float32)
+    zero = np.zeros(m, dtype=np.float32)
+    nblk = (n + block - 1) // block if kind == BHQ else 0
+    lead = np.zeros(max(nblk, 1), dtype=np.int32)
+    v = np.zeros((n, c), dtype=np.float32) if want_v else None
+    bad = _load().orc_quantize_grad(_ptr(h), n, c, kind, bits, block, seed,
+                                    stream, _ptr(codes), _ptr(inv_s),
+                                    _ptr(zero), _ptr(lead), _ptr(v))
+    if bad:
+        raise OracleError(f"{bad} non-finite gradient entries")
+    out = dict(codes=codes, inv_s=inv_s, zero=zero, kind=kind, bits=bits,
+               block=block, lead=lead[:nblk] if kind == BHQ else None)
+    if want_v:
+        out["v"] = v
+    return out
+
+
+def quantize_fwd(X, bits: int = 8) -> dict:
+    """Deterministic PTQ of a forward operand, Q_f / Q_theta (Sec. 2.1, App. E)."""
+    x = _f32(X)
+    n, c = x.shape
+    codes = np.zeros((n, c), dtype=np.uint8)
+    inv_s = np.zeros(1, dtype=np.float32)
+    zero = np.zeros(1, dtype=np.float32)
+    bad = _load().orc_quant_det(_ptr(x), n, c, bits, _ptr(codes), _ptr(inv_s),
+                                _ptr(zero))
+    if bad:
+        raise OracleError(f"{bad} non-finite entries")
+    return dict(codes=codes, inv_s=inv_s, zero=zero, kind=PTQ, bits=bits,
+                block=0, lead=None)
+
+
+def householder(nb: int, p: int) -> np.ndarray:
+    """Q = I - 2 n n^T / ||n||^2, n = 1/sqrt(N) 1 - e_p (Sec. 4.2)."""
+    Q = np.zeros((nb, nb))
+    _load().orc_householder(nb, p, _ptr(Q))
+    return Q
+
+
+def bhq_scales(lambda1: float, lambda2: float, nb: int, B: int) -> tuple:
+    """s1, s2 of App. D.4 for one group of nb rows."""
+    s1 = np.zeros(1)
+    s2 = np.zeros(1)
+    _load().orc_bhq_scales(float(lambda1), float(lambda2), nb, B, _ptr(s1),
+                           _ptr(s2))
+    return float(s1[0]), float(s2[0])
+
+
+def dequant(q: dict, codes=None) -> np.ndarray:
+    """The value the encoding represents, Eq. 9: diag(inv_s) Q_blk (codes + z').
+
+    ``codes`` may be given as floats (e.g. expected codes); the map is affine
+    in them, so dequant(E[codes]) = E[dequant(codes)].
+    """
+    src = q["codes"] if codes is None else codes
+    lib = _load()
+    if np.asarray(src).dtype == np.uint8:
+        cd = np.ascontiguousarray(src, dtype=np.uint8)
+        fn = lib.orc_dequant
+    else:
+        cd = np.ascontiguousarray(src, dtype=np.float64)
+        fn = lib.orc_dequant_f64
+    n, c = cd.shape
+    out = np.zeros((n, c))
+    inv_s = np.ascontiguousarray(q["inv_s"], dtype=np.float32)
+    zero = np.ascontiguousarray(q["zero"], dtype=np.float32)
+    lead = (np.ascontiguousarray(q["lead"], dtype=np.int32)
+            if q.get("lead") is not None else np.zeros(1, dtype=np.int32))
+    fn(_ptr(cd), n, c, q["kind"], max(q.get("block", 0), 1), _ptr(inv_s),
+       _ptr(zero), _ptr(lead), _ptr(out))
+    return out
+
+
+# --------------------------------------------------------------------------
+# Contractions (Eq. 6, App. E)
+# --------------------------------------------------------------------------
+def int_gemm(A, a_kmajor: bool, Bm, b_kmajor: bool, M: int, N: int, K: int,
+             oa: int, ob: int) -> np.ndarray:
+    """P_ij = sum_k (A_ik - oa)(B_kj - ob), exact in int64."""
+    a = np.ascontiguousarray(A, dtype=np.uint8)
+    b = np.ascontiguousarray(Bm, dtype=np.uint8)
+    out = np.zeros((M, N), dtype=np.int64)
+    _load().orc_int_gemm(_ptr(a), int(a_kmajor), _ptr(b), int(b_kmajor), M, N,
+                         K, oa, ob, _ptr(out))
+    return out
+
+
+def matmul(A: np.ndarray, Bm: np.ndarray, a_trans: bool = False) -> np.ndarray:
+    """Plain double product op(A) @ Bm with op(A) = A or A^T."""
+    a = np.ascontiguousarray(A, dtype=np.float64)
+    b = np.ascontiguousarray(Bm, dtype=np.float64)
+    K, N = b.shape
+    M = a.shape[1] if a_trans else a.shape[0]
+    out = np.zeros((M, N))
+    _load().orc_matmul_f64(_ptr(a), int(a_trans), _ptr(b), M, K, N, _ptr(out))
+    return out
+
+
+def grad_x(q_b2: dict, q_w: dict, codes_b2=None) -> np.ndarray:
+    """grad_X = Q_b2(dH) W~ (Eq. 6 in the N x C, C x D layout; App. E)."""
+    return matmul(dequant(q_b2, codes_b2), dequant(q_w))
+
+
+def grad_w(q_b1: dict, q_x: dict, codes_b1=None) -> np.ndarray:
+    """grad_W = Q_b1(dH)^T X~ (C x D; the transpose of Eq. 6's D x C form)."""
+    return matmul(dequant(q_b1, codes_b1), dequant(q_x), a_trans=True)
+
+
+def linear_backward(dH, X, W, kind: int, bits: int, block: int, seed: int,
+                    reuse_b2: bool = False) -> dict:
+    """One FQT backward of a linear layer (Eq. 6 with App. E's bifurcation):
+    Q_b2 (kind, bits) feeds grad_X, 8-bit stochastic PTQ Q_b1 feeds grad_W,
+    X~ and W~ are the deterministic 8-bit forward codes."""
+    q_x = quantize_fwd(X, 8)
+    q_w = quantize_fwd(W, 8)
+    q_b2 = quantize_grad(dH, kind, bits, block, seed, STREAM_B2)
+    q_b1 = q_b2 if reuse_b2 else quantize_grad(dH, PTQ, 8, 0, seed, STREAM_B1)
+    return dict(q_x=q_x, q_w=q_w, q_b2=q_b2, q_b1=q_b1,
+                grad_x=grad_x(q_b2, q_w), grad_w=grad_w(q_b1, q_x))

@@ -1,0 +1,155 @@
+"""Seeded synthetic inputs shaped like the paper's workloads.
+
+This module holds no arithmetic of the method: it only draws the layer
+tensors (output gradient dH, layer input X, weight W) that both the CUDA
+library and the CPU oracle consume.  Draws use numpy's counter-based Philox
+bit generator keyed by the data seed, so a (config, seed, size) triple gives
+the same arrays on any machine.
+
+The paper trains on CIFAR10, ImageNet and IWSLT14 (Sec. 5), which are not
+available here.  The gradients below stand in for them: rows (samples) with
+sparse, heavy-tailed per-sample magnitudes, the structure Sec. 4.1 attributes
+to cross-entropy gradients of a well-fit network (most rows near zero, a few
+outliers).  Conv layers are lowered to a linear layer on im2col rows
+(Sec. 2.1), padding zeros included.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import List, Optional, Tuple
+
+import numpy as np
+
+PTQ, PSQ, BHQ = 0, 1, 2
+KIND_NAMES = {PTQ: "ptq", PSQ: "psq", BHQ: "bhq"}
+
+
+def rng(seed: int) -> np.random.Generator:
+    return np.random.Generator(np.random.Philox(key=seed))
+
+
+def to_bf16_values(x: np.ndarray) -> np.ndarray:
+    """Round fp32 values to the nearest bf16 (ties to even), kept in fp32.
+
+    Used for workloads whose source tensors are bf16: the GPU receives the
+    bf16 tensor, the oracle its exact fp32 widening.
+    """
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    lsb = (u >> 16) & 1
+    r = (u + 0x7FFF + lsb) & 0xFFFF0000
+    return r.astype(np.uint32).view(np.float32)
+
+
+def im2col_nhwc(x: np.ndarray, kh: int, kw: int, stride: int,
+                pad: int) -> np.ndarray:
+    """im2col of an NHWC tensor: rows (n, oh, ow), columns (kh, kw, cin)."""
+    n, h, w, c = x.shape
+    xp = np.pad(x, ((0, 0), (pad, pad), (pad, pad), (0, 0)))
+    oh = (h + 2 * pad - kh) // stride + 1
+    ow = (w + 2 * pad - kw) // stride + 1
+    cols = np.empty((n, oh, ow, kh, kw, c), dtype=x.dtype)
+    for i in range(kh):
+        for j in range(kw):
+            cols[:, :, :, i, j, :] = xp[:, i:i + stride * oh:stride,
+                                        j:j + stride * ow:stride, :]
+    return cols.reshape(n * oh * ow, kh * kw * c)
+
+
+@dataclasses.dataclass
+class Layer:
+    """One layer backward problem: dH (N x C), X (N x D), W (C x D)."""
+    name: str
+    dH: np.ndarray
+    X: np.ndarray
+    W: np.ndarray
+    dtype: str  # "f32" or "bf16": the source tensor type handed to the GPU
+    runs: List[Tuple[int, int, int]]  # (kind, bits, block) for Q_b2
+
+    @property
+    def N(self) -> int:
+        return self.dH.shape[0]
+
+    @property
+    def C(self) -> int:
+        return self.dH.shape[1]
+
+    @property
+    def D(self) -> int:
+        return self.X.shape[1]
+
+
+def _lognormal_rows(g: np.random.Generator, n: int, sigma: float) -> np.ndarray:
+    return np.exp(sigma * g.standard_normal(n)).astype(np.float32)
+
+
+CONFIG_NAMES = [
+    "linear-128x256",
+    "resnet18-conv3x3-b128-32x32-64ch",
+    "resnet50-layer3-conv3x3-b256-14x14-256ch",
+    "transformer-ffn-8192tok-1024x4096-bf16",
+]
+
+
+def config(index: int, batch: Optional[int] = None, rows: Optional[int] = None,
+           seed: Optional[int] = None) -> List[Layer]:
+    """Layers of workload `index` (0-based).
+
+    `batch` shrinks the image batch of the conv workloads and `rows` the
+    token / sample count of the others, keeping every other shape and the
+    value distributions, so the same recipe yields oracle-sized cases.
+    """
+    g = rng(1234 + index if seed is None else seed)
+    if index == 0:
+        n = rows or 128
+        dH = (g.standard_normal((n, 256)).astype(np.float32)
+              * _lognormal_rows(g, n, 2.0)[:, None])
+        X = g.uniform(-1, 1, (n, 256)).astype(np.float32)
+        W = (0.02 * g.standard_normal((256, 256))).astype(np.float32)
+        return [Layer(CONFIG_NAMES[0], dH, X, W, "f32",
+                      [(PTQ, 8, 0), (PSQ, 8, 0), (BHQ, 5, 16)])]
+    if index == 1:
+        b = batch or 128
+        x = g.uniform(-1, 1, (b, 32, 32, 64)).astype(np.float32)
+        X = im2col_nhwc(x, 3, 3, 1, 1)
+        n = X.shape[0]
+        dH = g.standard_normal((n, 64)).astype(np.float32)
+        big = g.random(n) < 0.01
+        dH[big] *= 100.0
+        W = (np.sqrt(2.0 / 576) * g.standard_normal((64, 576))).astype(np.float32)
+        runs = [(k, b_, 16 if k == BHQ else 0) for k in (PTQ, PSQ, BHQ)
+                for b_ in (4, 5, 8)]
+        return [Layer(CONFIG_NAMES[1], dH, X, W, "f32", runs)]
+    if index == 2:
+        b = batch or 256
+        x = g.uniform(-1, 1, (b, 14, 14, 256)).astype(np.float32)
+        X = im2col_nhwc(x, 3, 3, 1, 1)
+        n = X.shape[0]
+        dH = (g.standard_normal((n, 256)).astype(np.float32)
+              * _lognormal_rows(g, n, 2.5)[:, None])
+        W = (np.sqrt(2.0 / 2304) * g.standard_normal((256, 2304))).astype(np.float32)
+        return [Layer(CONFIG_NAMES[2], dH, X, W, "f32",
+                      [(BHQ, 5, nb) for nb in (8, 16, 32, 64)])]
+    if index == 3:
+        n = rows or 8192
+        out = []
+        for name, c, d in (("ffn-up", 4096, 1024), ("ffn-down", 1024, 4096)):
+            z = g.standard_normal((n, c)).astype(np.float32)
+            chi = g.chisquare(3, (n, c)).astype(np.float32)
+            t3 = z / np.sqrt(chi / 3.0)
+            dH = to_bf16_values(t3 * _lognormal_rows(g, n, 1.5)[:, None])
+            X = to_bf16_values(g.standard_normal((n, d)).astype(np.float32))
+            W = to_bf16_values((0.02 * g.standard_normal((c, d))).astype(np.float32))
+            out.append(Layer(f"{CONFIG_NAMES[3]}:{name}", dH, X, W, "bf16",
+                             [(PTQ, 8, 0), (PSQ, 5, 0), (BHQ, 5, 16)]))
+        return out
+    raise ValueError(f"no workload {index}")
+
+
+def random_grad(g: np.random.Generator, n: int, c: int, sigma: float = 2.0,
+                outlier_frac: float = 0.0) -> np.ndarray:
+    """Generic per-sample-scaled gradient for edge-case tests."""
+    dH = (g.standard_normal((n, c)).astype(np.float32)
+          * _lognormal_rows(g, n, sigma)[:, None])
+    if outlier_frac > 0:
+        dH[g.random(n) < outlier_frac] *= 100.0
+    return dH

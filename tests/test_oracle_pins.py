@@ -1,0 +1,417 @@
+"""Pins of the CPU oracle to what the paper and the mathematics fix.
+
+None of these tests calls the CUDA library.  Each one checks the oracle
+against something other than itself: published known answers, exact
+expectations by enumeration of every rounding outcome, the paper's variance
+expressions and bounds, the Householder identities, and special cases that
+reduce to another quantizer or to a library routine.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle as orc
+from paper_2010_14298_gb300 import workloads as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _moments(v: np.ndarray, B: int):
+    """Exact mean and variance of every code, by enumerating all uniforms."""
+    m = np.zeros(v.shape)
+    var = np.zeros(v.shape)
+    for idx in np.ndindex(v.shape):
+        m[idx], var[idx] = orc.sr_moments(float(v[idx]), B)
+    return m, var
+
+
+def _blocks(n, nb):
+    return [(r0, min(nb, n - r0)) for r0 in range(0, n, nb)]
+
+
+# --------------------------------------------------------------------------
+# Philox4x32-10 and the uniforms
+# --------------------------------------------------------------------------
+def test_philox_known_answers():
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "philox4x32_10_kat.txt"))
+            if l.strip() and not l.startswith("#")]
+    assert len(rows) == 3
+    for r in rows:
+        vals = [int(x, 16) for x in r]
+        assert orc.philox4x32_10(vals[:4], vals[4:6]) == tuple(vals[6:10])
+
+
+def test_uniform_layout_reads_the_philox_block():
+    seed, stream = 0x1234_5678_9ABC_DEF0, 1
+    for q in (0, 1, 77, 1 << 33):
+        w = orc.philox4x32_10([q & 0xFFFFFFFF, q >> 32, stream, 0],
+                              [seed & 0xFFFFFFFF, seed >> 32])
+        for i in range(8):
+            expect = (w[i // 2] >> (16 * (i % 2))) & 0xFFFF
+            assert orc.u16(seed, stream, 8 * q + i) == expect
+
+
+def test_uniforms_are_uniform_and_streams_distinct():
+    n = 1 << 16
+    a = np.array([orc.u16(7, 0, i) for i in range(n)])
+    b = np.array([orc.u16(7, 1, i) for i in range(n)])
+    for u in (a, b):
+        hist = np.bincount(u >> 10, minlength=64)
+        chi2 = ((hist - n / 64) ** 2 / (n / 64)).sum()
+        assert chi2 < 130  # df = 63; p(chi2 > 130) ~ 1e-6
+    assert abs(np.corrcoef(a, b)[0, 1]) < 0.02
+    assert (a != b).mean() > 0.99
+
+
+# --------------------------------------------------------------------------
+# Stochastic rounding (Sec. 3.3, App. D: E[SR(X)] = X, Var = p (1 - p))
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("v", [0.0, 0.25, 0.5, 1.0, 3.7, 12.999, 100.3125,
+                               254.5, 254.99, 255.0, 1e-7, 17.000001])
+def test_sr_moments_match_the_definition(v):
+    B = 255
+    m, var = orc.sr_moments(v, B)
+    v32 = float(np.float32(v))
+    assert v32 - 2.0 ** -16 <= m <= v32 + 1e-12
+    p = m - np.floor(v32)
+    assert var == pytest.approx(p * (1 - p), abs=1e-12)
+    assert var <= 0.25 + 1e-12
+    if v32 == np.floor(v32):
+        assert m == v32 and var == 0.0
+
+
+def test_sr_takes_only_floor_or_ceil():
+    rs = np.random.Generator(np.random.Philox(3))
+    for v in rs.uniform(0, 31, 200).astype(np.float32):
+        for u in (0, 1, 12345, 40000, 65535):
+            c = orc.sr(v, u, 31)
+            assert c in (np.floor(v), min(np.ceil(v), 31))
+
+
+# --------------------------------------------------------------------------
+# Unbiasedness of every quantizer, exactly (enumerating all outcomes)
+# --------------------------------------------------------------------------
+CASES = [(orc.PTQ, 4, 0), (orc.PTQ, 8, 0), (orc.PSQ, 3, 0), (orc.PSQ, 8, 0),
+         (orc.BHQ, 4, 4), (orc.BHQ, 5, 3), (orc.BHQ, 8, 8), (orc.BHQ, 2, 1)]
+
+
+@pytest.mark.parametrize("kind,bits,block", CASES)
+def test_quantizer_is_unbiased_exactly(kind, bits, block):
+    g = wl.rng(11 + kind * 10 + bits)
+    h = wl.random_grad(g, 8, 12, sigma=2.0, outlier_frac=0.2)
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, kind, bits, block, seed=5, want_v=True)
+    v = q["v"]
+    assert v.min() >= 0.0 and v.max() <= B * (1 + 1e-5)
+    m, _ = _moments(v, B)
+    e_deq = orc.dequant(q, m)
+    nb = block if kind == orc.BHQ else (1 if kind == orc.PSQ else 8)
+    for r0, n in _blocks(8, nb):
+        scale = np.abs(h[r0:r0 + n]).max()
+        err = np.abs(e_deq[r0:r0 + n] - h[r0:r0 + n]).max()
+        assert err <= 2e-5 * scale, (r0, err, scale)
+
+
+# --------------------------------------------------------------------------
+# Exact variance against the paper's expressions
+# --------------------------------------------------------------------------
+def _exact_var_of_dequant(q, var_codes):
+    """Var of each dequantized entry: diag(inv_s) Q_blk acts on independent codes."""
+    n, c = var_codes.shape
+    inv_s = q["inv_s"].astype(np.float64)
+    if q["kind"] == orc.PTQ:
+        return var_codes * inv_s[0] ** 2
+    if q["kind"] == orc.PSQ:
+        return var_codes * (inv_s ** 2)[:, None]
+    out = np.zeros((n, c))
+    for b, (r0, nb) in enumerate(_blocks(n, q["block"])):
+        Q = orc.householder(nb, int(q["lead"][b]))
+        W = (inv_s[r0:r0 + nb, None] * Q) ** 2
+        out[r0:r0 + nb] = W @ var_codes[r0:r0 + nb]
+    return out
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_ptq_variance_bound(bits):
+    g = wl.rng(21)
+    h = wl.random_grad(g, 6, 16)
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, orc.PTQ, bits, want_v=True)
+    _, var = _moments(q["v"], B)
+    total = _exact_var_of_dequant(q, var).sum()
+    R = float(h.max() - h.min())
+    assert total <= h.size * R * R / (4 * B * B) * (1 + 1e-5)  # Eq. 8
+    assert total > 0
+
+
+@pytest.mark.parametrize("bits", [3, 5])
+def test_psq_variance_bound_and_gain(bits):
+    g = wl.rng(22)
+    h = wl.random_grad(g, 8, 16, sigma=2.0)
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, orc.PSQ, bits, want_v=True)
+    _, var = _moments(q["v"], B)
+    total = _exact_var_of_dequant(q, var).sum()
+    Ri = h.max(axis=1) - h.min(axis=1)
+    bound = h.shape[1] / (4 * B * B) * (Ri.astype(np.float64) ** 2).sum()
+    assert total <= bound * (1 + 1e-5)  # Sec. 4.1 / App. D.3
+    qp = orc.quantize_grad(h, orc.PTQ, bits, want_v=True)
+    _, varp = _moments(qp["v"], B)
+    assert total < _exact_var_of_dequant(qp, varp).sum()  # PSQ below PTQ
+
+
+@pytest.mark.parametrize("nb,bits", [(4, 4), (8, 5), (16, 8)])
+def test_bhq_variance_bound(nb, bits):
+    g = wl.rng(23 + nb)
+    h = (1e-3 * g.standard_normal((2 * nb, 10))).astype(np.float32)
+    h[0] = 10.0 * g.standard_normal(10)
+    h[nb + 3] = 30.0 * g.standard_normal(10)
+    # one large row per block, lambda2 / lambda1 ~ 0: the case of Sec. 4.2
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, orc.BHQ, bits, nb, want_v=True)
+    _, var = _moments(q["v"], B)
+    vd = _exact_var_of_dequant(q, var)
+    D = h.shape[1]
+    for b, (r0, n) in enumerate(_blocks(h.shape[0], nb)):
+        blk = h[r0:r0 + n].astype(np.float64)
+        p = int(np.argmax(np.abs(blk).max(axis=1)))
+        assert p == q["lead"][b]
+        lam1 = blk[p].max() - blk[p].min()
+        lam2 = 2 * np.delete(np.abs(blk).max(axis=1), p).max()
+        inv_s = q["inv_s"][r0:r0 + n].astype(np.float64)
+        frob = (inv_s ** 2).sum()  # ||S^-1||_F^2, Q orthogonal
+        var_blk = vd[r0:r0 + n].sum()
+        assert var_blk <= D / 4 * frob * (1 + 1e-6)  # matrix-quantizer bound
+        hh = (lam1 ** (2 / 3) * n ** (-1 / 3) + lam2 ** (2 / 3) * n ** (2 / 3)) ** 3
+        assert frob <= hh / B ** 2 * (1 + 1e-5)  # App. D.4
+    # in this regime BHQ has lower variance than PSQ (Sec. 4.2)
+    qs = orc.quantize_grad(h, orc.PSQ, bits, want_v=True)
+    _, vs = _moments(qs["v"], B)
+    assert vd.sum() < _exact_var_of_dequant(qs, vs).sum()
+
+
+def test_fewer_bits_cost_about_4x_variance():
+    g = wl.rng(24)
+    h = g.standard_normal((16, 32)).astype(np.float32)
+    tot = {}
+    for bits in (4, 5, 6):
+        q = orc.quantize_grad(h, orc.PTQ, bits, want_v=True)
+        _, var = _moments(q["v"], (1 << bits) - 1)
+        tot[bits] = _exact_var_of_dequant(q, var).sum()
+    for b in (5, 6):
+        expect = (((1 << b) - 1) / ((1 << (b - 1)) - 1)) ** 2  # Sec. 3.3
+        assert tot[b - 1] / tot[b] == pytest.approx(expect, rel=0.2)
+
+
+# --------------------------------------------------------------------------
+# Householder reflection and the BHQ construction (Sec. 4.2, App. D.4)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("nb,p", [(2, 0), (3, 2), (8, 5), (16, 0), (64, 63)])
+def test_householder_identities(nb, p):
+    Q = orc.householder(nb, p)
+    assert np.allclose(Q @ Q.T, np.eye(nb), atol=1e-12)
+    assert np.allclose(Q, Q.T, atol=1e-15)
+    e = np.zeros(nb)
+    e[p] = 1.0
+    assert np.allclose(Q @ e, np.ones(nb) / np.sqrt(nb), atol=1e-12)
+    x = np.random.Generator(np.random.Philox(nb)).standard_normal(nb)
+    assert np.linalg.norm(Q @ x) == pytest.approx(np.linalg.norm(x), rel=1e-12)
+
+
+def test_householder_single_row_is_identity():
+    assert np.array_equal(orc.householder(1, 0), np.eye(1))
+
+
+@pytest.mark.parametrize("lam1,lam2,nb", [(10.0, 0.1, 16), (1.0, 1.0, 8),
+                                           (3.0, 1e-4, 64), (2.0, 0.5, 2)])
+def test_bhq_scales_solve_the_constrained_problem(lam1, lam2, nb):
+    B = 31
+    s1, s2 = orc.bhq_scales(lam1, lam2, nb, B)
+    # The range constraint of App. D.4 holds with equality ...
+    assert lam1 * s1 / np.sqrt(nb) + lam2 * s2 * np.sqrt(nb) == pytest.approx(B)
+    # ... and s1, s2 minimise s1^-2 + N s2^-2 along it.
+    f = lambda a: a ** -2 + nb * ((B - lam1 * a / np.sqrt(nb)) / (lam2 * np.sqrt(nb))) ** -2
+    for eps in (1e-3, -1e-3):
+        assert f(s1 * (1 + eps)) > f(s1)
+    # and the objective equals the closed form of App. D.4.
+    hh = (lam1 ** (2 / 3) * nb ** (-1 / 3) + lam2 ** (2 / 3) * nb ** (2 / 3)) ** 3
+    assert s1 ** -2 + nb * s2 ** -2 == pytest.approx(hh / B ** 2, rel=1e-12)
+
+
+def test_bhq_range_stays_within_B():
+    g = wl.rng(31)
+    for trial in range(20):
+        nb = [2, 4, 8, 16, 32, 64][trial % 6]
+        h = wl.random_grad(g, 4 * nb + 3, 24, sigma=2.5, outlier_frac=0.05)
+        for bits in (2, 5, 8):
+            q = orc.quantize_grad(h, orc.BHQ, bits, nb, want_v=True)
+            B = (1 << bits) - 1
+            assert q["v"].min() >= 0.0
+            assert q["v"].max() <= B * (1 + 1e-5)
+
+
+def test_bhq_degenerate_blocks():
+    h = np.zeros((12, 8), dtype=np.float32)
+    h[4] = 3.0  # constant lead row, lambda1 = 0, lambda2 = 0
+    h[9] = np.linspace(-1, 2, 8)  # single live row in its block
+    q = orc.quantize_grad(h, orc.BHQ, 5, 4)
+    assert (q["codes"][:4] == 0).all() and (q["inv_s"][:4] == 0).all()
+    assert q["lead"].tolist() == [0, 0, 1]
+    deq = orc.dequant(q)
+    assert np.abs(deq - h).max() <= (3.0 / 31) + 1e-6
+    assert np.allclose(deq[:4], 0.0)
+    # rows that are zero dequantize to zero exactly (inv_s = 0)
+    assert (q["inv_s"][[5, 6, 7, 8, 10, 11]] == 0).all()
+
+
+def test_bhq_block_one_matches_psq():
+    g = wl.rng(32)
+    h = wl.random_grad(g, 64, 64)
+    a = orc.quantize_grad(h, orc.BHQ, 5, 1, seed=9)
+    b = orc.quantize_grad(h, orc.PSQ, 5, seed=9)
+    diff = a["codes"].astype(int) - b["codes"].astype(int)
+    assert (diff == 0).mean() > 0.999 and np.abs(diff).max() <= 1
+    assert np.allclose(a["inv_s"], b["inv_s"], rtol=1e-6)
+
+
+def test_psq_reduces_to_ptq_when_rows_share_a_range():
+    g = wl.rng(33)
+    base = g.standard_normal(32).astype(np.float32)
+    h = np.stack([g.permutation(base) for _ in range(10)])
+    a = orc.quantize_grad(h, orc.PSQ, 5, seed=4)
+    b = orc.quantize_grad(h, orc.PTQ, 5, seed=4)
+    assert np.array_equal(a["codes"], b["codes"])  # S = s I (Eq. 9 remark)
+    assert np.all(a["inv_s"] == b["inv_s"][0]) and np.all(a["zero"] == b["zero"][0])
+
+
+def test_constant_and_zero_rows():
+    h = np.zeros((4, 16), dtype=np.float32)
+    h[1] = 2.5
+    h[2] = np.arange(16)
+    for kind in (orc.PTQ, orc.PSQ):
+        q = orc.quantize_grad(h, kind, 4)
+        deq = orc.dequant(q)
+        if kind == orc.PSQ:
+            assert np.array_equal(q["codes"][:2], np.zeros((2, 16)))
+            assert np.allclose(deq[:2], h[:2])
+
+
+# --------------------------------------------------------------------------
+# Deterministic forward quantizer (Sec. 2.1, App. E)
+# --------------------------------------------------------------------------
+def test_forward_quantizer_rounds_half_to_even():
+    x = np.array([[0.0, 0.5, 1.5, 2.5, 3.5, 254.5, 255.0, 7.49]], dtype=np.float32)
+    q = orc.quantize_fwd(x, 8)  # min 0, max 255 -> s = 1
+    assert q["inv_s"][0] == 1.0
+    assert q["codes"].tolist() == [[0, 0, 2, 2, 4, 254, 255, 7]]
+
+
+def test_forward_quantizer_error_is_half_a_bin():
+    g = wl.rng(34)
+    x = g.uniform(-3, 5, (40, 50)).astype(np.float32)
+    q = orc.quantize_fwd(x, 8)
+    deq = orc.dequant(q)
+    assert q["codes"].min() == 0 and q["codes"].max() == 255
+    assert np.abs(deq - x).max() <= 0.5 * q["inv_s"][0] * (1 + 1e-4) + 1e-6
+
+
+# --------------------------------------------------------------------------
+# Contractions: integer GEMM and Thm 1
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("ak,bk", [(1, 0), (0, 0), (1, 1), (0, 1)])
+def test_int_gemm_matches_numpy(ak, bk):
+    g = wl.rng(41)
+    M, N, K = 7, 9, 33
+    A = g.integers(0, 256, (M, K)).astype(np.uint8)
+    Bm = g.integers(0, 32, (K, N)).astype(np.uint8)
+    a_st = A if ak else A.T.copy()
+    b_st = Bm.T.copy() if bk else Bm
+    P = orc.int_gemm(a_st, ak, b_st, bk, M, N, K, 128, 16)
+    ref = (A.astype(np.int64) - 128) @ (Bm.astype(np.int64) - 16)
+    assert np.array_equal(P, ref)
+
+
+def test_matmul_matches_numpy():
+    g = wl.rng(42)
+    A = g.standard_normal((5, 7))
+    Bm = g.standard_normal((7, 3))
+    assert np.allclose(orc.matmul(A, Bm), A @ Bm, rtol=1e-13)
+    assert np.allclose(orc.matmul(A.T.copy(), Bm, a_trans=True), A @ Bm, rtol=1e-13)
+
+
+@pytest.mark.parametrize("kind,bits,block", [(orc.PTQ, 5, 0), (orc.PSQ, 4, 0),
+                                             (orc.BHQ, 5, 4)])
+def test_fqt_gradients_are_unbiased_exactly(kind, bits, block):
+    """Thm 1: E[FQT gradient | batch] = QAT gradient, for both contractions."""
+    g = wl.rng(51)
+    dH = wl.random_grad(g, 8, 10, outlier_frac=0.25)
+    X = g.uniform(-1, 1, (8, 6)).astype(np.float32)
+    W = (0.3 * g.standard_normal((10, 6))).astype(np.float32)
+    qx, qw = orc.quantize_fwd(X), orc.quantize_fwd(W)
+    q2 = orc.quantize_grad(dH, kind, bits, block, want_v=True)
+    q1 = orc.quantize_grad(dH, orc.PTQ, 8, 0, stream=orc.STREAM_B1, want_v=True)
+    m2, _ = _moments(q2["v"], (1 << bits) - 1)
+    m1, _ = _moments(q1["v"], 255)
+    Wt, Xt = orc.dequant(qw), orc.dequant(qx)
+    e_gx = orc.matmul(orc.dequant(q2, m2), Wt)
+    e_gw = orc.matmul(orc.dequant(q1, m1), Xt, a_trans=True)
+    qat_gx = dH.astype(np.float64) @ Wt
+    qat_gw = dH.astype(np.float64).T @ Xt
+    assert np.abs(e_gx - qat_gx).max() <= 1e-4 * np.abs(qat_gx).max()
+    assert np.abs(e_gw - qat_gw).max() <= 1e-4 * np.abs(qat_gw).max()
+    # and a single draw is what grad_x / grad_w return
+    assert np.allclose(orc.grad_x(q2, qw), orc.matmul(orc.dequant(q2), Wt))
+
+
+@pytest.mark.parametrize("kind,bits,block", [(orc.PSQ, 4, 0), (orc.BHQ, 4, 8)])
+def test_monte_carlo_mean_and_variance(kind, bits, block):
+    """Over many seeds: per-entry z-scores of the mean, total variance and the
+    variance of grad_X (Prop. 3's equality form, independent codes)."""
+    g = wl.rng(61)
+    h = wl.random_grad(g, 16, 32, outlier_frac=0.1)
+    W = (0.5 * g.standard_normal((32, 8))).astype(np.float32)
+    B = (1 << bits) - 1
+    q0 = orc.quantize_grad(h, kind, bits, block, want_v=True)
+    _, var_codes = _moments(q0["v"], B)
+    vd = _exact_var_of_dequant(q0, var_codes)
+    Wt = orc.dequant(orc.quantize_fwd(W))
+    K = 768
+    s1 = np.zeros(h.shape)
+    s2 = np.zeros(h.shape)
+    gx = []
+    for seed in range(K):
+        q = orc.quantize_grad(h, kind, bits, block, seed=seed + 1000)
+        d = orc.dequant(q)
+        s1 += d
+        s2 += d * d
+        gx.append(d @ Wt)
+    mean = s1 / K
+    emp_var = s2 / K - mean ** 2
+    live = vd > 0
+    z = (mean - h)[live] / np.sqrt(vd[live] / K)
+    assert np.abs(z).max() < 5.5
+    assert emp_var.sum() / vd.sum() == pytest.approx(1.0, rel=0.1)
+    gx = np.array(gx)
+    # exact Var[grad_X] from the independent per-code variances
+    n = h.shape[0]
+    inv_s = q0["inv_s"].astype(np.float64)
+    if kind == orc.PSQ:
+        var_gx = ((inv_s ** 2)[:, None] * var_codes) @ (Wt ** 2)
+    else:
+        var_gx = np.zeros((n, Wt.shape[1]))
+        for b, (r0, nbk) in enumerate(_blocks(n, block)):
+            Q = orc.householder(nbk, int(q0["lead"][b]))
+            A = inv_s[r0:r0 + nbk, None] * Q
+            var_gx[r0:r0 + nbk] = (A ** 2) @ (var_codes[r0:r0 + nbk] @ (Wt ** 2))
+    assert gx.var(axis=0).sum() / var_gx.sum() == pytest.approx(1.0, rel=0.12)
+
+
+def test_linear_backward_shapes_and_bifurcation():
+    L = wl.config(0, rows=16)[0]
+    out = orc.linear_backward(L.dH, L.X, L.W, orc.BHQ, 5, 16, seed=0)
+    assert out["grad_x"].shape == (16, 256) and out["grad_w"].shape == (256, 256)
+    assert out["q_b1"]["bits"] == 8 and out["q_b1"]["kind"] == orc.PTQ
+    # stream 1 draws differ from stream 0 draws
+    q2p = orc.quantize_grad(L.dH, orc.PTQ, 8, 0, seed=0, stream=0)
+    assert not np.array_equal(q2p["codes"], out["q_b1"]["codes"])
