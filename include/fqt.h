@@ -1,0 +1,157 @@
+/*
+ * fqt.h -- C ABI of the GB300 library for the quantized backward pass of one
+ * linear (or im2col-lowered conv) layer under fully quantized training (FQT),
+ * "A Statistical Framework for Low-bitwidth Training of Deep Neural
+ * Networks" (Chen, Gai, Yao, Mahoney, Gonzalez, NeurIPS 2020).
+ *
+ * Notation (PyTorch layout): dH is N x C (N samples / tokens / im2col rows,
+ * C output features), X is N x D, W is C x D (out x in).  The paper's
+ * Theta is W^T, so its grad_Theta = X~^T Q(dH) (Eq. 6) is the transpose of
+ * grad_W returned here.  b = bits, B = 2^b - 1.
+ *
+ * Conventions for every entry point:
+ *  - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *    allocates nothing.  `stream` is a cudaStream_t passed as void* (NULL =
+ *    the legacy default stream).  Work is enqueued on `stream` and the call
+ *    returns without synchronising.
+ *  - Argument errors are returned synchronously and enqueue nothing.
+ *    Conditions found on the device (non-finite input, a wait that ran out)
+ *    are recorded in the status word at the start of the workspace and are
+ *    returned by fqt_sync_status().
+ *  - `workspace` is caller-owned device memory of at least
+ *    fqt_workspace_size() bytes, 256-byte aligned and zero-filled before its
+ *    first use.  Calls that share a workspace must be ordered (same stream
+ *    or synchronised); concurrent calls need separate workspaces.
+ *  - Outputs depend only on the inputs and the seed, not on the launch
+ *    configuration.  Alignment: every pointer 16-byte aligned; quantizer
+ *    inputs need cols % 8 == 0; GEMM operands need cols % 16 == 0.
+ */
+#ifndef FQT_H_
+#define FQT_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FQT_API __attribute__((visibility("default")))
+#else
+#define FQT_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FQT_OK = 0,
+  FQT_EINVAL = 1,          /* bad argument: null pointer, size, bits, layout */
+  FQT_EUNSUPPORTED = 2,    /* valid request this build does not implement */
+  FQT_ECUDA = 3,           /* a CUDA runtime / driver call failed */
+  FQT_ENONFINITE = 4,      /* input held NaN or Inf (device-side) */
+  FQT_ETIMEOUT = 5,        /* a bounded device-side wait gave up */
+  FQT_EWORKSPACE = 6       /* workspace missing, misaligned or too small */
+} fqt_status;
+
+typedef enum { FQT_PTQ = 0, FQT_PSQ = 1, FQT_BHQ = 2 } fqt_kind;
+typedef enum { FQT_F32 = 0, FQT_BF16 = 1 } fqt_dtype;
+
+/*
+ * A quantized matrix: the encoding of Eq. 9 (Sec. 4),
+ *     value = S^-1 (codes + z' 1^T) = diag(inv_s) Q_blk (codes + z' 1^T),
+ * with Q_blk = I for PTQ (Sec. 3.3) and PSQ (Sec. 4.1), and for BHQ
+ * (Sec. 4.2) the block-diagonal Householder reflections
+ * Q = I - 2 n n^T / ||n||^2, n = 1/sqrt(nb) 1 - e_p, one per block of
+ * `block` consecutive rows (nb = rows of that block, p = its lead row).
+ *
+ * The caller allocates every array (device memory) and sets the pointers;
+ * the quantize calls fill rows, cols, bits, kind and block.
+ */
+typedef struct fqt_qtensor {
+  int64_t rows, cols;
+  int32_t bits;      /* b in [2, 8] */
+  int32_t kind;      /* fqt_kind */
+  int32_t block;     /* BHQ rows per block (power of two, <= 128); else 0 */
+  int32_t reserved;
+  uint8_t *codes;    /* rows x cols, row-major, values in [0, 2^b - 1] */
+  float *inv_s;      /* PTQ: 1 entry; PSQ, BHQ: rows entries (1/s_i; BHQ rows
+                        of a block whose other rows are all zero hold 0) */
+  float *zero;       /* same count: z' in the scaled / transformed domain */
+  int32_t *row_sum;  /* rows entries: sum_j codes_ij, or NULL (not computed) */
+  int32_t *col_sum;  /* cols entries: sum_i codes_ij, or NULL (not computed) */
+  int32_t *lead;     /* BHQ: ceil(rows / block) entries, lead row offset p
+                        within each block; else unused (may be NULL) */
+} fqt_qtensor;
+
+/* Bytes of workspace a layer with dH N x C, X N x D, W C x D needs for any
+ * call below (quantizers and backward). */
+FQT_API size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D);
+
+/*
+ * Deterministic 8-bit (or `bits`-bit) PTQ of a forward operand, the
+ * activation quantizer Q_f of Eq. 3 and App. E: z = min X, s = B / R(X),
+ * codes = round_half_even(s (X - z)) (Sec. 2.1).  X: rows x cols, row-major,
+ * fp32 or bf16.  Fills out->codes, inv_s[0], zero[0] and, when non-NULL,
+ * row_sum and col_sum.
+ */
+FQT_API fqt_status fqt_quantize_act(const void *X, fqt_dtype dtype, int64_t rows,
+                            int64_t cols, int bits, fqt_qtensor *out,
+                            void *workspace, size_t ws_bytes, void *stream);
+
+/* The same quantizer for the weight, Q_theta of Eq. 3 (W: C x D). */
+FQT_API fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t rows,
+                               int64_t cols, int bits, fqt_qtensor *out,
+                               void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Gradient quantizers with unbiased stochastic rounding (Sec. 3.3, 4.1, 4.2)
+ * and the bifurcation of App. E:
+ *   q_b2 <- Q_b2(dH): kind (PTQ, PSQ, BHQ), `bits`, BHQ `block`; feeds grad_X.
+ *   q_b1 <- Q_b1(dH): 8-bit stochastic PTQ; feeds grad_W.  May be NULL.
+ * SR draws 16-bit uniforms from Philox4x32-10 keyed by `seed`, counter
+ * (flat_index / 8, stream, 0), stream 0 for q_b2 and 1 for q_b1.
+ * dH: N x C row-major, fp32 or bf16, C % 8 == 0.  BHQ: block a power of
+ * two <= 128 and block * C <= 65536.
+ */
+FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
+                             int64_t C, fqt_kind kind, int bits, int block,
+                             uint64_t seed, fqt_qtensor *q_b2,
+                             fqt_qtensor *q_b1, void *workspace,
+                             size_t ws_bytes, void *stream);
+
+/*
+ * The two low-bit contractions of Eq. 6 with App. E's bifurcation:
+ *   grad_X = Q_b2(dH) W~          (N x D, fp32, row-major; may be NULL)
+ *   grad_W = Q_b1(dH)^T X~        (C x D, fp32, row-major; may be NULL)
+ * The integer products of the codes are exact; dequantization and, for BHQ,
+ * the inverse Householder transform of each block are applied in the
+ * epilogue.  Needs q_b2->row_sum, qw->col_sum (grad_X) and q_b1->col_sum,
+ * qx->col_sum (grad_W).  q_b1 may be NULL when q_b2 is PTQ with col_sum
+ * set: grad_W then uses q_b2.  C % 16 == 0 and D % 16 == 0.
+ */
+FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,
+                               const fqt_qtensor *q_b1,
+                               const fqt_qtensor *qx, const fqt_qtensor *qw,
+                               float *grad_X, float *grad_W, void *workspace,
+                               size_t ws_bytes, void *stream);
+
+/* Synchronises `stream`, returns the first device-side condition recorded in
+ * `workspace` since the previous call (or FQT_OK) and clears it. */
+FQT_API fqt_status fqt_sync_status(void *workspace, void *stream);
+
+/* Exact integer contraction, for bit-exact tests of the GEMM core:
+ *   out_ij = sum_k (A_ik - 2^(a_bits-1)) (B_kj - 2^(b_bits-1))   (int64)
+ * A is M x K, stored row-major (a_kmajor = 1) or as its K x M transpose;
+ * B is K x N, stored as K x N row-major (b_kmajor = 0) or as N x K. */
+FQT_API fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
+                              const uint8_t *Bm, int b_kmajor, int b_bits,
+                              int64_t M, int64_t N, int64_t K, int64_t *out,
+                              void *workspace, size_t ws_bytes, void *stream);
+
+/* Static description of a status code. */
+FQT_API const char *fqt_status_string(fqt_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FQT_H_ */

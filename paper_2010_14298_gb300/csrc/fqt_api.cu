@@ -1,0 +1,227 @@
+// fqt_api.cu -- the extern "C" entry points of include/fqt.h: argument
+// validation, workspace carving, launches, and the device status word.
+#include <cuda_runtime.h>
+#include <string.h>
+
+#include "fqt.h"
+#include "fqt_common.cuh"
+#include "fqt_internal.h"
+
+namespace fqt {
+
+int device_sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 148;
+  if (dev < 64 && cached[dev]) return cached[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    n = 148;
+  if (dev < 64) cached[dev] = n;
+  return n;
+}
+
+static bool aligned(const void *p, size_t a) {
+  return (reinterpret_cast<uintptr_t>(p) % a) == 0;
+}
+
+static fqt_status check_ws(void *ws, size_t bytes, size_t need) {
+  if (!ws || !aligned(ws, 256) || bytes < need) return FQT_EWORKSPACE;
+  return FQT_OK;
+}
+
+// Deterministic PTQ of a forward operand (Q_f / Q_theta).
+static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
+                                   int64_t cols, int bits, fqt_qtensor *out,
+                                   void *ws, size_t ws_bytes, void *stream) {
+  if (rows < 0 || cols <= 0 || cols > (1 << 20) || bits < 2 || bits > 8) return FQT_EINVAL;
+  if (!out) return FQT_EINVAL;
+  if (rows > 0 && (!X || !out->codes || !out->inv_s || !out->zero)) return FQT_EINVAL;
+  if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
+  if (cols % 8) return FQT_EUNSUPPORTED;
+  if (!aligned(X, 16) || !aligned(out->codes, 16)) return FQT_EINVAL;
+  fqt_status s = check_ws(ws, ws_bytes, kGemmOffset);
+  if (s != FQT_OK) return s;
+  out->rows = rows;
+  out->cols = cols;
+  out->bits = bits;
+  out->kind = FQT_PTQ;
+  out->block = 0;
+  if (rows == 0) return FQT_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int nsm = device_sm_count();
+  char *w = static_cast<char *>(ws);
+  float2 *part = reinterpret_cast<float2 *>(w + kRangeOffset);
+  int npart = 0;
+  cudaError_t e = launch_range(X, dtype == FQT_BF16, rows * cols, part, &npart,
+                               out->col_sum, out->col_sum ? cols : 0, nullptr, 0,
+                               nsm, st);
+  if (e != cudaSuccess) return FQT_ECUDA;
+  QuantArgs a;
+  memset(&a, 0, sizeof(a));
+  a.h = X;
+  a.N = rows;
+  a.C = (int)cols;
+  a.kind = KIND_DET;
+  a.bits = bits;
+  a.block = 0;
+  a.c2 = out->codes;
+  a.inv2 = out->inv_s;
+  a.zero2 = out->zero;
+  a.rsum2 = out->row_sum;
+  a.csum2 = out->col_sum;
+  a.part = part;
+  a.npart = npart;
+  a.status = reinterpret_cast<int *>(w);
+  int nth, grid;
+  size_t smem;
+  s = quant_geometry(a, nsm, &nth, &grid, &smem);
+  if (s != FQT_OK) return s;
+  e = launch_quant(a, dtype == FQT_BF16, nth, grid, smem, st);
+  return e == cudaSuccess ? FQT_OK : FQT_ECUDA;
+}
+
+}  // namespace fqt
+
+using namespace fqt;
+
+extern "C" {
+
+size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
+  return kGemmOffset + gemm_workspace_bytes(N, C, D);
+}
+
+fqt_status fqt_quantize_act(const void *X, fqt_dtype dtype, int64_t rows,
+                            int64_t cols, int bits, fqt_qtensor *out,
+                            void *workspace, size_t ws_bytes, void *stream) {
+  return quantize_forward(X, dtype, rows, cols, bits, out, workspace, ws_bytes,
+                          stream);
+}
+
+fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t rows,
+                               int64_t cols, int bits, fqt_qtensor *out,
+                               void *workspace, size_t ws_bytes, void *stream) {
+  return quantize_forward(W, dtype, rows, cols, bits, out, workspace, ws_bytes,
+                          stream);
+}
+
+fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
+                             int64_t C, fqt_kind kind, int bits, int block,
+                             uint64_t seed, fqt_qtensor *q_b2,
+                             fqt_qtensor *q_b1, void *workspace,
+                             size_t ws_bytes, void *stream) {
+  if (N < 0 || C <= 0 || C > (1 << 20) || bits < 2 || bits > 8) return FQT_EINVAL;
+  if (!q_b2) return FQT_EINVAL;
+  // an empty batch has nothing to read or write (its tensors may be NULL)
+  if (N > 0 && (!dH || !q_b2->codes || !q_b2->inv_s || !q_b2->zero)) return FQT_EINVAL;
+  if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
+  if (kind != FQT_PTQ && kind != FQT_PSQ && kind != FQT_BHQ) return FQT_EINVAL;
+  if (kind == FQT_BHQ) {
+    if (block < 1 || block > 128 || (block & (block - 1))) return FQT_EINVAL;
+    if (N > 0 && !q_b2->lead) return FQT_EINVAL;
+  } else {
+    block = 0;
+  }
+  if (N > 0 && q_b1 && (!q_b1->codes || !q_b1->inv_s || !q_b1->zero)) return FQT_EINVAL;
+  if (C % 8) return FQT_EUNSUPPORTED;
+  if (!aligned(dH, 16) || !aligned(q_b2->codes, 16) || (q_b1 && !aligned(q_b1->codes, 16)))
+    return FQT_EINVAL;
+  fqt_status s = check_ws(workspace, ws_bytes, kGemmOffset);
+  if (s != FQT_OK) return s;
+  q_b2->rows = N;
+  q_b2->cols = C;
+  q_b2->bits = bits;
+  q_b2->kind = kind;
+  q_b2->block = block;
+  if (q_b1) {
+    q_b1->rows = N;
+    q_b1->cols = C;
+    q_b1->bits = 8;
+    q_b1->kind = FQT_PTQ;
+    q_b1->block = 0;
+  }
+  if (N == 0) return FQT_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int nsm = device_sm_count();
+  char *w = static_cast<char *>(workspace);
+  float2 *part = reinterpret_cast<float2 *>(w + kRangeOffset);
+  int npart = 0;
+  int32_t *csum = q_b1 ? q_b1->col_sum : q_b2->col_sum;
+  cudaError_t e = launch_range(dH, dtype == FQT_BF16, N * C, part, &npart, csum,
+                               csum ? C : 0, nullptr, 0, nsm, st);
+  if (e != cudaSuccess) return FQT_ECUDA;
+  QuantArgs a;
+  memset(&a, 0, sizeof(a));
+  a.h = dH;
+  a.N = N;
+  a.C = (int)C;
+  a.kind = (int)kind;
+  a.bits = bits;
+  a.block = block;
+  a.key0 = (uint32_t)seed;
+  a.key1 = (uint32_t)(seed >> 32);
+  a.c2 = q_b2->codes;
+  a.inv2 = q_b2->inv_s;
+  a.zero2 = q_b2->zero;
+  a.rsum2 = q_b2->row_sum;
+  a.csum2 = q_b1 ? nullptr : q_b2->col_sum;
+  a.lead2 = q_b2->lead;
+  if (q_b1) {
+    a.c1 = q_b1->codes;
+    a.inv1 = q_b1->inv_s;
+    a.zero1 = q_b1->zero;
+    a.rsum1 = q_b1->row_sum;
+    a.csum1 = q_b1->col_sum;
+  }
+  a.part = part;
+  a.npart = npart;
+  a.status = reinterpret_cast<int *>(w);
+  int nth, grid;
+  size_t smem;
+  s = quant_geometry(a, nsm, &nth, &grid, &smem);
+  if (s != FQT_OK) return s;
+  e = launch_quant(a, dtype == FQT_BF16, nth, grid, smem, st);
+  return e == cudaSuccess ? FQT_OK : FQT_ECUDA;
+}
+
+fqt_status fqt_linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
+                               const fqt_qtensor *qx, const fqt_qtensor *qw,
+                               float *grad_X, float *grad_W, void *workspace,
+                               size_t ws_bytes, void *stream) {
+  return linear_backward(q_b2, q_b1, qx, qw, grad_X, grad_W, workspace, ws_bytes,
+                         reinterpret_cast<cudaStream_t>(stream));
+}
+
+fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
+                              const uint8_t *Bm, int b_kmajor, int b_bits,
+                              int64_t M, int64_t N, int64_t K, int64_t *out,
+                              void *workspace, size_t ws_bytes, void *stream) {
+  return debug_int_gemm(A, a_kmajor, a_bits, Bm, b_kmajor, b_bits, M, N, K, out,
+                        workspace, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+fqt_status fqt_sync_status(void *workspace, void *stream) {
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return FQT_ECUDA;
+  if (!workspace) return FQT_EWORKSPACE;
+  int code = 0;
+  if (cudaMemcpy(&code, workspace, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return FQT_ECUDA;
+  if (code != 0 && cudaMemset(workspace, 0, sizeof(int)) != cudaSuccess) return FQT_ECUDA;
+  return static_cast<fqt_status>(code);
+}
+
+const char *fqt_status_string(fqt_status status) {
+  switch (status) {
+    case FQT_OK: return "ok";
+    case FQT_EINVAL: return "invalid argument";
+    case FQT_EUNSUPPORTED: return "unsupported shape or option";
+    case FQT_ECUDA: return "CUDA error";
+    case FQT_ENONFINITE: return "non-finite input";
+    case FQT_ETIMEOUT: return "device-side wait timed out";
+    case FQT_EWORKSPACE: return "workspace missing, misaligned or too small";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

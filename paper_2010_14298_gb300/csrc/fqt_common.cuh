@@ -1,0 +1,192 @@
+// fqt_common.cuh -- shared device helpers of the GB300 FQT library:
+// workspace layout, the Philox4x32-10 generator, stochastic rounding and the
+// PTX wrappers (mbarrier, bulk copies, fences) the kernels use.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "fqt.h"
+
+namespace fqt {
+
+// ---------------------------------------------------------------------------
+// Workspace layout (caller-owned device memory, zero-filled before first use)
+//   [0, 256)               header: int32 status word at offset 0
+//   [256, 256 + 32 KiB)    per-CTA (min, max) partials of the range pass
+//   [kGemmOffset, ...)     split-K int32 partial tiles of grad_W
+// ---------------------------------------------------------------------------
+constexpr size_t kHeaderBytes = 256;
+constexpr int kMaxRangeCtas = 4096;
+constexpr size_t kRangeOffset = kHeaderBytes;
+constexpr size_t kRangeBytes = sizeof(float2) * kMaxRangeCtas;
+constexpr size_t kGemmOffset = kRangeOffset + kRangeBytes;
+
+// Time limit of every device-side wait (mbarrier polls), in nanoseconds of
+// %globaltimer.  A wait that exceeds it records FQT_ETIMEOUT and the kernel
+// winds down; no legitimate wait in these kernels lasts a millisecond.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+__device__ __forceinline__ void record_status(int *status, int code) {
+  if (status) atomicCAS(status, 0, code);
+}
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of the 4x32
+// S-box, multipliers 0xD2511F53 / 0xCD9E8D57, Weyl key increments
+// 0x9E3779B9 / 0xBB67AE85.
+// ---------------------------------------------------------------------------
+struct PhiloxKey {
+  uint32_t k0, k1;
+};
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, PhiloxKey key) {
+  uint32_t k0 = key.k0, k1 = key.k1;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// Eight 16-bit uniforms for the aligned group of 8 consecutive flat indices
+// starting at 8*q of `stream`: uniform i is half (i mod 2) of word i / 2.
+__device__ __forceinline__ uint4 philox_oct(uint64_t q, uint32_t stream,
+                                            PhiloxKey key) {
+  return philox4x32_10(
+      make_uint4((uint32_t)q, (uint32_t)(q >> 32), stream, 0u), key);
+}
+
+__device__ __forceinline__ uint32_t u16_of(const uint4 &w, int i) {
+  const uint32_t word = (i >> 1) == 0 ? w.x : (i >> 1) == 1 ? w.y
+                        : (i >> 1) == 2 ? w.z : w.w;
+  return (i & 1) ? (word >> 16) : (word & 0xFFFFu);
+}
+
+// Stochastic rounding of v >= 0 onto 0..B (Sec. 3.3): the probability
+// frac(v) is realised in 16-bit fixed point, code = (floor(v 2^16) + u) >> 16.
+__device__ __forceinline__ uint32_t sr_code(float v, uint32_t u16, uint32_t B) {
+  v = fminf(v, (float)(B + 1u));
+  const uint32_t fixed = __float2uint_rz(__fmul_rn(v, 65536.0f));
+  const uint32_t code = (fixed + u16) >> 16;
+  return min(code, B);
+}
+
+// Scale B / R of the affine quantizers; R = 0 or an overflowing quotient
+// take s = 1 (all codes 0, value = z).
+__device__ __forceinline__ float affine_scale(float mn, float mx, uint32_t B) {
+  const float R = __fsub_rn(mx, mn);
+  if (!(R > 0.0f)) return 1.0f;
+  const float s = __fdiv_rn((float)B, R);
+  return isfinite(s) ? s : 1.0f;
+}
+
+// ---------------------------------------------------------------------------
+// Loads of 8 consecutive elements (an "oct") as floats.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void load_oct(const float *p, float (&x)[8]) {
+  const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
+  const float4 b = __ldg(reinterpret_cast<const float4 *>(p) + 1);
+  x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+  x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+}
+
+__device__ __forceinline__ void load_oct(const __nv_bfloat16 *p, float (&x)[8]) {
+  const uint4 a = __ldg(reinterpret_cast<const uint4 *>(p));
+  const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    x[2 * i] = __uint_as_float(w[i] << 16);
+    x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+__device__ __forceinline__ void store_codes8(uint8_t *dst, const uint32_t (&c)[8]) {
+  uint2 v;
+  v.x = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
+  v.y = c[4] | (c[5] << 8) | (c[6] << 16) | (c[7] << 24);
+  *reinterpret_cast<uint2 *>(dst) = v;
+}
+
+// ---------------------------------------------------------------------------
+// PTX wrappers: mbarrier, async-proxy fences, bulk / tensor copies.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(count));
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile(
+      "mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "r"(bytes)
+      : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Bounded wait: returns false (and records FQT_ETIMEOUT) if the phase with
+// the given parity has not completed within kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          int *status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    for (int i = 0; i < 64; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (global_ns() - t0 > kWaitLimitNs) {
+      record_status(status, FQT_ETIMEOUT);
+      return false;
+    }
+  }
+}
+
+// Sleeps about `ns` nanoseconds (used only on the abort path).
+__device__ __forceinline__ void sleep_ns(uint64_t ns) {
+  const uint64_t t0 = global_ns();
+  while (global_ns() - t0 < ns) __nanosleep(1000);
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+}  // namespace fqt

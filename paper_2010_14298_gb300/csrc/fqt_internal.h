@@ -1,0 +1,59 @@
+// fqt_internal.h -- declarations shared by the translation units of the
+// GB300 FQT library (kernel argument blocks and host launchers).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "fqt.h"
+
+namespace fqt {
+
+enum { KIND_PTQ = 0, KIND_PSQ = 1, KIND_BHQ = 2, KIND_DET = 3 };
+
+
+
+// Arguments of the quantizer kernel (see fqt_quant.cu for the mapping).
+struct QuantArgs {
+  const void *h;
+  int64_t N;
+  int C, CO;
+  int kind, bits, block;
+  uint32_t key0, key1;
+  // code set 2: Q_b2 (gradient) or the forward operand (KIND_DET)
+  uint8_t *c2;
+  float *inv2, *zero2;
+  int32_t *rsum2, *csum2, *lead2;
+  // code set 1: Q_b1, 8-bit stochastic PTQ (may be null)
+  uint8_t *c1;
+  float *inv1, *zero1;
+  int32_t *rsum1, *csum1;
+  const float2 *part;
+  int npart;
+  int *status;
+  // launch geometry
+  int TW, OPT, RL, RPL, GT, G, nchunk, unit_rows;
+  int64_t n_units;
+};
+
+fqt_status quant_geometry(QuantArgs &a, int num_sms, int *nth, int *grid,
+                          size_t *smem);
+cudaError_t launch_quant(const QuantArgs &a, bool bf16, int nth, int grid,
+                         size_t smem, cudaStream_t st);
+cudaError_t launch_range(const void *x, bool bf16, int64_t count, float2 *part,
+                         int *npart, int32_t *z0, int64_t nz0, int32_t *z1,
+                         int64_t nz1, int num_sms, cudaStream_t st);
+
+int device_sm_count();
+
+size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D);
+fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
+                           const fqt_qtensor *qx, const fqt_qtensor *qw,
+                           float *grad_X, float *grad_W, void *ws,
+                           size_t ws_bytes, cudaStream_t st);
+fqt_status debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
+                          const uint8_t *Bm, int b_kmajor, int b_bits, int64_t M,
+                          int64_t N, int64_t K, int64_t *out, void *ws,
+                          size_t ws_bytes, cudaStream_t st);
+
+}  // namespace fqt

@@ -1,0 +1,600 @@
+// fqt_quant.cu -- quantizer kernels of the GB300 FQT library.
+//
+//  k_range  : per-CTA (min, max) of a tensor and a non-finite flag (the
+//             dynamic range R(X) = max X - min X of Sec. 3.3); also clears
+//             the column-sum outputs the quantizer accumulates into.
+//  k_quant  : one templated kernel for
+//             KIND_PTQ  per-tensor stochastic quantizer (Sec. 3.3),
+//             KIND_PSQ  per-sample quantizer (Sec. 4.1),
+//             KIND_BHQ  block Householder quantizer (Sec. 4.2, App. D.4),
+//             KIND_DET  deterministic PTQ of the forward operands (Sec. 2.1),
+//             fused with the 8-bit stochastic PTQ Q_b1 of App. E.
+//
+// Thread mapping.  A row (sample) is handled by a team of TW consecutive
+// threads; each thread owns OPT "octs" (8 consecutive columns) of the row,
+// octs cl, cl + TW, ...  Rows of a unit are spread over RL row lanes, RPL
+// rows per lane.  For BHQ a unit is one block of `block` rows and a CTA runs
+// G such groups side by side.  Row reductions use shuffles inside the team
+// (TW <= 32) or shared memory (TW > 32); the BHQ column sums go through
+// shared memory in a fixed order.  When the row does not fit the registers
+// (nchunk > 1, only BHQ with long rows) every pass re-reads its chunk.
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "fqt_common.cuh"
+#include "fqt_internal.h"
+
+namespace fqt {
+
+constexpr int kMaxOct = 4;  // octs a thread keeps in registers per pass
+
+// ---------------------------------------------------------------------------
+// Range pass
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void __launch_bounds__(256) k_range(const T *__restrict__ x,
+                                               int64_t n_oct, float2 *part,
+                                               int32_t *z0, int64_t nz0,
+                                               int32_t *z1, int64_t nz1) {
+  float mn = INFINITY, mx = -INFINITY;
+  int bad = 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (; o + 3 * stride < n_oct; o += 4 * stride) {
+    float v[4][8];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) load_oct(x + (o + u * stride) * 8, v[u]);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        bad |= !isfinite(v[u][i]);
+        mn = fminf(mn, v[u][i]);
+        mx = fmaxf(mx, v[u][i]);
+      }
+  }
+  for (; o < n_oct; o += stride) {
+    float v[8];
+    load_oct(x + o * 8, v);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      bad |= !isfinite(v[i]);
+      mn = fminf(mn, v[i]);
+      mx = fmaxf(mx, v[i]);
+    }
+  }
+  const int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (int64_t i = g; i < nz0; i += stride) z0[i] = 0;
+  for (int64_t i = g; i < nz1; i += stride) z1[i] = 0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  __shared__ float smn[8], smx[8];
+  __shared__ int sbad[8];
+  const int w = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    smn[w] = mn;
+    smx[w] = mx;
+    sbad[w] = bad;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 1; i < (int)(blockDim.x >> 5); ++i) {
+      mn = fminf(mn, smn[i]);
+      mx = fmaxf(mx, smx[i]);
+      bad |= sbad[i];
+    }
+    part[blockIdx.x] = bad ? make_float2(NAN, NAN) : make_float2(mn, mx);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Team reductions (a team = TW consecutive threads owning one row)
+// ---------------------------------------------------------------------------
+struct OpMinMax {
+  __device__ float2 operator()(float2 a, float2 b) const {
+    return make_float2(fminf(a.x, b.x), fmaxf(a.y, b.y));
+  }
+};
+struct OpMin {
+  __device__ float operator()(float a, float b) const { return fminf(a, b); }
+};
+struct OpAdd {
+  __device__ int operator()(int a, int b) const { return a + b; }
+};
+
+__device__ __forceinline__ float shfl_x(float v, int off) {
+  return __shfl_xor_sync(0xffffffffu, v, off);
+}
+__device__ __forceinline__ int shfl_x(int v, int off) {
+  return __shfl_xor_sync(0xffffffffu, v, off);
+}
+__device__ __forceinline__ float2 shfl_x(float2 v, int off) {
+  return make_float2(__shfl_xor_sync(0xffffffffu, v.x, off),
+                     __shfl_xor_sync(0xffffffffu, v.y, off));
+}
+
+// Reduces v over the TW lanes of each team; every lane of the team receives
+// the result.  Must be reached by the whole CTA (barriers when TW > 32);
+// `red` holds 32 entries of V.
+template <class V, class Op>
+__device__ __forceinline__ V team_reduce(V v, int TW, V *red, Op op) {
+  if (TW <= 32) {
+    for (int off = TW >> 1; off > 0; off >>= 1) v = op(v, shfl_x(v, off));
+    return v;
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v = op(v, shfl_x(v, off));
+  const int warp = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) red[warp] = v;
+  __syncthreads();
+  const int w0 = (threadIdx.x / TW) * (TW >> 5);
+  V acc = red[w0];
+  for (int w = 1; w < (TW >> 5); ++w) acc = op(acc, red[w0 + w]);
+  __syncthreads();
+  return acc;
+}
+
+// ---------------------------------------------------------------------------
+// The quantizer kernel
+// ---------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ const T *row_ptr(const void *h, int64_t row, int C) {
+  return reinterpret_cast<const T *>(h) + row * (int64_t)C;
+}
+
+template <int KIND, typename T, int NTMAX>
+__global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  // with 1024 threads the register file allows no per-thread column sums
+  constexpr bool kRegColSums = NTMAX <= 256;
+  const int nth = blockDim.x, tid = threadIdx.x;
+  const int grp = tid / a.GT, gt = tid - grp * a.GT;
+  const int rl = gt / a.TW, cl = gt - rl * a.TW;
+  const int TW = a.TW, OPT = a.OPT, RL = a.RL, C = a.C, CO = a.CO;
+  const int chunk_octs = TW * OPT;
+  const int chunk_cols = chunk_octs * 8;
+
+  // shared memory carve-up (sizes computed by quant_smem_bytes on the host)
+  float2 *red2 = reinterpret_cast<float2 *>(smem);    // 32
+  float *redf = reinterpret_cast<float *>(red2 + 32);  // 32
+  int *redi = reinterpret_cast<int *>(redf + 32);      // 32
+  int *csum_s = redi + 32;                             // C
+  float *bpar = reinterpret_cast<float *>(csum_s + C);  // G * 8
+  float2 *rowst = reinterpret_cast<float2 *>(bpar + 8 * a.G);  // G * block
+  float *wcol = reinterpret_cast<float *>(rowst + a.G * a.block);  // G * C
+  float *colp = wcol + a.G * C;  // G * RL * chunk_cols
+
+  // ---- global range from the range-pass partials ----
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < a.npart; i += nth) {
+    const float2 p = a.part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if ((tid & 31) == 0) {
+    red2[tid >> 5] = make_float2(gmin, gmax);
+    redi[tid >> 5] = bad;
+  }
+  for (int i = tid; i < C; i += nth) csum_s[i] = 0;
+  __syncthreads();
+  gmin = red2[0].x;
+  gmax = red2[0].y;
+  bad = redi[0];
+  for (int w = 1; w < (nth >> 5); ++w) {
+    gmin = fminf(gmin, red2[w].x);
+    gmax = fmaxf(gmax, red2[w].y);
+    bad |= redi[w];
+  }
+  __syncthreads();
+  if (bad) {
+    if (blockIdx.x == 0 && tid == 0) record_status(a.status, FQT_ENONFINITE);
+    return;
+  }
+  const uint32_t B2 = (1u << a.bits) - 1u;
+  const float s_g2 = affine_scale(gmin, gmax, B2);    // PTQ / DET scale
+  const float s_g1 = affine_scale(gmin, gmax, 255u);  // Q_b1 scale
+  const bool has_b1 = a.c1 != nullptr;
+  if (blockIdx.x == 0 && tid == 0) {
+    if (KIND == KIND_PTQ || KIND == KIND_DET) {
+      a.inv2[0] = __fdiv_rn(1.0f, s_g2);
+      a.zero2[0] = __fmul_rn(s_g2, gmin);
+    }
+    if (has_b1) {
+      a.inv1[0] = __fdiv_rn(1.0f, s_g1);
+      a.zero1[0] = __fmul_rn(s_g1, gmin);
+    }
+  }
+  // column sums of the code set that feeds grad_W (Q_b1 when present)
+  int32_t *const csum_g = has_b1 ? a.csum1 : a.csum2;
+  const bool want_cs = csum_g != nullptr;
+  const bool reg_cs = kRegColSums && a.nchunk == 1;
+  int cs[kMaxOct][8];
+#pragma unroll
+  for (int k = 0; k < kMaxOct; ++k)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cs[k][j] = 0;
+
+  const PhiloxKey key = {a.key0, a.key1};
+  float x[kMaxOct][8];
+
+  for (int64_t ub = (int64_t)blockIdx.x * a.G; ub < a.n_units;
+       ub += (int64_t)gridDim.x * a.G) {
+    const int64_t u = ub + grp;
+    const bool uvalid = u < a.n_units;
+    const int64_t r0 = u * a.unit_rows;
+    const int nrows = uvalid ? (int)min((int64_t)a.unit_rows, a.N - r0) : 0;
+    const bool rvalid = rl < nrows;
+    const int64_t row = r0 + rl;
+
+    auto oct_of = [&](int ch, int k) { return ch * chunk_octs + cl + TW * k; };
+    auto oct_ok = [&](int ch, int k) {
+      return k < OPT && rvalid && oct_of(ch, k) < CO;
+    };
+    auto load_chunk = [&](int ch) {
+#pragma unroll
+      for (int k = 0; k < kMaxOct; ++k) {
+        if (oct_ok(ch, k)) {
+          load_oct(row_ptr<T>(a.h, row, C) + oct_of(ch, k) * 8, x[k]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) x[k][j] = 0.0f;
+        }
+      }
+    };
+
+    // ---------------- per-row statistics (PSQ, BHQ) ----------------
+    float2 st = make_float2(INFINITY, -INFINITY);
+    if (KIND == KIND_PSQ || KIND == KIND_BHQ) {
+      for (int ch = 0; ch < a.nchunk; ++ch) {
+        load_chunk(ch);
+#pragma unroll
+        for (int k = 0; k < kMaxOct; ++k) {
+          if (oct_ok(ch, k)) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              st.x = fminf(st.x, x[k][j]);
+              st.y = fmaxf(st.y, x[k][j]);
+            }
+          }
+        }
+      }
+      st = team_reduce(st, TW, red2, OpMinMax());
+    }
+
+    // ---------------- BHQ: block scalars, Householder, row minima ----------
+    float s_row = 0.0f, c_row = 0.0f;
+    if (KIND == KIND_BHQ) {
+      if (cl == 0 && rvalid) rowst[grp * a.block + rl] = st;
+      __syncthreads();
+      if (gt == 0 && uvalid) {
+        const float2 *rs = rowst + grp * a.block;
+        int p = 0;
+        float np = -1.0f;
+        for (int k = 0; k < nrows; ++k) {  // lead row: largest ||h_k||_inf
+          const float nk = fmaxf(fabsf(rs[k].x), fabsf(rs[k].y));
+          if (nk > np) { np = nk; p = k; }
+        }
+        float lam2 = 0.0f;
+        for (int k = 0; k < nrows; ++k)
+          if (k != p) lam2 = fmaxf(lam2, fmaxf(fabsf(rs[k].x), fabsf(rs[k].y)));
+        lam2 = 2.0f * lam2;
+        float s1f = 0.0f, s2f = 0.0f, rho = 0.0f, kap = 0.0f;
+        if (np > 0.0f) {
+          float lam1 = __fsub_rn(rs[p].y, rs[p].x);
+          if (!(lam1 > 0.0f)) lam1 = 2.0f * np;
+          const double Nd = (double)nrows;
+          double s1, s2 = 0.0;
+          if (lam2 > 0.0f) {  // s1, s2 of App. D.4
+            const double c1 = cbrt((double)lam1), c2 = cbrt((double)lam2);
+            const double den = c1 * c1 * pow(Nd, -1.0 / 3.0) +
+                               c2 * c2 * pow(Nd, 2.0 / 3.0);
+            s1 = (double)B2 * pow(Nd, 1.0 / 6.0) / (c1 * den);
+            s2 = (double)B2 * pow(Nd, 1.0 / 6.0) / (c2 * den);
+          } else {  // limit lambda2 -> 0: the other rows are zero
+            s1 = (double)B2 * sqrt(Nd) / (double)lam1;
+          }
+          s1f = (float)s1;
+          s2f = lam2 > 0.0f ? (float)s2 : 0.0f;
+          if (nrows > 1) {
+            const double r = 1.0 / sqrt(Nd);
+            rho = (float)r;
+            kap = (float)(1.0 / (1.0 - r));
+          }
+        }
+        float *bp = bpar + grp * 8;
+        bp[0] = s1f;
+        bp[1] = s2f;
+        bp[2] = rho;
+        bp[3] = kap;
+        bp[4] = __int_as_float(p);
+        a.lead2[u] = p;
+      }
+      __syncthreads();
+      const float *bp = bpar + grp * 8;
+      const int p = __float_as_int(bp[4]);
+      const bool lead = rl == p;
+      s_row = lead ? bp[0] : bp[1];
+      c_row = lead ? bp[2] - 1.0f : bp[2];  // rho - delta_kp
+      const float e_row = bp[3] * c_row;    // (rho - delta_kp) / (1 - rho)
+      // w_j = sum_k e_k s_k h_kj, so that (Q g)_k = g_k - c_k w (g = s h)
+      float *cp = colp + grp * RL * chunk_cols;
+      float *wc = wcol + grp * C;
+      float tmin = INFINITY;
+      for (int ch = 0; ch < a.nchunk; ++ch) {
+        if (a.nchunk > 1) load_chunk(ch);
+#pragma unroll
+        for (int k = 0; k < kMaxOct; ++k) {
+          if (k < OPT) {
+            float *dst = cp + rl * chunk_cols + (cl + TW * k) * 8;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              dst[j] = __fmul_rn(e_row, __fmul_rn(s_row, x[k][j]));
+          }
+        }
+        __syncthreads();
+        for (int c = gt; c < chunk_cols; c += a.GT) {
+          const int col = ch * chunk_cols + c;
+          if (col < C) {
+            float acc = 0.0f;
+            for (int r = 0; r < RL; ++r) acc += cp[r * chunk_cols + c];
+            wc[col] = acc;
+          }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < kMaxOct; ++k) {
+          if (oct_ok(ch, k)) {
+            const int col0 = oct_of(ch, k) * 8;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float t = fmaf(-c_row, wc[col0 + j], __fmul_rn(s_row, x[k][j]));
+              tmin = fminf(tmin, t);
+            }
+          }
+        }
+      }
+      st.x = team_reduce(tmin, TW, redf, OpMin());  // z'_k
+    }
+
+    // ---------------- scale of this thread's row ----------------
+    float s2, z2;
+    if (KIND == KIND_PSQ) {
+      s2 = affine_scale(st.x, st.y, B2);
+      z2 = st.x;
+    } else if (KIND == KIND_BHQ) {
+      s2 = s_row;
+      z2 = st.x;
+    } else {
+      s2 = s_g2;
+      z2 = gmin;
+    }
+
+    // ---------------- rounding, packing, sums ----------------
+    int rs2 = 0, rs1 = 0;
+    for (int ch = 0; ch < a.nchunk; ++ch) {
+      if (a.nchunk > 1 || KIND == KIND_PTQ || KIND == KIND_DET) load_chunk(ch);
+#pragma unroll
+      for (int k = 0; k < kMaxOct; ++k) {
+        if (!oct_ok(ch, k)) continue;
+        const int o = oct_of(ch, k);
+        const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)o;
+        uint32_t c[8];
+        if (KIND == KIND_DET) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float v = __fmul_rn(__fsub_rn(x[k][j], z2), s2);
+            const int r = __float2int_rn(v);
+            c[j] = (uint32_t)min(max(r, 0), (int)B2);
+          }
+        } else {
+          const uint4 w = philox_oct(q, 0u, key);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float v;
+            if (KIND == KIND_BHQ) {
+              const float t = fmaf(-c_row, wcol[grp * C + o * 8 + j],
+                                   __fmul_rn(s_row, x[k][j]));
+              v = __fsub_rn(t, z2);
+            } else {
+              v = __fmul_rn(__fsub_rn(x[k][j], z2), s2);
+            }
+            c[j] = sr_code(v, u16_of(w, j), B2);
+          }
+        }
+        store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) rs2 += (int)c[j];
+        const uint32_t *sumc = c;
+        uint32_t d[8];
+        if (has_b1) {
+          const uint4 w = philox_oct(q, 1u, key);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float v = __fmul_rn(__fsub_rn(x[k][j], gmin), s_g1);
+            d[j] = sr_code(v, u16_of(w, j), 255u);
+            rs1 += (int)d[j];
+          }
+          store_codes8(a.c1 + row * (int64_t)C + o * 8, d);
+          sumc = d;
+        }
+        if (want_cs) {
+          if (reg_cs) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) cs[k][j] += (int)sumc[j];
+          } else {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              if (sumc[j]) atomicAdd(&csum_s[o * 8 + j], (int)sumc[j]);
+          }
+        }
+      }
+    }
+
+    // ---------------- row metadata ----------------
+    if (a.rsum2) rs2 = team_reduce(rs2, TW, redi, OpAdd());
+    if (has_b1 && a.rsum1) rs1 = team_reduce(rs1, TW, redi, OpAdd());
+    if (cl == 0 && rvalid) {
+      if (a.rsum2) a.rsum2[row] = rs2;
+      if (has_b1 && a.rsum1) a.rsum1[row] = rs1;
+      if (KIND == KIND_PSQ) {
+        a.inv2[row] = __fdiv_rn(1.0f, s2);
+        a.zero2[row] = __fmul_rn(s2, z2);
+      } else if (KIND == KIND_BHQ) {
+        a.inv2[row] = s2 > 0.0f ? __fdiv_rn(1.0f, s2) : 0.0f;
+        a.zero2[row] = z2;
+      }
+    }
+    if (KIND == KIND_BHQ) __syncthreads();  // bpar / wcol / colp are reused
+  }
+
+  // ---------------- column sums ----------------
+  if (want_cs) {
+    if (reg_cs) {
+#pragma unroll
+      for (int k = 0; k < kMaxOct; ++k) {
+        const int o = cl + TW * k;
+        if (k < OPT && o < CO) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (cs[k][j]) atomicAdd(&csum_s[o * 8 + j], cs[k][j]);
+        }
+      }
+    }
+    __syncthreads();
+    for (int i = tid; i < C; i += nth)
+      if (csum_s[i]) atomicAdd(&csum_g[i], csum_s[i]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------
+static int pow2ceil(int v) {
+  int p = 1;
+  while (p < v) p <<= 1;
+  return p;
+}
+
+size_t quant_smem_bytes(const QuantArgs &a) {
+  const size_t chunk_cols = (size_t)a.TW * a.OPT * 8;
+  size_t b = sizeof(float2) * 32 + sizeof(float) * 32 + sizeof(int) * 32;
+  b += sizeof(int) * a.C;
+  b += sizeof(float) * 8 * a.G;
+  if (a.kind == KIND_BHQ) {
+    b += sizeof(float2) * a.G * a.block;
+    b += sizeof(float) * a.G * a.C;
+    b += sizeof(float) * a.G * a.RL * chunk_cols;
+  }
+  return b;
+}
+
+// Chooses the thread mapping of k_quant for an N x C problem: TW threads per
+// row, each holding OPT <= 4 octs per pass; nchunk passes cover long rows.
+fqt_status quant_geometry(QuantArgs &a, int num_sms, int *nth_out,
+                          int *grid_out, size_t *smem_out) {
+  const int C = a.C;
+  if (C <= 0 || C % 8) return FQT_EUNSUPPORTED;
+  const int CO = C / 8;
+  a.CO = CO;
+  int opt = CO < kMaxOct ? CO : kMaxOct;
+  int TW = pow2ceil((CO + opt - 1) / opt);
+  const int rows_per_unit = a.kind == KIND_BHQ ? a.block : 1;
+  // a group (one BHQ block, or one row) may use at most 1024 threads
+  while ((int64_t)TW * rows_per_unit > 1024 && TW > 1) TW >>= 1;
+  if ((int64_t)TW * rows_per_unit > 1024) return FQT_EUNSUPPORTED;
+  opt = (CO + TW - 1) / TW;
+  if (opt > kMaxOct) opt = kMaxOct;
+  const int nchunk = (CO + TW * opt - 1) / (TW * opt);
+  if (nchunk > 1 && a.kind != KIND_BHQ) return FQT_EUNSUPPORTED;
+  a.TW = TW;
+  a.OPT = opt;
+  a.RPL = 1;
+  a.nchunk = nchunk;
+  int nth;
+  if (a.kind == KIND_BHQ) {
+    a.RL = a.block;
+    a.GT = a.RL * TW;
+    nth = a.GT < 256 ? 256 : a.GT;
+    a.G = nth / a.GT;
+    a.unit_rows = a.block;
+    a.n_units = (a.N + a.block - 1) / a.block;
+  } else {
+    nth = TW < 256 ? 256 : TW;
+    a.RL = nth / TW;
+    a.GT = nth;
+    a.G = 1;
+    a.unit_rows = a.RL;
+    a.n_units = (a.N + a.RL - 1) / a.RL;
+  }
+  const size_t smem = quant_smem_bytes(a);
+  if (smem > 200 * 1024) return FQT_EUNSUPPORTED;
+  const int per_sm = nth <= 256 ? 4 : 1;
+  const int64_t need = (a.n_units + a.G - 1) / a.G;
+  int64_t grid = (int64_t)num_sms * per_sm;
+  if (grid > need) grid = need;
+  if (grid < 1) grid = 1;
+  *nth_out = nth;
+  *grid_out = (int)grid;
+  *smem_out = smem;
+  return FQT_OK;
+}
+
+template <int KIND, typename T>
+static cudaError_t launch_quant_t(const QuantArgs &a, int nth, int grid,
+                                  size_t smem, cudaStream_t st) {
+  auto fn = nth <= 256 ? k_quant<KIND, T, 256> : k_quant<KIND, T, 1024>;
+  cudaError_t e = cudaFuncSetAttribute(
+      fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  fn<<<grid, nth, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quant(const QuantArgs &a, bool bf16, int nth, int grid,
+                         size_t smem, cudaStream_t st) {
+  switch (a.kind * 2 + (bf16 ? 1 : 0)) {
+    case KIND_PTQ * 2: return launch_quant_t<KIND_PTQ, float>(a, nth, grid, smem, st);
+    case KIND_PTQ * 2 + 1: return launch_quant_t<KIND_PTQ, __nv_bfloat16>(a, nth, grid, smem, st);
+    case KIND_PSQ * 2: return launch_quant_t<KIND_PSQ, float>(a, nth, grid, smem, st);
+    case KIND_PSQ * 2 + 1: return launch_quant_t<KIND_PSQ, __nv_bfloat16>(a, nth, grid, smem, st);
+    case KIND_BHQ * 2: return launch_quant_t<KIND_BHQ, float>(a, nth, grid, smem, st);
+    case KIND_BHQ * 2 + 1: return launch_quant_t<KIND_BHQ, __nv_bfloat16>(a, nth, grid, smem, st);
+    case KIND_DET * 2: return launch_quant_t<KIND_DET, float>(a, nth, grid, smem, st);
+    case KIND_DET * 2 + 1: return launch_quant_t<KIND_DET, __nv_bfloat16>(a, nth, grid, smem, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_range(const void *x, bool bf16, int64_t count, float2 *part,
+                         int *npart, int32_t *z0, int64_t nz0, int32_t *z1,
+                         int64_t nz1, int num_sms, cudaStream_t st) {
+  const int64_t n_oct = count / 8;
+  int64_t grid = (n_oct + 255) / 256;
+  const int64_t cap = (int64_t)num_sms * 8;
+  if (grid > cap) grid = cap;
+  if (grid > kMaxRangeCtas) grid = kMaxRangeCtas;
+  if (grid < 1) grid = 1;
+  *npart = (int)grid;
+  if (bf16)
+    k_range<__nv_bfloat16><<<(int)grid, 256, 0, st>>>(
+        reinterpret_cast<const __nv_bfloat16 *>(x), n_oct, part, z0, nz0, z1, nz1);
+  else
+    k_range<float><<<(int)grid, 256, 0, st>>>(
+        reinterpret_cast<const float *>(x), n_oct, part, z0, nz0, z1, nz1);
+  return cudaGetLastError();
+}
+
+}  // namespace fqt

@@ -1,0 +1,295 @@
+"""ctypes binding of the C ABI in include/fqt.h.
+
+Argument marshalling only: every step of the hot path runs in the CUDA
+library ``_lib/libfqt.so``.  PyTorch provides device memory and streams.
+There is no CPU fallback: if the library is missing or no GPU is present the
+calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+PTQ, PSQ, BHQ = 0, 1, 2
+F32, BF16 = 0, 1
+STATUS = {0: "FQT_OK", 1: "FQT_EINVAL", 2: "FQT_EUNSUPPORTED", 3: "FQT_ECUDA",
+          4: "FQT_ENONFINITE", 5: "FQT_ETIMEOUT", 6: "FQT_EWORKSPACE"}
+
+_lib = None
+_lock = threading.Lock()
+
+
+class FqtError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {STATUS.get(status, status)}")
+
+
+class _QT(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("bits", ctypes.c_int32), ("kind", ctypes.c_int32),
+                ("block", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("codes", ctypes.c_void_p), ("inv_s", ctypes.c_void_p),
+                ("zero", ctypes.c_void_p), ("row_sum", ctypes.c_void_p),
+                ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p)]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True):
+    """Loads libfqt.so (building it with nvcc when absent)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if not os.path.exists(path):
+            if not build_if_missing:
+                raise FileNotFoundError(f"{path} is not built")
+            _build.build()
+        lib = ctypes.CDLL(path)
+        P, i64, u64, i32, sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint64,
+                                ctypes.c_int, ctypes.c_size_t)
+        QP = ctypes.POINTER(_QT)
+        lib.fqt_workspace_size.argtypes = [i64, i64, i64]
+        lib.fqt_workspace_size.restype = sz
+        for name in ("fqt_quantize_act", "fqt_quantize_weight"):
+            f = getattr(lib, name)
+            f.argtypes = [P, i32, i64, i64, i32, QP, P, sz, P]
+            f.restype = i32
+        lib.fqt_quantize_grad.argtypes = [P, i32, i64, i64, i32, i32, i32, u64,
+                                          QP, QP, P, sz, P]
+        lib.fqt_quantize_grad.restype = i32
+        lib.fqt_linear_backward.argtypes = [QP, QP, QP, QP, P, P, P, sz, P]
+        lib.fqt_linear_backward.restype = i32
+        lib.fqt_sync_status.argtypes = [P, P]
+        lib.fqt_sync_status.restype = i32
+        lib.fqt_debug_int_gemm.argtypes = [P, i32, i32, P, i32, i32, i64, i64,
+                                           i64, P, P, sz, P]
+        lib.fqt_debug_int_gemm.restype = i32
+        lib.fqt_status_string.argtypes = [i32]
+        lib.fqt_status_string.restype = ctypes.c_char_p
+        _lib = lib
+        return lib
+
+
+def _check(st: int, what: str):
+    if st != 0:
+        raise FqtError(st, what)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else None
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+class Workspace:
+    """Caller-owned device scratch (zero-filled once), see fqt_workspace_size."""
+
+    def __init__(self, N: int, C: int, D: int, device="cuda"):
+        self.nbytes = int(load().fqt_workspace_size(N, C, D))
+        self.buf = torch.zeros(self.nbytes, dtype=torch.uint8, device=device)
+
+    def ensure(self, N: int, C: int, D: int):
+        need = int(load().fqt_workspace_size(N, C, D))
+        if need > self.nbytes:
+            self.nbytes = need
+            self.buf = torch.zeros(need, dtype=torch.uint8, device=self.buf.device)
+        return self
+
+    @property
+    def ptr(self):
+        return ctypes.c_void_p(self.buf.data_ptr())
+
+
+@dataclass
+class QTensor:
+    """A quantized matrix (the fqt_qtensor of include/fqt.h) held in torch tensors."""
+    codes: torch.Tensor
+    inv_s: torch.Tensor
+    zero: torch.Tensor
+    row_sum: Optional[torch.Tensor]
+    col_sum: Optional[torch.Tensor]
+    lead: Optional[torch.Tensor]
+    kind: int = PTQ
+    bits: int = 8
+    block: int = 0
+
+    @staticmethod
+    def empty(rows: int, cols: int, kind: int, bits: int, block: int = 0,
+              row_sum: bool = True, col_sum: bool = True, device="cuda"):
+        m = 1 if kind == PTQ else rows
+        nblk = (rows + block - 1) // block if kind == BHQ else 0
+        return QTensor(
+            codes=torch.empty((rows, cols), dtype=torch.uint8, device=device),
+            inv_s=torch.empty(m, dtype=torch.float32, device=device),
+            zero=torch.empty(m, dtype=torch.float32, device=device),
+            row_sum=(torch.empty(rows, dtype=torch.int32, device=device)
+                     if row_sum else None),
+            col_sum=(torch.empty(cols, dtype=torch.int32, device=device)
+                     if col_sum else None),
+            lead=(torch.empty(max(nblk, 1), dtype=torch.int32, device=device)
+                  if kind == BHQ else None),
+            kind=kind, bits=bits, block=block)
+
+    def c_struct(self) -> _QT:
+        rows, cols = self.codes.shape
+        return _QT(rows, cols, self.bits, self.kind, self.block, 0,
+                   self.codes.data_ptr(), self.inv_s.data_ptr(),
+                   self.zero.data_ptr(),
+                   self.row_sum.data_ptr() if self.row_sum is not None else None,
+                   self.col_sum.data_ptr() if self.col_sum is not None else None,
+                   self.lead.data_ptr() if self.lead is not None else None)
+
+    def to_numpy(self) -> dict:
+        """Host copy in the oracle's dict layout."""
+        d = dict(codes=self.codes.cpu().numpy(), inv_s=self.inv_s.cpu().numpy(),
+                 zero=self.zero.cpu().numpy(), kind=self.kind, bits=self.bits,
+                 block=self.block,
+                 lead=self.lead.cpu().numpy() if self.kind == BHQ else None)
+        if self.row_sum is not None:
+            d["row_sum"] = self.row_sum.cpu().numpy()
+        if self.col_sum is not None:
+            d["col_sum"] = self.col_sum.cpu().numpy()
+        return d
+
+
+def workspace_size(N: int, C: int, D: int) -> int:
+    return int(load().fqt_workspace_size(N, C, D))
+
+
+def _fwd(name, X, bits, ws, out, row_sum, col_sum, stream):
+    lib = load()
+    rows, cols = X.shape
+    if out is None:
+        out = QTensor.empty(rows, cols, PTQ, bits, 0, row_sum, col_sum, X.device)
+    qs = out.c_struct()
+    st = getattr(lib, name)(_ptr(X), _dtype_code(X), rows, cols, bits,
+                            ctypes.byref(qs), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, name)
+    out.kind, out.bits, out.block = PTQ, bits, 0
+    return out
+
+
+def quantize_act(X: torch.Tensor, bits: int = 8, ws: Workspace = None,
+                 out: QTensor = None, row_sum: bool = False,
+                 col_sum: bool = True, stream=None) -> QTensor:
+    """X~ = Q_f(X): deterministic PTQ (Sec. 2.1, App. E)."""
+    ws = ws or Workspace(*X.shape, 16, device=X.device)
+    return _fwd("fqt_quantize_act", X.contiguous(), bits, ws, out, row_sum,
+                col_sum, stream)
+
+
+def quantize_weight(W: torch.Tensor, bits: int = 8, ws: Workspace = None,
+                    out: QTensor = None, row_sum: bool = False,
+                    col_sum: bool = True, stream=None) -> QTensor:
+    """W~ = Q_theta(W): deterministic PTQ (Sec. 2.1, App. E)."""
+    ws = ws or Workspace(*W.shape, 16, device=W.device)
+    return _fwd("fqt_quantize_weight", W.contiguous(), bits, ws, out, row_sum,
+                col_sum, stream)
+
+
+def quantize_grad(dH: torch.Tensor, kind: int, bits: int, block: int = 0,
+                  seed: int = 0, with_b1: bool = True, ws: Workspace = None,
+                  q_b2: QTensor = None, q_b1: QTensor = None,
+                  b2_col_sum: bool = False, stream=None):
+    """(Q_b2(dH), Q_b1(dH)) with stochastic rounding (Sec. 3.3, 4.1, 4.2, App. E)."""
+    lib = load()
+    dH = dH.contiguous()
+    N, C = dH.shape
+    ws = ws or Workspace(N, C, 16, device=dH.device)
+    if q_b2 is None:
+        q_b2 = QTensor.empty(N, C, kind, bits, block if kind == BHQ else 0,
+                             True, b2_col_sum or not with_b1, dH.device)
+    if with_b1 and q_b1 is None:
+        q_b1 = QTensor.empty(N, C, PTQ, 8, 0, False, True, dH.device)
+    s2 = q_b2.c_struct()
+    s1 = q_b1.c_struct() if with_b1 else None
+    st = lib.fqt_quantize_grad(_ptr(dH), _dtype_code(dH), N, C, kind, bits,
+                               block if kind == BHQ else 0,
+                               ctypes.c_uint64(seed & (2 ** 64 - 1)),
+                               ctypes.byref(s2),
+                               ctypes.byref(s1) if s1 is not None else None,
+                               ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "fqt_quantize_grad")
+    q_b2.kind, q_b2.bits, q_b2.block = kind, bits, block if kind == BHQ else 0
+    if with_b1:
+        q_b1.kind, q_b1.bits, q_b1.block = PTQ, 8, 0
+    return q_b2, (q_b1 if with_b1 else None)
+
+
+def linear_backward(q_b2: QTensor, q_b1: Optional[QTensor], qx: QTensor,
+                    qw: QTensor, grad_x: bool = True, grad_w: bool = True,
+                    ws: Workspace = None, out_x: torch.Tensor = None,
+                    out_w: torch.Tensor = None, stream=None):
+    """grad_X = Q_b2(dH) W~ and grad_W = Q_b1(dH)^T X~ (Eq. 6, App. E)."""
+    lib = load()
+    N, C = q_b2.codes.shape
+    D = qx.codes.shape[1] if qx is not None else qw.codes.shape[1]
+    dev = q_b2.codes.device
+    ws = (ws or Workspace(N, C, D, device=dev)).ensure(N, C, D)
+    gx = gw = None
+    if grad_x:
+        gx = out_x if out_x is not None else torch.empty((N, D), dtype=torch.float32,
+                                                         device=dev)
+    if grad_w:
+        gw = out_w if out_w is not None else torch.empty((C, D), dtype=torch.float32,
+                                                         device=dev)
+    s2 = q_b2.c_struct()
+    s1 = q_b1.c_struct() if q_b1 is not None else None
+    sx = qx.c_struct() if qx is not None else None
+    sw = qw.c_struct() if qw is not None else None
+    st = lib.fqt_linear_backward(ctypes.byref(s2),
+                                 ctypes.byref(s1) if s1 is not None else None,
+                                 ctypes.byref(sx) if sx is not None else None,
+                                 ctypes.byref(sw) if sw is not None else None,
+                                 _ptr(gx), _ptr(gw), ws.ptr, ws.nbytes,
+                                 _stream(stream))
+    _check(st, "fqt_linear_backward")
+    return gx, gw
+
+
+def debug_int_gemm(A: torch.Tensor, a_kmajor: bool, a_bits: int, B: torch.Tensor,
+                   b_kmajor: bool, b_bits: int, M: int, N: int, K: int,
+                   ws: Workspace = None, stream=None) -> torch.Tensor:
+    """Exact sum_k (A_ik - 2^(a-1))(B_kj - 2^(b-1)) as int64 (M x N)."""
+    lib = load()
+    out = torch.empty((M, N), dtype=torch.int64, device=A.device)
+    ws = ws or Workspace(K, M, N, device=A.device)
+    ws.ensure(K, M, N)
+    st = lib.fqt_debug_int_gemm(_ptr(A), int(a_kmajor), a_bits, _ptr(B),
+                                int(b_kmajor), b_bits, M, N, K, _ptr(out), ws.ptr,
+                                ws.nbytes, _stream(stream))
+    _check(st, "fqt_debug_int_gemm")
+    return out
+
+
+def sync_status(ws: Workspace, stream=None) -> int:
+    """Synchronises and returns (then clears) the device-side status word."""
+    return int(load().fqt_sync_status(ws.ptr, _stream(stream)))
+
+
+def status_string(code: int) -> str:
+    return load().fqt_status_string(code).decode()

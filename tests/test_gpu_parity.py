@@ -1,0 +1,290 @@
+"""GPU parity: the CUDA library against the CPU oracle, through the C ABI.
+
+Bars: bit-exact for integer work (PTQ / PSQ / deterministic codes, metadata,
+sums, the integer contraction); BHQ codes agree on >= 99.99% of entries and
+every mismatch is a +-1 flip at a stochastic-rounding boundary; gradients
+agree within max |g - r| / max(|r|, 1e-3 ||r_row||_inf) <= 1e-3 with the
+GPU's codes fed to the oracle's dequantize-then-multiply.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from paper_2010_14298_gb300 import fqt
+from paper_2010_14298_gb300 import workloads as wl
+from gpu_util import (grad_rel_err, oracle_rows_grad_x, sr_boundary_distance,
+                      to_dev)
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="no GPU")]
+
+GRAD_TOL = 1e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    fqt.load()
+    yield
+
+
+# --------------------------------------------------------------------------
+# Integer contraction core
+# --------------------------------------------------------------------------
+GEMM_CASES = [
+    # M, N, K, a_kmajor, b_kmajor, a_bits, b_bits
+    (300, 272, 208, 1, 0, 5, 8),      # grad_X layout, ragged tiles and K tail
+    (64, 576, 5000, 0, 0, 8, 8),      # grad_W layout, split-K, exact chunks
+    (128, 128, 64, 1, 1, 8, 8),
+    (256, 160, 1040, 0, 1, 8, 4),
+    (48, 32, 16, 1, 0, 2, 8),
+    (1000, 64, 1024, 1, 0, 8, 8),
+]
+
+
+@pytest.mark.parametrize("M,N,K,ak,bk,ab,bb", GEMM_CASES)
+def test_int_gemm_bit_exact(M, N, K, ak, bk, ab, bb):
+    g = wl.rng(M * 7 + N * 3 + K)
+    A = g.integers(0, 1 << ab, (M, K)).astype(np.uint8)
+    B = g.integers(0, 1 << bb, (K, N)).astype(np.uint8)
+    a_st = A if ak else np.ascontiguousarray(A.T)
+    b_st = np.ascontiguousarray(B.T) if bk else B
+    got = fqt.debug_int_gemm(torch.from_numpy(a_st).cuda(), ak, ab,
+                             torch.from_numpy(b_st).cuda(), bk, bb, M, N, K)
+    ref = orc.int_gemm(a_st, ak, b_st, bk, M, N, K, 1 << (ab - 1), 1 << (bb - 1))
+    assert np.array_equal(got.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("K", [1024, 4096, 8192 + 64])
+@pytest.mark.parametrize("fill", [(255, 255), (0, 0), (0, 255)])
+def test_int_gemm_exact_at_extreme_magnitudes(K, fill):
+    """Every product at its largest magnitude: partial sums reach the 2^24
+    limit of exact fp32 accumulation inside each chunk."""
+    M, N = 128, 128
+    A = np.full((M, K), fill[0], dtype=np.uint8)
+    B = np.full((K, N), fill[1], dtype=np.uint8)
+    got = fqt.debug_int_gemm(torch.from_numpy(A).cuda(), 1, 8,
+                             torch.from_numpy(B).cuda(), 0, 8, M, N, K)
+    expect = K * (int(fill[0]) - 128) * (int(fill[1]) - 128)
+    assert (got.cpu().numpy() == expect).all()
+
+
+# --------------------------------------------------------------------------
+# Quantizers
+# --------------------------------------------------------------------------
+def _check_b1(q1_gpu, dH, seed):
+    r1 = orc.quantize_grad(dH, orc.PTQ, 8, 0, seed, orc.STREAM_B1)
+    h1 = q1_gpu.to_numpy()
+    assert np.array_equal(h1["codes"], r1["codes"])
+    assert np.array_equal(h1["inv_s"], r1["inv_s"])
+    assert np.array_equal(h1["zero"], r1["zero"])
+    assert np.array_equal(h1["col_sum"], r1["codes"].astype(np.int64).sum(0))
+
+
+def _check_bhq_codes(got, ref, v, seed, stream=0):
+    diff = got.astype(np.int64) - ref.astype(np.int64)
+    agree = (diff == 0).mean()
+    assert agree >= 0.9999, agree
+    assert np.abs(diff).max() <= 1
+    idx = np.flatnonzero(diff.ravel())
+    if idx.size:
+        dist = sr_boundary_distance(v.ravel()[idx], seed, stream, idx)
+        assert dist.max() <= 256, dist.max()  # within 2^-8 bin of the threshold
+
+
+QUANT_CASES = [(0, None, orc.PTQ, 8, 0), (0, None, orc.PSQ, 8, 0),
+               (0, None, orc.BHQ, 5, 16), (1, 2, orc.PTQ, 4, 0),
+               (1, 2, orc.PSQ, 5, 0), (1, 2, orc.BHQ, 8, 16),
+               (2, 1, orc.BHQ, 5, 8), (2, 1, orc.BHQ, 5, 64),
+               (3, 64, orc.PSQ, 5, 0), (3, 64, orc.BHQ, 5, 16),
+               (3, 64, orc.PTQ, 8, 0)]
+
+
+@pytest.mark.parametrize("cfg,small,kind,bits,block", QUANT_CASES)
+def test_quantize_grad_matches_oracle(cfg, small, kind, bits, block):
+    kw = {}
+    if cfg in (1, 2):
+        kw["batch"] = small
+    elif cfg == 3:
+        kw["rows"] = small
+    seed = 1234567
+    for L in wl.config(cfg, **kw):
+        dH = L.dH
+        q2, q1 = fqt.quantize_grad(to_dev(dH, L.dtype), kind, bits, block, seed)
+        ref = orc.quantize_grad(dH, kind, bits, block, seed, orc.STREAM_B2,
+                                want_v=True)
+        h2 = q2.to_numpy()
+        assert np.array_equal(h2["row_sum"], h2["codes"].astype(np.int64).sum(1))
+        if kind == orc.BHQ:
+            assert np.array_equal(h2["lead"], ref["lead"])
+            _check_bhq_codes(h2["codes"], ref["codes"], ref["v"], seed)
+            assert np.allclose(h2["inv_s"], ref["inv_s"], rtol=1e-6, atol=0)
+            assert np.allclose(h2["zero"], ref["zero"], rtol=1e-5, atol=1e-4)
+        else:
+            assert np.array_equal(h2["codes"], ref["codes"])
+            assert np.array_equal(h2["inv_s"], ref["inv_s"])
+            assert np.array_equal(h2["zero"], ref["zero"])
+        _check_b1(q1, dH, seed)
+
+
+def test_quantize_fwd_matches_oracle():
+    L = wl.config(1, batch=2)[0]
+    for M in (L.X, L.W):
+        q = fqt.quantize_act(to_dev(M), 8, row_sum=True)
+        ref = orc.quantize_fwd(M, 8)
+        h = q.to_numpy()
+        assert np.array_equal(h["codes"], ref["codes"])
+        assert np.array_equal(h["inv_s"], ref["inv_s"])
+        assert np.array_equal(h["zero"], ref["zero"])
+        assert np.array_equal(h["col_sum"], ref["codes"].astype(np.int64).sum(0))
+        assert np.array_equal(h["row_sum"], ref["codes"].astype(np.int64).sum(1))
+
+
+def test_quantize_fwd_bf16():
+    L = wl.config(3, rows=64)[0]
+    q = fqt.quantize_weight(to_dev(L.W, "bf16"), 8)
+    ref = orc.quantize_fwd(L.W, 8)
+    assert np.array_equal(q.codes.cpu().numpy(), ref["codes"])
+
+
+# --------------------------------------------------------------------------
+# The whole backward
+# --------------------------------------------------------------------------
+def _backward(L, kind, bits, block, seed=3, reuse=False):
+    dev = lambda a: to_dev(a, L.dtype)
+    qx = fqt.quantize_act(dev(L.X), 8)
+    qw = fqt.quantize_weight(dev(L.W), 8)
+    q2, q1 = fqt.quantize_grad(dev(L.dH), kind, bits, block, seed,
+                               with_b1=not reuse, b2_col_sum=reuse)
+    gx, gw = fqt.linear_backward(q2, q1, qx, qw)
+    torch.cuda.synchronize()
+    return qx, qw, q2, q1, gx.cpu().numpy(), gw.cpu().numpy()
+
+
+BACKWARD_CASES = [(0, None, orc.PTQ, 8, 0), (0, None, orc.PSQ, 8, 0),
+                  (0, None, orc.BHQ, 5, 16), (1, 2, orc.PTQ, 4, 0),
+                  (1, 2, orc.BHQ, 5, 16), (2, 1, orc.BHQ, 5, 32),
+                  (2, 1, orc.BHQ, 5, 64), (3, 128, orc.BHQ, 5, 16),
+                  (3, 128, orc.PTQ, 8, 0)]
+
+
+@pytest.mark.parametrize("cfg,small,kind,bits,block", BACKWARD_CASES)
+def test_linear_backward_matches_oracle(cfg, small, kind, bits, block):
+    kw = {}
+    if cfg in (1, 2):
+        kw["batch"] = small
+    elif cfg == 3:
+        kw["rows"] = small
+    for L in wl.config(cfg, **kw):
+        qx, qw, q2, q1, gx, gw = _backward(L, kind, bits, block)
+        h2, h1, hx, hw = q2.to_numpy(), q1.to_numpy(), qx.to_numpy(), qw.to_numpy()
+        ref_x = orc.grad_x(h2, hw)
+        ref_w = orc.grad_w(h1, hx)
+        assert grad_rel_err(gx, ref_x) <= GRAD_TOL
+        assert grad_rel_err(gw, ref_w) <= GRAD_TOL
+
+
+def test_ptq_codes_reused_for_grad_w():
+    L = wl.config(0)[0]
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.PTQ, 8, 0, reuse=True)
+    assert q1 is None
+    ref_w = orc.grad_w(q2.to_numpy(), qx.to_numpy())
+    assert grad_rel_err(gw, ref_w) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("cfg,kind,bits,block", [(1, orc.BHQ, 5, 16),
+                                                 (1, orc.PSQ, 4, 0),
+                                                 (2, orc.BHQ, 5, 16)])
+def test_full_size_sampled(cfg, kind, bits, block):
+    """Full-size workloads in the bench's launch configuration: codes of all
+    rows, grad_X on sampled row blocks, grad_W on sampled columns."""
+    L = wl.config(cfg)[0]
+    qx, qw, q2, q1, gx, gw = _backward(L, kind, bits, block, seed=11)
+    h2, h1, hx, hw = q2.to_numpy(), q1.to_numpy(), qx.to_numpy(), qw.to_numpy()
+    ref2 = orc.quantize_grad(L.dH, kind, bits, block, 11, orc.STREAM_B2,
+                             want_v=True)
+    if kind == orc.BHQ:
+        _check_bhq_codes(h2["codes"], ref2["codes"], ref2["v"], 11)
+    else:
+        assert np.array_equal(h2["codes"], ref2["codes"])
+    _check_b1(q1, L.dH, 11)
+    g = wl.rng(5)
+    rows = np.sort(g.choice(L.N, 96, replace=False))
+    ref_x = oracle_rows_grad_x(h2, hw, h2["codes"], rows)
+    assert grad_rel_err(gx[rows], ref_x) <= GRAD_TOL
+    cols = np.sort(g.choice(L.D, 32, replace=False))
+    deq1 = orc.dequant(h1)
+    deqx = orc.dequant(hx)[:, cols]
+    ref_w = orc.matmul(deq1, deqx, a_trans=True)
+    assert grad_rel_err(gw[:, cols], ref_w) <= GRAD_TOL
+
+
+# --------------------------------------------------------------------------
+# Edge cases and device-side status
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("N", [1, 5, 17, 33])
+@pytest.mark.parametrize("kind,block", [(orc.PSQ, 0), (orc.BHQ, 16),
+                                        (orc.BHQ, 64), (orc.PTQ, 0)])
+def test_ragged_and_tiny(N, kind, block):
+    g = wl.rng(N)
+    dH = wl.random_grad(g, N, 48, outlier_frac=0.2)
+    X = g.uniform(-1, 1, (N, 32)).astype(np.float32)
+    W = g.standard_normal((48, 32)).astype(np.float32)
+    L = wl.Layer("edge", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, kind, 5, block)
+    ref = orc.quantize_grad(dH, kind, 5, block, 3, orc.STREAM_B2, want_v=True)
+    if kind == orc.BHQ:
+        _check_bhq_codes(q2.codes.cpu().numpy(), ref["codes"], ref["v"], 3)
+    else:
+        assert np.array_equal(q2.codes.cpu().numpy(), ref["codes"])
+    h2, h1 = q2.to_numpy(), q1.to_numpy()
+    assert grad_rel_err(gx, orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+    assert grad_rel_err(gw, orc.grad_w(h1, qx.to_numpy())) <= GRAD_TOL
+
+
+def test_zero_and_constant_gradients():
+    dH = np.zeros((64, 32), dtype=np.float32)
+    dH[10] = 1.5
+    dH[40:48] = -2.0
+    for kind, block in ((orc.PTQ, 0), (orc.PSQ, 0), (orc.BHQ, 16)):
+        q2, q1 = fqt.quantize_grad(to_dev(dH), kind, 4, block, 0)
+        ref = orc.quantize_grad(dH, kind, 4, block, 0)
+        assert np.array_equal(q2.codes.cpu().numpy(), ref["codes"])
+        assert np.allclose(q2.inv_s.cpu().numpy(), ref["inv_s"], rtol=1e-6)
+
+
+def test_empty_batch_is_a_no_op():
+    dH = torch.zeros((0, 64), device="cuda")
+    q2, q1 = fqt.quantize_grad(dH, orc.PSQ, 5, 0, 0)
+    assert q2.codes.shape == (0, 64)
+
+
+def test_nonfinite_input_is_reported_on_sync():
+    dH = np.ones((32, 64), dtype=np.float32)
+    dH[3, 5] = np.nan
+    ws = fqt.Workspace(32, 64, 16)
+    fqt.quantize_grad(to_dev(dH), orc.PSQ, 5, 0, 0, ws=ws)
+    assert fqt.sync_status(ws) == 4
+    assert fqt.sync_status(ws) == 0  # cleared
+    dH[3, 5] = np.inf
+    fqt.quantize_act(to_dev(dH), 8, ws=ws)
+    assert fqt.sync_status(ws) == 4
+
+
+def test_same_seed_same_codes_other_seed_other_codes():
+    L = wl.config(0)[0]
+    a, _ = fqt.quantize_grad(to_dev(L.dH), orc.BHQ, 5, 16, 77)
+    b, _ = fqt.quantize_grad(to_dev(L.dH), orc.BHQ, 5, 16, 77)
+    c, _ = fqt.quantize_grad(to_dev(L.dH), orc.BHQ, 5, 16, 78)
+    assert torch.equal(a.codes, b.codes)
+    assert not torch.equal(a.codes, c.codes)
+
+
+def test_argument_errors():
+    dH = torch.zeros((16, 12), device="cuda")  # C % 8 != 0
+    with pytest.raises(fqt.FqtError) as e:
+        fqt.quantize_grad(dH, orc.PSQ, 5, 0, 0)
+    assert e.value.status == 2
+    with pytest.raises(fqt.FqtError) as e:
+        fqt.quantize_grad(torch.zeros((16, 16), device="cuda"), orc.BHQ, 5, 3, 0)
+    assert e.value.status == 1
