@@ -1,0 +1,377 @@
+"""Benchmark of the FQT quantized backward on GB300.
+
+One step = one pass of the whole hot path over one batch of the ResNet-18
+3x3 conv backward (batch 128, 32x32, 64 -> 64 channels, im2col N = 131072,
+C = 64, D = 576):
+  X~ = Q_f(X), W~ = Q_theta(W)            (deterministic 8-bit PTQ)
+  Q_b2(dH) = BHQ 5-bit, block 16; Q_b1(dH) = 8-bit stochastic PTQ
+  grad_X = Q_b2(dH) W~,  grad_W = Q_b1(dH)^T X~
+The reported value is quantized-backward throughput in TOPS: both
+contractions count 2 N C D integer ops each.  Inputs are resident in HBM
+when timing starts; L2 is flushed (256 MiB write) between timed steps.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+The reference arm times the CPU oracle on a bounded sample of the same
+workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "quantized-backward TOPS and quantizer GB/s (1 GB300) vs roofline, oracle-exact"
+WORKLOAD = "resnet18-conv3x3-b128-32x32-64ch (im2col N=131072, C=64, D=576)"
+KIND, BITS, BLOCK = 2, 5, 16  # BHQ-5, block 16
+CONFIG_INDEX = 1
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _traffic_record(kernel: str):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if the
+    summary was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    import hashlib
+    src = os.path.join(ROOT, "paper_2010_14298_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in sorted(os.listdir(src)):
+        h.update(open(os.path.join(src, f), "rb").read())
+    digest = h.hexdigest()[:16]
+    for line in text.splitlines():
+        parts = [p.strip() for p in line.strip().strip("|").split("|")]
+        if len(parts) >= 3 and parts[0] == kernel and parts[2] == digest:
+            try:
+                return float(parts[1])
+            except ValueError:
+                return None
+    return None
+
+
+class Clocks:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.file = None
+
+    def __enter__(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.file is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        self.file.flush()
+        rows = []
+        for line in open(self.file.name):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        os.unlink(self.file.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4)
+                          if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2010_14298_gb300 import fqt
+    from paper_2010_14298_gb300 import workloads as wl
+
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    fqt.load(build_if_missing=True)
+    dev = torch.device("cuda", local)
+
+    L = wl.config(CONFIG_INDEX, seed=1234 + CONFIG_INDEX + 1000 * rank)[0]
+    N, C, D = L.N, L.C, L.D
+    dH = torch.from_numpy(L.dH).to(dev)
+    X = torch.from_numpy(L.X).to(dev)
+    W = torch.from_numpy(L.W).to(dev)
+    ws = fqt.Workspace(N, C, D, device=dev)
+    ws_fx = fqt.Workspace(N, D, 16, device=dev)
+    ws_fw = fqt.Workspace(C, D, 16, device=dev)
+    # the backward consumes the fp16 carriers of the codes (2 bytes per code)
+    qx = fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+    qw = fqt.QTensor.empty(C, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+    q2 = fqt.QTensor.empty(N, C, KIND, BITS, BLOCK, True, False, dev, u8=False)
+    q1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+    gx = torch.empty((N, D), dtype=torch.float32, device=dev)
+    gw = torch.empty((C, D), dtype=torch.float32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    names = ["quantize_act", "quantize_weight", "quantize_grad", "grad_x", "grad_w"]
+    launches_per_call = [2, 2, 2, 1, 2]
+
+    def step(seed, evs=None):
+        def mark(i):
+            if evs is not None:
+                evs[i].record(stream)
+        mark(0)
+        fqt.quantize_act(X, 8, ws=ws_fx, out=qx)
+        mark(1)
+        fqt.quantize_weight(W, 8, ws=ws_fw, out=qw)
+        mark(2)
+        fqt.quantize_grad(dH, KIND, BITS, BLOCK, seed, ws=ws, q_b2=q2, q_b1=q1)
+        mark(3)
+        fqt.linear_backward(q2, q1, qx, qw, grad_x=True, grad_w=False, ws=ws,
+                            out_x=gx)
+        mark(4)
+        fqt.linear_backward(q2, q1, qx, qw, grad_x=False, grad_w=True, ws=ws,
+                            out_w=gw)
+        mark(5)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if fqt.sync_status(ws) != 0:
+        raise RuntimeError("device-side status after warm-up")
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)]
+           for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with Clocks(local) as clk:
+        t_wall = time.perf_counter()
+        for i in range(args.steps):
+            flush.fill_(i & 0xFF)  # evict L2 between timed steps
+            step(1000 + i, evs[i])
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter() - t_wall
+    if world > 1:
+        dist.barrier()
+    per_call = np.zeros(5)
+    step_ms = []
+    for e in evs:
+        d = [e[j].elapsed_time(e[j + 1]) for j in range(5)]
+        per_call += np.array(d)
+        step_ms.append(sum(d))
+    ms_step = float(np.mean(step_ms))
+    per_call /= args.steps
+    if world > 1:
+        t = torch.tensor([ms_step], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_step = float(t.item())
+    status = fqt.sync_status(ws)
+
+    ops_step = 2 * 2 * N * C * D  # both contractions
+    value = ops_step * world / (ms_step * 1e-3) / 1e12
+
+    # ---- roofline of the dominant kernel (largest share of the step) ----
+    hbm_peak, peak_src = _peaks()
+    # algorithmic bytes: each input read once, each output written once;
+    # codes travel as 2-byte fp16 carriers
+    cb = 2
+    alg_bytes = {
+        "quantize_act": N * D * 4 + N * D * cb + D * 4,
+        "quantize_weight": C * D * 4 + C * D * cb + D * 4,
+        "quantize_grad": N * C * 4 + 2 * N * C * cb + N * (4 + 4 + 4) + (N // BLOCK) * 4 + C * 4,
+        "grad_x": N * C * cb + C * D * cb + N * D * 4 + N * 12 + (N // BLOCK) * 4 + D * 4,
+        "grad_w": N * C * cb + N * D * cb + C * D * 4 + (C + D) * 4,
+    }
+    kern_of = {"quantize_act": "k_quant", "quantize_weight": "k_quant",
+               "quantize_grad": "k_quant", "grad_x": "k_gemm", "grad_w": "k_gemm"}
+    dom = names[int(np.argmax(per_call))]
+    achieved = alg_bytes[dom] / (per_call[names.index(dom)] * 1e-3) / 1e9
+    traffic = _traffic_record(dom)
+    quant_gbs = alg_bytes["quantize_grad"] / (per_call[2] * 1e-3) / 1e9
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if args.e2e_steps > 0:
+        h_dH = torch.from_numpy(L.dH).pin_memory()
+        h_X = torch.from_numpy(L.X).pin_memory()
+        h_W = torch.from_numpy(L.W).pin_memory()
+        h_gx = torch.empty((N, D), dtype=torch.float32).pin_memory()
+        h_gw = torch.empty((C, D), dtype=torch.float32).pin_memory()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        tot = 0.0
+        for i in range(args.e2e_steps + 1):
+            flush.fill_(i & 0xFF)
+            torch.cuda.synchronize()
+            e0.record(stream)
+            dH.copy_(h_dH, non_blocking=True)
+            X.copy_(h_X, non_blocking=True)
+            W.copy_(h_W, non_blocking=True)
+            step(2000 + i)
+            h_gx.copy_(gx, non_blocking=True)
+            h_gw.copy_(gw, non_blocking=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if i > 0:  # first pass warms the pinned-copy path
+                tot += e0.elapsed_time(e1)
+        e2e_ms = tot / args.e2e_steps
+        e2e = {"value": ops_step * world / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
+               "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": int((N * C + N * D + C * D) * 4),
+               "d2h_bytes_per_step": int((N * D + C * D) * 4)}
+
+    result = {
+        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "u8 codes (fp16 carriers, exact int accumulation); f32 in/out",
+        "data": "synthetic (seeded; shapes and value distributions of the workload)",
+        "config": {"workload": WORKLOAD, "quantizer": "Q_b2=BHQ-5 block16, Q_b1=PTQ-8 stochastic, X~/W~=PTQ-8",
+                   "N": N, "C": C, "D": D, "global_batch": 128 * world,
+                   "parallelism": f"replicas x{world} (independent batches)",
+                   "l2": "flushed between timed steps (256 MiB write)",
+                   "wall_s": t_wall},
+        "per_call_ms": {k: float(v) for k, v in zip(names, per_call)},
+        "quantizer_gbs": quant_gbs,
+        "roofline": {"bound": "hbm", "kernel": kern_of[dom], "call": dom,
+                     "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "peak_source": peak_src,
+                     "algorithmic_bytes": alg_bytes[dom],
+                     "traffic": traffic},
+        "clocks": clk.summary(),
+        "e2e": e2e,
+        "gpu_launches": int(sum(launches_per_call) * args.steps),
+        "device_status": status,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(args.cpu_rows)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def _oracle_step(L, rows: int, seed: int):
+    """One oracle pass over the first `rows` rows (the whole hot path)."""
+    import oracle as orc
+    dH, X = L.dH[:rows], L.X[:rows]
+    orc.linear_backward(dH, X, L.W, KIND, BITS, BLOCK, seed)
+    return 2 * 2 * rows * L.C * L.D
+
+
+def cpu_baseline(rows: int):
+    from paper_2010_14298_gb300 import workloads as wl
+    import oracle
+    oracle.build()
+    L = wl.config(CONFIG_INDEX, batch=max(1, rows // 1024))[0]
+    rows = L.N
+    t = time.perf_counter()
+    ops = _oracle_step(L, rows, 0)
+    dt = time.perf_counter() - t
+    return {"value": ops / dt / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
+            "sample": f"{rows} im2col rows (batch {rows // 1024}) of the workload, "
+                      f"full hot path, {dt:.1f} s single-threaded"}
+
+
+def run_reference(args):
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    from paper_2010_14298_gb300 import workloads as wl
+    import oracle
+    oracle.build()
+    L = wl.config(CONFIG_INDEX, batch=max(1, args.ref_rows // 1024))[0]
+    rows = L.N
+    for i in range(args.warmup):
+        _oracle_step(L, min(rows, 1024), i)
+    t = time.perf_counter()
+    ops = 0
+    for i in range(args.steps):
+        ops += _oracle_step(L, rows, 100 + i)
+    dt = time.perf_counter() - t
+    value = ops / dt / 1e12
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS",
+           "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64 oracle (f32 codes)",
+           "data": "synthetic (seeded)",
+           "config": {"workload": WORKLOAD, "sample_rows": rows},
+           "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1,
+                            "kind": "oracle",
+                            "sample": f"{rows} im2col rows per step, full hot path"},
+           "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-rows", type=int, default=65536,
+                    help="rows of the CPU-baseline sample (about 10 s of oracle work)")
+    ap.add_argument("--ref-rows", type=int, default=8192,
+                    help="rows per reference-arm step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "native":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -64,7 +64,10 @@ typedef enum { FQT_F32 = 0, FQT_BF16 = 1 } fqt_dtype;
  * `block` consecutive rows (nb = rows of that block, p = its lead row).
  *
  * The caller allocates every array (device memory) and sets the pointers;
- * the quantize calls fill rows, cols, bits, kind and block.
+ * the quantize calls fill rows, cols, bits, kind and block and write every
+ * non-NULL output.  `codes` (1 byte per entry) and `codes_f16` (2 bytes, the
+ * same integers centred and widened) are two encodings of one code matrix;
+ * either may be NULL.
  */
 typedef struct fqt_qtensor {
   int64_t rows, cols;
@@ -80,6 +83,10 @@ typedef struct fqt_qtensor {
   int32_t *col_sum;  /* cols entries: sum_i codes_ij, or NULL (not computed) */
   int32_t *lead;     /* BHQ: ceil(rows / block) entries, lead row offset p
                         within each block; else unused (may be NULL) */
+  uint16_t *codes_f16; /* rows x cols, row-major: the centred code
+                        code - 2^(b-1) as an IEEE fp16 bit pattern (exact),
+                        the operand format of the tensor-core contractions;
+                        NULL = not written.  Required by fqt_linear_backward. */
 } fqt_qtensor;
 
 /* Bytes of workspace a layer with dH N x C, X N x D, W C x D needs for any
@@ -124,9 +131,10 @@ FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
  *   grad_W = Q_b1(dH)^T X~        (C x D, fp32, row-major; may be NULL)
  * The integer products of the codes are exact; dequantization and, for BHQ,
  * the inverse Householder transform of each block are applied in the
- * epilogue.  Needs q_b2->row_sum, qw->col_sum (grad_X) and q_b1->col_sum,
- * qx->col_sum (grad_W).  q_b1 may be NULL when q_b2 is PTQ with col_sum
- * set: grad_W then uses q_b2.  C % 16 == 0 and D % 16 == 0.
+ * epilogue.  Reads the operands' codes_f16 and needs q_b2->row_sum,
+ * qw->col_sum (grad_X) and q_b1->col_sum, qx->col_sum (grad_W).  q_b1 may be
+ * NULL when q_b2 is PTQ with col_sum set: grad_W then uses q_b2.
+ * C % 16 == 0 and D % 16 == 0.
  */
 FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,
                                const fqt_qtensor *q_b1,
@@ -141,7 +149,11 @@ FQT_API fqt_status fqt_sync_status(void *workspace, void *stream);
 /* Exact integer contraction, for bit-exact tests of the GEMM core:
  *   out_ij = sum_k (A_ik - 2^(a_bits-1)) (B_kj - 2^(b_bits-1))   (int64)
  * A is M x K, stored row-major (a_kmajor = 1) or as its K x M transpose;
- * B is K x N, stored as K x N row-major (b_kmajor = 0) or as N x K. */
+ * B is K x N, stored as K x N row-major (b_kmajor = 0) or as N x K; both
+ * u8 codes.  The stored row pitch must be a multiple of 8 and N % 4 == 0.
+ * The workspace must hold fqt_debug_workspace_size(M, N, K) bytes. */
+FQT_API size_t fqt_debug_workspace_size(int64_t M, int64_t N, int64_t K);
+
 FQT_API fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
                               const uint8_t *Bm, int b_kmajor, int b_bits,
                               int64_t M, int64_t N, int64_t K, int64_t *out,
@@ -149,6 +161,11 @@ FQT_API fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits
 
 /* Static description of a status code. */
 FQT_API const char *fqt_status_string(fqt_status status);
+
+/* After a call of this thread returned FQT_ECUDA: the name of the CUDA error
+ * behind it and the step that raised it (static storage, per thread);
+ * "none" otherwise.  Has no counterpart in the paper. */
+FQT_API const char *fqt_last_cuda_error(void);
 
 #ifdef __cplusplus
 }

@@ -1,6 +1,7 @@
 // fqt_api.cu -- the extern "C" entry points of include/fqt.h: argument
 // validation, workspace carving, launches, and the device status word.
 #include <cuda_runtime.h>
+#include <stdio.h>
 #include <string.h>
 
 #include "fqt.h"
@@ -21,6 +22,14 @@ int device_sm_count() {
   return n;
 }
 
+static thread_local char g_last_error[160] = "none";
+
+fqt_status cuda_fail(cudaError_t e, const char *where) {
+  if (e == cudaSuccess) return FQT_OK;
+  snprintf(g_last_error, sizeof(g_last_error), "%s: %s", where, cudaGetErrorName(e));
+  return FQT_ECUDA;
+}
+
 static bool aligned(const void *p, size_t a) {
   return (reinterpret_cast<uintptr_t>(p) % a) == 0;
 }
@@ -36,10 +45,12 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
                                    void *ws, size_t ws_bytes, void *stream) {
   if (rows < 0 || cols <= 0 || cols > (1 << 20) || bits < 2 || bits > 8) return FQT_EINVAL;
   if (!out) return FQT_EINVAL;
-  if (rows > 0 && (!X || !out->codes || !out->inv_s || !out->zero)) return FQT_EINVAL;
+  if (rows > 0 && (!X || (!out->codes && !out->codes_f16) || !out->inv_s || !out->zero))
+    return FQT_EINVAL;
   if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
   if (cols % 8) return FQT_EUNSUPPORTED;
-  if (!aligned(X, 16) || !aligned(out->codes, 16)) return FQT_EINVAL;
+  if (!aligned(X, 16) || !aligned(out->codes, 16) || !aligned(out->codes_f16, 16))
+    return FQT_EINVAL;
   fqt_status s = check_ws(ws, ws_bytes, kGemmOffset);
   if (s != FQT_OK) return s;
   out->rows = rows;
@@ -56,7 +67,7 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
   cudaError_t e = launch_range(X, dtype == FQT_BF16, rows * cols, part, &npart,
                                out->col_sum, out->col_sum ? cols : 0, nullptr, 0,
                                nsm, st);
-  if (e != cudaSuccess) return FQT_ECUDA;
+  if (e != cudaSuccess) return cuda_fail(e, "range pass");
   QuantArgs a;
   memset(&a, 0, sizeof(a));
   a.h = X;
@@ -66,6 +77,7 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
   a.bits = bits;
   a.block = 0;
   a.c2 = out->codes;
+  a.f2 = out->codes_f16;
   a.inv2 = out->inv_s;
   a.zero2 = out->zero;
   a.rsum2 = out->row_sum;
@@ -78,7 +90,7 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
   s = quant_geometry(a, nsm, &nth, &grid, &smem);
   if (s != FQT_OK) return s;
   e = launch_quant(a, dtype == FQT_BF16, nth, grid, smem, st);
-  return e == cudaSuccess ? FQT_OK : FQT_ECUDA;
+  return cuda_fail(e, "quantizer launch");
 }
 
 }  // namespace fqt
@@ -89,6 +101,10 @@ extern "C" {
 
 size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
   return kGemmOffset + gemm_workspace_bytes(N, C, D);
+}
+
+size_t fqt_debug_workspace_size(int64_t M, int64_t N, int64_t K) {
+  return debug_workspace_bytes(M, N, K);
 }
 
 fqt_status fqt_quantize_act(const void *X, fqt_dtype dtype, int64_t rows,
@@ -113,7 +129,8 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   if (N < 0 || C <= 0 || C > (1 << 20) || bits < 2 || bits > 8) return FQT_EINVAL;
   if (!q_b2) return FQT_EINVAL;
   // an empty batch has nothing to read or write (its tensors may be NULL)
-  if (N > 0 && (!dH || !q_b2->codes || !q_b2->inv_s || !q_b2->zero)) return FQT_EINVAL;
+  if (N > 0 && (!dH || (!q_b2->codes && !q_b2->codes_f16) || !q_b2->inv_s || !q_b2->zero))
+    return FQT_EINVAL;
   if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
   if (kind != FQT_PTQ && kind != FQT_PSQ && kind != FQT_BHQ) return FQT_EINVAL;
   if (kind == FQT_BHQ) {
@@ -122,9 +139,11 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   } else {
     block = 0;
   }
-  if (N > 0 && q_b1 && (!q_b1->codes || !q_b1->inv_s || !q_b1->zero)) return FQT_EINVAL;
+  if (N > 0 && q_b1 && ((!q_b1->codes && !q_b1->codes_f16) || !q_b1->inv_s || !q_b1->zero))
+    return FQT_EINVAL;
   if (C % 8) return FQT_EUNSUPPORTED;
-  if (!aligned(dH, 16) || !aligned(q_b2->codes, 16) || (q_b1 && !aligned(q_b1->codes, 16)))
+  if (!aligned(dH, 16) || !aligned(q_b2->codes, 16) || !aligned(q_b2->codes_f16, 16) ||
+      (q_b1 && (!aligned(q_b1->codes, 16) || !aligned(q_b1->codes_f16, 16))))
     return FQT_EINVAL;
   fqt_status s = check_ws(workspace, ws_bytes, kGemmOffset);
   if (s != FQT_OK) return s;
@@ -149,7 +168,7 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   int32_t *csum = q_b1 ? q_b1->col_sum : q_b2->col_sum;
   cudaError_t e = launch_range(dH, dtype == FQT_BF16, N * C, part, &npart, csum,
                                csum ? C : 0, nullptr, 0, nsm, st);
-  if (e != cudaSuccess) return FQT_ECUDA;
+  if (e != cudaSuccess) return cuda_fail(e, "range pass");
   QuantArgs a;
   memset(&a, 0, sizeof(a));
   a.h = dH;
@@ -161,6 +180,7 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   a.key0 = (uint32_t)seed;
   a.key1 = (uint32_t)(seed >> 32);
   a.c2 = q_b2->codes;
+  a.f2 = q_b2->codes_f16;
   a.inv2 = q_b2->inv_s;
   a.zero2 = q_b2->zero;
   a.rsum2 = q_b2->row_sum;
@@ -168,6 +188,7 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   a.lead2 = q_b2->lead;
   if (q_b1) {
     a.c1 = q_b1->codes;
+    a.f1 = q_b1->codes_f16;
     a.inv1 = q_b1->inv_s;
     a.zero1 = q_b1->zero;
     a.rsum1 = q_b1->row_sum;
@@ -178,10 +199,18 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   a.status = reinterpret_cast<int *>(w);
   int nth, grid;
   size_t smem;
+  const bool bf16 = dtype == FQT_BF16;
+  {
+    QuantArgs a2 = a;  // staged kernel for rows of up to 1024 columns
+    if (quant2_geometry(a2, bf16, nsm, &grid, &smem) == FQT_OK) {
+      e = launch_quant2(a2, bf16, grid, smem, st);
+      return cuda_fail(e, "staged quantizer launch");
+    }
+  }
   s = quant_geometry(a, nsm, &nth, &grid, &smem);
   if (s != FQT_OK) return s;
-  e = launch_quant(a, dtype == FQT_BF16, nth, grid, smem, st);
-  return e == cudaSuccess ? FQT_OK : FQT_ECUDA;
+  e = launch_quant(a, bf16, nth, grid, smem, st);
+  return cuda_fail(e, "quantizer launch");
 }
 
 fqt_status fqt_linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
@@ -202,14 +231,20 @@ fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
 
 fqt_status fqt_sync_status(void *workspace, void *stream) {
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaStreamSynchronize(st) != cudaSuccess) return FQT_ECUDA;
+  cudaError_t e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
   if (!workspace) return FQT_EWORKSPACE;
   int code = 0;
-  if (cudaMemcpy(&code, workspace, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
-    return FQT_ECUDA;
-  if (code != 0 && cudaMemset(workspace, 0, sizeof(int)) != cudaSuccess) return FQT_ECUDA;
+  e = cudaMemcpy(&code, workspace, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "status read");
+  if (code != 0) {
+    e = cudaMemset(workspace, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "status clear");
+  }
   return static_cast<fqt_status>(code);
 }
+
+const char *fqt_last_cuda_error(void) { return g_last_error; }
 
 const char *fqt_status_string(fqt_status status) {
   switch (status) {

@@ -5,6 +5,7 @@
 
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <stdint.h>
 
 #include "fqt.h"
@@ -113,6 +114,22 @@ __device__ __forceinline__ void store_codes8(uint8_t *dst, const uint32_t (&c)[8
   v.x = c[0] | (c[1] << 8) | (c[2] << 16) | (c[3] << 24);
   v.y = c[4] | (c[5] << 8) | (c[6] << 16) | (c[7] << 24);
   *reinterpret_cast<uint2 *>(dst) = v;
+}
+
+// Eight codes as the fp16 values code - off (exact for |.| <= 2048): the fp16
+// bit pattern 0x6400 | c is 1024 + c, and one packed subtraction recentres
+// two codes at a time.
+__device__ __forceinline__ void store_carriers8(uint16_t *dst, const uint32_t (&c)[8],
+                                                uint32_t off) {
+  const __half2 bias = __half2half2(__int2half_rn(1024 + (int)off));
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t h = (0x6400u | c[2 * i]) | ((0x6400u | c[2 * i + 1]) << 16);
+    __half2 v = __hsub2(*reinterpret_cast<const __half2 *>(&h), bias);
+    w[i] = *reinterpret_cast<uint32_t *>(&v);
+  }
+  *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 // ---------------------------------------------------------------------------

@@ -22,17 +22,19 @@ struct QuantArgs {
   uint32_t key0, key1;
   // code set 2: Q_b2 (gradient) or the forward operand (KIND_DET)
   uint8_t *c2;
+  uint16_t *f2;  // fp16 carriers of code set 2 (may be null)
   float *inv2, *zero2;
   int32_t *rsum2, *csum2, *lead2;
   // code set 1: Q_b1, 8-bit stochastic PTQ (may be null)
   uint8_t *c1;
+  uint16_t *f1;  // fp16 carriers of code set 1 (may be null)
   float *inv1, *zero1;
   int32_t *rsum1, *csum1;
   const float2 *part;
   int npart;
   int *status;
   // launch geometry
-  int TW, OPT, RL, RPL, GT, G, nchunk, unit_rows;
+  int TW, OPT, RL, RPL, GT, G, nchunk, unit_rows, stage_bytes;
   int64_t n_units;
 };
 
@@ -40,13 +42,22 @@ fqt_status quant_geometry(QuantArgs &a, int num_sms, int *nth, int *grid,
                           size_t *smem);
 cudaError_t launch_quant(const QuantArgs &a, bool bf16, int nth, int grid,
                          size_t smem, cudaStream_t st);
+fqt_status quant2_geometry(QuantArgs &a, bool bf16, int num_sms, int *grid,
+                           size_t *smem);
+cudaError_t launch_quant2(const QuantArgs &a, bool bf16, int grid, size_t smem,
+                          cudaStream_t st);
 cudaError_t launch_range(const void *x, bool bf16, int64_t count, float2 *part,
                          int *npart, int32_t *z0, int64_t nz0, int32_t *z1,
                          int64_t nz1, int num_sms, cudaStream_t st);
 
 int device_sm_count();
 
+// Records the CUDA error behind an FQT_ECUDA return (per thread) and returns
+// FQT_ECUDA, or FQT_OK for cudaSuccess.
+fqt_status cuda_fail(cudaError_t e, const char *where);
+
 size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D);
+size_t debug_workspace_bytes(int64_t M, int64_t N, int64_t K);
 fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
                            const fqt_qtensor *qx, const fqt_qtensor *qw,
                            float *grad_X, float *grad_W, void *ws,

@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
   const uint32_t B2 = (1u << a.bits) - 1u;
   const float s_g2 = affine_scale(gmin, gmax, B2);    // PTQ / DET scale
   const float s_g1 = affine_scale(gmin, gmax, 255u);  // Q_b1 scale
-  const bool has_b1 = a.c1 != nullptr;
+  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
   if (blockIdx.x == 0 && tid == 0) {
     if (KIND == KIND_PTQ || KIND == KIND_DET) {
       a.inv2[0] = __fdiv_rn(1.0f, s_g2);
@@ -414,7 +414,8 @@ __global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
             c[j] = sr_code(v, u16_of(w, j), B2);
           }
         }
-        store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+        if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+        if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + o * 8, c, (B2 + 1u) >> 1);
 #pragma unroll
         for (int j = 0; j < 8; ++j) rs2 += (int)c[j];
         const uint32_t *sumc = c;
@@ -427,7 +428,8 @@ __global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
             d[j] = sr_code(v, u16_of(w, j), 255u);
             rs1 += (int)d[j];
           }
-          store_codes8(a.c1 + row * (int64_t)C + o * 8, d);
+          if (a.c1) store_codes8(a.c1 + row * (int64_t)C + o * 8, d);
+          if (a.f1) store_carriers8(a.f1 + row * (int64_t)C + o * 8, d, 128u);
           sumc = d;
         }
         if (want_cs) {
@@ -475,6 +477,390 @@ __global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
     }
     __syncthreads();
     for (int i = tid; i < C; i += nth)
+      if (csum_s[i]) atomicAdd(&csum_g[i], csum_s[i]);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Staged quantizer (rows of up to 1024 columns).
+//
+// Units of consecutive rows are copied into shared memory with one
+// cp.async.bulk each (double-buffered: the next unit streams in while the
+// current one is processed).  Row work uses "row segments": LPR lanes of a
+// warp own one row, each lane OPL octs of it, so row reductions are short
+// shuffle trees and every shared-memory read of a warp is contiguous.  The
+// BHQ column sums of the Householder reflection (w_j = sum_k e_k s_k h_kj)
+// run one thread per (block, column) over the staged block.
+// ---------------------------------------------------------------------------
+constexpr int kQ2Threads = 256;
+
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src,
+                                         uint32_t bytes, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+template <typename T>
+__device__ __forceinline__ void load_oct_smem(const unsigned char *row, int o,
+                                              int lane, float (&x)[8]);
+
+template <>
+__device__ __forceinline__ void load_oct_smem<float>(const unsigned char *row,
+                                                     int o, int lane,
+                                                     float (&x)[8]) {
+  // two 16-byte halves; lanes 4..7 of each quarter warp start with the
+  // second half so that a quarter warp touches every bank once
+  const int h0 = (lane >> 2) & 1;
+  const float4 a = *reinterpret_cast<const float4 *>(row + o * 32 + h0 * 16);
+  const float4 b = *reinterpret_cast<const float4 *>(row + o * 32 + (h0 ^ 1) * 16);
+  const float4 lo = h0 ? b : a, hi = h0 ? a : b;
+  x[0] = lo.x; x[1] = lo.y; x[2] = lo.z; x[3] = lo.w;
+  x[4] = hi.x; x[5] = hi.y; x[6] = hi.z; x[7] = hi.w;
+}
+
+template <>
+__device__ __forceinline__ void load_oct_smem<__nv_bfloat16>(
+    const unsigned char *row, int o, int lane, float (&x)[8]) {
+  const uint4 v = *reinterpret_cast<const uint4 *>(row + o * 16);
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    x[2 * i] = __uint_as_float(w[i] << 16);
+    x[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+template <typename T>
+__device__ __forceinline__ float elem_smem(const unsigned char *base, int64_t idx) {
+  if (sizeof(T) == 4) return reinterpret_cast<const float *>(base)[idx];
+  const uint16_t b = reinterpret_cast<const uint16_t *>(base)[idx];
+  return __uint_as_float((uint32_t)b << 16);
+}
+
+// Reduction over the LPR lanes of a row segment (LPR a power of two <= 32).
+template <class V, class Op>
+__device__ __forceinline__ V seg_reduce(V v, int LPR, Op op) {
+  for (int off = LPR >> 1; off > 0; off >>= 1) v = op(v, shfl_x(v, off));
+  return v;
+}
+
+template <int KIND, typename T>
+__global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int C = a.C, CO = a.CO;
+  const int LPR = a.TW, OPL = a.OPT, R = a.RL;  // lanes per row, octs per lane, rows per warp step
+  const int U = a.unit_rows, nb = a.block > 0 ? a.block : 1;
+  const int G = a.G;  // BHQ blocks per unit
+  const int seg = lane / LPR, sl = lane - seg * LPR;
+  const int row_bytes = C * (int)sizeof(T);
+  const size_t stage_bytes = (size_t)a.stage_bytes;
+
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + 2 * stage_bytes);
+  float2 *red = reinterpret_cast<float2 *>(bar + 2);              // 8
+  int *redi = reinterpret_cast<int *>(red + 8);                   // 8
+  int *csum_s = redi + 8;                                          // C
+  float2 *rowst = reinterpret_cast<float2 *>(csum_s + C);         // U
+  float *bpar = reinterpret_cast<float *>(rowst + U);             // G * 8
+  float *wcol = bpar + 8 * G;                                      // G * C
+
+  // ---- global range from the range-pass partials ----
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < a.npart; i += kQ2Threads) {
+    const float2 p = a.part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmin, gmax);
+    redi[warp] = bad;
+  }
+  for (int i = tid; i < C; i += kQ2Threads) csum_s[i] = 0;
+  if (tid == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  gmin = red[0].x;
+  gmax = red[0].y;
+  bad = redi[0];
+  for (int w = 1; w < kQ2Threads / 32; ++w) {
+    gmin = fminf(gmin, red[w].x);
+    gmax = fmaxf(gmax, red[w].y);
+    bad |= redi[w];
+  }
+  if (bad) {
+    if (blockIdx.x == 0 && tid == 0) record_status(a.status, FQT_ENONFINITE);
+    return;
+  }
+  const uint32_t B2 = (1u << a.bits) - 1u;
+  const float s_g2 = affine_scale(gmin, gmax, B2);
+  const float s_g1 = affine_scale(gmin, gmax, 255u);
+  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
+  if (blockIdx.x == 0 && tid == 0) {
+    if (KIND == KIND_PTQ) {
+      a.inv2[0] = __fdiv_rn(1.0f, s_g2);
+      a.zero2[0] = __fmul_rn(s_g2, gmin);
+    }
+    if (has_b1) {
+      a.inv1[0] = __fdiv_rn(1.0f, s_g1);
+      a.zero1[0] = __fmul_rn(s_g1, gmin);
+    }
+  }
+  int32_t *const csum_g = has_b1 ? a.csum1 : a.csum2;
+  const bool want_cs = csum_g != nullptr;
+  int cs[kMaxOct][8];
+#pragma unroll
+  for (int k = 0; k < kMaxOct; ++k)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cs[k][j] = 0;
+  const PhiloxKey key = {a.key0, a.key1};
+
+  auto issue = [&](int64_t u, int b) {
+    const int64_t r0 = u * U;
+    const int rows = (int)min((int64_t)U, a.N - r0);
+    const uint32_t bytes = (uint32_t)rows * (uint32_t)row_bytes;
+    fence_proxy_async_smem();
+    mbar_expect_tx(&bar[b], bytes);
+    bulk_g2s(smem + (size_t)b * stage_bytes, reinterpret_cast<const unsigned char *>(a.h) + r0 * row_bytes,
+             bytes, &bar[b]);
+  };
+  if (tid == 0 && (int64_t)blockIdx.x < a.n_units) issue(blockIdx.x, 0);
+
+  int it = 0;
+  for (int64_t u = blockIdx.x; u < a.n_units; u += gridDim.x, ++it) {
+    const int b = it & 1;
+    if (tid == 0 && u + gridDim.x < a.n_units) issue(u + gridDim.x, b ^ 1);
+    const bool ok = mbar_wait(&bar[b], (uint32_t)(it >> 1) & 1u, a.status);
+    if (__syncthreads_or(!ok)) break;
+    const unsigned char *sh = smem + (size_t)b * stage_bytes;
+    const int64_t r0 = u * U;
+    const int rows = (int)min((int64_t)U, a.N - r0);
+    const int steps = (rows + 8 * R - 1) / (8 * R);
+
+    // ---------------- BHQ: statistics, block scalars, column sums ----------
+    if (KIND == KIND_BHQ) {
+      for (int st = 0; st < steps; ++st) {
+        const int r = (st * 8 + warp) * R + seg;
+        const bool rv = r < rows;
+        float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll
+        for (int k = 0; k < kMaxOct; ++k) {
+          const int o = sl + LPR * k;
+          if (k < OPL && rv && o < CO) {
+            float x[8];
+            load_oct_smem<T>(sh + (size_t)r * row_bytes, o, lane, x);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              mm.x = fminf(mm.x, x[j]);
+              mm.y = fmaxf(mm.y, x[j]);
+            }
+          }
+        }
+        mm = seg_reduce(mm, LPR, OpMinMax());
+        if (rv && sl == 0) rowst[r] = mm;
+      }
+      __syncthreads();
+      if (tid < G) {
+        const int k0 = tid * nb;
+        const int nrows = min(nb, rows - k0);
+        float s1f = 0.0f, s2f = 0.0f, rho = 0.0f, kap = 0.0f;
+        int p = 0;
+        if (nrows > 0) {
+          float np = -1.0f;
+          for (int k = 0; k < nrows; ++k) {  // lead row: largest ||h_k||_inf
+            const float2 q = rowst[k0 + k];
+            const float nk = fmaxf(fabsf(q.x), fabsf(q.y));
+            if (nk > np) { np = nk; p = k; }
+          }
+          float lam2 = 0.0f;
+          for (int k = 0; k < nrows; ++k) {
+            const float2 q = rowst[k0 + k];
+            if (k != p) lam2 = fmaxf(lam2, fmaxf(fabsf(q.x), fabsf(q.y)));
+          }
+          lam2 = 2.0f * lam2;
+          if (np > 0.0f) {
+            float lam1 = __fsub_rn(rowst[k0 + p].y, rowst[k0 + p].x);
+            if (!(lam1 > 0.0f)) lam1 = 2.0f * np;
+            const float Nf = (float)nrows;
+            if (lam2 > 0.0f) {  // s1, s2 of App. D.4
+              const float c1 = cbrtf(lam1), c2 = cbrtf(lam2);
+              const float n3 = cbrtf(Nf), n6 = sqrtf(n3);
+              const float den = c1 * c1 / n3 + c2 * c2 * n3 * n3;
+              s1f = (float)B2 * n6 / (c1 * den);
+              s2f = (float)B2 * n6 / (c2 * den);
+            } else {  // lambda2 -> 0: the other rows are zero
+              s1f = (float)B2 * sqrtf(Nf) / lam1;
+            }
+            if (nrows > 1) {
+              rho = 1.0f / sqrtf(Nf);
+              kap = 1.0f / (1.0f - rho);
+            }
+          }
+          a.lead2[(r0 / nb) + tid] = p;
+        }
+        float *bp = bpar + tid * 8;
+        bp[0] = s1f;
+        bp[1] = s2f;
+        bp[2] = rho;
+        bp[3] = kap;
+        bp[4] = __int_as_float(p);
+      }
+      __syncthreads();
+      // w_j of every block and column of the unit, rows in order
+      const int gu = (rows + nb - 1) / nb;
+      for (int item = tid; item < gu * C; item += kQ2Threads) {
+        const int bb = item / C, j = item - bb * C;
+        const float *bp = bpar + bb * 8;
+        const int p = __float_as_int(bp[4]);
+        const float s1f = bp[0], s2f = bp[1], rho = bp[2], kap = bp[3];
+        const int nrows = min(nb, rows - bb * nb);
+        float acc = 0.0f;
+        for (int k = 0; k < nrows; ++k) {
+          const float hv = elem_smem<T>(sh, (int64_t)(bb * nb + k) * C + j);
+          const bool lead = k == p;
+          const float e = kap * (lead ? rho - 1.0f : rho);
+          acc = fmaf(e, __fmul_rn(lead ? s1f : s2f, hv), acc);
+        }
+        wcol[bb * C + j] = acc;
+      }
+      __syncthreads();
+    }
+
+    // ---------------- per row: scale, rounding, packing, sums ----------------
+    for (int st = 0; st < steps; ++st) {
+      const int r = (st * 8 + warp) * R + seg;
+      const bool rv = r < rows;
+      const int64_t row = r0 + r;
+      float x[kMaxOct][8];
+#pragma unroll
+      for (int k = 0; k < kMaxOct; ++k) {
+        const int o = sl + LPR * k;
+        if (k < OPL && rv && o < CO) {
+          load_oct_smem<T>(sh + (size_t)r * row_bytes, o, lane, x[k]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) x[k][j] = 0.0f;
+        }
+      }
+      float s2 = s_g2, z2 = gmin, c_row = 0.0f;
+      const float *wrow = wcol;
+      if (KIND == KIND_PSQ) {
+        float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll
+        for (int k = 0; k < kMaxOct; ++k) {
+          if (k < OPL && rv && sl + LPR * k < CO) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              mm.x = fminf(mm.x, x[k][j]);
+              mm.y = fmaxf(mm.y, x[k][j]);
+            }
+          }
+        }
+        mm = seg_reduce(mm, LPR, OpMinMax());
+        s2 = affine_scale(mm.x, mm.y, B2);
+        z2 = mm.x;
+      } else if (KIND == KIND_BHQ) {
+        const int bb = rv ? r / nb : 0;
+        const float *bp = bpar + bb * 8;
+        const bool lead = rv && (r - bb * nb) == __float_as_int(bp[4]);
+        s2 = lead ? bp[0] : bp[1];
+        c_row = lead ? bp[2] - 1.0f : bp[2];
+        wrow = wcol + bb * C;
+        float tmin = INFINITY;
+#pragma unroll
+        for (int k = 0; k < kMaxOct; ++k) {
+          const int o = sl + LPR * k;
+          if (k < OPL && rv && o < CO) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              tmin = fminf(tmin, fmaf(-c_row, wrow[o * 8 + j], __fmul_rn(s2, x[k][j])));
+          }
+        }
+        z2 = seg_reduce(tmin, LPR, OpMin());
+      }
+      int rs2 = 0, rs1 = 0;
+#pragma unroll
+      for (int k = 0; k < kMaxOct; ++k) {
+        const int o = sl + LPR * k;
+        if (!(k < OPL && rv && o < CO)) continue;
+        const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)o;
+        uint32_t c[8];
+        const uint4 w2 = philox_oct(q, 0u, key);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float v;
+          if (KIND == KIND_BHQ) {
+            const float t = fmaf(-c_row, wrow[o * 8 + j], __fmul_rn(s2, x[k][j]));
+            v = __fsub_rn(t, z2);
+          } else {
+            v = __fmul_rn(__fsub_rn(x[k][j], z2), s2);
+          }
+          c[j] = sr_code(v, u16_of(w2, j), B2);
+          rs2 += (int)c[j];
+        }
+        if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+        if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + o * 8, c, (B2 + 1u) >> 1);
+        if (has_b1) {
+          const uint4 w1 = philox_oct(q, 1u, key);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float v = __fmul_rn(__fsub_rn(x[k][j], gmin), s_g1);
+            c[j] = sr_code(v, u16_of(w1, j), 255u);
+            rs1 += (int)c[j];
+          }
+          if (a.c1) store_codes8(a.c1 + row * (int64_t)C + o * 8, c);
+          if (a.f1) store_carriers8(a.f1 + row * (int64_t)C + o * 8, c, 128u);
+        }
+        if (want_cs) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) cs[k][j] += (int)c[j];
+        }
+      }
+      if (a.rsum2) rs2 = seg_reduce(rs2, LPR, OpAdd());
+      if (has_b1 && a.rsum1) rs1 = seg_reduce(rs1, LPR, OpAdd());
+      if (rv && sl == 0) {
+        if (a.rsum2) a.rsum2[row] = rs2;
+        if (has_b1 && a.rsum1) a.rsum1[row] = rs1;
+        if (KIND == KIND_PSQ) {
+          a.inv2[row] = __fdiv_rn(1.0f, s2);
+          a.zero2[row] = __fmul_rn(s2, z2);
+        } else if (KIND == KIND_BHQ) {
+          a.inv2[row] = s2 > 0.0f ? __fdiv_rn(1.0f, s2) : 0.0f;
+          a.zero2[row] = z2;
+        }
+      }
+    }
+    __syncthreads();  // the stage buffer and the BHQ tables are reused
+  }
+
+  // ---------------- column sums ----------------
+  if (want_cs) {
+#pragma unroll
+    for (int k = 0; k < kMaxOct; ++k) {
+      const int o = sl + LPR * k;
+      const bool valid = k < OPL && o < CO;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        // the segments of a warp own the same columns: fold them first
+        int v = valid ? cs[k][j] : 0;
+        for (int off = LPR; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if (valid && seg == 0 && v) atomicAdd(&csum_s[o * 8 + j], v);
+      }
+    }
+    __syncthreads();
+    for (int i = tid; i < C; i += kQ2Threads)
       if (csum_s[i]) atomicAdd(&csum_g[i], csum_s[i]);
   }
 }
@@ -550,6 +936,81 @@ fqt_status quant_geometry(QuantArgs &a, int num_sms, int *nth_out,
   *grid_out = (int)grid;
   *smem_out = smem;
   return FQT_OK;
+}
+
+// Geometry of the staged kernel; FQT_EUNSUPPORTED sends the call to k_quant.
+fqt_status quant2_geometry(QuantArgs &a, bool bf16, int num_sms, int *grid_out,
+                           size_t *smem_out) {
+  const int C = a.C;
+  if (C <= 0 || C % 8 || a.kind == KIND_DET) return FQT_EUNSUPPORTED;
+  const int CO = C / 8;
+  if (CO > 32 * kMaxOct) return FQT_EUNSUPPORTED;  // rows longer than 1024
+  const int esize = bf16 ? 2 : 4;
+  const int LPR = CO >= 32 ? 32 : pow2ceil(CO);
+  const int OPL = (CO + LPR - 1) / LPR;
+  const size_t row_bytes = (size_t)C * esize;
+  size_t stage = 32768;
+  int U, G;
+  if (a.kind == KIND_BHQ) {
+    const size_t blk = (size_t)a.block * row_bytes;
+    if (blk > stage) stage = (blk + 127) & ~(size_t)127;
+    if (stage > 98304) return FQT_EUNSUPPORTED;
+    U = (int)(stage / row_bytes / a.block) * a.block;
+    G = U / a.block;
+  } else {
+    U = (int)(stage / row_bytes);
+    G = 1;
+  }
+  if (U < 1) return FQT_EUNSUPPORTED;
+  a.CO = CO;
+  a.TW = LPR;
+  a.OPT = OPL;
+  a.RL = 32 / LPR;
+  a.RPL = 1;
+  a.GT = kQ2Threads;
+  a.G = G;
+  a.unit_rows = U;
+  a.nchunk = 1;
+  a.stage_bytes = (int)stage;
+  a.n_units = (a.N + U - 1) / U;
+  size_t smem = 2 * stage + 16 + sizeof(float2) * 8 + sizeof(int) * 8 +
+                sizeof(int) * (size_t)C + sizeof(float2) * (size_t)U +
+                sizeof(float) * 8 * (size_t)G;
+  if (a.kind == KIND_BHQ) smem += sizeof(float) * (size_t)G * C;
+  if (smem > 220 * 1024) return FQT_EUNSUPPORTED;
+  int per_sm = (int)((220 * 1024) / smem);
+  if (per_sm > 4) per_sm = 4;
+  if (per_sm < 1) per_sm = 1;
+  int64_t grid = (int64_t)num_sms * per_sm;
+  if (grid > a.n_units) grid = a.n_units;
+  if (grid < 1) grid = 1;
+  *grid_out = (int)grid;
+  *smem_out = smem;
+  return FQT_OK;
+}
+
+template <int KIND, typename T>
+static cudaError_t launch_quant2_t(const QuantArgs &a, int grid, size_t smem,
+                                   cudaStream_t st) {
+  auto fn = k_quant2<KIND, T>;
+  cudaError_t e = cudaFuncSetAttribute(
+      fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  fn<<<grid, kQ2Threads, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quant2(const QuantArgs &a, bool bf16, int grid, size_t smem,
+                          cudaStream_t st) {
+  switch (a.kind * 2 + (bf16 ? 1 : 0)) {
+    case KIND_PTQ * 2: return launch_quant2_t<KIND_PTQ, float>(a, grid, smem, st);
+    case KIND_PTQ * 2 + 1: return launch_quant2_t<KIND_PTQ, __nv_bfloat16>(a, grid, smem, st);
+    case KIND_PSQ * 2: return launch_quant2_t<KIND_PSQ, float>(a, grid, smem, st);
+    case KIND_PSQ * 2 + 1: return launch_quant2_t<KIND_PSQ, __nv_bfloat16>(a, grid, smem, st);
+    case KIND_BHQ * 2: return launch_quant2_t<KIND_BHQ, float>(a, grid, smem, st);
+    case KIND_BHQ * 2 + 1: return launch_quant2_t<KIND_BHQ, __nv_bfloat16>(a, grid, smem, st);
+  }
+  return cudaErrorInvalidValue;
 }
 
 template <int KIND, typename T>

@@ -38,7 +38,8 @@ class _QT(ctypes.Structure):
                 ("block", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("codes", ctypes.c_void_p), ("inv_s", ctypes.c_void_p),
                 ("zero", ctypes.c_void_p), ("row_sum", ctypes.c_void_p),
-                ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p)]
+                ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p),
+                ("codes_f16", ctypes.c_void_p)]
 
 
 def library_path() -> str:
@@ -62,6 +63,8 @@ def load(build_if_missing: bool = True):
         QP = ctypes.POINTER(_QT)
         lib.fqt_workspace_size.argtypes = [i64, i64, i64]
         lib.fqt_workspace_size.restype = sz
+        lib.fqt_debug_workspace_size.argtypes = [i64, i64, i64]
+        lib.fqt_debug_workspace_size.restype = sz
         for name in ("fqt_quantize_act", "fqt_quantize_weight"):
             f = getattr(lib, name)
             f.argtypes = [P, i32, i64, i64, i32, QP, P, sz, P]
@@ -78,12 +81,16 @@ def load(build_if_missing: bool = True):
         lib.fqt_debug_int_gemm.restype = i32
         lib.fqt_status_string.argtypes = [i32]
         lib.fqt_status_string.restype = ctypes.c_char_p
+        lib.fqt_last_cuda_error.argtypes = []
+        lib.fqt_last_cuda_error.restype = ctypes.c_char_p
         _lib = lib
         return lib
 
 
 def _check(st: int, what: str):
     if st != 0:
+        if st == 3:
+            what += " (" + load().fqt_last_cuda_error().decode() + ")"
         raise FqtError(st, what)
 
 
@@ -126,8 +133,13 @@ class Workspace:
 
 @dataclass
 class QTensor:
-    """A quantized matrix (the fqt_qtensor of include/fqt.h) held in torch tensors."""
-    codes: torch.Tensor
+    """A quantized matrix (the fqt_qtensor of include/fqt.h) held in torch tensors.
+
+    ``codes`` holds the integer codes (uint8), ``codes16`` the same codes
+    centred by 2^(b-1) as exact fp16 values (the tensor-core operand format);
+    either may be None.
+    """
+    codes: Optional[torch.Tensor]
     inv_s: torch.Tensor
     zero: torch.Tensor
     row_sum: Optional[torch.Tensor]
@@ -136,14 +148,23 @@ class QTensor:
     kind: int = PTQ
     bits: int = 8
     block: int = 0
+    codes16: Optional[torch.Tensor] = None
+
+    @property
+    def shape(self):
+        return (self.codes if self.codes is not None else self.codes16).shape
 
     @staticmethod
     def empty(rows: int, cols: int, kind: int, bits: int, block: int = 0,
-              row_sum: bool = True, col_sum: bool = True, device="cuda"):
+              row_sum: bool = True, col_sum: bool = True, device="cuda",
+              u8: bool = True, f16: bool = True):
         m = 1 if kind == PTQ else rows
         nblk = (rows + block - 1) // block if kind == BHQ else 0
         return QTensor(
-            codes=torch.empty((rows, cols), dtype=torch.uint8, device=device),
+            codes=(torch.empty((rows, cols), dtype=torch.uint8, device=device)
+                   if u8 else None),
+            codes16=(torch.empty((rows, cols), dtype=torch.float16, device=device)
+                     if f16 else None),
             inv_s=torch.empty(m, dtype=torch.float32, device=device),
             zero=torch.empty(m, dtype=torch.float32, device=device),
             row_sum=(torch.empty(rows, dtype=torch.int32, device=device)
@@ -155,17 +176,21 @@ class QTensor:
             kind=kind, bits=bits, block=block)
 
     def c_struct(self) -> _QT:
-        rows, cols = self.codes.shape
+        rows, cols = self.shape
+        p = lambda t: t.data_ptr() if t is not None else None
         return _QT(rows, cols, self.bits, self.kind, self.block, 0,
-                   self.codes.data_ptr(), self.inv_s.data_ptr(),
-                   self.zero.data_ptr(),
-                   self.row_sum.data_ptr() if self.row_sum is not None else None,
-                   self.col_sum.data_ptr() if self.col_sum is not None else None,
-                   self.lead.data_ptr() if self.lead is not None else None)
+                   p(self.codes), self.inv_s.data_ptr(), self.zero.data_ptr(),
+                   p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16))
+
+    def codes_from_f16(self) -> torch.Tensor:
+        """The uint8 codes recovered from the fp16 carriers."""
+        off = 1 << (self.bits - 1)
+        return (self.codes16.float() + off).round().to(torch.uint8)
 
     def to_numpy(self) -> dict:
         """Host copy in the oracle's dict layout."""
-        d = dict(codes=self.codes.cpu().numpy(), inv_s=self.inv_s.cpu().numpy(),
+        codes = self.codes if self.codes is not None else self.codes_from_f16()
+        d = dict(codes=codes.cpu().numpy(), inv_s=self.inv_s.cpu().numpy(),
                  zero=self.zero.cpu().numpy(), kind=self.kind, bits=self.bits,
                  block=self.block,
                  lead=self.lead.cpu().numpy() if self.kind == BHQ else None)
@@ -246,9 +271,9 @@ def linear_backward(q_b2: QTensor, q_b1: Optional[QTensor], qx: QTensor,
                     out_w: torch.Tensor = None, stream=None):
     """grad_X = Q_b2(dH) W~ and grad_W = Q_b1(dH)^T X~ (Eq. 6, App. E)."""
     lib = load()
-    N, C = q_b2.codes.shape
-    D = qx.codes.shape[1] if qx is not None else qw.codes.shape[1]
-    dev = q_b2.codes.device
+    N, C = q_b2.shape
+    D = qx.shape[1] if qx is not None else qw.shape[1]
+    dev = q_b2.inv_s.device
     ws = (ws or Workspace(N, C, D, device=dev)).ensure(N, C, D)
     gx = gw = None
     if grad_x:
@@ -277,8 +302,11 @@ def debug_int_gemm(A: torch.Tensor, a_kmajor: bool, a_bits: int, B: torch.Tensor
     """Exact sum_k (A_ik - 2^(a-1))(B_kj - 2^(b-1)) as int64 (M x N)."""
     lib = load()
     out = torch.empty((M, N), dtype=torch.int64, device=A.device)
-    ws = ws or Workspace(K, M, N, device=A.device)
-    ws.ensure(K, M, N)
+    need = int(lib.fqt_debug_workspace_size(M, N, K))
+    if ws is None or ws.nbytes < need:
+        ws = Workspace(1, 16, 16, device=A.device)
+        ws.nbytes = need
+        ws.buf = torch.zeros(need, dtype=torch.uint8, device=A.device)
     st = lib.fqt_debug_int_gemm(_ptr(A), int(a_kmajor), a_bits, _ptr(B),
                                 int(b_kmajor), b_bits, M, N, K, _ptr(out), ws.ptr,
                                 ws.nbytes, _stream(stream))

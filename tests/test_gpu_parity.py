@@ -127,6 +127,20 @@ def test_quantize_grad_matches_oracle(cfg, small, kind, bits, block):
         _check_b1(q1, dH, seed)
 
 
+@pytest.mark.parametrize("kind,bits,block", [(orc.PTQ, 4, 0), (orc.PSQ, 8, 0),
+                                             (orc.BHQ, 5, 16), (orc.BHQ, 5, 64)])
+def test_fp16_carriers_encode_the_codes(kind, bits, block):
+    """codes_f16 holds code - 2^(b-1) exactly, for both code sets."""
+    L = wl.config(2, batch=1)[0]
+    q2, q1 = fqt.quantize_grad(to_dev(L.dH), kind, bits, block, 9)
+    for q, b in ((q2, bits), (q1, 8)):
+        want = q.codes.to(torch.int32) - (1 << (b - 1))
+        got = q.codes16.float()
+        assert torch.equal(got, want.float())
+    qx = fqt.quantize_act(to_dev(L.X), 8)
+    assert torch.equal(qx.codes16.float(), qx.codes.float() - 128)
+
+
 def test_quantize_fwd_matches_oracle():
     L = wl.config(1, batch=2)[0]
     for M in (L.X, L.W):
