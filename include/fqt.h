@@ -142,6 +142,31 @@ FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,
                                float *grad_X, float *grad_W, void *workspace,
                                size_t ws_bytes, void *stream);
 
+/*
+ * grad_W = Q_b1(dH)^T X~ exactly as fqt_linear_backward computes it, for
+ * callers that cannot allocate device memory when they need the backward --
+ * a loop whose memory budget is frozen after warm-up, or a C host with no
+ * allocator of its own that must not call cudaMalloc (which may synchronise
+ * the device).  It takes no workspace: the split-K partials live in a fixed
+ * 8 MiB array inside the library, which every GPU that loads the library
+ * keeps until the process exits.  The paper has no counterpart; this is a
+ * deployment convenience.
+ *  - Limit: C * D * 4 bytes of partials per split must fit 8 MiB with few
+ *    enough splits to keep each below 2^31 / 2^(b1 + bx - 2) rows; larger
+ *    problems return FQT_EWORKSPACE without launching anything.
+ *  - The first call on a device looks up the array's device address (a
+ *    runtime call with that device current); make that first call before any
+ *    stream capture.
+ *  - All calls on a device share the array and it keeps the last call's
+ *    contents, so calls that overlap on the GPU (other streams, other host
+ *    threads) race and give wrong results: order them.
+ *  - Device-side conditions (a bounded wait that ran out) are not reported.
+ * Operands as for fqt_linear_backward (codes_f16, col_sum, 8-bit PTQ).
+ */
+FQT_API fqt_status fqt_grad_w_fixed_scratch(const fqt_qtensor *q_b1,
+                                            const fqt_qtensor *qx, float *grad_W,
+                                            void *stream);
+
 /* Synchronises `stream`, returns the first device-side condition recorded in
  * `workspace` since the previous call (or FQT_OK) and clears it. */
 FQT_API fqt_status fqt_sync_status(void *workspace, void *stream);

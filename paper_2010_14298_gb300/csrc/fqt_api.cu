@@ -221,6 +221,11 @@ fqt_status fqt_linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
                          reinterpret_cast<cudaStream_t>(stream));
 }
 
+fqt_status fqt_grad_w_fixed_scratch(const fqt_qtensor *q_b1, const fqt_qtensor *qx,
+                                    float *grad_W, void *stream) {
+  return grad_w_fixed_scratch(q_b1, qx, grad_W, reinterpret_cast<cudaStream_t>(stream));
+}
+
 fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
                               const uint8_t *Bm, int b_kmajor, int b_bits,
                               int64_t M, int64_t N, int64_t K, int64_t *out,

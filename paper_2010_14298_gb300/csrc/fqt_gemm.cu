@@ -983,4 +983,98 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
   return FQT_OK;
 }
 
+// ---------------------------------------------------------------------------
+// grad_W without a caller-provided workspace.
+//
+// Some callers cannot allocate device memory at the point where they need
+// the backward: for example a serving or training loop whose memory budget
+// is frozen after warm-up, or a plain C host that has no allocator of its
+// own to hand (and must not call cudaMalloc, which can synchronise the
+// device and stall other streams).  For them the split-K partials of grad_W
+// live in a fixed array inside the library.  Every GPU that loads the
+// library holds it until the process exits; all calls on a device share it.
+// ---------------------------------------------------------------------------
+constexpr size_t kFixedPartialBytes = (size_t)8 << 20;  // 8 MiB of int32 partials
+static __device__ __align__(256) unsigned char
+    g_fixed_scratch[kHeaderBytes + kFixedPartialBytes];
+
+// Device address of g_fixed_scratch on the current device, looked up once
+// per device (the host-side symbol is only a stand-in for it).
+static fqt_status fixed_scratch_address(void **out) {
+  static void *addr[64] = {nullptr};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "get device");
+  if (dev < 0 || dev >= 64) return FQT_EUNSUPPORTED;
+  if (!addr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_fixed_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "fixed scratch address");
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return FQT_OK;
+}
+
+fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
+                                float *grad_W, cudaStream_t st) {
+  if (!grad_W || !qa || !qx || !qa->codes_f16 || !qx->codes_f16 || !qa->col_sum ||
+      !qx->col_sum || !qa->inv_s || !qa->zero || !qx->inv_s || !qx->zero)
+    return FQT_EINVAL;
+  if (qa->kind != FQT_PTQ || qx->kind != FQT_PTQ) return FQT_EINVAL;
+  const int64_t Nr = qa->rows, C = qa->cols, D = qx->cols;
+  if (qx->rows != Nr || Nr < 0) return FQT_EINVAL;
+  if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
+  if (!aligned16(qa->codes_f16) || !aligned16(qx->codes_f16)) return FQT_EINVAL;
+  // the partials of every split must fit the fixed array
+  const size_t per_split = (size_t)C * (size_t)D * 4;
+  if (per_split == 0 || per_split > kFixedPartialBytes) return FQT_EWORKSPACE;
+  const int max_splits = (int)(kFixedPartialBytes / per_split);
+  SplitPlan p = plan_splits(C, D, Nr, qa->bits, qx->bits, device_sm_count(), true);
+  if (p.splits > max_splits) {
+    // fewer, longer splits; each must stay within the int32 partial bound
+    const int64_t max_terms = ((int64_t)1 << 31) >> (qa->bits + qx->bits - 2);
+    p.ks_blocks = (p.kb_total + max_splits - 1) / max_splits;
+    if (p.ks_blocks * BK > max_terms) return FQT_EWORKSPACE;
+    p.splits = (int)((p.kb_total + p.ks_blocks - 1) / p.ks_blocks);
+  }
+  void *base = nullptr;
+  fqt_status s = fixed_scratch_address(&base);
+  if (s != FQT_OK) return s;
+  int *status = static_cast<int *>(base);
+  int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(base) + kHeaderBytes);
+  // the status word must start each call at zero (the array keeps the last
+  // call's contents); the partials are fully rewritten by every split
+  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), st);
+  if (e != cudaSuccess) return cuda_fail(e, "fixed scratch clear");
+  if (Nr == 0) {
+    e = cudaMemsetAsync(grad_W, 0, per_split, st);
+    return cuda_fail(e, "grad_W clear");
+  }
+  GemmArgs g;
+  memset(&g, 0, sizeof(g));
+  g.status = status;
+  s = run_gemm(qa->codes_f16, 0, qa->bits, qx->codes_f16, 0, qx->bits, C, D, Nr, p, g,
+               part, true, st);
+  if (s != FQT_OK) return s;
+  ReduceArgs r;
+  memset(&r, 0, sizeof(r));
+  r.part = part;
+  r.splits = p.splits;
+  r.M = C;
+  r.N = D;
+  r.out_f32 = grad_W;
+  r.Kn = Nr;
+  r.oa = 1 << (qa->bits - 1);
+  r.ob = 1 << (qx->bits - 1);
+  r.cs_a = qa->col_sum;
+  r.cs_b = qx->col_sum;
+  r.inv_a = qa->inv_s;
+  r.zero_a = qa->zero;
+  r.inv_b = qx->inv_s;
+  r.zero_b = qx->zero;
+  launch_reduce(r, st);
+  return cuda_fail(cudaGetLastError(), "split-K reduce launch");
+}
+
 }  // namespace fqt

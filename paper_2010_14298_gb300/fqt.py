@@ -74,6 +74,8 @@ def load(build_if_missing: bool = True):
         lib.fqt_quantize_grad.restype = i32
         lib.fqt_linear_backward.argtypes = [QP, QP, QP, QP, P, P, P, sz, P]
         lib.fqt_linear_backward.restype = i32
+        lib.fqt_grad_w_fixed_scratch.argtypes = [QP, QP, P, P]
+        lib.fqt_grad_w_fixed_scratch.restype = i32
         lib.fqt_sync_status.argtypes = [P, P]
         lib.fqt_sync_status.restype = i32
         lib.fqt_debug_int_gemm.argtypes = [P, i32, i32, P, i32, i32, i64, i64,
@@ -294,6 +296,22 @@ def linear_backward(q_b2: QTensor, q_b1: Optional[QTensor], qx: QTensor,
                                  _stream(stream))
     _check(st, "fqt_linear_backward")
     return gx, gw
+
+
+def grad_w_fixed_scratch(q_b1: QTensor, qx: QTensor, out: torch.Tensor = None,
+                         stream=None) -> torch.Tensor:
+    """grad_W through fqt_grad_w_fixed_scratch: no workspace, the library's
+    fixed scratch array holds the split-K partials (for callers that cannot
+    allocate device memory at this point)."""
+    lib = load()
+    C, D = q_b1.shape[1], qx.shape[1]
+    if out is None:
+        out = torch.empty((C, D), dtype=torch.float32, device=q_b1.inv_s.device)
+    s1, sx = q_b1.c_struct(), qx.c_struct()
+    st = lib.fqt_grad_w_fixed_scratch(ctypes.byref(s1), ctypes.byref(sx), _ptr(out),
+                                      _stream(stream))
+    _check(st, "fqt_grad_w_fixed_scratch")
+    return out
 
 
 def debug_int_gemm(A: torch.Tensor, a_kmajor: bool, a_bits: int, B: torch.Tensor,
