@@ -179,6 +179,10 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   a.block = block;
   a.key0 = (uint32_t)seed;
   a.key1 = (uint32_t)(seed >> 32);
+  for (int r = 0; r < 10; ++r) {  // Philox4x32-10 round keys (Weyl sequence)
+    a.round_keys[2 * r] = a.key0 + (uint32_t)r * 0x9E3779B9u;
+    a.round_keys[2 * r + 1] = a.key1 + (uint32_t)r * 0xBB67AE85u;
+  }
   a.c2 = q_b2->codes;
   a.f2 = q_b2->codes_f16;
   a.inv2 = q_b2->inv_s;

@@ -38,21 +38,19 @@ __device__ __forceinline__ void record_status(int *status, int code) {
 // S-box, multipliers 0xD2511F53 / 0xCD9E8D57, Weyl key increments
 // 0x9E3779B9 / 0xBB67AE85.
 // ---------------------------------------------------------------------------
-struct PhiloxKey {
-  uint32_t k0, k1;
+// The ten round keys (k0 + r W0, k1 + r W1) depend on the seed only: the
+// host expands them once and they reach the kernels as launch parameters.
+struct PhiloxKeys {
+  uint32_t k[20];
 };
 
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, PhiloxKey key) {
-  uint32_t k0 = key.k0, k1 = key.k1;
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, const PhiloxKeys &key) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    const uint32_t lo0 = 0xD2511F53u * c.x;
-    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
-    const uint32_t lo1 = 0xCD9E8D57u * c.z;
-    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-    k0 += 0x9E3779B9u;
-    k1 += 0xBB67AE85u;
+    const uint64_t p0 = (uint64_t)0xD2511F53u * c.x;
+    const uint64_t p1 = (uint64_t)0xCD9E8D57u * c.z;
+    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ key.k[2 * r], (uint32_t)p1,
+                   (uint32_t)(p0 >> 32) ^ c.w ^ key.k[2 * r + 1], (uint32_t)p0);
   }
   return c;
 }
@@ -60,7 +58,7 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, PhiloxKey key) {
 // Eight 16-bit uniforms for the aligned group of 8 consecutive flat indices
 // starting at 8*q of `stream`: uniform i is half (i mod 2) of word i / 2.
 __device__ __forceinline__ uint4 philox_oct(uint64_t q, uint32_t stream,
-                                            PhiloxKey key) {
+                                            const PhiloxKeys &key) {
   return philox4x32_10(
       make_uint4((uint32_t)q, (uint32_t)(q >> 32), stream, 0u), key);
 }
@@ -73,11 +71,17 @@ __device__ __forceinline__ uint32_t u16_of(const uint4 &w, int i) {
 
 // Stochastic rounding of v >= 0 onto 0..B (Sec. 3.3): the probability
 // frac(v) is realised in 16-bit fixed point, code = (floor(v 2^16) + u) >> 16.
-__device__ __forceinline__ uint32_t sr_code(float v, uint32_t u16, uint32_t B) {
-  v = fminf(v, (float)(B + 1u));
-  const uint32_t fixed = __float2uint_rz(__fmul_rn(v, 65536.0f));
+// sr_code16 takes v * 2^16 (scaling by 2^16 is exact, so callers may fold it
+// into their scale factor).
+__device__ __forceinline__ uint32_t sr_code16(float v16, uint32_t u16, uint32_t B) {
+  v16 = fminf(v16, (float)((B + 1u) << 16));
+  const uint32_t fixed = __float2uint_rz(v16);
   const uint32_t code = (fixed + u16) >> 16;
   return min(code, B);
+}
+
+__device__ __forceinline__ uint32_t sr_code(float v, uint32_t u16, uint32_t B) {
+  return sr_code16(__fmul_rn(v, 65536.0f), u16, B);
 }
 
 // Scale B / R of the affine quantizers; R = 0 or an overflowing quotient
@@ -174,6 +178,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
   return ok != 0;
 }
 
+// try_wait that lets the hardware suspend the thread for up to `ns`
+// nanoseconds (it resumes as soon as the phase completes), so a waiting warp
+// does not take issue slots from the warps doing work.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t parity,
+                                                    uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
+      : "memory");
+  return ok != 0;
+}
+
 __device__ __forceinline__ uint64_t global_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -187,8 +207,8 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (;;) {
-    for (int i = 0; i < 64; ++i)
-      if (mbar_try_wait(bar, parity)) return true;
+    for (int i = 0; i < 8; ++i)
+      if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if (global_ns() - t0 > kWaitLimitNs) {
       record_status(status, FQT_ETIMEOUT);
       return false;

@@ -20,6 +20,7 @@ struct QuantArgs {
   int C, CO;
   int kind, bits, block;
   uint32_t key0, key1;
+  uint32_t round_keys[20];  // Philox4x32-10 key schedule of (key0, key1)
   // code set 2: Q_b2 (gradient) or the forward operand (KIND_DET)
   uint8_t *c2;
   uint16_t *f2;  // fp16 carriers of code set 2 (may be null)

@@ -206,6 +206,7 @@ __global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
   const uint32_t B2 = (1u << a.bits) - 1u;
   const float s_g2 = affine_scale(gmin, gmax, B2);    // PTQ / DET scale
   const float s_g1 = affine_scale(gmin, gmax, 255u);  // Q_b1 scale
+  const float s_g1_16 = __fmul_rn(s_g1, 65536.0f);
   const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
   if (blockIdx.x == 0 && tid == 0) {
     if (KIND == KIND_PTQ || KIND == KIND_DET) {
@@ -227,7 +228,9 @@ __global__ void __launch_bounds__(NTMAX) k_quant(const QuantArgs a) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) cs[k][j] = 0;
 
-  const PhiloxKey key = {a.key0, a.key1};
+  PhiloxKeys key;
+#pragma unroll
+  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
   float x[kMaxOct][8];
 
   for (int64_t ub = (int64_t)blockIdx.x * a.G; ub < a.n_units;
@@ -607,6 +610,7 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
   const uint32_t B2 = (1u << a.bits) - 1u;
   const float s_g2 = affine_scale(gmin, gmax, B2);
   const float s_g1 = affine_scale(gmin, gmax, 255u);
+  const float s_g1_16 = __fmul_rn(s_g1, 65536.0f);
   const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
   if (blockIdx.x == 0 && tid == 0) {
     if (KIND == KIND_PTQ) {
@@ -625,7 +629,9 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
   for (int k = 0; k < kMaxOct; ++k)
 #pragma unroll
     for (int j = 0; j < 8; ++j) cs[k][j] = 0;
-  const PhiloxKey key = {a.key0, a.key1};
+  PhiloxKeys key;
+#pragma unroll
+  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
 
   auto issue = [&](int64_t u, int b) {
     const int64_t r0 = u * U;
@@ -790,6 +796,7 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
         }
         z2 = seg_reduce(tmin, LPR, OpMin());
       }
+      const float s2_16 = __fmul_rn(s2, 65536.0f);
       int rs2 = 0, rs1 = 0;
 #pragma unroll
       for (int k = 0; k < kMaxOct; ++k) {
@@ -803,11 +810,11 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
           float v;
           if (KIND == KIND_BHQ) {
             const float t = fmaf(-c_row, wrow[o * 8 + j], __fmul_rn(s2, x[k][j]));
-            v = __fsub_rn(t, z2);
+            v = __fmul_rn(__fsub_rn(t, z2), 65536.0f);
           } else {
-            v = __fmul_rn(__fsub_rn(x[k][j], z2), s2);
+            v = __fmul_rn(__fsub_rn(x[k][j], z2), s2_16);  // = v 2^16 exactly
           }
-          c[j] = sr_code(v, u16_of(w2, j), B2);
+          c[j] = sr_code16(v, u16_of(w2, j), B2);
           rs2 += (int)c[j];
         }
         if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
@@ -816,8 +823,8 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
           const uint4 w1 = philox_oct(q, 1u, key);
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            const float v = __fmul_rn(__fsub_rn(x[k][j], gmin), s_g1);
-            c[j] = sr_code(v, u16_of(w1, j), 255u);
+            const float v = __fmul_rn(__fsub_rn(x[k][j], gmin), s_g1_16);
+            c[j] = sr_code16(v, u16_of(w1, j), 255u);
             rs1 += (int)c[j];
           }
           if (a.c1) store_codes8(a.c1 + row * (int64_t)C + o * 8, c);
