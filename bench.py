@@ -23,7 +23,6 @@ import os
 import statistics
 import subprocess
 import sys
-import tempfile
 import time
 
 import numpy as np
@@ -72,26 +71,55 @@ def _traffic_record(kernel: str):
 
 
 class Clocks:
-    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+    """Samples SM clocks and throttle reasons with nvidia-smi while running.
+
+    A reader thread stamps every sample with the host clock on arrival, so
+    the summary keeps only samples taken between mark_start() and
+    mark_end() (the timed region).  nvidia-smi is started before the region
+    and the caller waits for its first sample before starting the clock.
+    """
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
-    def __init__(self, index: int):
+    def __init__(self, index: int, period_ms: int = 50):
         self.index = index
+        self.period_ms = period_ms
         self.proc = None
-        self.file = None
+        self.rows = []  # (host time, fields)
+        self.t0 = self.t1 = None
+        self._thread = None
+
+    def _reader(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                self.rows.append((time.perf_counter(), parts))
 
     def __enter__(self):
+        import threading
         try:
-            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
-                stdout=self.file, stderr=subprocess.DEVNULL)
+                 "--format=csv,noheader,nounits", "-lms", str(self.period_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True, bufsize=1)
+            self._thread = threading.Thread(target=self._reader, daemon=True)
+            self._thread.start()
         except Exception:
             self.proc = None
         return self
+
+    def wait_first(self, timeout_s: float = 10.0):
+        t = time.perf_counter()
+        while self.proc is not None and not self.rows and time.perf_counter() - t < timeout_s:
+            time.sleep(0.01)
+
+    def mark_start(self):
+        self.t0 = time.perf_counter()
+
+    def mark_end(self):
+        self.t1 = time.perf_counter()
 
     def __exit__(self, *a):
         if self.proc is not None:
@@ -100,28 +128,30 @@ class Clocks:
                 self.proc.wait(timeout=5)
             except Exception:
                 self.proc.kill()
+            if self._thread is not None:
+                self._thread.join(timeout=2)
 
     def summary(self):
-        if self.proc is None or self.file is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
-        self.file.flush()
-        rows = []
-        for line in open(self.file.name):
-            parts = [p.strip() for p in line.split(",")]
-            if len(parts) >= 9:
-                rows.append(parts)
-        os.unlink(self.file.name)
-        if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
-        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
-                 "sw_power_cap"]
-        reasons = sorted({names[i] for r in rows for i in range(4)
+        if self.proc is None or not self.rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        t0 = self.t0 if self.t0 is not None else -1e30
+        t1 = self.t1 if self.t1 is not None else 1e30
+        inside = [r for t, r in self.rows if t0 <= t <= t1]
+        where = "timed region"
+        if not inside:  # region shorter than one period: the nearest sample after its start
+            after = [r for t, r in self.rows if t >= t0]
+            inside = after[:1] or [self.rows[-1][1]]
+            where = "first sample after the start of the timed region"
+        num = lambda v: v.replace(".", "", 1).isdigit()
+        sm = [float(r[1]) for r in inside if num(r[1])]
+        mx = [float(r[2]) for r in inside if num(r[2])]
+        pw = [float(r[3]) for r in inside if num(r[3])]
+        reasons = sorted({self.NAMES[i] for r in inside for i in range(4)
                           if r[5 + i].lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
-                "samples": len(rows)}
+                "power_w": statistics.median(pw) if pw else None,
+                "samples": len(inside), "sampled": where}
 
 
 def _dist():
@@ -162,7 +192,9 @@ def run_gpu(args):
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     names = ["quantize_act", "quantize_weight", "quantize_grad", "grad_x", "grad_w"]
-    launches_per_call = [2, 2, 2, 1, 2]
+    # range + codes; range + codes; range + BHQ codes + BHQ offsets; one
+    # contraction; contraction + split-K reduction
+    launches_per_call = [2, 2, 3 if KIND == 2 else 2, 1, 2]
 
     def step(seed, evs=None):
         def mark(i):
@@ -193,11 +225,14 @@ def run_gpu(args):
         dist.barrier()
     torch.cuda.synchronize()
     with Clocks(local) as clk:
+        clk.wait_first()
         t_wall = time.perf_counter()
+        clk.mark_start()
         for i in range(args.steps):
             flush.fill_(i & 0xFF)  # evict L2 between timed steps
             step(1000 + i, evs[i])
         torch.cuda.synchronize()
+        clk.mark_end()
         t_wall = time.perf_counter() - t_wall
     if world > 1:
         dist.barrier()
@@ -226,7 +261,7 @@ def run_gpu(args):
     alg_bytes = {
         "quantize_act": N * D * 4 + N * D * cb + D * 4,
         "quantize_weight": C * D * 4 + C * D * cb + D * 4,
-        "quantize_grad": N * C * 4 + 2 * N * C * cb + N * (4 + 4 + 4) + (N // BLOCK) * 4 + C * 4,
+        "quantize_grad": N * C * 4 + 2 * N * C * cb + N * (4 + 4 + 4 + 8) + (N // BLOCK) * 4 + C * 4,
         "grad_x": N * C * cb + C * D * cb + N * D * 4 + N * 12 + (N // BLOCK) * 4 + D * 4,
         "grad_w": N * C * cb + N * D * cb + C * D * 4 + (C + D) * 4,
     }
@@ -355,7 +390,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=5)

@@ -87,6 +87,13 @@ typedef struct fqt_qtensor {
                         code - 2^(b-1) as an IEEE fp16 bit pattern (exact),
                         the operand format of the tensor-core contractions;
                         NULL = not written.  Required by fqt_linear_backward. */
+  float *hz;         /* BHQ: rows entries, (Q_blk d)_i, where the offset
+                        2^(b-1) + zero_i = m_i + d_i with m_i = rint of its
+                        fp32 sum and |d_i| <= 1/2; NULL = not written; else
+                        unused.  With hr, required by fqt_linear_backward for
+                        a BHQ q_b2 with block > 1. */
+  float *hr;         /* BHQ: rows entries, (Q_blk R)_i with R_i = row_sum_i -
+                        cols 2^(b-1) + cols m_i */
 } fqt_qtensor;
 
 /* Bytes of workspace a layer with dH N x C, X N x D, W C x D needs for any
@@ -117,7 +124,8 @@ FQT_API fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t r
  * SR draws 16-bit uniforms from Philox4x32-10 keyed by `seed`, counter
  * (flat_index / 8, stream, 0), stream 0 for q_b2 and 1 for q_b1.
  * dH: N x C row-major, fp32 or bf16, C % 8 == 0.  BHQ: block a power of
- * two <= 128 and block * C <= 65536.
+ * two <= 128 and block * C <= 65536; q_b2->hz and q_b2->hr are written when
+ * non-NULL (row_sum must then be non-NULL too).
  */
 FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
                              int64_t C, fqt_kind kind, int bits, int block,
@@ -131,8 +139,9 @@ FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
  *   grad_W = Q_b1(dH)^T X~        (C x D, fp32, row-major; may be NULL)
  * The integer products of the codes are exact; dequantization and, for BHQ,
  * the inverse Householder transform of each block are applied in the
- * epilogue.  Reads the operands' codes_f16 and needs q_b2->row_sum,
- * qw->col_sum (grad_X) and q_b1->col_sum, qx->col_sum (grad_W).  q_b1 may be
+ * epilogue.  Reads the operands' codes_f16 and needs q_b2->row_sum (or, for
+ * BHQ with block > 1, q_b2->hz and q_b2->hr), qw->col_sum (grad_X) and
+ * q_b1->col_sum, qx->col_sum (grad_W).  q_b1 may be
  * NULL when q_b2 is PTQ with col_sum set: grad_W then uses q_b2.
  * C % 16 == 0 and D % 16 == 0.
  */

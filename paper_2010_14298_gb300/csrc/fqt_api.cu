@@ -141,6 +141,9 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   }
   if (N > 0 && q_b1 && ((!q_b1->codes && !q_b1->codes_f16) || !q_b1->inv_s || !q_b1->zero))
     return FQT_EINVAL;
+  // the grad_X offsets of BHQ (hz, hr) are reflected row sums: both or neither
+  const bool want_off = kind == FQT_BHQ && block > 1 && (q_b2->hz || q_b2->hr);
+  if (N > 0 && want_off && (!q_b2->hz || !q_b2->hr || !q_b2->row_sum)) return FQT_EINVAL;
   if (C % 8) return FQT_EUNSUPPORTED;
   if (!aligned(dH, 16) || !aligned(q_b2->codes, 16) || !aligned(q_b2->codes_f16, 16) ||
       (q_b1 && (!aligned(q_b1->codes, 16) || !aligned(q_b1->codes_f16, 16))))
@@ -208,13 +211,20 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
     QuantArgs a2 = a;  // staged kernel for rows of up to 1024 columns
     if (quant2_geometry(a2, bf16, nsm, &grid, &smem) == FQT_OK) {
       e = launch_quant2(a2, bf16, grid, smem, st);
-      return cuda_fail(e, "staged quantizer launch");
+      if (e != cudaSuccess) return cuda_fail(e, "staged quantizer launch");
+    } else {
+      s = quant_geometry(a, nsm, &nth, &grid, &smem);
+      if (s != FQT_OK) return s;
+      e = launch_quant(a, bf16, nth, grid, smem, st);
+      if (e != cudaSuccess) return cuda_fail(e, "quantizer launch");
     }
   }
-  s = quant_geometry(a, nsm, &nth, &grid, &smem);
-  if (s != FQT_OK) return s;
-  e = launch_quant(a, bf16, nth, grid, smem, st);
-  return cuda_fail(e, "quantizer launch");
+  if (want_off) {
+    e = launch_bhq_offsets(q_b2->zero, q_b2->row_sum, q_b2->lead, q_b2->hz, q_b2->hr, N,
+                           (int)C, bits, block, st);
+    if (e != cudaSuccess) return cuda_fail(e, "BHQ offsets launch");
+  }
+  return FQT_OK;
 }
 
 fqt_status fqt_linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,

@@ -226,4 +226,77 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// ---------------------------------------------------------------------------
+// Float-float arithmetic (an unevaluated sum h + l of two fp32 values, about
+// 48 significant bits) from the error-free transformations of Knuth (two-sum),
+// Dekker (fast two-sum) and the fused multiply-add product error.  The
+// inverse Householder transform of BHQ subtracts nearly equal quantities;
+// carrying them in float-float keeps the result accurate to fp32 rounding of
+// the result itself.
+// ---------------------------------------------------------------------------
+struct ff {
+  float h, l;
+};
+
+__device__ __forceinline__ ff two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return {s, e};
+}
+
+// requires |a| >= |b| (or a == 0)
+__device__ __forceinline__ ff fast_two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  return {s, __fsub_rn(b, __fsub_rn(s, a))};
+}
+
+__device__ __forceinline__ ff two_prod(float a, float b) {
+  const float p = __fmul_rn(a, b);
+  return {p, __fmaf_rn(a, b, -p)};
+}
+
+__device__ __forceinline__ ff ff_add(ff x, ff y) {
+  const ff s = two_sum(x.h, y.h);
+  return fast_two_sum(s.h, __fadd_rn(s.l, __fadd_rn(x.l, y.l)));
+}
+
+__device__ __forceinline__ ff ff_neg(ff x) { return {-x.h, -x.l}; }
+
+__device__ __forceinline__ ff ff_mul(ff x, ff y) {
+  const ff p = two_prod(x.h, y.h);
+  return fast_two_sum(p.h, __fmaf_rn(x.h, y.l, __fmaf_rn(x.l, y.h, p.l)));
+}
+
+// An integer (|v| < 2^53) as float-float, exactly for |v| < 2^48.
+__device__ __forceinline__ ff ff_from_int(long long v) {
+  const float h = __ll2float_rn(v);
+  return {h, __ll2float_rn(v - (long long)h)};
+}
+
+__device__ __forceinline__ float ff_round(ff x) { return __fadd_rn(x.h, x.l); }
+
+// Constants of the block Householder reflection of n >= 2 rows (Sec. 4.2):
+// rho = 1/sqrt(n) (the entries of n = rho 1 - e_p besides the lead) and
+// kappa = rho / (1 - rho) = 2 rho / ||n||^2, both in float-float.
+struct HhConst {
+  ff rho, kap;
+};
+
+__device__ __forceinline__ HhConst hh_const(int n) {
+  const float nf = (float)n;
+  const float rh = __fdiv_rn(1.0f, __fsqrt_rn(nf));
+  // one Newton step on 1/sqrt(n): rho = rh (1 + r / 2) with r = 1 - n rh^2
+  const ff p = two_prod(rh, rh);
+  const float r = __fsub_rn(__fmaf_rn(-nf, p.h, 1.0f), __fmul_rn(nf, p.l));
+  HhConst c;
+  c.rho = fast_two_sum(rh, __fmul_rn(__fmul_rn(0.5f, rh), r));
+  // kappa = rho / (1 - rho): quotient and one correction
+  const ff om = ff_add({1.0f, 0.0f}, ff_neg(c.rho));
+  const float q1 = __fdiv_rn(c.rho.h, om.h);
+  const ff rem = ff_add(c.rho, ff_neg(ff_mul({q1, 0.0f}, om)));
+  c.kap = fast_two_sum(q1, __fdiv_rn(rem.h, om.h));
+  return c;
+}
+
 }  // namespace fqt

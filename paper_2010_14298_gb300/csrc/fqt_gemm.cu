@@ -25,6 +25,7 @@
 #include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
+#include <math.h>
 #include <string.h>
 
 #include "fqt_common.cuh"
@@ -37,20 +38,20 @@ constexpr int kMaxStages = 8;  // operand stages (A and B fp16 tiles), chosen pe
 constexpr int kGemmThreads = 320;
 constexpr int kWarpTma = 0, kWarpMma = 1, kWarpEpi0 = 2;
 constexpr int kNumEpiWarps = 8;
-// two 128-column fp32 accumulators and one 128-column int32 running sum
+// two 128-column fp32 accumulators and 256 columns of int32 running sums
 constexpr uint32_t kTmemCols = 512;
 
 constexpr size_t kTileBytes = 16384;  // one 128 x 64 fp16 operand tile
 constexpr size_t kBoxBytes = 4096;   // one 32 x 32 fp32 / int32 output box
 // Shared memory, from a 1024-byte-aligned base:
-//   [0, kFixedBytes)           epilogue tables and barriers
+//   [0, kFixedBytes)           per-warp epilogue tables and barriers
 //   [kFixedBytes, +S * 32 KiB) S operand stages (A, B)
 //   [..., + 8 * R * 4 KiB)     R output boxes per epilogue warp (TMA store ring)
-constexpr size_t kOffCol = 0;                              // [8 warps] 64 + 64 floats
-constexpr size_t kOffRow = kOffCol + kNumEpiWarps * 512;   // [8 warps] 3 x 32 floats
-constexpr size_t kOffBhq = kOffRow + kNumEpiWarps * 384;   // [2][2][4][32] floats
-constexpr size_t kOffBar = kOffBhq + 2 * 2 * 4 * 32 * sizeof(float);
-constexpr size_t kNumBars = 2 * kMaxStages + 6;
+constexpr size_t kOffKp = 0;                                        // [8 warps][BN] float4
+constexpr size_t kOffLead = kOffKp + kNumEpiWarps * BN * 16;        // [8 warps][BN] int
+constexpr size_t kOffMsum = kOffLead + kNumEpiWarps * BN * 4;       // [8 warps][BN] int
+constexpr size_t kOffBar = kOffMsum + kNumEpiWarps * BN * 4;
+constexpr size_t kNumBars = 2 * kMaxStages + 4;
 constexpr size_t kFixedBytes = (kOffBar + kNumBars * 8 + 16 + 1023) & ~(size_t)1023;
 
 __host__ __device__ constexpr size_t gemm_smem_bytes(int stages, int ring) {
@@ -58,23 +59,27 @@ __host__ __device__ constexpr size_t gemm_smem_bytes(int stages, int ring) {
          (size_t)kNumEpiWarps * ring * kBoxBytes + 1024;  // + alignment slack
 }
 
+// MODE_GRADX: grad_X^T = W~^T Q_b2(dH)^T, i.e. M = D (output columns of
+// grad_X, TMEM lanes), N = rows of dH (TMEM columns), K = C, with the
+// dequantizing epilogue.  MODE_PARTIAL: raw int32 split-K partials.
 enum { MODE_GRADX = 0, MODE_PARTIAL = 1 };
 
 struct GemmArgs {
   int64_t M, N, K;            // out is M x N, reduction over K
   int a_kmajor, b_kmajor;     // operand storage (see fqt_debug_int_gemm)
   uint32_t mn_lbo, mn_sbo;    // MN-major descriptor strides (bytes)
-  int oa, ob;                 // centring offsets 2^(b-1)
   int kc_blocks;              // K-blocks per exact chunk
   int m_tiles, n_tiles, splits;
   int64_t ks_blocks, kb_total;
   int64_t n_items;
-  int mode;
   int stages, ring;           // operand stages, output boxes per epilogue warp
-  // grad_X epilogue (MODE_GRADX)
-  int kind, block;
-  const float *inv_s, *zero;   // Q_b2 metadata (1 or M entries)
+  // grad_X epilogue (MODE_GRADX); rows of Q_b2 are the N dimension
+  int kind;
+  int og, ow;                  // centring offsets 2^(b-1) of Q_b2 and W~ codes
+  const float *inv_s, *zero;   // Q_b2 metadata (1 or N entries)
   const int32_t *row_sum, *lead;
+  const float *hz, *hr;        // BHQ offsets (block > 1)
+  float flt_mmax;              // largest |m| of a tile for the fp32 form
   const int32_t *col_sum_w;    // W~ column sums over C
   const float *inv_sw, *zero_w;
   int *status;
@@ -221,10 +226,46 @@ __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+// 32 columns of this warp's 32 lanes, without waiting (see tmem_wait_ld).
+__device__ __forceinline__ void tmem_ld32_nw(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+        "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+        "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]),
+        "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+
+// One column of this warp's 32 lanes, without waiting.
+__device__ __forceinline__ uint32_t tmem_ld1_nw(uint32_t taddr) {
+  uint32_t v;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(v) : "r"(taddr));
+  return v;
+}
+
+// Waits for every tcgen05.ld this thread has issued.  The registers of the
+// loads are passed through so that no use is scheduled before the wait.
+template <int NR>
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[NR]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < NR; ++i) asm volatile("" : "+r"(r[i]));
+}
+
 // Byte offset of the 16-byte chunk `chunk` of row `row` in a 128-byte-swizzled
 // K-major tile (rows of 128 bytes, 1024-byte atoms of 8 rows).
 __device__ __forceinline__ uint32_t sw128_off(int row, int chunk) {
   return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+// Element (row, col) of a 32 x 32 fp32 output box in the 128-byte swizzle.
+__device__ __forceinline__ void st_box(uint8_t *tile, int row, int col, float v) {
+  *reinterpret_cast<float *>(tile + sw128_off(row, col >> 2) + ((col & 3) << 2)) = v;
 }
 
 struct Item {
@@ -245,22 +286,677 @@ __device__ __forceinline__ Item decode_item(const GemmArgs &g, int64_t it) {
   return r;
 }
 
-// Inverse Householder of the row blocks of one column of a 32-row box:
-// (Q V)_k = V_k - c_k w with w = sum_k e_k V_k over each block of NB rows,
-// then the row scale; rowv holds e_k, c_k and the scale of the 32 rows.
-template <int NB>
-__device__ __forceinline__ void householder_cols(float (&colv)[32], const float *rowv) {
+// ---------------------------------------------------------------------------
+// grad_X epilogue.  The accumulator holds P^T: TMEM lane = output column j of
+// grad_X, TMEM column = row k of dH, so each thread owns one column j and the
+// rows of a BHQ block are consecutive registers of one thread.
+//
+// Dequantization (Eq. 9).  With a the centred codes of Q_b2 (code - 2^(b-1)),
+// w those of W~, the row offset 2^(b-1) + z'_k = m_k + d_k (m_k an integer,
+// |d_k| <= 1/2) and y = 2^(bw-1) + z_w,
+//   V_kj = sum_c (a_kc + m_k + d_k)(w_cj + y) = I_kj + y R_k + d_k U_j,
+//   I_kj = P_kj + m_k CWc_j (an exact integer), CWc_j = sum_c w_cj,
+//   R_k = sum_c (a_kc + m_k), U_j = CWc_j + C y = col_sum_w_j + C z_w,
+// and grad_X = inv_sw diag(inv_s) Q_blk V.  The reflection is linear in the
+// rows: Q V = Q I + y (Q R) 1^T + (Q d) U^T, with Q R and Q d per row (hr,
+// hz; the identity for PTQ / PSQ).  Per block of nb rows with lead p,
+//   (Q I)_k = I_k - beta (k != p),  (Q I)_p = rho S,
+//   S = sum_k I_k, beta = kappa (rho S - I_p), rho = 1/sqrt(nb),
+//   kappa = rho / (1 - rho).
+// S and I_p are exact integers, beta is formed in float-float and split into
+// an integer and a remainder, so I_k - beta loses nothing to the cancellation
+// of the reflection: every term left in fp32 is small or row-constant.
+//
+// Two forms of the integer part: F (fp32, every |I| below 2^24 / (2 +
+// sqrt(nb)): one exact chunk and |m_k| <= mmax, checked per tile) and
+// integer (int64 arithmetic, any size).
+// ---------------------------------------------------------------------------
+// beta = kappa (rho S - I_p) split as bi + bf (bi an integer) and the lead
+// value rho S, for a block of nact >= 2 rows.
+struct BlockFix {
+  float bi, bf, lead;
+  long long bil;
+};
+
+__device__ __forceinline__ BlockFix block_fix(const HhConst &c, long long S, long long Ip) {
+  const ff rS = ff_mul(c.rho, ff_from_int(S));
+  const ff w = ff_add(rS, ff_neg(ff_from_int(Ip)));
+  const ff beta = ff_mul(c.kap, w);
+  BlockFix f;
+  f.bi = rintf(beta.h);
+  f.bf = __fadd_rn(__fsub_rn(beta.h, f.bi), beta.l);
+  f.bil = (long long)f.bi;
+  f.lead = ff_round(rS);
+  return f;
+}
+
+// out = sc (t + hz U) + sc y hr, with kq = (sc, sc hz, sc y hr, m)
+__device__ __forceinline__ float dequant(const float4 &kq, float t, float U) {
+  return __fmaf_rn(kq.x, t, __fmaf_rn(kq.y, U, kq.z));
+}
+
+// The integer parts I of 32 rows (one box) of this thread's column.
+//   F form: fp32 values, I = P + m CWc (one exact fma).
+//   integer form: int64, I = P + m CWc with P folded over chunks.
+template <bool F>
+struct Ints;
+
+template <>
+struct Ints<true> {
+  float v[32];
+  __device__ __forceinline__ long long ll(int i) const { return (long long)v[i]; }
+  __device__ __forceinline__ float f(int i) const { return v[i]; }
+  __device__ __forceinline__ float minus(int i, const BlockFix &b) const {
+    return __fsub_rn(__fsub_rn(v[i], b.bi), b.bf);
+  }
+};
+
+template <>
+struct Ints<false> {  // the int32 products; I = P + m CWc formed on use
+  int v[32];
+  const float4 *kp;
+  long long cw;
+  __device__ __forceinline__ long long ll(int i) const {
+    return (long long)v[i] + (long long)kp[i].w * cw;
+  }
+  __device__ __forceinline__ float f(int i) const { return __ll2float_rn(ll(i)); }
+  __device__ __forceinline__ float minus(int i, const BlockFix &b) const {
+    return __fsub_rn(__ll2float_rn(ll(i) - b.bil), b.bf);
+  }
+};
+
+// Loads the products of the 32 rows at TMEM column c0 and forms I.
+template <bool F>
+__device__ __forceinline__ void load_ints(uint32_t acc, uint32_t ints, bool multi, int c0,
+                                          const float4 *kp, float cwc, Ints<F> &I) {
+  uint32_t r[32];
+  tmem_ld32_nw(acc + (uint32_t)c0, r);
+  if constexpr (F) {
+    tmem_wait_ld(r);
 #pragma unroll
-  for (int b0 = 0; b0 < 32; b0 += NB) {
-    float w = 0.0f;
+    for (int i = 0; i < 32; ++i) I.v[i] = __fmaf_rn(kp[c0 + i].w, cwc, __uint_as_float(r[i]));
+  } else {
+    uint32_t s[32];
+    if (multi) tmem_ld32_nw(ints + (uint32_t)c0, s);
+    tmem_wait_ld(r);
+    if (multi) tmem_wait_ld(s);
+    I.kp = kp + c0;
+    I.cw = (long long)cwc;
 #pragma unroll
-    for (int r = 0; r < NB; ++r) w = fmaf(rowv[b0 + r], colv[b0 + r], w);
-#pragma unroll
-    for (int r = 0; r < NB; ++r)
-      colv[b0 + r] = rowv[64 + b0 + r] * fmaf(-rowv[32 + b0 + r], w, colv[b0 + r]);
+    for (int i = 0; i < 32; ++i)
+      I.v[i] = __float2int_rn(__uint_as_float(r[i])) + (multi ? (int)s[i] : 0);
   }
 }
 
+// I of one row (TMEM column col) of this thread's column.
+template <bool F>
+__device__ __forceinline__ long long load_int1(uint32_t acc, uint32_t ints, bool multi,
+                                               int col, float m, float cwc) {
+  uint32_t v[2];
+  v[0] = tmem_ld1_nw(acc + (uint32_t)col);
+  v[1] = (!F && multi) ? tmem_ld1_nw(ints + (uint32_t)col) : 0u;
+  tmem_wait_ld(v);
+  if (F) return (long long)__fmaf_rn(m, cwc, __uint_as_float(v[0]));
+  long long P = __float2int_rn(__uint_as_float(v[0]));
+  if (multi) P += (int)v[1];
+  return P + (long long)m * (long long)cwc;
+}
+
+// One box (32 rows r0 .. r0 + 31 of the tile) of blocks of NB <= 32 rows:
+// reflection, dequantization, store into the swizzled box.
+// lead products loaded per box: one per block of NB <= 32 rows
+__host__ __device__ constexpr int leads_per_box(int nb) { return nb > 1 && nb <= 32 ? 32 / nb : 1; }
+
+template <int NB, bool F>
+__device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip)[leads_per_box(NB)],
+                                          const HhConst &hc, const float4 *kp,
+                                          const int *leads, int r0, int64_t row0,
+                                          int64_t N, float U, uint8_t *tile, int lane) {
+  if (NB == 1) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) st_box(tile, i, lane, dequant(kp[r0 + i], I.f(i), U));
+    return;
+  }
+  constexpr int NBB = NB > 1 ? NB : 2;
+#pragma unroll
+  for (int b = 0; b < 32 / NBB; ++b) {
+    const int kb0 = r0 + b * NBB;
+    const int64_t left = N - (row0 + b * NBB);
+    const int nact = left >= NBB ? NBB : (int)(left > 0 ? left : 0);
+    if (nact < 2) {  // a one-row block is not transformed
+#pragma unroll
+      for (int l = 0; l < NBB; ++l)
+        st_box(tile, b * NBB + l, lane, dequant(kp[kb0 + l], I.f(b * NBB + l), U));
+      continue;
+    }
+    long long S = 0;
+#pragma unroll
+    for (int l = 0; l < NBB; ++l) S += I.ll(b * NBB + l);
+    const BlockFix f = block_fix(nact == NBB ? hc : hh_const(nact), S, Ip[b]);
+#pragma unroll
+    for (int l = 0; l < NBB; ++l)
+      st_box(tile, b * NBB + l, lane, dequant(kp[kb0 + l], I.minus(b * NBB + l, f), U));
+    const int p = leads[kb0 / NBB];  // the lead row: a later store of the same thread
+    st_box(tile, b * NBB + p, lane, dequant(kp[kb0 + p], f.lead, U));
+  }
+}
+
+// The final chunk of one tile for this warp: groups of GW rows (a box, or
+// one block of NB > 32 rows spanning several boxes).
+template <int NB, bool F>
+__device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uint32_t acc,
+                                           uint32_t ints, bool multi, const float4 *kp,
+                                           const int *leads, const HhConst &hc, float cwc,
+                                           float U, uint8_t *myring, int &nbox,
+                                           uint64_t *acce_set, const CUtensorMap *tmOut,
+                                           int q, int lane) {
+  constexpr int GW = NB > 32 ? NB : 32;
+  constexpr int NPP = leads_per_box(NB);
+#pragma unroll 1
+  for (int g0 = 0; g0 < BN; g0 += GW) {
+    // blocks of more than 32 rows: their sums over all boxes first
+    long long S_big = 0, Ip_big = 0;
+    int p_big = 0;
+    if (NB > 32) {
+#pragma unroll 1
+      for (int bx = 0; bx < GW / 32; ++bx) {
+        Ints<F> I;
+        load_ints<F>(acc, ints, multi, g0 + bx * 32, kp, cwc, I);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) S_big += I.ll(i);
+      }
+      p_big = leads[g0 / (NB > 32 ? NB : 1)];
+      Ip_big = load_int1<F>(acc, ints, multi, g0 + p_big, kp[g0 + p_big].w, cwc);
+    }
+#pragma unroll 1
+    for (int bx = 0; bx < GW / 32; ++bx) {
+      const int r0 = g0 + bx * 32;
+      uint8_t *tile = myring + (size_t)(nbox % g.ring) * kBoxBytes;
+      if (nbox >= g.ring) {
+        if (lane == 0) bulk_wait_read(g.ring - 1);
+        __syncwarp();
+      }
+      Ints<F> I;
+      load_ints<F>(acc, ints, multi, r0, kp, cwc, I);
+      long long Ip[NPP];
+#pragma unroll
+      for (int b = 0; b < NPP; ++b) {
+        Ip[b] = 0;
+        if (NB > 1 && NB <= 32) {
+          const int col = r0 + b * (32 / NPP) + leads[(r0 + b * (32 / NPP)) / (32 / NPP)];
+          Ip[b] = load_int1<F>(acc, ints, multi, col, kp[col].w, cwc);
+        }
+      }
+      if (r0 + 32 == BN) {  // the accumulator has been read in full
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acce_set);
+      }
+      if constexpr (NB <= 32) {
+        box_small<NB, F>(I, Ip, hc, kp, leads, r0, t.n0 + r0, g.N, U, tile, lane);
+      } else {
+        const int64_t left = g.N - (t.n0 + g0);
+        const int nact = left >= NB ? NB : (int)(left > 0 ? left : 0);
+        if (nact < 2) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) st_box(tile, i, lane, dequant(kp[r0 + i], I.f(i), U));
+        } else {
+          const BlockFix f = block_fix(nact == NB ? hc : hh_const(nact), S_big, Ip_big);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            st_box(tile, i, lane, dequant(kp[r0 + i], I.minus(i, f), U));
+          if (p_big >= bx * 32 && p_big < bx * 32 + 32)
+            st_box(tile, p_big - bx * 32, lane, dequant(kp[g0 + p_big], f.lead, U));
+        }
+      }
+      // hand the box to the TMA engine: rows t.n0 + r0 .., columns 32q ..
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(tmOut, (int32_t)(t.m0 + q * 32), (int32_t)(t.n0 + r0), tile);
+        bulk_commit();
+      }
+      ++nbox;
+    }
+  }
+}
+
+// fp32 integers of magnitude below 2^22 to int32 with one FADD: x + 1.5 2^23
+// holds x in its low mantissa bits.  (Conversions to and from 64-bit
+// integers run on the FP64 pipe, which is slow on this GPU; the fp32 form
+// uses none per element.)
+constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
+constexpr uint32_t kMagicBits = 0x4B400000u;
+
+__device__ __forceinline__ uint32_t magic_bits(float x) {
+  return __float_as_uint(__fadd_rn(x, kMagic));
+}
+
+__device__ __forceinline__ int magic_int(float x) { return (int)(magic_bits(x) - kMagicBits); }
+
+// An int32 as float-float (exact).
+__device__ __forceinline__ ff ff_from_i32(int v) {
+  const float h = __int2float_rn(v);
+  return {h, __int2float_rn(v - __float2int_rz(h))};
+}
+
+struct BlockFixF {
+  float bi, bf, lead;
+};
+
+__device__ __forceinline__ BlockFixF block_fix_f(const HhConst &c, int S, int Ip) {
+  const ff rS = ff_mul(c.rho, ff_from_i32(S));
+  const ff w = ff_add(rS, ff_neg(ff_from_i32(Ip)));
+  const ff beta = ff_mul(c.kap, w);
+  BlockFixF f;
+  f.bi = rintf(beta.h);
+  f.bf = __fadd_rn(__fsub_rn(beta.h, f.bi), beta.l);
+  f.lead = ff_round(rS);
+  return f;
+}
+
+// (Q I)_k of a non-lead row in the fp32 form: (P - bi) + m CWc is exact
+// (every magnitude below 2^24), then the remainder bf.
+__device__ __forceinline__ float reflect_f(float P, const float4 &kq, float cwc,
+                                           const BlockFixF &f) {
+  return __fsub_rn(__fmaf_rn(kq.w, cwc, __fsub_rn(P, f.bi)), f.bf);
+}
+
+// The final chunk of one tile in the fp32 form (one exact chunk, |P| < 2^22,
+// |m| <= mmax).  Block sums S = sum P + CWc sum m, I_p = P_p + m_p CWc.
+template <int NB>
+__device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, uint32_t acc,
+                                             const float4 *kp, const int *leads,
+                                             const int *msum, const HhConst &hc, float cwc,
+                                             float U, uint8_t *myring, int &nbox,
+                                             uint64_t *acce_set, const CUtensorMap *tmOut,
+                                             int q, int lane) {
+  constexpr int GW = NB > 32 ? NB : 32;
+  constexpr int NPP = leads_per_box(NB);
+  constexpr int NBD = NB > 1 ? NB : 1;
+  const int cwi = (int)cwc;
+#pragma unroll 1
+  for (int g0 = 0; g0 < BN; g0 += GW) {
+    int S_big = 0, Ip_big = 0, p_big = 0;
+    if constexpr (NB > 32) {
+      uint32_t sb = 0u;
+#pragma unroll 1
+      for (int bx = 0; bx < GW / 32; ++bx) {
+        uint32_t r[32];
+        tmem_ld32_nw(acc + (uint32_t)(g0 + bx * 32), r);
+        tmem_wait_ld(r);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) sb += magic_bits(__uint_as_float(r[i]));
+      }
+      S_big = (int)(sb - (uint32_t)NB * kMagicBits) + cwi * msum[g0 / NBD];
+      p_big = leads[g0 / NBD];
+      uint32_t v[1];
+      v[0] = tmem_ld1_nw(acc + (uint32_t)(g0 + p_big));
+      tmem_wait_ld(v);
+      Ip_big = magic_int(__uint_as_float(v[0])) + (int)kp[g0 + p_big].w * cwi;
+    }
+#pragma unroll 1
+    for (int bx = 0; bx < GW / 32; ++bx) {
+      const int r0 = g0 + bx * 32;
+      uint8_t *tile = myring + (size_t)(nbox % g.ring) * kBoxBytes;
+      if (nbox >= g.ring) {
+        if (lane == 0) bulk_wait_read(g.ring - 1);
+        __syncwarp();
+      }
+      uint32_t r[32];
+      tmem_ld32_nw(acc + (uint32_t)r0, r);
+      uint32_t pp[NPP];
+#pragma unroll
+      for (int b = 0; b < NPP; ++b)
+        pp[b] = (NB > 1 && NB <= 32)
+                    ? tmem_ld1_nw(acc + (uint32_t)(r0 + b * NBD + leads[(r0 + b * NBD) / NBD]))
+                    : 0u;
+      tmem_wait_ld(r);
+      tmem_wait_ld(pp);
+      if (r0 + 32 == BN) {  // the accumulator has been read in full
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acce_set);
+      }
+      // every output of the box is formed in registers before the first
+      // store, so the per-row loads from shared memory need not wait for
+      // the stores into the (possibly aliasing) box
+      float o[32];
+      int lead_row = -1;
+      float lead_val = 0.0f;
+      if constexpr (NB == 1) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float4 kq = kp[r0 + i];
+          o[i] = dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U);
+        }
+      } else if constexpr (NB <= 32) {
+        float lv[32 / NBD];
+        int lp[32 / NBD];
+#pragma unroll
+        for (int b = 0; b < 32 / NBD; ++b) {
+          const int kb0 = r0 + b * NBD;
+          const int64_t left = g.N - (t.n0 + kb0);
+          const int nact = left >= NBD ? NBD : (int)(left > 0 ? left : 0);
+          lp[b] = -1;
+          lv[b] = 0.0f;
+          if (nact < 2) {  // a one-row block is not transformed
+#pragma unroll
+            for (int l = 0; l < NBD; ++l) {
+              const float4 kq = kp[kb0 + l];
+              o[b * NBD + l] = dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[b * NBD + l])), U);
+            }
+            continue;
+          }
+          uint32_t sb = 0u;
+#pragma unroll
+          for (int l = 0; l < NBD; ++l) sb += magic_bits(__uint_as_float(r[b * NBD + l]));
+          const int S = (int)(sb - (uint32_t)NBD * kMagicBits) + cwi * msum[kb0 / NBD];
+          const int p = leads[kb0 / NBD];
+          const int Ip = magic_int(__uint_as_float(pp[b])) + (int)kp[kb0 + p].w * cwi;
+          const BlockFixF f = block_fix_f(nact == NBD ? hc : hh_const(nact), S, Ip);
+#pragma unroll
+          for (int l = 0; l < NBD; ++l) {
+            const float4 kq = kp[kb0 + l];
+            o[b * NBD + l] = dequant(kq, reflect_f(__uint_as_float(r[b * NBD + l]), kq, cwc, f), U);
+          }
+          lp[b] = b * NBD + p;
+          lv[b] = dequant(kp[kb0 + p], f.lead, U);
+        }
+#pragma unroll
+        for (int i = 0; i < 32; ++i) st_box(tile, i, lane, o[i]);
+        // the lead rows: later stores of the same thread
+#pragma unroll
+        for (int b = 0; b < 32 / NBD; ++b)
+          if (lp[b] >= 0) st_box(tile, lp[b], lane, lv[b]);
+      } else {
+        const int64_t left = g.N - (t.n0 + g0);
+        const int nact = left >= NB ? NB : (int)(left > 0 ? left : 0);
+        if (nact < 2) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float4 kq = kp[r0 + i];
+            o[i] = dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U);
+          }
+        } else {
+          const BlockFixF f = block_fix_f(nact == NB ? hc : hh_const(nact), S_big, Ip_big);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float4 kq = kp[r0 + i];
+            o[i] = dequant(kq, reflect_f(__uint_as_float(r[i]), kq, cwc, f), U);
+          }
+          if (p_big >= bx * 32 && p_big < bx * 32 + 32) {
+            lead_row = p_big - bx * 32;
+            lead_val = dequant(kp[g0 + p_big], f.lead, U);
+          }
+        }
+      }
+      if constexpr (NB == 1 || NB > 32) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) st_box(tile, i, lane, o[i]);
+        if (lead_row >= 0) st_box(tile, lead_row, lane, lead_val);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(tmOut, (int32_t)(t.m0 + q * 32), (int32_t)(t.n0 + r0), tile);
+        bulk_commit();
+      }
+      ++nbox;
+    }
+  }
+}
+
+template <int NB, bool FLT>
+__device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
+                                               uint8_t *ring, uint64_t *accf,
+                                               uint64_t *acce, uint32_t tmem,
+                                               const CUtensorMap *tmOut,
+                                               volatile int *abort_flag, int warp,
+                                               int lane) {
+  const int ew = warp - kWarpEpi0;
+  const int q = warp & 3;     // TMEM lane quadrant: columns j = 32q .. 32q + 31
+  const int set = ew >> 2;    // the accumulator (and tiles) this warp serves
+  uint8_t *myring = ring + (size_t)ew * g.ring * kBoxBytes;
+  float4 *kp = reinterpret_cast<float4 *>(smem + kOffKp) + (size_t)ew * BN;
+  int *leads = reinterpret_cast<int *>(smem + kOffLead) + (size_t)ew * BN;
+  int *msum = reinterpret_cast<int *>(smem + kOffMsum) + (size_t)ew * BN;
+  const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+  const uint32_t acc = lane_base + (uint32_t)(set * BN);
+  const uint32_t ints = lane_base + (uint32_t)(2 * BN + set * BN);
+  const float inv_sw = *g.inv_sw, zw = *g.zero_w;
+  const ff y = two_sum((float)g.ow, zw);
+  const int Cn = (int)g.K;
+  HhConst hc = {{0.0f, 0.0f}, {0.0f, 0.0f}};
+  if (NB > 1) hc = hh_const(NB);
+  int nbox = 0;
+  uint32_t ph = 0;
+  bool ok = true;
+  int64_t local = 0;
+  for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
+    if ((int)(local & 1) != set) continue;
+    const Item t = decode_item(g, it);
+    const int64_t nchunks = (t.kb1 - t.kb0 + g.kc_blocks - 1) / g.kc_blocks;
+    const int64_t j = t.m0 + q * 32 + lane;
+    const bool active = t.m0 + q * 32 < g.M;  // warp-uniform
+    float cwc = 0.0f, U = 0.0f;
+    bool tile_f = false;
+    if (active) {
+      // per-row parameters of the tile (lanes own rows n0 + lane + 32 i)
+      float mabs = 0.0f;
+      float mrow[BN / 32];
+#pragma unroll
+      for (int i = 0; i < BN / 32; ++i) {
+        const int64_t k = t.n0 + lane + 32 * i;
+        float sc = 0.0f, A = 0.0f, B = 0.0f, m = 0.0f;
+        if (k < g.N) {
+          const int64_t ri = g.kind == FQT_PTQ ? 0 : k;
+          sc = __fmul_rn(inv_sw, g.inv_s[ri]);
+          const ff x = two_sum((float)g.og, g.zero[ri]);
+          m = rintf(x.h);
+          float hd, hR;
+          if (NB > 1) {
+            hd = g.hz[k];
+            hR = g.hr[k];
+          } else {
+            // R = sum_c (a + m); rounding relative to R itself suffices for a
+            // row-constant term
+            hd = ff_round(fast_two_sum(__fsub_rn(x.h, m), x.l));
+            hR = __fadd_rn((float)(g.row_sum[k] - Cn * g.og), __fmul_rn((float)Cn, m));
+          }
+          A = __fmul_rn(sc, hd);
+          B = __fmul_rn(sc, __fmaf_rn(hR, y.h, __fmul_rn(hR, y.l)));
+        }
+        kp[lane + 32 * i] = make_float4(sc, A, B, m);
+        mabs = fmaxf(mabs, fabsf(m));
+        mrow[i] = m;
+      }
+      if (NB > 1) {
+        // sums of m over each block (the fp32 form's S = sum P + CWc sum m)
+        if (NB <= 32) {
+#pragma unroll
+          for (int i = 0; i < BN / 32; ++i) {
+            float v = mrow[i];
+#pragma unroll
+            for (int off = 1; off < (NB > 32 ? 32 : NB); off <<= 1)
+              v += __shfl_xor_sync(0xffffffffu, v, off);
+            if (lane % (NB > 32 ? 32 : NB) == 0) msum[(32 * i + lane) / (NB > 1 ? NB : 1)] = (int)v;
+          }
+        } else {
+          float tot[BN / 32];
+#pragma unroll
+          for (int i = 0; i < BN / 32; ++i) {
+            float v = mrow[i];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+            tot[i] = v;
+          }
+          if (lane == 0) {
+#pragma unroll
+            for (int b = 0; b < BN / (NB > 32 ? NB : 32); ++b) {
+              float v = 0.0f;
+#pragma unroll
+              for (int i = 0; i < (NB > 32 ? NB : 32) / 32; ++i) v += tot[b * ((NB > 32 ? NB : 32) / 32) + i];
+              msum[b] = (int)v;
+            }
+          }
+        }
+      }
+      if (NB > 1) {
+        for (int b = lane; b < BN / NB; b += 32) {
+          const int64_t kb = t.n0 / NB + b;
+          leads[b] = kb * NB < g.N ? g.lead[kb] : 0;
+        }
+      }
+      if (j < g.M) {
+        const int cs = __ldg(g.col_sum_w + j);
+        cwc = (float)(cs - Cn * g.ow);
+        U = __fmaf_rn((float)Cn, zw, (float)cs);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1)
+        mabs = fmaxf(mabs, __shfl_xor_sync(0xffffffffu, mabs, off));
+      tile_f = FLT && mabs <= g.flt_mmax;
+    }
+    __syncwarp();
+    for (int64_t c = 0; c < nchunks; ++c) {
+      const bool got = !*abort_flag && mbar_wait(&accf[set], ph, g.status);
+      if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
+      ph ^= 1u;
+      tc_fence_after();
+      const bool last_chunk = c + 1 == nchunks;
+      if (!last_chunk && active) {
+        // exact chunk boundary: fold the chunk into the int32 running sum
+#pragma unroll 1
+        for (int grp = 0; grp < BN / 32; ++grp) {
+          uint32_t r[32];
+          tmem_ld32_nw(acc + (uint32_t)(grp * 32), r);
+          tmem_wait_ld(r);
+          if (c > 0) {
+            uint32_t s[32];
+            tmem_ld32_nw(ints + (uint32_t)(grp * 32), s);
+            tmem_wait_ld(s);
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)s[i]);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
+          }
+          tmem_st32(ints + (uint32_t)(grp * 32), r);
+        }
+        tmem_wait_st();
+      }
+      if (!last_chunk || !active) {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acce[set]);
+        continue;
+      }
+      const bool multi = c > 0;
+      if (FLT && tile_f)
+        gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, myring, nbox, &acce[set],
+                         tmOut, q, lane);
+      else
+        gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, myring, nbox,
+                              &acce[set], tmOut, q, lane);
+    }
+    if (!ok) break;
+  }
+  if (!ok) *abort_flag = 1;
+  if (lane == 0) bulk_wait_all();
+  __syncwarp();
+}
+
+// ---------------------------------------------------------------------------
+// Split-K partial epilogue: each warp owns TMEM lanes 32q .. 32q + 31 (rows)
+// and 64 columns, stored as two 32 x 32 int32 boxes (3-D tensor map over
+// splits x M x N) from a ring of boxes.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void partial_epilogue(const GemmArgs &g, uint8_t *ring,
+                                                 uint64_t *accf, uint64_t *acce,
+                                                 uint32_t tmem, const CUtensorMap *tmOut,
+                                                 volatile int *abort_flag, int warp,
+                                                 int lane) {
+  const int ew = warp - kWarpEpi0;
+  const int q = warp & 3;
+  const int hcol = ew >> 2;  // column half: 64 * hcol .. +63
+  uint8_t *myring = ring + (size_t)ew * g.ring * kBoxBytes;
+  int nbox = 0;
+  const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+  const uint32_t int_cols = lane_base + (uint32_t)(2 * BN + hcol * 64);
+  int buf = 0;
+  uint32_t aph = 0u;  // bit b: phase parity of accumulator b
+  bool ok = true;
+  for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
+    const Item t = decode_item(g, it);
+    const int64_t nchunks = (t.kb1 - t.kb0 + g.kc_blocks - 1) / g.kc_blocks;
+    for (int64_t c = 0; c < nchunks; ++c) {
+      const bool got = !*abort_flag && mbar_wait(&accf[buf], (aph >> buf) & 1u, g.status);
+      if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t accb = lane_base + (uint32_t)(buf * BN + hcol * 64);
+      const bool last = c + 1 == nchunks;
+#pragma unroll
+      for (int grp = 0; grp < 2; ++grp) {
+        uint32_t r[32];
+        tmem_ld32_nw(accb + (uint32_t)(grp * 32), r);
+        tmem_wait_ld(r);
+        if (c > 0) {
+          uint32_t s[32];
+          tmem_ld32_nw(int_cols + (uint32_t)(grp * 32), s);
+          tmem_wait_ld(s);
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            r[j] = (uint32_t)(__float2int_rn(__uint_as_float(r[j])) + (int)s[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) r[j] = (uint32_t)__float2int_rn(__uint_as_float(r[j]));
+        }
+        if (!last) {
+          tmem_st32(int_cols + (uint32_t)(grp * 32), r);
+          continue;
+        }
+        if (grp == 1) {  // this accumulator is no longer read
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acce[buf]);
+        }
+        uint8_t *tile = myring + (size_t)(nbox % g.ring) * kBoxBytes;
+        if (nbox >= g.ring) {
+          if (lane == 0) bulk_wait_read(g.ring - 1);
+          __syncwarp();
+        }
+#pragma unroll
+        for (int j4 = 0; j4 < 8; ++j4)
+          *reinterpret_cast<uint4 *>(tile + sw128_off(lane, j4)) =
+              make_uint4(r[4 * j4], r[4 * j4 + 1], r[4 * j4 + 2], r[4 * j4 + 3]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(tmOut, (int32_t)(t.n0 + hcol * 64 + grp * 32), (int32_t)(t.m0 + q * 32),
+                       t.split, tile);
+          bulk_commit();
+        }
+        ++nbox;
+      }
+      if (!last) {
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acce[buf]);
+      }
+      aph ^= 1u << buf;
+      buf ^= 1;
+    }
+    if (!ok) break;
+  }
+  if (!ok) *abort_flag = 1;
+  if (lane == 0) bulk_wait_all();
+  __syncwarp();
+}
+
+template <int MODE, int NB, bool FLT>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap tmA,
            const __grid_constant__ CUtensorMap tmB,
@@ -274,9 +970,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint8_t *ring = ops + (size_t)nstages * 2 * kTileBytes;          // output boxes
   uint64_t *full = bars, *empty = bars + kMaxStages;
   uint64_t *accf = bars + 2 * kMaxStages, *acce = accf + 2;
-  uint64_t *xbar = accf + 4;  // BHQ row-block exchange, one per column half
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kNumBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  // grad_X: one accumulator per item, served by 4 epilogue warps (one per
+  // lane quadrant); partials: accumulators alternate per chunk, 8 warps each
+  constexpr bool kPerItem = MODE == MODE_GRADX;
+  constexpr uint32_t kEpiArrivals = kPerItem ? 4u : 8u;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -286,8 +985,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&accf[i], 1);
-      mbar_init(&acce[i], kNumEpiWarps);
-      mbar_init(&xbar[i], 4);
+      mbar_init(&acce[i], kEpiArrivals);
     }
     *abort_flag = 0;
     fence_barrier_init();
@@ -360,8 +1058,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // swizzle row, two 8-row K atoms (2048 bytes) for MN-major
       const uint64_t a_step = g.a_kmajor ? 2u : (2048u >> 4);
       const uint64_t b_step = g.b_kmajor ? 2u : (2048u >> 4);
-      for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
+      int64_t local = 0;
+      for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
         const Item t = decode_item(g, it);
+        if (kPerItem) buf = (int)(local & 1);
         for (int64_t c0 = t.kb0; c0 < t.kb1 && !*abort_flag; c0 += g.kc_blocks) {
           const int64_t c1 = min(t.kb1, c0 + g.kc_blocks);
           if (!mbar_wait(&acce[buf], ((aph >> buf) & 1u) ^ 1u, g.status)) { fail(); break; }
@@ -385,239 +1085,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
           umma_commit(&accf[buf]);
           aph ^= 1u << buf;
-          buf ^= 1;
+          if (!kPerItem) buf ^= 1;
         }
       }
     }
   } else if (warp >= kWarpEpi0) {
-    // ------------------------------------------------------------ epilogue
-    // Each warp owns TMEM lanes 32q..32q+31 (rows) and 64 columns, handled as
-    // two 32 x 32 boxes.  A box goes through a 128-byte-swizzled shared tile:
-    // rows are written by their owning lane; for BHQ a column-owner pass
-    // applies the inverse Householder of each block; the tile then leaves
-    // with coalesced 16-byte stores (8 lanes per 128-byte row segment).
-    const int ew = warp - kWarpEpi0;
-    const int q = warp & 3;    // TMEM lane quadrant = rows 32q .. 32q+31
-    const int hcol = ew >> 2;  // column half: 64 * hcol .. +63
-    uint8_t *myring = ring + (size_t)ew * g.ring * kBoxBytes;
-    int nbox = 0;  // boxes stored by this warp so far
-    float *cwf = reinterpret_cast<float *>(smem + kOffCol + (size_t)ew * 512);
-    float *csw = cwf + 64;
-    float *rowv = reinterpret_cast<float *>(smem + kOffRow + (size_t)ew * 384);
-    float *xch = reinterpret_cast<float *>(smem + kOffBhq);  // [2][2][4][32]
-    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
-    const uint32_t int_cols = lane_base + (uint32_t)(2 * BN + hcol * 64);
-    const bool gx = g.mode == MODE_GRADX;
-    const bool bhq = gx && g.kind == FQT_BHQ;
-    const int nb = bhq ? g.block : 1;
-    uint32_t xph = 0;
-    int buf = 0;
-    uint32_t aph = 0u;  // bit b: phase parity of accumulator b
-    for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
-      const Item t = decode_item(g, it);
-      const int64_t nchunks = (t.kb1 - t.kb0 + g.kc_blocks - 1) / g.kc_blocks;
-      const int64_t row = t.m0 + q * 32 + lane;
-      const int64_t col0 = t.n0 + hcol * 64;
-      const bool rv = row < g.M;
-      // raw per-row / per-column inputs, loaded before the accumulator wait
-      float inv_si = 0.0f, zi = 0.0f, zw = 0.0f, inv_sw = 0.0f;
-      int rsum = 0, lead_p = -1, cs0 = 0, cs1 = 0;
-      if (gx) {
-        const int64_t ri = g.kind == FQT_PTQ ? 0 : (rv ? row : 0);
-        inv_si = rv ? g.inv_s[ri] : 0.0f;
-        zi = g.zero[ri];
-        rsum = rv ? g.row_sum[row] : 0;
-        zw = *g.zero_w;
-        inv_sw = *g.inv_sw;
-        if (bhq && rv) lead_p = g.lead[row / nb];
-        const int64_t c0 = col0 + lane, c1 = col0 + 32 + lane;
-        cs0 = c0 < g.N ? __ldg(g.col_sum_w + c0) : 0;
-        cs1 = c1 < g.N ? __ldg(g.col_sum_w + c1) : 0;
-      }
-      bool ok = true;
-      for (int64_t c = 0; c < nchunks; ++c) {
-        const bool got = !*abort_flag && mbar_wait(&accf[buf], (aph >> buf) & 1u, g.status);
-        if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t accb = lane_base + (uint32_t)(buf * BN + hcol * 64);
-        if (c + 1 < nchunks) {
-          // exact chunk boundary: fold the chunk into the int32 running sum
-#pragma unroll
-          for (int grp = 0; grp < 2; ++grp) {
-            uint32_t r[32];
-            tmem_ld32(accb + (uint32_t)(grp * 32), r);
-            if (c > 0) {
-              uint32_t s[32];
-              tmem_ld32(int_cols + (uint32_t)(grp * 32), s);
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                r[j] = (uint32_t)(__float2int_rn(__uint_as_float(r[j])) + (int)s[j]);
-            } else {
-#pragma unroll
-              for (int j = 0; j < 32; ++j)
-                r[j] = (uint32_t)__float2int_rn(__uint_as_float(r[j]));
-            }
-            tmem_st32(int_cols + (uint32_t)(grp * 32), r);
-          }
-          tmem_wait_st();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&acce[buf]);
-          aph ^= 1u << buf;
-          buf ^= 1;
-          continue;
-        }
-
-        // ---- last chunk: the epilogue proper ----
-        // Dequantization (Eq. 9) of V_ij = sum_c (a_ic + z'_i)(w_cj + z'_w)
-        // from the exact centred product P_ij and integer row / column sums:
-        // with m = round(-z'), d = z' + m,
-        // V = P + alpha_i CW_j + rowc_i + d_i SW_j.
-        float alpha = 0.0f, rowc = 0.0f, di = 0.0f, scale = 0.0f, ck = 0.0f, ek = 0.0f;
-        if (gx) {
-          const int Cn = (int)g.K;
-          const int mi = __float2int_rn(-zi), mw = __float2int_rn(-zw);
-          di = zi + (float)mi;
-          const float dw = zw + (float)mw;
-          const int ai = g.oa - mi, beta = g.ob - mw;
-          alpha = (float)ai;
-          const long long rowI = (long long)beta * (rsum - (long long)Cn * g.oa) +
-                                 (long long)Cn * ai * beta;
-          rowc = (float)rowI + (dw * (float)(rsum - Cn * mi) + (float)Cn * di * dw);
-          scale = inv_sw * inv_si;
-          cwf[lane] = (float)(cs0 - Cn * g.ob);
-          cwf[32 + lane] = (float)(cs1 - Cn * g.ob);
-          csw[lane] = (float)(cs0 - Cn * mw);
-          csw[32 + lane] = (float)(cs1 - Cn * mw);
-          if (bhq) {
-            const int64_t b = row / nb;
-            const int64_t nb_act = min((int64_t)nb, g.M - b * nb);
-            if (rv && nb_act > 1) {  // Q = I - 2 n n^T / |n|^2, n = rho 1 - e_p
-              const float rho = 1.0f / sqrtf((float)nb_act);
-              ck = (row - b * nb == lead_p) ? rho - 1.0f : rho;
-              ek = ck / (1.0f - rho);
-            }
-            rowv[lane] = ek;
-            rowv[32 + lane] = ck;
-            rowv[64 + lane] = scale;
-          }
-          __syncwarp();
-        }
-#pragma unroll
-        for (int bx = 0; bx < 2; ++bx) {
-          // the ring slot of this box must have been read by its last store
-          uint8_t *tile = myring + (size_t)(nbox % g.ring) * kBoxBytes;
-          if (nbox >= g.ring) {
-            if (lane == 0) bulk_wait_read(g.ring - 1);
-            __syncwarp();
-          }
-          uint32_t r[32];
-          tmem_ld32(accb + (uint32_t)(bx * 32), r);
-          if (c > 0) {  // add the int32 running sum of the earlier chunks
-            uint32_t s[32];
-            tmem_ld32(int_cols + (uint32_t)(bx * 32), s);
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-              r[j] = (uint32_t)(__float2int_rn(__uint_as_float(r[j])) + (int)s[j]);
-          } else if (!gx) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) r[j] = (uint32_t)__float2int_rn(__uint_as_float(r[j]));
-          }
-          // r: exact int32 (multi-chunk or partial store) or exact fp32
-          const bool r_is_int = c > 0 || !gx;
-          if (bx == 1) {  // this accumulator is no longer read
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&acce[buf]);
-          }
-          if (gx) {
-            const float4 *cw4 = reinterpret_cast<const float4 *>(cwf) + bx * 8;
-            const float4 *sw4 = reinterpret_cast<const float4 *>(csw) + bx * 8;
-            const float rs = bhq ? 1.0f : scale;
-#pragma unroll
-            for (int j4 = 0; j4 < 8; ++j4) {
-              const float4 a = cw4[j4], b = sw4[j4];
-              const float ca[4] = {a.x, a.y, a.z, a.w}, cb[4] = {b.x, b.y, b.z, b.w};
-              float o[4];
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const int j = 4 * j4 + e;
-                const float pj = r_is_int ? (float)(int)r[j] : __uint_as_float(r[j]);
-                o[e] = rs * (fmaf(alpha, ca[e], pj) + fmaf(di, cb[e], rowc));
-              }
-              *reinterpret_cast<float4 *>(tile + sw128_off(lane, j4)) =
-                  make_float4(o[0], o[1], o[2], o[3]);
-            }
-          } else {
-#pragma unroll
-            for (int j4 = 0; j4 < 8; ++j4)
-              *reinterpret_cast<uint4 *>(tile + sw128_off(lane, j4)) =
-                  make_uint4(r[4 * j4], r[4 * j4 + 1], r[4 * j4 + 2], r[4 * j4 + 3]);
-          }
-          __syncwarp();
-          if (bhq) {
-            // column-owner pass: lane = column, rows of the box in order;
-            // (Q V)_k = V_k - c_k w, w = sum_k e_k V_k over the block's rows
-            float colv[32];
-            const int cofs = ((lane >> 2) << 4) | ((lane & 3) << 2);
-#pragma unroll
-            for (int rr = 0; rr < 32; ++rr)
-              colv[rr] = *reinterpret_cast<const float *>(
-                  tile + rr * 128 + (cofs ^ ((rr & 7) << 4)));
-            if (nb <= 32) {
-              switch (nb) {
-                case 1: householder_cols<1>(colv, rowv); break;
-                case 2: householder_cols<2>(colv, rowv); break;
-                case 4: householder_cols<4>(colv, rowv); break;
-                case 8: householder_cols<8>(colv, rowv); break;
-                case 16: householder_cols<16>(colv, rowv); break;
-                default: householder_cols<32>(colv, rowv); break;
-              }
-            } else {
-              // blocks of 64 / 128 rows span 2 / 4 quadrant warps: add the
-              // per-warp partial sums through shared memory, double-buffered,
-              // synchronised by an mbarrier of the 4 warps of this half
-              float wp = 0.0f;
-#pragma unroll
-              for (int rr = 0; rr < 32; ++rr) wp = fmaf(rowv[rr], colv[rr], wp);
-              float *area = xch + ((xph & 1u) * 2 + hcol) * 4 * 32;
-              area[q * 32 + lane] = wp;
-              __syncwarp();
-              if (lane == 0) mbar_arrive(&xbar[hcol]);
-              const bool got2 = mbar_wait(&xbar[hcol], xph & 1u, g.status);
-              if (!__all_sync(0xffffffffu, got2)) { ok = false; break; }
-              xph ^= 1u;
-              const int qn = nb / 32, q0 = (q / qn) * qn;
-              float w = 0.0f;
-              for (int qq = q0; qq < q0 + qn; ++qq) w += area[qq * 32 + lane];
-#pragma unroll
-              for (int rr = 0; rr < 32; ++rr)
-                colv[rr] = rowv[64 + rr] * fmaf(-rowv[32 + rr], w, colv[rr]);
-            }
-#pragma unroll
-            for (int rr = 0; rr < 32; ++rr)
-              *reinterpret_cast<float *>(tile + rr * 128 + (cofs ^ ((rr & 7) << 4))) =
-                  colv[rr];
-            __syncwarp();
-          }
-          // hand the box to the TMA engine
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            const int32_t cx = (int32_t)(col0 + bx * 32), cy = (int32_t)(t.m0 + q * 32);
-            if (gx) tma_store_2d(&tmOut, cx, cy, tile);
-            else tma_store_3d(&tmOut, cx, cy, t.split, tile);
-            bulk_commit();
-          }
-          ++nbox;
-        }
-        aph ^= 1u << buf;
-        buf ^= 1;
-      }
-      if (!ok) { fail(); break; }
-    }
-    if (lane == 0) bulk_wait_all();
-    __syncwarp();
+    if (MODE == MODE_GRADX)
+      gradx_epilogue<NB, FLT>(g, smem, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
+    else
+      partial_epilogue(g, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
   }
 
   tc_fence_before();
@@ -774,26 +1250,54 @@ size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D) {
   return (bytes + 255) & ~(size_t)255;
 }
 
+typedef void (*GemmKernel)(CUtensorMap, CUtensorMap, CUtensorMap, GemmArgs);
+
+// The kernel instance of a mode, BHQ block size (1 = no reflection) and
+// product representation (fp32-exact or int32).
+static GemmKernel gemm_kernel(int mode, int nb, bool flt) {
+  if (mode == MODE_PARTIAL) return k_gemm<MODE_PARTIAL, 1, false>;
+#define FQT_GX(NBV)                                                          \
+  case NBV:                                                                  \
+    return flt ? k_gemm<MODE_GRADX, NBV, true> : k_gemm<MODE_GRADX, NBV, false>;
+  switch (nb) {
+    FQT_GX(1)
+    FQT_GX(2)
+    FQT_GX(4)
+    FQT_GX(8)
+    FQT_GX(16)
+    FQT_GX(32)
+    FQT_GX(64)
+    FQT_GX(128)
+  }
+#undef FQT_GX
+  return nullptr;
+}
+
 // Launches the contraction of fp16 carrier operands: A is M x K (stored
 // M x K if a_kmajor, else K x M), B is the K x N operand (stored N x K if
-// b_kmajor, else K x N).
+// b_kmajor, else K x N).  Partials: out is splits x M x N int32.  grad_X:
+// out is the N x M fp32 transpose (rows of dH x columns of W~).
 static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
                            const uint16_t *Bm, int b_kmajor, int b_bits, int64_t M,
                            int64_t N, int64_t K, const SplitPlan &p, GemmArgs &g,
-                           void *out, bool out_is_partial, cudaStream_t st) {
+                           void *out, int mode, int nb, bool flt, cudaStream_t st) {
+  const bool partial = mode == MODE_PARTIAL;
   CUtensorMap ta, tb;
   bool ok = a_kmajor ? make_map_f16(&ta, A, (uint64_t)K, (uint64_t)M, BK, BM)
                      : make_map_f16(&ta, A, (uint64_t)M, (uint64_t)K, 64, BK);
   ok = ok && (b_kmajor ? make_map_f16(&tb, Bm, (uint64_t)K, (uint64_t)N, BK, BN)
                        : make_map_f16(&tb, Bm, (uint64_t)N, (uint64_t)K, 64, BK));
   CUtensorMap to;
-  ok = ok && make_map_out(&to, out, out_is_partial, (uint64_t)N, (uint64_t)M,
-                          out_is_partial ? (uint64_t)p.splits : 1);
+  ok = ok && (partial ? make_map_out(&to, out, true, (uint64_t)N, (uint64_t)M,
+                                     (uint64_t)p.splits)
+                      : make_map_out(&to, out, false, (uint64_t)M, (uint64_t)N, 1));
   if (!ok) return cuda_fail(cudaErrorInvalidValue, "tensor map encode");
+  GemmKernel kern = gemm_kernel(mode, nb, flt);
+  if (!kern) return FQT_EUNSUPPORTED;
   // HBM-bound output tiles (grad_X): deep store ring; long reductions
   // (split-K partials): deep operand ring
-  g.stages = out_is_partial ? 5 : 2;
-  g.ring = out_is_partial ? 1 : 4;
+  g.stages = partial ? 5 : 2;
+  g.ring = partial ? 1 : 4;
   g.M = M;
   g.N = N;
   g.K = K;
@@ -801,8 +1305,6 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   g.b_kmajor = b_kmajor;
   g.mn_lbo = (uint32_t)(kTileBytes / 2);  // second 64-wide MN atom column
   g.mn_sbo = 1024;                        // next 8-row K atom
-  g.oa = 1 << (a_bits - 1);
-  g.ob = 1 << (b_bits - 1);
   g.kc_blocks = exact_chunk_blocks(a_bits, b_bits);
   g.m_tiles = p.m_tiles;
   g.n_tiles = p.n_tiles;
@@ -810,19 +1312,14 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   g.ks_blocks = p.ks_blocks;
   g.kb_total = p.kb_total;
   g.n_items = (int64_t)p.m_tiles * p.n_tiles * p.splits;
-  g.mode = out_is_partial ? MODE_PARTIAL : MODE_GRADX;
   const size_t smem = gemm_smem_bytes(g.stages, g.ring);
-  static size_t attr_bytes = 0;
-  if (smem > attr_bytes) {
-    const cudaError_t e = cudaFuncSetAttribute(
-        k_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "gemm shared-memory attribute");
-    attr_bytes = smem;
-  }
+  const cudaError_t ea =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (ea != cudaSuccess) return cuda_fail(ea, "gemm shared-memory attribute");
   const int nsm = device_sm_count();
   int64_t grid = g.n_items < nsm ? g.n_items : nsm;
   if (grid < 1) grid = 1;
-  k_gemm<<<(int)grid, kGemmThreads, smem, st>>>(ta, tb, to, g);
+  kern<<<(int)grid, kGemmThreads, smem, st>>>(ta, tb, to, g);
   return cuda_fail(cudaGetLastError(), "gemm launch");
 }
 
@@ -884,7 +1381,7 @@ fqt_status debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
   memset(&g, 0, sizeof(g));
   g.status = reinterpret_cast<int *>(ws);
   fqt_status s = run_gemm(a16, a_kmajor, a_bits, b16, b_kmajor, b_bits, M, N, K, p,
-                          g, part, true, st);
+                          g, part, MODE_PARTIAL, 1, false, st);
   if (s != FQT_OK) return s;
   ReduceArgs r;
   memset(&r, 0, sizeof(r));
@@ -906,10 +1403,13 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
   int *status = reinterpret_cast<int *>(ws);
   const int nsm = device_sm_count();
   if (grad_X) {
-    if (!q_b2 || !qw || !q_b2->codes_f16 || !qw->codes_f16 || !q_b2->row_sum ||
-        !qw->col_sum || !q_b2->inv_s || !q_b2->zero || !qw->inv_s || !qw->zero)
+    if (!q_b2 || !qw || !q_b2->codes_f16 || !qw->codes_f16 || !qw->col_sum ||
+        !q_b2->inv_s || !q_b2->zero || !qw->inv_s || !qw->zero)
       return FQT_EINVAL;
-    if (q_b2->kind == FQT_BHQ && !q_b2->lead) return FQT_EINVAL;
+    const int nb = q_b2->kind == FQT_BHQ && q_b2->block > 1 ? q_b2->block : 1;
+    if (nb > 1 && (!q_b2->lead || !q_b2->hz || !q_b2->hr)) return FQT_EINVAL;
+    if (nb == 1 && !q_b2->row_sum) return FQT_EINVAL;
+    if (nb > 128 || (nb & (nb - 1))) return FQT_EINVAL;
     const int64_t Nr = q_b2->rows, C = q_b2->cols, D = qw->cols;
     if (qw->rows != C || qw->kind != FQT_PTQ) return FQT_EINVAL;
     if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
@@ -917,21 +1417,36 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     if (!aligned16(q_b2->codes_f16) || !aligned16(qw->codes_f16) || !aligned16(grad_X))
       return FQT_EINVAL;
     if (Nr > 0) {
-      const SplitPlan p = plan_splits(Nr, D, C, q_b2->bits, qw->bits, nsm, false);
+      // transposed: M = D (columns of W~), N = rows of dH, K = C
+      const SplitPlan p = plan_splits(D, Nr, C, qw->bits, q_b2->bits, nsm, false);
+      // fp32 form of the integer parts I = P + m CWc: one exact chunk,
+      // |P| < 2^22 and |I| (2 + sqrt(nb)) < 2^24 (|I| < 2^24 without
+      // reflection) for every row offset |m| <= mmax, with
+      // |I| <= C 2^(bw-1) (2^(b-1) + |m|)
+      const int64_t kc_terms = (int64_t)exact_chunk_blocks(qw->bits, q_b2->bits) * BK;
+      const double lim = nb == 1 ? 16777216.0 : 16777216.0 / (2.0 + sqrt((double)nb));
+      const double mmax = floor(lim / ((double)C * (double)(1 << (qw->bits - 1)))) -
+                          (double)(1 << (q_b2->bits - 1)) - 1.0;
+      const int64_t pmax = C << (qw->bits + q_b2->bits - 2);
+      const bool flt = C <= kc_terms && mmax >= 0.0 && pmax < ((int64_t)1 << 22);
       GemmArgs g;
       memset(&g, 0, sizeof(g));
       g.status = status;
       g.kind = q_b2->kind;
-      g.block = q_b2->kind == FQT_BHQ ? q_b2->block : 0;
+      g.og = 1 << (q_b2->bits - 1);
+      g.ow = 1 << (qw->bits - 1);
       g.inv_s = q_b2->inv_s;
       g.zero = q_b2->zero;
       g.row_sum = q_b2->row_sum;
       g.lead = q_b2->lead;
+      g.hz = q_b2->hz;
+      g.hr = q_b2->hr;
+      g.flt_mmax = flt ? (float)mmax : -1.0f;
       g.col_sum_w = qw->col_sum;
       g.inv_sw = qw->inv_s;
       g.zero_w = qw->zero;
-      fqt_status s = run_gemm(q_b2->codes_f16, 1, q_b2->bits, qw->codes_f16, 0, qw->bits,
-                              Nr, D, C, p, g, grad_X, false, st);
+      fqt_status s = run_gemm(qw->codes_f16, 0, qw->bits, q_b2->codes_f16, 1, q_b2->bits,
+                              D, Nr, C, p, g, grad_X, MODE_GRADX, nb, flt, st);
       if (s != FQT_OK) return s;
     }
   }
@@ -954,7 +1469,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       memset(&g, 0, sizeof(g));
       g.status = status;
       fqt_status s = run_gemm(qa->codes_f16, 0, qa->bits, qx->codes_f16, 0, qx->bits, C,
-                              D, Nr, p, g, part, true, st);
+                              D, Nr, p, g, part, MODE_PARTIAL, 1, false, st);
       if (s != FQT_OK) return s;
     } else {
       const cudaError_t e = cudaMemsetAsync(part, 0, (size_t)C * D * 4, st);
@@ -1055,7 +1570,7 @@ fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
   memset(&g, 0, sizeof(g));
   g.status = status;
   s = run_gemm(qa->codes_f16, 0, qa->bits, qx->codes_f16, 0, qx->bits, C, D, Nr, p, g,
-               part, true, st);
+               part, MODE_PARTIAL, 1, false, st);
   if (s != FQT_OK) return s;
   ReduceArgs r;
   memset(&r, 0, sizeof(r));

@@ -51,6 +51,10 @@ cudaError_t launch_range(const void *x, bool bf16, int64_t count, float2 *part,
                          int *npart, int32_t *z0, int64_t nz0, int32_t *z1,
                          int64_t nz1, int num_sms, cudaStream_t st);
 
+cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
+                               const int32_t *lead, float *hz, float *hr, int64_t N,
+                               int C, int bits, int block, cudaStream_t st);
+
 int device_sm_count();
 
 // Records the CUDA error behind an FQT_ECUDA return (per thread) and returns

@@ -873,6 +873,81 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Offsets of the BHQ grad_X epilogue.  Each row's offset 2^(b-1) + z' is
+// split into an integer m (which the epilogue folds into the exact integer
+// product) and a fraction d, |d| <= 1/2.  With a the centred codes, w the
+// centred codes of W~ and y = 2^(bw-1) + z_w,
+//   (a + m + d)(w + y) summed over c = [P + m CWc] + y R + d U,
+//   P = a w, CWc_j = sum_c w_cj, R_i = sum_c (a_ic + m_i), U_j = CWc_j + C y
+// (Eq. 9).  The reflection of Sec. 4.2 is linear in the rows, so the epilogue
+// needs hz = Q_blk d and hr = Q_blk R, reflected here in float-float, one
+// thread per row, a block of rows inside one CTA.
+// ---------------------------------------------------------------------------
+constexpr int kOffThreads = 128;
+
+__global__ void __launch_bounds__(kOffThreads)
+    k_bhq_offsets(const float *__restrict__ zero, const int32_t *__restrict__ rsum,
+                  const int32_t *__restrict__ lead, float *hz, float *hr, int64_t N,
+                  int C, int oa, int nb) {
+  __shared__ float2 ds[kOffThreads];
+  __shared__ long long Rs[kOffThreads];
+  const int t = threadIdx.x;
+  const int64_t r0 = (int64_t)blockIdx.x * kOffThreads;
+  const int64_t k = r0 + t;
+  const bool kv = k < N;
+  ff d = {0.0f, 0.0f};
+  long long R = 0;
+  if (kv) {
+    const ff x = two_sum((float)oa, zero[k]);
+    const float m = rintf(x.h);  // the epilogue rounds the same fp32 sum
+    d = fast_two_sum(__fsub_rn(x.h, m), x.l);
+    R = (long long)rsum[k] - (long long)C * oa + (long long)C * (long long)m;
+  }
+  ds[t] = make_float2(d.h, d.l);
+  Rs[t] = R;
+  __syncthreads();
+  if (!kv) return;
+  const int base = (t / nb) * nb;  // nb divides kOffThreads: blocks stay in the CTA
+  const int64_t kb = r0 + base;
+  const int nact = (int)min((int64_t)nb, N - kb);
+  if (nact < 2) {  // a one-row block is not transformed
+    hz[k] = ff_round(d);
+    hr[k] = ff_round(ff_from_int(R));
+    return;
+  }
+  const int p = lead[kb / nb];
+  ff sd = {0.0f, 0.0f};
+  long long sR = 0;
+  for (int l = 0; l < nact; ++l) {
+    sd = ff_add(sd, {ds[base + l].x, ds[base + l].y});
+    sR += Rs[base + l];
+  }
+  const HhConst c = hh_const(nact);
+  // (Q v)_k = v_k - kappa (rho sum(v) - v_p) off the lead row; rho sum(v) on it
+  const ff rsd = ff_mul(c.rho, sd);
+  const ff rsR = ff_mul(c.rho, ff_from_int(sR));
+  if (t - base == p) {
+    hz[k] = ff_round(rsd);
+    hr[k] = ff_round(rsR);
+    return;
+  }
+  const ff wd = ff_add(rsd, ff_neg({ds[base + p].x, ds[base + p].y}));
+  const ff wR = ff_add(rsR, ff_neg(ff_from_int(Rs[base + p])));
+  hz[k] = ff_round(ff_add(d, ff_neg(ff_mul(c.kap, wd))));
+  hr[k] = ff_round(ff_add(ff_from_int(R), ff_neg(ff_mul(c.kap, wR))));
+}
+
+cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
+                               const int32_t *lead, float *hz, float *hr, int64_t N,
+                               int C, int bits, int block, cudaStream_t st) {
+  if (N <= 0) return cudaSuccess;
+  const int64_t grid = (N + kOffThreads - 1) / kOffThreads;
+  k_bhq_offsets<<<(unsigned)grid, kOffThreads, 0, st>>>(zero, rsum, lead, hz, hr, N, C,
+                                                        1 << (bits - 1), block);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
 static int pow2ceil(int v) {

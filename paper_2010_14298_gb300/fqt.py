@@ -39,7 +39,8 @@ class _QT(ctypes.Structure):
                 ("codes", ctypes.c_void_p), ("inv_s", ctypes.c_void_p),
                 ("zero", ctypes.c_void_p), ("row_sum", ctypes.c_void_p),
                 ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p),
-                ("codes_f16", ctypes.c_void_p)]
+                ("codes_f16", ctypes.c_void_p), ("hz", ctypes.c_void_p),
+                ("hr", ctypes.c_void_p)]
 
 
 def library_path() -> str:
@@ -139,7 +140,8 @@ class QTensor:
 
     ``codes`` holds the integer codes (uint8), ``codes16`` the same codes
     centred by 2^(b-1) as exact fp16 values (the tensor-core operand format);
-    either may be None.
+    either may be None.  ``hz`` and ``hr`` (BHQ, block > 1) are the reflected
+    per-row offsets the grad_X epilogue reads.
     """
     codes: Optional[torch.Tensor]
     inv_s: torch.Tensor
@@ -151,6 +153,8 @@ class QTensor:
     bits: int = 8
     block: int = 0
     codes16: Optional[torch.Tensor] = None
+    hz: Optional[torch.Tensor] = None
+    hr: Optional[torch.Tensor] = None
 
     @property
     def shape(self):
@@ -162,6 +166,7 @@ class QTensor:
               u8: bool = True, f16: bool = True):
         m = 1 if kind == PTQ else rows
         nblk = (rows + block - 1) // block if kind == BHQ else 0
+        offsets = kind == BHQ and block > 1 and row_sum
         return QTensor(
             codes=(torch.empty((rows, cols), dtype=torch.uint8, device=device)
                    if u8 else None),
@@ -175,14 +180,19 @@ class QTensor:
                      if col_sum else None),
             lead=(torch.empty(max(nblk, 1), dtype=torch.int32, device=device)
                   if kind == BHQ else None),
-            kind=kind, bits=bits, block=block)
+            kind=kind, bits=bits, block=block,
+            hz=(torch.empty(rows, dtype=torch.float32, device=device)
+                if offsets else None),
+            hr=(torch.empty(rows, dtype=torch.float32, device=device)
+                if offsets else None))
 
     def c_struct(self) -> _QT:
         rows, cols = self.shape
         p = lambda t: t.data_ptr() if t is not None else None
         return _QT(rows, cols, self.bits, self.kind, self.block, 0,
                    p(self.codes), self.inv_s.data_ptr(), self.zero.data_ptr(),
-                   p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16))
+                   p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16),
+                   p(self.hz), p(self.hr))
 
     def codes_from_f16(self) -> torch.Tensor:
         """The uint8 codes recovered from the fp16 carriers."""

@@ -177,8 +177,10 @@ def _backward(L, kind, bits, block, seed=3, reuse=False):
 
 BACKWARD_CASES = [(0, None, orc.PTQ, 8, 0), (0, None, orc.PSQ, 8, 0),
                   (0, None, orc.BHQ, 5, 16), (1, 2, orc.PTQ, 4, 0),
-                  (1, 2, orc.BHQ, 5, 16), (2, 1, orc.BHQ, 5, 32),
-                  (2, 1, orc.BHQ, 5, 64), (3, 128, orc.BHQ, 5, 16),
+                  (1, 2, orc.BHQ, 5, 16), (2, 1, orc.BHQ, 5, 8),
+                  (2, 1, orc.BHQ, 5, 32), (2, 1, orc.BHQ, 5, 64),
+                  (2, 1, orc.BHQ, 4, 128), (0, None, orc.BHQ, 5, 2),
+                  (3, 128, orc.BHQ, 5, 16), (3, 128, orc.BHQ, 8, 16),
                   (3, 128, orc.PTQ, 8, 0)]
 
 
@@ -196,6 +198,34 @@ def test_linear_backward_matches_oracle(cfg, small, kind, bits, block):
         ref_w = orc.grad_w(h1, hx)
         assert grad_rel_err(gx, ref_x) <= GRAD_TOL
         assert grad_rel_err(gw, ref_w) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("N,block", [(256, 8), (200, 64), (131, 128), (77, 16)])
+def test_bhq_offsets_match_oracle(N, block):
+    """The reflected per-row terms of the grad_X epilogue against the
+    oracle's reflection (Sec. 4.2) of the GPU's own zero points and row sums:
+    2^(b-1) + z' = m + d with m the integer nearest its fp32 sum,
+    hz = Q_blk d and hr = Q_blk (row_sum - C 2^(b-1) + C m)."""
+    g = wl.rng(N + block)
+    C, bits = 64, 5
+    dH = wl.random_grad(g, N, C, outlier_frac=0.1)
+    q2, _ = fqt.quantize_grad(to_dev(dH), orc.BHQ, bits, block, 9, with_b1=False)
+    zero32 = q2.zero.cpu().numpy()
+    rsum = q2.row_sum.cpu().numpy().astype(np.float64)
+    lead = q2.lead.cpu().numpy()
+    hz, hr = q2.hz.cpu().numpy(), q2.hr.cpu().numpy()
+    oa = 2 ** (bits - 1)
+    m = np.rint(np.float32(oa) + zero32).astype(np.float64)  # ties to even
+    d = oa + zero32.astype(np.float64) - m
+    R = rsum - C * oa + C * m
+    assert np.all(np.abs(d) <= 0.5 + 1e-6)
+    for b0 in range(0, N, block):
+        nb = min(block, N - b0)
+        Q = orc.householder(nb, int(lead[b0 // block])) if nb > 1 else np.eye(1)
+        for got, x in ((hz, d[b0:b0 + nb]), (hr, R[b0:b0 + nb])):
+            ref = Q @ x
+            tol = 2.0 ** -23 * np.abs(ref) + 2.0 ** -36 * np.abs(x).max()
+            assert np.all(np.abs(got[b0:b0 + nb] - ref) <= tol)
 
 
 def test_ptq_codes_reused_for_grad_w():
