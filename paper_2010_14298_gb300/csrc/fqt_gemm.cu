@@ -35,9 +35,14 @@ namespace fqt {
 
 constexpr int BM = 128, BN = 128, BK = 64;
 constexpr int kMaxStages = 8;  // operand stages (A and B fp16 tiles), chosen per launch
-constexpr int kGemmThreads = 320;
 constexpr int kWarpTma = 0, kWarpMma = 1, kWarpEpi0 = 2;
-constexpr int kNumEpiWarps = 8;
+// grad_X: three sets of four epilogue warps (one per TMEM lane quadrant) take
+// the tiles in turn; split-K partials use the first eight
+constexpr int kGradxSets = 3;
+constexpr int kNumEpiWarps = 4 * kGradxSets;
+constexpr int kPartialEpiWarps = 8;
+constexpr int kWarpPar = kWarpEpi0 + kNumEpiWarps;  // grad_X: per-tile parameter loader
+constexpr int kGemmThreads = 32 * (kWarpPar + 1);
 // two 128-column fp32 accumulators and 256 columns of int32 running sums
 constexpr uint32_t kTmemCols = 512;
 
@@ -47,11 +52,18 @@ constexpr size_t kBoxBytes = 4096;   // one 32 x 32 fp32 / int32 output box
 //   [0, kFixedBytes)           per-warp epilogue tables and barriers
 //   [kFixedBytes, +S * 32 KiB) S operand stages (A, B)
 //   [..., + 8 * R * 4 KiB)     R output boxes per epilogue warp (TMA store ring)
-constexpr size_t kOffKp = 0;                                        // [8 warps][BN] float4
-constexpr size_t kOffLead = kOffKp + kNumEpiWarps * BN * 16;        // [8 warps][BN] int
-constexpr size_t kOffMsum = kOffLead + kNumEpiWarps * BN * 4;       // [8 warps][BN] int
-constexpr size_t kOffBar = kOffMsum + kNumEpiWarps * BN * 4;
-constexpr size_t kNumBars = 2 * kMaxStages + 4;
+// grad_X parameter stages (one per tile in flight), each:
+//   float4 kp[BN]  per row k: inv_sw inv_s_k, .. hz_k, .. y hr_k, m_k
+//   int leads[BN]  lead row of each block;  int msum[BN]  sum of m per block
+//   int cs[BM]     W~ column sums of the tile's columns;  int flag
+constexpr int kParStages = 4;
+constexpr size_t kParBytes = 4096;
+constexpr size_t kParLeads = 2048, kParMsum = 2560, kParCs = 3072, kParFlag = 3584;
+constexpr size_t kOffPar = 0;
+constexpr size_t kOffBar = kOffPar + kParStages * kParBytes;
+// operand full / empty, accumulator full / empty (4 each), parameter full /
+// empty (4 each)
+constexpr size_t kNumBars = 2 * kMaxStages + 16;
 constexpr size_t kFixedBytes = (kOffBar + kNumBars * 8 + 16 + 1023) & ~(size_t)1023;
 
 __host__ __device__ constexpr size_t gemm_smem_bytes(int stages, int ring) {
@@ -73,6 +85,7 @@ struct GemmArgs {
   int64_t ks_blocks, kb_total;
   int64_t n_items;
   int stages, ring;           // operand stages, output boxes per epilogue warp
+  int nacc;                   // TMEM accumulators in rotation (2 or 4)
   // grad_X epilogue (MODE_GRADX); rows of Q_b2 are the N dimension
   int kind;
   int og, ow;                  // centring offsets 2^(b-1) of Q_b2 and W~ codes
@@ -707,122 +720,186 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
   }
 }
 
+// The global inputs of one tile's parameters (lane-owned rows and columns).
+struct TileLoads {
+  float inv[BN / 32], zero[BN / 32], hz[BN / 32], hr[BN / 32];
+  int rs[BN / 32], cs[BM / 32], lead[2];
+};
+
+template <int NB>
+__device__ __forceinline__ void tile_loads(const GemmArgs &g, const Item &t, int lane,
+                                           TileLoads &L) {
+  constexpr int NBD = NB > 1 ? NB : 1;
+#pragma unroll
+  for (int i = 0; i < BN / 32; ++i) {
+    const int64_t k = t.n0 + lane + 32 * i;
+    const bool kv = k < g.N;
+    const int64_t ri = g.kind == FQT_PTQ ? 0 : (kv ? k : 0);
+    L.inv[i] = kv ? __ldg(g.inv_s + ri) : 0.0f;
+    L.zero[i] = kv ? __ldg(g.zero + ri) : 0.0f;
+    if (NB > 1) {
+      L.hz[i] = kv ? __ldg(g.hz + k) : 0.0f;
+      L.hr[i] = kv ? __ldg(g.hr + k) : 0.0f;
+      L.rs[i] = 0;
+    } else {
+      L.hz[i] = L.hr[i] = 0.0f;
+      L.rs[i] = kv ? __ldg(g.row_sum + k) : 0;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < BM / 32; ++i) {
+    const int64_t j = t.m0 + lane + 32 * i;
+    L.cs[i] = j < g.M ? __ldg(g.col_sum_w + j) : 0;
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {  // BN / NB <= 64 blocks per tile
+    const int b = lane + 32 * u;
+    L.lead[u] = 0;
+    if (NB > 1 && b < BN / NBD) {
+      const int64_t kb = t.n0 / NBD + b;
+      L.lead[u] = kb * NBD < g.N ? __ldg(g.lead + kb) : 0;
+    }
+  }
+}
+
+// Parameter loader of grad_X (one warp): for every tile of this CTA, in
+// order, the per-row terms of its rows and the column sums of its columns go
+// into a parameter stage ahead of the epilogue warps that use them.  The
+// global loads of the next tile are in flight while this tile's are used.
+template <int NB, bool FLT>
+__device__ __forceinline__ void gradx_params(const GemmArgs &g, uint8_t *smem, uint64_t *pfull,
+                                             uint64_t *pempty, volatile int *abort_flag,
+                                             int lane) {
+  const float inv_sw = *g.inv_sw, zw = *g.zero_w;
+  const ff y = two_sum((float)g.ow, zw);
+  const int Cn = (int)g.K;
+  TileLoads cur, nxt;
+  if ((int64_t)blockIdx.x < g.n_items) tile_loads<NB>(g, decode_item(g, blockIdx.x), lane, cur);
+  int64_t local = 0;
+  for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
+    if (it + gridDim.x < g.n_items) tile_loads<NB>(g, decode_item(g, it + gridDim.x), lane, nxt);
+    const int s = (int)(local % kParStages);
+    const uint32_t wrap = (uint32_t)(local / kParStages);
+    const bool got = mbar_wait(&pempty[s], (wrap & 1u) ^ 1u, g.status);
+    if (!__all_sync(0xffffffffu, got)) { *abort_flag = 1; break; }
+    const Item t = decode_item(g, it);
+    uint8_t *P = smem + kOffPar + (size_t)s * kParBytes;
+    float4 *kp = reinterpret_cast<float4 *>(P);
+    int *leads = reinterpret_cast<int *>(P + kParLeads);
+    int *msum = reinterpret_cast<int *>(P + kParMsum);
+    int *cs = reinterpret_cast<int *>(P + kParCs);
+    float mabs = 0.0f;
+    float mrow[BN / 32];
+#pragma unroll
+    for (int i = 0; i < BN / 32; ++i) {
+      const int64_t k = t.n0 + lane + 32 * i;
+      float sc = 0.0f, A = 0.0f, B = 0.0f, m = 0.0f;
+      if (k < g.N) {
+        sc = __fmul_rn(inv_sw, cur.inv[i]);
+        const ff x = two_sum((float)g.og, cur.zero[i]);
+        m = rintf(x.h);
+        float hd, hR;
+        if (NB > 1) {
+          hd = cur.hz[i];
+          hR = cur.hr[i];
+        } else {
+          // R = sum_c (a + m); rounding relative to R itself suffices for a
+          // row-constant term
+          hd = ff_round(fast_two_sum(__fsub_rn(x.h, m), x.l));
+          hR = __fadd_rn((float)(cur.rs[i] - Cn * g.og), __fmul_rn((float)Cn, m));
+        }
+        A = __fmul_rn(sc, hd);
+        B = __fmul_rn(sc, __fmaf_rn(hR, y.h, __fmul_rn(hR, y.l)));
+      }
+      kp[lane + 32 * i] = make_float4(sc, A, B, m);
+      mabs = fmaxf(mabs, fabsf(m));
+      mrow[i] = m;
+    }
+    if constexpr (NB > 1) {
+      // sums of m over each block (the fp32 form's S = sum P + CWc sum m)
+      constexpr int SEG = NB > 32 ? 32 : NB;
+#pragma unroll
+      for (int i = 0; i < BN / 32; ++i) {
+        float v = mrow[i];
+#pragma unroll
+        for (int off = 1; off < SEG; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        mrow[i] = v;
+      }
+      if constexpr (NB <= 32) {
+#pragma unroll
+        for (int i = 0; i < BN / 32; ++i)
+          if (lane % NB == 0) msum[(32 * i + lane) / NB] = (int)mrow[i];
+      } else if (lane == 0) {
+#pragma unroll
+        for (int b = 0; b < BN / NB; ++b) {
+          float v = 0.0f;
+#pragma unroll
+          for (int i = 0; i < NB / 32; ++i) v += mrow[b * (NB / 32) + i];
+          msum[b] = (int)v;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+        if (lane + 32 * u < BN / NB) leads[lane + 32 * u] = cur.lead[u];
+    }
+#pragma unroll
+    for (int i = 0; i < BM / 32; ++i) cs[lane + 32 * i] = cur.cs[i];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+      mabs = fmaxf(mabs, __shfl_xor_sync(0xffffffffu, mabs, off));
+    if (lane == 0) *reinterpret_cast<int *>(P + kParFlag) = FLT && mabs <= g.flt_mmax;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&pfull[s]);
+    cur = nxt;
+  }
+}
+
 template <int NB, bool FLT>
 __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
                                                uint8_t *ring, uint64_t *accf,
-                                               uint64_t *acce, uint32_t tmem,
+                                               uint64_t *acce, uint64_t *pfull,
+                                               uint64_t *pempty, uint32_t tmem,
                                                const CUtensorMap *tmOut,
                                                volatile int *abort_flag, int warp,
                                                int lane) {
   const int ew = warp - kWarpEpi0;
   const int q = warp & 3;     // TMEM lane quadrant: columns j = 32q .. 32q + 31
-  const int set = ew >> 2;    // the accumulator (and tiles) this warp serves
+  const int set = ew >> 2;    // the tiles (every third one) this warp serves
   uint8_t *myring = ring + (size_t)ew * g.ring * kBoxBytes;
-  float4 *kp = reinterpret_cast<float4 *>(smem + kOffKp) + (size_t)ew * BN;
-  int *leads = reinterpret_cast<int *>(smem + kOffLead) + (size_t)ew * BN;
-  int *msum = reinterpret_cast<int *>(smem + kOffMsum) + (size_t)ew * BN;
   const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
-  const uint32_t acc = lane_base + (uint32_t)(set * BN);
-  const uint32_t ints = lane_base + (uint32_t)(2 * BN + set * BN);
-  const float inv_sw = *g.inv_sw, zw = *g.zero_w;
-  const ff y = two_sum((float)g.ow, zw);
+  const float zw = *g.zero_w;
   const int Cn = (int)g.K;
   HhConst hc = {{0.0f, 0.0f}, {0.0f, 0.0f}};
   if (NB > 1) hc = hh_const(NB);
   int nbox = 0;
-  uint32_t ph = 0;
   bool ok = true;
   int64_t local = 0;
   for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
-    if ((int)(local & 1) != set) continue;
+    if ((int)(local % kGradxSets) != set) continue;
     const Item t = decode_item(g, it);
+    const int buf = (int)(local & (g.nacc - 1));
+    const uint32_t acc = lane_base + (uint32_t)(buf * BN);
+    // int32 running sums (two accumulators only): columns 256 + 128 buf
+    const uint32_t ints = lane_base + (uint32_t)(2 * BN + buf * BN);
     const int64_t nchunks = (t.kb1 - t.kb0 + g.kc_blocks - 1) / g.kc_blocks;
-    const int64_t j = t.m0 + q * 32 + lane;
     const bool active = t.m0 + q * 32 < g.M;  // warp-uniform
-    float cwc = 0.0f, U = 0.0f;
-    bool tile_f = false;
-    if (active) {
-      // per-row parameters of the tile (lanes own rows n0 + lane + 32 i)
-      float mabs = 0.0f;
-      float mrow[BN / 32];
-#pragma unroll
-      for (int i = 0; i < BN / 32; ++i) {
-        const int64_t k = t.n0 + lane + 32 * i;
-        float sc = 0.0f, A = 0.0f, B = 0.0f, m = 0.0f;
-        if (k < g.N) {
-          const int64_t ri = g.kind == FQT_PTQ ? 0 : k;
-          sc = __fmul_rn(inv_sw, g.inv_s[ri]);
-          const ff x = two_sum((float)g.og, g.zero[ri]);
-          m = rintf(x.h);
-          float hd, hR;
-          if (NB > 1) {
-            hd = g.hz[k];
-            hR = g.hr[k];
-          } else {
-            // R = sum_c (a + m); rounding relative to R itself suffices for a
-            // row-constant term
-            hd = ff_round(fast_two_sum(__fsub_rn(x.h, m), x.l));
-            hR = __fadd_rn((float)(g.row_sum[k] - Cn * g.og), __fmul_rn((float)Cn, m));
-          }
-          A = __fmul_rn(sc, hd);
-          B = __fmul_rn(sc, __fmaf_rn(hR, y.h, __fmul_rn(hR, y.l)));
-        }
-        kp[lane + 32 * i] = make_float4(sc, A, B, m);
-        mabs = fmaxf(mabs, fabsf(m));
-        mrow[i] = m;
-      }
-      if (NB > 1) {
-        // sums of m over each block (the fp32 form's S = sum P + CWc sum m)
-        if (NB <= 32) {
-#pragma unroll
-          for (int i = 0; i < BN / 32; ++i) {
-            float v = mrow[i];
-#pragma unroll
-            for (int off = 1; off < (NB > 32 ? 32 : NB); off <<= 1)
-              v += __shfl_xor_sync(0xffffffffu, v, off);
-            if (lane % (NB > 32 ? 32 : NB) == 0) msum[(32 * i + lane) / (NB > 1 ? NB : 1)] = (int)v;
-          }
-        } else {
-          float tot[BN / 32];
-#pragma unroll
-          for (int i = 0; i < BN / 32; ++i) {
-            float v = mrow[i];
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-            tot[i] = v;
-          }
-          if (lane == 0) {
-#pragma unroll
-            for (int b = 0; b < BN / (NB > 32 ? NB : 32); ++b) {
-              float v = 0.0f;
-#pragma unroll
-              for (int i = 0; i < (NB > 32 ? NB : 32) / 32; ++i) v += tot[b * ((NB > 32 ? NB : 32) / 32) + i];
-              msum[b] = (int)v;
-            }
-          }
-        }
-      }
-      if (NB > 1) {
-        for (int b = lane; b < BN / NB; b += 32) {
-          const int64_t kb = t.n0 / NB + b;
-          leads[b] = kb * NB < g.N ? g.lead[kb] : 0;
-        }
-      }
-      if (j < g.M) {
-        const int cs = __ldg(g.col_sum_w + j);
-        cwc = (float)(cs - Cn * g.ow);
-        U = __fmaf_rn((float)Cn, zw, (float)cs);
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1)
-        mabs = fmaxf(mabs, __shfl_xor_sync(0xffffffffu, mabs, off));
-      tile_f = FLT && mabs <= g.flt_mmax;
-    }
-    __syncwarp();
+    const int s = (int)(local % kParStages);
+    const bool gotp = mbar_wait(&pfull[s], (uint32_t)(local / kParStages) & 1u, g.status);
+    if (!__all_sync(0xffffffffu, gotp)) { ok = false; break; }
+    const uint8_t *P = smem + kOffPar + (size_t)s * kParBytes;
+    const float4 *kp = reinterpret_cast<const float4 *>(P);
+    const int *leads = reinterpret_cast<const int *>(P + kParLeads);
+    const int *msum = reinterpret_cast<const int *>(P + kParMsum);
+    const int cs = reinterpret_cast<const int *>(P + kParCs)[q * 32 + lane];
+    const bool tile_f = FLT && *reinterpret_cast<const int *>(P + kParFlag) != 0;
+    const float cwc = (float)(cs - Cn * g.ow);
+    const float U = __fmaf_rn((float)Cn, zw, (float)cs);
     for (int64_t c = 0; c < nchunks; ++c) {
-      const bool got = !*abort_flag && mbar_wait(&accf[set], ph, g.status);
+      // every tile has nchunks chunks: the use count of this accumulator
+      // before chunk c of this tile gives the phase
+      const uint32_t par = (uint32_t)(((local / g.nacc) * nchunks + c) & 1);
+      const bool got = !*abort_flag && mbar_wait(&accf[buf], par, g.status);
       if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
-      ph ^= 1u;
       tc_fence_after();
       const bool last_chunk = c + 1 == nchunks;
       if (!last_chunk && active) {
@@ -833,12 +910,12 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
           tmem_ld32_nw(acc + (uint32_t)(grp * 32), r);
           tmem_wait_ld(r);
           if (c > 0) {
-            uint32_t s[32];
-            tmem_ld32_nw(ints + (uint32_t)(grp * 32), s);
-            tmem_wait_ld(s);
+            uint32_t sr[32];
+            tmem_ld32_nw(ints + (uint32_t)(grp * 32), sr);
+            tmem_wait_ld(sr);
 #pragma unroll
             for (int i = 0; i < 32; ++i)
-              r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)s[i]);
+              r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)sr[i]);
           } else {
 #pragma unroll
             for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
@@ -850,17 +927,20 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
       if (!last_chunk || !active) {
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&acce[set]);
+        if (lane == 0) mbar_arrive(&acce[buf]);
         continue;
       }
       const bool multi = c > 0;
       if (FLT && tile_f)
-        gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, myring, nbox, &acce[set],
+        gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, myring, nbox, &acce[buf],
                          tmOut, q, lane);
       else
         gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, myring, nbox,
-                              &acce[set], tmOut, q, lane);
+                              &acce[buf], tmOut, q, lane);
     }
+    // the parameter stage is free again
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&pempty[s]);
     if (!ok) break;
   }
   if (!ok) *abort_flag = 1;
@@ -969,13 +1049,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint8_t *ops = smem + kFixedBytes;                                // operand stages
   uint8_t *ring = ops + (size_t)nstages * 2 * kTileBytes;          // output boxes
   uint64_t *full = bars, *empty = bars + kMaxStages;
-  uint64_t *accf = bars + 2 * kMaxStages, *acce = accf + 2;
+  uint64_t *accf = bars + 2 * kMaxStages, *acce = accf + 4;
+  uint64_t *pfull = acce + 4, *pempty = pfull + 4;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kNumBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   // grad_X: one accumulator per item, served by 4 epilogue warps (one per
   // lane quadrant); partials: accumulators alternate per chunk, 8 warps each
   constexpr bool kPerItem = MODE == MODE_GRADX;
-  constexpr uint32_t kEpiArrivals = kPerItem ? 4u : 8u;
+  constexpr uint32_t kEpiArrivals = kPerItem ? 4u : (uint32_t)kPartialEpiWarps;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -983,9 +1064,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < 4; ++i) {
       mbar_init(&accf[i], 1);
       mbar_init(&acce[i], kEpiArrivals);
+      mbar_init(&pfull[i], 1);
+      mbar_init(&pempty[i], 4);  // the 4 epilogue warps of the consuming set
     }
     *abort_flag = 0;
     fence_barrier_init();
@@ -1061,7 +1144,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       int64_t local = 0;
       for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
         const Item t = decode_item(g, it);
-        if (kPerItem) buf = (int)(local & 1);
+        if (kPerItem) buf = (int)(local & (g.nacc - 1));
         for (int64_t c0 = t.kb0; c0 < t.kb1 && !*abort_flag; c0 += g.kc_blocks) {
           const int64_t c1 = min(t.kb1, c0 + g.kc_blocks);
           if (!mbar_wait(&acce[buf], ((aph >> buf) & 1u) ^ 1u, g.status)) { fail(); break; }
@@ -1089,10 +1172,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
       }
     }
+  } else if (warp == kWarpPar) {
+    if (MODE == MODE_GRADX) gradx_params<NB, FLT>(g, smem, pfull, pempty, abort_flag, lane);
   } else if (warp >= kWarpEpi0) {
     if (MODE == MODE_GRADX)
-      gradx_epilogue<NB, FLT>(g, smem, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
-    else
+      gradx_epilogue<NB, FLT>(g, smem, ring, accf, acce, pfull, pempty, tmem, &tmOut,
+                              abort_flag, warp, lane);
+    else if (warp < kWarpEpi0 + kPartialEpiWarps)
       partial_epilogue(g, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
   }
 
@@ -1297,7 +1383,11 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   // HBM-bound output tiles (grad_X): deep store ring; long reductions
   // (split-K partials): deep operand ring
   g.stages = partial ? 5 : 2;
-  g.ring = partial ? 1 : 4;
+  g.ring = partial ? 1 : 3;
+  // grad_X with one exact chunk per tile: four accumulators in rotation, so
+  // the next tile of each epilogue set is ready when it finishes the last;
+  // otherwise two, and the other half of tensor memory holds running sums
+  g.nacc = (!partial && exact_chunk_blocks(a_bits, b_bits) >= (K + BK - 1) / BK) ? 4 : 2;
   g.M = M;
   g.N = N;
   g.K = K;
