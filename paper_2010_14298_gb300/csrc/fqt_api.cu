@@ -68,6 +68,10 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
                                out->col_sum, out->col_sum ? cols : 0, nullptr, 0,
                                nsm, st);
   if (e != cudaSuccess) return cuda_fail(e, "range pass");
+  if (!out->row_sum && cols / 8 <= 1024)
+    return launch_fwd_codes(X, dtype == FQT_BF16, rows, (int)cols, bits, out->codes_f16,
+                            out->codes, out->col_sum, part, npart, out->inv_s, out->zero,
+                            reinterpret_cast<int *>(w), nsm, st);
   QuantArgs a;
   memset(&a, 0, sizeof(a));
   a.h = X;

@@ -95,6 +95,7 @@ struct GemmArgs {
   float flt_mmax;              // largest |m| of a tile for the fp32 form
   const int32_t *col_sum_w;    // W~ column sums over C
   const float *inv_sw, *zero_w;
+  float *out;                  // grad_X (N x M row-major) for MODE_GRADX
   int *status;
 };
 
@@ -276,10 +277,31 @@ __device__ __forceinline__ uint32_t sw128_off(int row, int chunk) {
   return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
-// Element (row, col) of a 32 x 32 fp32 output box in the 128-byte swizzle.
-__device__ __forceinline__ void st_box(uint8_t *tile, int row, int col, float v) {
-  *reinterpret_cast<float *>(tile + sw128_off(row, col >> 2) + ((col & 3) << 2)) = v;
-}
+// The 32 rows r0 .. r0 + 31 of this thread's column j of grad_X.  The 32
+// lanes of a warp hold 32 consecutive columns, so every store of a row is one
+// coalesced 128-byte write; no staging is needed.
+struct BoxOut {
+  float *p;       // &grad_X[row r0][j]
+  int64_t ld;     // row stride (D)
+  int rows;       // rows of the box inside the matrix (0 .. 32)
+  bool jv;        // column j inside the matrix
+  __device__ __forceinline__ void st(int row, float v) const {
+    if (jv && row < rows) __stcs(p + row * ld, v);
+  }
+  // all 32 values of the box (then the lead-row overwrites, same thread)
+  __device__ __forceinline__ void st32(const float (&o)[32]) const {
+    if (!jv) return;
+    if (rows == 32) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) __stcs(p + i * ld, o[i]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i < rows) __stcs(p + i * ld, o[i]);
+    }
+  }
+};
+
 
 struct Item {
   int64_t m0, n0;
@@ -297,6 +319,18 @@ __device__ __forceinline__ Item decode_item(const GemmArgs &g, int64_t it) {
   r.kb0 = (int64_t)r.split * g.ks_blocks;
   r.kb1 = min(g.kb_total, r.kb0 + g.ks_blocks);
   return r;
+}
+
+__device__ __forceinline__ BoxOut box_out(const GemmArgs &g, const Item &t, int q, int lane,
+                                          int r0) {
+  BoxOut w;
+  const int64_t j = t.m0 + q * 32 + lane, row0 = t.n0 + r0;
+  w.jv = j < g.M;
+  const int64_t left = g.N - row0;
+  w.rows = left >= 32 ? 32 : (int)(left > 0 ? left : 0);
+  w.ld = g.M;
+  w.p = g.out + (w.rows > 0 && w.jv ? row0 * g.M + j : 0);
+  return w;
 }
 
 // ---------------------------------------------------------------------------
@@ -424,10 +458,10 @@ template <int NB, bool F>
 __device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip)[leads_per_box(NB)],
                                           const HhConst &hc, const float4 *kp,
                                           const int *leads, int r0, int64_t row0,
-                                          int64_t N, float U, uint8_t *tile, int lane) {
+                                          int64_t N, float U, const BoxOut &w) {
   if (NB == 1) {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) st_box(tile, i, lane, dequant(kp[r0 + i], I.f(i), U));
+    for (int i = 0; i < 32; ++i) w.st(i, dequant(kp[r0 + i], I.f(i), U));
     return;
   }
   constexpr int NBB = NB > 1 ? NB : 2;
@@ -438,8 +472,7 @@ __device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip
     const int nact = left >= NBB ? NBB : (int)(left > 0 ? left : 0);
     if (nact < 2) {  // a one-row block is not transformed
 #pragma unroll
-      for (int l = 0; l < NBB; ++l)
-        st_box(tile, b * NBB + l, lane, dequant(kp[kb0 + l], I.f(b * NBB + l), U));
+      for (int l = 0; l < NBB; ++l) w.st(b * NBB + l, dequant(kp[kb0 + l], I.f(b * NBB + l), U));
       continue;
     }
     long long S = 0;
@@ -447,10 +480,9 @@ __device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip
     for (int l = 0; l < NBB; ++l) S += I.ll(b * NBB + l);
     const BlockFix f = block_fix(nact == NBB ? hc : hh_const(nact), S, Ip[b]);
 #pragma unroll
-    for (int l = 0; l < NBB; ++l)
-      st_box(tile, b * NBB + l, lane, dequant(kp[kb0 + l], I.minus(b * NBB + l, f), U));
+    for (int l = 0; l < NBB; ++l) w.st(b * NBB + l, dequant(kp[kb0 + l], I.minus(b * NBB + l, f), U));
     const int p = leads[kb0 / NBB];  // the lead row: a later store of the same thread
-    st_box(tile, b * NBB + p, lane, dequant(kp[kb0 + p], f.lead, U));
+    w.st(b * NBB + p, dequant(kp[kb0 + p], f.lead, U));
   }
 }
 
@@ -460,9 +492,7 @@ template <int NB, bool F>
 __device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uint32_t acc,
                                            uint32_t ints, bool multi, const float4 *kp,
                                            const int *leads, const HhConst &hc, float cwc,
-                                           float U, uint8_t *myring, int &nbox,
-                                           uint64_t *acce_set, const CUtensorMap *tmOut,
-                                           int q, int lane) {
+                                           float U, uint64_t *acce_set, int q, int lane) {
   constexpr int GW = NB > 32 ? NB : 32;
   constexpr int NPP = leads_per_box(NB);
 #pragma unroll 1
@@ -484,11 +514,7 @@ __device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uin
 #pragma unroll 1
     for (int bx = 0; bx < GW / 32; ++bx) {
       const int r0 = g0 + bx * 32;
-      uint8_t *tile = myring + (size_t)(nbox % g.ring) * kBoxBytes;
-      if (nbox >= g.ring) {
-        if (lane == 0) bulk_wait_read(g.ring - 1);
-        __syncwarp();
-      }
+      const BoxOut w = box_out(g, t, q, lane, r0);
       Ints<F> I;
       load_ints<F>(acc, ints, multi, r0, kp, cwc, I);
       long long Ip[NPP];
@@ -506,30 +532,21 @@ __device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uin
         if (lane == 0) mbar_arrive(acce_set);
       }
       if constexpr (NB <= 32) {
-        box_small<NB, F>(I, Ip, hc, kp, leads, r0, t.n0 + r0, g.N, U, tile, lane);
+        box_small<NB, F>(I, Ip, hc, kp, leads, r0, t.n0 + r0, g.N, U, w);
       } else {
         const int64_t left = g.N - (t.n0 + g0);
         const int nact = left >= NB ? NB : (int)(left > 0 ? left : 0);
         if (nact < 2) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) st_box(tile, i, lane, dequant(kp[r0 + i], I.f(i), U));
+          for (int i = 0; i < 32; ++i) w.st(i, dequant(kp[r0 + i], I.f(i), U));
         } else {
           const BlockFix f = block_fix(nact == NB ? hc : hh_const(nact), S_big, Ip_big);
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            st_box(tile, i, lane, dequant(kp[r0 + i], I.minus(i, f), U));
+          for (int i = 0; i < 32; ++i) w.st(i, dequant(kp[r0 + i], I.minus(i, f), U));
           if (p_big >= bx * 32 && p_big < bx * 32 + 32)
-            st_box(tile, p_big - bx * 32, lane, dequant(kp[g0 + p_big], f.lead, U));
+            w.st(p_big - bx * 32, dequant(kp[g0 + p_big], f.lead, U));
         }
       }
-      // hand the box to the TMA engine: rows t.n0 + r0 .., columns 32q ..
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        tma_store_2d(tmOut, (int32_t)(t.m0 + q * 32), (int32_t)(t.n0 + r0), tile);
-        bulk_commit();
-      }
-      ++nbox;
     }
   }
 }
@@ -581,9 +598,7 @@ template <int NB>
 __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, uint32_t acc,
                                              const float4 *kp, const int *leads,
                                              const int *msum, const HhConst &hc, float cwc,
-                                             float U, uint8_t *myring, int &nbox,
-                                             uint64_t *acce_set, const CUtensorMap *tmOut,
-                                             int q, int lane) {
+                                             float U, uint64_t *acce_set, int q, int lane) {
   constexpr int GW = NB > 32 ? NB : 32;
   constexpr int NPP = leads_per_box(NB);
   constexpr int NBD = NB > 1 ? NB : 1;
@@ -611,11 +626,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
 #pragma unroll 1
     for (int bx = 0; bx < GW / 32; ++bx) {
       const int r0 = g0 + bx * 32;
-      uint8_t *tile = myring + (size_t)(nbox % g.ring) * kBoxBytes;
-      if (nbox >= g.ring) {
-        if (lane == 0) bulk_wait_read(g.ring - 1);
-        __syncwarp();
-      }
+      const BoxOut w = box_out(g, t, q, lane, r0);
       uint32_t r[32];
       tmem_ld32_nw(acc + (uint32_t)r0, r);
       uint32_t pp[NPP];
@@ -634,14 +645,14 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
       // every output of the box is formed in registers before the first
       // store, so the per-row loads from shared memory need not wait for
       // the stores into the (possibly aliasing) box
-      float o[32];
+      // outputs overwrite the products in place (r holds fp32 bit patterns)
       int lead_row = -1;
       float lead_val = 0.0f;
       if constexpr (NB == 1) {
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           const float4 kq = kp[r0 + i];
-          o[i] = dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U);
+          r[i] = __float_as_uint(dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U));
         }
       } else if constexpr (NB <= 32) {
         float lv[32 / NBD];
@@ -657,7 +668,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
 #pragma unroll
             for (int l = 0; l < NBD; ++l) {
               const float4 kq = kp[kb0 + l];
-              o[b * NBD + l] = dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[b * NBD + l])), U);
+              r[b * NBD + l] = __float_as_uint(dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[b * NBD + l])), U));
             }
             continue;
           }
@@ -671,17 +682,16 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
 #pragma unroll
           for (int l = 0; l < NBD; ++l) {
             const float4 kq = kp[kb0 + l];
-            o[b * NBD + l] = dequant(kq, reflect_f(__uint_as_float(r[b * NBD + l]), kq, cwc, f), U);
+            r[b * NBD + l] = __float_as_uint(dequant(kq, reflect_f(__uint_as_float(r[b * NBD + l]), kq, cwc, f), U));
           }
           lp[b] = b * NBD + p;
           lv[b] = dequant(kp[kb0 + p], f.lead, U);
         }
-#pragma unroll
-        for (int i = 0; i < 32; ++i) st_box(tile, i, lane, o[i]);
+        w.st32(reinterpret_cast<const float (&)[32]>(r));
         // the lead rows: later stores of the same thread
 #pragma unroll
         for (int b = 0; b < 32 / NBD; ++b)
-          if (lp[b] >= 0) st_box(tile, lp[b], lane, lv[b]);
+          if (lp[b] >= 0) w.st(lp[b], lv[b]);
       } else {
         const int64_t left = g.N - (t.n0 + g0);
         const int nact = left >= NB ? NB : (int)(left > 0 ? left : 0);
@@ -689,14 +699,14 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const float4 kq = kp[r0 + i];
-            o[i] = dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U);
+            r[i] = __float_as_uint(dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U));
           }
         } else {
           const BlockFixF f = block_fix_f(nact == NB ? hc : hh_const(nact), S_big, Ip_big);
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const float4 kq = kp[r0 + i];
-            o[i] = dequant(kq, reflect_f(__uint_as_float(r[i]), kq, cwc, f), U);
+            r[i] = __float_as_uint(dequant(kq, reflect_f(__uint_as_float(r[i]), kq, cwc, f), U));
           }
           if (p_big >= bx * 32 && p_big < bx * 32 + 32) {
             lead_row = p_big - bx * 32;
@@ -705,17 +715,9 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
         }
       }
       if constexpr (NB == 1 || NB > 32) {
-#pragma unroll
-        for (int i = 0; i < 32; ++i) st_box(tile, i, lane, o[i]);
-        if (lead_row >= 0) st_box(tile, lead_row, lane, lead_val);
+        w.st32(reinterpret_cast<const float (&)[32]>(r));
+        if (lead_row >= 0) w.st(lead_row, lead_val);
       }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        tma_store_2d(tmOut, (int32_t)(t.m0 + q * 32), (int32_t)(t.n0 + r0), tile);
-        bulk_commit();
-      }
-      ++nbox;
     }
   }
 }
@@ -865,13 +867,11 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
   const int ew = warp - kWarpEpi0;
   const int q = warp & 3;     // TMEM lane quadrant: columns j = 32q .. 32q + 31
   const int set = ew >> 2;    // the tiles (every third one) this warp serves
-  uint8_t *myring = ring + (size_t)ew * g.ring * kBoxBytes;
   const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
   const float zw = *g.zero_w;
   const int Cn = (int)g.K;
   HhConst hc = {{0.0f, 0.0f}, {0.0f, 0.0f}};
   if (NB > 1) hc = hh_const(NB);
-  int nbox = 0;
   bool ok = true;
   int64_t local = 0;
   for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
@@ -932,11 +932,10 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
       }
       const bool multi = c > 0;
       if (FLT && tile_f)
-        gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, myring, nbox, &acce[buf],
-                         tmOut, q, lane);
+        gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane);
       else
-        gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, myring, nbox,
-                              &acce[buf], tmOut, q, lane);
+        gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, &acce[buf], q,
+                              lane);
     }
     // the parameter stage is free again
     __syncwarp();
@@ -944,8 +943,6 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
     if (!ok) break;
   }
   if (!ok) *abort_flag = 1;
-  if (lane == 0) bulk_wait_all();
-  __syncwarp();
 }
 
 // ---------------------------------------------------------------------------
@@ -1383,7 +1380,8 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   // HBM-bound output tiles (grad_X): deep store ring; long reductions
   // (split-K partials): deep operand ring
   g.stages = partial ? 5 : 2;
-  g.ring = partial ? 1 : 3;
+  g.ring = partial ? 1 : 0;  // grad_X stores straight from registers
+  if (!partial) g.out = static_cast<float *>(out);
   // grad_X with one exact chunk per tile: four accumulators in rotation, so
   // the next tile of each epilogue set is ready when it finishes the last;
   // otherwise two, and the other half of tensor memory holds running sums

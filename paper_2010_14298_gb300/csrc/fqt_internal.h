@@ -51,6 +51,10 @@ cudaError_t launch_range(const void *x, bool bf16, int64_t count, float2 *part,
                          int *npart, int32_t *z0, int64_t nz0, int32_t *z1,
                          int64_t nz1, int num_sms, cudaStream_t st);
 
+fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, int bits,
+                            uint16_t *f16, uint8_t *c8, int32_t *col_sum, const float2 *part,
+                            int npart, float *inv_out, float *zero_out, int *status,
+                            int num_sms, cudaStream_t st);
 cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
                                const int32_t *lead, float *hz, float *hr, int64_t N,
                                int C, int bits, int block, cudaStream_t st);

@@ -873,6 +873,139 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Codes of a forward operand (deterministic PTQ, Sec. 2.1 and App. E):
+// code = round_half_even((x - z) s) clamped to [0, B], z = min X, s = B / R(X).
+// A thread owns one column oct (8 columns) in every row it visits, so its
+// column sums stay in registers; a CTA covers rpi rows per step.  Row groups
+// are visited from the end of the matrix, which the range pass read last
+// and left in L2.  Rounding adds 1.5 2^23 (exact round-half-even of values
+// below 2^22 by the FADD itself).
+// ---------------------------------------------------------------------------
+constexpr int kFwdUnroll = 4;
+constexpr int kFwdMaxThreads = 1024;
+
+template <typename T>
+__global__ void __launch_bounds__(kFwdMaxThreads)
+    k_fwd_codes(const T *__restrict__ X, int64_t rows, int cols, int rpi,
+                uint16_t *__restrict__ f16, uint8_t *__restrict__ c8,
+                int32_t *__restrict__ col_sum, const float2 *__restrict__ part, int npart,
+                float *inv_out, float *zero_out, int bits, int *status) {
+  extern __shared__ int csum_s[];  // cols
+  __shared__ float2 red[kFwdMaxThreads / 32];
+  __shared__ int redi[kFwdMaxThreads / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < npart; i += blockDim.x) {
+    const float2 p = part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmin, gmax);
+    redi[warp] = bad;
+  }
+  for (int i = tid; i < cols; i += blockDim.x) csum_s[i] = 0;
+  __syncthreads();
+  gmin = red[0].x;
+  gmax = red[0].y;
+  bad = redi[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+    gmin = fminf(gmin, red[w].x);
+    gmax = fmaxf(gmax, red[w].y);
+    bad |= redi[w];
+  }
+  if (bad) {
+    if (blockIdx.x == 0 && tid == 0) record_status(status, FQT_ENONFINITE);
+    return;
+  }
+  const uint32_t B = (1u << bits) - 1u;
+  const float s = affine_scale(gmin, gmax, B), z = gmin;
+  if (blockIdx.x == 0 && tid == 0) {
+    inv_out[0] = __fdiv_rn(1.0f, s);
+    zero_out[0] = __fmul_rn(s, z);
+  }
+  const int opr = cols / 8;
+  const int rl = tid / opr, o = tid - rl * opr;
+  const bool lane_on = rl < rpi;
+  int cs[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) cs[j] = 0;
+  const int64_t groups = (rows + rpi - 1) / rpi;
+  const uint32_t off = (B + 1u) >> 1;
+  for (int64_t i0 = blockIdx.x; i0 < groups; i0 += (int64_t)kFwdUnroll * gridDim.x) {
+    float x[kFwdUnroll][8];
+    int64_t row[kFwdUnroll];
+    bool ok[kFwdUnroll];
+#pragma unroll
+    for (int u = 0; u < kFwdUnroll; ++u) {
+      const int64_t gi = i0 + (int64_t)u * gridDim.x;
+      row[u] = (groups - 1 - gi) * rpi + rl;
+      ok[u] = lane_on && gi < groups && row[u] < rows;
+      if (ok[u]) load_oct(X + row[u] * cols + o * 8, x[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < kFwdUnroll; ++u) {
+      if (!ok[u]) continue;
+      uint32_t c[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float v = __fmul_rn(__fsub_rn(x[u][j], z), s);
+        const uint32_t r = __float_as_uint(__fadd_rn(v, 12582912.0f)) - 0x4B400000u;
+        c[j] = min(r, B);  // v >= 0: r is the rounded value
+        cs[j] += (int)c[j];
+      }
+      const int64_t e = row[u] * cols + o * 8;
+      if (f16) store_carriers8(f16 + e, c, off);
+      if (c8) store_codes8(c8 + e, c);
+    }
+  }
+  if (col_sum) {
+    if (lane_on) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (cs[j]) atomicAdd(&csum_s[o * 8 + j], cs[j]);
+    }
+    __syncthreads();
+    for (int i = tid; i < cols; i += blockDim.x)
+      if (csum_s[i]) atomicAdd(&col_sum[i], csum_s[i]);
+  }
+}
+
+fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, int bits,
+                            uint16_t *f16, uint8_t *c8, int32_t *col_sum, const float2 *part,
+                            int npart, float *inv_out, float *zero_out, int *status,
+                            int num_sms, cudaStream_t st) {
+  const int opr = cols / 8;
+  if (cols % 8 || opr > kFwdMaxThreads) return FQT_EUNSUPPORTED;
+  int rpi = 512 / opr;  // about 512 threads: two CTAs per SM
+  if (rpi < 1) rpi = 1;
+  const int nth = ((rpi * opr + 31) / 32) * 32;
+  const int64_t groups = (rows + rpi - 1) / rpi;
+  int64_t grid = (int64_t)num_sms * (kFwdMaxThreads * 2 / nth >= 2 ? 2 : 1) * 4;
+  const int64_t need = (groups + kFwdUnroll - 1) / kFwdUnroll;
+  if (grid > need) grid = need;
+  if (grid < 1) grid = 1;
+  const size_t smem = (size_t)cols * sizeof(int);
+  if (bf16)
+    k_fwd_codes<__nv_bfloat16><<<(int)grid, nth, smem, st>>>(
+        reinterpret_cast<const __nv_bfloat16 *>(X), rows, cols, rpi, f16, c8, col_sum, part,
+        npart, inv_out, zero_out, bits, status);
+  else
+    k_fwd_codes<float><<<(int)grid, nth, smem, st>>>(
+        reinterpret_cast<const float *>(X), rows, cols, rpi, f16, c8, col_sum, part, npart,
+        inv_out, zero_out, bits, status);
+  return cuda_fail(cudaGetLastError(), "forward codes launch");
+}
+
+// ---------------------------------------------------------------------------
 // Offsets of the BHQ grad_X epilogue.  Each row's offset 2^(b-1) + z' is
 // split into an integer m (which the epilogue folds into the exact integer
 // product) and a fraction d, |d| <= 1/2.  With a the centred codes, w the
