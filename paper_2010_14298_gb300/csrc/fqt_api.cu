@@ -211,6 +211,17 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   int nth, grid;
   size_t smem;
   const bool bf16 = dtype == FQT_BF16;
+  if (kind == FQT_BHQ) {
+    // one warp per block when the block fits a warp's registers; the warp
+    // kernel also writes the grad_X offsets
+    QuantArgs aw = a;
+    if (want_off) {
+      aw.hz = q_b2->hz;
+      aw.hr = q_b2->hr;
+    }
+    s = launch_bhq_warp(aw, bf16, nsm, st);
+    if (s != FQT_EUNSUPPORTED) return s;
+  }
   {
     QuantArgs a2 = a;  // staged kernel for rows of up to 1024 columns
     if (quant2_geometry(a2, bf16, nsm, &grid, &smem) == FQT_OK) {

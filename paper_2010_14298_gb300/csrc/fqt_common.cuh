@@ -73,9 +73,16 @@ __device__ __forceinline__ uint32_t u16_of(const uint4 &w, int i) {
 // frac(v) is realised in 16-bit fixed point, code = (floor(v 2^16) + u) >> 16.
 // sr_code16 takes v * 2^16 (scaling by 2^16 is exact, so callers may fold it
 // into their scale factor).
+// floor(v16) is read off the fp32 bits (integer shift of the significand by
+// the exponent, no conversion instruction): v16 is capped at 2^24 - 1, which
+// leaves every code unchanged (a capped v gives code B either way), so the
+// exponent is at most 23 and the right shift 150 - exponent_field >= 0 (a
+// funnel shift clamps shifts of 32 and more to 0, covering v16 < 1).
 __device__ __forceinline__ uint32_t sr_code16(float v16, uint32_t u16, uint32_t B) {
-  v16 = fminf(v16, (float)((B + 1u) << 16));
-  const uint32_t fixed = __float2uint_rz(v16);
+  v16 = fminf(v16, fminf((float)((B + 1u) << 16), 16777215.0f));
+  const uint32_t bits = __float_as_uint(v16);
+  const uint32_t sig = (bits & 0x7FFFFFu) | 0x800000u;
+  const uint32_t fixed = __funnelshift_rc(sig, 0u, 150u - (bits >> 23));
   const uint32_t code = (fixed + u16) >> 16;
   return min(code, B);
 }
@@ -275,6 +282,12 @@ __device__ __forceinline__ ff ff_from_int(long long v) {
 }
 
 __device__ __forceinline__ float ff_round(ff x) { return __fadd_rn(x.h, x.l); }
+
+// An int32 as float-float, exactly, with 32-bit conversions only.
+__device__ __forceinline__ ff ff_from_i32s(int v) {
+  const float h = __int2float_rn(v);
+  return {h, __int2float_rn(v - __float2int_rz(h))};
+}
 
 // Constants of the block Householder reflection of n >= 2 rows (Sec. 4.2):
 // rho = 1/sqrt(n) (the entries of n = rho 1 - e_p besides the lead) and

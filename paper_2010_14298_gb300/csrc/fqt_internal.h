@@ -31,6 +31,7 @@ struct QuantArgs {
   uint16_t *f1;  // fp16 carriers of code set 1 (may be null)
   float *inv1, *zero1;
   int32_t *rsum1, *csum1;
+  float *hz, *hr;  // BHQ grad_X offsets of code set 2 (may be null)
   const float2 *part;
   int npart;
   int *status;
@@ -55,6 +56,7 @@ fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, in
                             uint16_t *f16, uint8_t *c8, int32_t *col_sum, const float2 *part,
                             int npart, float *inv_out, float *zero_out, int *status,
                             int num_sms, cudaStream_t st);
+fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
                                const int32_t *lead, float *hz, float *hr, int64_t N,
                                int C, int bits, int block, cudaStream_t st);

@@ -106,6 +106,12 @@ struct OpMin {
 struct OpAdd {
   __device__ int operator()(int a, int b) const { return a + b; }
 };
+struct OpAddF {
+  __device__ float operator()(float a, float b) const { return a + b; }
+};
+struct OpMaxF {
+  __device__ float operator()(float a, float b) const { return fmaxf(a, b); }
+};
 
 __device__ __forceinline__ float shfl_x(float v, int off) {
   return __shfl_xor_sync(0xffffffffu, v, off);
@@ -870,6 +876,366 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
     for (int i = tid; i < C; i += kQ2Threads)
       if (csum_s[i]) atomicAdd(&csum_g[i], csum_s[i]);
   }
+}
+
+// ---------------------------------------------------------------------------
+// BHQ gradient quantizer, one warp per block of nb rows (Sec. 4.2, App. D.4)
+// fused with Q_b1 (App. E), for rows of C = 8 LPR columns, LPR in {8, 16,
+// 32}: lane l owns oct l % LPR of row l / LPR of each of the STEPS row groups
+// of the block (nb = (32 / LPR) STEPS).  The block stays in registers and
+// every reduction is a shuffle inside the warp, so the warps of an SM run
+// their blocks independently, without CTA barriers.  The grad_X offsets hz,
+// hr of the block (see k_bhq_offsets) are formed in the same pass.
+// ---------------------------------------------------------------------------
+template <class V, class Op>
+__device__ __forceinline__ V xor_reduce(V v, int from, Op op) {
+  for (int off = from; off < 32; off <<= 1) v = op(v, shfl_x(v, off));
+  return v;
+}
+
+template <typename T, int STEPS>
+__global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
+  __shared__ float2 red[8];
+  __shared__ int redi[8];
+  extern __shared__ int csum_s[];  // C column sums of the grad_W code set
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int C = a.C, CO = C / 8;
+  const int LPR = CO, RS = 32 / LPR, nb = a.block;
+  const int sub = lane / LPR, o = lane - sub * LPR;
+
+  // ---- global range (Q_b1 scale) from the range-pass partials ----
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < a.npart; i += blockDim.x) {
+    const float2 p = a.part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmin, gmax);
+    redi[warp] = bad;
+  }
+  for (int i = tid; i < C; i += blockDim.x) csum_s[i] = 0;
+  __syncthreads();
+  gmin = red[0].x;
+  gmax = red[0].y;
+  bad = redi[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+    gmin = fminf(gmin, red[w].x);
+    gmax = fmaxf(gmax, red[w].y);
+    bad |= redi[w];
+  }
+  if (bad) {
+    if (blockIdx.x == 0 && tid == 0) record_status(a.status, FQT_ENONFINITE);
+    return;
+  }
+  const uint32_t B2 = (1u << a.bits) - 1u;
+  const float s_g1 = affine_scale(gmin, gmax, 255u);
+  const float s_g1_16 = __fmul_rn(s_g1, 65536.0f);
+  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
+  if (blockIdx.x == 0 && tid == 0 && has_b1) {
+    a.inv1[0] = __fdiv_rn(1.0f, s_g1);
+    a.zero1[0] = __fmul_rn(s_g1, gmin);
+  }
+  int32_t *const csum_g = has_b1 ? a.csum1 : a.csum2;
+  PhiloxKeys key;
+#pragma unroll
+  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
+  const bool want_off = a.hz != nullptr;
+  int cs[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) cs[j] = 0;
+
+  const int64_t nblocks = (a.N + nb - 1) / nb;
+  const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
+  // the rows of the warp's next block are loaded while this one is worked
+  float xn[STEPS][8];
+  auto load_block = [&](int64_t blk) {
+    const int64_t r0 = blk * nb;
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      const int k = sub + RS * s;
+      if (blk < nblocks && r0 + k < a.N) {
+        load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + o * 8, xn[s]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) xn[s][j] = 0.0f;
+      }
+    }
+  };
+  int64_t blk = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
+  load_block(blk);
+  for (; blk < nblocks; blk += wstride) {
+    const int64_t r0 = blk * nb;
+    const int nrows = (int)min((int64_t)nb, a.N - r0);
+    float x[STEPS][8];
+    bool rv[STEPS];
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      rv[s] = sub + RS * s < nrows;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) x[s][j] = xn[s][j];
+    }
+    load_block(blk + wstride);
+    // ---- row statistics ----
+    float rmin[STEPS], rmax[STEPS];
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        mm.x = fminf(mm.x, x[s][j]);
+        mm.y = fmaxf(mm.y, x[s][j]);
+      }
+      mm = seg_reduce(mm, LPR, OpMinMax());
+      rmin[s] = mm.x;
+      rmax[s] = mm.y;
+    }
+    // ---- lead row (largest ||h_k||_inf, lowest index on ties), lambda2 ----
+    float bestv = -1.0f;
+    int bestk = 0x7fffffff;
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      const int k = sub + RS * s;
+      const float nk = fmaxf(fabsf(rmin[s]), fabsf(rmax[s]));
+      if (rv[s] && (nk > bestv || (nk == bestv && k < bestk))) {
+        bestv = nk;
+        bestk = k;
+      }
+    }
+    for (int off = LPR; off < 32; off <<= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bestv, off);
+      const int ok = __shfl_xor_sync(0xffffffffu, bestk, off);
+      if (ov > bestv || (ov == bestv && ok < bestk)) {
+        bestv = ov;
+        bestk = ok;
+      }
+    }
+    const int p = bestk < nrows ? bestk : 0;
+    const float np = bestv;
+    float l2 = 0.0f;
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      const int k = sub + RS * s;
+      if (rv[s] && k != p) l2 = fmaxf(l2, fmaxf(fabsf(rmin[s]), fabsf(rmax[s])));
+    }
+    l2 = xor_reduce(l2, LPR, OpMaxF());
+    const float lam2 = 2.0f * l2;
+    // range of the lead row, from the lanes that own it
+    float pmin = 0.0f, pmax = 0.0f;
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s)
+      if (s == p / RS) {
+        pmin = rmin[s];
+        pmax = rmax[s];
+      }
+    pmin = __shfl_sync(0xffffffffu, pmin, (p % RS) * LPR);
+    pmax = __shfl_sync(0xffffffffu, pmax, (p % RS) * LPR);
+    // ---- block scalars s1, s2 (App. D.4) and the reflection ----
+    float s1f = 0.0f, s2f = 0.0f, rho = 0.0f, kap = 0.0f;
+    if (np > 0.0f) {
+      float lam1 = __fsub_rn(pmax, pmin);
+      if (!(lam1 > 0.0f)) lam1 = 2.0f * np;
+      const float Nf = (float)nrows;
+      if (lam2 > 0.0f) {
+        const float c1 = cbrtf(lam1), c2 = cbrtf(lam2);
+        const float n3 = cbrtf(Nf), n6 = sqrtf(n3);
+        const float den = c1 * c1 / n3 + c2 * c2 * n3 * n3;
+        s1f = (float)B2 * n6 / (c1 * den);
+        s2f = (float)B2 * n6 / (c2 * den);
+      } else {
+        s1f = (float)B2 * sqrtf(Nf) / lam1;
+      }
+      if (nrows > 1) {
+        rho = 1.0f / sqrtf(Nf);
+        kap = 1.0f / (1.0f - rho);
+      }
+    }
+    // w_j = sum_k e_k s_k h_kj over the block (lane: its 8 columns)
+    float w[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w[j] = 0.0f;
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      const bool lead = (sub + RS * s) == p;
+      const float e = kap * (lead ? rho - 1.0f : rho);
+      const float sk = lead ? s1f : s2f;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = fmaf(e, __fmul_rn(sk, x[s][j]), w[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) w[j] = xor_reduce(w[j], LPR, OpAddF());
+    // ---- per row: transform, row minimum, rounding, packing, sums ----
+    ff sd = {0.0f, 0.0f};
+    int sR = 0;
+    float dv[STEPS];
+    int Rv[STEPS];
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s) {
+      const int k = sub + RS * s;
+      const int64_t row = r0 + k;
+      const bool lead = k == p;
+      const float sk = lead ? s1f : s2f;
+      const float ck = lead ? rho - 1.0f : rho;
+      float t[8];
+      float tmin = INFINITY;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        t[j] = fmaf(-ck, w[j], __fmul_rn(sk, x[s][j]));
+        tmin = fminf(tmin, t[j]);
+      }
+      const float z2 = seg_reduce(tmin, LPR, OpMin());
+      const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)o;
+      uint32_t c[8];
+      int rs2 = 0, rs1 = 0;
+      if (rv[s]) {
+        const uint4 w2 = philox_oct(q, 0u, key);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          c[j] = sr_code16(__fmul_rn(__fsub_rn(t[j], z2), 65536.0f), u16_of(w2, j), B2);
+          rs2 += (int)c[j];
+        }
+        if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+        if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + o * 8, c, (B2 + 1u) >> 1);
+        if (has_b1) {
+          const uint4 w1 = philox_oct(q, 1u, key);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float v = __fmul_rn(__fsub_rn(x[s][j], gmin), s_g1_16);
+            c[j] = sr_code16(v, u16_of(w1, j), 255u);
+            rs1 += (int)c[j];
+          }
+          if (a.c1) store_codes8(a.c1 + row * (int64_t)C + o * 8, c);
+          if (a.f1) store_carriers8(a.f1 + row * (int64_t)C + o * 8, c, 128u);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) cs[j] += (int)c[j];
+      }
+      rs2 = seg_reduce(rs2, LPR, OpAdd());
+      if (has_b1) rs1 = seg_reduce(rs1, LPR, OpAdd());
+      if (rv[s] && o == 0) {
+        if (a.rsum2) a.rsum2[row] = rs2;
+        if (has_b1 && a.rsum1) a.rsum1[row] = rs1;
+        a.inv2[row] = sk > 0.0f ? __fdiv_rn(1.0f, sk) : 0.0f;
+        a.zero2[row] = z2;
+      }
+      // the row's offset split 2^(b-1) + z' = m + d and R = sum_c (a + m);
+      // |z'| is a few times B sqrt(nb) here, so m and R fit int32 and m
+      // converts with the 1.5 2^23 FADD
+      const ff xo = two_sum((float)((B2 + 1u) >> 1), z2);
+      const float m = rintf(xo.h);
+      const ff d = fast_two_sum(__fsub_rn(xo.h, m), xo.l);
+      const int mi = (int)(__float_as_uint(__fadd_rn(m, 12582912.0f)) - 0x4B400000u);
+      const int R = rs2 - C * (int)((B2 + 1u) >> 1) + C * mi;
+      dv[s] = ff_round(d);
+      Rv[s] = R;
+      if (rv[s] && o == 0) {  // one lane per row adds the row's terms
+        sd = ff_add(sd, d);
+        sR += R;
+      }
+    }
+    if (want_off) {
+      // block sums of d (float-float) and R over the lanes that added them
+      for (int off = 1; off < 32; off <<= 1) {
+        const ff od = {__shfl_xor_sync(0xffffffffu, sd.h, off),
+                       __shfl_xor_sync(0xffffffffu, sd.l, off)};
+        sd = ff_add(sd, od);
+        sR += __shfl_xor_sync(0xffffffffu, sR, off);
+      }
+      float dp = 0.0f;
+      int Rp = 0;
+#pragma unroll
+      for (int s = 0; s < STEPS; ++s)
+        if (s == p / RS) {
+          dp = dv[s];
+          Rp = Rv[s];
+        }
+      dp = __shfl_sync(0xffffffffu, dp, (p % RS) * LPR);
+      Rp = __shfl_sync(0xffffffffu, Rp, (p % RS) * LPR);
+      if (nrows >= 2) {
+        const HhConst hcst = hh_const(nrows);
+        const ff rsd = ff_mul(hcst.rho, sd);
+        const ff rsR = ff_mul(hcst.rho, ff_from_i32s(sR));
+        const ff wd = ff_add(rsd, {-dp, 0.0f});
+        const ff wR = ff_add(rsR, ff_neg(ff_from_i32s(Rp)));
+#pragma unroll
+        for (int s = 0; s < STEPS; ++s) {
+          const int k = sub + RS * s;
+          if (!(rv[s] && o == 0)) continue;
+          float hzv, hrv;
+          if (k == p) {
+            hzv = ff_round(rsd);
+            hrv = ff_round(rsR);
+          } else {
+            hzv = ff_round(ff_add({dv[s], 0.0f}, ff_neg(ff_mul(hcst.kap, wd))));
+            hrv = ff_round(ff_add(ff_from_i32s(Rv[s]), ff_neg(ff_mul(hcst.kap, wR))));
+          }
+          a.hz[r0 + k] = hzv;
+          a.hr[r0 + k] = hrv;
+        }
+      } else {
+#pragma unroll
+        for (int s = 0; s < STEPS; ++s)
+          if (rv[s] && o == 0) {
+            a.hz[r0 + sub + RS * s] = dv[s];
+            a.hr[r0 + sub + RS * s] = ff_round(ff_from_i32s(Rv[s]));
+          }
+      }
+    }
+    if (o == 0 && sub == 0) a.lead2[blk] = p;
+  }
+  // ---- column sums of the grad_W code set ----
+  if (csum_g) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      int v = xor_reduce(cs[j], LPR, OpAdd());
+      if (sub == 0 && v) atomicAdd(&csum_s[o * 8 + j], v);
+    }
+    __syncthreads();
+    for (int i = tid; i < C; i += blockDim.x)
+      if (csum_s[i]) atomicAdd(&csum_g[i], csum_s[i]);
+  }
+}
+
+// Launches k_bhq_warp when the shape fits it: BHQ with rows of 64, 128 or
+// 256 columns and blocks of (32 / LPR) STEPS rows, STEPS in {1, 2, 4, 8}.
+fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st) {
+  if (a.kind != KIND_BHQ || a.C % 8) return FQT_EUNSUPPORTED;
+  const int CO = a.C / 8;
+  if (CO != 8 && CO != 16 && CO != 32) return FQT_EUNSUPPORTED;
+  const int RS = 32 / CO;
+  if (a.block % RS) return FQT_EUNSUPPORTED;
+  const int steps = a.block / RS;
+  if (steps != 1 && steps != 2 && steps != 4 && steps != 8) return FQT_EUNSUPPORTED;
+  const int64_t nblocks = (a.N + a.block - 1) / a.block;
+  int64_t grid = (nblocks + 7) / 8;
+  // persistent: the CTAs that fit at once (two per SM), each warp looping
+  const int64_t cap = (int64_t)num_sms * (steps >= 8 ? 1 : 2);
+  if (grid > cap) grid = cap;
+  if (grid < 1) grid = 1;
+  const size_t smem = sizeof(int) * (size_t)a.C;
+#define FQT_BW(S)                                                                     \
+  case S:                                                                             \
+    if (bf16)                                                                         \
+      k_bhq_warp<__nv_bfloat16, S><<<(int)grid, 256, smem, st>>>(a);                  \
+    else                                                                              \
+      k_bhq_warp<float, S><<<(int)grid, 256, smem, st>>>(a);                          \
+    break;
+  switch (steps) {
+    FQT_BW(1)
+    FQT_BW(2)
+    FQT_BW(4)
+    FQT_BW(8)
+  }
+#undef FQT_BW
+  return cuda_fail(cudaGetLastError(), "BHQ warp quantizer launch");
 }
 
 // ---------------------------------------------------------------------------
