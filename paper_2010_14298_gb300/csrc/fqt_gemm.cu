@@ -1312,8 +1312,10 @@ static SplitPlan plan_splits(int64_t M, int64_t N, int64_t K, int a_bits,
   if (p.kb_total < 1) p.kb_total = 1;
   int splits = 1;
   if (allow_split) {
+    // as many splits as keep every (tile, split) item in one wave of CTAs
     const int64_t tiles = (int64_t)p.m_tiles * p.n_tiles;
-    splits = (int)((num_sms + tiles - 1) / tiles);
+    splits = (int)(num_sms / tiles);
+    if (splits < 1) splits = 1;
     // int32 partials: a split reduces at most 2^31 / 2^(a+b-2) terms
     const int64_t max_terms = ((int64_t)1 << 31) >> (a_bits + b_bits - 2);
     const int64_t min_splits = (K + max_terms - 1) / max_terms;
