@@ -1206,29 +1206,53 @@ struct ReduceArgs {
   const float *inv_a, *zero_a, *inv_b, *zero_b;
 };
 
-__global__ void __launch_bounds__(256) k_reduce(const ReduceArgs r) {
+// A CTA sums 32 consecutive outputs over all splits: 8 groups of 32 threads
+// take every 8th split (loads of a group are one coalesced 128-byte row, four
+// in flight per thread), then the groups add up in shared memory.
+constexpr int kRedElems = 32, kRedGroups = 8;
+
+__global__ void __launch_bounds__(kRedElems * kRedGroups) k_reduce(const ReduceArgs r) {
+  __shared__ long long acc[kRedGroups][kRedElems];
   const int64_t total = r.M * r.N;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += stride) {
-    int64_t P = 0;
-    for (int s = 0; s < r.splits; ++s) P += r.part[(int64_t)s * total + idx];
-    if (r.out_i64) {
-      r.out_i64[idx] = P;
-      continue;
+  const int e = threadIdx.x % kRedElems, grp = threadIdx.x / kRedElems;
+  for (int64_t base = (int64_t)blockIdx.x * kRedElems; base < total;
+       base += (int64_t)gridDim.x * kRedElems) {
+    const int64_t idx = base + e;
+    long long P0 = 0, P1 = 0, P2 = 0, P3 = 0;
+    if (idx < total) {
+      int sp = grp;
+      for (; sp + 3 * kRedGroups < r.splits; sp += 4 * kRedGroups) {
+        P0 += r.part[(int64_t)sp * total + idx];
+        P1 += r.part[(int64_t)(sp + kRedGroups) * total + idx];
+        P2 += r.part[(int64_t)(sp + 2 * kRedGroups) * total + idx];
+        P3 += r.part[(int64_t)(sp + 3 * kRedGroups) * total + idx];
+      }
+      for (; sp < r.splits; sp += kRedGroups) P0 += r.part[(int64_t)sp * total + idx];
     }
-    const int64_t c = idx / r.N, d = idx - c * r.N;
-    const float za = *r.zero_a, zb = *r.zero_b;
-    const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
-    const float da = za + (float)ma, db = zb + (float)mb;
-    const int64_t ca = r.cs_a[c], cb = r.cs_b[d];
-    // I = sum (a - ma)(b - mb), exact, from the centred product P
-    const int64_t I = P + (r.oa - ma) * (cb - r.Kn * r.ob) +
-                      (r.ob - mb) * (ca - r.Kn * r.oa) +
-                      r.Kn * (r.oa - ma) * (r.ob - mb);
-    const float V = (float)I + db * (float)(ca - r.Kn * ma) +
-                    da * (float)(cb - r.Kn * mb) + (float)r.Kn * da * db;
-    r.out_f32[idx] = (*r.inv_a) * (*r.inv_b) * V;
+    acc[grp][e] = P0 + P1 + P2 + P3;
+    __syncthreads();
+    if (grp == 0 && idx < total) {
+      int64_t P = 0;
+#pragma unroll
+      for (int g2 = 0; g2 < kRedGroups; ++g2) P += acc[g2][e];
+      if (r.out_i64) {
+        r.out_i64[idx] = P;
+      } else {
+        const int64_t c = idx / r.N, d = idx - c * r.N;
+        const float za = *r.zero_a, zb = *r.zero_b;
+        const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
+        const float da = za + (float)ma, db = zb + (float)mb;
+        const int64_t ca = r.cs_a[c], cb = r.cs_b[d];
+        // I = sum (a - ma)(b - mb), exact, from the centred product P
+        const int64_t I = P + (r.oa - ma) * (cb - r.Kn * r.ob) +
+                          (r.ob - mb) * (ca - r.Kn * r.oa) +
+                          r.Kn * (r.oa - ma) * (r.ob - mb);
+        const float V = (float)I + db * (float)(ca - r.Kn * ma) +
+                        da * (float)(cb - r.Kn * mb) + (float)r.Kn * da * db;
+        r.out_f32[idx] = (*r.inv_a) * (*r.inv_b) * V;
+      }
+    }
+    __syncthreads();
   }
 }
 
@@ -1328,10 +1352,27 @@ static SplitPlan plan_splits(int64_t M, int64_t N, int64_t K, int a_bits,
   return p;
 }
 
+// The k_gradw plan for grad_W of C x D over K rows, or splits = 0 when the
+// shape does not fit it.
+struct WPlan {
+  int mt, ncb, Cn, stages, splits;
+  int64_t ks_blocks, kb_total;
+  size_t smem;
+};
+
+static WPlan gradw_plan(int64_t K, int64_t C, int64_t D, int b1, int bx, int num_sms);
+
 size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D) {
-  // grad_W: M = C, N = D, K = N (8-bit x 8-bit)
+  // grad_W: M = C, N = D, K = N (8-bit x 8-bit), by either kernel
   const SplitPlan p = plan_splits(C, D, N, 8, 8, device_sm_count(), true);
-  const size_t bytes = (size_t)p.splits * (size_t)C * (size_t)D * 4;
+  const int64_t splits_t = p.splits;
+  int64_t splits_w = 0;
+  for (int b = 2; b <= 8; ++b) {  // the plan depends on the Q_b1 / X~ bits
+    const WPlan w = gradw_plan(N, C, D, b, 8, device_sm_count());
+    if (w.splits > splits_w) splits_w = w.splits;
+  }
+  const int64_t splits = splits_t > splits_w ? splits_t : splits_w;
+  const size_t bytes = (size_t)splits * (size_t)C * (size_t)D * 4;
   return (bytes + 255) & ~(size_t)255;
 }
 
@@ -1425,11 +1466,11 @@ __global__ void k_u8_to_f16(const uint8_t *__restrict__ src, uint16_t *dst,
 
 static void launch_reduce(const ReduceArgs &r, cudaStream_t st) {
   const int64_t total = r.M * r.N;
-  int64_t grid = (total + 255) / 256;
-  const int64_t cap = (int64_t)device_sm_count() * 8;
+  int64_t grid = (total + kRedElems - 1) / kRedElems;
+  const int64_t cap = (int64_t)device_sm_count() * 16;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  k_reduce<<<(int)grid, 256, 0, st>>>(r);
+  k_reduce<<<(int)grid, kRedElems * kRedGroups, 0, st>>>(r);
 }
 
 static bool aligned16(const void *p) {
@@ -1482,6 +1523,241 @@ fqt_status debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
   r.out_i64 = out;
   launch_reduce(r, st);
   return cuda_fail(cudaGetLastError(), "split-K reduce launch");
+}
+
+// ---------------------------------------------------------------------------
+// grad_W with one CTA per range of K rows and all of C x D (when C <= 256
+// and ceil(D / 128) C <= 512 TMEM columns): out^T (D x C) = X~^T Q_b1 over
+// the range, as ceil(D / 128) tiles of M = 128 (D) by N = C.  Every k-block
+// of 64 rows loads X~'s rows (all D columns) and Q_b1's rows once, both
+// contiguous in memory, and issues one MMA group per D tile into its own
+// TMEM accumulator.  The range is one exact chunk (<= 2^(26 - b1 - bx)
+// terms); the epilogue writes int32 partials [split][C][D] that k_reduce
+// sums in int64.
+// ---------------------------------------------------------------------------
+constexpr int kWThreads = 320;  // TMA, MMA, 8 epilogue warps
+constexpr int kWBK = 32;           // rows of K per stage (two K = 16 MMA steps)
+constexpr size_t kWBox = 64 * kWBK * 2;  // one 64-wide fp16 box of a stage
+
+struct WArgs {
+  int64_t K;          // rows of dH / X
+  int C, D, Cn;       // Cn: C rounded up to 16 (MMA N)
+  int mt, ncb;        // D tiles of 128, 64-wide boxes of Q_b1
+  int splits;
+  int64_t ks_blocks, kb_total;
+  int stages;
+  int32_t *part;      // [splits][C][D]
+  int *status;
+};
+
+__host__ __device__ constexpr uint32_t make_idesc_mn_n(int n) {
+  // A and B MN-major, D fp32, M = 128, N = n
+  return (1u << 4) | (1u << 15) | (1u << 16) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(BM >> 4) << 24);
+}
+
+// The int32 value of an fp32 holding an exact integer of magnitude <= 2^24,
+// from its bits (no conversion instruction).
+__device__ __forceinline__ int exact_f2i(float x) {
+  const uint32_t bits = __float_as_uint(x);
+  const uint32_t e = (bits >> 23) & 0xFFu;
+  const uint32_t sig = (bits & 0x7FFFFFu) | 0x800000u;
+  const uint32_t mag = e >= 150u ? sig << (e - 150u) : __funnelshift_rc(sig, 0u, 150u - e);
+  return (bits >> 31) ? -(int)mag : (int)mag;
+}
+
+__global__ void __launch_bounds__(kWThreads, 1)
+    k_gradw(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmQ,
+            const WArgs w) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem);
+  uint64_t *full = bars, *empty = bars + kMaxStages, *accf = empty + kMaxStages,
+           *acce = accf + 1;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acce + 1);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  uint8_t *ops = smem + 1024;
+  const size_t xbytes = (size_t)w.mt * 2 * kWBox;  // per D tile: two 64-wide boxes
+  const size_t stage_bytes = xbytes + (size_t)w.ncb * kWBox;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < w.stages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(accf, 1);
+    mbar_init(acce, kPartialEpiWarps);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == kWarpMma) {
+    asm volatile(
+        "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+            smem_u32(tmem_slot)),
+        "r"(kTmemCols)
+        : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int64_t n_items = w.splits;
+
+  if (warp == kWarpTma) {
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0;
+      for (int64_t it = blockIdx.x; it < n_items && !*abort_flag; it += gridDim.x) {
+        const int64_t kb0 = it * w.ks_blocks, kb1 = min(w.kb_total, kb0 + w.ks_blocks);
+        for (int64_t kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, w.status)) { *abort_flag = 1; break; }
+          mbar_expect_tx(&full[s], (uint32_t)stage_bytes);
+          uint8_t *sx = ops + (size_t)s * stage_bytes;
+          uint8_t *sq = sx + xbytes;
+          const int32_t kc = (int32_t)(kb * kWBK);
+          for (int m = 0; m < w.mt; ++m) {
+            tma_load_2d(sx + (size_t)m * 2 * kWBox, &tmX, m * 128, kc, &full[s]);
+            tma_load_2d(sx + (size_t)m * 2 * kWBox + kWBox, &tmX, m * 128 + 64, kc, &full[s]);
+          }
+          for (int cb = 0; cb < w.ncb; ++cb)
+            tma_load_2d(sq + (size_t)cb * kWBox, &tmQ, cb * 64, kc, &full[s]);
+          if (++s == w.stages) { s = 0; ph ^= 1u; }
+        }
+      }
+      if (*abort_flag) {
+        sleep_ns(200000);
+      } else {
+        for (int i = 0; i < w.stages; ++i) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, w.status)) break;
+          if (++s == w.stages) { s = 0; ph ^= 1u; }
+        }
+      }
+    }
+  } else if (warp == kWarpMma) {
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0, eph = 0;
+      const uint32_t idesc = make_idesc_mn_n(w.Cn);
+      for (int64_t it = blockIdx.x; it < n_items && !*abort_flag; it += gridDim.x) {
+        const int64_t kb0 = it * w.ks_blocks, kb1 = min(w.kb_total, kb0 + w.ks_blocks);
+        if (!mbar_wait(acce, eph ^ 1u, w.status)) { *abort_flag = 1; break; }
+        eph ^= 1u;
+        tc_fence_after();
+        for (int64_t kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&full[s], ph, w.status)) { *abort_flag = 1; break; }
+          tc_fence_after();
+          const uint32_t x_addr = smem_u32(ops + (size_t)s * stage_bytes);
+          const uint32_t q_addr = x_addr + (uint32_t)xbytes;
+          const uint64_t dq = sw128_desc_mn(q_addr, (uint32_t)kWBox, 1024);
+          for (int m = 0; m < w.mt; ++m) {
+            const uint64_t dx =
+                sw128_desc_mn(x_addr + (uint32_t)(m * 2 * kWBox), (uint32_t)kWBox, 1024);
+#pragma unroll
+            for (int k = 0; k < kWBK / 16; ++k)
+              umma_f16(tmem + (uint32_t)(m * w.Cn), dx + (2048u >> 4) * k, dq + (2048u >> 4) * k,
+                       idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+          }
+          umma_commit(&empty[s]);
+          if (++s == w.stages) { s = 0; ph ^= 1u; }
+        }
+        umma_commit(accf);
+      }
+    }
+  } else {
+    // epilogue: warp (q, h) takes the D tiles m = h, h + 2, ...; a thread owns
+    // output column d = 128 m + 32 q + lane of grad_W^T
+    const int q = warp & 3, h = (warp - kWarpEpi0) >> 2;
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    uint32_t aph = 0;
+    for (int64_t it = blockIdx.x; it < n_items && !*abort_flag; it += gridDim.x) {
+      const bool got = mbar_wait(accf, aph, w.status);
+      if (!__all_sync(0xffffffffu, got)) { *abort_flag = 1; break; }
+      aph ^= 1u;
+      tc_fence_after();
+      int32_t *pp = w.part + it * (int64_t)w.C * w.D;
+      for (int m = h; m < w.mt; m += 2) {
+        const int d = m * 128 + q * 32 + lane;
+        for (int c0 = 0; c0 < w.Cn; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld32_nw(lane_base + (uint32_t)(m * w.Cn + c0), r);
+          tmem_wait_ld(r);
+          if (d < w.D) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (c0 + i < w.C) pp[(int64_t)(c0 + i) * w.D + d] = exact_f2i(__uint_as_float(r[i]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acce);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpMma) {
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+static WPlan gradw_plan(int64_t K, int64_t C, int64_t D, int b1, int bx, int num_sms) {
+  WPlan p;
+  memset(&p, 0, sizeof(p));
+  if (C <= 0 || C > 256 || C % 16 || D <= 0 || D % 8 || K <= 0) return p;
+  p.Cn = (int)C;
+  p.mt = (int)((D + 127) / 128);
+  if ((int64_t)p.mt * p.Cn > (int64_t)kTmemCols) return p;
+  p.ncb = (int)((C + 63) / 64);
+  const size_t stage = (size_t)p.mt * 2 * kWBox + (size_t)p.ncb * kWBox;
+  p.stages = (int)((220 * 1024 - 1024 - 1024) / stage);
+  if (p.stages > kMaxStages) p.stages = kMaxStages;
+  if (p.stages < 2) {
+    p.splits = 0;
+    return p;
+  }
+  p.smem = 1024 + (size_t)p.stages * stage + 1024;
+  p.kb_total = (K + kWBK - 1) / kWBK;
+  const int64_t kc = exact_chunk_blocks(b1, bx) * (BK / kWBK);  // k-blocks per exact chunk
+  int64_t splits = (p.kb_total + kc - 1) / kc;     // every range one exact chunk
+  if (splits < num_sms) splits = num_sms;
+  if (splits > p.kb_total) splits = p.kb_total;
+  p.ks_blocks = (p.kb_total + splits - 1) / splits;
+  p.splits = (int)((p.kb_total + p.ks_blocks - 1) / p.ks_blocks);
+  return p;
+}
+
+static fqt_status run_gradw(const uint16_t *X16, const uint16_t *Q16, int64_t K, int C, int D,
+                            const WPlan &p, int32_t *part, int *status, cudaStream_t st) {
+  CUtensorMap tx, tq;
+  bool ok = make_map_f16(&tx, X16, (uint64_t)D, (uint64_t)K, 64, kWBK);
+  ok = ok && make_map_f16(&tq, Q16, (uint64_t)C, (uint64_t)K, 64, kWBK);
+  if (!ok) return cuda_fail(cudaErrorInvalidValue, "tensor map encode");
+  WArgs w;
+  memset(&w, 0, sizeof(w));
+  w.K = K;
+  w.C = C;
+  w.D = D;
+  w.Cn = p.Cn;
+  w.mt = p.mt;
+  w.ncb = p.ncb;
+  w.splits = p.splits;
+  w.ks_blocks = p.ks_blocks;
+  w.kb_total = p.kb_total;
+  w.stages = p.stages;
+  w.part = part;
+  w.status = status;
+  const cudaError_t ea =
+      cudaFuncSetAttribute(k_gradw, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+  if (ea != cudaSuccess) return cuda_fail(ea, "grad_W shared-memory attribute");
+  const int nsm = device_sm_count();
+  const int grid = p.splits < nsm ? p.splits : nsm;
+  k_gradw<<<grid, kWThreads, p.smem, st>>>(tx, tq, w);
+  return cuda_fail(cudaGetLastError(), "grad_W launch");
 }
 
 fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
@@ -1551,10 +1827,16 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
     if (!aligned16(qa->codes_f16) || !aligned16(qx->codes_f16)) return FQT_EINVAL;
     const SplitPlan p = plan_splits(C, D, Nr, qa->bits, qx->bits, nsm, true);
-    const size_t need = kGemmOffset + (size_t)p.splits * (size_t)C * (size_t)D * 4;
+    const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, qa->bits, qx->bits, nsm) : WPlan{};
+    const int splits = wp.splits > 0 ? wp.splits : p.splits;
+    const size_t need = kGemmOffset + (size_t)splits * (size_t)C * (size_t)D * 4;
     if (ws_bytes < need) return FQT_EWORKSPACE;
     int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kGemmOffset);
-    if (Nr > 0) {
+    if (Nr > 0 && wp.splits > 0) {
+      fqt_status s = run_gradw(qx->codes_f16, qa->codes_f16, Nr, (int)C, (int)D, wp, part,
+                               status, st);
+      if (s != FQT_OK) return s;
+    } else if (Nr > 0) {
       GemmArgs g;
       memset(&g, 0, sizeof(g));
       g.status = status;
@@ -1568,7 +1850,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     ReduceArgs r;
     memset(&r, 0, sizeof(r));
     r.part = part;
-    r.splits = Nr > 0 ? p.splits : 1;
+    r.splits = Nr > 0 ? splits : 1;
     r.M = C;
     r.N = D;
     r.out_f32 = grad_W;
