@@ -255,6 +255,32 @@ __device__ __forceinline__ void tmem_ld32_nw(uint32_t taddr, uint32_t (&r)[32]) 
       : "r"(taddr));
 }
 
+__device__ __forceinline__ void tmem_ld16_nw(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+        "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]),
+        "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld8_nw(uint32_t taddr, uint32_t (&r)[8]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+        "=r"(r[6]), "=r"(r[7])
+      : "r"(taddr));
+}
+
+// W consecutive columns (W = 8, 16 or 32) of this warp's 32 lanes.
+template <int W>
+__device__ __forceinline__ void tmem_ldw_nw(uint32_t taddr, uint32_t (&r)[W]) {
+  if constexpr (W == 32) tmem_ld32_nw(taddr, r);
+  else if constexpr (W == 16) tmem_ld16_nw(taddr, r);
+  else tmem_ld8_nw(taddr, r);
+}
+
 // One column of this warp's 32 lanes, without waiting.
 __device__ __forceinline__ uint32_t tmem_ld1_nw(uint32_t taddr) {
   uint32_t v;
@@ -603,6 +629,95 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
   constexpr int NPP = leads_per_box(NB);
   constexpr int NBD = NB > 1 ? NB : 1;
   const int cwi = (int)cwc;
+  if constexpr (NB <= 32) {
+    // one block (NB >= 8) or 16 rows (no reflection) per step, loaded from
+    // TMEM on its own, so few values are live at a time
+    constexpr int CH = NB >= 8 ? NB : (NB == 1 ? 16 : 8);
+    constexpr int BPC = NB > 1 ? CH / NB : 0;  // blocks per chunk
+    const int64_t j = t.m0 + q * 32 + lane;
+    const bool jv = j < g.M;
+#pragma unroll 1
+    for (int r0 = 0; r0 < BN; r0 += CH) {
+      uint32_t r[CH];
+      tmem_ldw_nw<CH>(acc + (uint32_t)r0, r);
+      uint32_t pp[BPC > 0 ? BPC : 1];
+#pragma unroll
+      for (int b = 0; b < BPC; ++b)
+        pp[b] = tmem_ld1_nw(acc + (uint32_t)(r0 + b * NBD + leads[(r0 + b * NBD) / NBD]));
+      tmem_wait_ld(r);
+      if (BPC > 0) tmem_wait_ld(pp);
+      if (r0 + CH == BN) {  // the accumulator has been read in full
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acce_set);
+      }
+      const int64_t row0 = t.n0 + r0;
+      const int64_t left = g.N - row0;
+      const int rows = left >= CH ? CH : (int)(left > 0 ? left : 0);
+      float *po = g.out + (jv && rows > 0 ? row0 * g.M + j : 0);
+      if constexpr (NB == 1) {
+#pragma unroll
+        for (int i = 0; i < CH; ++i) {
+          const float4 kq = kp[r0 + i];
+          r[i] = __float_as_uint(dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[i])), U));
+        }
+      }
+      int lrow[BPC > 0 ? BPC : 1];
+      float lval[BPC > 0 ? BPC : 1];
+#pragma unroll
+      for (int b = 0; b < (BPC > 0 ? BPC : 1); ++b) {
+        lrow[b] = -1;
+        lval[b] = 0.0f;
+      }
+      if constexpr (NB > 1) {
+#pragma unroll
+        for (int b = 0; b < BPC; ++b) {
+          const int kb0 = r0 + b * NBD;
+          const int64_t lb = g.N - (t.n0 + kb0);
+          const int nact = lb >= NBD ? NBD : (int)(lb > 0 ? lb : 0);
+          if (nact < 2) {  // a one-row block is not transformed
+#pragma unroll
+            for (int l = 0; l < NBD; ++l) {
+              const float4 kq = kp[kb0 + l];
+              r[b * NBD + l] = __float_as_uint(
+                  dequant(kq, __fmaf_rn(kq.w, cwc, __uint_as_float(r[b * NBD + l])), U));
+            }
+            continue;
+          }
+          uint32_t sb = 0u;
+#pragma unroll
+          for (int l = 0; l < NBD; ++l) sb += magic_bits(__uint_as_float(r[b * NBD + l]));
+          const int S = (int)(sb - (uint32_t)NBD * kMagicBits) + cwi * msum[kb0 / NBD];
+          const int p = leads[kb0 / NBD];
+          const float4 kl = kp[kb0 + p];
+          const int Ip = magic_int(__uint_as_float(pp[b])) + (int)kl.w * cwi;
+          const BlockFixF f = block_fix_f(nact == NBD ? hc : hh_const(nact), S, Ip);
+#pragma unroll
+          for (int l = 0; l < NBD; ++l) {
+            const float4 kq = kp[kb0 + l];
+            r[b * NBD + l] = __float_as_uint(
+                dequant(kq, reflect_f(__uint_as_float(r[b * NBD + l]), kq, cwc, f), U));
+          }
+          lrow[b] = b * NBD + p;
+          lval[b] = dequant(kl, f.lead, U);
+        }
+      }
+      if (jv) {
+        if (rows == CH) {
+#pragma unroll
+          for (int i = 0; i < CH; ++i) __stcs(po + (int64_t)i * g.M, __uint_as_float(r[i]));
+        } else {
+#pragma unroll
+          for (int i = 0; i < CH; ++i)
+            if (i < rows) __stcs(po + (int64_t)i * g.M, __uint_as_float(r[i]));
+        }
+        // the lead rows: later stores of the same thread to the same address
+#pragma unroll
+        for (int b = 0; b < BPC; ++b)
+          if (lrow[b] >= 0 && lrow[b] < rows) __stcs(po + (int64_t)lrow[b] * g.M, lval[b]);
+      }
+    }
+  } else {
 #pragma unroll 1
   for (int g0 = 0; g0 < BN; g0 += GW) {
     int S_big = 0, Ip_big = 0, p_big = 0;
@@ -719,6 +834,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
         if (lead_row >= 0) w.st(lead_row, lead_val);
       }
     }
+  }
   }
 }
 
