@@ -887,20 +887,29 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
 // their blocks independently, without CTA barriers.  The grad_X offsets hz,
 // hr of the block (see k_bhq_offsets) are formed in the same pass.
 // ---------------------------------------------------------------------------
-template <class V, class Op>
-__device__ __forceinline__ V xor_reduce(V v, int from, Op op) {
-  for (int off = from; off < 32; off <<= 1) v = op(v, shfl_x(v, off));
+template <int FROM, class V, class Op>
+__device__ __forceinline__ V xor_reduce(V v, Op op) {
+#pragma unroll
+  for (int off = FROM; off < 32; off <<= 1) v = op(v, shfl_x(v, off));
   return v;
 }
 
-template <typename T, int STEPS>
+// Reduction over the LPR lanes of a row (LPR a power of two, compile time).
+template <int LPR, class V, class Op>
+__device__ __forceinline__ V row_reduce(V v, Op op) {
+#pragma unroll
+  for (int off = LPR >> 1; off > 0; off >>= 1) v = op(v, shfl_x(v, off));
+  return v;
+}
+
+template <typename T, int LPR, int STEPS>
 __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
   __shared__ float2 red[8];
   __shared__ int redi[8];
   extern __shared__ int csum_s[];  // C column sums of the grad_W code set
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int C = a.C, CO = C / 8;
-  const int LPR = CO, RS = 32 / LPR, nb = a.block;
+  constexpr int CO = LPR, RS = 32 / LPR, C = 8 * LPR;
+  const int nb = a.block;
   const int sub = lane / LPR, o = lane - sub * LPR;
 
   // ---- global range (Q_b1 scale) from the range-pass partials ----
@@ -955,35 +964,23 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
 
   const int64_t nblocks = (a.N + nb - 1) / nb;
   const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
-  // the rows of the warp's next block are loaded while this one is worked
-  float xn[STEPS][8];
-  auto load_block = [&](int64_t blk) {
-    const int64_t r0 = blk * nb;
-#pragma unroll
-    for (int s = 0; s < STEPS; ++s) {
-      const int k = sub + RS * s;
-      if (blk < nblocks && r0 + k < a.N) {
-        load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + o * 8, xn[s]);
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) xn[s][j] = 0.0f;
-      }
-    }
-  };
-  int64_t blk = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
-  load_block(blk);
-  for (; blk < nblocks; blk += wstride) {
+  for (int64_t blk = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; blk < nblocks;
+       blk += wstride) {
     const int64_t r0 = blk * nb;
     const int nrows = (int)min((int64_t)nb, a.N - r0);
     float x[STEPS][8];
     bool rv[STEPS];
 #pragma unroll
     for (int s = 0; s < STEPS; ++s) {
-      rv[s] = sub + RS * s < nrows;
+      const int k = sub + RS * s;
+      rv[s] = k < nrows;
+      if (rv[s]) {
+        load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + o * 8, x[s]);
+      } else {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) x[s][j] = xn[s][j];
+        for (int j = 0; j < 8; ++j) x[s][j] = 0.0f;
+      }
     }
-    load_block(blk + wstride);
     // ---- row statistics ----
     float rmin[STEPS], rmax[STEPS];
 #pragma unroll
@@ -994,7 +991,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
         mm.x = fminf(mm.x, x[s][j]);
         mm.y = fmaxf(mm.y, x[s][j]);
       }
-      mm = seg_reduce(mm, LPR, OpMinMax());
+      mm = row_reduce<LPR>(mm, OpMinMax());
       rmin[s] = mm.x;
       rmax[s] = mm.y;
     }
@@ -1010,6 +1007,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
         bestk = k;
       }
     }
+#pragma unroll
     for (int off = LPR; off < 32; off <<= 1) {
       const float ov = __shfl_xor_sync(0xffffffffu, bestv, off);
       const int ok = __shfl_xor_sync(0xffffffffu, bestk, off);
@@ -1026,7 +1024,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
       const int k = sub + RS * s;
       if (rv[s] && k != p) l2 = fmaxf(l2, fmaxf(fabsf(rmin[s]), fabsf(rmax[s])));
     }
-    l2 = xor_reduce(l2, LPR, OpMaxF());
+    l2 = xor_reduce<LPR>(l2, OpMaxF());
     const float lam2 = 2.0f * l2;
     // range of the lead row, from the lanes that own it
     float pmin = 0.0f, pmax = 0.0f;
@@ -1071,7 +1069,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
       for (int j = 0; j < 8; ++j) w[j] = fmaf(e, __fmul_rn(sk, x[s][j]), w[j]);
     }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) w[j] = xor_reduce(w[j], LPR, OpAddF());
+    for (int j = 0; j < 8; ++j) w[j] = xor_reduce<LPR>(w[j], OpAddF());
     // ---- per row: transform, row minimum, rounding, packing, sums ----
     ff sd = {0.0f, 0.0f};
     int sR = 0;
@@ -1091,7 +1089,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
         t[j] = fmaf(-ck, w[j], __fmul_rn(sk, x[s][j]));
         tmin = fminf(tmin, t[j]);
       }
-      const float z2 = seg_reduce(tmin, LPR, OpMin());
+      const float z2 = row_reduce<LPR>(tmin, OpMin());
       const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)o;
       uint32_t c[8];
       int rs2 = 0, rs1 = 0;
@@ -1118,8 +1116,8 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
 #pragma unroll
         for (int j = 0; j < 8; ++j) cs[j] += (int)c[j];
       }
-      rs2 = seg_reduce(rs2, LPR, OpAdd());
-      if (has_b1) rs1 = seg_reduce(rs1, LPR, OpAdd());
+      rs2 = row_reduce<LPR>(rs2, OpAdd());
+      if (has_b1) rs1 = row_reduce<LPR>(rs1, OpAdd());
       if (rv[s] && o == 0) {
         if (a.rsum2) a.rsum2[row] = rs2;
         if (has_b1 && a.rsum1) a.rsum1[row] = rs1;
@@ -1143,7 +1141,8 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
     }
     if (want_off) {
       // block sums of d (float-float) and R over the lanes that added them
-      for (int off = 1; off < 32; off <<= 1) {
+#pragma unroll
+      for (int off = LPR; off < 32; off <<= 1) {  // lanes o == 0 hold the rows' terms
         const ff od = {__shfl_xor_sync(0xffffffffu, sd.h, off),
                        __shfl_xor_sync(0xffffffffu, sd.l, off)};
         sd = ff_add(sd, od);
@@ -1195,7 +1194,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
   if (csum_g) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      int v = xor_reduce(cs[j], LPR, OpAdd());
+      int v = xor_reduce<LPR>(cs[j], OpAdd());
       if (sub == 0 && v) atomicAdd(&csum_s[o * 8 + j], v);
     }
     __syncthreads();
@@ -1221,19 +1220,25 @@ fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
   const size_t smem = sizeof(int) * (size_t)a.C;
-#define FQT_BW(S)                                                                     \
-  case S:                                                                             \
+#define FQT_BW(L, S)                                                                  \
+  if (CO == L && steps == S) {                                                        \
     if (bf16)                                                                         \
-      k_bhq_warp<__nv_bfloat16, S><<<(int)grid, 256, smem, st>>>(a);                  \
+      k_bhq_warp<__nv_bfloat16, L, S><<<(int)grid, 256, smem, st>>>(a);               \
     else                                                                              \
-      k_bhq_warp<float, S><<<(int)grid, 256, smem, st>>>(a);                          \
-    break;
-  switch (steps) {
-    FQT_BW(1)
-    FQT_BW(2)
-    FQT_BW(4)
-    FQT_BW(8)
+      k_bhq_warp<float, L, S><<<(int)grid, 256, smem, st>>>(a);                       \
   }
+  FQT_BW(8, 1)
+  FQT_BW(8, 2)
+  FQT_BW(8, 4)
+  FQT_BW(8, 8)
+  FQT_BW(16, 1)
+  FQT_BW(16, 2)
+  FQT_BW(16, 4)
+  FQT_BW(16, 8)
+  FQT_BW(32, 1)
+  FQT_BW(32, 2)
+  FQT_BW(32, 4)
+  FQT_BW(32, 8)
 #undef FQT_BW
   return cuda_fail(cudaGetLastError(), "BHQ warp quantizer launch");
 }
