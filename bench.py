@@ -192,9 +192,10 @@ def run_gpu(args):
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
     names = ["quantize_act", "quantize_weight", "quantize_grad", "grad_x", "grad_w"]
-    # range + codes; range + codes; range + BHQ codes + BHQ offsets; one
-    # contraction; contraction + split-K reduction
-    launches_per_call = [2, 2, 3 if KIND == 2 else 2, 1, 2]
+    # forward PTQ of X and of W: range + codes; Q_b2 / Q_b1: range +
+    # warp-per-block BHQ quantizer; grad_X: one contraction; grad_W:
+    # contraction + split-K reduction
+    launches_per_call = [2, 2, 2, 1, 2]
 
     def step(seed, evs=None):
         def mark(i):
@@ -265,8 +266,9 @@ def run_gpu(args):
         "grad_x": N * C * cb + C * D * cb + N * D * 4 + N * 12 + (N // BLOCK) * 4 + D * 4,
         "grad_w": N * C * cb + N * D * cb + C * D * 4 + (C + D) * 4,
     }
-    kern_of = {"quantize_act": "k_quant", "quantize_weight": "k_quant",
-               "quantize_grad": "k_quant", "grad_x": "k_gemm", "grad_w": "k_gemm"}
+    kern_of = {"quantize_act": "k_range + k_fwd_codes", "quantize_weight": "k_range + k_fwd_codes",
+               "quantize_grad": "k_range + k_bhq_warp", "grad_x": "k_gemm",
+               "grad_w": "k_gradw + k_reduce"}
     dom = names[int(np.argmax(per_call))]
     achieved = alg_bytes[dom] / (per_call[names.index(dom)] * 1e-3) / 1e9
     traffic = _traffic_record(dom)
