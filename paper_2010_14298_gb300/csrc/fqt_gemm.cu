@@ -86,6 +86,8 @@ struct GemmArgs {
   int64_t n_items;
   int stages, ring;           // operand stages, output boxes per epilogue warp
   int nacc;                   // TMEM accumulators in rotation (2 or 4)
+  int m_fast;                 // item order: M tiles fastest (grad_X: the D
+                              // tiles of the same output rows together)
   // grad_X epilogue (MODE_GRADX); rows of Q_b2 are the N dimension
   int kind;
   int og, ow;                  // centring offsets 2^(b-1) of Q_b2 and W~ codes
@@ -340,8 +342,13 @@ __device__ __forceinline__ Item decode_item(const GemmArgs &g, int64_t it) {
   const int64_t tiles = (int64_t)g.m_tiles * g.n_tiles;
   r.split = (int)(it / tiles);
   const int64_t t = it - (int64_t)r.split * tiles;
-  r.m0 = (t / g.n_tiles) * BM;
-  r.n0 = (t % g.n_tiles) * BN;
+  if (g.m_fast) {  // the M tiles of the same N rows side by side
+    r.m0 = (t % g.m_tiles) * BM;
+    r.n0 = (t / g.m_tiles) * BN;
+  } else {
+    r.m0 = (t / g.n_tiles) * BM;
+    r.n0 = (t % g.n_tiles) * BN;
+  }
   r.kb0 = (int64_t)r.split * g.ks_blocks;
   r.kb1 = min(g.kb_total, r.kb0 + g.ks_blocks);
   return r;
@@ -1545,6 +1552,7 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   // the next tile of each epilogue set is ready when it finishes the last;
   // otherwise two, and the other half of tensor memory holds running sums
   g.nacc = (!partial && exact_chunk_blocks(a_bits, b_bits) >= (K + BK - 1) / BK) ? 4 : 2;
+  g.m_fast = partial ? 0 : 1;
   g.M = M;
   g.N = N;
   g.K = K;
