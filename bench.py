@@ -331,6 +331,35 @@ def run_gpu(args):
                "h2d_bytes_per_step": int((N * C + N * D + C * D) * 4),
                "d2h_bytes_per_step": int((N * D + C * D) * 4)}
 
+    # ---- the quantized forward GEMM H = X~ W~^T on the same layer (the
+    # contraction core with the roles renamed), timed alone ----
+    fwd = None
+    if args.forward_steps > 0:
+        qxr = fqt.quantize_act(X, 8, row_sum=True)
+        qwr = fqt.quantize_weight(W, 8, row_sum=True)
+        H = torch.empty((N, C), dtype=torch.float32, device=dev)
+        wsf = fqt.Workspace(1, 16, 16, device=dev)
+        for _ in range(3):
+            fqt.linear_forward(qxr, qwr, ws=wsf, out=H)
+        tf = []
+        for i in range(args.forward_steps):
+            flush.fill_(i & 0xFF)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fqt.linear_forward(qxr, qwr, ws=wsf, out=H)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            tf.append(e0.elapsed_time(e1))
+        fwd_ms = float(np.median(tf))
+        fwd_bytes = N * D * cb + C * D * cb + N * C * 4 + N * 8 + C * 4
+        fwd = {"call": "linear_forward (H = X~ W~^T, one k_gemm launch)", "ms": fwd_ms,
+               "TOPS": 2 * N * C * D / (fwd_ms * 1e-3) / 1e12,
+               "algorithmic_bytes": fwd_bytes,
+               "GBs": fwd_bytes / (fwd_ms * 1e-3) / 1e9,
+               "frac_of_hbm": fwd_bytes / (fwd_ms * 1e-3) / 1e9 / hbm_peak,
+               "device_status": fqt.sync_status(wsf)}
+
     result = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -354,6 +383,7 @@ def run_gpu(args):
                      "traffic": traffic},
         "clocks": clk.summary(),
         "e2e": e2e,
+        "forward": fwd,
         "gpu_launches": int(sum(launches_per_call) * args.steps),
         "device_status": status,
     }
@@ -430,6 +460,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=8192,
                     help="rows per reference-arm step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--forward-steps", type=int, default=50,
+                    help="timed calls of the quantized forward GEMM (0: skip)")
     ap.add_argument("--eager", action="store_true",
                     help="time the C-ABI calls directly instead of graph replays")
     args = ap.parse_args()

@@ -152,6 +152,19 @@ FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,
                                size_t ws_bytes, void *stream);
 
 /*
+ * The quantized forward of the layer (Sec. 2.1, Eq. 3): H = X~ W~^T, the
+ * product of the dequantized 8-bit PTQ operands, N x C fp32 row-major.  The
+ * integer product of the codes is exact (fp16 carriers on the tensor cores,
+ * as for the backward); dequantization is applied in the epilogue.  Needs
+ * qx and qw from fqt_quantize_act / fqt_quantize_weight with codes_f16 and
+ * row_sum set (rows of X: N x D, rows of W: C x D).  D % 16 == 0 and
+ * C % 16 == 0.  `workspace` holds the status word only.
+ */
+FQT_API fqt_status fqt_linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw,
+                                      float *H, void *workspace, size_t ws_bytes,
+                                      void *stream);
+
+/*
  * grad_W = Q_b1(dH)^T X~ exactly as fqt_linear_backward computes it, for
  * callers that cannot allocate device memory when they need the backward --
  * a loop whose memory budget is frozen after warm-up, or a C host with no

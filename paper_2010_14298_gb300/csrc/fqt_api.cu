@@ -242,6 +242,11 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   return FQT_OK;
 }
 
+fqt_status fqt_linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H,
+                              void *workspace, size_t ws_bytes, void *stream) {
+  return linear_forward(qx, qw, H, workspace, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
 fqt_status fqt_linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
                                const fqt_qtensor *qx, const fqt_qtensor *qw,
                                float *grad_X, float *grad_W, void *workspace,

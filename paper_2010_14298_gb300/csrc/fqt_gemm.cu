@@ -1884,6 +1884,50 @@ static fqt_status run_gradw(const uint16_t *X16, const uint16_t *Q16, int64_t K,
   return cuda_fail(cudaGetLastError(), "grad_W launch");
 }
 
+// H = X~ W~^T (Sec. 2.1): the grad_X kernel with the roles renamed -- M = C
+// (rows of W~, K-major), N = rows of X~, K = D; the row terms of X~ take the
+// place of Q_b2's (PTQ: one scale, one zero, the row sums), W~'s row sums the
+// place of the column sums over the contraction.
+fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H, void *ws,
+                          size_t ws_bytes, cudaStream_t st) {
+  if (!qx || !qw || !H) return FQT_EINVAL;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < kHeaderBytes)
+    return FQT_EWORKSPACE;
+  if (qx->kind != FQT_PTQ || qw->kind != FQT_PTQ) return FQT_EINVAL;
+  const int64_t Nr = qx->rows, D = qx->cols, C = qw->rows;
+  if (qw->cols != D || Nr < 0) return FQT_EINVAL;
+  if (Nr == 0) return FQT_OK;
+  if (!qx->codes_f16 || !qw->codes_f16 || !qx->row_sum || !qw->row_sum || !qx->inv_s ||
+      !qx->zero || !qw->inv_s || !qw->zero)
+    return FQT_EINVAL;
+  if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
+  if (D > 8192) return FQT_EUNSUPPORTED;
+  if (!aligned16(qx->codes_f16) || !aligned16(qw->codes_f16) || !aligned16(H)) return FQT_EINVAL;
+  const int nsm = device_sm_count();
+  const SplitPlan p = plan_splits(C, Nr, D, qw->bits, qx->bits, nsm, false);
+  const int64_t kc_terms = (int64_t)exact_chunk_blocks(qw->bits, qx->bits) * BK;
+  const double mmax = floor(16777216.0 / ((double)D * (double)(1 << (qw->bits - 1)))) -
+                      (double)(1 << (qx->bits - 1)) - 1.0;
+  const int64_t pmax = D << (qw->bits + qx->bits - 2);
+  const bool flt = D <= kc_terms && mmax >= 0.0;  // no block sums: |P| < 2^24 suffices
+  (void)pmax;
+  GemmArgs g;
+  memset(&g, 0, sizeof(g));
+  g.status = reinterpret_cast<int *>(ws);
+  g.kind = FQT_PTQ;
+  g.og = 1 << (qx->bits - 1);
+  g.ow = 1 << (qw->bits - 1);
+  g.inv_s = qx->inv_s;
+  g.zero = qx->zero;
+  g.row_sum = qx->row_sum;
+  g.col_sum_w = qw->row_sum;
+  g.inv_sw = qw->inv_s;
+  g.zero_w = qw->zero;
+  g.flt_mmax = flt ? (float)mmax : -1.0f;
+  return run_gemm(qw->codes_f16, 1, qw->bits, qx->codes_f16, 1, qx->bits, C, Nr, D, p, g, H,
+                  MODE_GRADX, 1, flt, st);
+}
+
 fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
                            const fqt_qtensor *qx, const fqt_qtensor *qw,
                            float *grad_X, float *grad_W, void *ws,
@@ -1918,7 +1962,8 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       const double mmax = floor(lim / ((double)C * (double)(1 << (qw->bits - 1)))) -
                           (double)(1 << (q_b2->bits - 1)) - 1.0;
       const int64_t pmax = C << (qw->bits + q_b2->bits - 2);
-      const bool flt = C <= kc_terms && mmax >= 0.0 && pmax < ((int64_t)1 << 22);
+      // the block sums of the reflection read |P| < 2^22 off the fp32 bits
+      const bool flt = C <= kc_terms && mmax >= 0.0 && (nb == 1 || pmax < ((int64_t)1 << 22));
       GemmArgs g;
       memset(&g, 0, sizeof(g));
       g.status = status;

@@ -75,6 +75,8 @@ def load(build_if_missing: bool = True):
         lib.fqt_quantize_grad.restype = i32
         lib.fqt_linear_backward.argtypes = [QP, QP, QP, QP, P, P, P, sz, P]
         lib.fqt_linear_backward.restype = i32
+        lib.fqt_linear_forward.argtypes = [QP, QP, P, P, sz, P]
+        lib.fqt_linear_forward.restype = i32
         lib.fqt_grad_w_fixed_scratch.argtypes = [QP, QP, P, P]
         lib.fqt_grad_w_fixed_scratch.restype = i32
         lib.fqt_sync_status.argtypes = [P, P]
@@ -275,6 +277,25 @@ def quantize_grad(dH: torch.Tensor, kind: int, bits: int, block: int = 0,
     if with_b1:
         q_b1.kind, q_b1.bits, q_b1.block = PTQ, 8, 0
     return q_b2, (q_b1 if with_b1 else None)
+
+
+def linear_forward(qx: QTensor, qw: QTensor, ws: Workspace = None, out: torch.Tensor = None,
+                   stream=None) -> torch.Tensor:
+    """H = X~ W~^T (Sec. 2.1): the quantized forward of the layer (N x C fp32).
+    qx and qw need codes16 and row_sum (quantize_act / quantize_weight with
+    row_sum=True)."""
+    lib = load()
+    N, D = qx.shape
+    C = qw.shape[0]
+    dev = qx.inv_s.device
+    ws = ws or Workspace(1, 16, 16, device=dev)
+    if out is None:
+        out = torch.empty((N, C), dtype=torch.float32, device=dev)
+    sx, sw = qx.c_struct(), qw.c_struct()
+    st = lib.fqt_linear_forward(ctypes.byref(sx), ctypes.byref(sw), _ptr(out), ws.ptr,
+                                ws.nbytes, _stream(stream))
+    _check(st, "fqt_linear_forward")
+    return out
 
 
 def linear_backward(q_b2: QTensor, q_b1: Optional[QTensor], qx: QTensor,

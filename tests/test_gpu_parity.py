@@ -228,6 +228,28 @@ def test_bhq_offsets_match_oracle(N, block):
             assert np.all(np.abs(got[b0:b0 + nb] - ref) <= tol)
 
 
+@pytest.mark.parametrize("cfg,small", [(0, None), (1, 2), (2, 1), (3, 128)])
+def test_linear_forward_matches_oracle(cfg, small):
+    """H = X~ W~^T (Sec. 2.1) through the same contraction core, against the
+    oracle's dequantize-then-multiply of the GPU's forward codes."""
+    kw = {}
+    if cfg in (1, 2):
+        kw["batch"] = small
+    elif cfg == 3:
+        kw["rows"] = small
+    for L in wl.config(cfg, **kw):
+        dev = lambda a: to_dev(a, L.dtype)
+        qx = fqt.quantize_act(dev(L.X), 8, row_sum=True)
+        qw = fqt.quantize_weight(dev(L.W), 8, row_sum=True)
+        H = fqt.linear_forward(qx, qw)
+        torch.cuda.synchronize()
+        hx, hw = qx.to_numpy(), qw.to_numpy()
+        assert np.array_equal(hx["row_sum"], hx["codes"].astype(np.int64).sum(axis=1))
+        ref = orc.matmul(orc.dequant(hx), np.ascontiguousarray(orc.dequant(hw).T))
+        assert H.shape == (L.N, L.W.shape[0])
+        assert grad_rel_err(H.cpu().numpy(), ref) <= GRAD_TOL
+
+
 def test_ptq_codes_reused_for_grad_w():
     L = wl.config(0)[0]
     qx, qw, q2, q1, gx, gw = _backward(L, orc.PTQ, 8, 0, reuse=True)
