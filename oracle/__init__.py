@@ -9,6 +9,7 @@ operation, no FMA contraction) and in the plain loops here.
 Every function cites the passage of the paper it restates:
 
 * ``quantize_grad``  -- PTQ (Sec. 3.3), PSQ (Sec. 4.1), BHQ (Sec. 4.2, App. D.4)
+* ``bhq_grouping``   -- the adaptive BHQ groups of App. D.5 (block = 0)
 * ``quantize_fwd``   -- deterministic 8-bit PTQ of X and W (Sec. 2.1, App. E)
 * ``dequant``        -- Eq. 9: Q(dH) = S^-1 (codes + z' 1^T)
 * ``grad_x``/``grad_w`` -- Eq. 6 with the bifurcation of App. E
@@ -85,6 +86,13 @@ def _load():
         lib.orc_int_gemm.restype = None
         lib.orc_matmul_f64.argtypes = [P, i32, P, i64, i64, i64, P]
         lib.orc_matmul_f64.restype = None
+        lib.orc_bhq_grouping.argtypes = [P, i64, i64, P, P, P, P, P]
+        lib.orc_bhq_grouping.restype = i64
+        lib.orc_quant_bhq_groups.argtypes = [P, i64, i64, i32, P, P, i64, u64,
+                                             u32, P, P, P, P]
+        lib.orc_quant_bhq_groups.restype = i64
+        lib.orc_dequant_groups_f64.argtypes = [P, i64, i64, P, i64, P, P, P]
+        lib.orc_dequant_groups_f64.restype = None
         _lib = lib
         return lib
 
@@ -142,12 +150,17 @@ def quantize_grad(dH, kind: int, bits: int, block: int = 0, seed: int = 0,
 
     Returns codes (uint8, N x C), inv_s and zero (1 entry for PTQ, N otherwise),
     lead (BHQ: lead row of each block) and, with want_v, the pre-rounding
-    values v that SR acts on.
+    values v that SR acts on.  BHQ with block = 0 takes the adaptive groups
+    of App. D.5 (``bhq_grouping``): codes, inv_s, zero and v are then in the
+    grouped (stored) order, row k holding row perm[k] of dH, and the dict
+    also carries perm, gstart, gsize and G.
     """
     h = _f32(dH)
     n, c = h.shape
-    if kind == BHQ and block < 1:
-        raise OracleError("BHQ needs block >= 1")
+    if kind == BHQ and block < 0:
+        raise OracleError("BHQ needs block >= 0 (0 = adaptive groups)")
+    if kind == BHQ and block == 0:
+        return _quantize_bhq_adaptive(h, bits, seed, stream, want_v)
     codes = np.zeros((n, c), dtype=np.uint8)
     m = 1 if kind == PTQ else n
     inv_s = np.zeros(m, dtype=np.float32)
@@ -162,6 +175,55 @@ def quantize_grad(dH, kind: int, bits: int, block: int = 0, seed: int = 0,
         raise OracleError(f"{bad} non-finite gradient entries")
     out = dict(codes=codes, inv_s=inv_s, zero=zero, kind=kind, bits=bits,
                block=block, lead=lead[:nblk] if kind == BHQ else None)
+    if want_v:
+        out["v"] = v
+    return out
+
+
+def bhq_grouping(dH, want_v: bool = False) -> dict:
+    """Adaptive BHQ grouping of App. D.5 (reading R8 of fqt_oracle.c).
+
+    Rows sorted by M_i = ||h_i||_inf (descending, ties by index); for every
+    group count G the estimate V(G) of App. D.4's bound with the paper's
+    group sizes (N - G) M_i / sum M; G = argmin V; integer sizes by
+    cumulative rounding.  Returns perm (stored row -> dH row), gstart (G + 1
+    group starts, then N repeated up to N + 1 entries), gsize (per stored
+    row), G and, with want_v, V (V[G - 1] = V(G), N - 1 entries).
+    """
+    h = _f32(dH)
+    n, c = h.shape
+    perm = np.zeros(max(n, 1), dtype=np.int32)
+    gstart = np.zeros(n + 1, dtype=np.int32)
+    gsize = np.zeros(max(n, 1), dtype=np.int32)
+    G = np.zeros(1, dtype=np.int64)
+    V = np.zeros(max(n - 1, 1)) if want_v else None
+    bad = _load().orc_bhq_grouping(_ptr(h), n, c, _ptr(perm), _ptr(gstart),
+                                   _ptr(gsize), _ptr(G), _ptr(V))
+    if bad:
+        raise OracleError(f"{bad} non-finite gradient entries")
+    out = dict(perm=perm[:n], gstart=gstart, gsize=gsize[:n], G=int(G[0]))
+    if want_v:
+        out["V"] = V[:max(n - 1, 0)]
+    return out
+
+
+def _quantize_bhq_adaptive(h, bits, seed, stream, want_v):
+    n, c = h.shape
+    grp = bhq_grouping(h)
+    codes = np.zeros((n, c), dtype=np.uint8)
+    inv_s = np.zeros(n, dtype=np.float32)
+    zero = np.zeros(n, dtype=np.float32)
+    v = np.zeros((n, c), dtype=np.float32) if want_v else None
+    perm = np.ascontiguousarray(grp["perm"], dtype=np.int32)
+    gstart = np.ascontiguousarray(grp["gstart"], dtype=np.int32)
+    bad = _load().orc_quant_bhq_groups(_ptr(h), n, c, bits, _ptr(perm),
+                                       _ptr(gstart), grp["G"], seed, stream,
+                                       _ptr(codes), _ptr(inv_s), _ptr(zero),
+                                       _ptr(v))
+    if bad:
+        raise OracleError(f"{bad} non-finite gradient entries")
+    out = dict(codes=codes, inv_s=inv_s, zero=zero, kind=BHQ, bits=bits,
+               block=0, lead=None, **grp)
     if want_v:
         out["v"] = v
     return out
@@ -202,10 +264,23 @@ def dequant(q: dict, codes=None) -> np.ndarray:
     """The value the encoding represents, Eq. 9: diag(inv_s) Q_blk (codes + z').
 
     ``codes`` may be given as floats (e.g. expected codes); the map is affine
-    in them, so dequant(E[codes]) = E[dequant(codes)].
+    in them, so dequant(E[codes]) = E[dequant(codes)].  For the adaptive BHQ
+    groups (block = 0) the codes are in the stored order and the result is
+    returned in dH's row order (row perm[k] <- stored row k).
     """
     src = q["codes"] if codes is None else codes
     lib = _load()
+    if q["kind"] == BHQ and q.get("block", 0) == 0:
+        cd = np.ascontiguousarray(src, dtype=np.float64)
+        n, c = cd.shape
+        stored = np.zeros((n, c))
+        lib.orc_dequant_groups_f64(
+            _ptr(cd), n, c, _ptr(np.ascontiguousarray(q["gstart"], dtype=np.int32)),
+            q["G"], _ptr(np.ascontiguousarray(q["inv_s"], dtype=np.float32)),
+            _ptr(np.ascontiguousarray(q["zero"], dtype=np.float32)), _ptr(stored))
+        out = np.zeros((n, c))
+        out[np.asarray(q["perm"], dtype=np.int64)] = stored
+        return out
     if np.asarray(src).dtype == np.uint8:
         cd = np.ascontiguousarray(src, dtype=np.uint8)
         fn = lib.orc_dequant

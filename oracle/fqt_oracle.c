@@ -41,6 +41,11 @@
  *      1 / s and zero = s * z (PTQ/PSQ; Q_blk = I) or z' (BHQ).
  *  R7  Forward quantizers Q_f, Q_theta (Sec. 2.1, App. E): deterministic
  *      8-bit PTQ, round half to even, codes clamped to [0, B].
+ *  R8  Adaptive BHQ groups (App. D.5): as printed, the variance estimate
+ *      sum_i M_i^2 / size_i with size_i = (N - G) M_i / sum M equals
+ *      (sum_{i<=G} M_i)^2 / (N - G), which grows with G, so it would always
+ *      pick one group.  It is the small-row-free limit of App. D.4's bound;
+ *      the oracle keeps that bound's second term (see orc_bhq_grouping).
  */
 #include <math.h>
 #include <stdint.h>
@@ -221,11 +226,81 @@ void orc_bhq_scales(double lambda1, double lambda2, int nb, uint32_t B,
 }
 
 /* ------------------------------------------------------------------------ */
-/* Block Householder quantizer BHQ (Sec. 4.2, App. D.4; R4, R5):            */
-/* per block, S = Q diag(s1, s2, ..., s2) with the lead row p carrying s1,   */
-/* T = S H_blk, z'_k = min_j T_kj, codes = SR(T - z' 1^T).                   */
-/* `lead` receives p for every block.                                         */
+/* Block Householder quantizer BHQ (Sec. 4.2, App. D.4; R4, R5) for one      */
+/* group of nb rows: src[k] is the row of h that becomes stored row k0 + k,  */
+/* p the lead row within the group.  S = Q diag(s1, s2, ..., s2) with the    */
+/* lead row carrying s1, T = S H_grp, z'_k = min_j T_kj,                     */
+/* codes = SR(T - z' 1^T), drawn with the stored flat index (k0 + k) c + j.  */
+/* Scratch: Q nb*nb, g and t nb*c, mnr/mxr/nrm nb entries.                   */
 /* ------------------------------------------------------------------------ */
+static void bhq_group(const float *h, int64_t c, const int64_t *src, int nb,
+                      int p, int64_t k0, uint32_t B, uint64_t seed,
+                      uint32_t stream, uint8_t *codes, float *inv_s,
+                      float *zero, float *vout, double *Q, double *g, float *t,
+                      float *mnr, float *mxr, float *nrm) {
+  for (int k = 0; k < nb; ++k) {
+    orc_range(h + src[k] * c, c, &mnr[k], &mxr[k]);
+    float a = fabsf(mnr[k]), m = fabsf(mxr[k]);
+    nrm[k] = a > m ? a : m; /* ||h_k||_inf */
+  }
+  if (!(nrm[p] > 0.0f)) { /* whole group is zero */
+    for (int k = 0; k < nb; ++k) {
+      for (int64_t j = 0; j < c; ++j) {
+        codes[(k0 + k) * c + j] = 0;
+        if (vout) vout[(k0 + k) * c + j] = 0.0f;
+      }
+      inv_s[k0 + k] = 0.0f;
+      zero[k0 + k] = 0.0f;
+    }
+    return;
+  }
+  float lambda1 = mxr[p] - mnr[p];
+  if (!(lambda1 > 0.0f)) lambda1 = 2.0f * nrm[p];
+  float lambda2 = 0.0f;
+  for (int k = 0; k < nb; ++k)
+    if (k != p && nrm[k] > lambda2) lambda2 = nrm[k];
+  lambda2 = 2.0f * lambda2;
+  double s1, s2;
+  orc_bhq_scales((double)lambda1, (double)lambda2, nb, B, &s1, &s2);
+  float s1f = (float)s1;
+  float s2f = lambda2 > 0.0f ? (float)s2 : 0.0f; /* 0 marks the s2 -> inf limit */
+  /* g = diag(s) H_grp; rows other than p are zero when lambda2 = 0. */
+  for (int k = 0; k < nb; ++k) {
+    double sk = (k == p) ? (double)s1f : (double)s2f;
+    for (int64_t j = 0; j < c; ++j)
+      g[(size_t)k * c + j] = (k == p || lambda2 > 0.0f)
+                                 ? sk * (double)h[src[k] * c + j]
+                                 : 0.0;
+  }
+  orc_householder(nb, p, Q);
+  for (int k = 0; k < nb; ++k) {
+    for (int64_t j = 0; j < c; ++j) {
+      double acc = 0.0;
+      for (int m = 0; m < nb; ++m) acc += Q[k * nb + m] * g[(size_t)m * c + j];
+      t[(size_t)k * c + j] = (float)acc;
+    }
+  }
+  for (int k = 0; k < nb; ++k) {
+    float zk = INFINITY;
+    for (int64_t j = 0; j < c; ++j)
+      if (t[(size_t)k * c + j] < zk) zk = t[(size_t)k * c + j];
+    for (int64_t j = 0; j < c; ++j) {
+      int64_t i = (k0 + k) * c + j;
+      float v = t[(size_t)k * c + j] - zk;
+      if (vout) vout[i] = v;
+      codes[i] = (uint8_t)orc_sr(v, orc_u16(seed, stream, (uint64_t)i), B);
+    }
+    zero[k0 + k] = zk;
+    if (k == p)
+      inv_s[k0 + k] = 1.0f / s1f;
+    else
+      inv_s[k0 + k] = lambda2 > 0.0f ? 1.0f / s2f : 0.0f;
+  }
+}
+
+/* BHQ with contiguous blocks of `block` rows in original order (R4): the   */
+/* lead row p of a block is its first row of largest infinity norm.         */
+/* `lead` receives p for every block.                                        */
 int64_t orc_quant_bhq(const float *h, int64_t n, int64_t c, int bits,
                       int block, uint64_t seed, uint32_t stream,
                       uint8_t *codes, float *inv_s, float *zero, int32_t *lead,
@@ -240,73 +315,161 @@ int64_t orc_quant_bhq(const float *h, int64_t n, int64_t c, int bits,
   float *mnr = (float *)malloc(sizeof(float) * (size_t)block);
   float *mxr = (float *)malloc(sizeof(float) * (size_t)block);
   float *nrm = (float *)malloc(sizeof(float) * (size_t)block);
+  int64_t *src = (int64_t *)malloc(sizeof(int64_t) * (size_t)block);
   int64_t nblocks = (n + block - 1) / block;
   for (int64_t b = 0; b < nblocks; ++b) {
     int64_t r0 = b * block;
     int nb = (int)((n - r0) < block ? (n - r0) : block);
     int p = 0;
+    float best = -1.0f;
     for (int k = 0; k < nb; ++k) {
-      orc_range(h + (r0 + k) * c, c, &mnr[k], &mxr[k]);
-      float a = fabsf(mnr[k]), m = fabsf(mxr[k]);
-      nrm[k] = a > m ? a : m; /* ||h_k||_inf */
-      if (nrm[k] > nrm[p]) p = k;
+      float mn, mx;
+      orc_range(h + (r0 + k) * c, c, &mn, &mx);
+      float a = fabsf(mn), m = fabsf(mx);
+      float nk = a > m ? a : m;
+      if (nk > best) { best = nk; p = k; }
+      src[k] = r0 + k;
     }
     lead[b] = p;
-    if (!(nrm[p] > 0.0f)) { /* whole block is zero */
-      for (int k = 0; k < nb; ++k) {
-        for (int64_t j = 0; j < c; ++j) {
-          codes[(r0 + k) * c + j] = 0;
-          if (vout) vout[(r0 + k) * c + j] = 0.0f;
+    bhq_group(h, c, src, nb, p, r0, B, seed, stream, codes, inv_s, zero, vout,
+              Q, g, t, mnr, mxr, nrm);
+  }
+  free(Q); free(g); free(t); free(mnr); free(mxr); free(nrm); free(src);
+  return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Adaptive BHQ grouping (App. D.5; R8).                                     */
+/*  1. M_i = ||h_i||_inf; rows in descending M, ties by ascending row index. */
+/*  2. For G = 1 .. n-1 the first G rows are large and the other n - G      */
+/*     small; group i holds the i-th large row and size_i = (n - G) M_i /    */
+/*     S_G small rows, S_G = sum of the G large M_i.  The variance of the    */
+/*     grouping is estimated with App. D.4's bound per group,                */
+/*       V(G) = sum_i (M_i^(2/3) size_i^(-1/3) + L^(2/3) size_i^(2/3))^3,    */
+/*     L = M_(G+1), the largest small row: every group's small rows are at   */
+/*     most that large.  L -> 0 leaves sum_i M_i^2 / size_i, App. D.5's own  */
+/*     estimate.  A large row with M_i = 0 adds 0; S_G = 0 gives V = 0.      */
+/*     G = argmin V (the smallest G on ties); n = 1 gives G = 1.             */
+/*  3. Integer sizes by cumulative rounding: e_0 = 0,                        */
+/*     e_i = floor((n - G) (C_i / S_G) + 1/2) with C_i the sum of the first  */
+/*     i large M, e_G = n - G; group i takes e_i - e_(i-1) small rows.  The  */
+/*     small rows are dealt from the smallest up: group 1 takes the          */
+/*     e_1 smallest, group 2 the next e_2 - e_1, and so on.                  */
+/*  4. Stored order: group after group, each lead row first, then its small  */
+/*     rows in descending M.  perm[k] = row of h stored at k; gstart[i] =    */
+/*     first stored row of group i (i < G), gstart[G .. n] = n; gsize[k] =   */
+/*     size of the group holding stored row k.  V[G-1] = V(G) when V is     */
+/*     non-NULL (n - 1 entries).  Returns the number of non-finite entries.  */
+/* ------------------------------------------------------------------------ */
+typedef struct {
+  float m;
+  int64_t i;
+} orc_mrow;
+
+static int cmp_mrow(const void *a, const void *b) {
+  const orc_mrow *x = (const orc_mrow *)a, *y = (const orc_mrow *)b;
+  if (x->m != y->m) return x->m > y->m ? -1 : 1;
+  return x->i < y->i ? -1 : (x->i > y->i ? 1 : 0);
+}
+
+int64_t orc_bhq_grouping(const float *h, int64_t n, int64_t c, int32_t *perm,
+                         int32_t *gstart, int32_t *gsize, int64_t *G_out,
+                         double *V) {
+  float gmn, gmx;
+  int64_t bad = orc_range(h, n * c, &gmn, &gmx);
+  if (bad) return bad;
+  orc_mrow *r = (orc_mrow *)malloc(sizeof(orc_mrow) * (size_t)(n > 0 ? n : 1));
+  for (int64_t i = 0; i < n; ++i) {
+    float mn, mx;
+    orc_range(h + i * c, c, &mn, &mx);
+    float a = fabsf(mn), m = fabsf(mx);
+    r[i].m = a > m ? a : m;
+    r[i].i = i;
+  }
+  qsort(r, (size_t)n, sizeof(orc_mrow), cmp_mrow);
+  int64_t G = 1;
+  if (n >= 2) {
+    double best = INFINITY;
+    for (int64_t g = 1; g < n; ++g) {
+      double S = 0.0;
+      for (int64_t i = 0; i < g; ++i) S += (double)r[i].m;
+      double v = 0.0;
+      if (S > 0.0) {
+        double L = (double)r[g].m, cl = cbrt(L);
+        for (int64_t i = 0; i < g; ++i) {
+          double Mi = (double)r[i].m;
+          if (!(Mi > 0.0)) continue;
+          double size = (double)(n - g) * Mi / S;
+          double cm = cbrt(Mi), cs = cbrt(size);
+          double term = cm * cm / cs + cl * cl * cs * cs;
+          v += term * term * term;
         }
-        inv_s[r0 + k] = 0.0f;
-        zero[r0 + k] = 0.0f;
       }
-      continue;
-    }
-    float lambda1 = mxr[p] - mnr[p];
-    if (!(lambda1 > 0.0f)) lambda1 = 2.0f * nrm[p];
-    float lambda2 = 0.0f;
-    for (int k = 0; k < nb; ++k)
-      if (k != p && nrm[k] > lambda2) lambda2 = nrm[k];
-    lambda2 = 2.0f * lambda2;
-    double s1, s2;
-    orc_bhq_scales((double)lambda1, (double)lambda2, nb, B, &s1, &s2);
-    float s1f = (float)s1;
-    float s2f = lambda2 > 0.0f ? (float)s2 : 0.0f; /* 0 marks the s2 -> inf limit */
-    /* g = diag(s) H_blk; rows other than p are zero when lambda2 = 0. */
-    for (int k = 0; k < nb; ++k) {
-      double sk = (k == p) ? (double)s1f : (double)s2f;
-      for (int64_t j = 0; j < c; ++j)
-        g[(size_t)k * c + j] = (k == p || lambda2 > 0.0f)
-                                   ? sk * (double)h[(r0 + k) * c + j]
-                                   : 0.0;
-    }
-    orc_householder(nb, p, Q);
-    for (int k = 0; k < nb; ++k) {
-      for (int64_t j = 0; j < c; ++j) {
-        double acc = 0.0;
-        for (int m = 0; m < nb; ++m) acc += Q[k * nb + m] * g[(size_t)m * c + j];
-        t[(size_t)k * c + j] = (float)acc;
+      if (V) V[g - 1] = v;
+      if (v < best) {
+        best = v;
+        G = g;
       }
-    }
-    for (int k = 0; k < nb; ++k) {
-      float zk = INFINITY;
-      for (int64_t j = 0; j < c; ++j)
-        if (t[(size_t)k * c + j] < zk) zk = t[(size_t)k * c + j];
-      for (int64_t j = 0; j < c; ++j) {
-        int64_t i = (r0 + k) * c + j;
-        float v = t[(size_t)k * c + j] - zk;
-        if (vout) vout[i] = v;
-        codes[i] = (uint8_t)orc_sr(v, orc_u16(seed, stream, (uint64_t)i), B);
-      }
-      zero[r0 + k] = zk;
-      if (k == p)
-        inv_s[r0 + k] = 1.0f / s1f;
-      else
-        inv_s[r0 + k] = lambda2 > 0.0f ? 1.0f / s2f : 0.0f;
     }
   }
-  free(Q); free(g); free(t); free(mnr); free(mxr); free(nrm);
+  /* cumulative rounding of the sizes */
+  int64_t *e = (int64_t *)malloc(sizeof(int64_t) * (size_t)(G + 1));
+  double SG = 0.0;
+  for (int64_t i = 0; i < G; ++i) SG += (double)r[i].m;
+  e[0] = 0;
+  double Ci = 0.0;
+  for (int64_t i = 1; i <= G; ++i) {
+    Ci += (double)r[i - 1].m;
+    if (i == G)
+      e[i] = n - G;
+    else if (SG > 0.0)
+      e[i] = (int64_t)floor((double)(n - G) * (Ci / SG) + 0.5);
+    else
+      e[i] = 0;
+  }
+  for (int64_t i = 0; i < G; ++i) {
+    int64_t k0 = i + e[i], ns = e[i + 1] - e[i];
+    gstart[i] = (int32_t)k0;
+    perm[k0] = (int32_t)r[i].i;
+    for (int64_t t = 0; t < ns; ++t) perm[k0 + 1 + t] = (int32_t)r[n - e[i + 1] + t].i;
+    for (int64_t t = 0; t <= ns; ++t) gsize[k0 + t] = (int32_t)(ns + 1);
+  }
+  for (int64_t i = G; i <= n; ++i) gstart[i] = (int32_t)n;
+  *G_out = G;
+  free(e);
+  free(r);
+  return 0;
+}
+
+/* BHQ over explicit groups (App. D.5 grouping, R8): group i is stored rows */
+/* gstart[i] .. gstart[i+1]-1, read from rows perm[k] of h, lead first.     */
+int64_t orc_quant_bhq_groups(const float *h, int64_t n, int64_t c, int bits,
+                             const int32_t *perm, const int32_t *gstart,
+                             int64_t G, uint64_t seed, uint32_t stream,
+                             uint8_t *codes, float *inv_s, float *zero,
+                             float *vout) {
+  uint32_t B = (1u << bits) - 1u;
+  float gmn, gmx;
+  int64_t bad = orc_range(h, n * c, &gmn, &gmx);
+  if (bad) return bad;
+  int64_t mx = 1;
+  for (int64_t i = 0; i < G; ++i)
+    if (gstart[i + 1] - gstart[i] > mx) mx = gstart[i + 1] - gstart[i];
+  double *Q = (double *)malloc(sizeof(double) * (size_t)mx * (size_t)mx);
+  double *g = (double *)malloc(sizeof(double) * (size_t)mx * (size_t)c);
+  float *t = (float *)malloc(sizeof(float) * (size_t)mx * (size_t)c);
+  float *mnr = (float *)malloc(sizeof(float) * (size_t)mx);
+  float *mxr = (float *)malloc(sizeof(float) * (size_t)mx);
+  float *nrm = (float *)malloc(sizeof(float) * (size_t)mx);
+  int64_t *src = (int64_t *)malloc(sizeof(int64_t) * (size_t)mx);
+  for (int64_t i = 0; i < G; ++i) {
+    int64_t k0 = gstart[i];
+    int nb = (int)(gstart[i + 1] - k0);
+    for (int k = 0; k < nb; ++k) src[k] = perm[k0 + k];
+    bhq_group(h, c, src, nb, 0, k0, B, seed, stream, codes, inv_s, zero, vout,
+              Q, g, t, mnr, mxr, nrm);
+  }
+  free(Q); free(g); free(t); free(mnr); free(mxr); free(nrm); free(src);
   return 0;
 }
 
@@ -382,6 +545,32 @@ void orc_dequant_f64(const double *codes, int64_t n, int64_t c, int kind,
     }
   }
   free(Q);
+}
+
+/* Dequantization over explicit groups (R8), rows in stored order:        */
+/* out_k = inv_s_k (Q_grp (codes + z' 1^T))_k, the lead first in its group. */
+void orc_dequant_groups_f64(const double *codes, int64_t n, int64_t c,
+                            const int32_t *gstart, int64_t G,
+                            const float *inv_s, const float *zero,
+                            double *out) {
+  for (int64_t i = 0; i < G; ++i) {
+    int64_t r0 = gstart[i];
+    int nb = (int)(gstart[i + 1] - r0);
+    double *Q = (double *)malloc(sizeof(double) * (size_t)nb * (size_t)nb);
+    orc_householder(nb, 0, Q);
+    for (int k = 0; k < nb; ++k) {
+      double is = (double)inv_s[r0 + k];
+      for (int64_t j = 0; j < c; ++j) {
+        double acc = 0.0;
+        for (int m = 0; m < nb; ++m)
+          acc += Q[k * nb + m] *
+                 (codes[(r0 + m) * c + j] + (double)zero[r0 + m]);
+        out[(r0 + k) * c + j] = is * acc;
+      }
+    }
+    free(Q);
+  }
+  (void)n;
 }
 
 /* Same map for uint8 codes. */

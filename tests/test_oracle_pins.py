@@ -341,7 +341,7 @@ def test_matmul_matches_numpy():
 
 
 @pytest.mark.parametrize("kind,bits,block", [(orc.PTQ, 5, 0), (orc.PSQ, 4, 0),
-                                             (orc.BHQ, 5, 4)])
+                                             (orc.BHQ, 5, 4), (orc.BHQ, 5, 0)])
 def test_fqt_gradients_are_unbiased_exactly(kind, bits, block):
     """Thm 1: E[FQT gradient | batch] = QAT gradient, for both contractions."""
     g = wl.rng(51)
@@ -415,3 +415,173 @@ def test_linear_backward_shapes_and_bifurcation():
     # stream 1 draws differ from stream 0 draws
     q2p = orc.quantize_grad(L.dH, orc.PTQ, 8, 0, seed=0, stream=0)
     assert not np.array_equal(q2p["codes"], out["q_b1"]["codes"])
+
+
+# --------------------------------------------------------------------------
+# Adaptive BHQ grouping (App. D.5, reading R8 of the oracle)
+# --------------------------------------------------------------------------
+def _groups(q):
+    """(stored start, size) of every adaptive group."""
+    gs = q["gstart"]
+    return [(int(gs[i]), int(gs[i + 1] - gs[i])) for i in range(q["G"])]
+
+
+def test_bhq_grouping_worked_example():
+    """N = 4 rows with M = (1, 1, 8, 1).  Per group the estimate is
+    (M^(2/3) + L^(2/3) size)^3 / size, so by hand:
+    G = 1: size 3, L = 1:            (4 + 3)^3 / 3 = 343 / 3;
+    G = 2: sizes 16/9, 2/9, L = 1:   (52/9)^3 (9/16) + (11/9)^3 (9/2)
+                                     = 151256 / 1296;
+    G = 3: sizes 0.8, 0.1, 0.1:      4.8^3 / 0.8 + 2 (1.1^3 / 0.1) = 164.86.
+    G = 1 wins: one group, the row with M = 8 first, then rows 0, 1, 3."""
+    h = np.zeros((4, 8), np.float32)
+    h[:, 0] = [1, -1, 8, 1]
+    h[:, 3] = [0.5, 0.2, -3, 0.1]
+    g = orc.bhq_grouping(h, want_v=True)
+    assert np.allclose(g["V"], [343 / 3, 151256 / 1296, 164.86], rtol=1e-13, atol=0)
+    assert g["G"] == 1
+    assert list(g["perm"]) == [2, 0, 1, 3]
+    assert list(g["gstart"]) == [0, 4, 4, 4, 4]
+    assert list(g["gsize"]) == [4, 4, 4, 4]
+
+
+@pytest.mark.parametrize("n", [2, 10, 11, 64])
+def test_bhq_grouping_equal_rows(n):
+    """All M_i = c: size = (N - G) / G and V(G) = c^2 N^3 / (G (N - G)),
+    smallest at G = N / 2 (symmetric about it), i.e. pairs for even N; the
+    small rows are dealt from the end of the index order."""
+    c = 1.75
+    h = np.zeros((n, 16), np.float32)
+    h[:, 5] = c
+    h[1::2, 5] = -c
+    g = orc.bhq_grouping(h, want_v=True)
+    G = np.arange(1, n)
+    assert np.allclose(g["V"], c * c * n ** 3 / (G * (n - G)), rtol=1e-12, atol=0)
+    if n % 2 == 0:
+        assert g["G"] == n // 2
+        perm = g["perm"].reshape(-1, 2)
+        assert np.array_equal(perm[:, 0], np.arange(n // 2))
+        assert np.array_equal(perm[:, 1], n - 1 - np.arange(n // 2))
+        assert np.all(g["gsize"] == 2)
+    else:
+        assert g["G"] in ((n - 1) // 2, (n + 1) // 2)
+
+
+def test_bhq_grouping_small_rows_vanish():
+    """With the small rows all zero (L = 0) the estimate is App. D.5's own
+    sum_i M_i^2 / size_i = (sum_{i<=G} M_i)^2 / (N - G)."""
+    g0 = wl.rng(71)
+    n, K = 40, 6
+    h = np.zeros((n, 24), np.float32)
+    rows = g0.choice(n, K, replace=False)
+    h[rows] = g0.standard_normal((K, 24)) * np.array([9, 5, 3, 2, 1.5, 1.2])[:, None]
+    M = np.sort(np.abs(h).max(axis=1).astype(np.float64))[::-1]
+    g = orc.bhq_grouping(h, want_v=True)
+    for G in range(K, n):
+        assert g["V"][G - 1] == pytest.approx(M[:K].sum() ** 2 / (n - G), rel=1e-12)
+    assert g["G"] <= K
+    assert set(g["perm"][g["gstart"][:g["G"]]]) == set(rows[np.argsort(
+        -np.abs(h[rows]).max(axis=1))][:g["G"]])
+
+
+@pytest.mark.parametrize("n,seed", [(1, 0), (3, 1), (37, 2), (128, 3), (500, 4)])
+def test_bhq_grouping_invariants(n, seed):
+    """Partition, leads = the G largest rows, cumulative-rounding sizes within
+    one row of (N - G) M_i / S_G, small rows dealt from the smallest up, and
+    V(G) equal to its expansion in prefix sums of M^(1), M^(4/3), M^(5/3),
+    M^2 (term = M (t + M^(1/3) u)^3, t = (S_G / (N - G))^(1/3),
+    u = L^(2/3) ((N - G) / S_G)^(2/3))."""
+    g0 = wl.rng(80 + seed)
+    h = wl.random_grad(g0, n, 16, sigma=2.0, outlier_frac=0.05)
+    g = orc.bhq_grouping(h, want_v=True)
+    G, perm, gs = g["G"], g["perm"], g["gstart"]
+    assert np.array_equal(np.sort(perm), np.arange(n))
+    assert gs[0] == 0 and np.all(np.diff(gs[:G + 1]) >= 1) and np.all(gs[G:] == n)
+    M = np.abs(h).max(axis=1).astype(np.float64)
+    order = np.lexsort((np.arange(n), -M))
+    assert np.array_equal(perm[gs[:G]], order[:G])
+    if n == 1:
+        assert G == 1
+        return
+    Ms = M[order]
+    SG = Ms[:G].sum()
+    sizes = np.diff(gs[:G + 1]) - 1
+    assert sizes.sum() == n - G
+    assert np.all(np.abs(sizes - (n - G) * Ms[:G] / SG) <= 1.0 + 1e-9)
+    for i, (k0, nb) in enumerate(_groups(g)):
+        assert np.all(g["gsize"][k0:k0 + nb] == nb)
+        assert np.all(M[perm[k0 + 1:k0 + nb]] <= M[perm[k0]])
+        if i + 1 < G and nb > 1 and gs[i + 2] - gs[i + 1] > 1:
+            assert M[perm[k0 + 1:k0 + nb]].max() <= M[perm[gs[i + 1] + 1:gs[i + 2]]].min()
+    Gs = np.arange(1, n)
+    S = np.cumsum(Ms)[:-1]
+    t = (S / (n - Gs)) ** (1 / 3)
+    u = Ms[1:] ** (2 / 3) * ((n - Gs) / S) ** (2 / 3)
+    P = [np.cumsum(Ms ** e)[:-1] for e in (1.0, 4 / 3, 5 / 3, 2.0)]
+    V = t ** 3 * P[0] + 3 * t ** 2 * u * P[1] + 3 * t * u ** 2 * P[2] + u ** 3 * P[3]
+    assert np.allclose(g["V"], V, rtol=1e-10, atol=0)
+    assert g["V"][G - 1] == g["V"].min() and np.argmin(g["V"]) == G - 1
+
+
+def test_bhq_adaptive_single_group_is_the_blocked_bhq():
+    """One group in index order is the contiguous BHQ with block = N: same
+    codes, scales and zero points bit for bit."""
+    n = 8
+    h = np.zeros((n, 16), np.float32)
+    g0 = wl.rng(90)
+    h[0] = 40.0 * g0.standard_normal(16)
+    for k in range(1, n):
+        h[k] = g0.uniform(-0.5, 0.5, 16)
+        h[k, k] = 1.0 - 0.01 * k  # strictly decreasing M in index order
+    q = orc.quantize_grad(h, orc.BHQ, 5, 0, seed=4, want_v=True)
+    assert q["G"] == 1 and np.array_equal(q["perm"], np.arange(n))
+    r = orc.quantize_grad(h, orc.BHQ, 5, n, seed=4, want_v=True)
+    assert r["lead"][0] == 0
+    for key in ("codes", "inv_s", "zero", "v"):
+        assert np.array_equal(q[key], r[key]), key
+    assert np.array_equal(orc.dequant(q), orc.dequant(r))
+
+
+@pytest.mark.parametrize("bits,n", [(4, 12), (5, 9), (8, 16)])
+def test_bhq_adaptive_is_unbiased_exactly(bits, n):
+    g0 = wl.rng(100 + bits)
+    h = wl.random_grad(g0, n, 10, sigma=2.0, outlier_frac=0.2)
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, orc.BHQ, bits, 0, seed=5, want_v=True)
+    v = q["v"]
+    assert v.min() >= 0.0 and v.max() <= B * (1 + 1e-5)
+    m, _ = _moments(v, B)
+    e_deq = orc.dequant(q, m)
+    for k0, nb in _groups(q):
+        rows = q["perm"][k0:k0 + nb]
+        scale = np.abs(h[rows]).max()
+        assert np.abs(e_deq[rows] - h[rows]).max() <= 2e-5 * scale
+
+
+@pytest.mark.parametrize("bits", [4, 6])
+def test_bhq_adaptive_variance_bound(bits):
+    """Per adaptive group: exact variance <= D/4 ||S^-1||_F^2 and
+    ||S^-1||_F^2 <= App. D.4's bound with that group's lambda1, lambda2, n."""
+    g0 = wl.rng(110 + bits)
+    h = (1e-2 * g0.standard_normal((24, 10))).astype(np.float32)
+    h[3] = 10.0 * g0.standard_normal(10)
+    h[17] = 25.0 * g0.standard_normal(10)
+    h[9] = 4.0 * g0.standard_normal(10)
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, orc.BHQ, bits, 0, want_v=True)
+    _, var = _moments(q["v"], B)
+    D = h.shape[1]
+    assert q["G"] >= 2
+    for k0, nb in _groups(q):
+        rows = q["perm"][k0:k0 + nb]
+        inv_s = q["inv_s"][k0:k0 + nb].astype(np.float64)
+        Q = orc.householder(nb, 0)
+        vd = ((inv_s[:, None] * Q) ** 2) @ var[k0:k0 + nb]
+        frob = (inv_s ** 2).sum()
+        assert vd.sum() <= D / 4 * frob * (1 + 1e-6)
+        if nb > 1:
+            blk = h[rows].astype(np.float64)
+            lam1 = blk[0].max() - blk[0].min()
+            lam2 = 2 * np.abs(blk[1:]).max()
+            hh = (lam1 ** (2 / 3) * nb ** (-1 / 3) + lam2 ** (2 / 3) * nb ** (2 / 3)) ** 3
+            assert frob <= hh / B ** 2 * (1 + 1e-5)
