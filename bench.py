@@ -360,6 +360,50 @@ def run_gpu(args):
                "frac_of_hbm": fwd_bytes / (fwd_ms * 1e-3) / 1e9 / hbm_peak,
                "device_status": fqt.sync_status(wsf)}
 
+    # ---- adaptive BHQ groups (App. D.5) on the same layer: Q_b2 with the
+    # grouping chosen for this batch (sort, estimate, layout, group
+    # quantizer), then grad_X (contraction + the groups' reflection pass);
+    # one CUDA graph per call, timed alone ----
+    ada = None
+    if args.adaptive_steps > 0:
+        qa = fqt.QTensor.empty(N, C, fqt.BHQ, BITS, 0, True, False, dev, u8=False)
+        qa1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+        fa = [lambda: fqt.quantize_grad(dH, fqt.BHQ, BITS, 0, 7, ws=ws, q_b2=qa, q_b1=qa1),
+              lambda: fqt.linear_backward(qa, qa1, qx, qw, grad_x=True, grad_w=False, ws=ws,
+                                          out_x=gx)]
+        for _ in range(3):
+            for f in fa:
+                f()
+        torch.cuda.synchronize()
+        ga = []
+        for f in fa:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                f()
+            ga.append(g)
+        ta = [[], []]
+        for i in range(args.adaptive_steps):
+            flush.fill_(i & 0xFF)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            ev[0].record(stream)
+            ga[0].replay()
+            ev[1].record(stream)
+            ga[1].replay()
+            ev[2].record(stream)
+            torch.cuda.synchronize()
+            ta[0].append(ev[0].elapsed_time(ev[1]))
+            ta[1].append(ev[1].elapsed_time(ev[2]))
+        G = int((qa.gstart[:N] < N).sum().item())
+        grouped = int((qa.gsize > 1).sum().item())
+        ada = {"quantizer": f"BHQ-{BITS}, adaptive groups (block 0)",
+               "quantize_grad_ms": float(np.median(ta[0])),
+               "grad_x_ms": float(np.median(ta[1])),
+               "fixed_block16_ms": {"quantize_grad": float(per_call[2]),
+                                    "grad_x": float(per_call[3])},
+               "groups": G, "rows_in_multirow_groups": grouped,
+               "launches": {"quantize_grad": 10, "grad_x": 3},
+               "device_status": fqt.sync_status(ws)}
+
     result = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -384,6 +428,7 @@ def run_gpu(args):
         "clocks": clk.summary(),
         "e2e": e2e,
         "forward": fwd,
+        "adaptive_bhq": ada,
         "gpu_launches": int(sum(launches_per_call) * args.steps),
         "device_status": status,
     }
@@ -462,6 +507,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--forward-steps", type=int, default=50,
                     help="timed calls of the quantized forward GEMM (0: skip)")
+    ap.add_argument("--adaptive-steps", type=int, default=50,
+                    help="timed steps of the adaptive BHQ groups (0: skip)")
     ap.add_argument("--eager", action="store_true",
                     help="time the C-ABI calls directly instead of graph replays")
     args = ap.parse_args()

@@ -61,7 +61,9 @@ typedef enum { FQT_F32 = 0, FQT_BF16 = 1 } fqt_dtype;
  * with Q_blk = I for PTQ (Sec. 3.3) and PSQ (Sec. 4.1), and for BHQ
  * (Sec. 4.2) the block-diagonal Householder reflections
  * Q = I - 2 n n^T / ||n||^2, n = 1/sqrt(nb) 1 - e_p, one per block of
- * `block` consecutive rows (nb = rows of that block, p = its lead row).
+ * `block` consecutive rows (nb = rows of that block, p = its lead row), or,
+ * with block 0, one per adaptive group of App. D.5 (rows reordered by
+ * `perm`, each group's lead row first).
  *
  * The caller allocates every array (device memory) and sets the pointers;
  * the quantize calls fill rows, cols, bits, kind and block and write every
@@ -94,6 +96,15 @@ typedef struct fqt_qtensor {
                         a BHQ q_b2 with block > 1. */
   float *hr;         /* BHQ: rows entries, (Q_blk R)_i with R_i = row_sum_i -
                         cols 2^(b-1) + cols m_i */
+  int32_t *perm;     /* BHQ with block 0 (the adaptive groups of App. D.5):
+                        rows entries, perm[k] = row of dH held by stored row
+                        k; codes, inv_s, zero, row_sum, hz and hr are then in
+                        this stored order.  Else unused (may be NULL). */
+  int32_t *gstart;   /* BHQ block 0: rows + 1 entries, gstart[i] = first
+                        stored row of group i (its lead row), rows for every
+                        i >= G (the number of groups) */
+  int32_t *gsize;    /* BHQ block 0: rows entries, size of the group of each
+                        stored row */
 } fqt_qtensor;
 
 /* Bytes of workspace a layer with dH N x C, X N x D, W C x D needs for any
@@ -126,6 +137,15 @@ FQT_API fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t r
  * dH: N x C row-major, fp32 or bf16, C % 8 == 0.  BHQ: block a power of
  * two <= 128 and block * C <= 65536; q_b2->hz and q_b2->hr are written when
  * non-NULL (row_sum must then be non-NULL too).
+ * BHQ with block 0 takes the adaptive groups of App. D.5, as this library
+ * reads it: rows sorted by M_i = ||dH_i||_inf (descending, ties by index);
+ * for every group count G the estimate V(G) = sum_i (M_i^(2/3) s_i^(-1/3) +
+ * M_(G+1)^(2/3) s_i^(2/3))^3 of App. D.4's bound with the paper's group
+ * sizes s_i = (N - G) M_i / sum_(i<=G) M_i; G = argmin V (smallest on ties);
+ * integer sizes by cumulative rounding of the s_i, small rows dealt from the
+ * smallest up.  It writes q_b2->perm, gstart, gsize (required) and stores
+ * the groups one after another, SR uniforms drawn by stored index.  Needs
+ * C in {64, 128, 256}, N <= 2^20, and hz, hr, row_sum for the backward.
  */
 FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
                              int64_t C, fqt_kind kind, int bits, int block,
@@ -140,7 +160,11 @@ FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
  * The integer products of the codes are exact; dequantization and, for BHQ,
  * the inverse Householder transform of each block are applied in the
  * epilogue.  Reads the operands' codes_f16 and needs q_b2->row_sum (or, for
- * BHQ with block > 1, q_b2->hz and q_b2->hr), qw->col_sum (grad_X) and
+ * BHQ with block > 1, q_b2->hz and q_b2->hr; for block 0 all three and perm,
+ * gstart, gsize, in which case the inverse reflections of groups of two or
+ * more rows run as a separate pass over their grad_X rows, and the product
+ * must have the fp32-exact form: C 2^(bw + b - 2) < 2^24 and C at most one
+ * exact chunk, else FQT_EUNSUPPORTED), qw->col_sum (grad_X) and
  * q_b1->col_sum, qx->col_sum (grad_W).  q_b1 may be
  * NULL when q_b2 is PTQ with col_sum set: grad_W then uses q_b2.
  * C % 16 == 0 and D % 16 == 0.

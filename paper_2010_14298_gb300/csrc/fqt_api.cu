@@ -104,7 +104,12 @@ using namespace fqt;
 extern "C" {
 
 size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
-  return kGemmOffset + gemm_workspace_bytes(N, C, D);
+  size_t need = gemm_workspace_bytes(N, C, D);
+  const size_t grp = group_workspace_bytes(N);         // adaptive BHQ grouping
+  const size_t list = 256 + (size_t)(N > 0 ? N : 0) * 4;  // its grad_X work list
+  if (grp > need) need = grp;
+  if (list > need) need = list;
+  return kGemmOffset + need;
 }
 
 size_t fqt_debug_workspace_size(int64_t M, int64_t N, int64_t K) {
@@ -137,22 +142,28 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
     return FQT_EINVAL;
   if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
   if (kind != FQT_PTQ && kind != FQT_PSQ && kind != FQT_BHQ) return FQT_EINVAL;
+  // BHQ block 0: the adaptive groups of App. D.5
+  const bool adapt = kind == FQT_BHQ && block == 0;
   if (kind == FQT_BHQ) {
-    if (block < 1 || block > 128 || (block & (block - 1))) return FQT_EINVAL;
-    if (N > 0 && !q_b2->lead) return FQT_EINVAL;
+    if (block < 0 || block > 128 || (block & (block - 1))) return FQT_EINVAL;
+    if (N > 0 && !adapt && !q_b2->lead) return FQT_EINVAL;
+    if (N > 0 && adapt && (!q_b2->perm || !q_b2->gstart || !q_b2->gsize)) return FQT_EINVAL;
   } else {
     block = 0;
   }
   if (N > 0 && q_b1 && ((!q_b1->codes && !q_b1->codes_f16) || !q_b1->inv_s || !q_b1->zero))
     return FQT_EINVAL;
   // the grad_X offsets of BHQ (hz, hr) are reflected row sums: both or neither
-  const bool want_off = kind == FQT_BHQ && block > 1 && (q_b2->hz || q_b2->hr);
+  const bool want_off = kind == FQT_BHQ && block != 1 && (q_b2->hz || q_b2->hr);
   if (N > 0 && want_off && (!q_b2->hz || !q_b2->hr || !q_b2->row_sum)) return FQT_EINVAL;
   if (C % 8) return FQT_EUNSUPPORTED;
   if (!aligned(dH, 16) || !aligned(q_b2->codes, 16) || !aligned(q_b2->codes_f16, 16) ||
       (q_b1 && (!aligned(q_b1->codes, 16) || !aligned(q_b1->codes_f16, 16))))
     return FQT_EINVAL;
-  fqt_status s = check_ws(workspace, ws_bytes, kGemmOffset);
+  if (adapt && (C != 64 && C != 128 && C != 256)) return FQT_EUNSUPPORTED;
+  if (adapt && N > ((int64_t)1 << 20)) return FQT_EUNSUPPORTED;
+  fqt_status s = check_ws(workspace, ws_bytes,
+                          kGemmOffset + (adapt ? group_workspace_bytes(N) : 0));
   if (s != FQT_OK) return s;
   q_b2->rows = N;
   q_b2->cols = C;
@@ -172,7 +183,7 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   char *w = static_cast<char *>(workspace);
   float2 *part = reinterpret_cast<float2 *>(w + kRangeOffset);
   int npart = 0;
-  int32_t *csum = q_b1 ? q_b1->col_sum : q_b2->col_sum;
+  int32_t *csum = q_b1 ? q_b1->col_sum : (adapt ? nullptr : q_b2->col_sum);
   cudaError_t e = launch_range(dH, dtype == FQT_BF16, N * C, part, &npart, csum,
                                csum ? C : 0, nullptr, 0, nsm, st);
   if (e != cudaSuccess) return cuda_fail(e, "range pass");
@@ -211,6 +222,19 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   int nth, grid;
   size_t smem;
   const bool bf16 = dtype == FQT_BF16;
+  if (adapt) {
+    s = launch_bhq_grouping(dH, bf16, N, (int)C, q_b2->perm, q_b2->gstart, q_b2->gsize,
+                            w + kGemmOffset, ws_bytes - kGemmOffset, st);
+    if (s != FQT_OK) return s;
+    QuantArgs ag = a;
+    ag.perm = q_b2->perm;
+    ag.gstart = q_b2->gstart;
+    if (want_off) {
+      ag.hz = q_b2->hz;
+      ag.hr = q_b2->hr;
+    }
+    return launch_bhq_groups(ag, bf16, nsm, st);
+  }
   if (kind == FQT_BHQ) {
     // one warp per block when the block fits a warp's registers; the warp
     // kernel also writes the grad_X offsets

@@ -94,6 +94,9 @@ struct GemmArgs {
   const float *inv_s, *zero;   // Q_b2 metadata (1 or N entries)
   const int32_t *row_sum, *lead;
   const float *hz, *hr;        // BHQ offsets (block > 1)
+  const int32_t *perm, *gsize; // adaptive BHQ groups (NB = 0): output row and
+                               // group size of every stored row of Q_b2
+  float raw_mmax;              // NB = 0: largest |m| of a row finished here
   float flt_mmax;              // largest |m| of a tile for the fp32 form
   const int32_t *col_sum_w;    // W~ column sums over C
   const float *inv_sw, *zero_w;
@@ -639,7 +642,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
   if constexpr (NB <= 32) {
     // one block (NB >= 8) or 16 rows (no reflection) per step, loaded from
     // TMEM on its own, so few values are live at a time
-    constexpr int CH = NB >= 8 ? NB : (NB == 1 ? 16 : 8);
+    constexpr int CH = NB >= 8 ? NB : (NB <= 1 ? 16 : 8);
     constexpr int BPC = NB > 1 ? CH / NB : 0;  // blocks per chunk
     const int64_t j = t.m0 + q * 32 + lane;
     const bool jv = j < g.M;
@@ -662,7 +665,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
       const int64_t left = g.N - row0;
       const int rows = left >= CH ? CH : (int)(left > 0 ? left : 0);
       float *po = g.out + (jv && rows > 0 ? row0 * g.M + j : 0);
-      if constexpr (NB == 1) {
+      if constexpr (NB <= 1) {
 #pragma unroll
         for (int i = 0; i < CH; ++i) {
           const float4 kq = kp[r0 + i];
@@ -709,7 +712,14 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
           lval[b] = dequant(kl, f.lead, U);
         }
       }
-      if (jv) {
+      if constexpr (NB == 0) {
+        // adaptive groups: row r0 + i of the tile is row leads[r0 + i] of grad_X
+        if (jv) {
+#pragma unroll
+          for (int i = 0; i < CH; ++i)
+            if (i < rows) __stcs(g.out + (int64_t)leads[r0 + i] * g.M + j, __uint_as_float(r[i]));
+        }
+      } else if (jv) {
         if (rows == CH) {
 #pragma unroll
           for (int i = 0; i < CH; ++i) __stcs(po + (int64_t)i * g.M, __uint_as_float(r[i]));
@@ -849,6 +859,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
 struct TileLoads {
   float inv[BN / 32], zero[BN / 32], hz[BN / 32], hr[BN / 32];
   int rs[BN / 32], cs[BM / 32], lead[2];
+  int gs[BN / 32], pr[BN / 32];  // NB = 0: group size and output row
 };
 
 template <int NB>
@@ -869,6 +880,13 @@ __device__ __forceinline__ void tile_loads(const GemmArgs &g, const Item &t, int
     } else {
       L.hz[i] = L.hr[i] = 0.0f;
       L.rs[i] = kv ? __ldg(g.row_sum + k) : 0;
+    }
+    if (NB == 0) {
+      L.gs[i] = kv ? __ldg(g.gsize + k) : 1;
+      L.pr[i] = kv ? __ldg(g.perm + k) : 0;
+    } else {
+      L.gs[i] = 1;
+      L.pr[i] = 0;
     }
   }
 #pragma unroll
@@ -935,10 +953,20 @@ __device__ __forceinline__ void gradx_params(const GemmArgs &g, uint8_t *smem, u
         }
         A = __fmul_rn(sc, hd);
         B = __fmul_rn(sc, __fmaf_rn(hR, y.h, __fmul_rn(hR, y.l)));
+        if (NB == 0 && (cur.gs[i] > 1 || !(fabsf(m) <= g.raw_mmax))) {
+          // finished by the group pass: the exact integer product P alone
+          sc = 1.0f;
+          A = B = m = 0.0f;
+        }
       }
       kp[lane + 32 * i] = make_float4(sc, A, B, m);
       mabs = fmaxf(mabs, fabsf(m));
       mrow[i] = m;
+    }
+    if constexpr (NB == 0) {
+#pragma unroll
+      for (int i = 0; i < BN / 32; ++i)
+        leads[lane + 32 * i] = min(max(cur.pr[i], 0), (int)(g.N - 1));
     }
     if constexpr (NB > 1) {
       // sums of m over each block (the fp32 form's S = sum P + CWc sum m)
@@ -972,7 +1000,8 @@ __device__ __forceinline__ void gradx_params(const GemmArgs &g, uint8_t *smem, u
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1)
       mabs = fmaxf(mabs, __shfl_xor_sync(0xffffffffu, mabs, off));
-    if (lane == 0) *reinterpret_cast<int *>(P + kParFlag) = FLT && mabs <= g.flt_mmax;
+    if (lane == 0)
+      *reinterpret_cast<int *>(P + kParFlag) = NB == 0 || (FLT && mabs <= g.flt_mmax);
     __syncwarp();
     if (lane == 0) mbar_arrive(&pfull[s]);
     cur = nxt;
@@ -1054,11 +1083,15 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
         continue;
       }
       const bool multi = c > 0;
-      if (FLT && tile_f)
-        gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane);
-      else
-        gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, &acce[buf], q,
-                              lane);
+      if constexpr (NB == 0) {
+        gradx_tile_f<0>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane);
+      } else {
+        if (FLT && tile_f)
+          gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane);
+        else
+          gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, &acce[buf], q,
+                                lane);
+      }
     }
     // the parameter stage is free again
     __syncwarp();
@@ -1509,6 +1542,8 @@ static GemmKernel gemm_kernel(int mode, int nb, bool flt) {
   case NBV:                                                                  \
     return flt ? k_gemm<MODE_GRADX, NBV, true> : k_gemm<MODE_GRADX, NBV, false>;
   switch (nb) {
+    case 0:  // adaptive BHQ groups: fp32 form only
+      return flt ? k_gemm<MODE_GRADX, 0, true> : nullptr;
     FQT_GX(1)
     FQT_GX(2)
     FQT_GX(4)
@@ -1928,6 +1963,209 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
                   MODE_GRADX, 1, flt, st);
 }
 
+// ---------------------------------------------------------------------------
+// Adaptive BHQ groups (App. D.5).  After the contraction, the grad_X rows of
+// every group of two or more rows -- and of single rows whose offset m is
+// too large for the fp32 form -- hold the exact integer products P.  This
+// pass adds the offsets and applies the group's inverse Householder
+// reflection, the second of the two sparse-dense products Sec. 4.3 counts,
+// with the arithmetic of the fused epilogue: fp32 where every magnitude is
+// exact (block sums off the fp32 bits), int64 / float-float otherwise.
+// k_grp_list collects the groups that need it; k_grp_fix gives a warp one
+// (group, 128 columns) unit, each lane 4 consecutive columns.
+// ---------------------------------------------------------------------------
+struct FixArgs {
+  float *out;
+  int64_t N, D;
+  int C, og, ow, bw, b2;
+  const float *inv_s, *zero, *hz, *hr;
+  const int32_t *row_sum, *perm, *gstart;
+  const float *inv_sw, *zero_w;
+  const int32_t *col_sum_w;
+  float raw_mmax;
+  int small_p;  // every |P| < 2^22: the fp32 block sums apply
+  int32_t *list;
+  int *count;
+  int *status;
+};
+
+// Per-row terms of the epilogue: scale, the offsets (hd, hR) and m.
+struct RowTerms {
+  float sc, hd, hR, m;
+};
+
+__device__ __forceinline__ RowTerms row_terms(const FixArgs &f, int64_t k, float inv_sw,
+                                              bool reflected) {
+  RowTerms t;
+  t.sc = __fmul_rn(inv_sw, f.inv_s[k]);
+  const ff x = two_sum((float)f.og, f.zero[k]);
+  t.m = rintf(x.h);
+  if (reflected) {
+    t.hd = f.hz[k];
+    t.hR = f.hr[k];
+  } else {
+    t.hd = ff_round(fast_two_sum(__fsub_rn(x.h, t.m), x.l));
+    t.hR = __fadd_rn((float)(f.row_sum[k] - f.C * f.og), __fmul_rn((float)f.C, t.m));
+  }
+  return t;
+}
+
+__global__ void __launch_bounds__(256) k_grp_list(const FixArgs f) {
+  const int64_t gi = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  bool need = false;
+  if (gi < f.N) {
+    const int64_t k0 = f.gstart[gi];
+    if (k0 < f.N) {
+      const int64_t k1 = f.gstart[gi + 1];
+      if (k1 - k0 >= 2) {
+        need = true;
+      } else if (k1 - k0 == 1) {
+        const float m = rintf(two_sum((float)f.og, f.zero[k0]).h);
+        need = !(fabsf(m) <= f.raw_mmax);
+      }
+    }
+  }
+  const unsigned ball = __ballot_sync(0xffffffffu, need);
+  if (!ball) return;
+  const int lane = threadIdx.x & 31;
+  int base = 0;
+  if (lane == 0) base = atomicAdd(f.count, __popc(ball));
+  base = __shfl_sync(0xffffffffu, base, 0);
+  if (need) f.list[base + __popc(ball & ((1u << lane) - 1u))] = (int32_t)gi;
+}
+
+__global__ void __launch_bounds__(256) k_grp_fix(const FixArgs f) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
+  const int nchunk = (int)((f.D + 127) / 128);
+  const int64_t nunits = (int64_t)*f.count * nchunk;
+  const float inv_sw = *f.inv_sw, zw = *f.zero_w;
+  const ff y = two_sum((float)f.ow, zw);
+  const int Cn = f.C;
+  for (int64_t u = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); u < nunits;
+       u += nw) {
+    const int64_t gi = f.list[u / nchunk];
+    const int ch = (int)(u % nchunk);
+    if (gi < 0 || gi >= f.N) {
+      if (lane == 0) record_status(f.status, FQT_EINVAL);
+      continue;
+    }
+    const int64_t k0 = f.gstart[gi];
+    int64_t k1 = f.gstart[gi + 1];
+    if (k1 > f.N) k1 = f.N;
+    if (k0 < 0 || k1 <= k0) continue;
+    const int nb = (int)(k1 - k0);
+    const int64_t j = (int64_t)ch * 128 + lane * 4;
+    const bool jv = j < f.D;
+    float cwc[4], U[4];
+    int cwi[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int cs = jv ? f.col_sum_w[j + c] : 0;
+      cwc[c] = (float)(cs - Cn * f.ow);
+      cwi[c] = (int)cwc[c];
+      U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
+    }
+    const bool refl = nb >= 2;
+    // the fp32 form: |P| < 2^22 and |I| (2 + sqrt(nb)) < 2^24 for every row
+    bool fast = refl && f.small_p;
+    if (fast) {
+      const double lim = 16777216.0 / (2.0 + sqrt((double)nb));
+      const double mmax = floor(lim / ((double)Cn * (double)(1 << (f.bw - 1)))) -
+                          (double)(1 << (f.b2 - 1)) - 1.0;
+      for (int r = lane; r < nb; r += 32) {
+        const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
+        if (!((double)fabsf(m) <= mmax)) fast = false;
+      }
+      fast = __all_sync(0xffffffffu, fast);
+    }
+    auto prow = [&](int r) -> float * {
+      int64_t pr = f.perm[k0 + r];
+      if (pr < 0 || pr >= f.N) pr = 0;
+      return f.out + pr * f.D + j;
+    };
+    if (fast) {
+      const HhConst hc = hh_const(nb);
+      uint32_t sb[4] = {0u, 0u, 0u, 0u};
+      int msum = 0, Ip[4] = {0, 0, 0, 0};
+      for (int r = 0; r < nb; ++r) {
+        const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
+        msum += (int)m;
+        if (!jv) continue;
+        const float4 P = *reinterpret_cast<const float4 *>(prow(r));
+        const float pv[4] = {P.x, P.y, P.z, P.w};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          sb[c] += magic_bits(pv[c]);
+          if (r == 0) Ip[c] = magic_int(pv[c]) + (int)m * cwi[c];
+        }
+      }
+      BlockFixF bf[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int S = (int)(sb[c] - (uint32_t)nb * kMagicBits) + cwi[c] * msum;
+        bf[c] = block_fix_f(hc, S, Ip[c]);
+      }
+      for (int r = 0; r < nb; ++r) {
+        const RowTerms t = row_terms(f, k0 + r, inv_sw, true);
+        const float A = __fmul_rn(t.sc, t.hd);
+        const float B = __fmul_rn(t.sc, __fmaf_rn(t.hR, y.h, __fmul_rn(t.hR, y.l)));
+        const float4 kq = make_float4(t.sc, A, B, t.m);
+        if (!jv) continue;
+        float *po = prow(r);
+        const float4 P = *reinterpret_cast<const float4 *>(po);
+        const float pv[4] = {P.x, P.y, P.z, P.w};
+        float o4[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          o4[c] = r == 0 ? dequant(kq, bf[c].lead, U[c])
+                         : dequant(kq, reflect_f(pv[c], kq, cwc[c], bf[c]), U[c]);
+        __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+      }
+    } else {
+      // int64 integer parts I = P + m CWc, float-float reflection
+      long long S[4] = {0, 0, 0, 0}, Ipl[4] = {0, 0, 0, 0};
+      for (int r = 0; r < nb && jv; ++r) {
+        const long long m = __float2ll_rn(rintf(two_sum((float)f.og, f.zero[k0 + r]).h));
+        const float4 P = *reinterpret_cast<const float4 *>(prow(r));
+        const float pv[4] = {P.x, P.y, P.z, P.w};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const long long I = (long long)__float2int_rn(pv[c]) + m * cwi[c];
+          S[c] += I;
+          if (r == 0) Ipl[c] = I;
+        }
+      }
+      ff rS[4], beta[4];
+      if (refl) {
+        const HhConst hc = hh_const(nb);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          rS[c] = ff_mul(hc.rho, ff_from_int(S[c]));
+          beta[c] = ff_mul(hc.kap, ff_add(rS[c], ff_neg(ff_from_int(Ipl[c]))));
+        }
+      }
+      for (int r = 0; r < nb && jv; ++r) {
+        const RowTerms t = row_terms(f, k0 + r, inv_sw, refl);
+        float *po = prow(r);
+        const float4 P = *reinterpret_cast<const float4 *>(po);
+        const float pv[4] = {P.x, P.y, P.z, P.w};
+        const long long m = __float2ll_rn(t.m);
+        float o4[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const ff I = ff_from_int((long long)__float2int_rn(pv[c]) + m * cwi[c]);
+          ff v = !refl ? I : (r == 0 ? rS[c] : ff_add(I, ff_neg(beta[c])));
+          v = ff_add(v, two_prod(t.hd, U[c]));
+          v = ff_add(v, ff_mul({t.hR, 0.0f}, y));
+          o4[c] = __fmul_rn(t.sc, ff_round(v));
+        }
+        __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+      }
+    }
+  }
+}
+
 fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
                            const fqt_qtensor *qx, const fqt_qtensor *qw,
                            float *grad_X, float *grad_W, void *ws,
@@ -1940,9 +2178,13 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     if (!q_b2 || !qw || !q_b2->codes_f16 || !qw->codes_f16 || !qw->col_sum ||
         !q_b2->inv_s || !q_b2->zero || !qw->inv_s || !qw->zero)
       return FQT_EINVAL;
-    const int nb = q_b2->kind == FQT_BHQ && q_b2->block > 1 ? q_b2->block : 1;
+    // BHQ with block 0: the adaptive groups of App. D.5 (NB = 0 kernels)
+    const bool adapt = q_b2->kind == FQT_BHQ && q_b2->block == 0;
+    const int nb = adapt ? 0 : (q_b2->kind == FQT_BHQ && q_b2->block > 1 ? q_b2->block : 1);
     if (nb > 1 && (!q_b2->lead || !q_b2->hz || !q_b2->hr)) return FQT_EINVAL;
-    if (nb == 1 && !q_b2->row_sum) return FQT_EINVAL;
+    if (nb <= 1 && !q_b2->row_sum) return FQT_EINVAL;
+    if (adapt && (!q_b2->perm || !q_b2->gstart || !q_b2->gsize || !q_b2->hz || !q_b2->hr))
+      return FQT_EINVAL;
     if (nb > 128 || (nb & (nb - 1))) return FQT_EINVAL;
     const int64_t Nr = q_b2->rows, C = q_b2->cols, D = qw->cols;
     if (qw->rows != C || qw->kind != FQT_PTQ) return FQT_EINVAL;
@@ -1958,12 +2200,16 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       // reflection) for every row offset |m| <= mmax, with
       // |I| <= C 2^(bw-1) (2^(b-1) + |m|)
       const int64_t kc_terms = (int64_t)exact_chunk_blocks(qw->bits, q_b2->bits) * BK;
-      const double lim = nb == 1 ? 16777216.0 : 16777216.0 / (2.0 + sqrt((double)nb));
+      const double lim = nb <= 1 ? 16777216.0 : 16777216.0 / (2.0 + sqrt((double)nb));
       const double mmax = floor(lim / ((double)C * (double)(1 << (qw->bits - 1)))) -
                           (double)(1 << (q_b2->bits - 1)) - 1.0;
       const int64_t pmax = C << (qw->bits + q_b2->bits - 2);
       // the block sums of the reflection read |P| < 2^22 off the fp32 bits
-      const bool flt = C <= kc_terms && mmax >= 0.0 && (nb == 1 || pmax < ((int64_t)1 << 22));
+      const bool flt = C <= kc_terms && mmax >= 0.0 && (nb <= 1 || pmax < ((int64_t)1 << 22));
+      // the adaptive groups need the fp32 form (rows are scattered by perm)
+      if (adapt && !flt) return FQT_EUNSUPPORTED;
+      const size_t list_bytes = 256 + (size_t)Nr * 4;
+      if (adapt && ws_bytes < kGemmOffset + list_bytes) return FQT_EWORKSPACE;
       GemmArgs g;
       memset(&g, 0, sizeof(g));
       g.status = status;
@@ -1980,9 +2226,46 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       g.col_sum_w = qw->col_sum;
       g.inv_sw = qw->inv_s;
       g.zero_w = qw->zero;
+      g.perm = q_b2->perm;
+      g.gsize = q_b2->gsize;
+      g.raw_mmax = (float)mmax;
       fqt_status s = run_gemm(qw->codes_f16, 0, qw->bits, q_b2->codes_f16, 1, q_b2->bits,
                               D, Nr, C, p, g, grad_X, MODE_GRADX, nb, flt, st);
       if (s != FQT_OK) return s;
+      if (adapt) {
+        FixArgs f;
+        memset(&f, 0, sizeof(f));
+        f.out = grad_X;
+        f.N = Nr;
+        f.D = D;
+        f.C = (int)C;
+        f.og = g.og;
+        f.ow = g.ow;
+        f.bw = qw->bits;
+        f.b2 = q_b2->bits;
+        f.inv_s = q_b2->inv_s;
+        f.zero = q_b2->zero;
+        f.hz = q_b2->hz;
+        f.hr = q_b2->hr;
+        f.row_sum = q_b2->row_sum;
+        f.perm = q_b2->perm;
+        f.gstart = q_b2->gstart;
+        f.inv_sw = qw->inv_s;
+        f.zero_w = qw->zero;
+        f.col_sum_w = qw->col_sum;
+        f.raw_mmax = (float)mmax;
+        f.small_p = pmax < ((int64_t)1 << 22);
+        char *lw = static_cast<char *>(ws) + kGemmOffset;
+        f.count = reinterpret_cast<int *>(lw);
+        f.list = reinterpret_cast<int32_t *>(lw + 256);
+        f.status = status;
+        cudaError_t e = cudaMemsetAsync(f.count, 0, sizeof(int), st);
+        if (e != cudaSuccess) return cuda_fail(e, "group list clear");
+        k_grp_list<<<(int)((Nr + 255) / 256), 256, 0, st>>>(f);
+        k_grp_fix<<<nsm * 8, 256, 0, st>>>(f);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_fail(e, "group fix-up launch");
+      }
     }
   }
   if (grad_W) {

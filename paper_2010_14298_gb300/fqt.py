@@ -40,7 +40,8 @@ class _QT(ctypes.Structure):
                 ("zero", ctypes.c_void_p), ("row_sum", ctypes.c_void_p),
                 ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p),
                 ("codes_f16", ctypes.c_void_p), ("hz", ctypes.c_void_p),
-                ("hr", ctypes.c_void_p)]
+                ("hr", ctypes.c_void_p), ("perm", ctypes.c_void_p),
+                ("gstart", ctypes.c_void_p), ("gsize", ctypes.c_void_p)]
 
 
 def library_path() -> str:
@@ -142,8 +143,11 @@ class QTensor:
 
     ``codes`` holds the integer codes (uint8), ``codes16`` the same codes
     centred by 2^(b-1) as exact fp16 values (the tensor-core operand format);
-    either may be None.  ``hz`` and ``hr`` (BHQ, block > 1) are the reflected
-    per-row offsets the grad_X epilogue reads.
+    either may be None.  ``hz`` and ``hr`` (BHQ, block != 1) are the reflected
+    per-row offsets the grad_X epilogue reads.  BHQ with block 0 takes the
+    adaptive groups of App. D.5: rows are stored group by group, ``perm``
+    maps a stored row to its row of dH, ``gstart`` holds the group starts
+    (then N) and ``gsize`` every stored row's group size.
     """
     codes: Optional[torch.Tensor]
     inv_s: torch.Tensor
@@ -157,6 +161,9 @@ class QTensor:
     codes16: Optional[torch.Tensor] = None
     hz: Optional[torch.Tensor] = None
     hr: Optional[torch.Tensor] = None
+    perm: Optional[torch.Tensor] = None
+    gstart: Optional[torch.Tensor] = None
+    gsize: Optional[torch.Tensor] = None
 
     @property
     def shape(self):
@@ -167,8 +174,10 @@ class QTensor:
               row_sum: bool = True, col_sum: bool = True, device="cuda",
               u8: bool = True, f16: bool = True):
         m = 1 if kind == PTQ else rows
-        nblk = (rows + block - 1) // block if kind == BHQ else 0
-        offsets = kind == BHQ and block > 1 and row_sum
+        adaptive = kind == BHQ and block == 0
+        nblk = (rows + block - 1) // block if kind == BHQ and not adaptive else 0
+        offsets = kind == BHQ and block != 1 and row_sum
+        i32 = lambda n: torch.empty(n, dtype=torch.int32, device=device)
         return QTensor(
             codes=(torch.empty((rows, cols), dtype=torch.uint8, device=device)
                    if u8 else None),
@@ -180,13 +189,15 @@ class QTensor:
                      if row_sum else None),
             col_sum=(torch.empty(cols, dtype=torch.int32, device=device)
                      if col_sum else None),
-            lead=(torch.empty(max(nblk, 1), dtype=torch.int32, device=device)
-                  if kind == BHQ else None),
+            lead=i32(max(nblk, 1)) if kind == BHQ else None,
             kind=kind, bits=bits, block=block,
             hz=(torch.empty(rows, dtype=torch.float32, device=device)
                 if offsets else None),
             hr=(torch.empty(rows, dtype=torch.float32, device=device)
-                if offsets else None))
+                if offsets else None),
+            perm=i32(max(rows, 1)) if adaptive else None,
+            gstart=i32(rows + 1) if adaptive else None,
+            gsize=i32(max(rows, 1)) if adaptive else None)
 
     def c_struct(self) -> _QT:
         rows, cols = self.shape
@@ -194,7 +205,7 @@ class QTensor:
         return _QT(rows, cols, self.bits, self.kind, self.block, 0,
                    p(self.codes), self.inv_s.data_ptr(), self.zero.data_ptr(),
                    p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16),
-                   p(self.hz), p(self.hr))
+                   p(self.hz), p(self.hr), p(self.perm), p(self.gstart), p(self.gsize))
 
     def codes_from_f16(self) -> torch.Tensor:
         """The uint8 codes recovered from the fp16 carriers."""
@@ -207,7 +218,13 @@ class QTensor:
         d = dict(codes=codes.cpu().numpy(), inv_s=self.inv_s.cpu().numpy(),
                  zero=self.zero.cpu().numpy(), kind=self.kind, bits=self.bits,
                  block=self.block,
-                 lead=self.lead.cpu().numpy() if self.kind == BHQ else None)
+                 lead=(self.lead.cpu().numpy()
+                       if self.kind == BHQ and self.block != 0 else None))
+        if self.perm is not None:
+            n = codes.shape[0]
+            gs = self.gstart.cpu().numpy()
+            d.update(perm=self.perm.cpu().numpy()[:n], gstart=gs,
+                     gsize=self.gsize.cpu().numpy()[:n], G=int((gs[:n] < n).sum()))
         if self.row_sum is not None:
             d["row_sum"] = self.row_sum.cpu().numpy()
         if self.col_sum is not None:

@@ -55,3 +55,51 @@ def oracle_rows_grad_x(q2: dict, qw: dict, codes2: np.ndarray, rows: np.ndarray)
         for k in range(r1 - r0):
             out[r0 + k] = res[k]
     return np.stack([out[int(r)] for r in rows])
+
+
+def oracle_groups_grad_x(q2: dict, qw: dict, groups) -> dict:
+    """Oracle grad_X of whole adaptive BHQ groups (stored-order group ids),
+    keyed by dH row: each group dequantized on its own (App. D.5 groups are
+    independent) and multiplied by W~."""
+    Wt = orc.dequant(qw)
+    gs = q2["gstart"]
+    out = {}
+    for gi in groups:
+        k0, k1 = int(gs[gi]), int(gs[gi + 1])
+        nb = k1 - k0
+        sub = dict(q2)
+        sub.update(codes=q2["codes"][k0:k1], inv_s=q2["inv_s"][k0:k1],
+                   zero=q2["zero"][k0:k1], perm=np.arange(nb, dtype=np.int32),
+                   gstart=np.array([0, nb], dtype=np.int32), G=1)
+        res = orc.matmul(orc.dequant(sub), Wt)
+        for r in range(nb):
+            out[int(q2["perm"][k0 + r])] = res[r]
+    return out
+
+
+def grouping_closed_form(dH: np.ndarray):
+    """App. D.5 grouping estimate V(G) for every G, from prefix sums of the
+    sorted M^p (the expansion of the per-group cube), and the cumulative-
+    rounding small-row counts e_i for a given G.  Independent of the oracle's
+    direct per-G loop; used where that loop is too slow (large N)."""
+    M = np.abs(dH).max(axis=1).astype(np.float32).astype(np.float64)
+    n = M.size
+    order = np.lexsort((np.arange(n), -M))
+    Ms = M[order]
+    G = np.arange(1, n)
+    S = np.cumsum(Ms)
+    P = [np.cumsum(Ms ** e)[:-1] for e in (1.0, 4 / 3, 5 / 3, 2.0)]
+    with np.errstate(divide="ignore", invalid="ignore"):
+        t = (P[0] / (n - G)) ** (1 / 3)
+        u = Ms[1:] ** (2 / 3) * ((n - G) / P[0]) ** (2 / 3)
+        V = t ** 3 * P[0] + 3 * t ** 2 * u * P[1] + 3 * t * u ** 2 * P[2] + u ** 3 * P[3]
+    V = np.where(P[0] > 0, V, 0.0)
+
+    def sizes(g):
+        SG = S[g - 1]
+        e = np.zeros(g + 1, dtype=np.int64)
+        if SG > 0:
+            e[1:g] = np.floor((n - g) * (S[:g - 1] / SG) + 0.5)
+        e[g] = n - g
+        return e
+    return order, Ms, V, sizes

@@ -13,7 +13,8 @@ import torch
 import oracle as orc
 from paper_2010_14298_gb300 import fqt
 from paper_2010_14298_gb300 import workloads as wl
-from gpu_util import (grad_rel_err, oracle_rows_grad_x, sr_boundary_distance,
+from gpu_util import (grad_rel_err, grouping_closed_form, oracle_groups_grad_x,
+                      oracle_rows_grad_x, sr_boundary_distance,
                       to_dev)
 
 pytestmark = [pytest.mark.gpu,
@@ -83,8 +84,9 @@ def _check_b1(q1_gpu, dH, seed):
 
 def _check_bhq_codes(got, ref, v, seed, stream=0):
     diff = got.astype(np.int64) - ref.astype(np.int64)
-    agree = (diff == 0).mean()
-    assert agree >= 0.9999, agree
+    # the transform rounds differently on the two sides: a +-1 flip where t
+    # sits at an SR threshold, at most 1e-4 of the codes (two on small cases)
+    assert (diff != 0).sum() <= max(2, 1e-4 * diff.size), (diff != 0).mean()
     assert np.abs(diff).max() <= 1
     idx = np.flatnonzero(diff.ravel())
     if idx.size:
@@ -308,6 +310,44 @@ def test_ragged_and_tiny(N, kind, block):
     assert grad_rel_err(gw, orc.grad_w(h1, qx.to_numpy())) <= GRAD_TOL
 
 
+@pytest.mark.parametrize("C,N,block,dtype", [(64, 200, 16, "f32"), (64, 77, 8, "bf16"),
+                                             (128, 130, 16, "f32"), (256, 45, 8, "bf16"),
+                                             (64, 1000, 32, "f32"), (256, 300, 4, "f32")])
+def test_warp_quantizer_shapes(C, N, block, dtype):
+    """Shapes of the warp-per-block BHQ quantizer (rows of 64/128/256 columns,
+    ragged last block, bf16 input): codes against the oracle and the whole
+    backward against the oracle's dequantize-then-multiply."""
+    g = wl.rng(C + N + block)
+    dH = wl.random_grad(g, N, C, outlier_frac=0.1)
+    if dtype == "bf16":
+        dH = wl.to_bf16_values(dH)
+    X = g.uniform(-1, 1, (N, 48)).astype(np.float32)
+    W = g.standard_normal((C, 48)).astype(np.float32)
+    L = wl.Layer("warp", dH, X, W, dtype, [])
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.BHQ, 5, block)
+    ref = orc.quantize_grad(dH, orc.BHQ, 5, block, 3, orc.STREAM_B2, want_v=True)
+    _check_bhq_codes(q2.codes.cpu().numpy(), ref["codes"], ref["v"], 3)
+    assert np.array_equal(q2.lead.cpu().numpy(), ref["lead"])
+    _check_b1(q1, dH, 3)
+    h2, h1 = q2.to_numpy(), q1.to_numpy()
+    assert grad_rel_err(gx, orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+    assert grad_rel_err(gw, orc.grad_w(h1, qx.to_numpy())) <= GRAD_TOL
+
+
+@pytest.mark.parametrize("N,C,D", [(1000, 16, 48), (333, 48, 208), (4097, 64, 576),
+                                   (64, 256, 256), (2051, 32, 1024)])
+def test_grad_w_shapes(N, C, D):
+    """grad_W through the one-CTA-per-K-range kernel at ragged K, C < 64 and
+    several D tiles, against the oracle."""
+    g = wl.rng(N + C + D)
+    dH = wl.random_grad(g, N, C)
+    X = g.uniform(-1, 1, (N, D)).astype(np.float32)
+    W = g.standard_normal((C, D)).astype(np.float32)
+    L = wl.Layer("gw", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.PSQ, 5, 0)
+    assert grad_rel_err(gw, orc.grad_w(q1.to_numpy(), qx.to_numpy())) <= GRAD_TOL
+
+
 def test_zero_and_constant_gradients():
     dH = np.zeros((64, 32), dtype=np.float32)
     dH[10] = 1.5
@@ -354,3 +394,121 @@ def test_argument_errors():
     with pytest.raises(fqt.FqtError) as e:
         fqt.quantize_grad(torch.zeros((16, 16), device="cuda"), orc.BHQ, 5, 3, 0)
     assert e.value.status == 1
+
+
+# --------------------------------------------------------------------------
+# Adaptive BHQ groups (App. D.5; BHQ with block 0)
+# --------------------------------------------------------------------------
+def _adaptive_cases():
+    g = wl.rng(300)
+    out = []
+    for n, c in ((1, 64), (2, 64), (7, 128), (130, 64), (4097, 64), (5000, 256)):
+        out.append((f"random-{n}x{c}", wl.random_grad(g, n, c, sigma=2.0, outlier_frac=0.05)))
+    eq = np.zeros((64, 64), np.float32)
+    eq[:, 7] = 2.5
+    eq[1::2, 7] = -2.5
+    out.append(("equal-rows-64", eq))
+    out.append(("cfg0-128", wl.config(0)[0].dH[:, :128].copy()))
+    out.append(("cfg1-b2", wl.config(1, batch=2)[0].dH))
+    out.append(("cfg2-b1", wl.config(2, batch=1)[0].dH))
+    return out
+
+
+ADAPTIVE = _adaptive_cases()
+
+
+@pytest.mark.parametrize("idx", range(len(ADAPTIVE)), ids=[a[0] for a in ADAPTIVE])
+def test_bhq_grouping_matches_oracle(idx):
+    """perm, gstart, gsize and G of the GPU grouping equal the oracle's."""
+    name, dH = ADAPTIVE[idx]
+    q2, _ = fqt.quantize_grad(to_dev(dH), orc.BHQ, 5, 0, seed=3, with_b1=False)
+    torch.cuda.synchronize()
+    h2 = q2.to_numpy()
+    ref = orc.bhq_grouping(dH)
+    assert h2["G"] == ref["G"]
+    assert np.array_equal(h2["perm"], ref["perm"])
+    assert np.array_equal(h2["gstart"], ref["gstart"])
+    assert np.array_equal(h2["gsize"], ref["gsize"])
+
+
+@pytest.mark.parametrize("idx", range(len(ADAPTIVE)), ids=[a[0] for a in ADAPTIVE])
+@pytest.mark.parametrize("bits", [4, 5, 8])
+def test_bhq_adaptive_backward_matches_oracle(idx, bits):
+    """Codes (stored order) and Q_b1 against the oracle; grad_X (scattered
+    back to dH's row order) and grad_W against the oracle's
+    dequantize-then-multiply of the GPU codes."""
+    name, dH = ADAPTIVE[idx]
+    n, c = dH.shape
+    g = wl.rng(n + c + bits)
+    X = g.uniform(-1, 1, (n, 48)).astype(np.float32)
+    W = (0.05 * g.standard_normal((c, 48))).astype(np.float32)
+    L = wl.Layer(name, dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.BHQ, bits, 0)
+    ref = orc.quantize_grad(dH, orc.BHQ, bits, 0, 3, orc.STREAM_B2, want_v=True)
+    h2 = q2.to_numpy()
+    assert np.array_equal(h2["perm"], ref["perm"])
+    _check_bhq_codes(h2["codes"], ref["codes"], ref["v"], 3)
+    _check_b1(q1, dH, 3)
+    assert grad_rel_err(gx, orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+    assert grad_rel_err(gw, orc.grad_w(q1.to_numpy(), qx.to_numpy())) <= GRAD_TOL
+
+
+def test_bhq_adaptive_bf16_and_wide_rows():
+    g = wl.rng(310)
+    dH = wl.to_bf16_values(wl.random_grad(g, 900, 128, sigma=2.5, outlier_frac=0.1))
+    X = g.uniform(-1, 1, (900, 64)).astype(np.float32)
+    W = (0.05 * g.standard_normal((128, 64))).astype(np.float32)
+    L = wl.Layer("bf16", dH, X, W, "bf16", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.BHQ, 5, 0)
+    ref = orc.quantize_grad(dH, orc.BHQ, 5, 0, 3, orc.STREAM_B2, want_v=True)
+    h2 = q2.to_numpy()
+    assert np.array_equal(h2["perm"], ref["perm"])
+    _check_bhq_codes(h2["codes"], ref["codes"], ref["v"], 3)
+    assert grad_rel_err(gx, orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+
+
+def test_bhq_adaptive_large_offsets_take_the_exact_path():
+    """Rows of one sign with a tiny range have offsets m far beyond the fp32
+    form: the contraction leaves them raw and the group pass finishes them
+    in int64 / float-float."""
+    g = wl.rng(320)
+    dH = wl.random_grad(g, 300, 64, sigma=1.0)
+    dH[10] = 50.0 + 1e-4 * g.standard_normal(64)   # all positive, R ~ 5e-4
+    dH[11] = -20.0 + 1e-3 * g.standard_normal(64)
+    X = g.uniform(-1, 1, (300, 32)).astype(np.float32)
+    W = (0.05 * g.standard_normal((64, 32))).astype(np.float32)
+    L = wl.Layer("offsets", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.BHQ, 5, 0)
+    h2 = q2.to_numpy()
+    m = np.rint(np.float32(16) + h2["zero"])
+    # the fp32 form holds |m| <= 2^24 / (C 2^(bw-1)) - 2^(b-1) - 1 = 2031 here
+    assert np.abs(m).max() > 2031
+    assert grad_rel_err(gx, orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+
+
+def test_bhq_adaptive_full_size_sampled():
+    """The ResNet-18 conv workload at full size (131072 x 64): the grouping
+    against its definition (closed form of the estimate, leads, cumulative
+    rounding), grad_X on sampled whole groups."""
+    L = wl.config(1)[0]
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.BHQ, 5, 0, seed=11)
+    h2, hw = q2.to_numpy(), qw.to_numpy()
+    n = L.N
+    order, Ms, V, sizes = grouping_closed_form(L.dH)
+    G = h2["G"]
+    best = V.min()
+    assert V[G - 1] <= best * (1 + 1e-12)
+    if V[G - 1] > best:  # a near tie: the other choice is as good
+        assert np.argmin(V) + 1 != G
+    gs = h2["gstart"]
+    assert np.all(gs[G:] == n) and np.all(np.diff(gs[:G + 1]) >= 1)
+    assert np.array_equal(h2["perm"][gs[:G]], order[:G])
+    e = sizes(G)
+    assert np.array_equal(np.diff(gs[:G + 1]) - 1, np.diff(e))
+    assert np.array_equal(np.sort(h2["perm"]), np.arange(n))
+    g = wl.rng(7)
+    big = np.argsort(-(np.diff(gs[:G + 1])))[:8]
+    groups = np.unique(np.concatenate([big, g.choice(G, 56, replace=False)]))
+    ref = oracle_groups_grad_x(h2, hw, groups)
+    rows = np.array(sorted(ref))
+    assert grad_rel_err(gx[rows], np.stack([ref[r] for r in rows])) <= GRAD_TOL
