@@ -1984,6 +1984,7 @@ struct FixArgs {
   const int32_t *col_sum_w;
   float raw_mmax;
   int small_p;  // every |P| < 2^22: the fp32 block sums apply
+  float mmax_nb[33];  // groups of nb <= 32 rows: largest |m| of the fp32 form
   int32_t *list;
   int *count;
   int *status;
@@ -2034,7 +2035,125 @@ __global__ void __launch_bounds__(256) k_grp_list(const FixArgs f) {
   if (need) f.list[base + __popc(ball & ((1u << lane) - 1u))] = (int32_t)gi;
 }
 
-__global__ void __launch_bounds__(256) k_grp_fix(const FixArgs f) {
+// Any group (or a single row left raw): rows visited one by one; the fp32
+// form where it is exact, else int64 integer parts and float-float.
+__device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int nb, int64_t j,
+                                               bool jv, const float (&cwc)[4],
+                                               const int (&cwi)[4], const float (&U)[4],
+                                               float inv_sw, const ff &y) {
+  const int lane = threadIdx.x & 31;
+  const int Cn = f.C;
+  const bool refl = nb >= 2;
+  // the fp32 form: |P| < 2^22 and |I| (2 + sqrt(nb)) < 2^24 for every row
+  bool fast = refl && f.small_p;
+  if (fast) {
+    const double lim = 16777216.0 / (2.0 + sqrt((double)nb));
+    const double mmax = floor(lim / ((double)Cn * (double)(1 << (f.bw - 1)))) -
+                        (double)(1 << (f.b2 - 1)) - 1.0;
+    for (int r = lane; r < nb; r += 32) {
+      const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
+      if (!((double)fabsf(m) <= mmax)) fast = false;
+    }
+    fast = __all_sync(0xffffffffu, fast);
+  }
+  auto prow = [&](int r) -> float * {
+    int64_t pr = f.perm[k0 + r];
+    if (pr < 0 || pr >= f.N) pr = 0;
+    return f.out + pr * f.D + j;
+  };
+  if (fast) {
+    const HhConst hc = hh_const(nb);
+    uint32_t sb[4] = {0u, 0u, 0u, 0u};
+    int msum = 0, Ip[4] = {0, 0, 0, 0};
+    for (int r = 0; r < nb; ++r) {
+      const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
+      msum += (int)m;
+      if (!jv) continue;
+      const float4 P = *reinterpret_cast<const float4 *>(prow(r));
+      const float pv[4] = {P.x, P.y, P.z, P.w};
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        sb[c] += magic_bits(pv[c]);
+        if (r == 0) Ip[c] = magic_int(pv[c]) + (int)m * cwi[c];
+      }
+    }
+    BlockFixF bf[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int S = (int)(sb[c] - (uint32_t)nb * kMagicBits) + cwi[c] * msum;
+      bf[c] = block_fix_f(hc, S, Ip[c]);
+    }
+    for (int r = 0; r < nb; ++r) {
+      const RowTerms t = row_terms(f, k0 + r, inv_sw, true);
+      const float A = __fmul_rn(t.sc, t.hd);
+      const float B = __fmul_rn(t.sc, __fmaf_rn(t.hR, y.h, __fmul_rn(t.hR, y.l)));
+      const float4 kq = make_float4(t.sc, A, B, t.m);
+      if (!jv) continue;
+      float *po = prow(r);
+      const float4 P = *reinterpret_cast<const float4 *>(po);
+      const float pv[4] = {P.x, P.y, P.z, P.w};
+      float o4[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        o4[c] = r == 0 ? dequant(kq, bf[c].lead, U[c])
+                       : dequant(kq, reflect_f(pv[c], kq, cwc[c], bf[c]), U[c]);
+      __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+    }
+  } else {
+    // int64 integer parts I = P + m CWc, float-float reflection
+    long long S[4] = {0, 0, 0, 0}, Ipl[4] = {0, 0, 0, 0};
+    for (int r = 0; r < nb && jv; ++r) {
+      const long long m = __float2ll_rn(rintf(two_sum((float)f.og, f.zero[k0 + r]).h));
+      const float4 P = *reinterpret_cast<const float4 *>(prow(r));
+      const float pv[4] = {P.x, P.y, P.z, P.w};
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const long long I = (long long)__float2int_rn(pv[c]) + m * cwi[c];
+        S[c] += I;
+        if (r == 0) Ipl[c] = I;
+      }
+    }
+    ff rS[4], beta[4];
+    if (refl) {
+      const HhConst hc = hh_const(nb);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        rS[c] = ff_mul(hc.rho, ff_from_int(S[c]));
+        beta[c] = ff_mul(hc.kap, ff_add(rS[c], ff_neg(ff_from_int(Ipl[c]))));
+      }
+    }
+    for (int r = 0; r < nb && jv; ++r) {
+      const RowTerms t = row_terms(f, k0 + r, inv_sw, refl);
+      float *po = prow(r);
+      const float4 P = *reinterpret_cast<const float4 *>(po);
+      const float pv[4] = {P.x, P.y, P.z, P.w};
+      const long long m = __float2ll_rn(t.m);
+      float o4[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const ff I = ff_from_int((long long)__float2int_rn(pv[c]) + m * cwi[c]);
+        ff v = !refl ? I : (r == 0 ? rS[c] : ff_add(I, ff_neg(beta[c])));
+        v = ff_add(v, two_prod(t.hd, U[c]));
+        v = ff_add(v, ff_mul({t.hR, 0.0f}, y));
+        o4[c] = __fmul_rn(t.sc, ff_round(v));
+      }
+      __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+    }
+  }
+}
+
+// Groups of 2 .. 32 rows in the fp32 form: lane r loads the per-row terms
+// of row r once; the rows' products are read 8 at a time (independent
+// loads) and, for groups of up to 8 rows, kept in registers for the
+// second pass.
+constexpr int kFixBatch = 8;
+
+__device__ __forceinline__ float4 ld_row4(const FixArgs &f, int pr, int64_t j, bool jv) {
+  return jv ? *reinterpret_cast<const float4 *>(f.out + (int64_t)pr * f.D + j)
+            : make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+__global__ void __launch_bounds__(256, 3) k_grp_fix(const FixArgs f) {
   const int lane = threadIdx.x & 31;
   const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int nchunk = (int)((f.D + 127) / 128);
@@ -2066,101 +2185,86 @@ __global__ void __launch_bounds__(256) k_grp_fix(const FixArgs f) {
       cwi[c] = (int)cwc[c];
       U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
     }
-    const bool refl = nb >= 2;
-    // the fp32 form: |P| < 2^22 and |I| (2 + sqrt(nb)) < 2^24 for every row
-    bool fast = refl && f.small_p;
+    // ---- per-row terms, lane r for row r ----
+    bool fast = nb >= 2 && nb <= 32 && f.small_p;
+    float4 kq = make_float4(0.f, 0.f, 0.f, 0.f);
+    int pr = 0;
     if (fast) {
-      const double lim = 16777216.0 / (2.0 + sqrt((double)nb));
-      const double mmax = floor(lim / ((double)Cn * (double)(1 << (f.bw - 1)))) -
-                          (double)(1 << (f.b2 - 1)) - 1.0;
-      for (int r = lane; r < nb; r += 32) {
-        const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
-        if (!((double)fabsf(m) <= mmax)) fast = false;
+      const float mmax = f.mmax_nb[nb];
+      bool ok = true;
+      if (lane < nb) {
+        const RowTerms t = row_terms(f, k0 + lane, inv_sw, true);
+        kq = make_float4(t.sc, __fmul_rn(t.sc, t.hd),
+                         __fmul_rn(t.sc, __fmaf_rn(t.hR, y.h, __fmul_rn(t.hR, y.l))), t.m);
+        ok = fabsf(t.m) <= mmax;
+        const int p = f.perm[k0 + lane];
+        pr = p < 0 || p >= f.N ? 0 : p;
       }
-      fast = __all_sync(0xffffffffu, fast);
+      fast = __all_sync(0xffffffffu, ok);
     }
-    auto prow = [&](int r) -> float * {
-      int64_t pr = f.perm[k0 + r];
-      if (pr < 0 || pr >= f.N) pr = 0;
-      return f.out + pr * f.D + j;
-    };
-    if (fast) {
-      const HhConst hc = hh_const(nb);
-      uint32_t sb[4] = {0u, 0u, 0u, 0u};
-      int msum = 0, Ip[4] = {0, 0, 0, 0};
-      for (int r = 0; r < nb; ++r) {
-        const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
-        msum += (int)m;
-        if (!jv) continue;
-        const float4 P = *reinterpret_cast<const float4 *>(prow(r));
-        const float pv[4] = {P.x, P.y, P.z, P.w};
+    if (!fast) {
+      fix_group_general(f, k0, nb, j, jv, cwc, cwi, U, inv_sw, y);
+      continue;
+    }
+    int msum = (int)kq.w;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          sb[c] += magic_bits(pv[c]);
-          if (r == 0) Ip[c] = magic_int(pv[c]) + (int)m * cwi[c];
+    for (int off = 16; off > 0; off >>= 1) msum += __shfl_xor_sync(0xffffffffu, msum, off);
+    const HhConst hc = hh_const(nb);
+    // ---- pass 1: block sums S = sum P + CWc sum m, lead I_p ----
+    uint32_t sb[4] = {0u, 0u, 0u, 0u};
+    float4 Pb[kFixBatch];
+    float4 P0 = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r0 = 0; r0 < nb; r0 += kFixBatch) {
+#pragma unroll
+      for (int b = 0; b < kFixBatch; ++b) {
+        const int prb = __shfl_sync(0xffffffffu, pr, (r0 + b) & 31);
+        Pb[b] = r0 + b < nb ? ld_row4(f, prb, j, jv) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int b = 0; b < kFixBatch; ++b) {
+        if (r0 + b >= nb) break;
+        sb[0] += magic_bits(Pb[b].x);
+        sb[1] += magic_bits(Pb[b].y);
+        sb[2] += magic_bits(Pb[b].z);
+        sb[3] += magic_bits(Pb[b].w);
+      }
+      if (r0 == 0) P0 = Pb[0];
+    }
+    const float mp = __shfl_sync(0xffffffffu, kq.w, 0);
+    const float p0[4] = {P0.x, P0.y, P0.z, P0.w};
+    BlockFixF bf[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int S = (int)(sb[c] - (uint32_t)nb * kMagicBits) + cwi[c] * msum;
+      bf[c] = block_fix_f(hc, S, magic_int(p0[c]) + (int)mp * cwi[c]);
+    }
+    // ---- pass 2: offsets and the inverse reflection ----
+    for (int r0 = 0; r0 < nb; r0 += kFixBatch) {
+      if (nb > kFixBatch) {
+#pragma unroll
+        for (int b = 0; b < kFixBatch; ++b) {
+          const int prb = __shfl_sync(0xffffffffu, pr, (r0 + b) & 31);
+          Pb[b] = r0 + b < nb ? ld_row4(f, prb, j, jv) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
       }
-      BlockFixF bf[4];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int S = (int)(sb[c] - (uint32_t)nb * kMagicBits) + cwi[c] * msum;
-        bf[c] = block_fix_f(hc, S, Ip[c]);
-      }
-      for (int r = 0; r < nb; ++r) {
-        const RowTerms t = row_terms(f, k0 + r, inv_sw, true);
-        const float A = __fmul_rn(t.sc, t.hd);
-        const float B = __fmul_rn(t.sc, __fmaf_rn(t.hR, y.h, __fmul_rn(t.hR, y.l)));
-        const float4 kq = make_float4(t.sc, A, B, t.m);
-        if (!jv) continue;
-        float *po = prow(r);
-        const float4 P = *reinterpret_cast<const float4 *>(po);
-        const float pv[4] = {P.x, P.y, P.z, P.w};
+      for (int b = 0; b < kFixBatch; ++b) {
+        const int r = r0 + b;
+        const int src = r & 31;
+        const float4 q = make_float4(__shfl_sync(0xffffffffu, kq.x, src),
+                                     __shfl_sync(0xffffffffu, kq.y, src),
+                                     __shfl_sync(0xffffffffu, kq.z, src),
+                                     __shfl_sync(0xffffffffu, kq.w, src));
+        const int prb = __shfl_sync(0xffffffffu, pr, src);
+        if (r >= nb || !jv) continue;
+        const float pv[4] = {Pb[b].x, Pb[b].y, Pb[b].z, Pb[b].w};
         float o4[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c)
-          o4[c] = r == 0 ? dequant(kq, bf[c].lead, U[c])
-                         : dequant(kq, reflect_f(pv[c], kq, cwc[c], bf[c]), U[c]);
-        __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
-      }
-    } else {
-      // int64 integer parts I = P + m CWc, float-float reflection
-      long long S[4] = {0, 0, 0, 0}, Ipl[4] = {0, 0, 0, 0};
-      for (int r = 0; r < nb && jv; ++r) {
-        const long long m = __float2ll_rn(rintf(two_sum((float)f.og, f.zero[k0 + r]).h));
-        const float4 P = *reinterpret_cast<const float4 *>(prow(r));
-        const float pv[4] = {P.x, P.y, P.z, P.w};
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const long long I = (long long)__float2int_rn(pv[c]) + m * cwi[c];
-          S[c] += I;
-          if (r == 0) Ipl[c] = I;
-        }
-      }
-      ff rS[4], beta[4];
-      if (refl) {
-        const HhConst hc = hh_const(nb);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          rS[c] = ff_mul(hc.rho, ff_from_int(S[c]));
-          beta[c] = ff_mul(hc.kap, ff_add(rS[c], ff_neg(ff_from_int(Ipl[c]))));
-        }
-      }
-      for (int r = 0; r < nb && jv; ++r) {
-        const RowTerms t = row_terms(f, k0 + r, inv_sw, refl);
-        float *po = prow(r);
-        const float4 P = *reinterpret_cast<const float4 *>(po);
-        const float pv[4] = {P.x, P.y, P.z, P.w};
-        const long long m = __float2ll_rn(t.m);
-        float o4[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const ff I = ff_from_int((long long)__float2int_rn(pv[c]) + m * cwi[c]);
-          ff v = !refl ? I : (r == 0 ? rS[c] : ff_add(I, ff_neg(beta[c])));
-          v = ff_add(v, two_prod(t.hd, U[c]));
-          v = ff_add(v, ff_mul({t.hR, 0.0f}, y));
-          o4[c] = __fmul_rn(t.sc, ff_round(v));
-        }
-        __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+          o4[c] = r == 0 ? dequant(q, bf[c].lead, U[c])
+                         : dequant(q, reflect_f(pv[c], q, cwc[c], bf[c]), U[c]);
+        __stcs(reinterpret_cast<float4 *>(f.out + (int64_t)prb * f.D + j),
+               make_float4(o4[0], o4[1], o4[2], o4[3]));
       }
     }
   }
@@ -2255,6 +2359,11 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
         f.col_sum_w = qw->col_sum;
         f.raw_mmax = (float)mmax;
         f.small_p = pmax < ((int64_t)1 << 22);
+        for (int n = 2; n <= 32; ++n) {
+          const double l = 16777216.0 / (2.0 + sqrt((double)n));
+          f.mmax_nb[n] = (float)(floor(l / ((double)C * (double)(1 << (qw->bits - 1)))) -
+                                 (double)(1 << (q_b2->bits - 1)) - 1.0);
+        }
         char *lw = static_cast<char *>(ws) + kGemmOffset;
         f.count = reinterpret_cast<int *>(lw);
         f.list = reinterpret_cast<int32_t *>(lw + 256);

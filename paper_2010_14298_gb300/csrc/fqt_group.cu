@@ -45,11 +45,8 @@ namespace fqt {
 namespace {
 
 constexpr int kSortThreads = 256;
-constexpr int kSortItems = 16;
-constexpr int kSortTile = kSortThreads * kSortItems;  // keys per sort tile
-constexpr int kSortTileLog = 12;
-constexpr int kCntPitch = kSortThreads + 2;  // uint16 counters per digit row
-constexpr size_t kCntBytes = sizeof(uint16_t) * 256 * kCntPitch;
+// keys per sort tile: 1024 (4 per thread) up to 2^17 rows, else 4096
+__host__ __device__ constexpr int sort_ipt(int64_t N) { return N <= ((int64_t)1 << 17) ? 4 : 16; }
 constexpr int kScanTile = 1024;  // sorted rows per CTA of the choice kernels
 constexpr int kKeysThreads = 1024;
 // the sort's tile offsets are summed per CTA over all tiles: 256 tiles at most
@@ -83,9 +80,10 @@ __device__ __forceinline__ int cta_excl_scan256(int v, int *wsum) {
 // ---------------------------------------------------------------------------
 template <typename T>
 __global__ void __launch_bounds__(kKeysThreads) k_grp_keys(const T *__restrict__ h, int64_t N,
-                                                            int C, int lpr, uint32_t *keys,
-                                                            int32_t *vals, int32_t *hist,
-                                                            int nt, unsigned *count) {
+                                                            int C, int lpr, int tile,
+                                                            uint32_t *keys, int32_t *vals,
+                                                            int32_t *hist, int nt,
+                                                            unsigned *count) {
   __shared__ int cnt[256];
   const int tid = threadIdx.x;
   for (int i = tid; i < 256; i += blockDim.x) cnt[i] = 0;
@@ -99,11 +97,11 @@ __global__ void __launch_bounds__(kKeysThreads) k_grp_keys(const T *__restrict__
   const int lane = tid & 31, warp = tid >> 5;
   const int rpw = 32 / lpr, sub = lane / lpr, o = lane - sub * lpr;
   const int octs = C / 8;
-  const int64_t r0 = (int64_t)blockIdx.x * kSortTile;
-  for (int rr = warp * rpw + sub; rr - sub < kSortTile; rr += (kKeysThreads / 32) * rpw) {
+  const int64_t r0 = (int64_t)blockIdx.x * tile;
+  for (int rr = warp * rpw + sub; rr - sub < tile; rr += (kKeysThreads / 32) * rpw) {
     const int64_t row = r0 + rr;
     float m = 0.0f;
-    if (rr < kSortTile && row < N) {
+    if (rr < tile && row < N) {
       for (int c8 = o; c8 < octs; c8 += lpr) {
         float x[8];
         load_oct(h + row * C + c8 * 8, x);
@@ -112,7 +110,7 @@ __global__ void __launch_bounds__(kKeysThreads) k_grp_keys(const T *__restrict__
       }
     }
     m = warp_max_xor(m, lpr);
-    if (o == 0 && rr < kSortTile && row < N) {
+    if (o == 0 && rr < tile && row < N) {
       const uint32_t key = ~__float_as_uint(m);
       keys[row] = key;
       vals[row] = (int32_t)row;
@@ -124,196 +122,250 @@ __global__ void __launch_bounds__(kKeysThreads) k_grp_keys(const T *__restrict__
 }
 
 // ---------------------------------------------------------------------------
-// One stable pass over digit (key >> shift) & 255.  Thread t holds keys
-// t*16 .. t*16+15 of its tile (tile order = thread-major), counts its digits
-// into column t of a 256 x 256 counter table, and a digit-major scan of the
-// table gives every key its rank in the tile.  The tile's global offsets
-// come from the histograms of all tiles (digit start + earlier tiles).  The
-// next pass's histogram is accumulated from the output positions.
+// One stable pass over digit (key >> shift) & 255 of a tile of 256 * IPT
+// keys.  Thread t holds the keys at tile positions i * 256 + t (i < IPT), so
+// the tile order is (i, warp, lane).  Per round i every warp ranks its 32
+// keys among equal digits with match.any and counts them per digit; a
+// digit-major scan of the (round, warp) counts gives each key its place in
+// the tile.  The tile's global offsets come from the histograms of all
+// tiles (digit start + earlier tiles).  The next pass's histogram is
+// accumulated from the output positions.
 // ---------------------------------------------------------------------------
+template <int IPT>
 __global__ void __launch_bounds__(kSortThreads) k_grp_radix(
     const uint32_t *__restrict__ kin, const int32_t *__restrict__ vin, uint32_t *kout,
     int32_t *vout, int64_t N, int nt, int shift, const int32_t *__restrict__ hcur,
     int32_t *hnext) {
-  extern __shared__ uint16_t cnt[];
-  __shared__ int wsum[kSortThreads / 32];
+  constexpr int T = kSortThreads * IPT;
+  constexpr int W = kSortThreads / 32;
+  extern __shared__ uint16_t cnt_s[];  // [IPT][W][256] counts, then offsets
+  auto cnt = [&](int i, int w, int d) -> uint16_t & { return cnt_s[(i * W + w) * 256 + d]; };
+  __shared__ int wsum[W];
   __shared__ int gbase[256];
-  const int tid = threadIdx.x;
-  const int64_t i0 = (int64_t)blockIdx.x * kSortTile + (int64_t)tid * kSortItems;
-  uint32_t k[kSortItems];
-  int32_t v[kSortItems];
-  if (i0 + kSortItems <= N) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t t0 = (int64_t)blockIdx.x * T;
+  for (int e = tid; e < IPT * W * 256; e += kSortThreads) cnt_s[e] = 0;
+  uint32_t k[IPT];
+  int32_t v[IPT];
+  int rk[IPT];
 #pragma unroll
-    for (int q = 0; q < kSortItems / 4; ++q) {
-      const uint4 a = __ldg(reinterpret_cast<const uint4 *>(kin + i0) + q);
-      const int4 b = __ldg(reinterpret_cast<const int4 *>(vin + i0) + q);
-      k[4 * q] = a.x; k[4 * q + 1] = a.y; k[4 * q + 2] = a.z; k[4 * q + 3] = a.w;
-      v[4 * q] = b.x; v[4 * q + 1] = b.y; v[4 * q + 2] = b.z; v[4 * q + 3] = b.w;
+  for (int i = 0; i < IPT; ++i) {
+    const int64_t idx = t0 + i * kSortThreads + tid;
+    k[i] = idx < N ? __ldg(kin + idx) : 0u;
+    v[i] = idx < N ? __ldg(vin + idx) : 0;
+  }
+  __syncthreads();
+  const unsigned lt = (1u << lane) - 1u;
+#pragma unroll
+  for (int i = 0; i < IPT; ++i) {
+    const bool ok = t0 + i * kSortThreads + tid < N;
+    const uint32_t d = ok ? (k[i] >> shift) & 255u : 256u + lane;
+    const unsigned peers = __match_any_sync(0xffffffffu, d);
+    rk[i] = __popc(peers & lt);
+    if (ok && (peers & lt) == 0u) cnt(i, warp, d) = (uint16_t)__popc(peers);
+  }
+  __syncthreads();
+  // thread d: running offsets of digit d over (round, warp), its total
+  int run = 0;
+#pragma unroll
+  for (int i = 0; i < IPT; ++i)
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      const int c = cnt(i, w, tid);
+      cnt(i, w, tid) = (uint16_t)run;
+      run += c;
     }
-  } else {
+  // digit d over all tiles and over the earlier ones: 16 loads in flight
+  int pre = 0, all = 0;
+  int b = 0;
+  for (; b + 16 <= nt; b += 16) {
+    int hv[16];
 #pragma unroll
-    for (int i = 0; i < kSortItems; ++i) {
-      k[i] = i0 + i < N ? kin[i0 + i] : 0u;
-      v[i] = i0 + i < N ? vin[i0 + i] : 0;
+    for (int q = 0; q < 16; ++q) hv[q] = __ldg(hcur + (int64_t)(b + q) * 256 + tid);
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      all += hv[q];
+      if (b + q < (int)blockIdx.x) pre += hv[q];
     }
   }
-  for (int d = 0; d < 256; ++d) cnt[d * kCntPitch + tid] = 0;
-#pragma unroll
-  for (int i = 0; i < kSortItems; ++i)
-    if (i0 + i < N) ++cnt[((k[i] >> shift) & 255u) * kCntPitch + tid];
-  __syncthreads();
-  // thread d: the row of digit d
-  int tot = 0;
-  for (int t = 0; t < kSortThreads; ++t) tot += cnt[tid * kCntPitch + t];
-  const int dstart = cta_excl_scan256(tot, wsum);
-  int pre = 0, all = 0;
-  for (int b = 0; b < nt; ++b) {
+  for (; b < nt; ++b) {
     const int hv = __ldg(hcur + (int64_t)b * 256 + tid);
     all += hv;
     if (b < (int)blockIdx.x) pre += hv;
   }
   const int dglob = cta_excl_scan256(all, wsum);
-  int run = dstart;
-  for (int t = 0; t < kSortThreads; ++t) {
-    const int c = cnt[tid * kCntPitch + t];
-    cnt[tid * kCntPitch + t] = (uint16_t)run;
-    run += c;
-  }
-  gbase[tid] = dglob + pre - dstart;
+  gbase[tid] = dglob + pre;
   __syncthreads();
 #pragma unroll
-  for (int i = 0; i < kSortItems; ++i) {
-    if (i0 + i >= N) continue;
+  for (int i = 0; i < IPT; ++i) {
+    const bool ok = t0 + i * kSortThreads + tid < N;
     const uint32_t d = (k[i] >> shift) & 255u;
-    const int r = cnt[d * kCntPitch + tid];
-    cnt[d * kCntPitch + tid] = (uint16_t)(r + 1);
-    const int64_t pos = (int64_t)gbase[d] + r;
-    if (pos < 0 || pos >= N) continue;  // unreachable with consistent histograms
-    kout[pos] = k[i];
-    vout[pos] = v[i];
-    if (hnext) atomicAdd(&hnext[(pos >> kSortTileLog) * 256 + ((k[i] >> (shift + 8)) & 255u)], 1);
+    int64_t pos = ok ? (int64_t)gbase[d] + cnt(i, warp, d) + rk[i] : -1;
+    if (pos >= N) pos = -1;  // unreachable with consistent histograms
+    if (pos >= 0) {
+      kout[pos] = k[i];
+      vout[pos] = v[i];
+    }
+    if (hnext) {
+      const uint32_t key2 = pos >= 0 ? (uint32_t)((pos / T) * 256 + ((k[i] >> (shift + 8)) & 255u))
+                                     : 0xFFFFFFFFu - lane;
+      const unsigned peers = __match_any_sync(0xffffffffu, key2);
+      if (pos >= 0 && (peers & lt) == 0u) atomicAdd(&hnext[key2], __popc(peers));
+    }
   }
 }
 
-__device__ __forceinline__ double key_m(uint32_t key) {
-  return (double)__uint_as_float(~key);
+__device__ __forceinline__ float key_m(uint32_t key) { return __uint_as_float(~key); }
+
+// ---------------------------------------------------------------------------
+// The estimate V(G) is evaluated in float-float (about 2^-46 relative, on the
+// fp32 pipe; fp64 is a narrow pipe on this part).  Candidate estimates differ
+// by far more than that on real data; the decision is as precise as a
+// double-precision evaluation with the same summation order would be.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ ff ff_sub(ff a, ff b) { return ff_add(a, ff_neg(b)); }
+
+// 1 / x for x > 0: fp32 reciprocal and one correction in float-float.
+__device__ __forceinline__ ff ff_rcp(ff x) {
+  const float y0 = __frcp_rn(x.h);
+  const ff p = ff_mul(x, {y0, 0.0f});
+  const float e = __fsub_rn(__fsub_rn(1.0f, p.h), p.l);
+  return fast_two_sum(y0, __fmul_rn(y0, e));
 }
 
-// Sums of M^p (p = 1, 4/3, 5/3, 2) over one thread's 4 sorted rows.
-__device__ __forceinline__ void pow_terms(double M, double (&a)[4]) {
-  const double c = cbrt(M);
-  a[0] = M;
-  a[1] = M * c;
-  a[2] = M * c * c;
-  a[3] = M * M;
+// x^(1/3) for x >= 0: fp32 cube root and one Newton correction.
+__device__ __forceinline__ ff ff_cbrt(ff x) {
+  if (!(x.h > 0.0f)) return {0.0f, 0.0f};
+  const float c0 = cbrtf(x.h);
+  const ff c3 = ff_mul(two_prod(c0, c0), {c0, 0.0f});
+  const ff r = ff_sub(x, c3);
+  return fast_two_sum(c0, __fdiv_rn(r.h, __fmul_rn(3.0f, __fmul_rn(c0, c0))));
+}
+
+// M, M^(4/3), M^(5/3), M^2 of one row.
+__device__ __forceinline__ void pow_terms(float M, ff (&a)[4]) {
+  const ff c = ff_cbrt({M, 0.0f});
+  a[0] = {M, 0.0f};
+  a[1] = ff_mul({M, 0.0f}, c);
+  a[2] = ff_mul(a[1], c);
+  a[3] = two_prod(M, M);
+}
+
+__device__ __forceinline__ ff shfl_xor_ff(ff v, int off) {
+  return {__shfl_xor_sync(0xffffffffu, v.h, off), __shfl_xor_sync(0xffffffffu, v.l, off)};
 }
 
 // Sum over a 256-thread CTA in a fixed order (deterministic).
-__device__ __forceinline__ double cta_sum256(double v, double *red) {
+__device__ __forceinline__ ff cta_sum256(ff v, ff *red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  for (int off = 16; off > 0; off >>= 1) v = ff_add(v, shfl_xor_ff(v, off));
   if (lane == 0) red[warp] = v;
   __syncthreads();
-  double s = 0.0;
-  for (int w = 0; w < 8; ++w) s += red[w];
+  ff s = {0.0f, 0.0f};
+  for (int w = 0; w < 8; ++w) s = ff_add(s, red[w]);
   __syncthreads();
   return s;
 }
 
 __global__ void __launch_bounds__(256) k_grp_tsum(const uint32_t *__restrict__ keys, int64_t N,
-                                                  double *tsum) {
-  __shared__ double red[8];
+                                                  ff *tsum) {
+  __shared__ ff red[8];
   const int64_t i0 = (int64_t)blockIdx.x * kScanTile + threadIdx.x * 4;
-  double s[4] = {0.0, 0.0, 0.0, 0.0};
+  ff s[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
   for (int e = 0; e < 4; ++e) {
     if (i0 + e >= N) break;
-    double a[4];
+    ff a[4];
     pow_terms(key_m(keys[i0 + e]), a);
-    for (int q = 0; q < 4; ++q) s[q] += a[q];
+    for (int q = 0; q < 4; ++q) s[q] = ff_add(s[q], a[q]);
   }
   for (int q = 0; q < 4; ++q) {
-    const double t = cta_sum256(s[q], red);
+    const ff t = cta_sum256(s[q], red);
     if (threadIdx.x == 0) tsum[(int64_t)blockIdx.x * 4 + q] = t;
   }
 }
 
-// Exclusive prefix over a 256-thread CTA of one double per thread.
-__device__ __forceinline__ double cta_excl_scan256d(double v, double *red) {
+// Exclusive prefix over a 256-thread CTA of one float-float per thread.
+__device__ __forceinline__ ff cta_excl_scan256ff(ff v, ff *red) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  double x = v;
+  ff x = v;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
-    const double y = __shfl_up_sync(0xffffffffu, x, off);
-    if (lane >= off) x += y;
+    const ff y = {__shfl_up_sync(0xffffffffu, x.h, off), __shfl_up_sync(0xffffffffu, x.l, off)};
+    if (lane >= off) x = ff_add(x, y);
   }
   if (lane == 31) red[warp] = x;
   __syncthreads();
-  double base = 0.0;
-  for (int w = 0; w < warp; ++w) base += red[w];
+  ff base = {0.0f, 0.0f};
+  for (int w = 0; w < warp; ++w) base = ff_add(base, red[w]);
   __syncthreads();
-  return base + (x - v);
+  return ff_add(base, ff_sub(x, v));
 }
 
-struct Best {
-  double v;
+__device__ __forceinline__ bool better(ff v, long long g, ff bv, long long bg) {
+  return v.h < bv.h || (v.h == bv.h && (v.l < bv.l || (v.l == bv.l && g < bg)));
+}
+
+struct BestFF {
+  float h, l;
   long long g;
 };
 
-__device__ __forceinline__ bool better(double v, long long g, double bv, long long bg) {
-  return v < bv || (v == bv && g < bg);
-}
-
 __global__ void __launch_bounds__(256) k_grp_choose(const uint32_t *__restrict__ keys, int64_t N,
-                                                    const double *__restrict__ tsum, double *cincl,
-                                                    double2 *best, long long *Gout, double *SGout,
+                                                    const ff *__restrict__ tsum, ff *cincl,
+                                                    BestFF *best, long long *Gout, ff *SGout,
                                                     unsigned *count) {
-  __shared__ double red[8];
-  __shared__ double bv_s[8];
+  __shared__ ff red[8];
+  __shared__ ff bv_s[8];
   __shared__ long long bg_s[8];
   __shared__ int last;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = blockIdx.x;
   // sums over the earlier tiles
-  double base[4];
+  ff base[4];
   for (int q = 0; q < 4; ++q) {
-    double p = 0.0;
-    for (int bb = tid; bb < b; bb += 256) p += tsum[(int64_t)bb * 4 + q];
+    ff p = {0.0f, 0.0f};
+    for (int bb = tid; bb < b; bb += 256) p = ff_add(p, tsum[(int64_t)bb * 4 + q]);
     base[q] = cta_sum256(p, red);
   }
   const int64_t i0 = (int64_t)b * kScanTile + tid * 4;
-  double loc[4][4];
-  double tot[4] = {0.0, 0.0, 0.0, 0.0};
-  double Mv[5];
-  for (int e = 0; e < 5; ++e) Mv[e] = i0 + e < N ? key_m(keys[i0 + e]) : 0.0;
+  ff loc[4][4];
+  ff tot[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+  float Mv[5];
+  for (int e = 0; e < 5; ++e) Mv[e] = i0 + e < N ? key_m(keys[i0 + e]) : 0.0f;
   for (int e = 0; e < 4; ++e) {
-    double a[4] = {0.0, 0.0, 0.0, 0.0};
+    ff a[4] = {{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
     if (i0 + e < N) pow_terms(Mv[e], a);
     for (int q = 0; q < 4; ++q) {
-      tot[q] += a[q];
+      tot[q] = ff_add(tot[q], a[q]);
       loc[e][q] = tot[q];
     }
   }
-  double off[4];
-  for (int q = 0; q < 4; ++q) off[q] = cta_excl_scan256d(tot[q], red);
-  double bv = INFINITY;
+  ff off[4];
+  for (int q = 0; q < 4; ++q) off[q] = ff_add(base[q], cta_excl_scan256ff(tot[q], red));
+  ff bv = {INFINITY, 0.0f};
   long long bg = 0x7fffffffffffffffll;
   for (int e = 0; e < 4; ++e) {
     const int64_t i = i0 + e;
     if (i >= N) break;
-    double S[4];
-    for (int q = 0; q < 4; ++q) S[q] = base[q] + off[q] + loc[e][q];
+    ff S[4];
+    for (int q = 0; q < 4; ++q) S[q] = ff_add(off[q], loc[e][q]);
     cincl[i] = S[0];
     if (i + 1 >= N) break;  // G = N is not a candidate
     const long long G = i + 1;
-    const double nG = (double)(N - G), L = Mv[e + 1];
-    double V = 0.0;
-    if (S[0] > 0.0) {
-      const double t3 = S[0] / nG;
-      const double t = cbrt(t3);
-      const double cl = cbrt(L), r = cbrt(nG / S[0]);
-      const double u = cl * cl * r * r;
-      V = t3 * S[0] + 3.0 * t * t * u * S[1] + 3.0 * t * u * u * S[2] + u * u * u * S[3];
+    const float nG = (float)(N - G);  // exact: N <= 2^20
+    ff V = {0.0f, 0.0f};
+    if (S[0].h > 0.0f) {
+      const ff t3 = ff_mul(S[0], ff_rcp({nG, 0.0f}));  // t^3 = S1 / (N - G)
+      const ff t = ff_cbrt(t3);
+      const ff cl = ff_cbrt({Mv[e + 1], 0.0f});
+      const ff r = ff_rcp(t);
+      const ff u = ff_mul(ff_mul(cl, cl), ff_mul(r, r));  // L^(2/3) ((N-G)/S1)^(2/3)
+      const ff tu = ff_mul(t, u);
+      V = ff_mul(t3, S[0]);
+      V = ff_add(V, ff_mul(ff_mul({3.0f, 0.0f}, ff_mul(t, tu)), S[1]));
+      V = ff_add(V, ff_mul(ff_mul({3.0f, 0.0f}, ff_mul(tu, u)), S[2]));
+      V = ff_add(V, ff_mul(ff_mul(ff_mul(u, u), u), S[3]));
     }
     if (better(V, G, bv, bg)) {
       bv = V;
@@ -323,7 +375,7 @@ __global__ void __launch_bounds__(256) k_grp_choose(const uint32_t *__restrict__
   __threadfence();  // cincl is read by the last CTA
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    const double ov = __shfl_xor_sync(0xffffffffu, bv, o);
+    const ff ov = shfl_xor_ff(bv, o);
     const long long og = __shfl_xor_sync(0xffffffffu, bg, o);
     if (better(ov, og, bv, bg)) {
       bv = ov;
@@ -341,34 +393,40 @@ __global__ void __launch_bounds__(256) k_grp_choose(const uint32_t *__restrict__
         bv = bv_s[w];
         bg = bg_s[w];
       }
-    best[b] = make_double2(bv, (double)bg);
+    best[b] = BestFF{bv.h, bv.l, bg};
     __threadfence();
     last = atomicAdd(count, 1u) == gridDim.x - 1;
   }
   __syncthreads();
   if (!last || tid != 0) return;
   __threadfence();
-  double fv = INFINITY;
+  ff fv = {INFINITY, 0.0f};
   long long fg = 0x7fffffffffffffffll;
   for (int bb = 0; bb < (int)gridDim.x; ++bb) {
-    const double2 x = __ldcg(best + bb);
-    if (better(x.x, (long long)x.y, fv, fg)) {
-      fv = x.x;
-      fg = (long long)x.y;
+    const volatile BestFF *x = best + bb;
+    const ff xv = {x->h, x->l};
+    const long long xg = x->g;
+    if (better(xv, xg, fv, fg)) {
+      fv = xv;
+      fg = xg;
     }
   }
   if (fg < 1 || fg >= N) fg = 1;  // N = 1: one group
   *Gout = fg;
-  *SGout = __ldcg(cincl + fg - 1);
+  const volatile ff *cg = cincl + fg - 1;
+  *SGout = ff{cg->h, cg->l};
   *count = 0u;
 }
 
+// e_j of the cumulative rounding, in fp64 (two divisions per group) so that
+// exact ties (equal rows) round as in a double-precision evaluation.
 __device__ __forceinline__ int64_t cum_size(int64_t j, int64_t N, int64_t G, double SG,
-                                            const double *cincl) {
+                                            const ff *cincl) {
   if (j <= 0) return 0;
   if (j >= G) return N - G;
   if (!(SG > 0.0)) return 0;
-  const double q = (double)(N - G) * (cincl[j - 1] / SG);
+  const ff c = cincl[j - 1];
+  const double q = (double)(N - G) * (((double)c.h + (double)c.l) / SG);
   int64_t e = (int64_t)floor(q + 0.5);
   if (e < 0) e = 0;
   if (e > N - G) e = N - G;
@@ -376,8 +434,8 @@ __device__ __forceinline__ int64_t cum_size(int64_t j, int64_t N, int64_t G, dou
 }
 
 __global__ void __launch_bounds__(256) k_grp_layout(const int32_t *__restrict__ vals, int64_t N,
-                                                    const double *__restrict__ cincl,
-                                                    const long long *Gp, const double *SGp,
+                                                    const ff *__restrict__ cincl,
+                                                    const long long *Gp, const ff *SGp,
                                                     int32_t *perm, int32_t *gstart,
                                                     int32_t *gsize) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -387,7 +445,7 @@ __global__ void __launch_bounds__(256) k_grp_layout(const int32_t *__restrict__ 
     gstart[i] = (int32_t)N;
     return;
   }
-  const double SG = *SGp;
+  const double SG = (double)SGp->h + (double)SGp->l;
   const int64_t e0 = cum_size(i, N, G, SG, cincl);
   int64_t e1 = cum_size(i + 1, N, G, SG, cincl);
   if (e1 < e0) e1 = e0;
@@ -507,10 +565,98 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
   for (int j = 0; j < 8; ++j) cs[j] = 0;
   bool badp = false;
 
+  // One row per sub-warp for a slot of RS single-row groups: BHQ of one row
+  // is lambda2 = 0, s1 = B / R(h), no reflection (App. D.4 with N = 1).
+  auto do_singles = [&](int64_t k0) {
+    const int64_t row = k0 + sub;
+    int64_t src = __ldg(a.perm + row);
+    if (src < 0 || src >= N) {
+      badp = true;
+      src = 0;
+    }
+    float x[8];
+    load_oct(h + src * C + o * 8, x);
+    float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      mm.x = fminf(mm.x, x[j]);
+      mm.y = fmaxf(mm.y, x[j]);
+    }
+    mm = row_minmax<LPR>(mm);
+    const float np = fmaxf(fabsf(mm.x), fabsf(mm.y));
+    float s1f = 0.0f;
+    if (np > 0.0f) {
+      float lam1 = __fsub_rn(mm.y, mm.x);
+      if (!(lam1 > 0.0f)) lam1 = 2.0f * np;
+      s1f = (float)B2 * sqrtf(1.0f) / lam1;
+    }
+    float t[8];
+    float tmin = INFINITY;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      t[j] = __fmul_rn(s1f, x[j]);
+      tmin = fminf(tmin, t[j]);
+    }
+    const float z2 = row_min<LPR>(tmin);
+    uint32_t c[8];
+    int rs2 = 0, rs1 = 0;
+    const uint4 w2 = philox_oct((uint64_t)row * (uint64_t)CO + (uint64_t)o, 0u, key);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      c[j] = sr_code16(__fmul_rn(__fsub_rn(t[j], z2), 65536.0f), u16_of(w2, j), B2);
+      rs2 += (int)c[j];
+    }
+    if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+    if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + o * 8, c, og2);
+    if (has_b1) {
+      const uint4 w1 = philox_oct((uint64_t)src * (uint64_t)CO + (uint64_t)o, 1u, key);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float vv = __fmul_rn(__fsub_rn(x[j], gmin), s_g1_16);
+        c[j] = sr_code16(vv, u16_of(w1, j), 255u);
+        rs1 += (int)c[j];
+        cs[j] += (int)c[j];
+      }
+      if (a.c1) store_codes8(a.c1 + src * (int64_t)C + o * 8, c);
+      if (a.f1) store_carriers8(a.f1 + src * (int64_t)C + o * 8, c, 128u);
+    }
+    rs2 = row_add<LPR>(rs2);
+    if (has_b1) rs1 = row_add<LPR>(rs1);
+    if (o == 0) {
+      if (a.rsum2) a.rsum2[row] = rs2;
+      if (has_b1 && a.rsum1) a.rsum1[src] = rs1;
+      a.inv2[row] = s1f > 0.0f ? __fdiv_rn(1.0f, s1f) : 0.0f;
+      a.zero2[row] = z2;
+      if (a.hz) {
+        const ff xo = two_sum((float)og2, z2);
+        const float m = rintf(xo.h);
+        const ff d = fast_two_sum(__fsub_rn(xo.h, m), xo.l);
+        a.hz[row] = ff_round(d);
+        // R = sum_c (a + m); C is a power of two, so C m is exact
+        a.hr[row] = ff_round(two_sum((float)(rs2 - C * (int)og2), __fmul_rn((float)C, m)));
+      }
+    }
+  };
+
+  // A warp takes slots of RS consecutive groups: all single rows -> one step;
+  // otherwise the groups one after another, a warp each.
   const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t gi = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; gi < N; gi += wstride) {
+  for (int64_t g0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + warp) * RS; g0 < N;
+       g0 += wstride * RS) {
+    const int64_t gk = g0 + (lane < RS ? lane : 0);
+    const int64_t ka = gk < N ? __ldg(a.gstart + gk) : N;
+    const int64_t kb = gk < N ? __ldg(a.gstart + gk + 1) : N;
+    const int64_t s0 = __shfl_sync(0xffffffffu, ka, 0);
+    if (s0 >= N) break;  // groups past G are empty and gstart does not decrease
+    if (__all_sync(0xffffffffu, lane >= RS || (ka < N && kb == ka + 1))) {
+      do_singles(s0);
+      continue;
+    }
+  for (int gs = 0; gs < RS; ++gs) {
+    const int64_t gi = g0 + gs;
+    if (gi >= N) break;
     const int64_t k0 = __ldg(a.gstart + gi);
-    if (k0 >= N) break;  // groups past G are empty and gstart does not decrease
+    if (k0 >= N) break;
     int64_t k1 = __ldg(a.gstart + gi + 1);
     if (k1 > N) k1 = N;
     if (k1 <= k0) continue;
@@ -594,10 +740,8 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
       w[j] = fmaf(es, __fmul_rn(s2f, csm[j]), el * __fmul_rn(s1f, xl[j]));
 
     // ---- pass 2: transform, row minimum, rounding, packing, sums ----
-    ff sd = {0.0f, 0.0f};
-    long long sR = 0;
+    ff sd = {0.0f, 0.0f}, sR = {0.0f, 0.0f}, Rp = {0.0f, 0.0f};
     float dp = 0.0f;
-    long long Rp = 0;
     for (int r0 = 0; r0 < nb; r0 += RS) {
       const int r = r0 + sub;
       const bool v = r < nb;
@@ -652,7 +796,8 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
       const ff xo = two_sum((float)og2, z2);
       const float m = rintf(xo.h);
       const ff d = fast_two_sum(__fsub_rn(xo.h, m), xo.l);
-      const long long R = (long long)rs2 - (long long)C * og2 + (long long)C * __float2ll_rn(m);
+      // R = sum_c (a + m); C is a power of two, so C m is exact
+      const ff R = two_sum((float)(rs2 - C * (int)og2), __fmul_rn((float)C, m));
       if (v && o == 0) {
         if (a.rsum2) a.rsum2[row] = rs2;
         if (has_b1 && a.rsum1) a.rsum1[src] = rs1;
@@ -660,10 +805,10 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
         a.zero2[row] = z2;
         if (a.hz) {
           a.hz[row] = ff_round(d);
-          a.hr[row] = (float)R;
+          a.hr[row] = ff_round(R);
         }
         sd = ff_add(sd, d);
-        sR += R;
+        sR = ff_add(sR, R);
         if (lead) {
           dp = ff_round(d);
           Rp = R;
@@ -676,20 +821,24 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
       for (int off = LPR; off < 32; off <<= 1) {
         const ff od = {__shfl_xor_sync(0xffffffffu, sd.h, off),
                        __shfl_xor_sync(0xffffffffu, sd.l, off)};
+        const ff oR = {__shfl_xor_sync(0xffffffffu, sR.h, off),
+                       __shfl_xor_sync(0xffffffffu, sR.l, off)};
         sd = ff_add(sd, od);
-        sR += __shfl_xor_sync(0xffffffffu, sR, off);
+        sR = ff_add(sR, oR);
       }
       sd.h = __shfl_sync(0xffffffffu, sd.h, 0);
       sd.l = __shfl_sync(0xffffffffu, sd.l, 0);
-      sR = __shfl_sync(0xffffffffu, sR, 0);
+      sR.h = __shfl_sync(0xffffffffu, sR.h, 0);
+      sR.l = __shfl_sync(0xffffffffu, sR.l, 0);
       dp = __shfl_sync(0xffffffffu, dp, 0);
-      Rp = __shfl_sync(0xffffffffu, Rp, 0);
+      Rp.h = __shfl_sync(0xffffffffu, Rp.h, 0);
+      Rp.l = __shfl_sync(0xffffffffu, Rp.l, 0);
       __syncwarp();  // every row's unreflected d, R is in hz, hr
       const HhConst hcst = hh_const(nb);
       const ff rsd = ff_mul(hcst.rho, sd);
-      const ff rsR = ff_mul(hcst.rho, ff_from_int(sR));
+      const ff rsR = ff_mul(hcst.rho, sR);
       const ff wd = ff_add(rsd, {-dp, 0.0f});
-      const ff wR = ff_add(rsR, ff_neg(ff_from_int(Rp)));
+      const ff wR = ff_add(rsR, ff_neg(Rp));
       const ff kd = ff_mul(hcst.kap, wd), kR = ff_mul(hcst.kap, wR);
       for (int r = lane; r < nb; r += 32) {
         const int64_t row = k0 + r;
@@ -704,6 +853,7 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
       }
       __syncwarp();
     }
+  }
   }
   if (__any_sync(0xffffffffu, badp) && lane == 0) record_status(a.status, FQT_EINVAL);
   // ---- column sums of Q_b1 ----
@@ -723,15 +873,16 @@ struct GroupScratch {
   uint32_t *k0, *k1;
   int32_t *v0, *v1;
   int32_t *hist;
-  double *tsum, *cincl;
-  double2 *best;
+  ff *tsum, *cincl;
+  BestFF *best;
   long long *G;
-  double *SG;
+  ff *SG;
   unsigned *count;
 };
 
 size_t carve(char *base, int64_t N, GroupScratch *s) {
-  const int64_t nt = (N + kSortTile - 1) / kSortTile;
+  const int tile = kSortThreads * sort_ipt(N);
+  const int64_t nt = (N + tile - 1) / tile;
   const int64_t ntc = (N + kScanTile - 1) / kScanTile;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -739,12 +890,12 @@ size_t carve(char *base, int64_t N, GroupScratch *s) {
     off += (bytes + 255) & ~(size_t)255;
     return p;
   };
-  const size_t nk = (size_t)(nt * kSortTile);
+  const size_t nk = (size_t)(nt * tile);
   char *k0 = take(nk * 4), *k1 = take(nk * 4), *v0 = take(nk * 4), *v1 = take(nk * 4);
   char *hist = take((size_t)4 * nt * 256 * 4);
-  char *tsum = take((size_t)ntc * 4 * 8);
-  char *cincl = take((size_t)N * 8 + 8);
-  char *best = take((size_t)ntc * 16);
+  char *tsum = take((size_t)ntc * 4 * sizeof(ff));
+  char *cincl = take((size_t)N * sizeof(ff) + 8);
+  char *best = take((size_t)ntc * sizeof(BestFF));
   char *G = take(8), *SG = take(8), *count = take(8);
   if (s) {
     s->k0 = reinterpret_cast<uint32_t *>(k0);
@@ -752,11 +903,11 @@ size_t carve(char *base, int64_t N, GroupScratch *s) {
     s->v0 = reinterpret_cast<int32_t *>(v0);
     s->v1 = reinterpret_cast<int32_t *>(v1);
     s->hist = reinterpret_cast<int32_t *>(hist);
-    s->tsum = reinterpret_cast<double *>(tsum);
-    s->cincl = reinterpret_cast<double *>(cincl);
-    s->best = reinterpret_cast<double2 *>(best);
+    s->tsum = reinterpret_cast<ff *>(tsum);
+    s->cincl = reinterpret_cast<ff *>(cincl);
+    s->best = reinterpret_cast<BestFF *>(best);
     s->G = reinterpret_cast<long long *>(G);
-    s->SG = reinterpret_cast<double *>(SG);
+    s->SG = reinterpret_cast<ff *>(SG);
     s->count = reinterpret_cast<unsigned *>(count);
   }
   return off;
@@ -774,27 +925,34 @@ fqt_status launch_bhq_grouping(const void *dH, bool bf16, int64_t N, int C, int3
   GroupScratch s;
   if (carve(nullptr, N, nullptr) > scratch_bytes) return FQT_EWORKSPACE;
   carve(static_cast<char *>(scratch), N, &s);
-  const int nt = (int)((N + kSortTile - 1) / kSortTile);
+  const int ipt = sort_ipt(N);
+  const int tile = kSortThreads * ipt;
+  const int nt = (int)((N + tile - 1) / tile);
   const int ntc = (int)((N + kScanTile - 1) / kScanTile);
   int lpr = 1;
   while (lpr < 32 && lpr < C / 8) lpr <<= 1;
   if (bf16)
     k_grp_keys<__nv_bfloat16><<<nt, kKeysThreads, 0, st>>>(
-        static_cast<const __nv_bfloat16 *>(dH), N, C, lpr, s.k0, s.v0, s.hist, nt, s.count);
+        static_cast<const __nv_bfloat16 *>(dH), N, C, lpr, tile, s.k0, s.v0, s.hist, nt,
+        s.count);
   else
     k_grp_keys<float><<<nt, kKeysThreads, 0, st>>>(static_cast<const float *>(dH), N, C, lpr,
-                                                    s.k0, s.v0, s.hist, nt, s.count);
+                                                    tile, s.k0, s.v0, s.hist, nt, s.count);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "grouping keys launch");
-  e = cudaFuncSetAttribute(k_grp_radix, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           (int)kCntBytes);
+  e = cudaFuncSetAttribute(k_grp_radix<16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)(sizeof(uint16_t) * 16 * (kSortThreads / 32) * 256));
   if (e != cudaSuccess) return cuda_fail(e, "radix smem attribute");
   uint32_t *kin = s.k0, *kout = s.k1;
   int32_t *vin = s.v0, *vout = s.v1;
   for (int p = 0; p < 4; ++p) {
     int32_t *hc = s.hist + (int64_t)p * nt * 256;
     int32_t *hn = p < 3 ? hc + (int64_t)nt * 256 : nullptr;
-    k_grp_radix<<<nt, kSortThreads, kCntBytes, st>>>(kin, vin, kout, vout, N, nt, 8 * p, hc, hn);
+    const size_t csm = sizeof(uint16_t) * ipt * (kSortThreads / 32) * 256;
+    if (ipt == 4)
+      k_grp_radix<4><<<nt, kSortThreads, csm, st>>>(kin, vin, kout, vout, N, nt, 8 * p, hc, hn);
+    else
+      k_grp_radix<16><<<nt, kSortThreads, csm, st>>>(kin, vin, kout, vout, N, nt, 8 * p, hc, hn);
     uint32_t *tk = kin;
     kin = kout;
     kout = tk;
