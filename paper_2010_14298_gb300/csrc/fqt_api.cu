@@ -223,10 +223,12 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   size_t smem;
   const bool bf16 = dtype == FQT_BF16;
   if (adapt) {
+    unsigned *slots = nullptr;
     s = launch_bhq_grouping(dH, bf16, N, (int)C, q_b2->perm, q_b2->gstart, q_b2->gsize,
-                            w + kGemmOffset, ws_bytes - kGemmOffset, st);
+                            w + kGemmOffset, ws_bytes - kGemmOffset, &slots, st);
     if (s != FQT_OK) return s;
     QuantArgs ag = a;
+    ag.slots = slots;
     ag.perm = q_b2->perm;
     ag.gstart = q_b2->gstart;
     if (want_off) {

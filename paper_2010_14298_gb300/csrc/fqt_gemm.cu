@@ -2157,14 +2157,13 @@ __global__ void __launch_bounds__(256, 3) k_grp_fix(const FixArgs f) {
   const int lane = threadIdx.x & 31;
   const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int nchunk = (int)((f.D + 127) / 128);
-  const int64_t nunits = (int64_t)*f.count * nchunk;
+  const int64_t nunits = (int64_t)*f.count;
   const float inv_sw = *f.inv_sw, zw = *f.zero_w;
   const ff y = two_sum((float)f.ow, zw);
   const int Cn = f.C;
   for (int64_t u = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); u < nunits;
        u += nw) {
-    const int64_t gi = f.list[u / nchunk];
-    const int ch = (int)(u % nchunk);
+    const int64_t gi = f.list[u];
     if (gi < 0 || gi >= f.N) {
       if (lane == 0) record_status(f.status, FQT_EINVAL);
       continue;
@@ -2174,18 +2173,7 @@ __global__ void __launch_bounds__(256, 3) k_grp_fix(const FixArgs f) {
     if (k1 > f.N) k1 = f.N;
     if (k0 < 0 || k1 <= k0) continue;
     const int nb = (int)(k1 - k0);
-    const int64_t j = (int64_t)ch * 128 + lane * 4;
-    const bool jv = j < f.D;
-    float cwc[4], U[4];
-    int cwi[4];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int cs = jv ? f.col_sum_w[j + c] : 0;
-      cwc[c] = (float)(cs - Cn * f.ow);
-      cwi[c] = (int)cwc[c];
-      U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
-    }
-    // ---- per-row terms, lane r for row r ----
+    // ---- per-row terms, lane r for row r (groups of up to 32 rows) ----
     bool fast = nb >= 2 && nb <= 32 && f.small_p;
     float4 kq = make_float4(0.f, 0.f, 0.f, 0.f);
     int pr = 0;
@@ -2202,69 +2190,82 @@ __global__ void __launch_bounds__(256, 3) k_grp_fix(const FixArgs f) {
       }
       fast = __all_sync(0xffffffffu, ok);
     }
-    if (!fast) {
-      fix_group_general(f, k0, nb, j, jv, cwc, cwi, U, inv_sw, y);
-      continue;
-    }
     int msum = (int)kq.w;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) msum += __shfl_xor_sync(0xffffffffu, msum, off);
-    const HhConst hc = hh_const(nb);
-    // ---- pass 1: block sums S = sum P + CWc sum m, lead I_p ----
-    uint32_t sb[4] = {0u, 0u, 0u, 0u};
-    float4 Pb[kFixBatch];
-    float4 P0 = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int r0 = 0; r0 < nb; r0 += kFixBatch) {
-#pragma unroll
-      for (int b = 0; b < kFixBatch; ++b) {
-        const int prb = __shfl_sync(0xffffffffu, pr, (r0 + b) & 31);
-        Pb[b] = r0 + b < nb ? ld_row4(f, prb, j, jv) : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-#pragma unroll
-      for (int b = 0; b < kFixBatch; ++b) {
-        if (r0 + b >= nb) break;
-        sb[0] += magic_bits(Pb[b].x);
-        sb[1] += magic_bits(Pb[b].y);
-        sb[2] += magic_bits(Pb[b].z);
-        sb[3] += magic_bits(Pb[b].w);
-      }
-      if (r0 == 0) P0 = Pb[0];
-    }
     const float mp = __shfl_sync(0xffffffffu, kq.w, 0);
-    const float p0[4] = {P0.x, P0.y, P0.z, P0.w};
-    BlockFixF bf[4];
+    const HhConst hc = hh_const(nb >= 2 ? nb : 2);
+    for (int ch = 0; ch < nchunk; ++ch) {
+      const int64_t j = (int64_t)ch * 128 + lane * 4;
+      const bool jv = j < f.D;
+      float cwc[4], U[4];
+      int cwi[4];
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int S = (int)(sb[c] - (uint32_t)nb * kMagicBits) + cwi[c] * msum;
-      bf[c] = block_fix_f(hc, S, magic_int(p0[c]) + (int)mp * cwi[c]);
-    }
-    // ---- pass 2: offsets and the inverse reflection ----
-    for (int r0 = 0; r0 < nb; r0 += kFixBatch) {
-      if (nb > kFixBatch) {
+      for (int c = 0; c < 4; ++c) {
+        const int cs = jv ? f.col_sum_w[j + c] : 0;
+        cwc[c] = (float)(cs - Cn * f.ow);
+        cwi[c] = (int)cwc[c];
+        U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
+      }
+      if (!fast) {
+        fix_group_general(f, k0, nb, j, jv, cwc, cwi, U, inv_sw, y);
+        continue;
+      }
+      // ---- pass 1: block sums S = sum P + CWc sum m, lead I_p ----
+      uint32_t sb[4] = {0u, 0u, 0u, 0u};
+      float4 Pb[kFixBatch];
+      float4 P0 = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int r0 = 0; r0 < nb; r0 += kFixBatch) {
 #pragma unroll
         for (int b = 0; b < kFixBatch; ++b) {
           const int prb = __shfl_sync(0xffffffffu, pr, (r0 + b) & 31);
           Pb[b] = r0 + b < nb ? ld_row4(f, prb, j, jv) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
+#pragma unroll
+        for (int b = 0; b < kFixBatch; ++b) {
+          if (r0 + b >= nb) break;
+          sb[0] += magic_bits(Pb[b].x);
+          sb[1] += magic_bits(Pb[b].y);
+          sb[2] += magic_bits(Pb[b].z);
+          sb[3] += magic_bits(Pb[b].w);
+        }
+        if (r0 == 0) P0 = Pb[0];
       }
+      const float p0[4] = {P0.x, P0.y, P0.z, P0.w};
+      BlockFixF bf[4];
 #pragma unroll
-      for (int b = 0; b < kFixBatch; ++b) {
-        const int r = r0 + b;
-        const int src = r & 31;
-        const float4 q = make_float4(__shfl_sync(0xffffffffu, kq.x, src),
-                                     __shfl_sync(0xffffffffu, kq.y, src),
-                                     __shfl_sync(0xffffffffu, kq.z, src),
-                                     __shfl_sync(0xffffffffu, kq.w, src));
-        const int prb = __shfl_sync(0xffffffffu, pr, src);
-        if (r >= nb || !jv) continue;
-        const float pv[4] = {Pb[b].x, Pb[b].y, Pb[b].z, Pb[b].w};
-        float o4[4];
+      for (int c = 0; c < 4; ++c) {
+        const int S = (int)(sb[c] - (uint32_t)nb * kMagicBits) + cwi[c] * msum;
+        bf[c] = block_fix_f(hc, S, magic_int(p0[c]) + (int)mp * cwi[c]);
+      }
+      // ---- pass 2: offsets and the inverse reflection ----
+      for (int r0 = 0; r0 < nb; r0 += kFixBatch) {
+        if (nb > kFixBatch) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
-          o4[c] = r == 0 ? dequant(q, bf[c].lead, U[c])
-                         : dequant(q, reflect_f(pv[c], q, cwc[c], bf[c]), U[c]);
-        __stcs(reinterpret_cast<float4 *>(f.out + (int64_t)prb * f.D + j),
-               make_float4(o4[0], o4[1], o4[2], o4[3]));
+          for (int b = 0; b < kFixBatch; ++b) {
+            const int prb = __shfl_sync(0xffffffffu, pr, (r0 + b) & 31);
+            Pb[b] = r0 + b < nb ? ld_row4(f, prb, j, jv) : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        }
+#pragma unroll
+        for (int b = 0; b < kFixBatch; ++b) {
+          const int r = r0 + b;
+          const int src = r & 31;
+          const float4 q = make_float4(__shfl_sync(0xffffffffu, kq.x, src),
+                                       __shfl_sync(0xffffffffu, kq.y, src),
+                                       __shfl_sync(0xffffffffu, kq.z, src),
+                                       __shfl_sync(0xffffffffu, kq.w, src));
+          const int prb = __shfl_sync(0xffffffffu, pr, src);
+          if (r >= nb || !jv) continue;
+          const float pv[4] = {Pb[b].x, Pb[b].y, Pb[b].z, Pb[b].w};
+          float o4[4];
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+            o4[c] = r == 0 ? dequant(q, bf[c].lead, U[c])
+                           : dequant(q, reflect_f(pv[c], q, cwc[c], bf[c]), U[c]);
+          __stcs(reinterpret_cast<float4 *>(f.out + (int64_t)prb * f.D + j),
+                 make_float4(o4[0], o4[1], o4[2], o4[3]));
+        }
       }
     }
   }

@@ -437,8 +437,9 @@ __global__ void __launch_bounds__(256) k_grp_layout(const int32_t *__restrict__ 
                                                     const ff *__restrict__ cincl,
                                                     const long long *Gp, const ff *SGp,
                                                     int32_t *perm, int32_t *gstart,
-                                                    int32_t *gsize) {
+                                                    int32_t *gsize, unsigned *slots) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i == 0) *slots = 0u;
   if (i > N) return;
   const int64_t G = *Gp;
   if (i >= G) {
@@ -638,11 +639,13 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
     }
   };
 
-  // A warp takes slots of RS consecutive groups: all single rows -> one step;
-  // otherwise the groups one after another, a warp each.
-  const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t g0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + warp) * RS; g0 < N;
-       g0 += wstride * RS) {
+  // A warp takes slots of RS consecutive groups from a queue: all single
+  // rows -> one step; otherwise the groups one after another, a warp each.
+  for (;;) {
+    unsigned slot = 0u;
+    if (lane == 0) slot = atomicAdd(a.slots, 1u);
+    const int64_t g0 = (int64_t)__shfl_sync(0xffffffffu, slot, 0) * RS;
+    if (g0 >= N) break;
     const int64_t gk = g0 + (lane < RS ? lane : 0);
     const int64_t ka = gk < N ? __ldg(a.gstart + gk) : N;
     const int64_t kb = gk < N ? __ldg(a.gstart + gk + 1) : N;
@@ -878,6 +881,7 @@ struct GroupScratch {
   long long *G;
   ff *SG;
   unsigned *count;
+  unsigned *slots;  // work queue of the group quantizer
 };
 
 size_t carve(char *base, int64_t N, GroupScratch *s) {
@@ -896,7 +900,7 @@ size_t carve(char *base, int64_t N, GroupScratch *s) {
   char *tsum = take((size_t)ntc * 4 * sizeof(ff));
   char *cincl = take((size_t)N * sizeof(ff) + 8);
   char *best = take((size_t)ntc * sizeof(BestFF));
-  char *G = take(8), *SG = take(8), *count = take(8);
+  char *G = take(8), *SG = take(8), *count = take(8), *slots = take(8);
   if (s) {
     s->k0 = reinterpret_cast<uint32_t *>(k0);
     s->k1 = reinterpret_cast<uint32_t *>(k1);
@@ -909,6 +913,7 @@ size_t carve(char *base, int64_t N, GroupScratch *s) {
     s->G = reinterpret_cast<long long *>(G);
     s->SG = reinterpret_cast<ff *>(SG);
     s->count = reinterpret_cast<unsigned *>(count);
+    s->slots = reinterpret_cast<unsigned *>(slots);
   }
   return off;
 }
@@ -919,7 +924,7 @@ size_t group_workspace_bytes(int64_t N) { return N > 0 ? carve(nullptr, N, nullp
 
 fqt_status launch_bhq_grouping(const void *dH, bool bf16, int64_t N, int C, int32_t *perm,
                                int32_t *gstart, int32_t *gsize, void *scratch,
-                               size_t scratch_bytes, cudaStream_t st) {
+                               size_t scratch_bytes, unsigned **slot_counter, cudaStream_t st) {
   if (N <= 0) return FQT_OK;
   if (N > kMaxGroupRows) return FQT_EUNSUPPORTED;
   GroupScratch s;
@@ -966,7 +971,8 @@ fqt_status launch_bhq_grouping(const void *dH, bool bf16, int64_t N, int C, int3
   k_grp_tsum<<<ntc, 256, 0, st>>>(kin, N, s.tsum);
   k_grp_choose<<<ntc, 256, 0, st>>>(kin, N, s.tsum, s.cincl, s.best, s.G, s.SG, s.count);
   k_grp_layout<<<(int)((N + 1 + 255) / 256), 256, 0, st>>>(vin, N, s.cincl, s.G, s.SG, perm,
-                                                             gstart, gsize);
+                                                             gstart, gsize, s.slots);
+  if (slot_counter) *slot_counter = s.slots;
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "grouping choice launch");
   return FQT_OK;

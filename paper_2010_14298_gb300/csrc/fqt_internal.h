@@ -33,6 +33,7 @@ struct QuantArgs {
   int32_t *rsum1, *csum1;
   float *hz, *hr;  // BHQ grad_X offsets of code set 2 (may be null)
   const int32_t *perm, *gstart;  // adaptive BHQ groups (block 0)
+  unsigned *slots;               // their work queue (zeroed by the grouping)
   const float2 *part;
   int npart;
   int *status;
@@ -65,7 +66,7 @@ cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
 size_t group_workspace_bytes(int64_t N);
 fqt_status launch_bhq_grouping(const void *dH, bool bf16, int64_t N, int C, int32_t *perm,
                                int32_t *gstart, int32_t *gsize, void *scratch,
-                               size_t scratch_bytes, cudaStream_t st);
+                               size_t scratch_bytes, unsigned **slot_counter, cudaStream_t st);
 fqt_status launch_bhq_groups(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 
 int device_sm_count();
