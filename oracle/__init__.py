@@ -10,6 +10,8 @@ Every function cites the passage of the paper it restates:
 
 * ``quantize_grad``  -- PTQ (Sec. 3.3), PSQ (Sec. 4.1), BHQ (Sec. 4.2, App. D.4)
 * ``bhq_grouping``   -- the adaptive BHQ groups of App. D.5 (block = 0)
+* SHIFT quantizer   -- per-tensor range, per-sample power-of-two shifts (Sec. 4.3)
+* ``grad_w_shifted`` -- grad_W with the shifted integer accumulators of Sec. 4.3
 * ``quantize_fwd``   -- deterministic 8-bit PTQ of X and W (Sec. 2.1, App. E)
 * ``dequant``        -- Eq. 9: Q(dH) = S^-1 (codes + z' 1^T)
 * ``grad_x``/``grad_w`` -- Eq. 6 with the bifurcation of App. E
@@ -31,7 +33,7 @@ _LIB_PATH = os.path.join(_BUILD, "libfqt_oracle.so")
 _lib = None
 _lock = threading.Lock()
 
-PTQ, PSQ, BHQ = 0, 1, 2
+PTQ, PSQ, BHQ, SHIFT = 0, 1, 2, 3
 STREAM_B2, STREAM_B1 = 0, 1
 
 
@@ -150,7 +152,9 @@ def quantize_grad(dH, kind: int, bits: int, block: int = 0, seed: int = 0,
 
     Returns codes (uint8, N x C), inv_s and zero (1 entry for PTQ, N otherwise),
     lead (BHQ: lead row of each block) and, with want_v, the pre-rounding
-    values v that SR acts on.  BHQ with block = 0 takes the adaptive groups
+    values v that SR acts on.  SHIFT (kind 3) is the per-tensor-range,
+    per-sample-shift quantizer of Sec. 4.3 (reading R9 of fqt_oracle.c); its
+    dict carries ``shift`` (per row) instead of lead.  BHQ with block = 0 takes the adaptive groups
     of App. D.5 (``bhq_grouping``): codes, inv_s, zero and v are then in the
     grouped (stored) order, row k holding row perm[k] of dH, and the dict
     also carries perm, gstart, gsize and G.
@@ -166,18 +170,46 @@ def quantize_grad(dH, kind: int, bits: int, block: int = 0, seed: int = 0,
     inv_s = np.zeros(m, dtype=np.float32)
     zero = np.zeros(m, dtype=np.float32)
     nblk = (n + block - 1) // block if kind == BHQ else 0
-    lead = np.zeros(max(nblk, 1), dtype=np.int32)
+    # BHQ: lead row of each block; SHIFT: the shift of each row
+    lead = np.zeros(max(n if kind == SHIFT else nblk, 1), dtype=np.int32)
     v = np.zeros((n, c), dtype=np.float32) if want_v else None
-    bad = _load().orc_quantize_grad(_ptr(h), n, c, kind, bits, block, seed,
-                                    stream, _ptr(codes), _ptr(inv_s),
-                                    _ptr(zero), _ptr(lead), _ptr(v))
+    bad = _load().orc_quantize_grad(_ptr(h), n, c, kind, bits,
+                                    block if kind == BHQ else 0, seed, stream,
+                                    _ptr(codes), _ptr(inv_s), _ptr(zero),
+                                    _ptr(lead), _ptr(v))
     if bad:
         raise OracleError(f"{bad} non-finite gradient entries")
     out = dict(codes=codes, inv_s=inv_s, zero=zero, kind=kind, bits=bits,
-               block=block, lead=lead[:nblk] if kind == BHQ else None)
+               block=block if kind == BHQ else 0,
+               lead=lead[:nblk] if kind == BHQ else None)
+    if kind == SHIFT:
+        out["shift"] = lead[:n].copy()
     if want_v:
         out["v"] = v
     return out
+
+
+def shifted_codes(q: dict) -> np.ndarray:
+    """Integer codes of the shift quantizer on the common scale 1 / (16 s)
+    (Sec. 4.3): a_ic = 2^(4 - shift_i) (code_ic - 2^(b-1)), exact in int64."""
+    z0 = 1 << (q["bits"] - 1)
+    sh = np.asarray(q["shift"], dtype=np.int64)
+    return (np.asarray(q["codes"], dtype=np.int64) - z0) << (4 - sh)[:, None]
+
+
+def grad_w_shifted(q: dict, q_x: dict) -> np.ndarray:
+    """grad_W = Q(dH)^T X~ for the shift quantizer, as Sec. 4.3 describes the
+    hardware form: every sample's integer products are shifted by its
+    2^(4 - shift_i) before the sum over samples (exact int64), and one scale
+    1 / (16 s) is applied at the end.  X~ = inv_sx (codes_x + zero_x)."""
+    a = shifted_codes(q)                                   # N x C, int64
+    cx = np.asarray(q_x["codes"], dtype=np.int64)          # N x D
+    P = a.T @ cx                                           # exact
+    colsum_a = a.sum(axis=0)                               # C
+    inv16s = float(np.float64(q["inv_s"][0]) * 2.0 ** (int(q["shift"][0]) - 4)) \
+        if len(q["shift"]) else 0.0
+    ix, zx = float(q_x["inv_s"][0]), float(q_x["zero"][0])
+    return inv16s * ix * (P.astype(np.float64) + zx * colsum_a[:, None].astype(np.float64))
 
 
 def bhq_grouping(dH, want_v: bool = False) -> dict:

@@ -41,6 +41,13 @@
  *      1 / s and zero = s * z (PTQ/PSQ; Q_blk = I) or z' (BHQ).
  *  R7  Forward quantizers Q_f, Q_theta (Sec. 2.1, App. E): deterministic
  *      8-bit PTQ, round half to even, codes clamped to [0, B].
+ *  R9  Shift quantizer (Sec. 4.3, left open by the paper): the range is
+ *      per tensor and symmetric, [-M, M], so that every row shares the
+ *      integer midpoint code 2^(b-1) as its zero point; a per-row zero point
+ *      would add a per-row offset that shifted integer accumulators cannot
+ *      absorb, and a per-tensor minimum as zero point leaves no room to
+ *      shift rows that straddle 0.  Shifts are capped at 4 (the paper's
+ *      [0, 4]).
  *  R8  Adaptive BHQ groups (App. D.5): as printed, the variance estimate
  *      sum_i M_i^2 / size_i with size_i = (N - G) M_i / sum M equals
  *      (sum_{i<=G} M_i)^2 / (N - G), which grows with G, so it would always
@@ -473,7 +480,51 @@ int64_t orc_quant_bhq_groups(const float *h, int64_t n, int64_t c, int bits,
   return 0;
 }
 
-/* Gradient quantizer dispatch: kind 0 = PTQ, 1 = PSQ, 2 = BHQ. */
+/* ------------------------------------------------------------------------ */
+/* Per-sample power-of-two shift quantizer (Sec. 4.3; R9): one symmetric     */
+/* per-tensor range [-M, M], M = max |dH|, base scale s = (2^(b-1) - 1) / M, */
+/* and per row a shift sh_i, the largest integer in [0, 4] with              */
+/* 2^sh_i ||h_i||_inf <= M.  Row i is quantized with s 2^sh_i around the     */
+/* integer midpoint z0 = 2^(b-1): v = (s 2^sh_i) h + z0, code = SR(v), so    */
+/* value = (code - z0) / (s 2^sh_i): inv_s_i = (1/s) 2^-sh_i, zero_i = -z0   */
+/* (R6's encoding, per row).  M = 0 (or s not finite) takes s = 1.           */
+/* `shift` receives sh_i.                                                    */
+/* ------------------------------------------------------------------------ */
+int64_t orc_quant_shift(const float *h, int64_t n, int64_t c, int bits,
+                        uint64_t seed, uint32_t stream, uint8_t *codes,
+                        float *inv_s, float *zero, int32_t *shift, float *vout) {
+  uint32_t B = (1u << bits) - 1u;
+  float z0 = (float)(1u << (bits - 1));
+  float gmn, gmx;
+  int64_t bad = orc_range(h, n * c, &gmn, &gmx);
+  if (bad) return bad;
+  float M = fabsf(gmn) > fabsf(gmx) ? fabsf(gmn) : fabsf(gmx);
+  float s = (float)((1u << (bits - 1)) - 1u) / M;
+  if (!(M > 0.0f) || !isfinite(s)) s = 1.0f;
+  float inv = 1.0f / s;
+  for (int64_t r = 0; r < n; ++r) {
+    const float *row = h + r * c;
+    float mn, mx;
+    orc_range(row, c, &mn, &mx);
+    float Mi = fabsf(mn) > fabsf(mx) ? fabsf(mn) : fabsf(mx);
+    int sh = 0;
+    while (sh < 4 && ldexpf(Mi, sh + 1) <= M) ++sh;
+    float sr = ldexpf(s, sh); /* exact: a power-of-two multiple */
+    for (int64_t j = 0; j < c; ++j) {
+      int64_t i = r * c + j;
+      float v = sr * row[j] + z0;
+      if (vout) vout[i] = v;
+      codes[i] = (uint8_t)orc_sr(v, orc_u16(seed, stream, (uint64_t)i), B);
+    }
+    inv_s[r] = ldexpf(inv, -sh);
+    zero[r] = -z0;
+    shift[r] = sh;
+  }
+  return 0;
+}
+
+/* Gradient quantizer dispatch: kind 0 = PTQ, 1 = PSQ, 2 = BHQ, 3 = the shift
+ * quantizer (`lead` then receives the per-row shifts). */
 int64_t orc_quantize_grad(const float *h, int64_t n, int64_t c, int kind,
                           int bits, int block, uint64_t seed, uint32_t stream,
                           uint8_t *codes, float *inv_s, float *zero,
@@ -482,6 +533,8 @@ int64_t orc_quantize_grad(const float *h, int64_t n, int64_t c, int kind,
     return orc_quant_ptq(h, n, c, bits, seed, stream, codes, inv_s, zero, vout);
   if (kind == 1)
     return orc_quant_psq(h, n, c, bits, seed, stream, codes, inv_s, zero, vout);
+  if (kind == 3)
+    return orc_quant_shift(h, n, c, bits, seed, stream, codes, inv_s, zero, lead, vout);
   return orc_quant_bhq(h, n, c, bits, block, seed, stream, codes, inv_s, zero,
                        lead, vout);
 }

@@ -585,3 +585,99 @@ def test_bhq_adaptive_variance_bound(bits):
             lam2 = 2 * np.abs(blk[1:]).max()
             hh = (lam1 ** (2 / 3) * nb ** (-1 / 3) + lam2 ** (2 / 3) * nb ** (2 / 3)) ** 3
             assert frob <= hh / B ** 2 * (1 + 1e-5)
+
+
+# --------------------------------------------------------------------------
+# Per-sample power-of-two shift quantizer (Sec. 4.3, reading R9 of the oracle)
+# --------------------------------------------------------------------------
+def test_shift_quantizer_shift_values():
+    """Rows scaled by known powers of two: shift_i is the largest integer in
+    [0, 4] with 2^shift ||h_i||_inf <= M (equality allowed), capped at 4."""
+    base = np.linspace(-1.0, 1.0, 16, dtype=np.float32)  # ||.||_inf = 1
+    scales = [1.0, 0.5, 0.5 * 0.999, 0.25, 0.125, 1 / 16, 1 / 64, 0.0, 0.75]
+    want = [0, 1, 1, 2, 3, 4, 4, 4, 0]
+    h = np.stack([base * np.float32(a) for a in scales]).astype(np.float32)
+    q = orc.quantize_grad(h, orc.SHIFT, 5, 0, seed=1)
+    assert list(q["shift"]) == want
+    s = np.float32(15) / np.float32(1.0)  # (2^(b-1) - 1) / M
+    assert np.array_equal(q["inv_s"], np.float32(1) / s * np.float32(2.0) ** -np.array(want, np.float32))
+    assert np.all(q["zero"] == -16)
+
+
+@pytest.mark.parametrize("bits", [3, 5, 8])
+def test_shift_quantizer_is_unbiased_exactly_and_in_range(bits):
+    g = wl.rng(120 + bits)
+    h = wl.random_grad(g, 10, 12, sigma=2.0, outlier_frac=0.2)
+    B = (1 << bits) - 1
+    q = orc.quantize_grad(h, orc.SHIFT, bits, 0, seed=7, want_v=True)
+    v = q["v"]
+    assert v.min() >= 1.0 - 1e-5 and v.max() <= B + 1e-5  # |s 2^sh h| <= 2^(b-1) - 1
+    m, var = _moments(v, B)
+    e = orc.dequant(q, m)
+    # E[code] falls below v by less than 2^-16 of a bin (R1), v is fp32
+    inv = q["inv_s"].astype(np.float64)[:, None]
+    assert np.all(np.abs(e - h) <= inv * 2.0 ** -15)
+    # per-entry variance p(1-p) / (s 2^sh)^2 <= 1 / (4 (s 2^sh)^2)
+    assert np.all(var * inv ** 2 <= 0.25 * inv ** 2 * (1 + 1e-9))
+
+
+def test_shift_quantizer_beats_the_symmetric_per_tensor_range():
+    """Rows far below the largest get up to 16x finer steps: the exact
+    variance falls below the unshifted (shift 0) quantizer's, by up to 256x per
+    such row (Sec. 4.3's motivation, Sec. 4.1's per-sample argument)."""
+    g = wl.rng(130)
+    h = (0.01 * g.standard_normal((8, 16))).astype(np.float32)
+    h[2] = 5.0 * g.standard_normal(16)
+    bits = 4
+    q = orc.quantize_grad(h, orc.SHIFT, bits, 0, want_v=True)
+    _, var = _moments(q["v"], (1 << bits) - 1)
+    vq = var * (q["inv_s"].astype(np.float64) ** 2)[:, None]
+    assert q["shift"][2] == 0 and np.all(np.delete(q["shift"], 2) == 4)
+    # the same rows with every shift forced to 0: step 1/s instead of 1/(16 s)
+    step0 = q["inv_s"][2].astype(np.float64)
+    small = np.delete(np.arange(8), 2)
+    assert vq[small].sum() <= small.size * 16 * 0.25 * (step0 / 16) ** 2 * (1 + 1e-9)
+    assert vq[small].max() < 0.25 * step0 ** 2 / 200
+
+
+def test_shift_quantizer_equal_rows_is_symmetric_ptq():
+    g = wl.rng(131)
+    base = g.standard_normal(16).astype(np.float32)
+    h = np.stack([base if k % 2 else -base for k in range(6)])
+    q = orc.quantize_grad(h, orc.SHIFT, 6, 0, seed=2)
+    assert np.all(q["shift"] == 0)
+    assert np.all(q["inv_s"] == q["inv_s"][0])
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_shifted_accumulators_equal_the_dequantized_product(bits):
+    """Sec. 4.3's hardware form: integer products of each sample shifted by
+    2^(4 - shift_i) before the sum over samples, one scale at the end, equals
+    grad_W of the dequantized codes (Eq. 6) up to double rounding."""
+    g = wl.rng(140 + bits)
+    dH = wl.random_grad(g, 40, 16, sigma=2.5, outlier_frac=0.1)
+    X = g.uniform(-1, 1, (40, 24)).astype(np.float32)
+    q = orc.quantize_grad(dH, orc.SHIFT, bits, 0, seed=9)
+    qx = orc.quantize_fwd(X)
+    a = orc.shifted_codes(q)
+    assert np.abs(a).max() <= 16 * ((1 << (bits - 1)) - 1)  # fits an fp16 carrier exactly
+    ref = orc.grad_w(q, qx)
+    got = orc.grad_w_shifted(q, qx)
+    assert np.abs(got - ref).max() <= 1e-12 * np.abs(ref).max()
+
+
+def test_shift_gradients_are_unbiased_exactly():
+    """Thm 1 with the shift quantizer feeding both contractions (no
+    bifurcation): E[grad_X] and E[grad_W] equal the QAT gradients."""
+    g = wl.rng(150)
+    dH = wl.random_grad(g, 8, 10, outlier_frac=0.25)
+    X = g.uniform(-1, 1, (8, 6)).astype(np.float32)
+    W = (0.3 * g.standard_normal((10, 6))).astype(np.float32)
+    qx, qw = orc.quantize_fwd(X), orc.quantize_fwd(W)
+    q = orc.quantize_grad(dH, orc.SHIFT, 4, 0, want_v=True)
+    m, _ = _moments(q["v"], 15)
+    Wt, Xt = orc.dequant(qw), orc.dequant(qx)
+    e = orc.dequant(q, m)
+    assert np.abs(orc.matmul(e, Wt) - dH.astype(np.float64) @ Wt).max() <= 1e-4 * np.abs(dH @ Wt).max()
+    assert np.abs(orc.matmul(e, Xt, a_trans=True) - dH.astype(np.float64).T @ Xt).max() <= \
+        1e-4 * np.abs(dH.T @ Xt).max()
