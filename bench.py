@@ -404,6 +404,51 @@ def run_gpu(args):
                "launches": {"quantize_grad": 10, "grad_x": 3},
                "device_status": fqt.sync_status(ws)}
 
+    # ---- the per-sample power-of-two shift quantizer (Sec. 4.3) on the same
+    # layer: one code set feeds both contractions (no Q_b1); one CUDA graph
+    # per call, timed alone ----
+    shf = None
+    if args.shift_steps > 0:
+        qs = fqt.QTensor.empty(N, C, fqt.SHIFT, BITS, 0, True, False, dev, u8=False)
+        fs = [lambda: fqt.quantize_grad(dH, fqt.SHIFT, BITS, 0, 11, with_b1=False, ws=ws,
+                                        q_b2=qs),
+              lambda: fqt.linear_backward(qs, None, qx, qw, grad_x=True, grad_w=False, ws=ws,
+                                          out_x=gx),
+              lambda: fqt.linear_backward(qs, None, qx, qw, grad_x=False, grad_w=True, ws=ws,
+                                          out_w=gw)]
+        for _ in range(3):
+            for f in fs:
+                f()
+        torch.cuda.synchronize()
+        gs_ = []
+        for f in fs:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                f()
+            gs_.append(g)
+        tsh = [[], [], []]
+        for i in range(args.shift_steps):
+            flush.fill_(i & 0xFF)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            for k in range(3):
+                ev[k].record(stream)
+                gs_[k].replay()
+            ev[3].record(stream)
+            torch.cuda.synchronize()
+            for k in range(3):
+                tsh[k].append(ev[k].elapsed_time(ev[k + 1]))
+        sh = qs.shift.cpu().numpy()
+        shf = {"quantizer": f"SHIFT-{BITS} (per-tensor range, per-row shifts in [0, 4])",
+               "quantize_grad_ms": float(np.median(tsh[0])),
+               "grad_x_ms": float(np.median(tsh[1])),
+               "grad_w_ms": float(np.median(tsh[2])),
+               "bifurcated_bhq16_ms": {"quantize_grad": float(per_call[2]),
+                                       "grad_x": float(per_call[3]),
+                                       "grad_w": float(per_call[4])},
+               "rows_per_shift": [int((sh == k).sum()) for k in range(5)],
+               "launches": {"quantize_grad": 2, "grad_x": 1, "grad_w": 2},
+               "device_status": fqt.sync_status(ws)}
+
     result = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -429,6 +474,7 @@ def run_gpu(args):
         "e2e": e2e,
         "forward": fwd,
         "adaptive_bhq": ada,
+        "shift_quantizer": shf,
         "gpu_launches": int(sum(launches_per_call) * args.steps),
         "device_status": status,
     }
@@ -509,6 +555,8 @@ def main():
                     help="timed calls of the quantized forward GEMM (0: skip)")
     ap.add_argument("--adaptive-steps", type=int, default=50,
                     help="timed steps of the adaptive BHQ groups (0: skip)")
+    ap.add_argument("--shift-steps", type=int, default=50,
+                    help="timed steps of the shift quantizer path (0: skip)")
     ap.add_argument("--eager", action="store_true",
                     help="time the C-ABI calls directly instead of graph replays")
     args = ap.parse_args()

@@ -52,7 +52,7 @@ typedef enum {
   FQT_EWORKSPACE = 6       /* workspace missing, misaligned or too small */
 } fqt_status;
 
-typedef enum { FQT_PTQ = 0, FQT_PSQ = 1, FQT_BHQ = 2 } fqt_kind;
+typedef enum { FQT_PTQ = 0, FQT_PSQ = 1, FQT_BHQ = 2, FQT_SHIFT = 3 } fqt_kind;
 typedef enum { FQT_F32 = 0, FQT_BF16 = 1 } fqt_dtype;
 
 /*
@@ -105,6 +105,14 @@ typedef struct fqt_qtensor {
                         i >= G (the number of groups) */
   int32_t *gsize;    /* BHQ block 0: rows entries, size of the group of each
                         stored row */
+  uint16_t *shift_f16; /* FQT_SHIFT: rows x cols, the codes on the common scale
+                        of all rows, a = 2^(4 - shift_i) (code - 2^(b-1)), as
+                        exact fp16 (|a| <= 16 (2^(b-1) - 1)): the grad_W
+                        operand.  Else unused (may be NULL). */
+  int32_t *shift;    /* FQT_SHIFT: rows entries, shift_i in [0, 4] */
+  int32_t *shift_col_sum; /* FQT_SHIFT: cols entries, sum_i a_ic */
+  float *shift_scale; /* FQT_SHIFT: 2 entries, the common scale 2^-4 / s of a
+                        and 0 (its zero point) */
 } fqt_qtensor;
 
 /* Bytes of workspace a layer with dH N x C, X N x D, W C x D needs for any
@@ -128,8 +136,8 @@ FQT_API fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t r
                                void *workspace, size_t ws_bytes, void *stream);
 
 /*
- * Gradient quantizers with unbiased stochastic rounding (Sec. 3.3, 4.1, 4.2)
- * and the bifurcation of App. E:
+ * Gradient quantizers with unbiased stochastic rounding (Sec. 3.3, 4.1, 4.2,
+ * 4.3) and the bifurcation of App. E:
  *   q_b2 <- Q_b2(dH): kind (PTQ, PSQ, BHQ), `bits`, BHQ `block`; feeds grad_X.
  *   q_b1 <- Q_b1(dH): 8-bit stochastic PTQ; feeds grad_W.  May be NULL.
  * SR draws 16-bit uniforms from Philox4x32-10 keyed by `seed`, counter
@@ -146,6 +154,16 @@ FQT_API fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t r
  * smallest up.  It writes q_b2->perm, gstart, gsize (required) and stores
  * the groups one after another, SR uniforms drawn by stored index.  Needs
  * C in {64, 128, 256}, N <= 2^20, and hz, hr, row_sum for the backward.
+ * FQT_SHIFT is the per-sample power-of-two shift quantizer that Sec. 4.3
+ * proposes for hardware, as this library reads it: one symmetric per-tensor
+ * range [-M, M], M = max |dH|, s = (2^(b-1) - 1) / M; row i uses the scale
+ * s 2^shift_i, shift_i the largest integer in [0, 4] with
+ * 2^shift_i ||dH_i||_inf <= M, around the midpoint code 2^(b-1):
+ * code = SR(s 2^shift_i dH_ij + 2^(b-1)); inv_s_i = 2^-shift_i / s,
+ * zero_i = -2^(b-1).  It also writes shift, shift_f16, shift_col_sum and
+ * shift_scale (required): grad_W then contracts the shifted integer codes
+ * (the samples' accumulators shifted before the sum, Sec. 4.3), so q_b1 may
+ * be NULL (no bifurcation).  Needs C in {64, 128, 256, 512, 1024}.
  */
 FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
                              int64_t C, fqt_kind kind, int bits, int block,
@@ -166,7 +184,8 @@ FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
  * must have the fp32-exact form: C 2^(bw + b - 2) < 2^24 and C at most one
  * exact chunk, else FQT_EUNSUPPORTED), qw->col_sum (grad_X) and
  * q_b1->col_sum, qx->col_sum (grad_W).  q_b1 may be
- * NULL when q_b2 is PTQ with col_sum set: grad_W then uses q_b2.
+ * NULL when q_b2 is PTQ with col_sum set, or FQT_SHIFT: grad_W then uses
+ * q_b2 (for FQT_SHIFT its shift_f16, shift_col_sum and shift_scale).
  * C % 16 == 0 and D % 16 == 0.
  */
 FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,

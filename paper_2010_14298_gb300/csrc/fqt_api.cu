@@ -141,7 +141,16 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   if (N > 0 && (!dH || (!q_b2->codes && !q_b2->codes_f16) || !q_b2->inv_s || !q_b2->zero))
     return FQT_EINVAL;
   if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
-  if (kind != FQT_PTQ && kind != FQT_PSQ && kind != FQT_BHQ) return FQT_EINVAL;
+  if (kind != FQT_PTQ && kind != FQT_PSQ && kind != FQT_BHQ && kind != FQT_SHIFT)
+    return FQT_EINVAL;
+  if (kind == FQT_SHIFT) {
+    if (N > 0 && (!q_b2->shift_f16 || !q_b2->shift || !q_b2->shift_col_sum ||
+                  !q_b2->shift_scale))
+      return FQT_EINVAL;
+    if (C % 8 || (C / 8 != 8 && C / 8 != 16 && C / 8 != 32 && C / 8 != 64 && C / 8 != 128))
+      return FQT_EUNSUPPORTED;
+    if (!aligned(q_b2->shift_f16, 16)) return FQT_EINVAL;
+  }
   // BHQ block 0: the adaptive groups of App. D.5
   const bool adapt = kind == FQT_BHQ && block == 0;
   if (kind == FQT_BHQ) {
@@ -184,8 +193,10 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   float2 *part = reinterpret_cast<float2 *>(w + kRangeOffset);
   int npart = 0;
   int32_t *csum = q_b1 ? q_b1->col_sum : (adapt ? nullptr : q_b2->col_sum);
+  // the column sums the quantizer accumulates into are cleared by the range pass
+  int32_t *csum2 = kind == FQT_SHIFT ? q_b2->shift_col_sum : nullptr;
   cudaError_t e = launch_range(dH, dtype == FQT_BF16, N * C, part, &npart, csum,
-                               csum ? C : 0, nullptr, 0, nsm, st);
+                               csum ? C : 0, csum2, csum2 ? C : 0, nsm, st);
   if (e != cudaSuccess) return cuda_fail(e, "range pass");
   QuantArgs a;
   memset(&a, 0, sizeof(a));
@@ -222,6 +233,15 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   int nth, grid;
   size_t smem;
   const bool bf16 = dtype == FQT_BF16;
+  if (kind == FQT_SHIFT) {
+    QuantArgs as = a;
+    as.fs = q_b2->shift_f16;
+    as.shift = q_b2->shift;
+    as.scs = q_b2->shift_col_sum;
+    as.sscale = q_b2->shift_scale;
+    as.csum2 = nullptr;
+    return launch_shift(as, bf16, nsm, st);
+  }
   if (adapt) {
     unsigned *slots = nullptr;
     s = launch_bhq_grouping(dH, bf16, N, (int)C, q_b2->perm, q_b2->gstart, q_b2->gsize,

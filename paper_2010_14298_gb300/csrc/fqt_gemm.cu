@@ -1518,16 +1518,24 @@ struct WPlan {
 
 static WPlan gradw_plan(int64_t K, int64_t C, int64_t D, int b1, int bx, int num_sms);
 
+// grad_W takes k_gradw (one exact chunk per K range) unless its plan would
+// need more than two ranges per SM (wide operands, e.g. the shift
+// quantizer's 12-bit shifted codes); then the split-K tile kernel, whose
+// ranges fold several exact chunks.
+static bool use_gradw(const WPlan &w, int num_sms) {
+  return w.splits > 0 && w.splits <= 2 * num_sms;
+}
+
 size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D) {
-  // grad_W: M = C, N = D, K = N (8-bit x 8-bit), by either kernel
-  const SplitPlan p = plan_splits(C, D, N, 8, 8, device_sm_count(), true);
-  const int64_t splits_t = p.splits;
-  int64_t splits_w = 0;
-  for (int b = 2; b <= 8; ++b) {  // the plan depends on the Q_b1 / X~ bits
-    const WPlan w = gradw_plan(N, C, D, b, 8, device_sm_count());
-    if (w.splits > splits_w) splits_w = w.splits;
+  // grad_W: M = C, N = D, K = N, by either kernel; the operand bits run from
+  // 2 (Q_b1) to 12 (shifted 8-bit codes of the shift quantizer)
+  const int nsm = device_sm_count();
+  int64_t splits = 0;
+  for (int b = 2; b <= 12; ++b) {
+    const WPlan w = gradw_plan(N, C, D, b, 8, nsm);
+    const int64_t sp = use_gradw(w, nsm) ? w.splits : plan_splits(C, D, N, b, 8, nsm, true).splits;
+    if (sp > splits) splits = sp;
   }
-  const int64_t splits = splits_t > splits_w ? splits_t : splits_w;
   const size_t bytes = (size_t)splits * (size_t)C * (size_t)D * 4;
   return (bytes + 255) & ~(size_t)255;
 }
@@ -2380,30 +2388,37 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
   }
   if (grad_W) {
     const fqt_qtensor *qa = q_b1 ? q_b1 : q_b2;
-    if (!qa || !qx || !qa->codes_f16 || !qx->codes_f16 || !qa->col_sum || !qx->col_sum ||
-        !qa->inv_s || !qa->zero || !qx->inv_s || !qx->zero)
+    // the shift quantizer feeds grad_W itself: its codes on the common scale
+    const bool shifted = qa && qa->kind == FQT_SHIFT;
+    if (!qa || !qx || !qx->codes_f16 || !qx->col_sum || !qx->inv_s || !qx->zero)
       return FQT_EINVAL;
-    if (qa->kind != FQT_PTQ || qx->kind != FQT_PTQ) return FQT_EINVAL;
+    if (shifted ? (!qa->shift_f16 || !qa->shift_col_sum || !qa->shift_scale)
+                : (!qa->codes_f16 || !qa->col_sum || !qa->inv_s || !qa->zero))
+      return FQT_EINVAL;
+    if ((!shifted && qa->kind != FQT_PTQ) || qx->kind != FQT_PTQ) return FQT_EINVAL;
+    const uint16_t *A16 = shifted ? qa->shift_f16 : qa->codes_f16;
+    // |shifted code| <= 16 (2^(b-1) - 1) < 2^(b+3): b + 4 bits of centred magnitude
+    const int a_bits = shifted ? qa->bits + 4 : qa->bits;
     const int64_t Nr = qa->rows, C = qa->cols, D = qx->cols;
     if (qx->rows != Nr) return FQT_EINVAL;
     if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
-    if (!aligned16(qa->codes_f16) || !aligned16(qx->codes_f16)) return FQT_EINVAL;
-    const SplitPlan p = plan_splits(C, D, Nr, qa->bits, qx->bits, nsm, true);
-    const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, qa->bits, qx->bits, nsm) : WPlan{};
-    const int splits = wp.splits > 0 ? wp.splits : p.splits;
+    if (!aligned16(A16) || !aligned16(qx->codes_f16)) return FQT_EINVAL;
+    const SplitPlan p = plan_splits(C, D, Nr, a_bits, qx->bits, nsm, true);
+    const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, a_bits, qx->bits, nsm) : WPlan{};
+    const bool w_ok = use_gradw(wp, nsm);
+    const int splits = w_ok ? wp.splits : p.splits;
     const size_t need = kGemmOffset + (size_t)splits * (size_t)C * (size_t)D * 4;
     if (ws_bytes < need) return FQT_EWORKSPACE;
     int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kGemmOffset);
-    if (Nr > 0 && wp.splits > 0) {
-      fqt_status s = run_gradw(qx->codes_f16, qa->codes_f16, Nr, (int)C, (int)D, wp, part,
-                               status, st);
+    if (Nr > 0 && w_ok) {
+      fqt_status s = run_gradw(qx->codes_f16, A16, Nr, (int)C, (int)D, wp, part, status, st);
       if (s != FQT_OK) return s;
     } else if (Nr > 0) {
       GemmArgs g;
       memset(&g, 0, sizeof(g));
       g.status = status;
-      fqt_status s = run_gemm(qa->codes_f16, 0, qa->bits, qx->codes_f16, 0, qx->bits, C,
-                              D, Nr, p, g, part, MODE_PARTIAL, 1, false, st);
+      fqt_status s = run_gemm(A16, 0, a_bits, qx->codes_f16, 0, qx->bits, C, D, Nr, p, g,
+                              part, MODE_PARTIAL, 1, false, st);
       if (s != FQT_OK) return s;
     } else {
       const cudaError_t e = cudaMemsetAsync(part, 0, (size_t)C * D * 4, st);
@@ -2417,12 +2432,13 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     r.N = D;
     r.out_f32 = grad_W;
     r.Kn = Nr;
-    r.oa = 1 << (qa->bits - 1);
+    // shifted codes are their own carriers (offset 0, zero point 0)
+    r.oa = shifted ? 0 : 1 << (qa->bits - 1);
     r.ob = 1 << (qx->bits - 1);
-    r.cs_a = qa->col_sum;
+    r.cs_a = shifted ? qa->shift_col_sum : qa->col_sum;
     r.cs_b = qx->col_sum;
-    r.inv_a = qa->inv_s;
-    r.zero_a = qa->zero;
+    r.inv_a = shifted ? qa->shift_scale : qa->inv_s;
+    r.zero_a = shifted ? qa->shift_scale + 1 : qa->zero;
     r.inv_b = qx->inv_s;
     r.zero_b = qx->zero;
     launch_reduce(r, st);

@@ -9,7 +9,7 @@
 
 namespace fqt {
 
-enum { KIND_PTQ = 0, KIND_PSQ = 1, KIND_BHQ = 2, KIND_DET = 3 };
+enum { KIND_PTQ = 0, KIND_PSQ = 1, KIND_BHQ = 2, KIND_SHIFT = 3, KIND_DET = 4 };
 
 
 
@@ -34,6 +34,11 @@ struct QuantArgs {
   float *hz, *hr;  // BHQ grad_X offsets of code set 2 (may be null)
   const int32_t *perm, *gstart;  // adaptive BHQ groups (block 0)
   unsigned *slots;               // their work queue (zeroed by the grouping)
+  // the shift quantizer (KIND_SHIFT): shifted carriers, shifts, their column
+  // sums and the common scale / zero point
+  uint16_t *fs;
+  int32_t *shift, *scs;
+  float *sscale;
   const float2 *part;
   int npart;
   int *status;
@@ -59,6 +64,7 @@ fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, in
                             int npart, float *inv_out, float *zero_out, int *status,
                             int num_sms, cudaStream_t st);
 fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
+fqt_status launch_shift(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
                                const int32_t *lead, float *hz, float *hr, int64_t N,
                                int C, int bits, int block, cudaStream_t st);

@@ -1244,6 +1244,220 @@ fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st
 }
 
 // ---------------------------------------------------------------------------
+// Per-sample power-of-two shift quantizer (Sec. 4.3; the reading is stated in
+// include/fqt.h): one symmetric per-tensor range [-M, M] from the range pass,
+// s = (2^(b-1) - 1) / M, and per row the largest shift in [0, 4] with
+// 2^shift ||h_i||_inf <= M; code = SR(s 2^shift h + 2^(b-1)).  A row is held
+// by LPR lanes, OPL octs (8 columns) each, in registers; a warp step covers
+// RS = 32 / LPR rows.  Besides the grad_X encoding (codes, centred fp16
+// carriers, row sums, inv_s = 2^-shift / s, zero = -2^(b-1)) it writes the
+// grad_W operand: the codes on the common scale 2^-4 / s, a = 2^(4 - shift)
+// (code - 2^(b-1)), as exact fp16, and their column sums.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void store_shifted8(uint16_t *dst, const uint32_t (&c)[8],
+                                               uint32_t off, float mul) {
+  const __half2 bias = __half2half2(__int2half_rn(1024 + (int)off));
+  const __half2 m2 = __float2half2_rn(mul);  // a power of two: exact products
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t hb = (0x6400u | c[2 * i]) | ((0x6400u | c[2 * i + 1]) << 16);
+    __half2 v = __hmul2(__hsub2(*reinterpret_cast<const __half2 *>(&hb), bias), m2);
+    w[i] = *reinterpret_cast<uint32_t *>(&v);
+  }
+  *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+template <typename T, int LPR, int OPL>
+__global__ void __launch_bounds__(256) k_shift(const QuantArgs a) {
+  __shared__ float2 red[8];
+  __shared__ int redi[8];
+  extern __shared__ int csum_s[];  // [C] shifted-code column sums, [C] Q_b1 column sums
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int RS = 32 / LPR, C = 8 * LPR * OPL, CO = C / 8;
+  const int sub = lane / LPR, o = lane - sub * LPR;
+
+  // ---- global range from the range-pass partials ----
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < a.npart; i += blockDim.x) {
+    const float2 p = a.part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmin, gmax);
+    redi[warp] = bad;
+  }
+  for (int i = tid; i < 2 * C; i += blockDim.x) csum_s[i] = 0;
+  __syncthreads();
+  gmin = red[0].x;
+  gmax = red[0].y;
+  bad = redi[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+    gmin = fminf(gmin, red[w].x);
+    gmax = fmaxf(gmax, red[w].y);
+    bad |= redi[w];
+  }
+  if (bad) {
+    if (blockIdx.x == 0 && tid == 0) record_status(a.status, FQT_ENONFINITE);
+    return;
+  }
+  const uint32_t B = (1u << a.bits) - 1u, z0 = 1u << (a.bits - 1);
+  const float M = fmaxf(fabsf(gmin), fabsf(gmax));
+  float s = __fdiv_rn((float)(z0 - 1u), M);
+  if (!(M > 0.0f) || !isfinite(s)) s = 1.0f;
+  const float inv = __fdiv_rn(1.0f, s);
+  const float s_g1 = affine_scale(gmin, gmax, 255u);
+  const float s_g1_16 = __fmul_rn(s_g1, 65536.0f);
+  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
+  if (blockIdx.x == 0 && tid == 0) {
+    a.sscale[0] = __fmul_rn(inv, 0.0625f);
+    a.sscale[1] = 0.0f;
+    if (has_b1) {
+      a.inv1[0] = __fdiv_rn(1.0f, s_g1);
+      a.zero1[0] = __fmul_rn(s_g1, gmin);
+    }
+  }
+  PhiloxKeys key;
+#pragma unroll
+  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
+  int csA[OPL][8], cs1[OPL][8];
+#pragma unroll
+  for (int q = 0; q < OPL; ++q)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) csA[q][j] = cs1[q][j] = 0;
+  const T *h = reinterpret_cast<const T *>(a.h);
+  const int64_t step = (int64_t)gridDim.x * (blockDim.x >> 5) * RS;
+  for (int64_t r0 = ((int64_t)blockIdx.x * (blockDim.x >> 5) + warp) * RS; r0 < a.N;
+       r0 += step) {
+    const int64_t row = r0 + sub;
+    const bool v = row < a.N;
+    float x[OPL][8];
+#pragma unroll
+    for (int q = 0; q < OPL; ++q) {
+      if (v) {
+        load_oct(h + row * C + (q * LPR + o) * 8, x[q]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) x[q][j] = 0.0f;
+      }
+    }
+    float mi = 0.0f;
+#pragma unroll
+    for (int q = 0; q < OPL; ++q)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) mi = fmaxf(mi, fabsf(x[q][j]));
+    mi = row_reduce<LPR>(mi, OpMaxF());
+    // largest shift in [0, 4] with 2^shift ||h_i||_inf <= M (exact products)
+    int sh = 0;
+#pragma unroll
+    for (int k = 1; k <= 4; ++k)
+      if (__fmul_rn(mi, (float)(1 << k)) <= M) sh = k;
+    const float sr = __fmul_rn(s, (float)(1 << sh));
+    const float mul = (float)(1 << (4 - sh));
+    int rs2 = 0, rs1 = 0;
+#pragma unroll
+    for (int q = 0; q < OPL; ++q) {
+      if (!v) continue;
+      const int oct = q * LPR + o;
+      const uint64_t qi = (uint64_t)row * (uint64_t)CO + (uint64_t)oct;
+      const uint4 w2 = philox_oct(qi, 0u, key);
+      uint32_t c[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float vv = __fadd_rn(__fmul_rn(sr, x[q][j]), (float)z0);
+        c[j] = sr_code16(__fmul_rn(vv, 65536.0f), u16_of(w2, j), B);
+        rs2 += (int)c[j];
+        csA[q][j] += ((int)c[j] - (int)z0) * (1 << (4 - sh));
+      }
+      if (a.c2) store_codes8(a.c2 + row * (int64_t)C + oct * 8, c);
+      if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + oct * 8, c, z0);
+      store_shifted8(a.fs + row * (int64_t)C + oct * 8, c, z0, mul);
+      if (has_b1) {
+        const uint4 w1 = philox_oct(qi, 1u, key);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float vv = __fmul_rn(__fsub_rn(x[q][j], gmin), s_g1_16);
+          c[j] = sr_code16(vv, u16_of(w1, j), 255u);
+          rs1 += (int)c[j];
+          cs1[q][j] += (int)c[j];
+        }
+        if (a.c1) store_codes8(a.c1 + row * (int64_t)C + oct * 8, c);
+        if (a.f1) store_carriers8(a.f1 + row * (int64_t)C + oct * 8, c, 128u);
+      }
+    }
+    rs2 = row_reduce<LPR>(rs2, OpAdd());
+    if (has_b1) rs1 = row_reduce<LPR>(rs1, OpAdd());
+    if (v && o == 0) {
+      if (a.rsum2) a.rsum2[row] = rs2;
+      if (has_b1 && a.rsum1) a.rsum1[row] = rs1;
+      a.inv2[row] = __fmul_rn(inv, __fdiv_rn(1.0f, (float)(1 << sh)));
+      a.zero2[row] = -(float)z0;
+      a.shift[row] = sh;
+    }
+  }
+  // ---- column sums: rows of a step, then the CTA, then global ----
+#pragma unroll
+  for (int q = 0; q < OPL; ++q)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int va = xor_reduce<LPR>(csA[q][j], OpAdd());
+      const int v1 = has_b1 ? xor_reduce<LPR>(cs1[q][j], OpAdd()) : 0;
+      if (sub == 0) {
+        if (va) atomicAdd(&csum_s[(q * LPR + o) * 8 + j], va);
+        if (v1) atomicAdd(&csum_s[C + (q * LPR + o) * 8 + j], v1);
+      }
+    }
+  __syncthreads();
+  for (int i = tid; i < C; i += blockDim.x) {
+    if (csum_s[i]) atomicAdd(&a.scs[i], csum_s[i]);
+    if (has_b1 && a.csum1 && csum_s[C + i]) atomicAdd(&a.csum1[i], csum_s[C + i]);
+  }
+}
+
+fqt_status launch_shift(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st) {
+  if (a.C % 8) return FQT_EUNSUPPORTED;
+  const int CO = a.C / 8;
+  int lpr, opl;
+  switch (CO) {
+    case 8: lpr = 8; opl = 1; break;
+    case 16: lpr = 16; opl = 1; break;
+    case 32: lpr = 32; opl = 1; break;
+    case 64: lpr = 32; opl = 2; break;
+    case 128: lpr = 32; opl = 4; break;
+    default: return FQT_EUNSUPPORTED;
+  }
+  const int rs = 32 / lpr;
+  int64_t grid = (a.N + 8 * rs - 1) / (8 * rs);
+  const int64_t cap = (int64_t)num_sms * 4;
+  if (grid > cap) grid = cap;
+  if (grid < 1) grid = 1;
+  const size_t smem = 2 * sizeof(int) * (size_t)a.C;
+#define FQT_SH(L, P)                                                                   \
+  if (lpr == L && opl == P) {                                                          \
+    if (bf16)                                                                          \
+      k_shift<__nv_bfloat16, L, P><<<(int)grid, 256, smem, st>>>(a);                   \
+    else                                                                               \
+      k_shift<float, L, P><<<(int)grid, 256, smem, st>>>(a);                           \
+  }
+  FQT_SH(8, 1)
+  FQT_SH(16, 1)
+  FQT_SH(32, 1)
+  FQT_SH(32, 2)
+  FQT_SH(32, 4)
+#undef FQT_SH
+  return cuda_fail(cudaGetLastError(), "shift quantizer launch");
+}
+
+// ---------------------------------------------------------------------------
 // Codes of a forward operand (deterministic PTQ, Sec. 2.1 and App. E):
 // code = round_half_even((x - z) s) clamped to [0, B], z = min X, s = B / R(X).
 // A thread owns one column oct (8 columns) in every row it visits, so its

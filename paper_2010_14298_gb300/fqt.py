@@ -17,7 +17,7 @@ import torch
 
 from . import build as _build
 
-PTQ, PSQ, BHQ = 0, 1, 2
+PTQ, PSQ, BHQ, SHIFT = 0, 1, 2, 3
 F32, BF16 = 0, 1
 STATUS = {0: "FQT_OK", 1: "FQT_EINVAL", 2: "FQT_EUNSUPPORTED", 3: "FQT_ECUDA",
           4: "FQT_ENONFINITE", 5: "FQT_ETIMEOUT", 6: "FQT_EWORKSPACE"}
@@ -41,7 +41,9 @@ class _QT(ctypes.Structure):
                 ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p),
                 ("codes_f16", ctypes.c_void_p), ("hz", ctypes.c_void_p),
                 ("hr", ctypes.c_void_p), ("perm", ctypes.c_void_p),
-                ("gstart", ctypes.c_void_p), ("gsize", ctypes.c_void_p)]
+                ("gstart", ctypes.c_void_p), ("gsize", ctypes.c_void_p),
+                ("shift_f16", ctypes.c_void_p), ("shift", ctypes.c_void_p),
+                ("shift_col_sum", ctypes.c_void_p), ("shift_scale", ctypes.c_void_p)]
 
 
 def library_path() -> str:
@@ -147,7 +149,10 @@ class QTensor:
     per-row offsets the grad_X epilogue reads.  BHQ with block 0 takes the
     adaptive groups of App. D.5: rows are stored group by group, ``perm``
     maps a stored row to its row of dH, ``gstart`` holds the group starts
-    (then N) and ``gsize`` every stored row's group size.
+    (then N) and ``gsize`` every stored row's group size.  SHIFT (the
+    per-sample power-of-two shift quantizer of Sec. 4.3) also carries
+    ``shift`` (per row), ``shift16`` (the codes on the common scale, the
+    grad_W operand), ``shift_col_sum`` and ``shift_scale`` (2^-4 / s, 0).
     """
     codes: Optional[torch.Tensor]
     inv_s: torch.Tensor
@@ -164,6 +169,10 @@ class QTensor:
     perm: Optional[torch.Tensor] = None
     gstart: Optional[torch.Tensor] = None
     gsize: Optional[torch.Tensor] = None
+    shift16: Optional[torch.Tensor] = None
+    shift: Optional[torch.Tensor] = None
+    shift_col_sum: Optional[torch.Tensor] = None
+    shift_scale: Optional[torch.Tensor] = None
 
     @property
     def shape(self):
@@ -197,7 +206,13 @@ class QTensor:
                 if offsets else None),
             perm=i32(max(rows, 1)) if adaptive else None,
             gstart=i32(rows + 1) if adaptive else None,
-            gsize=i32(max(rows, 1)) if adaptive else None)
+            gsize=i32(max(rows, 1)) if adaptive else None,
+            shift16=(torch.empty((rows, cols), dtype=torch.float16, device=device)
+                     if kind == SHIFT else None),
+            shift=i32(max(rows, 1)) if kind == SHIFT else None,
+            shift_col_sum=i32(cols) if kind == SHIFT else None,
+            shift_scale=(torch.empty(2, dtype=torch.float32, device=device)
+                         if kind == SHIFT else None))
 
     def c_struct(self) -> _QT:
         rows, cols = self.shape
@@ -205,7 +220,8 @@ class QTensor:
         return _QT(rows, cols, self.bits, self.kind, self.block, 0,
                    p(self.codes), self.inv_s.data_ptr(), self.zero.data_ptr(),
                    p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16),
-                   p(self.hz), p(self.hr), p(self.perm), p(self.gstart), p(self.gsize))
+                   p(self.hz), p(self.hr), p(self.perm), p(self.gstart), p(self.gsize),
+                   p(self.shift16), p(self.shift), p(self.shift_col_sum), p(self.shift_scale))
 
     def codes_from_f16(self) -> torch.Tensor:
         """The uint8 codes recovered from the fp16 carriers."""
@@ -220,6 +236,8 @@ class QTensor:
                  block=self.block,
                  lead=(self.lead.cpu().numpy()
                        if self.kind == BHQ and self.block != 0 else None))
+        if self.shift is not None:
+            d["shift"] = self.shift.cpu().numpy()[:codes.shape[0]]
         if self.perm is not None:
             n = codes.shape[0]
             gs = self.gstart.cpu().numpy()

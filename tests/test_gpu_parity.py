@@ -512,3 +512,88 @@ def test_bhq_adaptive_full_size_sampled():
     ref = oracle_groups_grad_x(h2, hw, groups)
     rows = np.array(sorted(ref))
     assert grad_rel_err(gx[rows], np.stack([ref[r] for r in rows])) <= GRAD_TOL
+
+
+# --------------------------------------------------------------------------
+# Per-sample power-of-two shift quantizer (Sec. 4.3; kind SHIFT)
+# --------------------------------------------------------------------------
+SHIFT_C = (64, 128, 256, 512, 1024)
+
+
+def _shift_layers(cfg, small):
+    kw = {}
+    if cfg in (1, 2):
+        kw["batch"] = small
+    elif cfg in (0, 3):
+        kw["rows"] = small
+    return [L for L in wl.config(cfg, **kw) if L.C in SHIFT_C]
+
+
+@pytest.mark.parametrize("cfg,small", [(0, None), (1, 2), (2, 1), (3, 256)])
+@pytest.mark.parametrize("bits", [4, 5, 8])
+def test_shift_quantizer_matches_oracle(cfg, small, bits):
+    """Codes, shifts, scales and zero points bit for bit (both sides decide
+    in fp32 with the same operations); the shifted grad_W operand and its
+    column sums exactly."""
+    for L in _shift_layers(cfg, small):
+        q2, _ = fqt.quantize_grad(to_dev(L.dH, L.dtype), fqt.SHIFT, bits, 0, seed=5,
+                                  with_b1=False)
+        torch.cuda.synchronize()
+        h2 = q2.to_numpy()
+        ref = orc.quantize_grad(L.dH, orc.SHIFT, bits, 0, 5, orc.STREAM_B2)
+        for key in ("codes", "inv_s", "zero", "shift"):
+            assert np.array_equal(h2[key], ref[key]), key
+        a = orc.shifted_codes(ref)
+        assert np.array_equal(q2.shift16.float().cpu().numpy().astype(np.int64), a)
+        assert np.array_equal(q2.shift_col_sum.cpu().numpy(), a.sum(axis=0))
+        assert np.array_equal(h2["row_sum"], ref["codes"].astype(np.int64).sum(1))
+        sc = q2.shift_scale.cpu().numpy()
+        assert sc[1] == 0.0
+        assert sc[0] == np.float32(ref["inv_s"][0] * np.float32(2.0 ** (int(ref["shift"][0]) - 4)))
+
+
+@pytest.mark.parametrize("cfg,small", [(0, None), (1, 2), (2, 1), (3, 256)])
+@pytest.mark.parametrize("bits", [4, 5, 8])
+def test_shift_backward_matches_oracle(cfg, small, bits):
+    """No bifurcation: the shift codes feed grad_X (as a per-row encoding)
+    and grad_W (shifted integer accumulators, Sec. 4.3)."""
+    for L in _shift_layers(cfg, small):
+        dev = lambda x: to_dev(x, L.dtype)
+        ws = fqt.Workspace(L.N, L.C, L.D)
+        qx = fqt.quantize_act(dev(L.X), 8)
+        qw = fqt.quantize_weight(dev(L.W), 8)
+        q2, q1 = fqt.quantize_grad(dev(L.dH), fqt.SHIFT, bits, 0, seed=3, with_b1=False,
+                                   ws=ws)
+        gx, gw = fqt.linear_backward(q2, None, qx, qw, ws=ws)
+        assert fqt.sync_status(ws) == 0
+        h2, hx, hw = q2.to_numpy(), qx.to_numpy(), qw.to_numpy()
+        assert grad_rel_err(gx.cpu().numpy(), orc.grad_x(h2, hw)) <= GRAD_TOL
+        ref_w = orc.grad_w_shifted(h2, hx)
+        assert grad_rel_err(gw.cpu().numpy(), ref_w) <= GRAD_TOL
+        assert np.abs(ref_w - orc.grad_w(h2, hx)).max() <= 1e-9 * np.abs(ref_w).max()
+
+
+@pytest.mark.parametrize("N,C", [(1, 64), (7, 128), (333, 256), (1000, 512), (65, 1024)])
+def test_shift_shapes_ragged_and_bf16(N, C):
+    g = wl.rng(N + C)
+    dH = wl.to_bf16_values(wl.random_grad(g, N, C, sigma=2.5, outlier_frac=0.1))
+    X = g.uniform(-1, 1, (N, 32)).astype(np.float32)
+    W = (0.05 * g.standard_normal((C, 32))).astype(np.float32)
+    qx = fqt.quantize_act(to_dev(X), 8)
+    qw = fqt.quantize_weight(to_dev(W), 8)
+    q2, _ = fqt.quantize_grad(to_dev(dH, "bf16"), fqt.SHIFT, 5, 0, seed=9, with_b1=False)
+    gx, gw = fqt.linear_backward(q2, None, qx, qw)
+    torch.cuda.synchronize()
+    h2 = q2.to_numpy()
+    ref = orc.quantize_grad(dH, orc.SHIFT, 5, 0, 9, orc.STREAM_B2)
+    assert np.array_equal(h2["codes"], ref["codes"]) and np.array_equal(h2["shift"], ref["shift"])
+    assert grad_rel_err(gx.cpu().numpy(), orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+    assert grad_rel_err(gw.cpu().numpy(), orc.grad_w_shifted(h2, qx.to_numpy())) <= GRAD_TOL
+
+
+def test_shift_with_a_bifurcated_q_b1_too():
+    """The shift kind may still emit the 8-bit PTQ Q_b1 in the same pass."""
+    L = wl.config(1, batch=2)[0]
+    q2, q1 = fqt.quantize_grad(to_dev(L.dH), fqt.SHIFT, 5, 0, seed=3, with_b1=True)
+    torch.cuda.synchronize()
+    _check_b1(q1, L.dH, 3)
