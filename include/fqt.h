@@ -113,6 +113,10 @@ typedef struct fqt_qtensor {
   int32_t *shift_col_sum; /* FQT_SHIFT: cols entries, sum_i a_ic */
   float *shift_scale; /* FQT_SHIFT: 2 entries, the common scale 2^-4 / s of a
                         and 0 (its zero point) */
+  int32_t conv[8];   /* written by fqt_quantize_act_conv: {n, h, w, c, kh, kw,
+                        pad, 0}, the geometry of an implicit im2col operand;
+                        all zero for an ordinary matrix (the other quantize
+                        calls clear it) */
 } fqt_qtensor;
 
 /* Bytes of workspace a layer with dH N x C, X N x D, W C x D needs for any
@@ -129,6 +133,28 @@ FQT_API size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D);
 FQT_API fqt_status fqt_quantize_act(const void *X, fqt_dtype dtype, int64_t rows,
                             int64_t cols, int bits, fqt_qtensor *out,
                             void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Q_f of a stride-1 convolution's input without forming its im2col matrix:
+ * X is an NHWC tensor n x h x w x c (fp32 or bf16); the quantized operand is
+ * the im2col matrix of kh x kw taps with `pad` zeros on every side
+ * (rows = n oh ow output pixels, oh = h + 2 pad - kh + 1, ow likewise;
+ * cols = kh kw c, tap-major then channel), exactly the codes that
+ * fqt_quantize_act gives for that matrix: z = min and s = B / R over X and,
+ * when pad > 0, the padding zeros (Sec. 2.1, App. E).  Storage is NHWC:
+ * out->codes_f16 (n h w x c) holds code - code(0.0), so that a zero carrier
+ * encodes the padding; out->codes (optional) the codes; inv_s[0], zero[0];
+ * out->col_sum (required, kh kw c + 1 entries) the column sums of the
+ * im2col matrix followed by code(0.0); out->conv the geometry.  row_sum must
+ * be NULL.  c % 8 == 0, c <= 4096.  The workspace holds the status word and range
+ * partials only (fqt_workspace_size(n h w, c, 16) bytes suffice).
+ * fqt_linear_backward reads such an operand as qx for grad_W (stride 1,
+ * c % 64 == 0, ow % 32 == 0).
+ */
+FQT_API fqt_status fqt_quantize_act_conv(const void *X, fqt_dtype dtype, int64_t n, int64_t h,
+                                         int64_t w, int64_t c, int kh, int kw, int pad,
+                                         int bits, fqt_qtensor *out, void *workspace,
+                                         size_t ws_bytes, void *stream);
 
 /* The same quantizer for the weight, Q_theta of Eq. 3 (W: C x D). */
 FQT_API fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t rows,

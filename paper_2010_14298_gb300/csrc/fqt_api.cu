@@ -58,6 +58,7 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
   out->bits = bits;
   out->kind = FQT_PTQ;
   out->block = 0;
+  memset(out->conv, 0, sizeof(out->conv));
   if (rows == 0) return FQT_OK;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int nsm = device_sm_count();
@@ -97,11 +98,65 @@ static fqt_status quantize_forward(const void *X, fqt_dtype dtype, int64_t rows,
   return cuda_fail(e, "quantizer launch");
 }
 
+// Q_f of a stride-1 conv input as its implicit im2col matrix (see fqt.h).
+static fqt_status quantize_conv(const void *X, fqt_dtype dtype, int64_t n, int64_t h,
+                                int64_t wd, int64_t c, int kh, int kw, int pad, int bits,
+                                fqt_qtensor *out, void *ws, size_t ws_bytes, void *stream) {
+  if (!out || bits < 2 || bits > 8 || n < 0 || h <= 0 || wd <= 0 || c <= 0 || kh <= 0 ||
+      kw <= 0 || pad < 0)
+    return FQT_EINVAL;
+  const int64_t oh = h + 2 * pad - kh + 1, ow = wd + 2 * pad - kw + 1;
+  if (oh <= 0 || ow <= 0 || h > (1 << 16) || wd > (1 << 16) || c > (1 << 16)) return FQT_EINVAL;
+  if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
+  if (n > 0 && (!X || !out->codes_f16 || !out->inv_s || !out->zero || !out->col_sum))
+    return FQT_EINVAL;
+  if (out->row_sum) return FQT_EUNSUPPORTED;  // row sums of the im2col rows: not built
+  if (c % 8 || c > 4096) return FQT_EUNSUPPORTED;  // column sums stage c ints in shared memory
+  if (!aligned(X, 16) || !aligned(out->codes, 16) || !aligned(out->codes_f16, 16))
+    return FQT_EINVAL;
+  const int64_t pixels = n * h * wd;
+  fqt_status s = check_ws(ws, ws_bytes, kGemmOffset);
+  if (s != FQT_OK) return s;
+  out->rows = n * oh * ow;
+  out->cols = (int64_t)kh * kw * c;
+  out->bits = bits;
+  out->kind = FQT_PTQ;
+  out->block = 0;
+  const int32_t geo[7] = {(int32_t)n, (int32_t)h, (int32_t)wd, (int32_t)c, kh, kw, pad};
+  memcpy(out->conv, geo, sizeof(geo));
+  out->conv[7] = 0;
+  if (n == 0) return FQT_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int nsm = device_sm_count();
+  char *w = static_cast<char *>(ws);
+  float2 *part = reinterpret_cast<float2 *>(w + kRangeOffset);
+  int npart = 0;
+  cudaError_t e = launch_range(X, dtype == FQT_BF16, pixels * c, part, &npart, out->col_sum,
+                               (int64_t)kh * kw * c, nullptr, 0, nsm, st);
+  if (e != cudaSuccess) return cuda_fail(e, "range pass");
+  // code(0.0), the carriers' centre, follows the column sums (device memory)
+  int32_t *zc = out->col_sum + (int64_t)kh * kw * c;
+  s = launch_fwd_codes(X, dtype == FQT_BF16, pixels, (int)c, bits, out->codes_f16, out->codes,
+                       nullptr, part, npart, out->inv_s, out->zero, reinterpret_cast<int *>(w),
+                       nsm, st, pad > 0 ? 1 : 0, zc);
+  if (s != FQT_OK) return s;
+  return launch_conv_colsum(out->codes_f16, n, (int)h, (int)wd, (int)c, kh, kw, pad,
+                            out->col_sum, st);
+}
+
 }  // namespace fqt
 
 using namespace fqt;
 
 extern "C" {
+
+fqt_status fqt_quantize_act_conv(const void *X, fqt_dtype dtype, int64_t n, int64_t h,
+                                 int64_t w, int64_t c, int kh, int kw, int pad, int bits,
+                                 fqt_qtensor *out, void *workspace, size_t ws_bytes,
+                                 void *stream) {
+  return quantize_conv(X, dtype, n, h, w, c, kh, kw, pad, bits, out, workspace, ws_bytes,
+                       stream);
+}
 
 size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
   size_t need = gemm_workspace_bytes(N, C, D);

@@ -117,6 +117,17 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map,
       : "memory");
 }
 
+__device__ __forceinline__ void tma_load_4d(void *dst, const CUtensorMap *map, int32_t c0,
+                                            int32_t c1, int32_t c2, int32_t c3,
+                                            uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3),
+      "r"(smem_u32(bar))
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int32_t c0,
                                              int32_t c1, const void *src) {
   asm volatile(
@@ -1358,6 +1369,7 @@ struct ReduceArgs {
   // grad_W = inv_s1 inv_sx sum_n (a_nc + z'_1)(x_nd + z'_x)
   int64_t Kn;        // rows N of dH / X
   int oa, ob;
+  const int32_t *ob_dev;       // if set, ob is read here (a conv operand's code(0.0))
   const int32_t *cs_a, *cs_b;  // column sums of Q_b1 codes (M) and X~ codes (N)
   const float *inv_a, *zero_a, *inv_b, *zero_b;
 };
@@ -1399,10 +1411,11 @@ __global__ void __launch_bounds__(kRedElems * kRedGroups) k_reduce(const ReduceA
         const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
         const float da = za + (float)ma, db = zb + (float)mb;
         const int64_t ca = r.cs_a[c], cb = r.cs_b[d];
+        const int64_t ob = r.ob_dev ? (int64_t)*r.ob_dev : (int64_t)r.ob;
         // I = sum (a - ma)(b - mb), exact, from the centred product P
-        const int64_t I = P + (r.oa - ma) * (cb - r.Kn * r.ob) +
-                          (r.ob - mb) * (ca - r.Kn * r.oa) +
-                          r.Kn * (r.oa - ma) * (r.ob - mb);
+        const int64_t I = P + (r.oa - ma) * (cb - r.Kn * ob) +
+                          (ob - mb) * (ca - r.Kn * r.oa) +
+                          r.Kn * (r.oa - ma) * (ob - mb);
         const float V = (float)I + db * (float)(ca - r.Kn * ma) +
                         da * (float)(cb - r.Kn * mb) + (float)r.Kn * da * db;
         r.out_f32[idx] = (*r.inv_a) * (*r.inv_b) * V;
@@ -1715,6 +1728,9 @@ struct WArgs {
   int stages;
   int32_t *part;      // [splits][C][D]
   int *status;
+  // implicit im2col operand (stride 1): X~ is read as 4-D boxes of an NHWC
+  // tensor at shifted pixel coordinates; padding comes back as zero carriers
+  int conv, ih, iw, oh, ow, cin, kw, pad, taps;
 };
 
 __host__ __device__ constexpr uint32_t make_idesc_mn_n(int n) {
@@ -1783,9 +1799,28 @@ __global__ void __launch_bounds__(kWThreads, 1)
           uint8_t *sx = ops + (size_t)s * stage_bytes;
           uint8_t *sq = sx + xbytes;
           const int32_t kc = (int32_t)(kb * kWBK);
-          for (int m = 0; m < w.mt; ++m) {
-            tma_load_2d(sx + (size_t)m * 2 * kWBox, &tmX, m * 128, kc, &full[s]);
-            tma_load_2d(sx + (size_t)m * 2 * kWBox + kWBox, &tmX, m * 128 + 64, kc, &full[s]);
+          if (w.conv) {
+            // 32 output pixels of one output row (ow % 32 == 0); box (64 channels
+            // of one tap) x 32 pixels read at the tap's offset
+            const int64_t p0 = kb * kWBK;
+            const int ox0 = (int)(p0 % w.ow);
+            const int64_t t = p0 / w.ow;
+            const int oy = (int)(t % w.oh), nimg = (int)(t / w.oh);
+            for (int m = 0; m < 2 * w.mt; ++m) {
+              const int d0 = m * 64, tap = d0 / w.cin, cg = d0 - tap * w.cin;
+              uint8_t *dst = sx + (size_t)m * kWBox;
+              if (tap < w.taps) {
+                const int ky = tap / w.kw, kx = tap - ky * w.kw;
+                tma_load_4d(dst, &tmX, cg, ox0 + kx - w.pad, oy + ky - w.pad, nimg, &full[s]);
+              } else {  // past the last tap: a box outside the tensor (zeros)
+                tma_load_4d(dst, &tmX, 0, 0, w.ih + 8, nimg, &full[s]);
+              }
+            }
+          } else {
+            for (int m = 0; m < w.mt; ++m) {
+              tma_load_2d(sx + (size_t)m * 2 * kWBox, &tmX, m * 128, kc, &full[s]);
+              tma_load_2d(sx + (size_t)m * 2 * kWBox + kWBox, &tmX, m * 128 + 64, kc, &full[s]);
+            }
           }
           for (int cb = 0; cb < w.ncb; ++cb)
             tma_load_2d(sq + (size_t)cb * kWBox, &tmQ, cb * 64, kc, &full[s]);
@@ -1898,10 +1933,29 @@ static WPlan gradw_plan(int64_t K, int64_t C, int64_t D, int b1, int bx, int num
   return p;
 }
 
+// 4-D map of NHWC fp16 carriers (c, w, h, n), boxes of 64 channels x 32
+// pixels of one image row, 128-byte swizzle: the same shared-memory image as
+// a 64 x 32 box of the im2col matrix.
+static bool make_map_f16_nhwc(CUtensorMap *m, const void *base, uint64_t n, uint64_t h,
+                              uint64_t w, uint64_t c) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {c, w, h, n};
+  cuuint64_t strides[3] = {c * 2, w * c * 2, h * w * c * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)kWBK, 1, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(base), dims, strides,
+            box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 static fqt_status run_gradw(const uint16_t *X16, const uint16_t *Q16, int64_t K, int C, int D,
-                            const WPlan &p, int32_t *part, int *status, cudaStream_t st) {
+                            const WPlan &p, int32_t *part, int *status, cudaStream_t st,
+                            const int32_t *conv = nullptr) {
   CUtensorMap tx, tq;
-  bool ok = make_map_f16(&tx, X16, (uint64_t)D, (uint64_t)K, 64, kWBK);
+  bool ok = conv ? make_map_f16_nhwc(&tx, X16, (uint64_t)conv[0], (uint64_t)conv[1],
+                                     (uint64_t)conv[2], (uint64_t)conv[3])
+                 : make_map_f16(&tx, X16, (uint64_t)D, (uint64_t)K, 64, kWBK);
   ok = ok && make_map_f16(&tq, Q16, (uint64_t)C, (uint64_t)K, 64, kWBK);
   if (!ok) return cuda_fail(cudaErrorInvalidValue, "tensor map encode");
   WArgs w;
@@ -1918,6 +1972,17 @@ static fqt_status run_gradw(const uint16_t *X16, const uint16_t *Q16, int64_t K,
   w.stages = p.stages;
   w.part = part;
   w.status = status;
+  if (conv) {
+    w.conv = 1;
+    w.ih = conv[1];
+    w.iw = conv[2];
+    w.cin = conv[3];
+    w.kw = conv[5];
+    w.pad = conv[6];
+    w.oh = conv[1] + 2 * conv[6] - conv[4] + 1;
+    w.ow = conv[2] + 2 * conv[6] - conv[5] + 1;
+    w.taps = conv[4] * conv[5];
+  }
   const cudaError_t ea =
       cudaFuncSetAttribute(k_gradw, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
   if (ea != cudaSuccess) return cuda_fail(ea, "grad_W shared-memory attribute");
@@ -2399,19 +2464,31 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     const uint16_t *A16 = shifted ? qa->shift_f16 : qa->codes_f16;
     // |shifted code| <= 16 (2^(b-1) - 1) < 2^(b+3): b + 4 bits of centred magnitude
     const int a_bits = shifted ? qa->bits + 4 : qa->bits;
+    // an implicit im2col operand: carriers centred at code(0.0), |.| < 2^b
+    const bool conv = qx->conv[0] > 0;
+    const int x_bits = conv ? qx->bits + 1 : qx->bits;
     const int64_t Nr = qa->rows, C = qa->cols, D = qx->cols;
     if (qx->rows != Nr) return FQT_EINVAL;
     if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
     if (!aligned16(A16) || !aligned16(qx->codes_f16)) return FQT_EINVAL;
-    const SplitPlan p = plan_splits(C, D, Nr, a_bits, qx->bits, nsm, true);
-    const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, a_bits, qx->bits, nsm) : WPlan{};
+    if (conv) {
+      const int32_t *g = qx->conv;
+      const int64_t oh = (int64_t)g[1] + 2 * g[6] - g[4] + 1, ow = (int64_t)g[2] + 2 * g[6] - g[5] + 1;
+      if (oh <= 0 || ow <= 0 || (int64_t)g[0] * oh * ow != Nr || (int64_t)g[4] * g[5] * g[3] != D)
+        return FQT_EINVAL;
+      if (g[3] % 64 || ow % kWBK) return FQT_EUNSUPPORTED;
+    }
+    const SplitPlan p = plan_splits(C, D, Nr, a_bits, x_bits, nsm, true);
+    const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, a_bits, x_bits, nsm) : WPlan{};
     const bool w_ok = use_gradw(wp, nsm);
+    if (conv && Nr > 0 && !w_ok) return FQT_EUNSUPPORTED;  // the tile kernel reads plain matrices
     const int splits = w_ok ? wp.splits : p.splits;
     const size_t need = kGemmOffset + (size_t)splits * (size_t)C * (size_t)D * 4;
     if (ws_bytes < need) return FQT_EWORKSPACE;
     int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kGemmOffset);
     if (Nr > 0 && w_ok) {
-      fqt_status s = run_gradw(qx->codes_f16, A16, Nr, (int)C, (int)D, wp, part, status, st);
+      fqt_status s = run_gradw(qx->codes_f16, A16, Nr, (int)C, (int)D, wp, part, status, st,
+                               conv ? qx->conv : nullptr);
       if (s != FQT_OK) return s;
     } else if (Nr > 0) {
       GemmArgs g;
@@ -2437,6 +2514,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     r.ob = 1 << (qx->bits - 1);
     r.cs_a = shifted ? qa->shift_col_sum : qa->col_sum;
     r.cs_b = qx->col_sum;
+    r.ob_dev = conv ? qx->col_sum + D : nullptr;
     r.inv_a = shifted ? qa->shift_scale : qa->inv_s;
     r.zero_a = shifted ? qa->shift_scale + 1 : qa->zero;
     r.inv_b = qx->inv_s;

@@ -1474,7 +1474,8 @@ __global__ void __launch_bounds__(kFwdMaxThreads)
     k_fwd_codes(const T *__restrict__ X, int64_t rows, int cols, int rpi,
                 uint16_t *__restrict__ f16, uint8_t *__restrict__ c8,
                 int32_t *__restrict__ col_sum, const float2 *__restrict__ part, int npart,
-                float *inv_out, float *zero_out, int bits, int *status) {
+                float *inv_out, float *zero_out, int bits, int *status, int conv_zero,
+                int32_t *code_zero_out) {
   extern __shared__ int csum_s[];  // cols
   __shared__ float2 red[kFwdMaxThreads / 32];
   __shared__ int redi[kFwdMaxThreads / 32];
@@ -1512,10 +1513,22 @@ __global__ void __launch_bounds__(kFwdMaxThreads)
     return;
   }
   const uint32_t B = (1u << bits) - 1u;
+  if (conv_zero) {  // the im2col matrix also holds the padding zeros
+    gmin = fminf(gmin, 0.0f);
+    gmax = fmaxf(gmax, 0.0f);
+  }
   const float s = affine_scale(gmin, gmax, B), z = gmin;
+  // carriers are centred at 2^(b-1), or at the code of 0.0 for a conv operand
+  // whose padding the loads fill with zero carriers
+  uint32_t off = (B + 1u) >> 1;
+  if (conv_zero) {
+    const float v0 = __fmul_rn(__fsub_rn(0.0f, z), s);
+    off = min(__float_as_uint(__fadd_rn(v0, 12582912.0f)) - 0x4B400000u, B);
+  }
   if (blockIdx.x == 0 && tid == 0) {
     inv_out[0] = __fdiv_rn(1.0f, s);
     zero_out[0] = __fmul_rn(s, z);
+    if (code_zero_out) *code_zero_out = (int32_t)off;
   }
   const int opr = cols / 8;
   const int rl = tid / opr, o = tid - rl * opr;
@@ -1524,7 +1537,6 @@ __global__ void __launch_bounds__(kFwdMaxThreads)
 #pragma unroll
   for (int j = 0; j < 8; ++j) cs[j] = 0;
   const int64_t groups = (rows + rpi - 1) / rpi;
-  const uint32_t off = (B + 1u) >> 1;
   for (int64_t i0 = blockIdx.x; i0 < groups; i0 += (int64_t)kFwdUnroll * gridDim.x) {
     float x[kFwdUnroll][8];
     int64_t row[kFwdUnroll];
@@ -1567,7 +1579,8 @@ __global__ void __launch_bounds__(kFwdMaxThreads)
 fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, int bits,
                             uint16_t *f16, uint8_t *c8, int32_t *col_sum, const float2 *part,
                             int npart, float *inv_out, float *zero_out, int *status,
-                            int num_sms, cudaStream_t st) {
+                            int num_sms, cudaStream_t st, int conv_zero,
+                            int32_t *code_zero_out) {
   const int opr = cols / 8;
   if (cols % 8 || opr > kFwdMaxThreads) return FQT_EUNSUPPORTED;
   int rpi = 512 / opr;  // about 512 threads: two CTAs per SM
@@ -1582,12 +1595,78 @@ fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, in
   if (bf16)
     k_fwd_codes<__nv_bfloat16><<<(int)grid, nth, smem, st>>>(
         reinterpret_cast<const __nv_bfloat16 *>(X), rows, cols, rpi, f16, c8, col_sum, part,
-        npart, inv_out, zero_out, bits, status);
+        npart, inv_out, zero_out, bits, status, conv_zero, code_zero_out);
   else
     k_fwd_codes<float><<<(int)grid, nth, smem, st>>>(
         reinterpret_cast<const float *>(X), rows, cols, rpi, f16, c8, col_sum, part, npart,
-        inv_out, zero_out, bits, status);
+        inv_out, zero_out, bits, status, conv_zero, code_zero_out);
   return cuda_fail(cudaGetLastError(), "forward codes launch");
+}
+
+// ---------------------------------------------------------------------------
+// Column sums of the implicit im2col matrix of a conv operand (stride 1):
+// im2col column (ky, kx, ch) holds, for every output pixel (n, oy, ox), the
+// code of input pixel (oy + ky - pad, ox + kx - pad) or the code of 0.0 in
+// the padding.  With carriers a = code - code(0) (zero in the padding), the
+// sum is rows code(0) + the carriers over the input rectangle that tap
+// (ky, kx) reads.  One CTA per (tap, image) sums its rectangle (the carriers
+// are in L2 after the codes pass) and adds into the column sums, which the
+// range pass cleared; code(0) sits after them.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_conv_colsum(const uint16_t *__restrict__ f16, int h,
+                                                     int w, int c, int kh, int kw, int pad,
+                                                     int oh, int ow, int64_t rows,
+                                                     int32_t *col_sum) {
+  extern __shared__ int acc_s[];  // c
+  const int taps = kh * kw;
+  const int tap = (int)(blockIdx.x % taps);
+  const int64_t img = blockIdx.x / taps;
+  const int ky = tap / kw, kx = tap - ky * kw;
+  const int y0 = max(0, ky - pad), y1 = min(h, ky - pad + oh);
+  const int x0 = max(0, kx - pad), x1 = min(w, kx - pad + ow);
+  const int octs = c / 8;
+  for (int i = threadIdx.x; i < c; i += blockDim.x) acc_s[i] = 0;
+  __syncthreads();
+  const int lanes = blockDim.x >= octs ? blockDim.x / octs : 1;
+  const int rw = x1 - x0, npix = (y1 > y0 && rw > 0) ? (y1 - y0) * rw : 0;
+  for (int oc = threadIdx.x % octs; oc < octs; oc += blockDim.x) {
+    const int pl = blockDim.x >= octs ? (int)threadIdx.x / octs : 0;
+    if (pl >= lanes) continue;
+    int a8[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int p = pl; p < npix; p += lanes) {
+      const int y = y0 + p / rw, x = x0 + p % rw;
+      const uint4 v = __ldg(reinterpret_cast<const uint4 *>(
+          f16 + ((img * h + y) * (int64_t)w + x) * c + oc * 8));
+      const uint32_t wds[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const __half2 hh = *reinterpret_cast<const __half2 *>(&wds[q]);
+        const float2 f = __half22float2(hh);
+        a8[2 * q] += (int)f.x;
+        a8[2 * q + 1] += (int)f.y;
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      if (a8[j]) atomicAdd(&acc_s[oc * 8 + j], a8[j]);
+  }
+  __syncthreads();
+  const int zc = col_sum[(int64_t)taps * c];
+  for (int i = threadIdx.x; i < c; i += blockDim.x) {
+    const int v = acc_s[i] + (img == 0 ? (int)(rows * (int64_t)zc) : 0);
+    if (v) atomicAdd(&col_sum[(int64_t)tap * c + i], v);
+  }
+}
+
+fqt_status launch_conv_colsum(const uint16_t *f16, int64_t n, int h, int w, int c, int kh,
+                              int kw, int pad, int32_t *col_sum, cudaStream_t st) {
+  const int oh = h + 2 * pad - kh + 1, ow = w + 2 * pad - kw + 1;
+  const int64_t grid = n * kh * kw;
+  if (grid <= 0) return FQT_OK;
+  if (grid > 0x7fffffff) return FQT_EUNSUPPORTED;
+  k_conv_colsum<<<(int)grid, 256, sizeof(int) * (size_t)c, st>>>(f16, h, w, c, kh, kw, pad, oh,
+                                                                 ow, n * oh * ow, col_sum);
+  return cuda_fail(cudaGetLastError(), "conv column sums launch");
 }
 
 // ---------------------------------------------------------------------------

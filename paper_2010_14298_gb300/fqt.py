@@ -43,7 +43,8 @@ class _QT(ctypes.Structure):
                 ("hr", ctypes.c_void_p), ("perm", ctypes.c_void_p),
                 ("gstart", ctypes.c_void_p), ("gsize", ctypes.c_void_p),
                 ("shift_f16", ctypes.c_void_p), ("shift", ctypes.c_void_p),
-                ("shift_col_sum", ctypes.c_void_p), ("shift_scale", ctypes.c_void_p)]
+                ("shift_col_sum", ctypes.c_void_p), ("shift_scale", ctypes.c_void_p),
+                ("conv", ctypes.c_int32 * 8)]
 
 
 def library_path() -> str:
@@ -79,6 +80,10 @@ def load(build_if_missing: bool = True):
         lib.fqt_linear_backward.argtypes = [QP, QP, QP, QP, P, P, P, sz, P]
         lib.fqt_linear_backward.restype = i32
         lib.fqt_linear_forward.argtypes = [QP, QP, P, P, sz, P]
+        lib.fqt_linear_forward.restype = i32
+        lib.fqt_quantize_act_conv.argtypes = [P, i32, i64, i64, i64, i64, i32, i32, i32, i32,
+                                              QP, P, sz, P]
+        lib.fqt_quantize_act_conv.restype = i32
         lib.fqt_linear_forward.restype = i32
         lib.fqt_grad_w_fixed_scratch.argtypes = [QP, QP, P, P]
         lib.fqt_grad_w_fixed_scratch.restype = i32
@@ -173,9 +178,13 @@ class QTensor:
     shift: Optional[torch.Tensor] = None
     shift_col_sum: Optional[torch.Tensor] = None
     shift_scale: Optional[torch.Tensor] = None
+    conv: Optional[tuple] = None   # implicit im2col operand: (n, h, w, c, kh, kw, pad, 0)
+    logical: Optional[tuple] = None  # (rows, cols) of that im2col matrix
 
     @property
     def shape(self):
+        if self.logical is not None:
+            return self.logical
         return (self.codes if self.codes is not None else self.codes16).shape
 
     @staticmethod
@@ -221,7 +230,8 @@ class QTensor:
                    p(self.codes), self.inv_s.data_ptr(), self.zero.data_ptr(),
                    p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16),
                    p(self.hz), p(self.hr), p(self.perm), p(self.gstart), p(self.gsize),
-                   p(self.shift16), p(self.shift), p(self.shift_col_sum), p(self.shift_scale))
+                   p(self.shift16), p(self.shift), p(self.shift_col_sum), p(self.shift_scale),
+                   (ctypes.c_int32 * 8)(*(self.conv or (0,) * 8)))
 
     def codes_from_f16(self) -> torch.Tensor:
         """The uint8 codes recovered from the fp16 carriers."""
@@ -274,6 +284,37 @@ def quantize_act(X: torch.Tensor, bits: int = 8, ws: Workspace = None,
     ws = ws or Workspace(*X.shape, 16, device=X.device)
     return _fwd("fqt_quantize_act", X.contiguous(), bits, ws, out, row_sum,
                 col_sum, stream)
+
+
+def quantize_act_conv(X: torch.Tensor, kh: int, kw: int, pad: int, bits: int = 8,
+                      ws: Workspace = None, out: QTensor = None, u8: bool = False,
+                      stream=None) -> QTensor:
+    """X~ = Q_f(im2col(X)) for a stride-1 convolution, without forming the
+    im2col matrix (Sec. 2.1, App. E): X is NHWC; the codes are stored NHWC,
+    centred at the code of 0.0 (fqt_quantize_act_conv)."""
+    lib = load()
+    X = X.contiguous()
+    n, h, w, c = X.shape
+    oh, ow = h + 2 * pad - kh + 1, w + 2 * pad - kw + 1
+    dev = X.device
+    ws = ws or Workspace(n * h * w, c, 16, device=dev)
+    if out is None:
+        out = QTensor(
+            codes=(torch.empty((n * h * w, c), dtype=torch.uint8, device=dev) if u8 else None),
+            codes16=torch.empty((n * h * w, c), dtype=torch.float16, device=dev),
+            inv_s=torch.empty(1, dtype=torch.float32, device=dev),
+            zero=torch.empty(1, dtype=torch.float32, device=dev),
+            row_sum=None,
+            col_sum=torch.empty(kh * kw * c + 1, dtype=torch.int32, device=dev),
+            lead=None)
+    out.logical = (n * oh * ow, kh * kw * c)
+    qs = out.c_struct()
+    st = lib.fqt_quantize_act_conv(_ptr(X), _dtype_code(X), n, h, w, c, kh, kw, pad, bits,
+                                   ctypes.byref(qs), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "fqt_quantize_act_conv")
+    out.kind, out.bits, out.block = PTQ, bits, 0
+    out.conv = tuple(qs.conv)
+    return out
 
 
 def quantize_weight(W: torch.Tensor, bits: int = 8, ws: Workspace = None,

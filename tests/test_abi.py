@@ -19,6 +19,7 @@ def test_header_declares_the_boundary():
     names = set(declared_symbols())
     for required in ("fqt_quantize_act", "fqt_quantize_weight",
                      "fqt_quantize_grad", "fqt_linear_backward", "fqt_linear_forward",
+                     "fqt_quantize_act_conv",
                      "fqt_workspace_size", "fqt_sync_status",
                      "fqt_status_string", "fqt_debug_int_gemm"):
         assert required in names

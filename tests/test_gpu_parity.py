@@ -597,3 +597,69 @@ def test_shift_with_a_bifurcated_q_b1_too():
     q2, q1 = fqt.quantize_grad(to_dev(L.dH), fqt.SHIFT, 5, 0, seed=3, with_b1=True)
     torch.cuda.synchronize()
     _check_b1(q1, L.dH, 3)
+
+
+# --------------------------------------------------------------------------
+# Implicit im2col operand (NEXT n3, the X~ side): NHWC codes, shifted loads
+# --------------------------------------------------------------------------
+def _conv_codes_as_im2col(q, x_shape, kh, kw, pad):
+    """The im2col matrix of the GPU's NHWC codes (padding = code of 0.0)."""
+    n, h, w, c = x_shape
+    zc = int(q.col_sum[-1].item())
+    nhwc = (q.codes16.float().cpu().numpy().astype(np.int64) + zc).reshape(n, h, w, c)
+    full = np.full((n, h + 2 * pad, w + 2 * pad, c), zc, dtype=np.int64)
+    full[:, pad:pad + h, pad:pad + w] = nhwc
+    oh, ow = h + 2 * pad - kh + 1, w + 2 * pad - kw + 1
+    cols = np.empty((n, oh, ow, kh, kw, c), dtype=np.int64)
+    for i in range(kh):
+        for j in range(kw):
+            cols[:, :, :, i, j, :] = full[:, i:i + oh, j:j + ow, :]
+    return cols.reshape(n * oh * ow, kh * kw * c), zc
+
+
+@pytest.mark.parametrize("n,h,w,c,pad,dtype", [(2, 32, 32, 64, 1, "f32"), (1, 32, 32, 128, 1, "bf16"),
+                                               (3, 8, 12, 16, 1, "f32"), (2, 9, 9, 64, 0, "f32")])
+def test_conv_quantizer_equals_the_im2col_quantizer(n, h, w, c, pad, dtype):
+    g = wl.rng(n * h + c + pad)
+    x = g.uniform(-1, 1, (n, h, w, c)).astype(np.float32)
+    x[0, 0, 0, :4] = 3.0  # the range is not symmetric
+    if dtype == "bf16":
+        x = wl.to_bf16_values(x)
+    xi = wl.im2col_nhwc(x, 3, 3, 1, pad)
+    ref = orc.quantize_fwd(xi, 8)
+    q = fqt.quantize_act_conv(to_dev(x, dtype), 3, 3, pad, 8)
+    torch.cuda.synchronize()
+    assert q.shape == xi.shape
+    got, zc = _conv_codes_as_im2col(q, x.shape, 3, 3, pad)
+    assert np.array_equal(got, ref["codes"].astype(np.int64))
+    assert np.array_equal(q.inv_s.cpu().numpy(), ref["inv_s"])
+    assert np.array_equal(q.zero.cpu().numpy(), ref["zero"])
+    assert np.array_equal(q.col_sum[:-1].cpu().numpy(), ref["codes"].astype(np.int64).sum(0))
+
+
+@pytest.mark.parametrize("batch", [2, 128])
+def test_conv_grad_w_equals_the_explicit_path(batch):
+    """grad_W with X~ read as shifted NHWC boxes equals grad_W over the
+    materialized im2col codes bit for bit (the contraction is exact), and the
+    oracle within the tolerance (sampled columns at batch 128)."""
+    g = wl.rng(400 + batch)
+    x = g.uniform(-1, 1, (batch, 32, 32, 64)).astype(np.float32)
+    xi = wl.im2col_nhwc(x, 3, 3, 1, 1)
+    N = xi.shape[0]
+    dH = g.standard_normal((N, 64)).astype(np.float32)
+    dH[g.random(N) < 0.01] *= 100.0
+    W = (np.sqrt(2.0 / 576) * g.standard_normal((64, 576))).astype(np.float32)
+    qw = fqt.quantize_weight(to_dev(W), 8)
+    q2, q1 = fqt.quantize_grad(to_dev(dH), orc.BHQ, 5, 16, seed=3)
+    ws = fqt.Workspace(N, 64, 576)
+    qx = fqt.quantize_act(to_dev(xi), 8)
+    qc = fqt.quantize_act_conv(to_dev(x), 3, 3, 1, 8)
+    _, gw = fqt.linear_backward(q2, q1, qx, qw, grad_x=False, ws=ws)
+    _, gwc = fqt.linear_backward(q2, q1, qc, qw, grad_x=False, ws=ws)
+    assert fqt.sync_status(ws) == 0
+    gw, gwc = gw.cpu().numpy(), gwc.cpu().numpy()
+    assert np.array_equal(gw, gwc)
+    h1, hx = q1.to_numpy(), qx.to_numpy()
+    cols = np.arange(576) if batch == 2 else np.sort(wl.rng(5).choice(576, 48, replace=False))
+    ref = orc.matmul(orc.dequant(h1), orc.dequant(hx)[:, cols], a_trans=True)
+    assert grad_rel_err(gwc[:, cols], ref) <= GRAD_TOL
