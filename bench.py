@@ -449,6 +449,59 @@ def run_gpu(args):
                "launches": {"quantize_grad": 2, "grad_x": 1, "grad_w": 2},
                "device_status": fqt.sync_status(ws)}
 
+    # ---- the same step with X~ as an implicit im2col operand: the forward
+    # PTQ reads the NHWC input once (the im2col matrix is never formed) and
+    # grad_W reads its boxes at shifted pixel coordinates; codes and grad_W
+    # are bit-identical to the explicit path ----
+    imp = None
+    if args.implicit_steps > 0 and L.x_nhwc is not None:
+        xn = torch.from_numpy(L.x_nhwc).to(dev)
+        nb, hh, ww, cc = L.x_nhwc.shape
+        qc = None
+
+        def qconv():
+            nonlocal qc
+            qc = fqt.quantize_act_conv(xn, 3, 3, 1, 8, ws=ws_fx, out=qc)
+        qconv()
+        fi = [qconv,
+              lambda: fqt.quantize_weight(W, 8, ws=ws_fw, out=qw),
+              lambda: fqt.quantize_grad(dH, KIND, BITS, BLOCK, 1000, ws=ws, q_b2=q2, q_b1=q1),
+              lambda: fqt.linear_backward(q2, q1, qx, qw, grad_x=True, grad_w=False, ws=ws,
+                                          out_x=gx),
+              lambda: fqt.linear_backward(q2, q1, qc, qw, grad_x=False, grad_w=True, ws=ws,
+                                          out_w=gw)]
+        for _ in range(3):
+            for f in fi:
+                f()
+        torch.cuda.synchronize()
+        gi = []
+        for f in fi:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                f()
+            gi.append(g)
+        ti = [[] for _ in fi]
+        for i in range(args.implicit_steps):
+            flush.fill_(i & 0xFF)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(fi) + 1)]
+            for k in range(len(fi)):
+                ev[k].record(stream)
+                gi[k].replay()
+            ev[-1].record(stream)
+            torch.cuda.synchronize()
+            for k in range(len(fi)):
+                ti[k].append(ev[k].elapsed_time(ev[k + 1]))
+        per = [float(np.median(t)) for t in ti]
+        ms_imp = sum(per)
+        imp = {"x_input": f"NHWC {nb}x{hh}x{ww}x{cc}, 3x3 taps, pad 1, stride 1",
+               "per_call_ms": dict(zip(["quantize_act_conv", "quantize_weight", "quantize_grad",
+                                        "grad_x", "grad_w"], per)),
+               "ms_per_step": ms_imp,
+               "TOPS": ops_step / (ms_imp * 1e-3) / 1e12,
+               "explicit_ms": {"quantize_act": float(per_call[0]), "grad_w": float(per_call[4])},
+               "launches_per_step": 10,
+               "device_status": fqt.sync_status(ws)}
+
     result = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -475,6 +528,7 @@ def run_gpu(args):
         "forward": fwd,
         "adaptive_bhq": ada,
         "shift_quantizer": shf,
+        "implicit_im2col": imp,
         "gpu_launches": int(sum(launches_per_call) * args.steps),
         "device_status": status,
     }
@@ -557,6 +611,8 @@ def main():
                     help="timed steps of the adaptive BHQ groups (0: skip)")
     ap.add_argument("--shift-steps", type=int, default=50,
                     help="timed steps of the shift quantizer path (0: skip)")
+    ap.add_argument("--implicit-steps", type=int, default=50,
+                    help="timed steps with the implicit im2col X operand (0: skip)")
     ap.add_argument("--eager", action="store_true",
                     help="time the C-ABI calls directly instead of graph replays")
     args = ap.parse_args()

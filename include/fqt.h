@@ -142,8 +142,8 @@ FQT_API fqt_status fqt_quantize_act(const void *X, fqt_dtype dtype, int64_t rows
  * cols = kh kw c, tap-major then channel), exactly the codes that
  * fqt_quantize_act gives for that matrix: z = min and s = B / R over X and,
  * when pad > 0, the padding zeros (Sec. 2.1, App. E).  Storage is NHWC:
- * out->codes_f16 (n h w x c) holds code - code(0.0), so that a zero carrier
- * encodes the padding; out->codes (optional) the codes; inv_s[0], zero[0];
+ * out->codes_f16 (n h w x c) holds code - 2^(b-1) as for any operand;
+ * out->codes (optional) the codes; inv_s[0], zero[0];
  * out->col_sum (required, kh kw c + 1 entries) the column sums of the
  * im2col matrix followed by code(0.0); out->conv the geometry.  row_sum must
  * be NULL.  c % 8 == 0, c <= 4096.  The workspace holds the status word and range

@@ -134,13 +134,13 @@ static fqt_status quantize_conv(const void *X, fqt_dtype dtype, int64_t n, int64
   cudaError_t e = launch_range(X, dtype == FQT_BF16, pixels * c, part, &npart, out->col_sum,
                                (int64_t)kh * kw * c, nullptr, 0, nsm, st);
   if (e != cudaSuccess) return cuda_fail(e, "range pass");
-  // code(0.0), the carriers' centre, follows the column sums (device memory)
+  // code(0.0), the padding's code, follows the column sums (device memory)
   int32_t *zc = out->col_sum + (int64_t)kh * kw * c;
   s = launch_fwd_codes(X, dtype == FQT_BF16, pixels, (int)c, bits, out->codes_f16, out->codes,
                        nullptr, part, npart, out->inv_s, out->zero, reinterpret_cast<int *>(w),
                        nsm, st, pad > 0 ? 1 : 0, zc);
   if (s != FQT_OK) return s;
-  return launch_conv_colsum(out->codes_f16, n, (int)h, (int)wd, (int)c, kh, kw, pad,
+  return launch_conv_colsum(out->codes_f16, n, (int)h, (int)wd, (int)c, kh, kw, pad, bits,
                             out->col_sum, st);
 }
 

@@ -1369,7 +1369,11 @@ struct ReduceArgs {
   // grad_W = inv_s1 inv_sx sum_n (a_nc + z'_1)(x_nd + z'_x)
   int64_t Kn;        // rows N of dH / X
   int oa, ob;
-  const int32_t *ob_dev;       // if set, ob is read here (a conv operand's code(0.0))
+  // an implicit im2col X~: its padding entered the product as code 2^(bx-1);
+  // P += (code(0) - ob) pad_a[c][tap(d)], pad_a = the A carriers summed over
+  // the rows whose tap reads padding (C x taps), tap(d) = d / cin
+  const int32_t *pad_a, *code_zero;
+  int taps, cin;
   const int32_t *cs_a, *cs_b;  // column sums of Q_b1 codes (M) and X~ codes (N)
   const float *inv_a, *zero_a, *inv_b, *zero_b;
 };
@@ -1411,7 +1415,8 @@ __global__ void __launch_bounds__(kRedElems * kRedGroups) k_reduce(const ReduceA
         const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
         const float da = za + (float)ma, db = zb + (float)mb;
         const int64_t ca = r.cs_a[c], cb = r.cs_b[d];
-        const int64_t ob = r.ob_dev ? (int64_t)*r.ob_dev : (int64_t)r.ob;
+        const int64_t ob = r.ob;
+        if (r.pad_a) P += ((int64_t)*r.code_zero - ob) * r.pad_a[c * r.taps + d / r.cin];
         // I = sum (a - ma)(b - mb), exact, from the centred product P
         const int64_t I = P + (r.oa - ma) * (cb - r.Kn * ob) +
                           (ob - mb) * (ca - r.Kn * r.oa) +
@@ -1549,7 +1554,8 @@ size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D) {
     const int64_t sp = use_gradw(w, nsm) ? w.splits : plan_splits(C, D, N, b, 8, nsm, true).splits;
     if (sp > splits) splits = sp;
   }
-  const size_t bytes = (size_t)splits * (size_t)C * (size_t)D * 4;
+  // + the padding table of an implicit im2col X~ (C x taps, taps <= D)
+  const size_t bytes = (size_t)splits * (size_t)C * (size_t)D * 4 + (size_t)C * D * 4;
   return (bytes + 255) & ~(size_t)255;
 }
 
@@ -1730,7 +1736,7 @@ struct WArgs {
   int *status;
   // implicit im2col operand (stride 1): X~ is read as 4-D boxes of an NHWC
   // tensor at shifted pixel coordinates; padding comes back as zero carriers
-  int conv, ih, iw, oh, ow, cin, kw, pad, taps;
+  int conv, ih, iw, oh, ow, cin, kh, kw, pad, taps;
 };
 
 __host__ __device__ constexpr uint32_t make_idesc_mn_n(int n) {
@@ -1791,8 +1797,17 @@ __global__ void __launch_bounds__(kWThreads, 1)
     if (lane == 0) {
       int s = 0;
       uint32_t ph = 0;
+      // implicit im2col: the pixel position advances per K block; the D
+      // boxes walk (channel group, tap) without divisions
       for (int64_t it = blockIdx.x; it < n_items && !*abort_flag; it += gridDim.x) {
         const int64_t kb0 = it * w.ks_blocks, kb1 = min(w.kb_total, kb0 + w.ks_blocks);
+        int ox0 = 0, oy = 0, nimg = 0;
+        if (w.conv) {
+          const int64_t p0 = kb0 * kWBK, t = p0 / w.ow;
+          ox0 = (int)(p0 - t * w.ow);
+          oy = (int)(t % w.oh);
+          nimg = (int)(t / w.oh);
+        }
         for (int64_t kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, w.status)) { *abort_flag = 1; break; }
           mbar_expect_tx(&full[s], (uint32_t)stage_bytes);
@@ -1802,18 +1817,29 @@ __global__ void __launch_bounds__(kWThreads, 1)
           if (w.conv) {
             // 32 output pixels of one output row (ow % 32 == 0); box (64 channels
             // of one tap) x 32 pixels read at the tap's offset
-            const int64_t p0 = kb * kWBK;
-            const int ox0 = (int)(p0 % w.ow);
-            const int64_t t = p0 / w.ow;
-            const int oy = (int)(t % w.oh), nimg = (int)(t / w.oh);
+            int cg = 0, kx = 0, ky = 0;
             for (int m = 0; m < 2 * w.mt; ++m) {
-              const int d0 = m * 64, tap = d0 / w.cin, cg = d0 - tap * w.cin;
-              uint8_t *dst = sx + (size_t)m * kWBox;
-              if (tap < w.taps) {
-                const int ky = tap / w.kw, kx = tap - ky * w.kw;
-                tma_load_4d(dst, &tmX, cg, ox0 + kx - w.pad, oy + ky - w.pad, nimg, &full[s]);
-              } else {  // past the last tap: a box outside the tensor (zeros)
-                tma_load_4d(dst, &tmX, 0, 0, w.ih + 8, nimg, &full[s]);
+              if (ky < w.kh)
+                tma_load_4d(sx + (size_t)m * kWBox, &tmX, cg, ox0 + kx - w.pad,
+                            oy + ky - w.pad, nimg, &full[s]);
+              else  // past the last tap: a box outside the tensor (zeros)
+                tma_load_4d(sx + (size_t)m * kWBox, &tmX, 0, 0, w.ih + w.oh + 8, nimg,
+                            &full[s]);
+              cg += 64;
+              if (cg == w.cin) {
+                cg = 0;
+                if (++kx == w.kw) {
+                  kx = 0;
+                  ++ky;
+                }
+              }
+            }
+            ox0 += kWBK;
+            if (ox0 == w.ow) {
+              ox0 = 0;
+              if (++oy == w.oh) {
+                oy = 0;
+                ++nimg;
               }
             }
           } else {
@@ -1977,6 +2003,7 @@ static fqt_status run_gradw(const uint16_t *X16, const uint16_t *Q16, int64_t K,
     w.ih = conv[1];
     w.iw = conv[2];
     w.cin = conv[3];
+    w.kh = conv[4];
     w.kw = conv[5];
     w.pad = conv[6];
     w.oh = conv[1] + 2 * conv[6] - conv[4] + 1;
@@ -2034,6 +2061,49 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
   g.flt_mmax = flt ? (float)mmax : -1.0f;
   return run_gemm(qw->codes_f16, 1, qw->bits, qx->codes_f16, 1, qx->bits, C, Nr, D, p, g, H,
                   MODE_GRADX, 1, flt, st);
+}
+
+// ---------------------------------------------------------------------------
+// Implicit im2col X~ (stride 1): per tap (ky, kx), the sum over the output
+// pixels whose input pixel (oy + ky - pad, ox + kx - pad) lies in the padding
+// of the A operand's carriers (C per row), for the padding correction of
+// k_reduce.  One CTA per (tap, image) visits only that image's padding
+// pixels for the tap: whole rows above / below, then the left / right
+// columns of the other rows; threads over (channel, pixel lane).
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_conv_padsum(const uint16_t *__restrict__ A16, int C,
+                                                     int h, int w, int kw, int pad, int oh,
+                                                     int ow, int taps, int32_t *pad_a) {
+  const int tap = (int)(blockIdx.x % taps);
+  const int64_t img = blockIdx.x / taps;
+  const int ky = tap / kw, kx = tap - ky * kw;
+  const int top = min(oh, max(0, pad - ky)), bot = min(oh - top, max(0, oh - (h + pad - ky)));
+  const int left = min(ow, max(0, pad - kx)), right = min(ow - left, max(0, ow - (w + pad - kx)));
+  const int rows_out = top + bot, cols_out = left + right;
+  const int full_px = rows_out * ow;  // the pixel counts of one image fit int
+  const int count = full_px + (oh - rows_out) * cols_out;
+  const int lanes = blockDim.x >= C ? blockDim.x / C : 1;
+  for (int ch = threadIdx.x % C; ch < C; ch += blockDim.x) {
+    const int pl = blockDim.x >= C ? (int)threadIdx.x / C : 0;
+    if (pl >= lanes) continue;
+    int acc = 0;
+    for (int t = pl; t < count; t += lanes) {
+      int oy, ox;
+      if (t < full_px) {
+        const int r = t / ow;
+        oy = r < top ? r : oh - bot + (r - top);
+        ox = t - r * ow;
+      } else {
+        const int u = t - full_px, r = u / cols_out, cc = u - r * cols_out;
+        oy = top + r;
+        ox = cc < left ? cc : ow - right + (cc - left);
+      }
+      const int64_t p = (img * oh + oy) * (int64_t)ow + ox;
+      const uint16_t hb = __ldg(A16 + p * C + ch);
+      acc += (int)__half2float(*reinterpret_cast<const __half *>(&hb));
+    }
+    if (acc) atomicAdd(&pad_a[ch * taps + tap], acc);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -2464,9 +2534,9 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     const uint16_t *A16 = shifted ? qa->shift_f16 : qa->codes_f16;
     // |shifted code| <= 16 (2^(b-1) - 1) < 2^(b+3): b + 4 bits of centred magnitude
     const int a_bits = shifted ? qa->bits + 4 : qa->bits;
-    // an implicit im2col operand: carriers centred at code(0.0), |.| < 2^b
+    // an implicit im2col operand (its padding is corrected in the reduction)
     const bool conv = qx->conv[0] > 0;
-    const int x_bits = conv ? qx->bits + 1 : qx->bits;
+    const int x_bits = qx->bits;
     const int64_t Nr = qa->rows, C = qa->cols, D = qx->cols;
     if (qx->rows != Nr) return FQT_EINVAL;
     if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
@@ -2483,9 +2553,22 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     const bool w_ok = use_gradw(wp, nsm);
     if (conv && Nr > 0 && !w_ok) return FQT_EUNSUPPORTED;  // the tile kernel reads plain matrices
     const int splits = w_ok ? wp.splits : p.splits;
-    const size_t need = kGemmOffset + (size_t)splits * (size_t)C * (size_t)D * 4;
+    const size_t pbytes = (size_t)splits * (size_t)C * (size_t)D * 4;
+    const int taps = conv ? qx->conv[4] * qx->conv[5] : 0;
+    const size_t need = kGemmOffset + pbytes + (conv ? (size_t)C * taps * 4 : 0);
     if (ws_bytes < need) return FQT_EWORKSPACE;
     int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kGemmOffset);
+    int32_t *pad_a = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kGemmOffset + pbytes);
+    if (conv && Nr > 0) {
+      const int32_t *g = qx->conv;
+      const int oh = g[1] + 2 * g[6] - g[4] + 1, ow = g[2] + 2 * g[6] - g[5] + 1;
+      cudaError_t e = cudaMemsetAsync(pad_a, 0, (size_t)C * taps * 4, st);
+      if (e != cudaSuccess) return cuda_fail(e, "padding sums clear");
+      k_conv_padsum<<<(int)((int64_t)g[0] * taps), 256, 0, st>>>(A16, (int)C, g[1], g[2], g[5],
+                                                                 g[6], oh, ow, taps, pad_a);
+      e = cudaGetLastError();
+      if (e != cudaSuccess) return cuda_fail(e, "padding sums launch");
+    }
     if (Nr > 0 && w_ok) {
       fqt_status s = run_gradw(qx->codes_f16, A16, Nr, (int)C, (int)D, wp, part, status, st,
                                conv ? qx->conv : nullptr);
@@ -2514,7 +2597,12 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     r.ob = 1 << (qx->bits - 1);
     r.cs_a = shifted ? qa->shift_col_sum : qa->col_sum;
     r.cs_b = qx->col_sum;
-    r.ob_dev = conv ? qx->col_sum + D : nullptr;
+    if (conv) {
+      r.pad_a = pad_a;
+      r.code_zero = qx->col_sum + D;
+      r.taps = taps;
+      r.cin = qx->conv[3];
+    }
     r.inv_a = shifted ? qa->shift_scale : qa->inv_s;
     r.zero_a = shifted ? qa->shift_scale + 1 : qa->zero;
     r.inv_b = qx->inv_s;

@@ -65,7 +65,7 @@ fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, in
                             int num_sms, cudaStream_t st, int conv_zero = 0,
                             int32_t *code_zero_out = nullptr);
 fqt_status launch_conv_colsum(const uint16_t *f16, int64_t n, int h, int w, int c, int kh,
-                              int kw, int pad, int32_t *col_sum, cudaStream_t st);
+                              int kw, int pad, int bits, int32_t *col_sum, cudaStream_t st);
 fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 fqt_status launch_shift(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,

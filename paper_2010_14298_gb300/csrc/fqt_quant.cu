@@ -1518,17 +1518,14 @@ __global__ void __launch_bounds__(kFwdMaxThreads)
     gmax = fmaxf(gmax, 0.0f);
   }
   const float s = affine_scale(gmin, gmax, B), z = gmin;
-  // carriers are centred at 2^(b-1), or at the code of 0.0 for a conv operand
-  // whose padding the loads fill with zero carriers
-  uint32_t off = (B + 1u) >> 1;
-  if (conv_zero) {
-    const float v0 = __fmul_rn(__fsub_rn(0.0f, z), s);
-    off = min(__float_as_uint(__fadd_rn(v0, 12582912.0f)) - 0x4B400000u, B);
-  }
+  const uint32_t off = (B + 1u) >> 1;  // carriers: code - 2^(b-1)
   if (blockIdx.x == 0 && tid == 0) {
     inv_out[0] = __fdiv_rn(1.0f, s);
     zero_out[0] = __fmul_rn(s, z);
-    if (code_zero_out) *code_zero_out = (int32_t)off;
+    if (code_zero_out) {  // the code of 0.0 (a conv operand's padding)
+      const float v0 = __fmul_rn(__fsub_rn(0.0f, z), s);
+      *code_zero_out = (int32_t)min(__float_as_uint(__fadd_rn(v0, 12582912.0f)) - 0x4B400000u, B);
+    }
   }
   const int opr = cols / 8;
   const int rl = tid / opr, o = tid - rl * opr;
@@ -1607,15 +1604,16 @@ fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, in
 // Column sums of the implicit im2col matrix of a conv operand (stride 1):
 // im2col column (ky, kx, ch) holds, for every output pixel (n, oy, ox), the
 // code of input pixel (oy + ky - pad, ox + kx - pad) or the code of 0.0 in
-// the padding.  With carriers a = code - code(0) (zero in the padding), the
-// sum is rows code(0) + the carriers over the input rectangle that tap
-// (ky, kx) reads.  One CTA per (tap, image) sums its rectangle (the carriers
-// are in L2 after the codes pass) and adds into the column sums, which the
-// range pass cleared; code(0) sits after them.
+// the padding.  With carriers a = code - 2^(b-1), the sum is the carriers
+// over the input rectangle that tap (ky, kx) reads, plus 2^(b-1) for each of
+// its n_valid entries and code(0) for each of the rows - n_valid padding
+// entries.  One CTA per (tap, image) sums its rectangle (the carriers are in
+// L2 after the codes pass) and adds into the column sums, which the range
+// pass cleared; code(0) sits after them.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_conv_colsum(const uint16_t *__restrict__ f16, int h,
                                                      int w, int c, int kh, int kw, int pad,
-                                                     int oh, int ow, int64_t rows,
+                                                     int oh, int ow, int64_t nimg, int centre,
                                                      int32_t *col_sum) {
   extern __shared__ int acc_s[];  // c
   const int taps = kh * kw;
@@ -1652,20 +1650,101 @@ __global__ void __launch_bounds__(256) k_conv_colsum(const uint16_t *__restrict_
   }
   __syncthreads();
   const int zc = col_sum[(int64_t)taps * c];
+  const int64_t rows = nimg * oh * ow, nvalid = nimg * (int64_t)npix;
+  const int base = img == 0 ? (int)(nvalid * centre + (rows - nvalid) * (int64_t)zc) : 0;
   for (int i = threadIdx.x; i < c; i += blockDim.x) {
-    const int v = acc_s[i] + (img == 0 ? (int)(rows * (int64_t)zc) : 0);
+    const int v = acc_s[i] + base;
     if (v) atomicAdd(&col_sum[(int64_t)tap * c + i], v);
   }
 }
 
+// The same sums in one pass for kernels of up to 9 taps: one CTA per image,
+// every input pixel's carriers added into the taps that read it (registers),
+// then shared memory, then the column sums.
+constexpr int kConvMaxTaps = 9;
+
+__global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict__ f16, int h,
+                                                      int w, int c, int kh, int kw, int pad,
+                                                      int oh, int ow, int64_t nimg,
+                                                      int centre, int32_t *col_sum) {
+  extern __shared__ int acc_s[];  // taps x c
+  const int taps = kh * kw;
+  const int64_t img = blockIdx.x;
+  for (int i = threadIdx.x; i < taps * c; i += blockDim.x) acc_s[i] = 0;
+  __syncthreads();
+  int tky[kConvMaxTaps], tkx[kConvMaxTaps];
+#pragma unroll
+  for (int t = 0; t < kConvMaxTaps; ++t) {
+    tky[t] = t < taps ? t / kw : 0;
+    tkx[t] = t < taps ? t - (t / kw) * kw : 0;
+  }
+  const int octs = c / 8;
+  const int lanes = blockDim.x >= octs ? blockDim.x / octs : 1;
+  for (int oc = threadIdx.x % octs; oc < octs; oc += blockDim.x) {
+    const int pl = blockDim.x >= octs ? (int)threadIdx.x / octs : 0;
+    if (pl >= lanes) continue;
+    int a[kConvMaxTaps][8];
+#pragma unroll
+    for (int t = 0; t < kConvMaxTaps; ++t)
+#pragma unroll
+      for (int j = 0; j < 8; ++j) a[t][j] = 0;
+    for (int p = pl; p < h * w; p += lanes) {
+      const int y = p / w, x = p - y * w;
+      const uint4 v = __ldg(reinterpret_cast<const uint4 *>(
+          f16 + ((img * h + y) * (int64_t)w + x) * c + oc * 8));
+      const uint32_t wds[4] = {v.x, v.y, v.z, v.w};
+      int e[8];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&wds[q]));
+        e[2 * q] = (int)f.x;
+        e[2 * q + 1] = (int)f.y;
+      }
+#pragma unroll
+      for (int t = 0; t < kConvMaxTaps; ++t) {
+        const int oy = y - tky[t] + pad, ox = x - tkx[t] + pad;
+        if (t < taps && oy >= 0 && oy < oh && ox >= 0 && ox < ow) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) a[t][j] += e[j];
+        }
+      }
+    }
+#pragma unroll
+    for (int t = 0; t < kConvMaxTaps; ++t)
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (t < taps && a[t][j]) atomicAdd(&acc_s[t * c + oc * 8 + j], a[t][j]);
+  }
+  __syncthreads();
+  const int zc = col_sum[(int64_t)taps * c];
+  const int64_t rows = nimg * oh * ow;
+  for (int i = threadIdx.x; i < taps * c; i += blockDim.x) {
+    int v = acc_s[i];
+    if (img == 0) {
+      const int t = i / c, ky = t / kw, kx = t - ky * kw;
+      const int ry = min(h, ky - pad + oh) - max(0, ky - pad);
+      const int rx = min(w, kx - pad + ow) - max(0, kx - pad);
+      const int64_t nvalid = nimg * (int64_t)(ry > 0 && rx > 0 ? ry * rx : 0);
+      v += (int)(nvalid * centre + (rows - nvalid) * (int64_t)zc);
+    }
+    if (v) atomicAdd(&col_sum[i], v);
+  }
+}
+
 fqt_status launch_conv_colsum(const uint16_t *f16, int64_t n, int h, int w, int c, int kh,
-                              int kw, int pad, int32_t *col_sum, cudaStream_t st) {
+                              int kw, int pad, int bits, int32_t *col_sum, cudaStream_t st) {
   const int oh = h + 2 * pad - kh + 1, ow = w + 2 * pad - kw + 1;
+  if (n <= 0) return FQT_OK;
+  if (kh * kw <= kConvMaxTaps && (size_t)kh * kw * c * sizeof(int) <= 48 * 1024 &&
+      n <= 0x7fffffff) {
+    k_conv_colsum1<<<(int)n, 256, sizeof(int) * (size_t)kh * kw * c, st>>>(
+        f16, h, w, c, kh, kw, pad, oh, ow, n, 1 << (bits - 1), col_sum);
+    return cuda_fail(cudaGetLastError(), "conv column sums launch");
+  }
   const int64_t grid = n * kh * kw;
-  if (grid <= 0) return FQT_OK;
   if (grid > 0x7fffffff) return FQT_EUNSUPPORTED;
-  k_conv_colsum<<<(int)grid, 256, sizeof(int) * (size_t)c, st>>>(f16, h, w, c, kh, kw, pad, oh,
-                                                                 ow, n * oh * ow, col_sum);
+  k_conv_colsum<<<(int)grid, 256, sizeof(int) * (size_t)c, st>>>(
+      f16, h, w, c, kh, kw, pad, oh, ow, n, 1 << (bits - 1), col_sum);
   return cuda_fail(cudaGetLastError(), "conv column sums launch");
 }
 

@@ -290,8 +290,9 @@ def quantize_act_conv(X: torch.Tensor, kh: int, kw: int, pad: int, bits: int = 8
                       ws: Workspace = None, out: QTensor = None, u8: bool = False,
                       stream=None) -> QTensor:
     """X~ = Q_f(im2col(X)) for a stride-1 convolution, without forming the
-    im2col matrix (Sec. 2.1, App. E): X is NHWC; the codes are stored NHWC,
-    centred at the code of 0.0 (fqt_quantize_act_conv)."""
+    im2col matrix (Sec. 2.1, App. E): X is NHWC; the codes are stored NHWC
+    and col_sum ends with the code of 0.0, the padding's code
+    (fqt_quantize_act_conv)."""
     lib = load()
     X = X.contiguous()
     n, h, w, c = X.shape

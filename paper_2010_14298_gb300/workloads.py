@@ -64,6 +64,7 @@ class Layer:
     W: np.ndarray
     dtype: str  # "f32" or "bf16": the source tensor type handed to the GPU
     runs: List[Tuple[int, int, int]]  # (kind, bits, block) for Q_b2
+    x_nhwc: Optional[np.ndarray] = None  # conv layers: the NHWC input X is the im2col of
 
     @property
     def N(self) -> int:
@@ -118,7 +119,7 @@ def config(index: int, batch: Optional[int] = None, rows: Optional[int] = None,
         W = (np.sqrt(2.0 / 576) * g.standard_normal((64, 576))).astype(np.float32)
         runs = [(k, b_, 16 if k == BHQ else 0) for k in (PTQ, PSQ, BHQ)
                 for b_ in (4, 5, 8)]
-        return [Layer(CONFIG_NAMES[1], dH, X, W, "f32", runs)]
+        return [Layer(CONFIG_NAMES[1], dH, X, W, "f32", runs, x)]
     if index == 2:
         b = batch or 256
         x = g.uniform(-1, 1, (b, 14, 14, 256)).astype(np.float32)
@@ -128,7 +129,7 @@ def config(index: int, batch: Optional[int] = None, rows: Optional[int] = None,
               * _lognormal_rows(g, n, 2.5)[:, None])
         W = (np.sqrt(2.0 / 2304) * g.standard_normal((256, 2304))).astype(np.float32)
         return [Layer(CONFIG_NAMES[2], dH, X, W, "f32",
-                      [(BHQ, 5, nb) for nb in (8, 16, 32, 64)])]
+                      [(BHQ, 5, nb) for nb in (8, 16, 32, 64)], x)]
     if index == 3:
         n = rows or 8192
         out = []

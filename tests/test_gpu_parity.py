@@ -605,8 +605,9 @@ def test_shift_with_a_bifurcated_q_b1_too():
 def _conv_codes_as_im2col(q, x_shape, kh, kw, pad):
     """The im2col matrix of the GPU's NHWC codes (padding = code of 0.0)."""
     n, h, w, c = x_shape
-    zc = int(q.col_sum[-1].item())
-    nhwc = (q.codes16.float().cpu().numpy().astype(np.int64) + zc).reshape(n, h, w, c)
+    zc = int(q.col_sum[-1].item())  # the code of 0.0: the padding's code
+    nhwc = (q.codes16.float().cpu().numpy().astype(np.int64)
+            + (1 << (q.bits - 1))).reshape(n, h, w, c)
     full = np.full((n, h + 2 * pad, w + 2 * pad, c), zc, dtype=np.int64)
     full[:, pad:pad + h, pad:pad + w] = nhwc
     oh, ow = h + 2 * pad - kh + 1, w + 2 * pad - kw + 1
