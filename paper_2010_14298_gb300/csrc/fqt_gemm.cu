@@ -2072,37 +2072,53 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
 // columns of the other rows; threads over (channel, pixel lane).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_conv_padsum(const uint16_t *__restrict__ A16, int C,
-                                                     int h, int w, int kw, int pad, int oh,
-                                                     int ow, int taps, int32_t *pad_a) {
-  const int tap = (int)(blockIdx.x % taps);
-  const int64_t img = blockIdx.x / taps;
+                                                     int64_t nimg, int h, int w, int kw,
+                                                     int pad, int oh, int ow, int taps,
+                                                     int32_t *pad_a) {
+  // a warp per (tap, image); lane = a pair of channels; 8 pixels in flight
+  const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (wid >= nimg * taps) return;
+  const int tap = (int)(wid % taps);
+  const int64_t img = wid / taps;
   const int ky = tap / kw, kx = tap - ky * kw;
   const int top = min(oh, max(0, pad - ky)), bot = min(oh - top, max(0, oh - (h + pad - ky)));
   const int left = min(ow, max(0, pad - kx)), right = min(ow - left, max(0, ow - (w + pad - kx)));
   const int rows_out = top + bot, cols_out = left + right;
   const int full_px = rows_out * ow;  // the pixel counts of one image fit int
   const int count = full_px + (oh - rows_out) * cols_out;
-  const int lanes = blockDim.x >= C ? blockDim.x / C : 1;
-  for (int ch = threadIdx.x % C; ch < C; ch += blockDim.x) {
-    const int pl = blockDim.x >= C ? (int)threadIdx.x / C : 0;
-    if (pl >= lanes) continue;
-    int acc = 0;
-    for (int t = pl; t < count; t += lanes) {
-      int oy, ox;
-      if (t < full_px) {
-        const int r = t / ow;
-        oy = r < top ? r : oh - bot + (r - top);
-        ox = t - r * ow;
-      } else {
-        const int u = t - full_px, r = u / cols_out, cc = u - r * cols_out;
-        oy = top + r;
-        ox = cc < left ? cc : ow - right + (cc - left);
+  for (int c2 = lane; c2 < C / 2; c2 += 32) {
+    int acc0 = 0, acc1 = 0;
+    for (int t0 = 0; t0 < count; t0 += 8) {
+      uint32_t v[8];
+#pragma unroll
+      for (int b = 0; b < 8; ++b) {
+        const int t = t0 + b;
+        v[b] = 0u;
+        if (t < count) {
+          int oy, ox;
+          if (t < full_px) {
+            const int r = t / ow;
+            oy = r < top ? r : oh - bot + (r - top);
+            ox = t - r * ow;
+          } else {
+            const int u = t - full_px, r = u / cols_out, cc = u - r * cols_out;
+            oy = top + r;
+            ox = cc < left ? cc : ow - right + (cc - left);
+          }
+          const int64_t pp = (img * oh + oy) * (int64_t)ow + ox;
+          v[b] = __ldg(reinterpret_cast<const uint32_t *>(A16 + pp * C) + c2);
+        }
       }
-      const int64_t p = (img * oh + oy) * (int64_t)ow + ox;
-      const uint16_t hb = __ldg(A16 + p * C + ch);
-      acc += (int)__half2float(*reinterpret_cast<const __half *>(&hb));
+#pragma unroll
+      for (int b = 0; b < 8; ++b) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&v[b]));
+        acc0 += (int)f.x;
+        acc1 += (int)f.y;
+      }
     }
-    if (acc) atomicAdd(&pad_a[ch * taps + tap], acc);
+    if (acc0) atomicAdd(&pad_a[(2 * c2) * taps + tap], acc0);
+    if (acc1) atomicAdd(&pad_a[(2 * c2 + 1) * taps + tap], acc1);
   }
 }
 
@@ -2564,8 +2580,9 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       const int oh = g[1] + 2 * g[6] - g[4] + 1, ow = g[2] + 2 * g[6] - g[5] + 1;
       cudaError_t e = cudaMemsetAsync(pad_a, 0, (size_t)C * taps * 4, st);
       if (e != cudaSuccess) return cuda_fail(e, "padding sums clear");
-      k_conv_padsum<<<(int)((int64_t)g[0] * taps), 256, 0, st>>>(A16, (int)C, g[1], g[2], g[5],
-                                                                 g[6], oh, ow, taps, pad_a);
+      const int64_t warps = (int64_t)g[0] * taps;
+      k_conv_padsum<<<(int)((warps + 7) / 8), 256, 0, st>>>(A16, (int)C, g[0], g[1], g[2], g[5],
+                                                            g[6], oh, ow, taps, pad_a);
       e = cudaGetLastError();
       if (e != cudaSuccess) return cuda_fail(e, "padding sums launch");
     }

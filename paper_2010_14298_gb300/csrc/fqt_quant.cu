@@ -1662,6 +1662,7 @@ __global__ void __launch_bounds__(256) k_conv_colsum(const uint16_t *__restrict_
 // every input pixel's carriers added into the taps that read it (registers),
 // then shared memory, then the column sums.
 constexpr int kConvMaxTaps = 9;
+constexpr int kConvSlices = 4;
 
 __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict__ f16, int h,
                                                       int w, int c, int kh, int kw, int pad,
@@ -1669,7 +1670,10 @@ __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict
                                                       int centre, int32_t *col_sum) {
   extern __shared__ int acc_s[];  // taps x c
   const int taps = kh * kw;
-  const int64_t img = blockIdx.x;
+  // CTA = (image, slice of kConvSlices input rows)
+  const int64_t img = blockIdx.x / kConvSlices;
+  const int slice = (int)(blockIdx.x % kConvSlices);
+  const int ys = (h * slice) / kConvSlices, ye = (h * (slice + 1)) / kConvSlices;
   for (int i = threadIdx.x; i < taps * c; i += blockDim.x) acc_s[i] = 0;
   __syncthreads();
   int tky[kConvMaxTaps], tkx[kConvMaxTaps];
@@ -1688,7 +1692,7 @@ __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict
     for (int t = 0; t < kConvMaxTaps; ++t)
 #pragma unroll
       for (int j = 0; j < 8; ++j) a[t][j] = 0;
-    for (int p = pl; p < h * w; p += lanes) {
+    for (int p = ys * w + pl; p < ye * w; p += lanes) {
       const int y = p / w, x = p - y * w;
       const uint4 v = __ldg(reinterpret_cast<const uint4 *>(
           f16 + ((img * h + y) * (int64_t)w + x) * c + oc * 8));
@@ -1709,18 +1713,26 @@ __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict
         }
       }
     }
+    // lanes of a warp that share a channel oct add up by shuffles first
+    const bool shfl_ok = octs <= 32 && (32 % octs) == 0;
 #pragma unroll
     for (int t = 0; t < kConvMaxTaps; ++t)
 #pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (t < taps && a[t][j]) atomicAdd(&acc_s[t * c + oc * 8 + j], a[t][j]);
+      for (int j = 0; j < 8; ++j) {
+        int v = a[t][j];
+        if (shfl_ok) {
+          for (int off = octs; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+          if ((int)(threadIdx.x & 31) >= octs) v = 0;
+        }
+        if (t < taps && v) atomicAdd(&acc_s[t * c + oc * 8 + j], v);
+      }
   }
   __syncthreads();
   const int zc = col_sum[(int64_t)taps * c];
   const int64_t rows = nimg * oh * ow;
   for (int i = threadIdx.x; i < taps * c; i += blockDim.x) {
     int v = acc_s[i];
-    if (img == 0) {
+    if (img == 0 && slice == 0) {
       const int t = i / c, ky = t / kw, kx = t - ky * kw;
       const int ry = min(h, ky - pad + oh) - max(0, ky - pad);
       const int rx = min(w, kx - pad + ow) - max(0, kx - pad);
@@ -1736,8 +1748,8 @@ fqt_status launch_conv_colsum(const uint16_t *f16, int64_t n, int h, int w, int 
   const int oh = h + 2 * pad - kh + 1, ow = w + 2 * pad - kw + 1;
   if (n <= 0) return FQT_OK;
   if (kh * kw <= kConvMaxTaps && (size_t)kh * kw * c * sizeof(int) <= 48 * 1024 &&
-      n <= 0x7fffffff) {
-    k_conv_colsum1<<<(int)n, 256, sizeof(int) * (size_t)kh * kw * c, st>>>(
+      n * kConvSlices <= 0x7fffffff) {
+    k_conv_colsum1<<<(int)(n * kConvSlices), 256, sizeof(int) * (size_t)kh * kw * c, st>>>(
         f16, h, w, c, kh, kw, pad, oh, ow, n, 1 << (bits - 1), col_sum);
     return cuda_fail(cudaGetLastError(), "conv column sums launch");
   }
