@@ -161,6 +161,24 @@ def _dist():
     return ws, rank, local
 
 
+def rank_seed(rank: int) -> int:
+    """Seed of a rank's synthetic batch: replicas process independent batches
+    of the same shapes and distributions (weak scaling)."""
+    return 1234 + CONFIG_INDEX + 1000 * rank
+
+
+def max_over_ranks(value: float, device) -> float:
+    """The job's time is the slowest rank's: MAX all-reduce of one float
+    (the only collective; none is on the data path)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -174,7 +192,7 @@ def run_gpu(args):
     fqt.load(build_if_missing=True)
     dev = torch.device("cuda", local)
 
-    L = wl.config(CONFIG_INDEX, seed=1234 + CONFIG_INDEX + 1000 * rank)[0]
+    L = wl.config(CONFIG_INDEX, seed=rank_seed(rank))[0]
     N, C, D = L.N, L.C, L.D
     dH = torch.from_numpy(L.dH).to(dev)
     X = torch.from_numpy(L.X).to(dev)
@@ -265,10 +283,7 @@ def run_gpu(args):
         step_ms.append(sum(d))
     ms_step = float(np.mean(step_ms))
     per_call /= args.steps
-    if world > 1:
-        t = torch.tensor([ms_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_step = float(t.item())
+    ms_step = max_over_ranks(ms_step, dev)
     status = fqt.sync_status(ws)
 
     ops_step = 2 * 2 * N * C * D  # both contractions
