@@ -664,3 +664,57 @@ def test_conv_grad_w_equals_the_explicit_path(batch):
     cols = np.arange(576) if batch == 2 else np.sort(wl.rng(5).choice(576, 48, replace=False))
     ref = orc.matmul(orc.dequant(h1), orc.dequant(hx)[:, cols], a_trans=True)
     assert grad_rel_err(gwc[:, cols], ref) <= GRAD_TOL
+
+
+# --------------------------------------------------------------------------
+# Unbiasedness of the GPU quantizers over seeds (Sec. 3.3, 4.1-4.3; the
+# premise of Thm 1): the mean of the dequantized GPU codes is dH, with the
+# spread the exact per-code variances predict.
+# --------------------------------------------------------------------------
+def _code_moments(v, B):
+    var = np.zeros(v.shape)
+    for idx in np.ndindex(v.shape):
+        var[idx] = orc.sr_moments(float(v[idx]), B)[1]
+    return var
+
+
+@pytest.mark.parametrize("kind,bits,block", [(orc.PSQ, 4, 0), (orc.BHQ, 4, 8), (orc.SHIFT, 4, 0)])
+def test_gpu_quantizers_are_unbiased_monte_carlo(kind, bits, block):
+    g = wl.rng(500 + kind)
+    h = wl.random_grad(g, 16, 64, sigma=1.5, outlier_frac=0.1)
+    B = (1 << bits) - 1
+    ref = orc.quantize_grad(h, kind, bits, block, 0, want_v=True)
+    vc = _code_moments(ref["v"], B)
+    inv = ref["inv_s"].astype(np.float64)
+    if kind == orc.BHQ:
+        vd = np.zeros(h.shape)
+        for b, r0 in enumerate(range(0, 16, block)):
+            Q = orc.householder(block, int(ref["lead"][b]))
+            vd[r0:r0 + block] = ((inv[r0:r0 + block, None] * Q) ** 2) @ vc[r0:r0 + block]
+    else:
+        vd = vc * (inv ** 2)[:, None]
+    K = 512
+    dH = to_dev(h)
+    s1 = np.zeros(h.shape)
+    s2 = np.zeros(h.shape)
+    for seed in range(K):
+        q2, _ = fqt.quantize_grad(dH, kind, bits, block, seed=seed + 77, with_b1=False)
+        d = orc.dequant(q2.to_numpy())
+        s1 += d
+        s2 += d * d
+    mean = s1 / K
+    # the z bound needs the normal approximation of each entry's count of
+    # round-ups: p (1 - p) K >= 8 (BHQ entries mix a block's codes: its
+    # smallest code variance decides)
+    if kind == orc.BHQ:
+        vmin = np.zeros(h.shape)
+        for r0 in range(0, 16, block):
+            vmin[r0:r0 + block] = vc[r0:r0 + block].min(axis=0)
+    else:
+        vmin = vc
+    live = (vd > 0) & (vmin * K >= 8)
+    assert live.mean() > 0.5
+    z = (mean - h)[live] / np.sqrt(vd[live] / K)
+    assert np.abs(z).max() < 5.5
+    emp = (s2 / K - mean ** 2).sum()
+    assert emp / vd.sum() == pytest.approx(1.0, rel=0.12)
