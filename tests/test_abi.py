@@ -54,3 +54,56 @@ def test_argument_errors_are_synchronous_and_need_no_gpu():
     st = lib.fqt_quantize_act(ctypes.cast(buf, ctypes.c_void_p), 0, 4, 8, 9,
                               ctypes.byref(qs), None, 0, None)
     assert st == 1
+
+
+def _aligned(n=1 << 16):
+    """A 256-byte aligned host buffer standing in for a device pointer in
+    calls that must fail validation before touching it."""
+    raw = ctypes.create_string_buffer(n + 256)
+    addr = (ctypes.addressof(raw) + 255) & ~255
+    return raw, ctypes.c_void_p(addr)
+
+
+def test_new_entry_points_validate_without_gpu():
+    """The adaptive groups, the shift quantizer and the implicit im2col
+    operand reject bad requests synchronously, before any CUDA call."""
+    from paper_2010_14298_gb300 import fqt
+    lib = fqt.load()
+    raw, p = _aligned()
+    q = fqt._QT()
+    q.codes_f16 = p.value
+    q.inv_s = p.value
+    q.zero = p.value
+    BHQ, SHIFT = 2, 3
+    # adaptive BHQ (block 0) needs perm / gstart / gsize
+    st = lib.fqt_quantize_grad(p, 0, 16, 64, BHQ, 5, 0, 0, ctypes.byref(q), None, p, 256,
+                               None)
+    assert st == 1
+    # unknown kind
+    assert lib.fqt_quantize_grad(p, 0, 16, 64, 7, 5, 0, 0, ctypes.byref(q), None, p, 256,
+                                 None) == 1
+    # the shift quantizer needs its grad_W operand arrays
+    assert lib.fqt_quantize_grad(p, 0, 16, 64, SHIFT, 5, 0, 0, ctypes.byref(q), None, p, 256,
+                                 None) == 1
+    q.shift_f16 = p.value
+    q.shift = p.value
+    q.shift_col_sum = p.value
+    q.shift_scale = p.value
+    # ... and rows of 64 .. 1024 columns
+    assert lib.fqt_quantize_grad(p, 0, 16, 72, SHIFT, 5, 0, 0, ctypes.byref(q), None, p, 256,
+                                 None) == 2
+    # the implicit im2col quantizer: row sums are not built, bad geometry fails
+    qc = fqt._QT()
+    qc.codes_f16 = p.value
+    qc.inv_s = p.value
+    qc.zero = p.value
+    qc.col_sum = p.value
+    qc.row_sum = p.value
+    assert lib.fqt_quantize_act_conv(p, 0, 2, 8, 8, 64, 3, 3, 1, 8, ctypes.byref(qc), p, 256,
+                                     None) == 2
+    qc.row_sum = None
+    assert lib.fqt_quantize_act_conv(p, 0, 2, 2, 2, 64, 5, 5, 0, 8, ctypes.byref(qc), p, 256,
+                                     None) == 1  # 5x5 taps on a 2x2 image
+    assert lib.fqt_quantize_act_conv(p, 0, 2, 8, 8, 60, 3, 3, 1, 8, ctypes.byref(qc), p, 256,
+                                     None) == 2  # c % 8 != 0
+    del raw
