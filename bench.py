@@ -561,6 +561,127 @@ def run_gpu(args):
                "launches_per_step": 10,
                "device_status": fqt.sync_status(ws)}
 
+    def time_graphs(fns, steps):
+        """Median ms of each call, replayed as one CUDA graph per call, L2
+        flushed before each round."""
+        for _ in range(3):
+            for f in fns:
+                f()
+        torch.cuda.synchronize()
+        gs_ = []
+        for f in fns:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                f()
+            gs_.append(g)
+        tt = [[] for _ in fns]
+        for i in range(steps):
+            flush.fill_(i & 0xFF)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(fns) + 1)]
+            for k, g in enumerate(gs_):
+                ev[k].record(stream)
+                g.replay()
+            ev[-1].record(stream)
+            torch.cuda.synchronize()
+            for k in range(len(fns)):
+                tt[k].append(ev[k].elapsed_time(ev[k + 1]))
+        return [float(np.median(t)) for t in tt]
+
+    bf16_peak = 1862.7
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            bf16_peak = float(json.load(f)["bf16_tflops"])
+    except Exception:
+        pass
+
+    # ---- the other full-size workloads: one backward step per layer, each
+    # contraction against its binding roofline (HBM bytes with 2-byte code
+    # carriers, or the tensor peak of the fp16 kind = the measured bf16 peak) ----
+    others = None
+    if args.config_steps > 0:
+        others = []
+        for cfg in (2, 3):
+            for Lo in wl.config(cfg):
+                No, Co, Do = Lo.N, Lo.C, Lo.D
+                dt = torch.bfloat16 if Lo.dtype == "bf16" else torch.float32
+                to = lambda a: torch.from_numpy(a).to(dev).to(dt)
+                dHo, Xo, Wo = to(Lo.dH), to(Lo.X), to(Lo.W)
+                wso = fqt.Workspace(No, Co, Do, device=dev)
+                qxo = fqt.QTensor.empty(No, Do, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+                qwo = fqt.QTensor.empty(Co, Do, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+                q2o = fqt.QTensor.empty(No, Co, fqt.BHQ, 5, 16, True, False, dev, u8=False)
+                q1o = fqt.QTensor.empty(No, Co, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+                gxo = torch.empty((No, Do), dtype=torch.float32, device=dev)
+                gwo = torch.empty((Co, Do), dtype=torch.float32, device=dev)
+                wfx = fqt.Workspace(No, Do, 16, device=dev)
+                wfw = fqt.Workspace(Co, Do, 16, device=dev)
+                fo = [lambda: fqt.quantize_act(Xo, 8, ws=wfx, out=qxo),
+                      lambda: fqt.quantize_weight(Wo, 8, ws=wfw, out=qwo),
+                      lambda: fqt.quantize_grad(dHo, fqt.BHQ, 5, 16, 5, ws=wso, q_b2=q2o,
+                                                q_b1=q1o),
+                      lambda: fqt.linear_backward(q2o, q1o, qxo, qwo, grad_x=True, grad_w=False,
+                                                  ws=wso, out_x=gxo),
+                      lambda: fqt.linear_backward(q2o, q1o, qxo, qwo, grad_x=False, grad_w=True,
+                                                  ws=wso, out_w=gwo)]
+                per = time_graphs(fo, args.config_steps)
+                ops = 2 * No * Co * Do
+                eb = 2 if Lo.dtype == "bf16" else 4
+                bytes_x = No * Co * 2 + Co * Do * 2 + No * Do * 4 + No * 12 + (No // 16) * 4
+                bytes_w = No * Co * 2 + No * Do * 2 + Co * Do * 4 + (Co + Do) * 4
+                roof = {}
+                for name, ms, by in (("grad_x", per[3], bytes_x), ("grad_w", per[4], bytes_w)):
+                    gbs = by / (ms * 1e-3) / 1e9
+                    tops = ops / (ms * 1e-3) / 1e12
+                    hbm_bound = ops / by < bf16_peak * 1e12 / (hbm_peak * 1e9)
+                    roof[name] = {"bound": "hbm" if hbm_bound else "tensor", "ms": ms,
+                                  "TOPS": tops, "GBs": gbs,
+                                  "frac": gbs / hbm_peak if hbm_bound else tops / bf16_peak,
+                                  "ops_per_byte": ops / by}
+                others.append({"workload": Lo.name, "N": No, "C": Co, "D": Do,
+                               "dtype": Lo.dtype, "quantizer": "BHQ-5 block 16 + Q_b1 PTQ-8",
+                               "per_call_ms": dict(zip(["quantize_act", "quantize_weight",
+                                                        "quantize_grad", "grad_x", "grad_w"],
+                                                       per)),
+                               "ms_per_step": sum(per),
+                               "TOPS": 2 * ops / (sum(per) * 1e-3) / 1e12,
+                               "quantize_grad_GBs": (No * Co * eb + 2 * No * Co * 2 + No * 20)
+                               / (per[2] * 1e-3) / 1e9,
+                               "roofline": roof, "device_status": fqt.sync_status(wso)})
+                del dHo, Xo, Wo, qxo, qwo, q2o, q1o, gxo, gwo, wso, wfx, wfw
+                torch.cuda.empty_cache()
+
+    # ---- the paper's own overhead shape (Sec. 4.3): a conv layer with
+    # N = 128, C = 64, 56 x 56, i.e. dH of 401408 im2col rows x 64; the paper
+    # timed its CPU routines there (context only, another machine) ----
+    ovh = None
+    if args.config_steps > 0:
+        gp = wl.rng(480)
+        dHp = torch.from_numpy(wl.random_grad(gp, 128 * 56 * 56, 64, sigma=2.0,
+                                              outlier_frac=0.01)).to(dev)
+        Np = dHp.shape[0]
+        wsp = fqt.Workspace(Np, 64, 16, device=dev)
+        qsets = {}
+        for name, kind, bits, block in (("PTQ-8", fqt.PTQ, 8, 0), ("PSQ-8", fqt.PSQ, 8, 0),
+                                        ("BHQ-5 block 16", fqt.BHQ, 5, 16),
+                                        ("BHQ-5 adaptive groups", fqt.BHQ, 5, 0)):
+            qsets[name] = (fqt.QTensor.empty(Np, 64, kind, bits, block, True, False, dev, u8=False),
+                           fqt.QTensor.empty(Np, 64, fqt.PTQ, 8, 0, False, True, dev, u8=False),
+                           kind, bits, block)
+        fns = [(lambda q=q: fqt.quantize_grad(dHp, q[2], q[3], q[4], 3, ws=wsp, q_b2=q[0],
+                                              q_b1=q[1])) for q in qsets.values()]
+        per = time_graphs(fns, args.config_steps)
+        ovh = {"shape": "dH 401408 x 64 fp32 (conv N=128, C=64, 56x56)",
+               "quantize_grad_ms": dict(zip(qsets.keys(), per)),
+               "includes": "range pass, scales / transform, SR of Q_b2 and of the 8-bit Q_b1, "
+                           "packing, row and column sums (and the grouping, adaptive)",
+               "paper_cpu_ms": {"per-tensor range": 11.0, "per-sample range": 24.0,
+                                "Householder transform": 21.0, "BHQ construction": 0.003,
+                                "INT8 conv layer": 480.0},
+               "paper_cpu_note": "1 Intel CPU core, CPU TensorFlow + AVX (Sec. 4.3): context only",
+               "device_status": fqt.sync_status(wsp)}
+        del dHp, qsets, wsp
+        torch.cuda.empty_cache()
+
     result = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -588,6 +709,8 @@ def run_gpu(args):
         "adaptive_bhq": ada,
         "shift_quantizer": shf,
         "implicit_im2col": imp,
+        "other_workloads": others,
+        "paper_overhead_shape": ovh,
         "gpu_launches": int(sum(launches_per_call) * args.steps),
         "device_status": status,
     }
@@ -672,6 +795,9 @@ def main():
                     help="timed steps of the shift quantizer path (0: skip)")
     ap.add_argument("--implicit-steps", type=int, default=50,
                     help="timed steps with the implicit im2col X operand (0: skip)")
+    ap.add_argument("--config-steps", type=int, default=20,
+                    help="timed steps of the other full-size workloads and of the paper's "
+                         "overhead shape (0: skip)")
     ap.add_argument("--eager", action="store_true",
                     help="time the C-ABI calls directly instead of graph replays")
     args = ap.parse_args()

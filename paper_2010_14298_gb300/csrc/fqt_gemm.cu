@@ -1609,6 +1609,13 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   // (split-K partials): deep operand ring
   g.stages = partial ? 5 : 2;
   g.ring = partial ? 1 : 0;  // grad_X stores straight from registers
+  // grad_X tiles with a long reduction (K of many blocks: a contraction that
+  // is tensor-bound rather than bound by its output) keep more operand
+  // stages in flight
+  if (!partial && (K + BK - 1) / BK > 2) {
+    while (g.stages < kMaxStages && gemm_smem_bytes(g.stages + 1, g.ring) <= 227 * 1024)
+      ++g.stages;
+  }
   if (!partial) g.out = static_cast<float *>(out);
   // grad_X with one exact chunk per tile: four accumulators in rotation, so
   // the next tile of each epilogue set is ready when it finishes the last;
