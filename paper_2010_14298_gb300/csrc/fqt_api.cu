@@ -161,7 +161,7 @@ fqt_status fqt_quantize_act_conv(const void *X, fqt_dtype dtype, int64_t n, int6
 size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
   size_t need = gemm_workspace_bytes(N, C, D);
   const size_t grp = group_workspace_bytes(N);         // adaptive BHQ grouping
-  const size_t list = 256 + (size_t)(N > 0 ? N : 0) * 4;  // its grad_X work list
+  const size_t list = group_list_bytes(N);               // its grad_X work lists
   if (grp > need) need = grp;
   if (list > need) need = list;
   return kGemmOffset + need;

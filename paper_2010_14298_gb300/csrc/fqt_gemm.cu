@@ -2138,7 +2138,8 @@ __global__ void __launch_bounds__(256) k_conv_padsum(const uint16_t *__restrict_
 // with the arithmetic of the fused epilogue: fp32 where every magnitude is
 // exact (block sums off the fp32 bits), int64 / float-float otherwise.
 // k_grp_list collects the groups that need it; k_grp_fix gives a warp one
-// (group, 128 columns) unit, each lane 4 consecutive columns.
+// (group, 128 columns) unit, each lane 4 consecutive columns, and
+// k_grp_fix_big a CTA to each group of more than 32 rows.
 // ---------------------------------------------------------------------------
 struct FixArgs {
   float *out;
@@ -2151,8 +2152,8 @@ struct FixArgs {
   float raw_mmax;
   int small_p;  // every |P| < 2^22: the fp32 block sums apply
   float mmax_nb[33];  // groups of nb <= 32 rows: largest |m| of the fp32 form
-  int32_t *list;
-  int *count;
+  int32_t *list, *list_big;
+  int *count, *count_big;
   int *status;
 };
 
@@ -2184,7 +2185,11 @@ __global__ void __launch_bounds__(256) k_grp_list(const FixArgs f) {
     const int64_t k0 = f.gstart[gi];
     if (k0 < f.N) {
       const int64_t k1 = f.gstart[gi + 1];
-      if (k1 - k0 >= 2) {
+      if (k1 - k0 > 32) {
+        // a CTA of its own (k_grp_fix_big)
+        const int slot = atomicAdd(f.count_big, 1);
+        f.list_big[slot] = (int32_t)gi;
+      } else if (k1 - k0 >= 2) {
         need = true;
       } else if (k1 - k0 == 1) {
         const float m = rintf(two_sum((float)f.og, f.zero[k0]).h);
@@ -2304,6 +2309,129 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
         o4[c] = __fmul_rn(t.sc, ff_round(v));
       }
       __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+    }
+  }
+}
+
+// Groups of more than 32 rows: a CTA each, its warps taking every NW-th
+// row (kBigBatch rows in flight per warp) with the int64 integer parts and
+// float-float reflection of fix_group_general; the block sums S go through
+// shared memory in warp order.
+constexpr int kBigFixWarps = 16, kBigBatch = 4;
+
+__global__ void __launch_bounds__(kBigFixWarps * 32) k_grp_fix_big(const FixArgs f) {
+  constexpr int NW = kBigFixWarps;
+  __shared__ long long s_part[NW][128];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nchunk = (int)((f.D + 127) / 128);
+  const int nunits = *f.count_big;
+  const float inv_sw = *f.inv_sw, zw = *f.zero_w;
+  const ff y = two_sum((float)f.ow, zw);
+  const int Cn = f.C;
+  for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+    const int64_t gi = f.list_big[u];
+    if (gi < 0 || gi >= f.N) {
+      if (threadIdx.x == 0) record_status(f.status, FQT_EINVAL);
+      continue;
+    }
+    const int64_t k0 = f.gstart[gi];
+    int64_t k1 = f.gstart[gi + 1];
+    if (k1 > f.N) k1 = f.N;
+    if (k0 < 0 || k1 - k0 < 2) continue;
+    const int nb = (int)(k1 - k0);
+    const HhConst hc = hh_const(nb);
+    auto prow = [&](int r) -> int64_t {
+      int64_t pr = f.perm[k0 + r];
+      return pr < 0 || pr >= f.N ? 0 : pr;
+    };
+    for (int ch = 0; ch < nchunk; ++ch) {
+      const int64_t j = (int64_t)ch * 128 + lane * 4;
+      const bool jv = j < f.D;
+      int cwi[4];
+      float U[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int cs = jv ? f.col_sum_w[j + c] : 0;
+        cwi[c] = cs - Cn * f.ow;
+        U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
+      }
+      // ---- pass 1: S = sum_k I_k, I = P + m CWc ----
+      long long S[4] = {0, 0, 0, 0};
+      for (int r0 = warp; r0 < nb; r0 += NW * kBigBatch) {
+        float4 P[kBigBatch];
+        long long m[kBigBatch];
+#pragma unroll
+        for (int b = 0; b < kBigBatch; ++b) {
+          const int r = r0 + b * NW;
+          const bool v = r < nb && jv;
+          m[b] = v ? __float2ll_rn(rintf(two_sum((float)f.og, f.zero[k0 + r]).h)) : 0;
+          P[b] = v ? *reinterpret_cast<const float4 *>(f.out + prow(r) * f.D + j)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int b = 0; b < kBigBatch; ++b) {
+          S[0] += (long long)__float2int_rn(P[b].x) + m[b] * cwi[0];
+          S[1] += (long long)__float2int_rn(P[b].y) + m[b] * cwi[1];
+          S[2] += (long long)__float2int_rn(P[b].z) + m[b] * cwi[2];
+          S[3] += (long long)__float2int_rn(P[b].w) + m[b] * cwi[3];
+        }
+      }
+#pragma unroll
+      for (int c = 0; c < 4; ++c) s_part[warp][lane * 4 + c] = S[c];
+      // the lead row's integer parts (row 0 of the group)
+      long long Ipl[4] = {0, 0, 0, 0};
+      if (jv) {
+        const long long m0 = __float2ll_rn(rintf(two_sum((float)f.og, f.zero[k0]).h));
+        const float4 P0 = *reinterpret_cast<const float4 *>(f.out + prow(0) * f.D + j);
+        Ipl[0] = (long long)__float2int_rn(P0.x) + m0 * cwi[0];
+        Ipl[1] = (long long)__float2int_rn(P0.y) + m0 * cwi[1];
+        Ipl[2] = (long long)__float2int_rn(P0.z) + m0 * cwi[2];
+        Ipl[3] = (long long)__float2int_rn(P0.w) + m0 * cwi[3];
+      }
+      __syncthreads();
+      ff rS[4], beta[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        long long tot = 0;
+        for (int w = 0; w < NW; ++w) tot += s_part[w][lane * 4 + c];
+        rS[c] = ff_mul(hc.rho, ff_from_int(tot));
+        beta[c] = ff_mul(hc.kap, ff_add(rS[c], ff_neg(ff_from_int(Ipl[c]))));
+      }
+      // every warp has read the lead row and the sums before any row is
+      // overwritten, and before the next chunk reuses s_part
+      __syncthreads();
+      // ---- pass 2: offsets and the inverse reflection ----
+      for (int r0 = warp; r0 < nb; r0 += NW * kBigBatch) {
+        float4 P[kBigBatch];
+        int64_t pr[kBigBatch];
+#pragma unroll
+        for (int b = 0; b < kBigBatch; ++b) {
+          const int r = r0 + b * NW;
+          const bool v = r < nb && jv;
+          pr[b] = v ? prow(r) : 0;
+          P[b] = v ? *reinterpret_cast<const float4 *>(f.out + pr[b] * f.D + j)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int b = 0; b < kBigBatch; ++b) {
+          const int r = r0 + b * NW;
+          if (r >= nb || !jv) continue;
+          const RowTerms t = row_terms(f, k0 + r, inv_sw, true);
+          const long long m = __float2ll_rn(t.m);
+          const float pv[4] = {P[b].x, P[b].y, P[b].z, P[b].w};
+          float o4[4];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const ff I = ff_from_int((long long)__float2int_rn(pv[c]) + m * cwi[c]);
+            ff v = r == 0 ? rS[c] : ff_add(I, ff_neg(beta[c]));
+            v = ff_add(v, two_prod(t.hd, U[c]));
+            v = ff_add(v, ff_mul({t.hR, 0.0f}, y));
+            o4[c] = __fmul_rn(t.sc, ff_round(v));
+          }
+          __stcs(reinterpret_cast<float4 *>(f.out + pr[b] * f.D + j),
+                 make_float4(o4[0], o4[1], o4[2], o4[3]));
+        }
+      }
     }
   }
 }
@@ -2479,7 +2607,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       const bool flt = C <= kc_terms && mmax >= 0.0 && (nb <= 1 || pmax < ((int64_t)1 << 22));
       // the adaptive groups need the fp32 form (rows are scattered by perm)
       if (adapt && !flt) return FQT_EUNSUPPORTED;
-      const size_t list_bytes = 256 + (size_t)Nr * 4;
+      const size_t list_bytes = group_list_bytes(Nr);
       if (adapt && ws_bytes < kGemmOffset + list_bytes) return FQT_EWORKSPACE;
       GemmArgs g;
       memset(&g, 0, sizeof(g));
@@ -2533,11 +2661,14 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
         }
         char *lw = static_cast<char *>(ws) + kGemmOffset;
         f.count = reinterpret_cast<int *>(lw);
+        f.count_big = reinterpret_cast<int *>(lw + 4);
         f.list = reinterpret_cast<int32_t *>(lw + 256);
+        f.list_big = reinterpret_cast<int32_t *>(lw + 256 + (((size_t)Nr * 4 + 255) & ~(size_t)255));
         f.status = status;
-        cudaError_t e = cudaMemsetAsync(f.count, 0, sizeof(int), st);
+        cudaError_t e = cudaMemsetAsync(f.count, 0, 2 * sizeof(int), st);
         if (e != cudaSuccess) return cuda_fail(e, "group list clear");
         k_grp_list<<<(int)((Nr + 255) / 256), 256, 0, st>>>(f);
+        k_grp_fix_big<<<nsm * 2, kBigFixWarps * 32, 0, st>>>(f);
         k_grp_fix<<<nsm * 8, 256, 0, st>>>(f);
         e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_fail(e, "group fix-up launch");

@@ -49,6 +49,11 @@ constexpr int kSortThreads = 256;
 __host__ __device__ constexpr int sort_ipt(int64_t N) { return N <= ((int64_t)1 << 17) ? 4 : 16; }
 constexpr int kScanTile = 1024;  // sorted rows per CTA of the choice kernels
 constexpr int kKeysThreads = 1024;
+// Groups of more than kBigGroup rows are quantized by a CTA each.  Group
+// sizes follow the sorted norms (non-increasing up to the rounding), so
+// every such group has an index below N / kBigGroup + 1.
+constexpr int kBigGroup = 64;
+__host__ __device__ inline int64_t big_grid(int64_t N) { return N / kBigGroup + 1; }
 // the sort's tile offsets are summed per CTA over all tiles: 256 tiles at most
 constexpr int64_t kMaxGroupRows = (int64_t)1 << 20;
 
@@ -664,6 +669,8 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
     if (k1 > N) k1 = N;
     if (k1 <= k0) continue;
     const int nb = (int)(k1 - k0);
+    // groups of more than kBigGroup rows get a whole CTA (k_bhq_groups_big)
+    if (nb > kBigGroup && gi < big_grid(N)) continue;
 
     // ---- pass 1: lead row, lambda2, column sums of the small rows ----
     float xl[8], csm[8];
@@ -872,6 +879,292 @@ __global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// BHQ of one large group per CTA: the eight warps split the group's rows in
+// every pass (RS rows per warp step), and the column sums of the small rows,
+// lambda2, and the group sums of the offsets d and R go through shared
+// memory in a fixed order.  Same arithmetic as k_bhq_groups.
+// ---------------------------------------------------------------------------
+template <typename T, int LPR>
+__global__ void __launch_bounds__(256) k_bhq_groups_big(const QuantArgs a) {
+  constexpr int CO = LPR, RS = 32 / LPR, C = 8 * LPR, NW = 8;
+  __shared__ float2 red[NW];
+  __shared__ int redi[NW];
+  __shared__ float col_s[NW][C];   // per-warp column sums, then lead row / w
+  __shared__ float lead_s[C];
+  __shared__ float misc_s[NW][4];  // l2, pmin, pmax per warp
+  __shared__ ff sd_s[NW], sR_s[NW];
+  __shared__ float dp_s;
+  __shared__ ff Rp_s;
+  extern __shared__ int csum_s[];  // C column sums of Q_b1
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int sub = lane / LPR, o = lane - sub * LPR;
+  const int64_t N = a.N;
+  const int64_t gi = blockIdx.x;
+  if (gi >= N) return;
+  const int64_t k0 = __ldg(a.gstart + gi);
+  if (k0 >= N) return;
+  int64_t k1 = __ldg(a.gstart + gi + 1);
+  if (k1 > N) k1 = N;
+  if (k1 - k0 <= kBigGroup) return;
+  const int nb = (int)(k1 - k0);
+  const T *h = reinterpret_cast<const T *>(a.h);
+
+  // ---- global range (Q_b1 scale) from the range-pass partials ----
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < a.npart; i += blockDim.x) {
+    const float2 p = a.part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmin, gmax);
+    redi[warp] = bad;
+  }
+  for (int i = tid; i < C; i += blockDim.x) csum_s[i] = 0;
+  __syncthreads();
+  gmin = red[0].x;
+  gmax = red[0].y;
+  bad = redi[0];
+  for (int w = 1; w < NW; ++w) {
+    gmin = fminf(gmin, red[w].x);
+    gmax = fmaxf(gmax, red[w].y);
+    bad |= redi[w];
+  }
+  if (bad) return;  // k_bhq_groups records the status
+  const uint32_t B2 = (1u << a.bits) - 1u;
+  const uint32_t og2 = (B2 + 1u) >> 1;
+  const float s_g1 = affine_scale(gmin, gmax, 255u);
+  const float s_g1_16 = __fmul_rn(s_g1, 65536.0f);
+  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
+  PhiloxKeys key;
+#pragma unroll
+  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
+  bool badp = false;
+
+  // ---- pass 1: lead row, lambda2, column sums of the small rows ----
+  float csm[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) csm[j] = 0.0f;
+  float l2 = 0.0f;
+  for (int r0 = warp * RS; r0 < nb; r0 += NW * RS) {
+    const int r = r0 + sub;
+    const bool v = r < nb;
+    int64_t src = v ? (int64_t)__ldg(a.perm + k0 + r) : 0;
+    if (src < 0 || src >= N) {
+      badp = true;
+      src = 0;
+    }
+    float x[8];
+    if (v) {
+      load_oct(h + src * C + o * 8, x);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) x[j] = 0.0f;
+    }
+    float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      mm.x = fminf(mm.x, x[j]);
+      mm.y = fmaxf(mm.y, x[j]);
+    }
+    mm = row_minmax<LPR>(mm);
+    if (v) {
+      if (r == 0) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) lead_s[o * 8 + j] = x[j];
+        if (o == 0) {
+          misc_s[0][1] = mm.x;
+          misc_s[0][2] = mm.y;
+        }
+      } else {
+        l2 = fmaxf(l2, fmaxf(fabsf(mm.x), fabsf(mm.y)));
+#pragma unroll
+        for (int j = 0; j < 8; ++j) csm[j] += x[j];
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) csm[j] = sub_add<LPR>(csm[j]);
+  l2 = sub_max<LPR>(l2);
+  if (sub == 0) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) col_s[warp][o * 8 + j] = csm[j];
+  }
+  if (lane == 0) misc_s[warp][0] = l2;
+  __syncthreads();
+  // reduce over the warps in a fixed order
+  l2 = 0.0f;
+  for (int w = 0; w < NW; ++w) l2 = fmaxf(l2, misc_s[w][0]);
+  const float pmin = misc_s[0][1], pmax = misc_s[0][2];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    float sacc = 0.0f;
+    for (int w = 0; w < NW; ++w) sacc += col_s[w][o * 8 + j];
+    csm[j] = sacc;
+  }
+  float xl[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) xl[j] = lead_s[o * 8 + j];
+  const float lam2 = 2.0f * l2;
+  const float np = fmaxf(fabsf(pmin), fabsf(pmax));
+  float s1f = 0.0f, s2f = 0.0f, rho = 0.0f, kap = 0.0f;
+  if (np > 0.0f) {
+    float lam1 = __fsub_rn(pmax, pmin);
+    if (!(lam1 > 0.0f)) lam1 = 2.0f * np;
+    const float Nf = (float)nb;
+    if (lam2 > 0.0f) {
+      const float c1 = cbrtf(lam1), c2 = cbrtf(lam2);
+      const float n3 = cbrtf(Nf), n6 = sqrtf(n3);
+      const float den = c1 * c1 / n3 + c2 * c2 * n3 * n3;
+      s1f = (float)B2 * n6 / (c1 * den);
+      s2f = (float)B2 * n6 / (c2 * den);
+    } else {
+      s1f = (float)B2 * sqrtf(Nf) / lam1;
+    }
+    rho = 1.0f / sqrtf(Nf);
+    kap = 1.0f / (1.0f - rho);
+  }
+  const float el = kap * (rho - 1.0f), es = kap * rho;
+  float w[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) w[j] = fmaf(es, __fmul_rn(s2f, csm[j]), el * __fmul_rn(s1f, xl[j]));
+
+  // ---- pass 2: transform, row minimum, rounding, packing, sums ----
+  ff sd = {0.0f, 0.0f}, sR = {0.0f, 0.0f};
+  int cs[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) cs[j] = 0;
+  for (int r0 = warp * RS; r0 < nb; r0 += NW * RS) {
+    const int r = r0 + sub;
+    const bool v = r < nb;
+    int64_t src = v ? (int64_t)__ldg(a.perm + k0 + r) : 0;
+    if (src < 0 || src >= N) src = 0;
+    float x[8];
+    if (v) {
+      load_oct(h + src * C + o * 8, x);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) x[j] = 0.0f;
+    }
+    const bool lead = r == 0;
+    const float sk = lead ? s1f : s2f;
+    const float ck = lead ? rho - 1.0f : rho;
+    float t[8];
+    float tmin = INFINITY;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      t[j] = fmaf(-ck, w[j], __fmul_rn(sk, x[j]));
+      tmin = fminf(tmin, t[j]);
+    }
+    const float z2 = row_min<LPR>(tmin);
+    const int64_t row = k0 + r;
+    uint32_t c[8];
+    int rs2 = 0, rs1 = 0;
+    if (v) {
+      const uint4 w2 = philox_oct((uint64_t)row * (uint64_t)CO + (uint64_t)o, 0u, key);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c[j] = sr_code16(__fmul_rn(__fsub_rn(t[j], z2), 65536.0f), u16_of(w2, j), B2);
+        rs2 += (int)c[j];
+      }
+      if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
+      if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + o * 8, c, og2);
+      if (has_b1) {
+        const uint4 w1 = philox_oct((uint64_t)src * (uint64_t)CO + (uint64_t)o, 1u, key);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float vv = __fmul_rn(__fsub_rn(x[j], gmin), s_g1_16);
+          c[j] = sr_code16(vv, u16_of(w1, j), 255u);
+          rs1 += (int)c[j];
+          cs[j] += (int)c[j];
+        }
+        if (a.c1) store_codes8(a.c1 + src * (int64_t)C + o * 8, c);
+        if (a.f1) store_carriers8(a.f1 + src * (int64_t)C + o * 8, c, 128u);
+      }
+    }
+    rs2 = row_add<LPR>(rs2);
+    if (has_b1) rs1 = row_add<LPR>(rs1);
+    const ff xo = two_sum((float)og2, z2);
+    const float m = rintf(xo.h);
+    const ff d = fast_two_sum(__fsub_rn(xo.h, m), xo.l);
+    const ff R = two_sum((float)(rs2 - C * (int)og2), __fmul_rn((float)C, m));
+    if (v && o == 0) {
+      if (a.rsum2) a.rsum2[row] = rs2;
+      if (has_b1 && a.rsum1) a.rsum1[src] = rs1;
+      a.inv2[row] = sk > 0.0f ? __fdiv_rn(1.0f, sk) : 0.0f;
+      a.zero2[row] = z2;
+      if (a.hz) {
+        a.hz[row] = ff_round(d);
+        a.hr[row] = ff_round(R);
+      }
+      sd = ff_add(sd, d);
+      sR = ff_add(sR, R);
+      if (lead) {
+        dp_s = ff_round(d);
+        Rp_s = R;
+      }
+    }
+  }
+#pragma unroll
+  for (int off = LPR; off < 32; off <<= 1) {
+    const ff od = {__shfl_xor_sync(0xffffffffu, sd.h, off), __shfl_xor_sync(0xffffffffu, sd.l, off)};
+    const ff oR = {__shfl_xor_sync(0xffffffffu, sR.h, off), __shfl_xor_sync(0xffffffffu, sR.l, off)};
+    sd = ff_add(sd, od);
+    sR = ff_add(sR, oR);
+  }
+  if (lane == 0) {
+    sd_s[warp] = sd;
+    sR_s[warp] = sR;
+  }
+  // ---- column sums of Q_b1 ----
+  if (has_b1 && a.csum1) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int v = sub_addi<LPR>(cs[j]);
+      if (sub == 0 && v) atomicAdd(&csum_s[o * 8 + j], v);
+    }
+  }
+  __syncthreads();  // hz, hr of every row are in global memory; sums in shared
+  if (a.hz) {
+    sd = {0.0f, 0.0f};
+    sR = {0.0f, 0.0f};
+    for (int w2 = 0; w2 < NW; ++w2) {
+      sd = ff_add(sd, sd_s[w2]);
+      sR = ff_add(sR, sR_s[w2]);
+    }
+    const HhConst hcst = hh_const(nb);
+    const ff rsd = ff_mul(hcst.rho, sd);
+    const ff rsR = ff_mul(hcst.rho, sR);
+    const ff wd = ff_add(rsd, {-dp_s, 0.0f});
+    const ff wR = ff_add(rsR, ff_neg(Rp_s));
+    const ff kd = ff_mul(hcst.kap, wd), kR = ff_mul(hcst.kap, wR);
+    for (int r = tid; r < nb; r += blockDim.x) {
+      const int64_t row = k0 + r;
+      if (r == 0) {
+        a.hz[row] = ff_round(rsd);
+        a.hr[row] = ff_round(rsR);
+      } else {
+        const float dr = a.hz[row], Rr = a.hr[row];
+        a.hz[row] = ff_round(ff_add({dr, 0.0f}, ff_neg(kd)));
+        a.hr[row] = ff_round(ff_add({Rr, 0.0f}, ff_neg(kR)));
+      }
+    }
+  }
+  if (__any_sync(0xffffffffu, badp) && lane == 0) record_status(a.status, FQT_EINVAL);
+  if (has_b1 && a.csum1)
+    for (int i = tid; i < C; i += blockDim.x)
+      if (csum_s[i]) atomicAdd(&a.csum1[i], csum_s[i]);
+}
+
 struct GroupScratch {
   uint32_t *k0, *k1;
   int32_t *v0, *v1;
@@ -984,12 +1277,17 @@ fqt_status launch_bhq_groups(QuantArgs &a, bool bf16, int num_sms, cudaStream_t 
   if (CO != 8 && CO != 16 && CO != 32) return FQT_EUNSUPPORTED;
   const int grid = num_sms * 2;
   const size_t smem = sizeof(int) * (size_t)a.C;
+  const int64_t bgrid = big_grid(a.N);
+  if (bgrid > 0x7fffffff) return FQT_EUNSUPPORTED;
 #define FQT_BG(L)                                                                      \
   if (CO == L) {                                                                       \
-    if (bf16)                                                                          \
+    if (bf16) {                                                                        \
       k_bhq_groups<__nv_bfloat16, L><<<grid, 256, smem, st>>>(a);                      \
-    else                                                                               \
+      k_bhq_groups_big<__nv_bfloat16, L><<<(int)bgrid, 256, smem, st>>>(a);            \
+    } else {                                                                           \
       k_bhq_groups<float, L><<<grid, 256, smem, st>>>(a);                              \
+      k_bhq_groups_big<float, L><<<(int)bgrid, 256, smem, st>>>(a);                    \
+    }                                                                                  \
   }
   FQT_BG(8)
   FQT_BG(16)

@@ -73,6 +73,12 @@ cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
                                int C, int bits, int block, cudaStream_t st);
 
 size_t group_workspace_bytes(int64_t N);
+// grad_X work lists of the adaptive groups: two counters, the groups of up to
+// 32 rows (at most N) and the larger ones (at most N / 33)
+inline size_t group_list_bytes(int64_t N) {
+  const size_t n = N > 0 ? (size_t)N : 0;
+  return 256 + ((n * 4 + 255) & ~(size_t)255) + (n / 32 + 1) * 4;
+}
 fqt_status launch_bhq_grouping(const void *dH, bool bf16, int64_t N, int C, int32_t *perm,
                                int32_t *gstart, int32_t *gsize, void *scratch,
                                size_t scratch_bytes, unsigned **slot_counter, cudaStream_t st);

@@ -411,6 +411,14 @@ def _adaptive_cases():
     out.append(("cfg0-128", wl.config(0)[0].dH[:, :128].copy()))
     out.append(("cfg1-b2", wl.config(1, batch=2)[0].dH))
     out.append(("cfg2-b1", wl.config(2, batch=1)[0].dH))
+    # row scales spread over orders of magnitude: groups of 33 .. 64 rows
+    # (a warp's quantizer, a CTA's fix-up) and of 65 .. 591 rows (a CTA each)
+    ln = g.standard_normal((20000, 64)) * np.exp(3.0 * g.standard_normal((20000, 1)))
+    out.append(("lognormal-rows-20000x64", ln.astype(np.float32)))
+    # a few outlier rows among many small ones: a handful of groups of 250+
+    ol = 1e-3 * g.standard_normal((6000, 128))
+    ol[:5] *= 1e4
+    out.append(("outliers-6000x128", ol.astype(np.float32)))
     return out
 
 
