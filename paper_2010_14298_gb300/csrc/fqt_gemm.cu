@@ -35,14 +35,35 @@ namespace fqt {
 
 constexpr int BM = 128, BN = 128, BK = 64;
 constexpr int kMaxStages = 8;  // operand stages (A and B fp16 tiles), chosen per launch
-constexpr int kWarpTma = 0, kWarpMma = 1, kWarpEpi0 = 2;
-// grad_X: three sets of four epilogue warps (one per TMEM lane quadrant) take
-// the tiles in turn; split-K partials use the first eight
-constexpr int kGradxSets = 3;
-constexpr int kNumEpiWarps = 4 * kGradxSets;
+constexpr int kWarpTma = 0, kWarpMma = 1, kWarpEpi0 = 2;  // k_gradw's roles
 constexpr int kPartialEpiWarps = 8;
-constexpr int kWarpPar = kWarpEpi0 + kNumEpiWarps;  // grad_X: per-tile parameter loader
-constexpr int kGemmThreads = 32 * (kWarpPar + 1);
+// k_gemm: warpgroup 0 holds the TMA producer, the MMA issuer and grad_X's
+// per-tile parameter loader (warp 3 idles); the epilogue warps follow in
+// sets of four (one per TMEM lane quadrant) that take the tiles in turn.
+// The epilogue's arithmetic comes in three forms (FORM):
+//   0  int64 integer parts for every tile (several exact chunks, large C);
+//   1  the fp32 form for tiles whose row offsets allow it, int64 for the
+//      others, in the same epilogue (the fp32 form's offset bound is small);
+//   2  the fp32 form only: the rare tiles outside it are stored raw and
+//      finished by the CTA after its last tile (gradx_raw_fix).
+// FORM 2 has four sets: without the int64 path, warpgroup 0 can hand
+// registers to the epilogue warpgroups (setmaxnreg) and 104 per thread
+// suffice; tiles with a long reduction use three of the sets (g.sets), so
+// that the tensor cores fill a fourth accumulator while three are drained.
+// Otherwise three sets at 128 registers; split-K partials use the first
+// eight epilogue warps.
+constexpr int kGemmWarpPar = 2, kGemmWarpEpi0 = 4;
+template <int MODE, int FORM>
+struct GemmLayout {
+  static constexpr int sets = (MODE == 0 && FORM == 2) ? 4 : 3;  // MODE 0: grad_X
+  static constexpr int threads = 32 * (kGemmWarpEpi0 + 4 * sets);
+  // registers per thread of the launch, and the split (0: no setmaxnreg)
+  static constexpr int launch_regs = ((65536 / threads) / 8) * 8;
+  static constexpr int regs_ctl = sets == 4 ? 64 : 0;
+  static constexpr int regs_epi = sets == 4 ? 104 : 0;
+  static_assert(regs_ctl == 0 || 128 * regs_ctl + 32 * 4 * sets * regs_epi <= threads * launch_regs,
+                "register split above the launch's registers");
+};
 // two 128-column fp32 accumulators and 256 columns of int32 running sums
 constexpr uint32_t kTmemCols = 512;
 
@@ -64,11 +85,16 @@ constexpr size_t kOffBar = kOffPar + kParStages * kParBytes;
 // operand full / empty, accumulator full / empty (4 each), parameter full /
 // empty (4 each)
 constexpr size_t kNumBars = 2 * kMaxStages + 16;
-constexpr size_t kFixedBytes = (kOffBar + kNumBars * 8 + 16 + 1023) & ~(size_t)1023;
+// grad_X in the fp32 form with fixed blocks: one bit per tile of this CTA
+// (in its order) for the tiles left raw, finished by the CTA at the end
+constexpr size_t kOffRaw = (kOffBar + kNumBars * 8 + 16 + 15) & ~(size_t)15;
+constexpr size_t kRawMaskBytes = 4096;
+constexpr int64_t kMaxLocalTiles = (int64_t)kRawMaskBytes * 8;
+constexpr size_t kFixedBytes = (kOffRaw + kRawMaskBytes + 1023) & ~(size_t)1023;
 
 __host__ __device__ constexpr size_t gemm_smem_bytes(int stages, int ring) {
   return kFixedBytes + (size_t)stages * 2 * kTileBytes +
-         (size_t)kNumEpiWarps * ring * kBoxBytes + 1024;  // + alignment slack
+         (size_t)kPartialEpiWarps * ring * kBoxBytes + 1024;  // + alignment slack
 }
 
 // MODE_GRADX: grad_X^T = W~^T Q_b2(dH)^T, i.e. M = D (output columns of
@@ -101,6 +127,9 @@ struct GemmArgs {
   const int32_t *col_sum_w;    // W~ column sums over C
   const float *inv_sw, *zero_w;
   float *out;                  // grad_X (N x M row-major) for MODE_GRADX
+  int sets;                    // grad_X epilogue sets in use (3 or 4)
+  int bw, b2;                  // code bits of W~ and of Q_b2
+  int small_p;                 // every |P| < 2^22 (block sums off the fp32 bits)
   int *status;
 };
 
@@ -641,11 +670,14 @@ __device__ __forceinline__ float reflect_f(float P, const float4 &kq, float cwc,
 
 // The final chunk of one tile in the fp32 form (one exact chunk, |P| < 2^22,
 // |m| <= mmax).  Block sums S = sum P + CWc sum m, I_p = P_p + m_p CWc.
+// raw: a tile outside the fp32 form, whose row terms are units (1, 0, 0, 0):
+// no block is transformed, so the stores are its exact products P.
 template <int NB>
 __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, uint32_t acc,
                                              const float4 *kp, const int *leads,
                                              const int *msum, const HhConst &hc, float cwc,
-                                             float U, uint64_t *acce_set, int q, int lane) {
+                                             float U, uint64_t *acce_set, int q, int lane,
+                                             bool raw) {
   constexpr int GW = NB > 32 ? NB : 32;
   constexpr int NPP = leads_per_box(NB);
   constexpr int NBD = NB > 1 ? NB : 1;
@@ -696,7 +728,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
           const int kb0 = r0 + b * NBD;
           const int64_t lb = g.N - (t.n0 + kb0);
           const int nact = lb >= NBD ? NBD : (int)(lb > 0 ? lb : 0);
-          if (nact < 2) {  // a one-row block is not transformed
+          if (nact < 2 || raw) {  // a one-row block is not transformed
 #pragma unroll
             for (int l = 0; l < NBD; ++l) {
               const float4 kq = kp[kb0 + l];
@@ -807,7 +839,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
           const int nact = left >= NBD ? NBD : (int)(left > 0 ? left : 0);
           lp[b] = -1;
           lv[b] = 0.0f;
-          if (nact < 2) {  // a one-row block is not transformed
+          if (nact < 2 || raw) {  // a one-row block is not transformed
 #pragma unroll
             for (int l = 0; l < NBD; ++l) {
               const float4 kq = kp[kb0 + l];
@@ -838,7 +870,7 @@ __device__ __forceinline__ void gradx_tile_f(const GemmArgs &g, const Item &t, u
       } else {
         const int64_t left = g.N - (t.n0 + g0);
         const int nact = left >= NB ? NB : (int)(left > 0 ? left : 0);
-        if (nact < 2) {
+        if (nact < 2 || raw) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const float4 kq = kp[r0 + i];
@@ -920,10 +952,11 @@ __device__ __forceinline__ void tile_loads(const GemmArgs &g, const Item &t, int
 // order, the per-row terms of its rows and the column sums of its columns go
 // into a parameter stage ahead of the epilogue warps that use them.  The
 // global loads of the next tile are in flight while this tile's are used.
-template <int NB, bool FLT>
+template <int NB, int FORM>
 __device__ __forceinline__ void gradx_params(const GemmArgs &g, uint8_t *smem, uint64_t *pfull,
                                              uint64_t *pempty, volatile int *abort_flag,
                                              int lane) {
+  uint32_t *raw_mask = reinterpret_cast<uint32_t *>(smem + kOffRaw);
   const float inv_sw = *g.inv_sw, zw = *g.zero_w;
   const ff y = two_sum((float)g.ow, zw);
   const int Cn = (int)g.K;
@@ -1011,15 +1044,25 @@ __device__ __forceinline__ void gradx_params(const GemmArgs &g, uint8_t *smem, u
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1)
       mabs = fmaxf(mabs, __shfl_xor_sync(0xffffffffu, mabs, off));
+    // fp32 form with fixed blocks: a tile with a row offset beyond it keeps
+    // the exact products P (unit row terms); its bit sends it to the CTA's
+    // final pass (gradx_raw_fix)
+    const bool raw = FORM == 2 && NB != 0 && !(mabs <= g.flt_mmax);
+    if (raw) {
+#pragma unroll
+      for (int i = 0; i < BN / 32; ++i) kp[lane + 32 * i] = make_float4(1.0f, 0.0f, 0.0f, 0.0f);
+      if (lane == 0 && local < kMaxLocalTiles) raw_mask[local >> 5] |= 1u << (local & 31);
+    }
     if (lane == 0)
-      *reinterpret_cast<int *>(P + kParFlag) = NB == 0 || (FLT && mabs <= g.flt_mmax);
+      *reinterpret_cast<int *>(P + kParFlag) =
+          NB == 0 || (FORM == 2 && !raw) || (FORM == 1 && mabs <= g.flt_mmax);
     __syncwarp();
     if (lane == 0) mbar_arrive(&pfull[s]);
     cur = nxt;
   }
 }
 
-template <int NB, bool FLT>
+template <int NB, int FORM>
 __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
                                                uint8_t *ring, uint64_t *accf,
                                                uint64_t *acce, uint64_t *pfull,
@@ -1027,18 +1070,19 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
                                                const CUtensorMap *tmOut,
                                                volatile int *abort_flag, int warp,
                                                int lane) {
-  const int ew = warp - kWarpEpi0;
+  const int ew = warp - kGemmWarpEpi0;
   const int q = warp & 3;     // TMEM lane quadrant: columns j = 32q .. 32q + 31
-  const int set = ew >> 2;    // the tiles (every third one) this warp serves
+  const int set = ew >> 2;    // the tiles (every g.sets-th one) this warp serves
   const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
   const float zw = *g.zero_w;
   const int Cn = (int)g.K;
   HhConst hc = {{0.0f, 0.0f}, {0.0f, 0.0f}};
   if (NB > 1) hc = hh_const(NB);
   bool ok = true;
-  int64_t local = 0;
-  for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
-    if ((int)(local % kGradxSets) != set) continue;
+  // this CTA's tiles local = set, set + g.sets, ... (item blockIdx.x + local * grid)
+  for (int64_t local = set; set < g.sets; local += g.sets) {
+    const int64_t it = (int64_t)blockIdx.x + local * (int64_t)gridDim.x;
+    if (it >= g.n_items || *abort_flag) break;
     const Item t = decode_item(g, it);
     const int buf = (int)(local & (g.nacc - 1));
     const uint32_t acc = lane_base + (uint32_t)(buf * BN);
@@ -1054,7 +1098,7 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
     const int *leads = reinterpret_cast<const int *>(P + kParLeads);
     const int *msum = reinterpret_cast<const int *>(P + kParMsum);
     const int cs = reinterpret_cast<const int *>(P + kParCs)[q * 32 + lane];
-    const bool tile_f = FLT && *reinterpret_cast<const int *>(P + kParFlag) != 0;
+    const bool tile_f = FORM != 0 && *reinterpret_cast<const int *>(P + kParFlag) != 0;
     const float cwc = (float)(cs - Cn * g.ow);
     const float U = __fmaf_rn((float)Cn, zw, (float)cs);
     for (int64_t c = 0; c < nchunks; ++c) {
@@ -1095,13 +1139,18 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
       }
       const bool multi = c > 0;
       if constexpr (NB == 0) {
-        gradx_tile_f<0>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane);
+        gradx_tile_f<0>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane, false);
       } else {
-        if (FLT && tile_f)
-          gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane);
-        else
+        if constexpr (FORM == 2) {
+          // a tile outside the fp32 form has unit row terms (kq = (1, 0, 0, 0)):
+          // the one-row epilogue stores its exact products P for gradx_raw_fix
+          gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane, !tile_f);
+        } else if (FORM == 1 && tile_f) {
+          gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane, false);
+        } else {
           gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, &acce[buf], q,
                                 lane);
+        }
       }
     }
     // the parameter stage is free again
@@ -1122,7 +1171,7 @@ __device__ __forceinline__ void partial_epilogue(const GemmArgs &g, uint8_t *rin
                                                  uint32_t tmem, const CUtensorMap *tmOut,
                                                  volatile int *abort_flag, int warp,
                                                  int lane) {
-  const int ew = warp - kWarpEpi0;
+  const int ew = warp - kGemmWarpEpi0;
   const int q = warp & 3;
   const int hcol = ew >> 2;  // column half: 64 * hcol .. +63
   uint8_t *myring = ring + (size_t)ew * g.ring * kBoxBytes;
@@ -1200,8 +1249,14 @@ __device__ __forceinline__ void partial_epilogue(const GemmArgs &g, uint8_t *rin
   __syncwarp();
 }
 
-template <int MODE, int NB, bool FLT>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// The tiles of this CTA left raw by the fp32-form epilogue (defined with the
+// group fix-up, whose arithmetic it shares).
+template <int NB>
+__device__ __noinline__ void gradx_raw_fix(const GemmArgs &g, const uint32_t *raw_mask, int ew,
+                                           int nwarps, int lane);
+
+template <int MODE, int NB, int FORM>
+__global__ void __launch_bounds__(GemmLayout<MODE, FORM>::threads, 1)
     k_gemm(const __grid_constant__ CUtensorMap tmA,
            const __grid_constant__ CUtensorMap tmB,
            const __grid_constant__ CUtensorMap tmOut, const GemmArgs g) {
@@ -1237,6 +1292,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
+  if (MODE == MODE_GRADX && FORM == 2 && NB != 0)
+    for (int i = threadIdx.x; i < (int)(kRawMaskBytes / 4); i += blockDim.x)
+      reinterpret_cast<uint32_t *>(smem + kOffRaw)[i] = 0u;
   if (warp == kWarpMma) {
     asm volatile(
         "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -1249,9 +1307,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  using LY = GemmLayout<MODE, FORM>;
 
   auto fail = [&]() { *abort_flag = 1; };
 
+  // Every warp of a warpgroup executes the same setmaxnreg, and each role's
+  // code follows its own warpgroup's setmaxnreg.
+  if (warp >= kGemmWarpEpi0) {
+    if constexpr (LY::regs_epi > 0)
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(LY::regs_epi));
+    if (MODE == MODE_GRADX) {
+      gradx_epilogue<NB, FORM>(g, smem, ring, accf, acce, pfull, pempty, tmem, &tmOut,
+                               abort_flag, warp, lane);
+      if constexpr (FORM == 2 && NB != 0) {
+        // every epilogue warp arrives here once; then the tiles left raw
+        // (their products stored by this CTA) are finished
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * 4 * LY::sets) : "memory");
+        if (!*abort_flag)
+          gradx_raw_fix<NB>(g, reinterpret_cast<const uint32_t *>(smem + kOffRaw),
+                            warp - kGemmWarpEpi0, 4 * LY::sets, lane);
+      }
+    }
+    else if (warp < kGemmWarpEpi0 + kPartialEpiWarps)
+      partial_epilogue(g, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
+  } else {
+  if constexpr (LY::regs_ctl > 0)
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(LY::regs_ctl));
   if (warp == kWarpTma) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
@@ -1336,14 +1417,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
       }
     }
-  } else if (warp == kWarpPar) {
-    if (MODE == MODE_GRADX) gradx_params<NB, FLT>(g, smem, pfull, pempty, abort_flag, lane);
-  } else if (warp >= kWarpEpi0) {
-    if (MODE == MODE_GRADX)
-      gradx_epilogue<NB, FLT>(g, smem, ring, accf, acce, pfull, pempty, tmem, &tmOut,
-                              abort_flag, warp, lane);
-    else if (warp < kWarpEpi0 + kPartialEpiWarps)
-      partial_epilogue(g, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
+  } else if (warp == kGemmWarpPar) {
+    if (MODE == MODE_GRADX) gradx_params<NB, FORM>(g, smem, pfull, pempty, abort_flag, lane);
+  }
   }
 
   tc_fence_before();
@@ -1563,14 +1639,26 @@ typedef void (*GemmKernel)(CUtensorMap, CUtensorMap, CUtensorMap, GemmArgs);
 
 // The kernel instance of a mode, BHQ block size (1 = no reflection) and
 // product representation (fp32-exact or int32).
-static GemmKernel gemm_kernel(int mode, int nb, bool flt) {
-  if (mode == MODE_PARTIAL) return k_gemm<MODE_PARTIAL, 1, false>;
+// The epilogue form (see GemmLayout) of a contraction whose fp32 form holds
+// rows with |m| <= mmax, for codes of b bits.  A row whose values straddle 0
+// has z' in [-(2^b - 1), 0], so |m| <= 2^(b-1): with mmax at least that, only
+// rows of one sign far from 0 leave the form, and form 2 finishes them in a
+// final pass; otherwise many tiles can, and form 1 keeps both paths.
+static int epilogue_form(bool flt, double mmax, int b) {
+  if (!flt) return 0;
+  return mmax >= (double)(1 << (b - 1)) ? 2 : 1;
+}
+
+static GemmKernel gemm_kernel(int mode, int nb, int form) {
+  if (mode == MODE_PARTIAL) return k_gemm<MODE_PARTIAL, 1, 0>;
 #define FQT_GX(NBV)                                                          \
   case NBV:                                                                  \
-    return flt ? k_gemm<MODE_GRADX, NBV, true> : k_gemm<MODE_GRADX, NBV, false>;
+    return form == 2   ? k_gemm<MODE_GRADX, NBV, 2>                           \
+           : form == 1 ? k_gemm<MODE_GRADX, NBV, 1>                           \
+                       : k_gemm<MODE_GRADX, NBV, 0>;
   switch (nb) {
-    case 0:  // adaptive BHQ groups: fp32 form only
-      return flt ? k_gemm<MODE_GRADX, 0, true> : nullptr;
+    case 0:  // adaptive BHQ groups: fp32 form only (raw rows go to the group pass)
+      return form == 2 ? k_gemm<MODE_GRADX, 0, 2> : nullptr;
     FQT_GX(1)
     FQT_GX(2)
     FQT_GX(4)
@@ -1591,7 +1679,7 @@ static GemmKernel gemm_kernel(int mode, int nb, bool flt) {
 static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
                            const uint16_t *Bm, int b_kmajor, int b_bits, int64_t M,
                            int64_t N, int64_t K, const SplitPlan &p, GemmArgs &g,
-                           void *out, int mode, int nb, bool flt, cudaStream_t st) {
+                           void *out, int mode, int nb, int form, cudaStream_t st) {
   const bool partial = mode == MODE_PARTIAL;
   CUtensorMap ta, tb;
   bool ok = a_kmajor ? make_map_f16(&ta, A, (uint64_t)K, (uint64_t)M, BK, BM)
@@ -1603,8 +1691,26 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
                                      (uint64_t)p.splits)
                       : make_map_out(&to, out, false, (uint64_t)M, (uint64_t)N, 1));
   if (!ok) return cuda_fail(cudaErrorInvalidValue, "tensor map encode");
-  GemmKernel kern = gemm_kernel(mode, nb, flt);
+  GemmKernel kern = gemm_kernel(mode, nb, form);
   if (!kern) return FQT_EUNSUPPORTED;
+  const bool four = !partial && form == 2;  // GemmLayout: four epilogue sets
+  const int threads = four ? GemmLayout<0, 2>::threads : GemmLayout<0, 0>::threads;
+  if (four) {
+    // the register split needs the launch's registers per thread: with fewer,
+    // setmaxnreg.inc would wait for registers that do not exist
+    using LY = GemmLayout<0, 2>;
+    cudaFuncAttributes fa;
+    const cudaError_t e = cudaFuncGetAttributes(&fa, kern);
+    if (e != cudaSuccess) return cuda_fail(e, "gemm attributes");
+    if ((int64_t)fa.numRegs * LY::threads < 128 * LY::regs_ctl + 32 * 4 * LY::sets * LY::regs_epi)
+      return FQT_EUNSUPPORTED;
+  }
+  // the fp32 form: four epilogue sets for tiles bound by their output, three
+  // for long reductions; the code bits for the final pass over raw tiles
+  g.sets = (four && (K + BK - 1) / BK <= 2) ? 4 : 3;
+  g.bw = a_bits;
+  g.b2 = b_bits;
+  g.small_p = (K << (a_bits + b_bits - 2)) < ((int64_t)1 << 22);
   // HBM-bound output tiles (grad_X): deep store ring; long reductions
   // (split-K partials): deep operand ring
   g.stages = partial ? 5 : 2;
@@ -1643,7 +1749,9 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   const int nsm = device_sm_count();
   int64_t grid = g.n_items < nsm ? g.n_items : nsm;
   if (grid < 1) grid = 1;
-  kern<<<(int)grid, kGemmThreads, smem, st>>>(ta, tb, to, g);
+  // the raw-tile bits of a CTA cover kMaxLocalTiles of its tiles
+  if (four && nb != 0 && (g.n_items + grid - 1) / grid > kMaxLocalTiles) return FQT_EUNSUPPORTED;
+  kern<<<(int)grid, threads, smem, st>>>(ta, tb, to, g);
   return cuda_fail(cudaGetLastError(), "gemm launch");
 }
 
@@ -2067,7 +2175,7 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
   g.zero_w = qw->zero;
   g.flt_mmax = flt ? (float)mmax : -1.0f;
   return run_gemm(qw->codes_f16, 1, qw->bits, qx->codes_f16, 1, qx->bits, C, Nr, D, p, g, H,
-                  MODE_GRADX, 1, flt, st);
+                  MODE_GRADX, 1, epilogue_form(flt, mmax, qx->bits), st);
 }
 
 // ---------------------------------------------------------------------------
@@ -2154,6 +2262,10 @@ struct FixArgs {
   float mmax_nb[33];  // groups of nb <= 32 rows: largest |m| of the fp32 form
   int32_t *list, *list_big;
   int *count, *count_big;
+  // fixed blocks (gradx_raw_fix): block size, per-tensor Q_b2 metadata
+  // (PTQ) and the lead row of every block
+  int nbk, per_tensor;
+  const int32_t *lead;
   int *status;
 };
 
@@ -2162,13 +2274,19 @@ struct RowTerms {
   float sc, hd, hR, m;
 };
 
+__device__ __forceinline__ float zero_of(const FixArgs &f, int64_t k) {
+  return f.zero[f.per_tensor ? 0 : k];
+}
+
 __device__ __forceinline__ RowTerms row_terms(const FixArgs &f, int64_t k, float inv_sw,
                                               bool reflected) {
   RowTerms t;
-  t.sc = __fmul_rn(inv_sw, f.inv_s[k]);
-  const ff x = two_sum((float)f.og, f.zero[k]);
+  t.sc = __fmul_rn(inv_sw, f.inv_s[f.per_tensor ? 0 : k]);
+  const ff x = two_sum((float)f.og, zero_of(f, k));
   t.m = rintf(x.h);
-  if (reflected) {
+  // BHQ rows (no row sums here) read their offsets from hz, hr even for a
+  // one-row block, where they are the unreflected d and R
+  if (reflected || !f.row_sum) {
     t.hd = f.hz[k];
     t.hR = f.hr[k];
   } else {
@@ -2207,11 +2325,13 @@ __global__ void __launch_bounds__(256) k_grp_list(const FixArgs f) {
 }
 
 // Any group (or a single row left raw): rows visited one by one; the fp32
-// form where it is exact, else int64 integer parts and float-float.
+// form where it is exact, else int64 integer parts and float-float.  The
+// lead row is row `lead` of the group (0 for the stored groups); rows are
+// perm[k] of grad_X, or k itself without perm.
 __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int nb, int64_t j,
                                                bool jv, const float (&cwc)[4],
                                                const int (&cwi)[4], const float (&U)[4],
-                                               float inv_sw, const ff &y) {
+                                               float inv_sw, const ff &y, int lead) {
   const int lane = threadIdx.x & 31;
   const int Cn = f.C;
   const bool refl = nb >= 2;
@@ -2222,13 +2342,13 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
     const double mmax = floor(lim / ((double)Cn * (double)(1 << (f.bw - 1)))) -
                         (double)(1 << (f.b2 - 1)) - 1.0;
     for (int r = lane; r < nb; r += 32) {
-      const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
+      const float m = rintf(two_sum((float)f.og, zero_of(f, k0 + r)).h);
       if (!((double)fabsf(m) <= mmax)) fast = false;
     }
     fast = __all_sync(0xffffffffu, fast);
   }
   auto prow = [&](int r) -> float * {
-    int64_t pr = f.perm[k0 + r];
+    int64_t pr = f.perm ? (int64_t)f.perm[k0 + r] : k0 + r;
     if (pr < 0 || pr >= f.N) pr = 0;
     return f.out + pr * f.D + j;
   };
@@ -2237,7 +2357,7 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
     uint32_t sb[4] = {0u, 0u, 0u, 0u};
     int msum = 0, Ip[4] = {0, 0, 0, 0};
     for (int r = 0; r < nb; ++r) {
-      const float m = rintf(two_sum((float)f.og, f.zero[k0 + r]).h);
+      const float m = rintf(two_sum((float)f.og, zero_of(f, k0 + r)).h);
       msum += (int)m;
       if (!jv) continue;
       const float4 P = *reinterpret_cast<const float4 *>(prow(r));
@@ -2245,7 +2365,7 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         sb[c] += magic_bits(pv[c]);
-        if (r == 0) Ip[c] = magic_int(pv[c]) + (int)m * cwi[c];
+        if (r == lead) Ip[c] = magic_int(pv[c]) + (int)m * cwi[c];
       }
     }
     BlockFixF bf[4];
@@ -2266,7 +2386,7 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
       float o4[4];
 #pragma unroll
       for (int c = 0; c < 4; ++c)
-        o4[c] = r == 0 ? dequant(kq, bf[c].lead, U[c])
+        o4[c] = r == lead ? dequant(kq, bf[c].lead, U[c])
                        : dequant(kq, reflect_f(pv[c], kq, cwc[c], bf[c]), U[c]);
       __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
     }
@@ -2274,14 +2394,14 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
     // int64 integer parts I = P + m CWc, float-float reflection
     long long S[4] = {0, 0, 0, 0}, Ipl[4] = {0, 0, 0, 0};
     for (int r = 0; r < nb && jv; ++r) {
-      const long long m = __float2ll_rn(rintf(two_sum((float)f.og, f.zero[k0 + r]).h));
+      const long long m = __float2ll_rn(rintf(two_sum((float)f.og, zero_of(f, k0 + r)).h));
       const float4 P = *reinterpret_cast<const float4 *>(prow(r));
       const float pv[4] = {P.x, P.y, P.z, P.w};
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         const long long I = (long long)__float2int_rn(pv[c]) + m * cwi[c];
         S[c] += I;
-        if (r == 0) Ipl[c] = I;
+        if (r == lead) Ipl[c] = I;
       }
     }
     ff rS[4], beta[4];
@@ -2303,12 +2423,86 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         const ff I = ff_from_int((long long)__float2int_rn(pv[c]) + m * cwi[c]);
-        ff v = !refl ? I : (r == 0 ? rS[c] : ff_add(I, ff_neg(beta[c])));
+        ff v = !refl ? I : (r == lead ? rS[c] : ff_add(I, ff_neg(beta[c])));
         v = ff_add(v, two_prod(t.hd, U[c]));
         v = ff_add(v, ff_mul({t.hR, 0.0f}, y));
         o4[c] = __fmul_rn(t.sc, ff_round(v));
       }
       __stcs(reinterpret_cast<float4 *>(po), make_float4(o4[0], o4[1], o4[2], o4[3]));
+    }
+  }
+}
+
+// Tiles of a fixed-block grad_X (or of the forward) in the fp32 form that the
+// contraction left raw (a row offset m beyond the form): after its last
+// tile, every epilogue warp of the CTA takes every nwarps-th (tile, block)
+// unit of the CTA's raw tiles -- each lane 4 of the tile's 128 columns --
+// with the arithmetic of fix_group_general (int64 integer parts and
+// float-float where the fp32 form is not exact).  NB = 1: one row per unit.
+template <int NB>
+__device__ __noinline__ void gradx_raw_fix(const GemmArgs &g, const uint32_t *raw_mask, int ew,
+                                           int nwarps, int lane) {
+  constexpr int NBD = NB > 1 ? NB : 1;
+  constexpr int BPT = BN / NBD;  // units per tile
+  int64_t n_local = (g.n_items - (int64_t)blockIdx.x + gridDim.x - 1) / gridDim.x;
+  if (n_local > kMaxLocalTiles) n_local = kMaxLocalTiles;
+  const int nwords = (int)((n_local + 31) / 32);
+  bool any = false;
+  for (int w = 0; w < nwords; ++w) any |= raw_mask[w] != 0u;
+  if (!any) return;
+  FixArgs f;
+  memset(&f, 0, sizeof(f));
+  f.out = g.out;
+  f.N = g.N;
+  f.D = g.M;
+  f.C = (int)g.K;
+  f.og = g.og;
+  f.ow = g.ow;
+  f.bw = g.bw;
+  f.b2 = g.b2;
+  f.inv_s = g.inv_s;
+  f.zero = g.zero;
+  f.hz = g.hz;
+  f.hr = g.hr;
+  f.row_sum = NB > 1 ? nullptr : g.row_sum;
+  f.inv_sw = g.inv_sw;
+  f.zero_w = g.zero_w;
+  f.col_sum_w = g.col_sum_w;
+  f.small_p = g.small_p;
+  f.nbk = NB;
+  f.per_tensor = g.kind == FQT_PTQ;
+  f.lead = g.lead;
+  f.status = g.status;
+  const float inv_sw = *g.inv_sw, zw = *g.zero_w;
+  const ff y = two_sum((float)g.ow, zw);
+  const int Cn = (int)g.K;
+  int64_t u = 0;
+  for (int w = 0; w < nwords; ++w) {
+    uint32_t bits = raw_mask[w];
+    while (bits) {
+      const int l = w * 32 + __ffs(bits) - 1;
+      bits &= bits - 1u;
+      const Item t = decode_item(g, (int64_t)blockIdx.x + (int64_t)l * gridDim.x);
+      for (int b = 0; b < BPT; ++b, ++u) {
+        if ((int)(u % nwarps) != ew) continue;
+        const int64_t k0 = t.n0 + (int64_t)b * NBD;
+        if (k0 >= g.N) continue;
+        const int nb = (int)min((int64_t)NBD, g.N - k0);
+        const int64_t j = t.m0 + lane * 4;
+        const bool jv = j < g.M;
+        float cwc[4], U[4];
+        int cwi[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int cs = jv ? g.col_sum_w[j + c] : 0;
+          cwc[c] = (float)(cs - Cn * g.ow);
+          cwi[c] = (int)cwc[c];
+          U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
+        }
+        int lead = NBD > 1 ? g.lead[k0 / NBD] : 0;
+        if (lead < 0 || lead >= nb) lead = 0;
+        fix_group_general(f, k0, nb, j, jv, cwc, cwi, U, inv_sw, y, lead);
+      }
     }
   }
 }
@@ -2502,7 +2696,7 @@ __global__ void __launch_bounds__(256, 3) k_grp_fix(const FixArgs f) {
         U[c] = __fmaf_rn((float)Cn, zw, (float)cs);
       }
       if (!fast) {
-        fix_group_general(f, k0, nb, j, jv, cwc, cwi, U, inv_sw, y);
+        fix_group_general(f, k0, nb, j, jv, cwc, cwi, U, inv_sw, y, 0);
         continue;
       }
       // ---- pass 1: block sums S = sum P + CWc sum m, lead I_p ----
@@ -2629,7 +2823,8 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       g.gsize = q_b2->gsize;
       g.raw_mmax = (float)mmax;
       fqt_status s = run_gemm(qw->codes_f16, 0, qw->bits, q_b2->codes_f16, 1, q_b2->bits,
-                              D, Nr, C, p, g, grad_X, MODE_GRADX, nb, flt, st);
+                              D, Nr, C, p, g, grad_X, MODE_GRADX, nb,
+                              adapt ? 2 : epilogue_form(flt, mmax, q_b2->bits), st);
       if (s != FQT_OK) return s;
       if (adapt) {
         FixArgs f;

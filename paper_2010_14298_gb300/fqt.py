@@ -365,7 +365,7 @@ def linear_forward(qx: QTensor, qw: QTensor, ws: Workspace = None, out: torch.Te
     N, D = qx.shape
     C = qw.shape[0]
     dev = qx.inv_s.device
-    ws = ws or Workspace(1, 16, 16, device=dev)
+    ws = ws or Workspace(N, C, D, device=dev)
     if out is None:
         out = torch.empty((N, C), dtype=torch.float32, device=dev)
     sx, sw = qx.c_struct(), qw.c_struct()

@@ -252,6 +252,59 @@ def test_linear_forward_matches_oracle(cfg, small):
         assert grad_rel_err(H.cpu().numpy(), ref) <= GRAD_TOL
 
 
+def _offset_rows(g, n, c, rows, base=50.0, spread=1e-4):
+    """Rows of one sign with a tiny range: their zero points put the row
+    offset m far beyond the fp32 form of the contraction."""
+    dH = wl.random_grad(g, n, c, sigma=1.0)
+    for i, r in enumerate(rows):
+        dH[r] = (base if i % 2 == 0 else -0.4 * base) + spread * g.standard_normal(c)
+    return dH
+
+
+@pytest.mark.parametrize("kind,bits,block", [(orc.BHQ, 5, 16), (orc.BHQ, 4, 2),
+                                             (orc.BHQ, 5, 128), (orc.PSQ, 8, 0),
+                                             (orc.PSQ, 4, 0)])
+def test_tiles_outside_the_fp32_form(kind, bits, block):
+    """Tiles with a row whose offset m exceeds the fp32 form are stored raw
+    by the contraction and finished by the tile pass (int64 integer parts,
+    float-float reflection); the other tiles stay in the fused epilogue."""
+    g = wl.rng(330 + bits + block)
+    n, c, d = 300, 64, 208  # row tiles 0..127, 128..255, 256..299; ragged columns
+    dH = _offset_rows(g, n, c, [10, 140, 299], base=5000.0, spread=1e-2)
+    X = g.uniform(-1, 1, (n, d)).astype(np.float32)
+    W = (0.05 * g.standard_normal((c, d))).astype(np.float32)
+    L = wl.Layer("offsets", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, kind, bits, block)
+    h2, hw = q2.to_numpy(), qw.to_numpy()
+    m = np.rint(np.float32(2 ** (bits - 1)) + h2["zero"].astype(np.float32))
+    nb = max(block, 1)
+    lim = 2.0 ** 24 / (2.0 + np.sqrt(nb)) if nb > 1 else 2.0 ** 24
+    mmax = np.floor(lim / (c * 2.0 ** 7)) - 2 ** (bits - 1) - 1
+    assert np.abs(m).max() > mmax  # at least one tile leaves the fp32 form
+    assert grad_rel_err(gx, orc.grad_x(h2, hw)) <= GRAD_TOL
+
+
+def test_per_tensor_offset_sends_every_tile_to_the_tile_pass():
+    """PTQ of an all-positive dH with a tiny range: one zero point for all
+    rows, so every tile of grad_X -- and every tile of the forward for an X
+    of that kind -- is finished by the tile pass."""
+    g = wl.rng(341)
+    n, c, d = 260, 64, 144
+    dH = (50.0 + 1e-4 * g.standard_normal((n, c))).astype(np.float32)
+    X = (20.0 + 1e-3 * g.standard_normal((n, d))).astype(np.float32)
+    W = (0.05 * g.standard_normal((c, d))).astype(np.float32)
+    L = wl.Layer("ptq-offset", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.PTQ, 5, 0)
+    assert grad_rel_err(gx, orc.grad_x(q2.to_numpy(), qw.to_numpy())) <= GRAD_TOL
+    qxr = fqt.quantize_act(to_dev(X), 8, row_sum=True)
+    qwr = fqt.quantize_weight(to_dev(W), 8, row_sum=True)
+    H = fqt.linear_forward(qxr, qwr)
+    torch.cuda.synchronize()
+    hx, hwr = qxr.to_numpy(), qwr.to_numpy()
+    ref = orc.matmul(orc.dequant(hx), np.ascontiguousarray(orc.dequant(hwr).T))
+    assert grad_rel_err(H.cpu().numpy(), ref) <= GRAD_TOL
+
+
 def test_ptq_codes_reused_for_grad_w():
     L = wl.config(0)[0]
     qx, qw, q2, q1, gx, gw = _backward(L, orc.PTQ, 8, 0, reuse=True)
