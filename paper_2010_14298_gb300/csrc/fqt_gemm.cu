@@ -48,19 +48,19 @@ constexpr int kPartialEpiWarps = 8;
 //      finished by the CTA after its last tile (gradx_raw_fix).
 // FORM 2 has four sets: without the int64 path, warpgroup 0 can hand
 // registers to the epilogue warpgroups (setmaxnreg) and 104 per thread
-// suffice; tiles with a long reduction use three of the sets (g.sets), so
+// suffice (96 for one-row blocks, whose parameter loader keeps 80); tiles with a long reduction use three of the sets (g.sets), so
 // that the tensor cores fill a fourth accumulator while three are drained.
 // Otherwise three sets at 128 registers; split-K partials use the first
 // eight epilogue warps.
 constexpr int kGemmWarpPar = 2, kGemmWarpEpi0 = 4;
-template <int MODE, int FORM>
+template <int MODE, int FORM, int NB = 16>
 struct GemmLayout {
   static constexpr int sets = (MODE == 0 && FORM == 2) ? 4 : 3;  // MODE 0: grad_X
   static constexpr int threads = 32 * (kGemmWarpEpi0 + 4 * sets);
   // registers per thread of the launch, and the split (0: no setmaxnreg)
   static constexpr int launch_regs = ((65536 / threads) / 8) * 8;
-  static constexpr int regs_ctl = sets == 4 ? 64 : 0;
-  static constexpr int regs_epi = sets == 4 ? 104 : 0;
+  static constexpr int regs_ctl = sets == 4 ? (NB == 1 ? 80 : 64) : 0;
+  static constexpr int regs_epi = sets == 4 ? (NB == 1 ? 96 : 104) : 0;
   static_assert(regs_ctl == 0 || 128 * regs_ctl + 32 * 4 * sets * regs_epi <= threads * launch_regs,
                 "register split above the launch's registers");
 };
@@ -1256,7 +1256,7 @@ __device__ __noinline__ void gradx_raw_fix(const GemmArgs &g, const uint32_t *ra
                                            int nwarps, int lane);
 
 template <int MODE, int NB, int FORM>
-__global__ void __launch_bounds__(GemmLayout<MODE, FORM>::threads, 1)
+__global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
     k_gemm(const __grid_constant__ CUtensorMap tmA,
            const __grid_constant__ CUtensorMap tmB,
            const __grid_constant__ CUtensorMap tmOut, const GemmArgs g) {
@@ -1307,7 +1307,7 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM>::threads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  using LY = GemmLayout<MODE, FORM>;
+  using LY = GemmLayout<MODE, FORM, NB>;
 
   auto fail = [&]() { *abort_flag = 1; };
 
@@ -1698,12 +1698,14 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   if (four) {
     // the register split needs the launch's registers per thread: with fewer,
     // setmaxnreg.inc would wait for registers that do not exist
-    using LY = GemmLayout<0, 2>;
+    using L16 = GemmLayout<0, 2, 16>;
+    using L1 = GemmLayout<0, 2, 1>;
+    const int64_t need = nb == 1 ? 128 * L1::regs_ctl + 32 * 4 * L1::sets * L1::regs_epi
+                                 : 128 * L16::regs_ctl + 32 * 4 * L16::sets * L16::regs_epi;
     cudaFuncAttributes fa;
     const cudaError_t e = cudaFuncGetAttributes(&fa, kern);
     if (e != cudaSuccess) return cuda_fail(e, "gemm attributes");
-    if ((int64_t)fa.numRegs * LY::threads < 128 * LY::regs_ctl + 32 * 4 * LY::sets * LY::regs_epi)
-      return FQT_EUNSUPPORTED;
+    if ((int64_t)fa.numRegs * L16::threads < need) return FQT_EUNSUPPORTED;
   }
   // the fp32 form: four epilogue sets for tiles bound by their output, three
   // for long reductions; the code bits for the final pass over raw tiles
