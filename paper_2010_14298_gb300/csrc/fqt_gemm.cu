@@ -48,7 +48,7 @@ constexpr int kPartialEpiWarps = 8;
 //      finished by the CTA after its last tile (gradx_raw_fix).
 // FORM 2 has four sets: without the int64 path, warpgroup 0 can hand
 // registers to the epilogue warpgroups (setmaxnreg) and 104 per thread
-// suffice (96 for one-row blocks, whose parameter loader keeps 80); tiles with a long reduction use three of the sets (g.sets), so
+// suffice (96 for blocks of up to 16 rows, whose parameter loader keeps 80); tiles with a long reduction use three of the sets (g.sets), so
 // that the tensor cores fill a fourth accumulator while three are drained.
 // Otherwise three sets at 128 registers; split-K partials use the first
 // eight epilogue warps.
@@ -59,8 +59,8 @@ struct GemmLayout {
   static constexpr int threads = 32 * (kGemmWarpEpi0 + 4 * sets);
   // registers per thread of the launch, and the split (0: no setmaxnreg)
   static constexpr int launch_regs = ((65536 / threads) / 8) * 8;
-  static constexpr int regs_ctl = sets == 4 ? (NB == 1 ? 80 : 64) : 0;
-  static constexpr int regs_epi = sets == 4 ? (NB == 1 ? 96 : 104) : 0;
+  static constexpr int regs_ctl = sets == 4 ? (NB <= 16 ? 80 : 64) : 0;
+  static constexpr int regs_epi = sets == 4 ? (NB <= 16 ? 96 : 104) : 0;
   static_assert(regs_ctl == 0 || 128 * regs_ctl + 32 * 4 * sets * regs_epi <= threads * launch_regs,
                 "register split above the launch's registers");
 };
@@ -1699,9 +1699,9 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
     // the register split needs the launch's registers per thread: with fewer,
     // setmaxnreg.inc would wait for registers that do not exist
     using L16 = GemmLayout<0, 2, 16>;
-    using L1 = GemmLayout<0, 2, 1>;
-    const int64_t need = nb == 1 ? 128 * L1::regs_ctl + 32 * 4 * L1::sets * L1::regs_epi
-                                 : 128 * L16::regs_ctl + 32 * 4 * L16::sets * L16::regs_epi;
+    using L32 = GemmLayout<0, 2, 32>;
+    const int64_t need = nb <= 16 ? 128 * L16::regs_ctl + 32 * 4 * L16::sets * L16::regs_epi
+                                  : 128 * L32::regs_ctl + 32 * 4 * L32::sets * L32::regs_epi;
     cudaFuncAttributes fa;
     const cudaError_t e = cudaFuncGetAttributes(&fa, kern);
     if (e != cudaSuccess) return cuda_fail(e, "gemm attributes");

@@ -511,7 +511,7 @@ __device__ __forceinline__ int sub_addi(int v) {
 }
 
 template <typename T, int LPR>
-__global__ void __launch_bounds__(256, 2) k_bhq_groups(const QuantArgs a) {
+__global__ void __launch_bounds__(256, 3) k_bhq_groups(const QuantArgs a) {
   __shared__ float2 red[8];
   __shared__ int redi[8];
   extern __shared__ int csum_s[];  // C column sums of Q_b1
@@ -1275,7 +1275,7 @@ fqt_status launch_bhq_groups(QuantArgs &a, bool bf16, int num_sms, cudaStream_t 
   if (a.C % 8) return FQT_EUNSUPPORTED;
   const int CO = a.C / 8;
   if (CO != 8 && CO != 16 && CO != 32) return FQT_EUNSUPPORTED;
-  const int grid = num_sms * 2;
+  const int grid = num_sms * 3;
   const size_t smem = sizeof(int) * (size_t)a.C;
   const int64_t bgrid = big_grid(a.N);
   if (bgrid > 0x7fffffff) return FQT_EUNSUPPORTED;
