@@ -2643,7 +2643,7 @@ __device__ __forceinline__ float4 ld_row4(const FixArgs &f, int pr, int64_t j, b
             : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
-__global__ void __launch_bounds__(256, 3) k_grp_fix(const FixArgs f) {
+__global__ void __launch_bounds__(256, 4) k_grp_fix(const FixArgs f) {
   const int lane = threadIdx.x & 31;
   const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int nchunk = (int)((f.D + 127) / 128);
