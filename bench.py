@@ -650,6 +650,74 @@ def run_gpu(args):
                 del dHo, Xo, Wo, qxo, qwo, q2o, q1o, gxo, gwo, wso, wfx, wfw
                 torch.cuda.empty_cache()
 
+    # ---- the full ResNet-50 backward sweep at batch 256, 224 x 224: every conv
+    # (and the fc) lowered to im2col, BHQ-5/16 + Q_b1 PTQ-8 gradients, 8-bit
+    # X~ and W~; inputs drawn on the device from the same recipe as
+    # workloads.resnet50_layer (the host draw is 40+ GB) ----
+    sweep = None
+    if args.sweep_steps > 0:
+        import torch.nn.functional as F
+        layers_out = []
+        tot = {"quantize_act": 0.0, "quantize_weight": 0.0, "quantize_grad": 0.0,
+               "grad_x": 0.0, "grad_w": 0.0}
+        ops_all = 0
+        st_all = 0
+        bsz = 256
+        for li, sh in enumerate(wl.resnet50_shapes()):
+            gen = torch.Generator(device=dev)
+            gen.manual_seed(1234 + 4 + li)
+            Ns, Dp, Cp = sh.rows(bsz), sh.D_pad, sh.C_pad
+            x = torch.rand((bsz, sh.cin, sh.h, sh.h), generator=gen, device=dev) * 2.0 - 1.0
+            cols = F.unfold(x, sh.k, padding=sh.pad, stride=sh.stride)
+            del x
+            Xs = torch.zeros((Ns, Dp), dtype=torch.float32, device=dev)
+            Xs[:, :sh.D] = cols.view(bsz, sh.cin, sh.k * sh.k, -1).permute(0, 3, 2, 1).reshape(Ns, sh.D)
+            del cols
+            dHs = torch.zeros((Ns, Cp), dtype=torch.float32, device=dev)
+            dHs[:, :sh.cout] = (torch.randn((Ns, sh.cout), generator=gen, device=dev)
+                                * torch.exp(2.0 * torch.randn((Ns, 1), generator=gen, device=dev)))
+            Ws = torch.zeros((Cp, Dp), dtype=torch.float32, device=dev)
+            Ws[:sh.cout, :sh.D] = (torch.randn((sh.cout, sh.D), generator=gen, device=dev)
+                                   * float(np.sqrt(2.0 / sh.D)))
+            wss = fqt.Workspace(Ns, Cp, Dp, device=dev)
+            qxs = fqt.QTensor.empty(Ns, Dp, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+            qws = fqt.QTensor.empty(Cp, Dp, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+            q2s = fqt.QTensor.empty(Ns, Cp, fqt.BHQ, 5, 16, True, False, dev, u8=False)
+            q1s = fqt.QTensor.empty(Ns, Cp, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+            gxs = torch.empty((Ns, Dp), dtype=torch.float32, device=dev)
+            gws = torch.empty((Cp, Dp), dtype=torch.float32, device=dev)
+            wfxs = fqt.Workspace(Ns, Dp, 16, device=dev)
+            wfws = fqt.Workspace(Cp, Dp, 16, device=dev)
+            fs = [lambda: fqt.quantize_act(Xs, 8, ws=wfxs, out=qxs),
+                  lambda: fqt.quantize_weight(Ws, 8, ws=wfws, out=qws),
+                  lambda: fqt.quantize_grad(dHs, fqt.BHQ, 5, 16, 5, ws=wss, q_b2=q2s, q_b1=q1s),
+                  lambda: fqt.linear_backward(q2s, q1s, qxs, qws, grad_x=True, grad_w=False,
+                                              ws=wss, out_x=gxs),
+                  lambda: fqt.linear_backward(q2s, q1s, qxs, qws, grad_x=False, grad_w=True,
+                                              ws=wss, out_w=gws)]
+            per = time_graphs(fs, args.sweep_steps)
+            for k_, v_ in zip(tot, per):
+                tot[k_] += v_
+            ops_l = 2 * 2 * Ns * sh.cout * sh.D
+            ops_all += ops_l
+            st_all |= fqt.sync_status(wss)
+            layers_out.append({"layer": sh.name, "N": Ns, "C": sh.cout, "D": sh.D,
+                               "backward_ms": per[2] + per[3] + per[4], "grad_x_ms": per[3],
+                               "TOPS": ops_l / ((per[3] + per[4]) * 1e-3) / 1e12})
+            del Xs, dHs, Ws, wss, qxs, qws, q2s, q1s, gxs, gws, wfxs, wfws
+            torch.cuda.empty_cache()
+        bwd = tot["quantize_grad"] + tot["grad_x"] + tot["grad_w"]
+        slow = sorted(layers_out, key=lambda r: -r["backward_ms"])[:5]
+        sweep = {"workload": "ResNet-50 v1.5 backward sweep, batch 256, 224 x 224: 53 convs + fc "
+                             "via im2col (stem D 147 -> 160 and fc C 1000 -> 1008 zero-padded)",
+                 "layers": len(layers_out), "quantizer": "BHQ-5 block 16 + Q_b1 PTQ-8; X~, W~ PTQ-8",
+                 "backward_ms": bwd, "ops": ops_all, "TOPS": ops_all / (bwd * 1e-3) / 1e12,
+                 "per_call_ms_sum": tot,
+                 "forward_quantizers_ms": tot["quantize_act"] + tot["quantize_weight"],
+                 # the stem's grad_X (w.r.t. the image) is not needed in training
+                 "stem_grad_x_ms": next(r for r in layers_out if r["layer"] == "conv1")["grad_x_ms"],
+                 "slowest_layers": slow, "device_status": st_all}
+
     # ---- the paper's own overhead shape (Sec. 4.3): a conv layer with
     # N = 128, C = 64, 56 x 56, i.e. dH of 401408 im2col rows x 64; the paper
     # timed its CPU routines there (context only, another machine) ----
@@ -711,6 +779,7 @@ def run_gpu(args):
         "implicit_im2col": imp,
         "other_workloads": others,
         "paper_overhead_shape": ovh,
+        "resnet50_sweep": sweep,
         "gpu_launches": int(sum(launches_per_call) * args.steps),
         "device_status": status,
     }
@@ -795,6 +864,8 @@ def main():
                     help="timed steps of the shift quantizer path (0: skip)")
     ap.add_argument("--implicit-steps", type=int, default=50,
                     help="timed steps with the implicit im2col X operand (0: skip)")
+    ap.add_argument("--sweep-steps", type=int, default=5,
+                    help="timed rounds per layer of the ResNet-50 sweep (0: skip)")
     ap.add_argument("--config-steps", type=int, default=20,
                     help="timed steps of the other full-size workloads and of the paper's "
                          "overhead shape (0: skip)")

@@ -88,7 +88,89 @@ CONFIG_NAMES = [
     "resnet18-conv3x3-b128-32x32-64ch",
     "resnet50-layer3-conv3x3-b256-14x14-256ch",
     "transformer-ffn-8192tok-1024x4096-bf16",
+    "resnet50-sweep-b256-224x224",
 ]
+
+
+@dataclasses.dataclass(frozen=True)
+class ConvShape:
+    """One layer of the ResNet-50 sweep lowered to im2col: a k x k conv of
+    cin -> cout channels on an h x h input (stride, padding); the final fc is
+    a 1 x 1 conv on a 1 x 1 map."""
+    name: str
+    cin: int
+    cout: int
+    k: int
+    stride: int
+    pad: int
+    h: int
+
+    @property
+    def hout(self) -> int:
+        return (self.h + 2 * self.pad - self.k) // self.stride + 1
+
+    def rows(self, batch: int) -> int:
+        return batch * self.hout * self.hout
+
+    @property
+    def D(self) -> int:  # im2col columns (kh, kw, cin)
+        return self.k * self.k * self.cin
+
+    @property
+    def D_pad(self) -> int:  # to a multiple of 16 for the contractions
+        return (self.D + 15) // 16 * 16
+
+    @property
+    def C_pad(self) -> int:
+        return (self.cout + 15) // 16 * 16
+
+
+def resnet50_shapes() -> List[ConvShape]:
+    """The 53 convolutions of ResNet-50 v1.5 (stride 2 on the 3 x 3 conv of the
+    first bottleneck of a stage; four projection shortcuts) and the fc, at a
+    224 x 224 input, in forward order."""
+    out = [ConvShape("conv1", 3, 64, 7, 2, 3, 224)]
+    cin, h = 64, 56  # after the 3 x 3 / 2 max pool
+    for stage, (blocks, width) in enumerate(((3, 64), (4, 128), (6, 256), (3, 512)), start=1):
+        cout = 4 * width
+        for b in range(blocks):
+            s = 2 if (b == 0 and stage > 1) else 1
+            pre = f"layer{stage}.{b}"
+            out.append(ConvShape(pre + ".conv1", cin, width, 1, 1, 0, h))
+            out.append(ConvShape(pre + ".conv2", width, width, 3, s, 1, h))
+            h2 = (h + 2 - 3) // s + 1
+            out.append(ConvShape(pre + ".conv3", width, cout, 1, 1, 0, h2))
+            if b == 0:
+                out.append(ConvShape(pre + ".downsample", cin, cout, 1, s, 0, h))
+            cin, h = cout, h2
+    out.append(ConvShape("fc", 2048, 1000, 1, 1, 0, 1))
+    return out
+
+
+def resnet50_layer(shape: ConvShape, batch: int, seed: int) -> "Layer":
+    """One layer of the ResNet-50 sweep: input U[-1, 1] at the layer's NHWC
+    input shape, lowered to im2col; dH rows N(0, 1) scaled per sample by
+    lognormal(0, 2); W Kaiming normal N(0, 2/D).  D and C are padded to
+    multiples of 16 with zero columns (the stem's D = 147 -> 160, the fc's
+    C = 1000 -> 1008): the padded columns of X and W are zero and so are the
+    padded columns of dH; the outputs of the real columns are those of the
+    unpadded layer."""
+    g = rng(seed)
+    x = g.uniform(-1, 1, (batch, shape.h, shape.h, shape.cin)).astype(np.float32)
+    X = im2col_nhwc(x, shape.k, shape.k, shape.stride, shape.pad)
+    n = X.shape[0]
+    if shape.D_pad != shape.D:
+        X = np.concatenate([X, np.zeros((n, shape.D_pad - shape.D), np.float32)], axis=1)
+    dH = (g.standard_normal((n, shape.cout)).astype(np.float32)
+          * _lognormal_rows(g, n, 2.0)[:, None])
+    W = (np.sqrt(2.0 / shape.D) * g.standard_normal((shape.cout, shape.D))).astype(np.float32)
+    if shape.C_pad != shape.cout:
+        dH = np.concatenate([dH, np.zeros((n, shape.C_pad - shape.cout), np.float32)], axis=1)
+        W = np.concatenate([W, np.zeros((shape.C_pad - shape.cout, shape.D), np.float32)], axis=0)
+    if shape.D_pad != shape.D:
+        W = np.concatenate([W, np.zeros((W.shape[0], shape.D_pad - shape.D), np.float32)], axis=1)
+    return Layer(f"{CONFIG_NAMES[4]}:{shape.name}", np.ascontiguousarray(dH),
+                 np.ascontiguousarray(X), np.ascontiguousarray(W), "f32", [(BHQ, 5, 16)])
 
 
 def config(index: int, batch: Optional[int] = None, rows: Optional[int] = None,
@@ -143,6 +225,12 @@ def config(index: int, batch: Optional[int] = None, rows: Optional[int] = None,
             out.append(Layer(f"{CONFIG_NAMES[3]}:{name}", dH, X, W, "bf16",
                              [(PTQ, 8, 0), (PSQ, 5, 0), (BHQ, 5, 16)]))
         return out
+    if index == 4:
+        # full size is 40+ GB of fp32 inputs: the bench draws it on the device
+        # from the same shape table; here, small batches for the oracle
+        b = batch or 1
+        base = 1234 + index if seed is None else seed
+        return [resnet50_layer(sh, b, base + i) for i, sh in enumerate(resnet50_shapes())]
     raise ValueError(f"no workload {index}")
 
 

@@ -202,6 +202,24 @@ def test_linear_backward_matches_oracle(cfg, small, kind, bits, block):
         assert grad_rel_err(gw, ref_w) <= GRAD_TOL
 
 
+RESNET50 = wl.config(4, batch=1)
+
+
+@pytest.mark.parametrize("idx", range(len(RESNET50)), ids=[L.name.split(":")[1] for L in RESNET50])
+def test_resnet50_sweep_layer_matches_oracle(idx):
+    """Every layer of the ResNet-50 sweep (batch 1; the stem's D and the fc's
+    C zero-padded to multiples of 16): BHQ-5/16 codes against the oracle's,
+    grad_X and grad_W against the oracle's dequantize-then-multiply of the
+    GPU's codes."""
+    L = RESNET50[idx]
+    qx, qw, q2, q1, gx, gw = _backward(L, orc.BHQ, 5, 16)
+    h2 = q2.to_numpy()
+    ref = orc.quantize_grad(L.dH, orc.BHQ, 5, 16, 3, orc.STREAM_B2, want_v=True)
+    _check_bhq_codes(h2["codes"], ref["codes"], ref["v"], 3)
+    assert grad_rel_err(gx, orc.grad_x(h2, qw.to_numpy())) <= GRAD_TOL
+    assert grad_rel_err(gw, orc.grad_w(q1.to_numpy(), qx.to_numpy())) <= GRAD_TOL
+
+
 @pytest.mark.parametrize("N,block", [(256, 8), (200, 64), (131, 128), (77, 16)])
 def test_bhq_offsets_match_oracle(N, block):
     """The reflected per-row terms of the grad_X epilogue against the
