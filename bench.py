@@ -330,7 +330,17 @@ def run_gpu(args):
         sets = [dict(dH=dH, X=X, W=W, gx=gx, gw=gw),
                 dict(dH=torch.empty_like(dH), X=torch.empty_like(X), W=torch.empty_like(W),
                      gx=torch.empty_like(gx), gw=torch.empty_like(gw))]
-        s_in, s_cmp, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        s_cmp = torch.cuda.Stream(dev)
+        # each direction's copies can be split by rows over several streams
+        # (several copy engines); one stream per direction measured fastest
+        ncs = max(1, args.e2e_copy_streams)
+        s_ins = [torch.cuda.Stream(dev) for _ in range(ncs)]
+        s_outs = [torch.cuda.Stream(dev) for _ in range(ncs)]
+
+        def split_rows(t):
+            n_ = t.shape[0]
+            step_ = (n_ + ncs - 1) // ncs
+            return [t[i:i + step_] for i in range(0, n_, step_)]
 
         def e2e_calls(b, seed):
             return [lambda: fqt.quantize_act(b["X"], 8, ws=ws_fx, out=qx),
@@ -344,30 +354,42 @@ def run_gpu(args):
             done_cmp, done_out = [None, None], [None, None]
             for i in range(nsteps):
                 b = sets[i & 1]
-                with torch.cuda.stream(s_in):
-                    if done_cmp[i & 1] is not None:  # step i-2 has read these inputs
-                        s_in.wait_event(done_cmp[i & 1])
-                    for k, hsrc in (("dH", h_dH), ("X", h_X), ("W", h_W)):
-                        b[k].copy_(hsrc, non_blocking=True)
-                    ein = torch.cuda.Event()
-                    ein.record(s_in)
+                eins = []
+                for si, s_in in enumerate(s_ins):
+                    with torch.cuda.stream(s_in):
+                        if done_cmp[i & 1] is not None:  # step i-2 has read these inputs
+                            s_in.wait_event(done_cmp[i & 1])
+                        for k, hsrc in (("dH", h_dH), ("X", h_X), ("W", h_W)):
+                            dst_, src_ = split_rows(b[k]), split_rows(hsrc)
+                            if si < len(dst_):
+                                dst_[si].copy_(src_[si], non_blocking=True)
+                        ein = torch.cuda.Event()
+                        ein.record(s_in)
+                        eins.append(ein)
                 with torch.cuda.stream(s_cmp):
-                    s_cmp.wait_event(ein)
+                    for ein in eins:
+                        s_cmp.wait_event(ein)
                     if done_out[i & 1] is not None:  # step i-2's gradients have left
-                        s_cmp.wait_event(done_out[i & 1])
+                        for eo in done_out[i & 1]:
+                            s_cmp.wait_event(eo)
                     for f in e2e_calls(b, seed0 + i):
                         f()
                     ec = torch.cuda.Event()
                     ec.record(s_cmp)
                     done_cmp[i & 1] = ec
-                with torch.cuda.stream(s_out):
-                    s_out.wait_event(ec)
-                    h_gx.copy_(b["gx"], non_blocking=True)
-                    h_gw.copy_(b["gw"], non_blocking=True)
-                    eo = torch.cuda.Event()
-                    eo.record(s_out)
-                    done_out[i & 1] = eo
-            for st_ in (s_in, s_cmp, s_out):
+                eos = []
+                for si, s_out in enumerate(s_outs):
+                    with torch.cuda.stream(s_out):
+                        s_out.wait_event(ec)
+                        for hdst, k in ((h_gx, "gx"), (h_gw, "gw")):
+                            dst_, src_ = split_rows(hdst), split_rows(b[k])
+                            if si < len(dst_):
+                                dst_[si].copy_(src_[si], non_blocking=True)
+                        eo = torch.cuda.Event()
+                        eo.record(s_out)
+                        eos.append(eo)
+                done_out[i & 1] = eos
+            for st_ in s_ins + [s_cmp] + s_outs:
                 stream.wait_stream(st_)
 
         run_e2e(2, 2000)  # warms the pinned-copy path and the streams
@@ -377,7 +399,7 @@ def run_gpu(args):
         flush.fill_(7)
         torch.cuda.synchronize()
         e0.record(stream)
-        for st_ in (s_in, s_cmp, s_out):
+        for st_ in s_ins + [s_cmp] + s_outs:
             st_.wait_stream(stream)
         run_e2e(args.e2e_steps, 3000)
         e1.record(stream)
@@ -387,8 +409,9 @@ def run_gpu(args):
                "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int((N * C + N * D + C * D) * 4),
                "d2h_bytes_per_step": int((N * D + C * D) * 4),
-               "schedule": "2-deep pipeline: H2D / C-ABI calls / D2H on three streams, "
-                           "double-buffered device inputs and outputs, eager calls"}
+               "schedule": f"2-deep pipeline: H2D on {ncs} streams / C-ABI calls / D2H on "
+                           f"{ncs} streams (each copy split by rows), double-buffered device "
+                           "inputs and outputs, eager calls"}
 
     # ---- the quantized forward GEMM H = X~ W~^T on the same layer (the
     # contraction core with the roles renamed), timed alone ----
@@ -851,6 +874,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--e2e-copy-streams", type=int, default=1,
+                    help="streams per copy direction in the end-to-end pipeline")
     ap.add_argument("--cpu-rows", type=int, default=65536,
                     help="rows of the CPU-baseline sample (about 10 s of oracle work)")
     ap.add_argument("--ref-rows", type=int, default=8192,
