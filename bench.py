@@ -409,9 +409,11 @@ def run_gpu(args):
                "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int((N * C + N * D + C * D) * 4),
                "d2h_bytes_per_step": int((N * D + C * D) * 4),
-               "schedule": f"2-deep pipeline: H2D on {ncs} streams / C-ABI calls / D2H on "
-                           f"{ncs} streams (each copy split by rows), double-buffered device "
-                           "inputs and outputs, eager calls"}
+               "schedule": ("2-deep pipeline: H2D / C-ABI calls / D2H on three streams, "
+                            "double-buffered device inputs and outputs, eager calls" if ncs == 1 else
+                            f"2-deep pipeline: H2D on {ncs} streams / C-ABI calls / D2H on {ncs} "
+                            "streams (each copy split by rows), double-buffered device inputs and "
+                            "outputs, eager calls")}
 
     # ---- the quantized forward GEMM H = X~ W~^T on the same layer (the
     # contraction core with the roles renamed), timed alone ----
