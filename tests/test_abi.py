@@ -107,3 +107,27 @@ def test_new_entry_points_validate_without_gpu():
     assert lib.fqt_quantize_act_conv(p, 0, 2, 8, 8, 60, 3, 3, 1, 8, ctypes.byref(qc), p, 256,
                                      None) == 2  # c % 8 != 0
     del raw
+
+
+def test_adaptive_group_limits_without_gpu():
+    """Adaptive BHQ groups (block 0): rows of 64, 128 or 256 columns and at
+    most 2^20 rows (the radix sort's per-tile prefix); other requests are
+    refused synchronously with FQT_EUNSUPPORTED."""
+    from paper_2010_14298_gb300 import fqt
+    lib = fqt.load()
+    raw, p = _aligned()
+    q = fqt._QT()
+    for name in ("codes_f16", "inv_s", "zero", "row_sum", "hz", "hr", "perm", "gstart",
+                 "gsize"):
+        setattr(q, name, p.value)
+    BHQ = 2
+    assert lib.fqt_quantize_grad(p, 0, 64, 512, BHQ, 5, 0, 0, ctypes.byref(q), None, p, 256,
+                                 None) == 2
+    assert lib.fqt_quantize_grad(p, 0, (1 << 20) + 1, 64, BHQ, 5, 0, 0, ctypes.byref(q), None,
+                                 p, 256, None) == 2
+    # block sizes other than 0 or a power of two up to 128 are invalid
+    assert lib.fqt_quantize_grad(p, 0, 64, 64, BHQ, 5, 24, 0, ctypes.byref(q), None, p, 256,
+                                 None) == 1
+    assert lib.fqt_quantize_grad(p, 0, 64, 64, BHQ, 5, 256, 0, ctypes.byref(q), None, p, 256,
+                                 None) == 1
+    del raw
