@@ -131,3 +131,37 @@ def test_adaptive_group_limits_without_gpu():
     assert lib.fqt_quantize_grad(p, 0, 64, 64, BHQ, 5, 256, 0, ctypes.byref(q), None, p, 256,
                                  None) == 1
     del raw
+
+
+def test_backward_shape_checks_without_gpu():
+    """fqt_linear_backward refuses, before any launch: contraction widths
+    that are not multiples of 16 or exceed the int32 epilogue bound
+    (FQT_EUNSUPPORTED), mismatched operands and BHQ tensors without their
+    lead rows or offsets (FQT_EINVAL), a misaligned workspace
+    (FQT_EWORKSPACE)."""
+    from paper_2010_14298_gb300 import fqt
+    lib = fqt.load()
+    raw, p = _aligned()
+
+    def qt(rows, cols, kind=0, block=0, **fields):
+        q = fqt._QT()
+        q.rows, q.cols, q.bits, q.kind, q.block = rows, cols, 8, kind, block
+        for name in ("codes_f16", "inv_s", "zero", "row_sum", "col_sum"):
+            setattr(q, name, p.value)
+        for k, v in fields.items():
+            setattr(q, k, v)
+        return q
+
+    def run(q2, qw, ws=p):
+        return lib.fqt_linear_backward(ctypes.byref(q2), None, None, ctypes.byref(qw), p, None,
+                                       ws, 1 << 16, None)
+
+    assert run(qt(256, 72), qt(72, 64)) == 2            # C % 16
+    assert run(qt(256, 64), qt(64, 40)) == 2            # D % 16
+    assert run(qt(256, 8208), qt(8208, 64)) == 2        # C above the int32 epilogue bound
+    assert run(qt(256, 64), qt(128, 64)) == 1           # W~ rows != C
+    assert run(qt(256, 64, kind=2, block=16), qt(64, 64)) == 1  # BHQ without lead / hz / hr
+    assert run(qt(256, 64, kind=2, block=16, lead=p.value, hz=p.value), qt(64, 64)) == 1
+    misaligned = ctypes.c_void_p(p.value + 64)
+    assert run(qt(256, 64), qt(64, 64), ws=misaligned) == 6
+    del raw
