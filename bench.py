@@ -810,6 +810,10 @@ def run_gpu(args):
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(args.cpu_rows)
+        if ovh is not None:
+            # the paper timed its CPU quantizer routines on this shape (Sec.
+            # 4.3); the oracle's whole gradient quantizers on one core beside it
+            ovh["oracle_cpu_ms"] = oracle_overhead_shape()
     if rank == 0:
         print(json.dumps(result), flush=True)
     if world > 1:
@@ -836,6 +840,22 @@ def cpu_baseline(rows: int):
     return {"value": ops / dt / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
             "sample": f"{rows} im2col rows (batch {rows // 1024}) of the workload, "
                       f"full hot path, {dt:.1f} s single-threaded"}
+
+
+def oracle_overhead_shape():
+    """The oracle's gradient quantizers (range, scales / transform, SR, sums;
+    Q_b2 only) on the paper's overhead shape, dH 401408 x 64, one core."""
+    import oracle as orc
+    from paper_2010_14298_gb300 import workloads as wl
+    orc.build()
+    dH = wl.random_grad(wl.rng(480), 128 * 56 * 56, 64, sigma=2.0, outlier_frac=0.01)
+    out = {}
+    for name, kind, bits, block in (("PTQ-8", orc.PTQ, 8, 0), ("PSQ-8", orc.PSQ, 8, 0),
+                                    ("BHQ-5 block 16", orc.BHQ, 5, 16)):
+        t = time.perf_counter()
+        orc.quantize_grad(dH, kind, bits, block, 0, orc.STREAM_B2)
+        out[name] = (time.perf_counter() - t) * 1e3
+    return out
 
 
 def run_reference(args):
