@@ -251,12 +251,22 @@ FQT_API fqt_status fqt_linear_forward(const fqt_qtensor *qx, const fqt_qtensor *
  *  - All calls on a device share the array and it keeps the last call's
  *    contents, so calls that overlap on the GPU (other streams, other host
  *    threads) race and give wrong results: order them.
- *  - Device-side conditions (a bounded wait that ran out) are not reported.
- * Operands as for fqt_linear_backward (codes_f16, col_sum, 8-bit PTQ).
+ *  - Device-side conditions (a bounded wait that ran out) are recorded in
+ *    the array's status word and returned by fqt_fixed_scratch_sync_status.
+ * Operands as for fqt_linear_backward (codes_f16, col_sum, PTQ), but plain
+ * matrices only: an implicit im2col operand (from fqt_quantize_act_conv,
+ * conv[0] > 0) returns FQT_EUNSUPPORTED before anything is enqueued.
  */
 FQT_API fqt_status fqt_grad_w_fixed_scratch(const fqt_qtensor *q_b1,
                                             const fqt_qtensor *qx, float *grad_W,
                                             void *stream);
+
+/* Synchronises `stream`, returns the first device-side condition recorded by
+ * fqt_grad_w_fixed_scratch calls on the current device since the previous
+ * call of this function (or FQT_OK) and clears it.  Allocates nothing; like
+ * the first fqt_grad_w_fixed_scratch call it looks up the array's address
+ * once per device.  Has no counterpart in the paper. */
+FQT_API fqt_status fqt_fixed_scratch_sync_status(void *stream);
 
 /* Synchronises `stream`, returns the first device-side condition recorded in
  * `workspace` since the previous call (or FQT_OK) and clears it. */
@@ -274,6 +284,18 @@ FQT_API fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits
                               const uint8_t *Bm, int b_kmajor, int b_bits,
                               int64_t M, int64_t N, int64_t K, int64_t *out,
                               void *workspace, size_t ws_bytes, void *stream);
+
+/* Check of the device-side timeout path: one thread waits on an mbarrier
+ * that nothing arrives at, with the bounded wait the contraction kernels
+ * use, here bounded by limit_ns (at most 10 s, else FQT_EINVAL) instead of
+ * their 2 s.  When it runs out the kernel records FQT_ETIMEOUT and returns.
+ * The condition goes to `workspace` (then read by fqt_sync_status; at least
+ * 256 bytes, 256-byte aligned) or, with workspace NULL, to the fixed array
+ * of fqt_grad_w_fixed_scratch (read by fqt_fixed_scratch_sync_status).
+ * No bulk copy or tensor-core operation is in flight during the wait.  Has
+ * no counterpart in the paper. */
+FQT_API fqt_status fqt_debug_wait_timeout(void *workspace, size_t ws_bytes,
+                                          uint64_t limit_ns, void *stream);
 
 /* Static description of a status code. */
 FQT_API const char *fqt_status_string(fqt_status status);

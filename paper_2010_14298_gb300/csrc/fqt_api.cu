@@ -384,6 +384,29 @@ fqt_status fqt_sync_status(void *workspace, void *stream) {
   return static_cast<fqt_status>(code);
 }
 
+fqt_status fqt_fixed_scratch_sync_status(void *stream) {
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+  int *word = nullptr;
+  const fqt_status s = fixed_scratch_status(&word);
+  if (s != FQT_OK) return s;
+  int code = 0;
+  e = cudaMemcpy(&code, word, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "status read");
+  if (code != 0) {
+    e = cudaMemset(word, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "status clear");
+  }
+  return static_cast<fqt_status>(code);
+}
+
+fqt_status fqt_debug_wait_timeout(void *workspace, size_t ws_bytes, uint64_t limit_ns,
+                                  void *stream) {
+  return debug_wait_timeout(workspace, ws_bytes, limit_ns,
+                            reinterpret_cast<cudaStream_t>(stream));
+}
+
 const char *fqt_last_cuda_error(void) { return g_last_error; }
 
 const char *fqt_status_string(fqt_status status) {

@@ -208,19 +208,25 @@ __device__ __forceinline__ uint64_t global_ns() {
 }
 
 // Bounded wait: returns false (and records FQT_ETIMEOUT) if the phase with
-// the given parity has not completed within kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
-                                          int *status) {
+// the given parity has not completed within limit_ns nanoseconds.
+__device__ __forceinline__ bool mbar_wait_limit(uint64_t *bar, uint32_t parity,
+                                                int *status, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (;;) {
     for (int i = 0; i < 8; ++i)
       if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
-    if (global_ns() - t0 > kWaitLimitNs) {
+    if (global_ns() - t0 > limit_ns) {
       record_status(status, FQT_ETIMEOUT);
       return false;
     }
   }
+}
+
+// The kernels' wait: bounded by kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          int *status) {
+  return mbar_wait_limit(bar, parity, status, kWaitLimitNs);
 }
 
 // Sleeps about `ns` nanoseconds (used only on the abort path).

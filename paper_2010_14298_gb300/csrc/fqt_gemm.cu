@@ -3005,6 +3005,9 @@ fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
       !qx->col_sum || !qa->inv_s || !qa->zero || !qx->inv_s || !qx->zero)
     return FQT_EINVAL;
   if (qa->kind != FQT_PTQ || qx->kind != FQT_PTQ) return FQT_EINVAL;
+  // an implicit im2col operand stores NHWC codes, not the Nr x D matrix the
+  // tile kernel below reads: refuse it before anything is enqueued
+  if (qa->conv[0] > 0 || qx->conv[0] > 0) return FQT_EUNSUPPORTED;
   const int64_t Nr = qa->rows, C = qa->cols, D = qx->cols;
   if (qx->rows != Nr || Nr < 0) return FQT_EINVAL;
   if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
@@ -3024,14 +3027,13 @@ fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
   void *base = nullptr;
   fqt_status s = fixed_scratch_address(&base);
   if (s != FQT_OK) return s;
+  // the status word keeps the first condition recorded since the last
+  // fqt_fixed_scratch_sync_status (it is zero when the library loads); the
+  // partials are fully rewritten by every split, so nothing else needs clearing
   int *status = static_cast<int *>(base);
   int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(base) + kHeaderBytes);
-  // the status word must start each call at zero (the array keeps the last
-  // call's contents); the partials are fully rewritten by every split
-  cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int), st);
-  if (e != cudaSuccess) return cuda_fail(e, "fixed scratch clear");
   if (Nr == 0) {
-    e = cudaMemsetAsync(grad_W, 0, per_split, st);
+    const cudaError_t e = cudaMemsetAsync(grad_W, 0, per_split, st);
     return cuda_fail(e, "grad_W clear");
   }
   GemmArgs g;
@@ -3058,6 +3060,48 @@ fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
   r.zero_b = qx->zero;
   launch_reduce(r, st);
   return cuda_fail(cudaGetLastError(), "split-K reduce launch");
+}
+
+// Status word of the fixed array (its first int): the device-side conditions
+// of fqt_grad_w_fixed_scratch calls land there, as they land in a caller's
+// workspace for the other calls.
+fqt_status fixed_scratch_status(int **out) {
+  void *base = nullptr;
+  const fqt_status s = fixed_scratch_address(&base);
+  if (s == FQT_OK) *out = static_cast<int *>(base);
+  return s;
+}
+
+// ---------------------------------------------------------------------------
+// A wait on an mbarrier that nothing arrives at, bounded by limit_ns: the
+// same bounded wait the contraction kernels use, made to run out on purpose
+// so that the timeout path (FQT_ETIMEOUT in the status word, the kernel
+// returns, the context stays usable) can be checked.  No bulk copy or
+// tensor-core operation is in flight.
+// ---------------------------------------------------------------------------
+__global__ void k_wait_nothing(int *status, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait_limit(&bar, 0, status, limit_ns);
+}
+
+fqt_status debug_wait_timeout(void *ws, size_t ws_bytes, uint64_t limit_ns,
+                              cudaStream_t st) {
+  if (limit_ns > 10000000000ull) return FQT_EINVAL;  // at most 10 s
+  int *status = nullptr;
+  if (ws) {
+    if (ws_bytes < kHeaderBytes || ((uintptr_t)ws & 255)) return FQT_EWORKSPACE;
+    status = static_cast<int *>(ws);
+  } else {
+    const fqt_status s = fixed_scratch_status(&status);
+    if (s != FQT_OK) return s;
+  }
+  k_wait_nothing<<<1, 32, 0, st>>>(status, limit_ns);
+  return cuda_fail(cudaGetLastError(), "wait test launch");
 }
 
 }  // namespace fqt

@@ -94,6 +94,8 @@ size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D);
 size_t debug_workspace_bytes(int64_t M, int64_t N, int64_t K);
 fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
                                 float *grad_W, cudaStream_t st);
+fqt_status fixed_scratch_status(int **out);
+fqt_status debug_wait_timeout(void *ws, size_t ws_bytes, uint64_t limit_ns, cudaStream_t st);
 fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H, void *ws,
                           size_t ws_bytes, cudaStream_t st);
 fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,

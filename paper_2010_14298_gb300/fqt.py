@@ -89,6 +89,10 @@ def load(build_if_missing: bool = True):
         lib.fqt_grad_w_fixed_scratch.restype = i32
         lib.fqt_sync_status.argtypes = [P, P]
         lib.fqt_sync_status.restype = i32
+        lib.fqt_fixed_scratch_sync_status.argtypes = [P]
+        lib.fqt_fixed_scratch_sync_status.restype = i32
+        lib.fqt_debug_wait_timeout.argtypes = [P, sz, u64, P]
+        lib.fqt_debug_wait_timeout.restype = i32
         lib.fqt_debug_int_gemm.argtypes = [P, i32, i32, P, i32, i32, i64, i64,
                                            i64, P, P, sz, P]
         lib.fqt_debug_int_gemm.restype = i32
@@ -443,6 +447,22 @@ def debug_int_gemm(A: torch.Tensor, a_kmajor: bool, a_bits: int, B: torch.Tensor
 def sync_status(ws: Workspace, stream=None) -> int:
     """Synchronises and returns (then clears) the device-side status word."""
     return int(load().fqt_sync_status(ws.ptr, _stream(stream)))
+
+
+def fixed_scratch_sync_status(stream=None) -> int:
+    """Synchronises and returns (then clears) the status word of the fixed
+    array behind grad_w_fixed_scratch."""
+    return int(load().fqt_fixed_scratch_sync_status(_stream(stream)))
+
+
+def debug_wait_timeout(limit_ns: int, ws: Optional[Workspace] = None, stream=None):
+    """Enqueues a bounded wait that is made to run out after limit_ns; its
+    FQT_ETIMEOUT lands in ws (or, with ws None, the fixed array's word)."""
+    lib = load()
+    st = lib.fqt_debug_wait_timeout(ws.ptr if ws is not None else None,
+                                    ws.nbytes if ws is not None else 0,
+                                    ctypes.c_uint64(limit_ns), _stream(stream))
+    _check(st, "fqt_debug_wait_timeout")
 
 
 def status_string(code: int) -> str:

@@ -165,3 +165,30 @@ def test_backward_shape_checks_without_gpu():
     misaligned = ctypes.c_void_p(p.value + 64)
     assert run(qt(256, 64), qt(64, 64), ws=misaligned) == 6
     del raw
+
+
+def test_fixed_scratch_and_wait_test_refusals_without_gpu():
+    """fqt_grad_w_fixed_scratch refuses an implicit im2col operand
+    (FQT_EUNSUPPORTED) and fqt_debug_wait_timeout a limit above 10 s or a
+    misaligned workspace, all before any CUDA call."""
+    from paper_2010_14298_gb300 import fqt
+    lib = fqt.load()
+    raw, p = _aligned()
+
+    def qt(rows, cols, conv=None):
+        q = fqt._QT()
+        q.rows, q.cols, q.bits, q.kind = rows, cols, 8, 0
+        for name in ("codes_f16", "inv_s", "zero", "col_sum"):
+            setattr(q, name, p.value)
+        if conv:
+            q.conv = (ctypes.c_int32 * 8)(*conv)
+        return q
+
+    q1 = qt(2048, 64)
+    qx = qt(2048, 576, conv=(2, 32, 32, 64, 3, 3, 1, 0))
+    assert lib.fqt_grad_w_fixed_scratch(ctypes.byref(q1), ctypes.byref(qx), p, None) == 2
+    assert lib.fqt_grad_w_fixed_scratch(ctypes.byref(qx), ctypes.byref(q1), p, None) == 2
+    assert lib.fqt_debug_wait_timeout(p, 256, 10_000_000_001, None) == 1
+    assert lib.fqt_debug_wait_timeout(ctypes.c_void_p(p.value + 16), 256, 1000, None) == 6
+    assert lib.fqt_debug_wait_timeout(p, 128, 1000, None) == 6
+    del raw
