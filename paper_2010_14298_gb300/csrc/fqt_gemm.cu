@@ -84,7 +84,7 @@ constexpr size_t kOffPar = 0;
 constexpr size_t kOffBar = kOffPar + kParStages * kParBytes;
 // operand full / empty, accumulator full / empty (4 each), parameter full /
 // empty (4 each)
-constexpr size_t kNumBars = 2 * kMaxStages + 16;
+constexpr size_t kNumBars = 2 * kMaxStages + 17;  // ... + the MMA drain barrier
 // grad_X in the fp32 form with fixed blocks: one bit per tile of this CTA
 // (in its order) for the tiles left raw, finished by the CTA at the end
 constexpr size_t kOffRaw = (kOffBar + kNumBars * 8 + 16 + 15) & ~(size_t)15;
@@ -1269,7 +1269,7 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
   uint8_t *ring = ops + (size_t)nstages * 2 * kTileBytes;          // output boxes
   uint64_t *full = bars, *empty = bars + kMaxStages;
   uint64_t *accf = bars + 2 * kMaxStages, *acce = accf + 4;
-  uint64_t *pfull = acce + 4, *pempty = pfull + 4;
+  uint64_t *pfull = acce + 4, *pempty = pfull + 4, *drain = pempty + 4;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kNumBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   // grad_X: one accumulator per item, served by 4 epilogue warps (one per
@@ -1289,6 +1289,7 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
       mbar_init(&pfull[i], 1);
       mbar_init(&pempty[i], 4);  // the 4 epilogue warps of the consuming set
     }
+    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -1416,6 +1417,10 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
           if (!kPerItem) buf ^= 1;
         }
       }
+      // every MMA this thread issued has completed before TMEM is released
+      // (after an abort the epilogue may have stopped waiting for them)
+      umma_commit(drain);
+      mbar_wait(drain, 0, g.status);
     }
   } else if (warp == kGemmWarpPar) {
     if (MODE == MODE_GRADX) gradx_params<NB, FORM>(g, smem, pfull, pempty, abort_flag, lane);
@@ -1879,8 +1884,8 @@ __global__ void __launch_bounds__(kWThreads, 1)
   uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem);
   uint64_t *full = bars, *empty = bars + kMaxStages, *accf = empty + kMaxStages,
-           *acce = accf + 1;
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(acce + 1);
+           *acce = accf + 1, *drain = acce + 1;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   uint8_t *ops = smem + 1024;
   const size_t xbytes = (size_t)w.mt * 2 * kWBox;  // per D tile: two 64-wide boxes
@@ -1893,6 +1898,7 @@ __global__ void __launch_bounds__(kWThreads, 1)
     }
     mbar_init(accf, 1);
     mbar_init(acce, kPartialEpiWarps);
+    mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -2008,6 +2014,9 @@ __global__ void __launch_bounds__(kWThreads, 1)
         }
         umma_commit(accf);
       }
+      // every MMA this thread issued has completed before TMEM is released
+      umma_commit(drain);
+      mbar_wait(drain, 0, w.status);
     }
   } else {
     // epilogue: warp (q, h) takes the D tiles m = h, h + 2, ...; a thread owns
