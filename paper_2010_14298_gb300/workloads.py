@@ -161,7 +161,7 @@ def resnet50_layer(shape: ConvShape, batch: int, seed: int) -> "Layer":
     n = X.shape[0]
     if shape.D_pad != shape.D:
         X = np.concatenate([X, np.zeros((n, shape.D_pad - shape.D), np.float32)], axis=1)
-    dH = (g.standard_normal((n, shape.cout)).astype(np.float32)
+    dH = (g.standard_normal((n, shape.cout), dtype=np.float32)
           * _lognormal_rows(g, n, 2.0)[:, None])
     W = (np.sqrt(2.0 / shape.D) * g.standard_normal((shape.cout, shape.D))).astype(np.float32)
     if shape.C_pad != shape.cout:

@@ -82,12 +82,24 @@ def _check_b1(q1_gpu, dH, seed):
     assert np.array_equal(h1["col_sum"], r1["codes"].astype(np.int64).sum(0))
 
 
+# BHQ codes of every case compared in this module: the >= 99.99% agreement
+# bar is a rate, so it is applied to each case of at least AGREE_MIN codes on
+# its own and to the pool of all cases (test_bhq_code_agreement_pooled).
+AGREE_MIN = 10_000
+_BHQ_POOL = {"codes": 0, "flips": 0}
+
+
 def _check_bhq_codes(got, ref, v, seed, stream=0):
     diff = got.astype(np.int64) - ref.astype(np.int64)
-    # the transform rounds differently on the two sides: a +-1 flip where t
-    # sits at an SR threshold, at most 1e-4 of the codes (two on small cases)
-    assert (diff != 0).sum() <= max(2, 1e-4 * diff.size), (diff != 0).mean()
-    assert np.abs(diff).max() <= 1
+    flips = int((diff != 0).sum())
+    _BHQ_POOL["codes"] += diff.size
+    _BHQ_POOL["flips"] += flips
+    # the transform rounds differently on the two sides (fp32 on the GPU,
+    # double rounded to fp32 in the oracle): a mismatch is a +-1 flip where
+    # v sits at its SR threshold
+    assert np.abs(diff).max(initial=0) <= 1
+    if diff.size >= AGREE_MIN:
+        assert flips <= 1e-4 * diff.size, flips / diff.size
     idx = np.flatnonzero(diff.ravel())
     if idx.size:
         dist = sr_boundary_distance(v.ravel()[idx], seed, stream, idx)
@@ -797,3 +809,89 @@ def test_gpu_quantizers_are_unbiased_monte_carlo(kind, bits, block):
     assert np.abs(z).max() < 5.5
     emp = (s2 / K - mean ** 2).sum()
     assert emp / vd.sum() == pytest.approx(1.0, rel=0.12)
+
+
+# --------------------------------------------------------------------------
+# Full-size workloads of the transformer FFN pair and the ResNet-50 sweep,
+# at the sizes the bench times (sampled outputs)
+# --------------------------------------------------------------------------
+def _grad_w_columns(h1: dict, hx: dict, cols: np.ndarray) -> np.ndarray:
+    """The oracle's dequantize-then-multiply grad_W on a subset of the
+    columns of a per-tensor X~ (its dequantization is column-separable); the
+    double product of the two dequantized matrices is a BLAS dgemm here (the
+    oracle's plain loop takes minutes at millions of rows)."""
+    sub = dict(hx)
+    sub["codes"] = np.ascontiguousarray(hx["codes"][:, cols])
+    return orc.dequant(h1).T @ orc.dequant(sub)
+
+
+def _sampled_check(L, kind, bits, block, seed, n_rows=96, n_cols=32):
+    """Every code of Q_b2 and Q_b1 against the oracle's, grad_X on sampled
+    rows (whole quantizer blocks) and grad_W on sampled columns against the
+    oracle's dequantize-then-multiply of the GPU's codes."""
+    qx, qw, q2, q1, gx, gw = _backward(L, kind, bits, block, seed=seed)
+    h2, h1, hx, hw = q2.to_numpy(), q1.to_numpy(), qx.to_numpy(), qw.to_numpy()
+    ref2 = orc.quantize_grad(L.dH, kind, bits, block, seed, orc.STREAM_B2,
+                             want_v=kind == orc.BHQ)
+    if kind == orc.BHQ:
+        _check_bhq_codes(h2["codes"], ref2["codes"], ref2["v"], seed)
+        assert np.array_equal(h2["lead"], ref2["lead"])
+    else:
+        assert np.array_equal(h2["codes"], ref2["codes"])
+        assert np.array_equal(h2["inv_s"], ref2["inv_s"])
+        assert np.array_equal(h2["zero"], ref2["zero"])
+    del ref2
+    _check_b1(q1, L.dH, seed)
+    ref_f = orc.quantize_fwd(L.X, 8)
+    assert np.array_equal(hx["codes"], ref_f["codes"])
+    del ref_f
+    g = wl.rng(L.N + L.C + L.D)
+    rows = np.sort(g.choice(L.N, min(n_rows, L.N), replace=False))
+    rows = np.union1d(rows, [0, L.N - 1])  # the first and the ragged last block
+    ref_x = oracle_rows_grad_x(h2, hw, h2["codes"], rows)
+    assert grad_rel_err(gx[rows], ref_x) <= GRAD_TOL
+    cols = np.sort(g.choice(L.D, min(n_cols, L.D), replace=False))
+    cols = np.union1d(cols, [0, L.D - 1])
+    assert grad_rel_err(gw[:, cols], _grad_w_columns(h1, hx, cols)) <= GRAD_TOL
+
+
+_FFN = {}
+
+
+def _ffn_layer(i):
+    if not _FFN:
+        _FFN.update(enumerate(wl.config(3)))
+    return _FFN[i]
+
+
+@pytest.mark.parametrize("kind,bits,block", [(orc.PTQ, 8, 0), (orc.PSQ, 5, 0),
+                                             (orc.BHQ, 5, 16)])
+@pytest.mark.parametrize("layer", [0, 1], ids=["ffn-up", "ffn-down"])
+def test_ffn_full_size_sampled(layer, kind, bits, block):
+    """The transformer FFN pair at 8192 tokens from bf16 tensors (C = 4096
+    and 1024): the int64 and mixed epilogue forms, several exact chunks per
+    split-K range of grad_W, at the shapes the bench times."""
+    _sampled_check(_ffn_layer(layer), kind, bits, block, seed=13)
+
+
+R50_FULL = ["conv1", "layer1.0.conv2", "layer1.0.conv3", "fc"]
+
+
+@pytest.mark.parametrize("name", R50_FULL)
+def test_resnet50_full_batch_layer_sampled(name):
+    """Layers of the ResNet-50 sweep at batch 256: the stem (N = 3,211,264
+    im2col rows, D 147 -> 160), a 3 x 3 and a 1 x 1 layer of stage 1
+    (N = 802,816, C = 64 and 256) and the fc (C 1000 -> 1008); BHQ-5/16 with
+    Q_b1, as the bench runs them."""
+    shapes = wl.resnet50_shapes()
+    i = [s.name for s in shapes].index(name)
+    L = wl.resnet50_layer(shapes[i], 256, 1234 + 4 + i)
+    _sampled_check(L, orc.BHQ, 5, 16, seed=3)
+
+
+def test_bhq_code_agreement_pooled():
+    """The >= 99.99% BHQ code agreement over every case this module compared
+    (cases below AGREE_MIN codes cannot show a 1e-4 rate on their own)."""
+    if _BHQ_POOL["codes"] == 0:
+        pytest.skip("no BHQ case ran")
+    assert _BHQ_POOL["flips"] <= 1e-4 * _BHQ_POOL["codes"], _BHQ_POOL
