@@ -1,19 +1,22 @@
 """Benchmark of the FQT quantized backward on GB300.
 
-One step = one pass of the whole hot path over one batch of the ResNet-18
-3x3 conv backward (batch 128, 32x32, 64 -> 64 channels, im2col N = 131072,
-C = 64, D = 576):
+One step = one pass of the whole hot path over the full ResNet-50 v1.5
+backward at batch 256, 224 x 224 (53 convolutions and the fc, each lowered to
+im2col; 4.19 TOP of integer contractions):  for every layer
   X~ = Q_f(X), W~ = Q_theta(W)            (deterministic 8-bit PTQ)
   Q_b2(dH) = BHQ 5-bit, block 16; Q_b1(dH) = 8-bit stochastic PTQ
   grad_X = Q_b2(dH) W~,  grad_W = Q_b1(dH)^T X~
 The reported value is quantized-backward throughput in TOPS: both
-contractions count 2 N C D integer ops each.  Inputs are resident in HBM
-when timing starts; L2 is flushed (256 MiB write) between timed steps.
+contractions count 2 N C D integer ops each.  Every layer's inputs (34 GB of
+fp32 dH, X, W) are resident in HBM when timing starts; a step moves far more
+than the 129 MB L2, so no flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
 The reference arm times the CPU oracle on a bounded sample of the same
-workload on the host cores.
+workload (every layer at batch 1) on all host cores.  The other workloads
+(the linear layer, the ResNet-18 and ResNet-50 layer3 convs, the transformer
+FFN pair) and the method's variants are reported as extras.
 """
 from __future__ import annotations
 
@@ -32,23 +35,29 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "quantized-backward TOPS and quantizer GB/s (1 GB300) vs roofline, oracle-exact"
-WORKLOAD = "resnet18-conv3x3-b128-32x32-64ch (im2col N=131072, C=64, D=576)"
-KIND, BITS, BLOCK = 2, 5, 16  # BHQ-5, block 16
-CONFIG_INDEX = 1
+WORKLOAD = ("resnet50-sweep-b256-224x224: ResNet-50 v1.5 backward, batch 256, 53 convs + fc "
+            "via im2col (stem D 147 -> 160, fc C 1000 -> 1008 zero-padded)")
+KIND, BITS, BLOCK = 2, 5, 16  # Q_b2 = BHQ-5, block 16
+SWEEP_BATCH = 256
+CALLS = ["quantize_act", "quantize_weight", "quantize_grad", "grad_x", "grad_w"]
+KERNELS = {"quantize_act": "k_range + k_fwd_codes", "quantize_weight": "k_range + k_fwd_codes",
+           "quantize_grad": "k_range + k_bhq_warp", "grad_x": "k_gemm",
+           "grad_w": "k_gradw (or split-K k_gemm) + k_reduce"}
 
 
 def _peaks():
+    """(HBM GB/s, bf16 dense TFLOP/s burst, source)."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             p = json.load(f)
-        return float(p["hbm_gbs"]), "measured"
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
     except Exception:
-        return 6800.0, "fallback"
+        return 6800.0, 1900.0, "fallback"
 
 
-def _traffic_record(kernel: str):
-    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if the
-    summary was taken on the current kernel source."""
+def _traffic_record(kernel: str, workload: str):
+    """Per-launch DRAM bytes of `kernel` on `workload` from the committed ncu
+    summary, if that summary was taken on the current kernel sources."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.md")
     try:
         text = open(path).read()
@@ -62,9 +71,9 @@ def _traffic_record(kernel: str):
     digest = h.hexdigest()[:16]
     for line in text.splitlines():
         parts = [p.strip() for p in line.strip().strip("|").split("|")]
-        if len(parts) >= 3 and parts[0] == kernel and parts[2] == digest:
+        if len(parts) >= 4 and parts[0] == kernel and parts[1] == workload and parts[3] == digest:
             try:
-                return float(parts[1])
+                return float(parts[2])
             except ValueError:
                 return None
     return None
@@ -161,10 +170,10 @@ def _dist():
     return ws, rank, local
 
 
-def rank_seed(rank: int) -> int:
-    """Seed of a rank's synthetic batch: replicas process independent batches
+def rank_seed(rank: int, layer: int) -> int:
+    """Seed of a rank's synthetic layer: replicas process independent batches
     of the same shapes and distributions (weak scaling)."""
-    return 1234 + CONFIG_INDEX + 1000 * rank
+    return 1234 + 4 + layer + 1000 * rank
 
 
 def max_over_ranks(value: float, device) -> float:
@@ -179,6 +188,157 @@ def max_over_ranks(value: float, device) -> float:
     return float(t.item())
 
 
+# ---------------------------------------------------------------------------
+# Algorithmic work per call: each input read once, each output written once,
+# codes at 1 byte each, per-row / per-column metadata at 4 bytes per entry.
+# (The library's contractions read 2-byte fp16 carriers of the codes; the
+# carriers, a PTQ range pass's second read of its input and any re-read from
+# L2 are traffic, not algorithmic bytes.)
+# ---------------------------------------------------------------------------
+def alg_bytes(N: int, C: int, D: int, eb: int = 4, block: int = BLOCK) -> dict:
+    nblk = (N + block - 1) // block if block else 0
+    return {
+        "quantize_act": N * D * eb + N * D + D * 4 + 8,
+        "quantize_weight": C * D * eb + C * D + D * 4 + 8,
+        "quantize_grad": N * C * eb + 2 * N * C + N * 20 + nblk * 4 + C * 4 + 8,
+        "grad_x": N * C + C * D + N * D * 4 + N * 12 + nblk * 4 + D * 4,
+        "grad_w": N * C + N * D + C * D * 4 + (C + D) * 4,
+    }
+
+
+def launches(C: int, kind: int = KIND, block: int = BLOCK) -> dict:
+    """Kernels each call launches (fixed by the library's dispatch)."""
+    warp_bhq = kind == KIND and block > 0 and C in (64, 128, 256)
+    return {"quantize_act": 2, "quantize_weight": 2,
+            "quantize_grad": 2 if (warp_bhq or kind != KIND) else 3,
+            "grad_x": 1, "grad_w": 2}
+
+
+def sweep_layer_tensors(sh, batch: int, seed: int, dev):
+    """One layer of the sweep drawn on the device with torch's seeded
+    generator: the recipe of workloads.resnet50_layer (input U[-1, 1] at the
+    layer's input shape lowered by im2col, dH N(0, 1) rows scaled by
+    lognormal(0, 2), W N(0, 2 / D); D and C zero-padded to multiples of 16)."""
+    import torch
+    import torch.nn.functional as F
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(seed)
+    Ns, Dp, Cp = sh.rows(batch), sh.D_pad, sh.C_pad
+    X = torch.zeros((Ns, Dp), dtype=torch.float32, device=dev)
+    # im2col in slices of the batch (the unfolded tensor of a whole layer can
+    # exceed 2 GB)
+    per = max(1, batch // 8)
+    r0 = 0
+    for b0 in range(0, batch, per):
+        nb = min(per, batch - b0)
+        x = torch.rand((nb, sh.cin, sh.h, sh.h), generator=gen, device=dev) * 2.0 - 1.0
+        cols = F.unfold(x, sh.k, padding=sh.pad, stride=sh.stride)
+        rows = nb * sh.hout * sh.hout
+        X[r0:r0 + rows, :sh.D] = (cols.view(nb, sh.cin, sh.k * sh.k, -1).permute(0, 3, 2, 1)
+                                  .reshape(rows, sh.D))
+        r0 += rows
+        del x, cols
+    dH = torch.zeros((Ns, Cp), dtype=torch.float32, device=dev)
+    dH[:, :sh.cout] = (torch.randn((Ns, sh.cout), generator=gen, device=dev)
+                       * torch.exp(2.0 * torch.randn((Ns, 1), generator=gen, device=dev)))
+    W = torch.zeros((Cp, Dp), dtype=torch.float32, device=dev)
+    W[:sh.cout, :sh.D] = (torch.randn((sh.cout, sh.D), generator=gen, device=dev)
+                          * float(np.sqrt(2.0 / sh.D)))
+    return dH, X, W
+
+
+class LayerState:
+    """Device-resident operands, codes and outputs of one layer and its five
+    C-ABI calls (Q_f, Q_theta, Q_b2 + Q_b1, grad_X, grad_W)."""
+
+    def __init__(self, fqt, dH, X, W, ws, kind=KIND, bits=BITS, block=BLOCK, seed=5):
+        dev = dH.device
+        N, C = dH.shape
+        D = X.shape[1]
+        self.N, self.C, self.D = N, C, D
+        self.dH, self.X, self.W = dH, X, W
+        self.kind, self.bits, self.block, self.seed = kind, bits, block, seed
+        self.qx = fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+        self.qw = fqt.QTensor.empty(C, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+        self.q2 = fqt.QTensor.empty(N, C, kind, bits, block, True, False, dev, u8=False)
+        self.q1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+        self.gx = torch_empty((N, D), dev)
+        self.gw = torch_empty((C, D), dev)
+        self.ws = ws
+        self.fqt = fqt
+
+    def calls(self, dH=None, X=None, W=None, gx=None, gw=None, seed=None):
+        f, ws = self.fqt, self.ws
+        dH = self.dH if dH is None else dH
+        X = self.X if X is None else X
+        W = self.W if W is None else W
+        gx = self.gx if gx is None else gx
+        gw = self.gw if gw is None else gw
+        seed = self.seed if seed is None else seed
+        return [
+            lambda: f.quantize_act(X, 8, ws=ws, out=self.qx),
+            lambda: f.quantize_weight(W, 8, ws=ws, out=self.qw),
+            lambda: f.quantize_grad(dH, self.kind, self.bits, self.block, seed, ws=ws,
+                                    q_b2=self.q2, q_b1=self.q1),
+            lambda: f.linear_backward(self.q2, self.q1, self.qx, self.qw, grad_x=True,
+                                      grad_w=False, ws=ws, out_x=gx),
+            lambda: f.linear_backward(self.q2, self.q1, self.qx, self.qw, grad_x=False,
+                                      grad_w=True, ws=ws, out_w=gw),
+        ]
+
+
+def torch_empty(shape, dev):
+    import torch
+    return torch.empty(shape, dtype=torch.float32, device=dev)
+
+
+def capture(fns):
+    """One CUDA graph per call (the library's launches on the capturing
+    stream): the timed replays carry no host launch overhead."""
+    import torch
+    graphs = []
+    for f in fns:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            f()
+        graphs.append(g)
+    return graphs
+
+
+def roofline_of(call: str, rows, hbm_peak: float, bf16_peak: float):
+    """Roofline of one call type over the sweep's layers.  rows: per layer
+    (ms, algorithmic bytes, ops).  A contraction is HBM-bound on a layer when
+    its ops per algorithmic byte are below the ridge (tensor peak of the fp16
+    kind = the measured bf16 peak, over the measured HBM copy bandwidth);
+    `achieved` aggregates the launches on the binding side that takes most
+    of the call's time."""
+    ridge = bf16_peak * 1e12 / (hbm_peak * 1e9)
+    hb = [(ms, by, op) for ms, by, op in rows if not op or op / by < ridge]
+    tb = [(ms, by, op) for ms, by, op in rows if op and op / by >= ridge]
+    t_h, t_t = sum(r[0] for r in hb), sum(r[0] for r in tb)
+    out = {"call": call, "kernel": KERNELS[call],
+           "launches_per_call": 1 if call == "grad_x" else 2,
+           "ms": t_h + t_t}
+    if hb:
+        gbs = sum(r[1] for r in hb) / (t_h * 1e-3) / 1e9
+        out["hbm_bound_layers"] = {"n": len(hb), "ms": t_h, "achieved_GBs": gbs,
+                                   "frac": gbs / hbm_peak}
+    if tb:
+        tops = sum(r[2] for r in tb) / (t_t * 1e-3) / 1e12
+        out["tensor_bound_layers"] = {"n": len(tb), "ms": t_t, "achieved_TOPS": tops,
+                                      "frac": tops / bf16_peak}
+    if t_h >= t_t:
+        by = sum(r[1] for r in hb)
+        out.update(bound="hbm", achieved=by / (t_h * 1e-3) / 1e9, peak=hbm_peak, unit="GB/s",
+                   algorithmic_bytes=by, launches=len(hb))
+    else:
+        op = sum(r[2] for r in tb)
+        out.update(bound="tensor", achieved=op / (t_t * 1e-3) / 1e12, peak=bf16_peak,
+                   unit="TFLOP/s", algorithmic_ops=op, launches=len(tb))
+    out["frac"] = out["achieved"] / out["peak"]
+    return out
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -191,74 +351,42 @@ def run_gpu(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     fqt.load(build_if_missing=True)
     dev = torch.device("cuda", local)
-
-    L = wl.config(CONFIG_INDEX, seed=rank_seed(rank))[0]
-    N, C, D = L.N, L.C, L.D
-    dH = torch.from_numpy(L.dH).to(dev)
-    X = torch.from_numpy(L.X).to(dev)
-    W = torch.from_numpy(L.W).to(dev)
-    ws = fqt.Workspace(N, C, D, device=dev)
-    ws_fx = fqt.Workspace(N, D, 16, device=dev)
-    ws_fw = fqt.Workspace(C, D, 16, device=dev)
-    # the backward consumes the fp16 carriers of the codes (2 bytes per code)
-    qx = fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-    qw = fqt.QTensor.empty(C, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-    q2 = fqt.QTensor.empty(N, C, KIND, BITS, BLOCK, True, False, dev, u8=False)
-    q1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-    gx = torch.empty((N, D), dtype=torch.float32, device=dev)
-    gw = torch.empty((C, D), dtype=torch.float32, device=dev)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
-    names = ["quantize_act", "quantize_weight", "quantize_grad", "grad_x", "grad_w"]
-    # forward PTQ of X and of W: range + codes; Q_b2 / Q_b1: range +
-    # warp-per-block BHQ quantizer; grad_X: one contraction; grad_W:
-    # contraction + split-K reduction
-    launches_per_call = [2, 2, 2, 1, 2]
+    hbm_peak, bf16_peak, peak_src = _peaks()
 
-    def calls(seed):
-        return [
-            lambda: fqt.quantize_act(X, 8, ws=ws_fx, out=qx),
-            lambda: fqt.quantize_weight(W, 8, ws=ws_fw, out=qw),
-            lambda: fqt.quantize_grad(dH, KIND, BITS, BLOCK, seed, ws=ws, q_b2=q2, q_b1=q1),
-            lambda: fqt.linear_backward(q2, q1, qx, qw, grad_x=True, grad_w=False, ws=ws,
-                                        out_x=gx),
-            lambda: fqt.linear_backward(q2, q1, qx, qw, grad_x=False, grad_w=True, ws=ws,
-                                        out_w=gw),
-        ]
+    # ---- the sweep's layers, resident in HBM ----
+    shapes = wl.resnet50_shapes()
+    B = SWEEP_BATCH
+    big = max(shapes, key=lambda s: fqt.workspace_size(s.rows(B), s.C_pad, s.D_pad))
+    ws = fqt.Workspace(big.rows(B), big.C_pad, big.D_pad, device=dev)  # calls run in order
+    layers = []
+    for li, sh in enumerate(shapes):
+        dH, X, W = sweep_layer_tensors(sh, B, rank_seed(rank, li), dev)
+        layers.append(LayerState(fqt, dH, X, W, ws))
+    nl = len(layers)
+    ops_layer = [4 * sh.rows(B) * sh.cout * sh.D for sh in shapes]
+    ops_step = sum(ops_layer)
+    byt = [alg_bytes(L.N, L.C, L.D) for L in layers]
+    nlaunch = sum(sum(launches(L.C).values()) for L in layers)
 
-    graphs = None
-
-    def step(seed, evs=None):
-        def mark(i):
-            if evs is not None:
-                evs[i].record(stream)
-        fns = [g.replay for g in graphs] if graphs is not None else calls(seed)
-        for i, f in enumerate(fns):
-            mark(i)
-            f()
-        mark(5)
-
-    for i in range(args.warmup):
-        step(i)
+    for _ in range(args.warmup):
+        for L in layers:
+            for f in L.calls():
+                f()
     torch.cuda.synchronize()
     if fqt.sync_status(ws) != 0:
         raise RuntimeError("device-side status after warm-up")
-    if not args.eager:
-        # one CUDA graph per call (the library's launches on the capturing
-        # stream), so the timed steps carry no host launch overhead; the
-        # gradient quantizer's seed is fixed at capture
-        graphs = []
-        for f in calls(1000):
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                f()
-            graphs.append(g)
-        for i in range(2):
-            step(0)
-        torch.cuda.synchronize()
-        if fqt.sync_status(ws) != 0:
-            raise RuntimeError("device-side status after graph warm-up")
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)]
+    graphs = [capture(L.calls()) for L in layers]
+    for _ in range(2):
+        for gl in graphs:
+            for g in gl:
+                g.replay()
+    torch.cuda.synchronize()
+    if fqt.sync_status(ws) != 0:
+        raise RuntimeError("device-side status after graph warm-up")
+
+    ncalls = nl * len(CALLS)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(ncalls + 1)]
            for _ in range(args.steps)]
     if world > 1:
         dist.barrier()
@@ -268,342 +396,185 @@ def run_gpu(args):
         t_wall = time.perf_counter()
         clk.mark_start()
         for i in range(args.steps):
-            flush.fill_(i & 0xFF)  # evict L2 between timed steps
-            step(1000 + i, evs[i])
+            e, k = evs[i], 0
+            for gl in graphs:
+                for g in gl:
+                    e[k].record(stream)
+                    g.replay()
+                    k += 1
+            e[k].record(stream)
         torch.cuda.synchronize()
         clk.mark_end()
         t_wall = time.perf_counter() - t_wall
     if world > 1:
         dist.barrier()
-    per_call = np.zeros(5)
+    per = np.zeros((nl, len(CALLS)))
     step_ms = []
     for e in evs:
-        d = [e[j].elapsed_time(e[j + 1]) for j in range(5)]
-        per_call += np.array(d)
-        step_ms.append(sum(d))
-    ms_step = float(np.mean(step_ms))
-    per_call /= args.steps
-    ms_step = max_over_ranks(ms_step, dev)
+        d = np.array([e[j].elapsed_time(e[j + 1]) for j in range(ncalls)])
+        per += d.reshape(nl, len(CALLS))
+        step_ms.append(e[0].elapsed_time(e[ncalls]))
+    per /= args.steps
+    ms_step = max_over_ranks(float(np.mean(step_ms)), dev)
     status = fqt.sync_status(ws)
-
-    ops_step = 2 * 2 * N * C * D  # both contractions
     value = ops_step * world / (ms_step * 1e-3) / 1e12
 
-    # ---- roofline of the dominant kernel (largest share of the step) ----
-    hbm_peak, peak_src = _peaks()
-    # algorithmic bytes: each input read once, each output written once;
-    # codes travel as 2-byte fp16 carriers
-    cb = 2
-    alg_bytes = {
-        "quantize_act": N * D * 4 + N * D * cb + D * 4,
-        "quantize_weight": C * D * 4 + C * D * cb + D * 4,
-        "quantize_grad": N * C * 4 + 2 * N * C * cb + N * (4 + 4 + 4 + 8) + (N // BLOCK) * 4 + C * 4,
-        "grad_x": N * C * cb + C * D * cb + N * D * 4 + N * 12 + (N // BLOCK) * 4 + D * 4,
-        "grad_w": N * C * cb + N * D * cb + C * D * 4 + (C + D) * 4,
+    # ---- rooflines: every call type over the layers; the dominant one is
+    # the call with the largest share of the step ----
+    roofs = {}
+    for ci, c in enumerate(CALLS):
+        rows = [(per[li, ci], byt[li][c], ops_layer[li] // 2 if c in ("grad_x", "grad_w") else 0)
+                for li in range(nl)]
+        roofs[c] = roofline_of(c, rows, hbm_peak, bf16_peak)
+    call_ms = {c: float(per[:, ci].sum()) for ci, c in enumerate(CALLS)}
+    dom = max(CALLS, key=lambda c: call_ms[c])
+    r = roofs[dom]
+    roofline = {"bound": r["bound"], "achieved": r["achieved"], "peak": r["peak"],
+                "unit": r["unit"], "frac": r["frac"],
+                "traffic": _traffic_record(KERNELS[dom], "resnet50-sweep-b256"),
+                "kernel": r["kernel"], "call": dom, "peak_source": peak_src,
+                "launches": r["launches"],
+                "per_launch": ("algorithmic bytes and CUDA-event time summed over the "
+                               f"{r['launches']} {r['bound']}-bound launches of the step")}
+    slow = sorted(range(nl), key=lambda li: -per[li].sum())[:6]
+    result = {
+        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "u8 codes (fp16 carriers, exact int accumulation); f32 in/out",
+        "data": "synthetic (seeded on the device; shapes and value distributions of the workload)",
+        "config": {"workload": WORKLOAD, "layers": nl, "global_batch": B * world,
+                   "quantizer": "Q_b2=BHQ-5 block16, Q_b1=PTQ-8 stochastic, X~/W~=PTQ-8",
+                   "ops_per_step": ops_step,
+                   "parallelism": f"replicas x{world} (independent batches)",
+                   "l2": "no flush: inputs larger than L2 (a step reads 34 GB of fp32 inputs)",
+                   "launch": "one CUDA graph per C-ABI call, events between calls",
+                   "wall_s": t_wall},
+        "roofline": roofline,
+        "per_call_ms": call_ms,
+        "rooflines": roofs,
+        "slowest_layers": [{"layer": shapes[li].name, "N": layers[li].N, "C": shapes[li].cout,
+                            "D": shapes[li].D,
+                            "ms": dict(zip(CALLS, [float(v) for v in per[li]]))}
+                           for li in slow],
+        "stem_grad_x_ms": float(per[0, 3]),
+        "clocks": clk.summary(),
+        "gpu_launches": int(nlaunch * args.steps),
+        "device_status": status,
     }
-    kern_of = {"quantize_act": "k_range + k_fwd_codes", "quantize_weight": "k_range + k_fwd_codes",
-               "quantize_grad": "k_range + k_bhq_warp", "grad_x": "k_gemm",
-               "grad_w": "k_gradw + k_reduce"}
-    # The dominant kernel is the grad_X contraction (k_gemm, the largest
-    # share of the ncu launch list); it is the only kernel of its call, so
-    # the call's events time it alone.  The other calls launch two kernels
-    # each; their whole-call bandwidth is reported beside it.
-    dom = "grad_x"
-    achieved = alg_bytes[dom] / (per_call[names.index(dom)] * 1e-3) / 1e9
-    traffic = _traffic_record(dom)
-    quant_gbs = alg_bytes["quantize_grad"] / (per_call[2] * 1e-3) / 1e9
-    call_gbs = {k: alg_bytes[k] / (per_call[i] * 1e-3) / 1e9 for i, k in enumerate(names)}
-
-    # ---- end to end through the public API with host buffers ----
-    # Every step copies its inputs (dH, X, W) from pinned host memory, runs
-    # the five C-ABI calls and copies both gradients back.  Steps are
-    # pipelined two deep on three streams (host-to-device copies, calls,
-    # device-to-host copies) with double-buffered device inputs and outputs,
-    # so the copies of neighbouring steps overlap each other and the calls.
-    e2e = None
     if args.e2e_steps > 0:
-        h_dH = torch.from_numpy(L.dH).pin_memory()
-        h_X = torch.from_numpy(L.X).pin_memory()
-        h_W = torch.from_numpy(L.W).pin_memory()
-        h_gx = torch.empty((N, D), dtype=torch.float32).pin_memory()
-        h_gw = torch.empty((C, D), dtype=torch.float32).pin_memory()
-        sets = [dict(dH=dH, X=X, W=W, gx=gx, gw=gw),
-                dict(dH=torch.empty_like(dH), X=torch.empty_like(X), W=torch.empty_like(W),
-                     gx=torch.empty_like(gx), gw=torch.empty_like(gw))]
-        s_cmp = torch.cuda.Stream(dev)
-        # each direction's copies can be split by rows over several streams
-        # (several copy engines); one stream per direction measured fastest
-        ncs = max(1, args.e2e_copy_streams)
-        s_ins = [torch.cuda.Stream(dev) for _ in range(ncs)]
-        s_outs = [torch.cuda.Stream(dev) for _ in range(ncs)]
+        result["e2e"] = e2e_sweep(fqt, layers, shapes, ops_step * world, args, dev, stream)
+    if args.extras:
+        result["extras"] = run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(args.cpu_batch)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
 
-        def split_rows(t):
-            n_ = t.shape[0]
-            step_ = (n_ + ncs - 1) // ncs
-            return [t[i:i + step_] for i in range(0, n_, step_)]
 
-        def e2e_calls(b, seed):
-            return [lambda: fqt.quantize_act(b["X"], 8, ws=ws_fx, out=qx),
-                    lambda: fqt.quantize_weight(b["W"], 8, ws=ws_fw, out=qw),
-                    lambda: fqt.quantize_grad(b["dH"], KIND, BITS, BLOCK, seed, ws=ws, q_b2=q2,
-                                              q_b1=q1),
-                    lambda: fqt.linear_backward(q2, q1, qx, qw, ws=ws, out_x=b["gx"],
-                                                out_w=b["gw"])]
+def e2e_sweep(fqt, layers, shapes, ops_step, args, dev, stream):
+    """The same step through the public API with host buffers: every layer's
+    dH, X and W are copied from pinned host memory and its grad_X and grad_W
+    copied back, every step.  Layers are pipelined on three streams
+    (host-to-device copies, the C-ABI calls, device-to-host copies) through
+    two device staging sets sized for the largest layer, so the copies of
+    neighbouring layers overlap each other and the calls."""
+    import torch
+    h_in, h_out = [], []
+    try:
+        for L in layers:
+            ins = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in (L.dH, L.X, L.W)]
+            for h, t in zip(ins, (L.dH, L.X, L.W)):
+                h.copy_(t)
+            h_in.append(ins)
+            h_out.append([torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                          for t in (L.gx, L.gw)])
+    except RuntimeError as exc:  # pinned host memory exhausted
+        return {"value": None, "unit": "TOPS", "error": f"pinned host buffers: {exc}"[:200]}
+    sz = {k: max(getattr(L, k).numel() for L in layers) for k in ("dH", "X", "W", "gx", "gw")}
+    sets = [{k: torch.empty(n, dtype=torch.float32, device=dev) for k, n in sz.items()}
+            for _ in range(2)]
+    view = lambda s, k, t: s[k][:t.numel()].view(t.shape)
+    s_in, s_cmp, s_out = (torch.cuda.Stream(dev) for _ in range(3))
+    done_cmp, done_out = [None, None], [None, None]
 
-        def run_e2e(nsteps, seed0):
-            done_cmp, done_out = [None, None], [None, None]
-            for i in range(nsteps):
-                b = sets[i & 1]
-                eins = []
-                for si, s_in in enumerate(s_ins):
-                    with torch.cuda.stream(s_in):
-                        if done_cmp[i & 1] is not None:  # step i-2 has read these inputs
-                            s_in.wait_event(done_cmp[i & 1])
-                        for k, hsrc in (("dH", h_dH), ("X", h_X), ("W", h_W)):
-                            dst_, src_ = split_rows(b[k]), split_rows(hsrc)
-                            if si < len(dst_):
-                                dst_[si].copy_(src_[si], non_blocking=True)
-                        ein = torch.cuda.Event()
-                        ein.record(s_in)
-                        eins.append(ein)
+    def run(nsteps, seed0):
+        g = 0
+        for i in range(nsteps):
+            for li, L in enumerate(layers):
+                s = sets[g & 1]
+                with torch.cuda.stream(s_in):
+                    if done_cmp[g & 1] is not None:  # the layer before has read the set
+                        s_in.wait_event(done_cmp[g & 1])
+                    for k, h in zip(("dH", "X", "W"), h_in[li]):
+                        view(s, k, h).copy_(h, non_blocking=True)
+                    ein = torch.cuda.Event()
+                    ein.record(s_in)
                 with torch.cuda.stream(s_cmp):
-                    for ein in eins:
-                        s_cmp.wait_event(ein)
-                    if done_out[i & 1] is not None:  # step i-2's gradients have left
-                        for eo in done_out[i & 1]:
-                            s_cmp.wait_event(eo)
-                    for f in e2e_calls(b, seed0 + i):
+                    s_cmp.wait_event(ein)
+                    if done_out[g & 1] is not None:  # its gradients have left
+                        s_cmp.wait_event(done_out[g & 1])
+                    for f in L.calls(dH=view(s, "dH", L.dH), X=view(s, "X", L.X),
+                                     W=view(s, "W", L.W), gx=view(s, "gx", L.gx),
+                                     gw=view(s, "gw", L.gw), seed=seed0 + i):
                         f()
                     ec = torch.cuda.Event()
                     ec.record(s_cmp)
-                    done_cmp[i & 1] = ec
-                eos = []
-                for si, s_out in enumerate(s_outs):
-                    with torch.cuda.stream(s_out):
-                        s_out.wait_event(ec)
-                        for hdst, k in ((h_gx, "gx"), (h_gw, "gw")):
-                            dst_, src_ = split_rows(hdst), split_rows(b[k])
-                            if si < len(dst_):
-                                dst_[si].copy_(src_[si], non_blocking=True)
-                        eo = torch.cuda.Event()
-                        eo.record(s_out)
-                        eos.append(eo)
-                done_out[i & 1] = eos
-            for st_ in s_ins + [s_cmp] + s_outs:
-                stream.wait_stream(st_)
+                    done_cmp[g & 1] = ec
+                with torch.cuda.stream(s_out):
+                    s_out.wait_event(ec)
+                    for k, h in zip(("gx", "gw"), h_out[li]):
+                        h.copy_(view(s, k, h), non_blocking=True)
+                    eo = torch.cuda.Event()
+                    eo.record(s_out)
+                    done_out[g & 1] = eo
+                g += 1
+        for st_ in (s_in, s_cmp, s_out):
+            stream.wait_stream(st_)
 
-        run_e2e(2, 2000)  # warms the pinned-copy path and the streams
-        torch.cuda.synchronize()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        flush.fill_(7)
-        torch.cuda.synchronize()
-        e0.record(stream)
-        for st_ in s_ins + [s_cmp] + s_outs:
-            st_.wait_stream(stream)
-        run_e2e(args.e2e_steps, 3000)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
-        e2e = {"value": ops_step * world / (e2e_ms * 1e-3) / 1e12, "unit": "TOPS",
-               "ms_per_step": e2e_ms,
-               "h2d_bytes_per_step": int((N * C + N * D + C * D) * 4),
-               "d2h_bytes_per_step": int((N * D + C * D) * 4),
-               "schedule": ("2-deep pipeline: H2D / C-ABI calls / D2H on three streams, "
-                            "double-buffered device inputs and outputs, eager calls" if ncs == 1 else
-                            f"2-deep pipeline: H2D on {ncs} streams / C-ABI calls / D2H on {ncs} "
-                            "streams (each copy split by rows), double-buffered device inputs and "
-                            "outputs, eager calls")}
+    run(1, 2000)  # warms the pinned-copy path and the streams
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for st_ in (s_in, s_cmp, s_out):
+        st_.wait_stream(stream)
+    run(args.e2e_steps, 3000)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.e2e_steps
+    h2d = sum(sum(t.numel() * 4 for t in (L.dH, L.X, L.W)) for L in layers)
+    d2h = sum(sum(t.numel() * 4 for t in (L.gx, L.gw)) for L in layers)
+    status = fqt.sync_status(layers[0].ws)
+    del h_in, h_out, sets
+    return {"value": ops_step / (ms * 1e-3) / 1e12, "unit": "TOPS", "ms_per_step": ms,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "schedule": "layers pipelined on three streams (H2D / C-ABI calls / D2H), two "
+                        "device staging sets, pinned host buffers per layer, eager calls",
+            "device_status": status}
 
-    # ---- the quantized forward GEMM H = X~ W~^T on the same layer (the
-    # contraction core with the roles renamed), timed alone ----
-    fwd = None
-    if args.forward_steps > 0:
-        qxr = fqt.quantize_act(X, 8, row_sum=True)
-        qwr = fqt.quantize_weight(W, 8, row_sum=True)
-        H = torch.empty((N, C), dtype=torch.float32, device=dev)
-        wsf = fqt.Workspace(1, 16, 16, device=dev)
-        for _ in range(3):
-            fqt.linear_forward(qxr, qwr, ws=wsf, out=H)
-        tf = []
-        for i in range(args.forward_steps):
-            flush.fill_(i & 0xFF)
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            fqt.linear_forward(qxr, qwr, ws=wsf, out=H)
-            e1.record(stream)
-            torch.cuda.synchronize()
-            tf.append(e0.elapsed_time(e1))
-        fwd_ms = float(np.median(tf))
-        fwd_bytes = N * D * cb + C * D * cb + N * C * 4 + N * 8 + C * 4
-        fwd = {"call": "linear_forward (H = X~ W~^T, one k_gemm launch)", "ms": fwd_ms,
-               "TOPS": 2 * N * C * D / (fwd_ms * 1e-3) / 1e12,
-               "algorithmic_bytes": fwd_bytes,
-               "GBs": fwd_bytes / (fwd_ms * 1e-3) / 1e9,
-               "frac_of_hbm": fwd_bytes / (fwd_ms * 1e-3) / 1e9 / hbm_peak,
-               "device_status": fqt.sync_status(wsf)}
 
-    # ---- adaptive BHQ groups (App. D.5) on the same layer: Q_b2 with the
-    # grouping chosen for this batch (sort, estimate, layout, group
-    # quantizer), then grad_X (contraction + the groups' reflection pass);
-    # one CUDA graph per call, timed alone ----
-    ada = None
-    if args.adaptive_steps > 0:
-        qa = fqt.QTensor.empty(N, C, fqt.BHQ, BITS, 0, True, False, dev, u8=False)
-        qa1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-        fa = [lambda: fqt.quantize_grad(dH, fqt.BHQ, BITS, 0, 7, ws=ws, q_b2=qa, q_b1=qa1),
-              lambda: fqt.linear_backward(qa, qa1, qx, qw, grad_x=True, grad_w=False, ws=ws,
-                                          out_x=gx)]
-        for _ in range(3):
-            for f in fa:
-                f()
-        torch.cuda.synchronize()
-        ga = []
-        for f in fa:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                f()
-            ga.append(g)
-        ta = [[], []]
-        for i in range(args.adaptive_steps):
-            flush.fill_(i & 0xFF)
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-            ev[0].record(stream)
-            ga[0].replay()
-            ev[1].record(stream)
-            ga[1].replay()
-            ev[2].record(stream)
-            torch.cuda.synchronize()
-            ta[0].append(ev[0].elapsed_time(ev[1]))
-            ta[1].append(ev[1].elapsed_time(ev[2]))
-        G = int((qa.gstart[:N] < N).sum().item())
-        grouped = int((qa.gsize > 1).sum().item())
-        ada = {"quantizer": f"BHQ-{BITS}, adaptive groups (block 0)",
-               "quantize_grad_ms": float(np.median(ta[0])),
-               "grad_x_ms": float(np.median(ta[1])),
-               "fixed_block16_ms": {"quantize_grad": float(per_call[2]),
-                                    "grad_x": float(per_call[3])},
-               "groups": G, "rows_in_multirow_groups": grouped,
-               "launches": {"quantize_grad": 10, "grad_x": 3},
-               "device_status": fqt.sync_status(ws)}
+def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
+    """The other workloads and the method's variants, each call replayed as
+    one CUDA graph and timed alone (median over rounds, L2 flushed before
+    each round)."""
+    import torch
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    steps = args.extra_steps
 
-    # ---- the per-sample power-of-two shift quantizer (Sec. 4.3) on the same
-    # layer: one code set feeds both contractions (no Q_b1); one CUDA graph
-    # per call, timed alone ----
-    shf = None
-    if args.shift_steps > 0:
-        qs = fqt.QTensor.empty(N, C, fqt.SHIFT, BITS, 0, True, False, dev, u8=False)
-        fs = [lambda: fqt.quantize_grad(dH, fqt.SHIFT, BITS, 0, 11, with_b1=False, ws=ws,
-                                        q_b2=qs),
-              lambda: fqt.linear_backward(qs, None, qx, qw, grad_x=True, grad_w=False, ws=ws,
-                                          out_x=gx),
-              lambda: fqt.linear_backward(qs, None, qx, qw, grad_x=False, grad_w=True, ws=ws,
-                                          out_w=gw)]
-        for _ in range(3):
-            for f in fs:
-                f()
-        torch.cuda.synchronize()
-        gs_ = []
-        for f in fs:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                f()
-            gs_.append(g)
-        tsh = [[], [], []]
-        for i in range(args.shift_steps):
-            flush.fill_(i & 0xFF)
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-            for k in range(3):
-                ev[k].record(stream)
-                gs_[k].replay()
-            ev[3].record(stream)
-            torch.cuda.synchronize()
-            for k in range(3):
-                tsh[k].append(ev[k].elapsed_time(ev[k + 1]))
-        sh = qs.shift.cpu().numpy()
-        shf = {"quantizer": f"SHIFT-{BITS} (per-tensor range, per-row shifts in [0, 4])",
-               "quantize_grad_ms": float(np.median(tsh[0])),
-               "grad_x_ms": float(np.median(tsh[1])),
-               "grad_w_ms": float(np.median(tsh[2])),
-               "bifurcated_bhq16_ms": {"quantize_grad": float(per_call[2]),
-                                       "grad_x": float(per_call[3]),
-                                       "grad_w": float(per_call[4])},
-               "rows_per_shift": [int((sh == k).sum()) for k in range(5)],
-               "launches": {"quantize_grad": 2, "grad_x": 1, "grad_w": 2},
-               "device_status": fqt.sync_status(ws)}
-
-    # ---- the same step with X~ as an implicit im2col operand: the forward
-    # PTQ reads the NHWC input once (the im2col matrix is never formed) and
-    # grad_W reads its boxes at shifted pixel coordinates; codes and grad_W
-    # are bit-identical to the explicit path ----
-    imp = None
-    if args.implicit_steps > 0 and L.x_nhwc is not None:
-        xn = torch.from_numpy(L.x_nhwc).to(dev)
-        nb, hh, ww, cc = L.x_nhwc.shape
-        qc = None
-
-        def qconv():
-            nonlocal qc
-            qc = fqt.quantize_act_conv(xn, 3, 3, 1, 8, ws=ws_fx, out=qc)
-        qconv()
-        fi = [qconv,
-              lambda: fqt.quantize_weight(W, 8, ws=ws_fw, out=qw),
-              lambda: fqt.quantize_grad(dH, KIND, BITS, BLOCK, 1000, ws=ws, q_b2=q2, q_b1=q1),
-              lambda: fqt.linear_backward(q2, q1, qx, qw, grad_x=True, grad_w=False, ws=ws,
-                                          out_x=gx),
-              lambda: fqt.linear_backward(q2, q1, qc, qw, grad_x=False, grad_w=True, ws=ws,
-                                          out_w=gw)]
-        for _ in range(3):
-            for f in fi:
-                f()
-        torch.cuda.synchronize()
-        gi = []
-        for f in fi:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                f()
-            gi.append(g)
-        ti = [[] for _ in fi]
-        for i in range(args.implicit_steps):
-            flush.fill_(i & 0xFF)
-            ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(fi) + 1)]
-            for k in range(len(fi)):
-                ev[k].record(stream)
-                gi[k].replay()
-            ev[-1].record(stream)
-            torch.cuda.synchronize()
-            for k in range(len(fi)):
-                ti[k].append(ev[k].elapsed_time(ev[k + 1]))
-        per = [float(np.median(t)) for t in ti]
-        ms_imp = sum(per)
-        imp = {"x_input": f"NHWC {nb}x{hh}x{ww}x{cc}, 3x3 taps, pad 1, stride 1",
-               "per_call_ms": dict(zip(["quantize_act_conv", "quantize_weight", "quantize_grad",
-                                        "grad_x", "grad_w"], per)),
-               "ms_per_step": ms_imp,
-               "TOPS": ops_step / (ms_imp * 1e-3) / 1e12,
-               "explicit_ms": {"quantize_act": float(per_call[0]), "grad_w": float(per_call[4])},
-               "launches_per_step": 10,
-               "device_status": fqt.sync_status(ws)}
-
-    def time_graphs(fns, steps):
-        """Median ms of each call, replayed as one CUDA graph per call, L2
-        flushed before each round."""
+    def time_graphs(fns):
         for _ in range(3):
             for f in fns:
                 f()
         torch.cuda.synchronize()
-        gs_ = []
-        for f in fns:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                f()
-            gs_.append(g)
+        gs = capture(fns)
         tt = [[] for _ in fns]
         for i in range(steps):
             flush.fill_(i & 0xFF)
             ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(fns) + 1)]
-            for k, g in enumerate(gs_):
+            for k, g in enumerate(gs):
                 ev[k].record(stream)
                 g.replay()
             ev[-1].record(stream)
@@ -612,250 +583,220 @@ def run_gpu(args):
                 tt[k].append(ev[k].elapsed_time(ev[k + 1]))
         return [float(np.median(t)) for t in tt]
 
-    bf16_peak = 1862.7
-    try:
-        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            bf16_peak = float(json.load(f)["bf16_tflops"])
-    except Exception:
-        pass
+    def on_dev(Lw):
+        dt = torch.bfloat16 if Lw.dtype == "bf16" else torch.float32
+        return [torch.from_numpy(a).to(dev).to(dt) for a in (Lw.dH, Lw.X, Lw.W)]
 
-    # ---- the other full-size workloads: one backward step per layer, each
-    # contraction against its binding roofline (HBM bytes with 2-byte code
-    # carriers, or the tensor peak of the fp16 kind = the measured bf16 peak) ----
-    others = None
-    if args.config_steps > 0:
-        others = []
-        for cfg in (2, 3):
-            for Lo in wl.config(cfg):
-                No, Co, Do = Lo.N, Lo.C, Lo.D
-                dt = torch.bfloat16 if Lo.dtype == "bf16" else torch.float32
-                to = lambda a: torch.from_numpy(a).to(dev).to(dt)
-                dHo, Xo, Wo = to(Lo.dH), to(Lo.X), to(Lo.W)
-                wso = fqt.Workspace(No, Co, Do, device=dev)
-                qxo = fqt.QTensor.empty(No, Do, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-                qwo = fqt.QTensor.empty(Co, Do, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-                q2o = fqt.QTensor.empty(No, Co, fqt.BHQ, 5, 16, True, False, dev, u8=False)
-                q1o = fqt.QTensor.empty(No, Co, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-                gxo = torch.empty((No, Do), dtype=torch.float32, device=dev)
-                gwo = torch.empty((Co, Do), dtype=torch.float32, device=dev)
-                wfx = fqt.Workspace(No, Do, 16, device=dev)
-                wfw = fqt.Workspace(Co, Do, 16, device=dev)
-                fo = [lambda: fqt.quantize_act(Xo, 8, ws=wfx, out=qxo),
-                      lambda: fqt.quantize_weight(Wo, 8, ws=wfw, out=qwo),
-                      lambda: fqt.quantize_grad(dHo, fqt.BHQ, 5, 16, 5, ws=wso, q_b2=q2o,
-                                                q_b1=q1o),
-                      lambda: fqt.linear_backward(q2o, q1o, qxo, qwo, grad_x=True, grad_w=False,
-                                                  ws=wso, out_x=gxo),
-                      lambda: fqt.linear_backward(q2o, q1o, qxo, qwo, grad_x=False, grad_w=True,
-                                                  ws=wso, out_w=gwo)]
-                per = time_graphs(fo, args.config_steps)
-                ops = 2 * No * Co * Do
-                eb = 2 if Lo.dtype == "bf16" else 4
-                bytes_x = No * Co * 2 + Co * Do * 2 + No * Do * 4 + No * 12 + (No // 16) * 4
-                bytes_w = No * Co * 2 + No * Do * 2 + Co * Do * 4 + (Co + Do) * 4
-                roof = {}
-                for name, ms, by in (("grad_x", per[3], bytes_x), ("grad_w", per[4], bytes_w)):
-                    gbs = by / (ms * 1e-3) / 1e9
-                    tops = ops / (ms * 1e-3) / 1e12
-                    hbm_bound = ops / by < bf16_peak * 1e12 / (hbm_peak * 1e9)
-                    roof[name] = {"bound": "hbm" if hbm_bound else "tensor", "ms": ms,
-                                  "TOPS": tops, "GBs": gbs,
-                                  "frac": gbs / hbm_peak if hbm_bound else tops / bf16_peak,
-                                  "ops_per_byte": ops / by}
-                others.append({"workload": Lo.name, "N": No, "C": Co, "D": Do,
-                               "dtype": Lo.dtype, "quantizer": "BHQ-5 block 16 + Q_b1 PTQ-8",
-                               "per_call_ms": dict(zip(["quantize_act", "quantize_weight",
-                                                        "quantize_grad", "grad_x", "grad_w"],
-                                                       per)),
-                               "ms_per_step": sum(per),
-                               "TOPS": 2 * ops / (sum(per) * 1e-3) / 1e12,
-                               "quantize_grad_GBs": (No * Co * eb + 2 * No * Co * 2 + No * 20)
-                               / (per[2] * 1e-3) / 1e9,
-                               "roofline": roof, "device_status": fqt.sync_status(wso)})
-                del dHo, Xo, Wo, qxo, qwo, q2o, q1o, gxo, gwo, wso, wfx, wfw
-                torch.cuda.empty_cache()
-
-    # ---- the full ResNet-50 backward sweep at batch 256, 224 x 224: every conv
-    # (and the fc) lowered to im2col, BHQ-5/16 + Q_b1 PTQ-8 gradients, 8-bit
-    # X~ and W~; inputs drawn on the device from the same recipe as
-    # workloads.resnet50_layer (the host draw is 40+ GB) ----
-    sweep = None
-    if args.sweep_steps > 0:
-        import torch.nn.functional as F
-        layers_out = []
-        tot = {"quantize_act": 0.0, "quantize_weight": 0.0, "quantize_grad": 0.0,
-               "grad_x": 0.0, "grad_w": 0.0}
-        ops_all = 0
-        st_all = 0
-        bsz = 256
-        for li, sh in enumerate(wl.resnet50_shapes()):
-            gen = torch.Generator(device=dev)
-            gen.manual_seed(1234 + 4 + li)
-            Ns, Dp, Cp = sh.rows(bsz), sh.D_pad, sh.C_pad
-            x = torch.rand((bsz, sh.cin, sh.h, sh.h), generator=gen, device=dev) * 2.0 - 1.0
-            cols = F.unfold(x, sh.k, padding=sh.pad, stride=sh.stride)
-            del x
-            Xs = torch.zeros((Ns, Dp), dtype=torch.float32, device=dev)
-            Xs[:, :sh.D] = cols.view(bsz, sh.cin, sh.k * sh.k, -1).permute(0, 3, 2, 1).reshape(Ns, sh.D)
-            del cols
-            dHs = torch.zeros((Ns, Cp), dtype=torch.float32, device=dev)
-            dHs[:, :sh.cout] = (torch.randn((Ns, sh.cout), generator=gen, device=dev)
-                                * torch.exp(2.0 * torch.randn((Ns, 1), generator=gen, device=dev)))
-            Ws = torch.zeros((Cp, Dp), dtype=torch.float32, device=dev)
-            Ws[:sh.cout, :sh.D] = (torch.randn((sh.cout, sh.D), generator=gen, device=dev)
-                                   * float(np.sqrt(2.0 / sh.D)))
-            wss = fqt.Workspace(Ns, Cp, Dp, device=dev)
-            qxs = fqt.QTensor.empty(Ns, Dp, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-            qws = fqt.QTensor.empty(Cp, Dp, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-            q2s = fqt.QTensor.empty(Ns, Cp, fqt.BHQ, 5, 16, True, False, dev, u8=False)
-            q1s = fqt.QTensor.empty(Ns, Cp, fqt.PTQ, 8, 0, False, True, dev, u8=False)
-            gxs = torch.empty((Ns, Dp), dtype=torch.float32, device=dev)
-            gws = torch.empty((Cp, Dp), dtype=torch.float32, device=dev)
-            wfxs = fqt.Workspace(Ns, Dp, 16, device=dev)
-            wfws = fqt.Workspace(Cp, Dp, 16, device=dev)
-            fs = [lambda: fqt.quantize_act(Xs, 8, ws=wfxs, out=qxs),
-                  lambda: fqt.quantize_weight(Ws, 8, ws=wfws, out=qws),
-                  lambda: fqt.quantize_grad(dHs, fqt.BHQ, 5, 16, 5, ws=wss, q_b2=q2s, q_b1=q1s),
-                  lambda: fqt.linear_backward(q2s, q1s, qxs, qws, grad_x=True, grad_w=False,
-                                              ws=wss, out_x=gxs),
-                  lambda: fqt.linear_backward(q2s, q1s, qxs, qws, grad_x=False, grad_w=True,
-                                              ws=wss, out_w=gws)]
-            per = time_graphs(fs, args.sweep_steps)
-            for k_, v_ in zip(tot, per):
-                tot[k_] += v_
-            ops_l = 2 * 2 * Ns * sh.cout * sh.D
-            ops_all += ops_l
-            st_all |= fqt.sync_status(wss)
-            layers_out.append({"layer": sh.name, "N": Ns, "C": sh.cout, "D": sh.D,
-                               "backward_ms": per[2] + per[3] + per[4], "grad_x_ms": per[3],
-                               "TOPS": ops_l / ((per[3] + per[4]) * 1e-3) / 1e12})
-            del Xs, dHs, Ws, wss, qxs, qws, q2s, q1s, gxs, gws, wfxs, wfws
-            torch.cuda.empty_cache()
-        bwd = tot["quantize_grad"] + tot["grad_x"] + tot["grad_w"]
-        slow = sorted(layers_out, key=lambda r: -r["backward_ms"])[:5]
-        sweep = {"workload": "ResNet-50 v1.5 backward sweep, batch 256, 224 x 224: 53 convs + fc "
-                             "via im2col (stem D 147 -> 160 and fc C 1000 -> 1008 zero-padded)",
-                 "layers": len(layers_out), "quantizer": "BHQ-5 block 16 + Q_b1 PTQ-8; X~, W~ PTQ-8",
-                 "backward_ms": bwd, "ops": ops_all, "TOPS": ops_all / (bwd * 1e-3) / 1e12,
-                 "per_call_ms_sum": tot,
-                 "forward_quantizers_ms": tot["quantize_act"] + tot["quantize_weight"],
-                 # the stem's grad_X (w.r.t. the image) is not needed in training
-                 "stem_grad_x_ms": next(r for r in layers_out if r["layer"] == "conv1")["grad_x_ms"],
-                 "slowest_layers": slow, "device_status": st_all}
-
-    # ---- the paper's own overhead shape (Sec. 4.3): a conv layer with
-    # N = 128, C = 64, 56 x 56, i.e. dH of 401408 im2col rows x 64; the paper
-    # timed its CPU routines there (context only, another machine) ----
-    ovh = None
-    if args.config_steps > 0:
-        gp = wl.rng(480)
-        dHp = torch.from_numpy(wl.random_grad(gp, 128 * 56 * 56, 64, sigma=2.0,
-                                              outlier_frac=0.01)).to(dev)
-        Np = dHp.shape[0]
-        wsp = fqt.Workspace(Np, 64, 16, device=dev)
-        qsets = {}
-        for name, kind, bits, block in (("PTQ-8", fqt.PTQ, 8, 0), ("PSQ-8", fqt.PSQ, 8, 0),
-                                        ("BHQ-5 block 16", fqt.BHQ, 5, 16),
-                                        ("BHQ-5 adaptive groups", fqt.BHQ, 5, 0)):
-            qsets[name] = (fqt.QTensor.empty(Np, 64, kind, bits, block, True, False, dev, u8=False),
-                           fqt.QTensor.empty(Np, 64, fqt.PTQ, 8, 0, False, True, dev, u8=False),
-                           kind, bits, block)
-        fns = [(lambda q=q: fqt.quantize_grad(dHp, q[2], q[3], q[4], 3, ws=wsp, q_b2=q[0],
-                                              q_b1=q[1])) for q in qsets.values()]
-        per = time_graphs(fns, args.config_steps)
-        ovh = {"shape": "dH 401408 x 64 fp32 (conv N=128, C=64, 56x56)",
-               "quantize_grad_ms": dict(zip(qsets.keys(), per)),
-               "includes": "range pass, scales / transform, SR of Q_b2 and of the 8-bit Q_b1, "
-                           "packing, row and column sums (and the grouping, adaptive)",
-               "paper_cpu_ms": {"per-tensor range": 11.0, "per-sample range": 24.0,
-                                "Householder transform": 21.0, "BHQ construction": 0.003,
-                                "INT8 conv layer": 480.0},
-               "paper_cpu_note": "1 Intel CPU core, CPU TensorFlow + AVX (Sec. 4.3): context only",
-               "device_status": fqt.sync_status(wsp)}
-        del dHp, qsets, wsp
+    def layer_runs(Lw, runs):
+        dH, X, W = on_dev(Lw)
+        eb = 2 if Lw.dtype == "bf16" else 4
+        ws = fqt.Workspace(Lw.N, Lw.C, Lw.D, device=dev)
+        out = []
+        for kind, bits, block in runs:
+            st = LayerState(fqt, dH, X, W, ws, kind, bits, block, seed=5)
+            per = time_graphs(st.calls())
+            by = alg_bytes(Lw.N, Lw.C, Lw.D, eb, block if kind == KIND else 0)
+            ops = 2 * Lw.N * Lw.C * Lw.D
+            roof = {}
+            for c, ms in (("grad_x", per[3]), ("grad_w", per[4])):
+                r = roofline_of(c, [(ms, by[c], ops)], hbm_peak, bf16_peak)
+                roof[c] = {"bound": r["bound"], "frac": r["frac"], "achieved": r["achieved"],
+                           "unit": r["unit"]}
+            name = {0: "PTQ", 1: "PSQ", 2: "BHQ"}[kind] + f"-{bits}" + (
+                f" block {block}" if kind == KIND else "")
+            out.append({"Q_b2": name, "per_call_ms": dict(zip(CALLS, per)),
+                        "ms_per_step": sum(per), "TOPS": 2 * ops / (sum(per) * 1e-3) / 1e12,
+                        "quantize_grad_GBs": by["quantize_grad"] / (per[2] * 1e-3) / 1e9,
+                        "roofline": roof, "device_status": fqt.sync_status(ws)})
+            del st
+        del dH, X, W, ws
         torch.cuda.empty_cache()
+        return out
 
-    result = {
-        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "u8 codes (fp16 carriers, exact int accumulation); f32 in/out",
-        "data": "synthetic (seeded; shapes and value distributions of the workload)",
-        "config": {"workload": WORKLOAD, "quantizer": "Q_b2=BHQ-5 block16, Q_b1=PTQ-8 stochastic, X~/W~=PTQ-8",
-                   "N": N, "C": C, "D": D, "global_batch": 128 * world,
-                   "parallelism": f"replicas x{world} (independent batches)",
-                   "l2": "flushed between timed steps (256 MiB write)",
-                   "launch": ("eager C-ABI calls" if args.eager else
-                              "one CUDA graph per call, captured from the C-ABI calls"),
-                   "wall_s": t_wall},
-        "per_call_ms": {k: float(v) for k, v in zip(names, per_call)},
-        "per_call_gbs": {k: float(v) for k, v in call_gbs.items()},
-        "quantizer_gbs": quant_gbs,
-        "roofline": {"bound": "hbm", "kernel": kern_of[dom], "call": dom,
-                     "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved / hbm_peak, "peak_source": peak_src,
-                     "algorithmic_bytes": alg_bytes[dom],
-                     "traffic": traffic},
-        "clocks": clk.summary(),
-        "e2e": e2e,
-        "forward": fwd,
-        "adaptive_bhq": ada,
-        "shift_quantizer": shf,
-        "implicit_im2col": imp,
-        "other_workloads": others,
-        "paper_overhead_shape": ovh,
-        "resnet50_sweep": sweep,
-        "gpu_launches": int(sum(launches_per_call) * args.steps),
-        "device_status": status,
-    }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(args.cpu_rows)
-        if ovh is not None:
-            # the paper timed its CPU quantizer routines on this shape (Sec.
-            # 4.3); the oracle's whole gradient quantizers on one core beside it
-            ovh["oracle_cpu_ms"] = oracle_overhead_shape()
-    if rank == 0:
-        print(json.dumps(result), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    ex = {}
+    # linear layer 128 x 256: launch-bound, reported as latency
+    L1 = wl.config(0)[0]
+    ex["linear-128x256"] = {
+        "latency": [{"Q_b2": r["Q_b2"], "step_us": r["ms_per_step"] * 1e3,
+                     "per_call_us": {k: v * 1e3 for k, v in r["per_call_ms"].items()}}
+                    for r in layer_runs(L1, [(0, 8, 0), (1, 8, 0), (KIND, 5, 16)])]}
+    L2 = wl.config(1)[0]
+    ex["resnet18-conv3x3"] = {"N": L2.N, "C": L2.C, "D": L2.D, "runs": layer_runs(
+        L2, [(k, b, 16 if k == KIND else 0) for k in (0, 1, KIND) for b in (4, 5, 8)])}
+    L3 = wl.config(2)[0]
+    ex["resnet50-layer3-conv3x3"] = {"N": L3.N, "C": L3.C, "D": L3.D, "runs": layer_runs(
+        L3, [(KIND, 5, nb) for nb in (8, 16, 32, 64)])}
+    del L3
+    for Lf in wl.config(3):
+        ex[Lf.name.split(":")[0] + ":" + Lf.name.split(":")[1]] = {
+            "N": Lf.N, "C": Lf.C, "D": Lf.D, "dtype": "bf16",
+            "runs": layer_runs(Lf, [(0, 8, 0), (1, 5, 0), (KIND, 5, 16)])}
+
+    # variants on the ResNet-18 conv layer
+    dH, X, W = on_dev(L2)
+    N, C, D = L2.N, L2.C, L2.D
+    ws = fqt.Workspace(N, C, D, device=dev)
+    base = LayerState(fqt, dH, X, W, ws)
+    per_base = time_graphs(base.calls())
+    qa = fqt.QTensor.empty(N, C, fqt.BHQ, BITS, 0, True, False, dev, u8=False)
+    qa1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+    pa = time_graphs([
+        lambda: fqt.quantize_grad(dH, fqt.BHQ, BITS, 0, 7, ws=ws, q_b2=qa, q_b1=qa1),
+        lambda: fqt.linear_backward(qa, qa1, base.qx, base.qw, grad_x=True, grad_w=False,
+                                    ws=ws, out_x=base.gx)])
+    ex["adaptive_bhq"] = {"quantizer": f"BHQ-{BITS}, adaptive groups (block 0)",
+                          "quantize_grad_ms": pa[0], "grad_x_ms": pa[1],
+                          "fixed_block16_ms": {"quantize_grad": per_base[2],
+                                               "grad_x": per_base[3]},
+                          "groups": int((qa.gstart[:N] < N).sum().item()),
+                          "device_status": fqt.sync_status(ws)}
+    qs = fqt.QTensor.empty(N, C, fqt.SHIFT, BITS, 0, True, False, dev, u8=False)
+    ps = time_graphs([
+        lambda: fqt.quantize_grad(dH, fqt.SHIFT, BITS, 0, 11, with_b1=False, ws=ws, q_b2=qs),
+        lambda: fqt.linear_backward(qs, None, base.qx, base.qw, grad_x=True, grad_w=False,
+                                    ws=ws, out_x=base.gx),
+        lambda: fqt.linear_backward(qs, None, base.qx, base.qw, grad_x=False, grad_w=True,
+                                    ws=ws, out_w=base.gw)])
+    ex["shift_quantizer"] = {"quantizer": f"SHIFT-{BITS} (per-tensor range, per-row shifts "
+                                          "in [0, 4]; no Q_b1)",
+                             "quantize_grad_ms": ps[0], "grad_x_ms": ps[1], "grad_w_ms": ps[2],
+                             "device_status": fqt.sync_status(ws)}
+    xn = torch.from_numpy(L2.x_nhwc).to(dev)
+    box = {}
+
+    def qconv():
+        box["qc"] = fqt.quantize_act_conv(xn, 3, 3, 1, 8, ws=ws, out=box.get("qc"))
+    qconv()
+    pi = time_graphs([qconv, lambda: fqt.linear_backward(base.q2, base.q1, box["qc"], base.qw,
+                                                         grad_x=False, grad_w=True, ws=ws,
+                                                         out_w=base.gw)])
+    ex["implicit_im2col"] = {"x_input": "NHWC 128x32x32x64, 3x3 taps, pad 1, stride 1",
+                             "quantize_act_conv_ms": pi[0], "grad_w_ms": pi[1],
+                             "explicit_ms": {"quantize_act": per_base[0], "grad_w": per_base[4]},
+                             "device_status": fqt.sync_status(ws)}
+    qxr = fqt.quantize_act(X, 8, row_sum=True)
+    qwr = fqt.quantize_weight(W, 8, row_sum=True)
+    H = torch.empty((N, C), dtype=torch.float32, device=dev)
+    pf = time_graphs([lambda: fqt.linear_forward(qxr, qwr, ws=ws, out=H)])
+    fb = N * D + C * D + N * C * 4 + N * 8 + C * 4
+    ex["forward"] = {"call": "linear_forward (H = X~ W~^T, one k_gemm launch)", "ms": pf[0],
+                     "TOPS": 2 * N * C * D / (pf[0] * 1e-3) / 1e12,
+                     "GBs": fb / (pf[0] * 1e-3) / 1e9,
+                     "frac_of_hbm": fb / (pf[0] * 1e-3) / 1e9 / hbm_peak}
+    del dH, X, W, ws, base, qa, qa1, qs, xn, box, qxr, qwr, H
+    torch.cuda.empty_cache()
+
+    # the paper's own overhead shape (Sec. 4.3): dH of a conv with N = 128,
+    # C = 64, 56 x 56 (401408 im2col rows); the paper timed its CPU routines
+    # there (context only, another machine)
+    dHp = torch.from_numpy(wl.random_grad(wl.rng(480), 128 * 56 * 56, 64, sigma=2.0,
+                                          outlier_frac=0.01)).to(dev)
+    Np = dHp.shape[0]
+    wsp = fqt.Workspace(Np, 64, 16, device=dev)
+    qsets = {}
+    for name, kind, bits, block in (("PTQ-8", 0, 8, 0), ("PSQ-8", 1, 8, 0),
+                                    ("BHQ-5 block 16", KIND, 5, 16),
+                                    ("BHQ-5 adaptive groups", KIND, 5, 0)):
+        qsets[name] = (fqt.QTensor.empty(Np, 64, kind, bits, block, True, False, dev, u8=False),
+                       fqt.QTensor.empty(Np, 64, fqt.PTQ, 8, 0, False, True, dev, u8=False),
+                       kind, bits, block)
+    po = time_graphs([(lambda q=q: fqt.quantize_grad(dHp, q[2], q[3], q[4], 3, ws=wsp,
+                                                      q_b2=q[0], q_b1=q[1]))
+                      for q in qsets.values()])
+    ex["paper_overhead_shape"] = {
+        "shape": "dH 401408 x 64 fp32 (conv N=128, C=64, 56x56)",
+        "quantize_grad_ms": dict(zip(qsets.keys(), po)),
+        "paper_cpu_ms": {"per-tensor range": 11.0, "per-sample range": 24.0,
+                         "Householder transform": 21.0, "INT8 conv layer": 480.0},
+        "paper_cpu_note": "1 Intel CPU core, CPU TensorFlow + AVX (Sec. 4.3): context only",
+        "device_status": fqt.sync_status(wsp)}
+    del dHp, qsets, wsp, flush
+    torch.cuda.empty_cache()
+    return ex
 
 
-def _oracle_step(L, rows: int, seed: int):
-    """One oracle pass over the first `rows` rows (the whole hot path)."""
-    import oracle as orc
-    dH, X = L.dH[:rows], L.X[:rows]
-    orc.linear_backward(dH, X, L.W, KIND, BITS, BLOCK, seed)
-    return 2 * 2 * rows * L.C * L.D
+# ---------------------------------------------------------------------------
+# The CPU oracle on the host cores: one spawned process per core, each owning
+# a fixed share of the sweep's layers (round robin), all starting each timed
+# step together at a barrier; a step's time is the span from the first
+# start to the last finish.  The oracle itself is single-threaded C.
+# ---------------------------------------------------------------------------
+def _oracle_worker(w, nproc, batch, steps, layer_ids, barrier, queue):
+    os.environ["OMP_NUM_THREADS"] = "1"
+    os.environ["OPENBLAS_NUM_THREADS"] = "1"
+    try:
+        import oracle as orc
+        from paper_2010_14298_gb300 import workloads as wl
+        shapes = wl.resnet50_shapes()
+        mine = [li for i, li in enumerate(layer_ids) if i % nproc == w]
+        data = [(shapes[li], wl.resnet50_layer(shapes[li], batch, rank_seed(0, li)))
+                for li in mine]
+        out = []
+        for s in range(steps):
+            barrier.wait(timeout=900)
+            t0 = time.time()
+            ops = 0
+            for sh, L in data:
+                orc.linear_backward(L.dH, L.X, L.W, KIND, BITS, BLOCK, s)
+                ops += 4 * sh.rows(batch) * sh.cout * sh.D
+            out.append((t0, time.time(), ops))
+        queue.put((w, out, None))
+    except Exception as exc:  # reported by the parent
+        queue.put((w, None, repr(exc)[:300]))
 
 
-def cpu_baseline(rows: int):
-    from paper_2010_14298_gb300 import workloads as wl
+def oracle_sweep(batch: int, steps: int, nproc: int, layer_ids=None):
+    """[(seconds, ops)] per step of the oracle's full hot path over the
+    sweep's layers at `batch`, on `nproc` processes."""
+    import multiprocessing as mp
     import oracle
-    oracle.build()
-    L = wl.config(CONFIG_INDEX, batch=max(1, rows // 1024))[0]
-    rows = L.N
-    t = time.perf_counter()
-    ops = _oracle_step(L, rows, 0)
-    dt = time.perf_counter() - t
-    return {"value": ops / dt / 1e12, "unit": "TOPS", "cores": 1, "kind": "oracle",
-            "sample": f"{rows} im2col rows (batch {rows // 1024}) of the workload, "
-                      f"full hot path, {dt:.1f} s single-threaded"}
-
-
-def oracle_overhead_shape():
-    """The oracle's gradient quantizers (range, scales / transform, SR, sums;
-    Q_b2 only) on the paper's overhead shape, dH 401408 x 64, one core."""
-    import oracle as orc
     from paper_2010_14298_gb300 import workloads as wl
-    orc.build()
-    dH = wl.random_grad(wl.rng(480), 128 * 56 * 56, 64, sigma=2.0, outlier_frac=0.01)
-    out = {}
-    for name, kind, bits, block in (("PTQ-8", orc.PTQ, 8, 0), ("PSQ-8", orc.PSQ, 8, 0),
-                                    ("BHQ-5 block 16", orc.BHQ, 5, 16)):
-        t = time.perf_counter()
-        orc.quantize_grad(dH, kind, bits, block, 0, orc.STREAM_B2)
-        out[name] = (time.perf_counter() - t) * 1e3
-    return out
+    oracle.build()
+    if layer_ids is None:
+        layer_ids = list(range(len(wl.resnet50_shapes())))
+    nproc = max(1, min(nproc, len(layer_ids)))
+    ctx = mp.get_context("spawn")
+    barrier = ctx.Barrier(nproc)
+    queue = ctx.Queue()
+    procs = [ctx.Process(target=_oracle_worker,
+                         args=(w, nproc, batch, steps, layer_ids, barrier, queue), daemon=True)
+             for w in range(nproc)]
+    for p in procs:
+        p.start()
+    res = {}
+    try:
+        for _ in range(nproc):
+            w, out, err = queue.get(timeout=1800)
+            if err is not None:
+                raise RuntimeError(f"oracle worker {w}: {err}")
+            res[w] = out
+    finally:
+        for p in procs:
+            p.join(timeout=30)
+            if p.is_alive():
+                p.terminate()
+    return [(max(res[w][s][1] for w in res) - min(res[w][s][0] for w in res),
+             sum(res[w][s][2] for w in res)) for s in range(steps)]
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(batch: int):
+    cores = host_cores()
+    par = oracle_sweep(batch, 1, cores)
+    one = oracle_sweep(1, 1, 1)
+    (dt, ops), (dt1, ops1) = par[0], one[0]
+    return {"value": ops / dt / 1e12, "unit": "TOPS", "cores": cores, "kind": "oracle",
+            "sample": f"every layer of the sweep at batch {batch} (instead of 256), full hot "
+                      f"path, {cores} processes of the single-threaded oracle (layers dealt "
+                      f"round robin): {dt:.1f} s wall for {ops / 1e9:.1f} GOP",
+            "single_thread": {"value": ops1 / dt1 / 1e12, "unit": "TOPS", "cores": 1,
+                              "sample": f"every layer at batch 1, one process: {dt1:.1f} s"}}
 
 
 def run_reference(args):
@@ -863,27 +804,26 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2010_14298_gb300 import workloads as wl
-    import oracle
-    oracle.build()
-    L = wl.config(CONFIG_INDEX, batch=max(1, args.ref_rows // 1024))[0]
-    rows = L.N
-    for i in range(args.warmup):
-        _oracle_step(L, min(rows, 1024), i)
-    t = time.perf_counter()
-    ops = 0
-    for i in range(args.steps):
-        ops += _oracle_step(L, rows, 100 + i)
-    dt = time.perf_counter() - t
+    cores = host_cores()
+    nl = len(wl.resnet50_shapes())
+    # each step: the whole sweep at batch 1 (about 0.5 s on 16 cores); long
+    # runs take every m-th layer per step so that the run stays in minutes
+    m = max(1, -(-args.steps // 200))
+    ids = list(range(0, nl, m))
+    res = oracle_sweep(1, args.warmup + args.steps, cores, ids)[args.warmup:]
+    dt = sum(r[0] for r in res)
+    ops = sum(r[1] for r in res)
     value = ops / dt / 1e12
+    sample = (f"{len(ids)} of the sweep's {nl} layers at batch 1 per step, full hot path, "
+              f"{cores} processes of the single-threaded oracle")
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS",
            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
-           "scaling": "weak", "vs_baseline": None, "dtype": "f64 oracle (f32 codes)",
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64 oracle (u8 codes)",
            "data": "synthetic (seeded)",
-           "config": {"workload": WORKLOAD, "sample_rows": rows},
-           "cpu_baseline": {"value": value, "unit": "TOPS", "cores": 1,
-                            "kind": "oracle",
-                            "sample": f"{rows} im2col rows per step, full hot path"},
+           "config": {"workload": WORKLOAD, "sample": sample},
+           "cpu_baseline": {"value": value, "unit": "TOPS", "cores": cores, "kind": "oracle",
+                            "sample": sample},
            "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out), flush=True)
@@ -892,32 +832,18 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
-    ap.add_argument("--e2e-steps", type=int, default=20)
-    ap.add_argument("--e2e-copy-streams", type=int, default=1,
-                    help="streams per copy direction in the end-to-end pipeline")
-    ap.add_argument("--cpu-rows", type=int, default=65536,
-                    help="rows of the CPU-baseline sample (about 10 s of oracle work)")
-    ap.add_argument("--ref-rows", type=int, default=8192,
-                    help="rows per reference-arm step")
+    ap.add_argument("--e2e-steps", type=int, default=3,
+                    help="timed end-to-end steps through the C ABI with host buffers (0: skip)")
+    ap.add_argument("--cpu-batch", type=int, default=4,
+                    help="batch of the CPU-baseline sample (every layer of the sweep)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--forward-steps", type=int, default=50,
-                    help="timed calls of the quantized forward GEMM (0: skip)")
-    ap.add_argument("--adaptive-steps", type=int, default=50,
-                    help="timed steps of the adaptive BHQ groups (0: skip)")
-    ap.add_argument("--shift-steps", type=int, default=50,
-                    help="timed steps of the shift quantizer path (0: skip)")
-    ap.add_argument("--implicit-steps", type=int, default=50,
-                    help="timed steps with the implicit im2col X operand (0: skip)")
-    ap.add_argument("--sweep-steps", type=int, default=5,
-                    help="timed rounds per layer of the ResNet-50 sweep (0: skip)")
-    ap.add_argument("--config-steps", type=int, default=20,
-                    help="timed steps of the other full-size workloads and of the paper's "
-                         "overhead shape (0: skip)")
-    ap.add_argument("--eager", action="store_true",
-                    help="time the C-ABI calls directly instead of graph replays")
+    ap.add_argument("--no-extras", dest="extras", action="store_false",
+                    help="skip the other workloads and the variants")
+    ap.add_argument("--extra-steps", type=int, default=10,
+                    help="timed rounds per call of the other workloads")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "native":
         args.warmup = 3

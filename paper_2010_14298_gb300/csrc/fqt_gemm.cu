@@ -1734,6 +1734,15 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   // the next tile of each epilogue set is ready when it finishes the last;
   // otherwise two, and the other half of tensor memory holds running sums
   g.nacc = (!partial && exact_chunk_blocks(a_bits, b_bits) >= (K + BK - 1) / BK) ? 4 : 2;
+  // Several exact chunks per tile (two accumulators): one epilogue set per
+  // accumulator, so that each accumulator's chunks are drained by one set in
+  // order.  An mbarrier parity wait cannot tell a phase from the one two
+  // phases later; with three sets, the set of tile L + 2 could start waiting
+  // on accumulator L mod 2 while tile L's chunks still pass through it (the
+  // parameter ring holds that set back only until tile L - 4 is done).  With
+  // one chunk per tile, tile L's parameters wait for tile L - 4 (the same
+  // accumulator of four) to be drained, which is enough.
+  if (!partial && g.nacc == 2) g.sets = 2;
   g.m_fast = partial ? 0 : 1;
   g.M = M;
   g.N = N;

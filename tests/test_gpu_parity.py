@@ -889,6 +889,24 @@ def test_resnet50_full_batch_layer_sampled(name):
     _sampled_check(L, orc.BHQ, 5, 16, seed=3)
 
 
+@pytest.mark.parametrize("kind,bits", [(orc.PTQ, 8), (orc.PSQ, 8), (orc.BHQ, 8)])
+def test_grad_x_several_chunks_and_tiles_per_cta(kind, bits):
+    """grad_X with two exact chunks per tile (8-bit codes, C = 2048) and at
+    least three tiles per CTA (480 tiles): the accumulators are reused by
+    later tiles while earlier tiles' chunks drain."""
+    g = wl.rng(2048)
+    n, c, d = 7680, 2048, 1024
+    dH = wl.random_grad(g, n, c, sigma=1.5)
+    X = g.standard_normal((n, d)).astype(np.float32)
+    W = (0.02 * g.standard_normal((c, d))).astype(np.float32)
+    L = wl.Layer("chunks", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, kind, bits, 16 if kind == orc.BHQ else 0, seed=4)
+    h2, hw = q2.to_numpy(), qw.to_numpy()
+    rows = np.sort(wl.rng(7).choice(n, 160, replace=False))
+    ref_x = oracle_rows_grad_x(h2, hw, h2["codes"], rows)
+    assert grad_rel_err(gx[rows], ref_x) <= GRAD_TOL
+
+
 def test_bhq_code_agreement_pooled():
     """The >= 99.99% BHQ code agreement over every case this module compared
     (cases below AGREE_MIN codes cannot show a 1e-4 rate on their own)."""

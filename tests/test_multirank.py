@@ -34,8 +34,9 @@ def _worker(rank, world, port, q):
     w, r, _ = bench._dist()
     dist.barrier()
     slowest = bench.max_over_ranks(1.0 + 2.0 * r, torch.device("cpu"))
-    L = wl.config(bench.CONFIG_INDEX, batch=1, seed=bench.rank_seed(r))[0]
-    q.put((r, w, slowest, bench.rank_seed(r), float(L.dH[:4, :4].sum())))
+    sh = wl.resnet50_shapes()[5]
+    L = wl.resnet50_layer(sh, 1, bench.rank_seed(r, 5))
+    q.put((r, w, slowest, bench.rank_seed(r, 5), float(L.dH[:4, :4].sum())))
     dist.barrier()
     dist.destroy_process_group()
 
@@ -61,8 +62,7 @@ def test_two_ranks_take_the_slowest_time_and_distinct_batches():
 def test_reference_arm_under_torchrun_prints_once():
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
            "--master-addr", "127.0.0.1", "--master-port", str(_free_port()), "bench.py",
-           "--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "0",
-           "--ref-rows", "1024"]
+           "--impl", "reference", "--gpus", "2", "--steps", "1", "--warmup", "0"]
     r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
@@ -70,3 +70,4 @@ def test_reference_arm_under_torchrun_prints_once():
     rec = json.loads(lines[0])
     assert rec["impl"] == "reference" and rec["n_gpus"] == 2 and rec["value"] > 0
     assert rec["e2e"]["h2d_bytes_per_step"] == 0
+    assert rec["cpu_baseline"]["cores"] >= 1 and rec["cpu_baseline"]["kind"] == "oracle"
