@@ -162,7 +162,9 @@ size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
   size_t need = gemm_workspace_bytes(N, C, D);
   const size_t grp = group_workspace_bytes(N);         // adaptive BHQ grouping
   const size_t list = group_list_bytes(N);               // its grad_X work lists
+  const size_t bhq = bhq_pass_bytes(N, C);                // two-pass BHQ scratch
   if (grp > need) need = grp;
+  if (bhq > need) need = bhq;
   if (list > need) need = list;
   return kGemmOffset + need;
 }
@@ -226,8 +228,13 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
     return FQT_EINVAL;
   if (adapt && (C != 64 && C != 128 && C != 256)) return FQT_EUNSUPPORTED;
   if (adapt && N > ((int64_t)1 << 20)) return FQT_EUNSUPPORTED;
+  // fixed BHQ blocks of supported shapes: the two-pass quantizer, whose
+  // statistics pass also takes the range (no separate range pass)
+  const bool two_pass = kind == FQT_BHQ && !adapt &&
+                        bhq_pass_supported((int)C, block, dtype == FQT_BF16);
   fqt_status s = check_ws(workspace, ws_bytes,
-                          kGemmOffset + (adapt ? group_workspace_bytes(N) : 0));
+                          kGemmOffset + (adapt ? group_workspace_bytes(N)
+                                         : two_pass ? bhq_pass_bytes(N, C) : 0));
   if (s != FQT_OK) return s;
   q_b2->rows = N;
   q_b2->cols = C;
@@ -250,9 +257,12 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   int32_t *csum = q_b1 ? q_b1->col_sum : (adapt ? nullptr : q_b2->col_sum);
   // the column sums the quantizer accumulates into are cleared by the range pass
   int32_t *csum2 = kind == FQT_SHIFT ? q_b2->shift_col_sum : nullptr;
-  cudaError_t e = launch_range(dH, dtype == FQT_BF16, N * C, part, &npart, csum,
-                               csum ? C : 0, csum2, csum2 ? C : 0, nsm, st);
-  if (e != cudaSuccess) return cuda_fail(e, "range pass");
+  cudaError_t e = cudaSuccess;
+  if (!two_pass) {
+    e = launch_range(dH, dtype == FQT_BF16, N * C, part, &npart, csum, csum ? C : 0, csum2,
+                     csum2 ? C : 0, nsm, st);
+    if (e != cudaSuccess) return cuda_fail(e, "range pass");
+  }
   QuantArgs a;
   memset(&a, 0, sizeof(a));
   a.h = dH;
@@ -312,16 +322,13 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
     }
     return launch_bhq_groups(ag, bf16, nsm, st);
   }
-  if (kind == FQT_BHQ) {
-    // one warp per block when the block fits a warp's registers; the warp
-    // kernel also writes the grad_X offsets
+  if (two_pass) {
     QuantArgs aw = a;
     if (want_off) {
       aw.hz = q_b2->hz;
       aw.hr = q_b2->hr;
     }
-    s = launch_bhq_warp(aw, bf16, nsm, st);
-    if (s != FQT_EUNSUPPORTED) return s;
+    return launch_bhq_passes(aw, bf16, nsm, w + kGemmOffset, part, st);
   }
   {
     QuantArgs a2 = a;  // staged kernel for rows of up to 1024 columns

@@ -467,7 +467,7 @@ __global__ void __launch_bounds__(256) k_grp_layout(const int32_t *__restrict__ 
 // (LPR lanes per row, 8 columns per lane).  Pass 1 reads the rows for the
 // lead row's range, lambda2 and the column sums of the small rows; pass 2
 // re-reads them (L2) for the transform, the row minima, SR and packing; the
-// grad_X offsets hz, hr are reflected at the end (see k_bhq_warp).
+// grad_X offsets hz, hr are reflected at the end (see k_bhq_team).
 // ---------------------------------------------------------------------------
 template <int LPR>
 __device__ __forceinline__ float2 row_minmax(float2 v) {

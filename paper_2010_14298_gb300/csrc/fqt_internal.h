@@ -66,7 +66,10 @@ fqt_status launch_fwd_codes(const void *X, bool bf16, int64_t rows, int cols, in
                             int32_t *code_zero_out = nullptr);
 fqt_status launch_conv_colsum(const uint16_t *f16, int64_t n, int h, int w, int c, int kh,
                               int kw, int pad, int bits, int32_t *col_sum, cudaStream_t st);
-fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
+bool bhq_pass_supported(int C, int block, bool bf16);
+size_t bhq_pass_bytes(int64_t N, int64_t C);
+fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch,
+                             float2 *part, cudaStream_t st);
 fqt_status launch_shift(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
                                const int32_t *lead, float *hz, float *hr, int64_t N,

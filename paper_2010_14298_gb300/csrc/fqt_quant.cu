@@ -879,13 +879,26 @@ __global__ void __launch_bounds__(kQ2Threads) k_quant2(const QuantArgs a) {
 }
 
 // ---------------------------------------------------------------------------
-// BHQ gradient quantizer, one warp per block of nb rows (Sec. 4.2, App. D.4)
-// fused with Q_b1 (App. E), for rows of C = 8 LPR columns, LPR in {8, 16,
-// 32}: lane l owns oct l % LPR of row l / LPR of each of the STEPS row groups
-// of the block (nb = (32 / LPR) STEPS).  The block stays in registers and
-// every reduction is a shuffle inside the warp, so the warps of an SM run
-// their blocks independently, without CTA barriers.  The grad_X offsets hz,
-// hr of the block (see k_bhq_offsets) are formed in the same pass.
+// BHQ gradient quantizer for fixed blocks (Sec. 4.2, App. D.4) fused with
+// Q_b1 (App. E), in two passes over dH.  The statistics pass holds each
+// block in registers: a team of TEAM warps per block of nb rows, each warp
+// owning a slab of 8 LPR columns (TEAM > 1 only with LPR = 32, slabs of 256
+// columns), lane l owning oct l % LPR of the slab in row l / LPR of each of
+// the STEPS row groups (nb = (32 / LPR) STEPS); row reductions are shuffles
+// inside a warp and one shared-memory exchange at a named barrier of the
+// team.  Its per-entry work is light (statistics, column sums, row minima),
+// so the unrolled block fits the instruction cache.  The code pass streams
+// the rows with rolled loops (rounding, packing, sums need no block-wide
+// exchange once z'_k and w_j are known); k_bhq_offsets then reflects the
+// grad_X offsets hz, hr of each block.
+//
+// Stochastic rounding runs on the fp32 pipe: with U = 128 + u 2^-16 (u the
+// 16-bit uniform, exact in fp32), floor(v + u 2^-16) = floor(rd(v + U)) - 128
+// because rounding down never crosses an integer, and a second round-down
+// addition of 2^23 + 0x6400 - 128 leaves 0x4B006400 + code in the bits:
+// code = floor(v + u 2^-16) = (floor(v 2^16) + u) >> 16, the rule of sr_code16
+// (R1) for v in [0, B].  Byte 0 of those bits is the code and byte 1 is 0x64,
+// so one byte permutation packs two fp16 carriers 1024 + code.
 // ---------------------------------------------------------------------------
 template <int FROM, class V, class Op>
 __device__ __forceinline__ V xor_reduce(V v, Op op) {
@@ -902,70 +915,110 @@ __device__ __forceinline__ V row_reduce(V v, Op op) {
   return v;
 }
 
-template <typename T, int LPR, int STEPS>
-__global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
+constexpr float kSrMagic = 8414080.0f;     // 2^23 + 0x6400 - 128
+constexpr uint32_t kSrBits = 0x4B006400u;  // bits of 2^23 + 0x6400
+
+// 128 + u 2^-16 for the low and the high 16-bit uniform of a Philox word
+__device__ __forceinline__ float sr_u_lo(uint32_t w) {
+  return __uint_as_float(0x43000000u | (w & 0xFFFFu));
+}
+__device__ __forceinline__ float sr_u_hi(uint32_t w) {
+  return __uint_as_float(__byte_perm(w, 0x43000000u, 0x7632));
+}
+// uniform j (0..7) of an oct: half (j mod 2) of word j / 2
+__device__ __forceinline__ float sr_u(const uint4 &w, int j) {
+  const uint32_t word = (j >> 1) == 0 ? w.x : (j >> 1) == 1 ? w.y : (j >> 1) == 2 ? w.z : w.w;
+  return (j & 1) ? sr_u_hi(word) : sr_u_lo(word);
+}
+
+// kSrBits + code, code = SR(v) for v in [0, B] (v already clamped)
+__device__ __forceinline__ uint32_t sr_bits(float v, float U) {
+  return __float_as_uint(__fadd_rd(__fadd_rd(v, U), kSrMagic));
+}
+
+// Eight codes (kSrBits + code) as centred fp16 carriers code - off.
+__device__ __forceinline__ void store_carriers_bits(uint16_t *dst, const uint32_t (&b)[8],
+                                                    __half2 bias) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t h = __byte_perm(b[2 * i], b[2 * i + 1], 0x5410);
+    __half2 v = __hsub2(*reinterpret_cast<const __half2 *>(&h), bias);
+    w[i] = *reinterpret_cast<uint32_t *>(&v);
+  }
+  *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Eight codes (kSrBits + code) as bytes.
+__device__ __forceinline__ void store_codes_bits(uint8_t *dst, const uint32_t (&b)[8]) {
+  uint2 v;
+  v.x = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+  v.y = __byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410);
+  *reinterpret_cast<uint2 *>(dst) = v;
+}
+
+// Named barrier of one team of TEAM warps (ids 1..8; 0 is __syncthreads).
+template <int TEAM>
+__device__ __forceinline__ void team_sync(int team) {
+  if constexpr (TEAM > 1)
+    asm volatile("bar.sync %0, %1;" ::"r"(1 + team), "n"(32 * TEAM) : "memory");
+}
+
+constexpr int kTeamRows = 16;  // rows of a block when TEAM > 1 (LPR = 32, STEPS <= 16)
+
+// Per-block results of the statistics pass, read by the code pass: lead row
+// p (as an integer bit pattern), s1, s2 and rho = 1/sqrt(nb) (0 for a block
+// of one row or of zeros), followed in the workspace by w_j for every block.
+struct BhqBlock {
+  float p, s1, s2, rho;
+};
+
+// Workspace bytes of the two-pass BHQ quantizer for blocks of at least 4
+// rows: the per-block record and the C column sums w of every block.
+size_t bhq_pass_bytes(int64_t N, int64_t C) {
+  const int64_t nblk = (N + 3) / 4;
+  return (size_t)nblk * sizeof(BhqBlock) + (size_t)nblk * (size_t)C * sizeof(float) + 512;
+}
+
+// ---------------------------------------------------------------------------
+// Statistics pass of BHQ (the first of the two passes over dH): for every
+// block its row statistics, lead row, lambda1, lambda2, s1, s2 (App. D.4),
+// the reflection's column sums w_j = sum_k e_k s_k h_kj and the row minima
+// z'_k of T = Q diag(s) H (Sec. 4.2), plus the per-CTA (min, max) and
+// non-finite flag of the whole tensor (the range of Q_b1) and the clearing of
+// the column sums the code pass accumulates into.
+// ---------------------------------------------------------------------------
+template <typename T, int LPR, int STEPS, int TEAM>
+__global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
+    k_bhq_stats(const QuantArgs a, BhqBlock *__restrict__ bst, float *__restrict__ wsum,
+                float2 *__restrict__ part) {
+  static_assert(TEAM == 1 || (LPR == 32 && STEPS <= kTeamRows), "team layout");
+  constexpr int RS = 32 / LPR, SLAB = 8 * LPR, C = SLAB * TEAM;
+  constexpr int TPC = 8 / TEAM;  // teams per CTA
+  constexpr int XW = TEAM > 1 ? 8 : 1;
+  __shared__ float2 xs_mm[XW][kTeamRows];
+  __shared__ float xs_tm[XW][kTeamRows];
   __shared__ float2 red[8];
   __shared__ int redi[8];
-  extern __shared__ int csum_s[];  // C column sums of the grad_W code set
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int CO = LPR, RS = 32 / LPR, C = 8 * LPR;
+  const int team = warp / TEAM, wi = warp - team * TEAM;
   const int nb = a.block;
   const int sub = lane / LPR, o = lane - sub * LPR;
-
-  // ---- global range (Q_b1 scale) from the range-pass partials ----
-  float gmin = INFINITY, gmax = -INFINITY;
-  int bad = 0;
-  for (int i = tid; i < a.npart; i += blockDim.x) {
-    const float2 p = a.part[i];
-    bad |= isnan(p.x);
-    gmin = fminf(gmin, p.x);
-    gmax = fmaxf(gmax, p.y);
+  const int col0 = (wi * LPR + o) * 8;
+  const float fB2 = (float)((1u << a.bits) - 1u);
+  // the code pass accumulates column sums into these
+  {
+    const int64_t g = (int64_t)blockIdx.x * blockDim.x + tid;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = g; i < C; i += stride) {
+      if (a.csum1) a.csum1[i] = 0;
+      if (a.csum2) a.csum2[i] = 0;
+    }
   }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
-    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
-    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
-  }
-  if (lane == 0) {
-    red[warp] = make_float2(gmin, gmax);
-    redi[warp] = bad;
-  }
-  for (int i = tid; i < C; i += blockDim.x) csum_s[i] = 0;
-  __syncthreads();
-  gmin = red[0].x;
-  gmax = red[0].y;
-  bad = redi[0];
-  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
-    gmin = fminf(gmin, red[w].x);
-    gmax = fmaxf(gmax, red[w].y);
-    bad |= redi[w];
-  }
-  if (bad) {
-    if (blockIdx.x == 0 && tid == 0) record_status(a.status, FQT_ENONFINITE);
-    return;
-  }
-  const uint32_t B2 = (1u << a.bits) - 1u;
-  const float s_g1 = affine_scale(gmin, gmax, 255u);
-  const float s_g1_16 = __fmul_rn(s_g1, 65536.0f);
-  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
-  if (blockIdx.x == 0 && tid == 0 && has_b1) {
-    a.inv1[0] = __fdiv_rn(1.0f, s_g1);
-    a.zero1[0] = __fmul_rn(s_g1, gmin);
-  }
-  int32_t *const csum_g = has_b1 ? a.csum1 : a.csum2;
-  PhiloxKeys key;
-#pragma unroll
-  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
-  const bool want_off = a.hz != nullptr;
-  int cs[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) cs[j] = 0;
-
+  float gmn = INFINITY, gmx = -INFINITY, nanacc = 0.0f;
   const int64_t nblocks = (a.N + nb - 1) / nb;
-  const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t blk = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; blk < nblocks;
-       blk += wstride) {
+  const int64_t tstride = (int64_t)gridDim.x * TPC;
+  for (int64_t blk = (int64_t)blockIdx.x * TPC + team; blk < nblocks; blk += tstride) {
     const int64_t r0 = blk * nb;
     const int nrows = (int)min((int64_t)nb, a.N - r0);
     float x[STEPS][8];
@@ -975,13 +1028,13 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
       const int k = sub + RS * s;
       rv[s] = k < nrows;
       if (rv[s]) {
-        load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + o * 8, x[s]);
+        load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + col0, x[s]);
       } else {
 #pragma unroll
         for (int j = 0; j < 8; ++j) x[s][j] = 0.0f;
       }
     }
-    // ---- row statistics ----
+    // ---- row statistics (and a NaN that any non-finite entry leaves) ----
     float rmin[STEPS], rmax[STEPS];
 #pragma unroll
     for (int s = 0; s < STEPS; ++s) {
@@ -990,11 +1043,35 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
       for (int j = 0; j < 8; ++j) {
         mm.x = fminf(mm.x, x[s][j]);
         mm.y = fmaxf(mm.y, x[s][j]);
+        nanacc = fmaf(x[s][j], 0.0f, nanacc);
       }
       mm = row_reduce<LPR>(mm, OpMinMax());
       rmin[s] = mm.x;
       rmax[s] = mm.y;
     }
+    if constexpr (TEAM > 1) {
+      if (lane == 0) {
+#pragma unroll
+        for (int s = 0; s < STEPS; ++s) xs_mm[warp][s] = make_float2(rmin[s], rmax[s]);
+      }
+      team_sync<TEAM>(team);
+      float2 mine = make_float2(INFINITY, -INFINITY);
+      if (lane < STEPS) {
+#pragma unroll
+        for (int w2 = 0; w2 < TEAM; ++w2) mine = OpMinMax()(mine, xs_mm[team * TEAM + w2][lane]);
+      }
+#pragma unroll
+      for (int s = 0; s < STEPS; ++s) {
+        rmin[s] = __shfl_sync(0xffffffffu, mine.x, s);
+        rmax[s] = __shfl_sync(0xffffffffu, mine.y, s);
+      }
+    }
+#pragma unroll
+    for (int s = 0; s < STEPS; ++s)
+      if (rv[s]) {
+        gmn = fminf(gmn, rmin[s]);
+        gmx = fmaxf(gmx, rmax[s]);
+      }
     // ---- lead row (largest ||h_k||_inf, lowest index on ties), lambda2 ----
     float bestv = -1.0f;
     int bestk = 0x7fffffff;
@@ -1046,10 +1123,10 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
         const float c1 = cbrtf(lam1), c2 = cbrtf(lam2);
         const float n3 = cbrtf(Nf), n6 = sqrtf(n3);
         const float den = c1 * c1 / n3 + c2 * c2 * n3 * n3;
-        s1f = (float)B2 * n6 / (c1 * den);
-        s2f = (float)B2 * n6 / (c2 * den);
+        s1f = fB2 * n6 / (c1 * den);
+        s2f = fB2 * n6 / (c2 * den);
       } else {
-        s1f = (float)B2 * sqrtf(Nf) / lam1;
+        s1f = fB2 * sqrtf(Nf) / lam1;
       }
       if (nrows > 1) {
         rho = 1.0f / sqrtf(Nf);
@@ -1063,184 +1140,353 @@ __global__ void __launch_bounds__(256, 2) k_bhq_warp(const QuantArgs a) {
 #pragma unroll
     for (int s = 0; s < STEPS; ++s) {
       const bool lead = (sub + RS * s) == p;
-      const float e = kap * (lead ? rho - 1.0f : rho);
-      const float sk = lead ? s1f : s2f;
+      const float esk = __fmul_rn(kap * (lead ? rho - 1.0f : rho), lead ? s1f : s2f);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) w[j] = fmaf(e, __fmul_rn(sk, x[s][j]), w[j]);
+      for (int j = 0; j < 8; ++j) w[j] = fmaf(esk, x[s][j], w[j]);
     }
 #pragma unroll
     for (int j = 0; j < 8; ++j) w[j] = xor_reduce<LPR>(w[j], OpAddF());
-    // ---- per row: transform, row minimum, rounding, packing, sums ----
-    ff sd = {0.0f, 0.0f};
-    int sR = 0;
-    float dv[STEPS];
-    int Rv[STEPS];
+    // ---- row minima of T; the code pass recomputes each t_kj with this
+    // same sequence of roundings, so z'_k is exactly its row minimum ----
+    float tmin[STEPS];
 #pragma unroll
     for (int s = 0; s < STEPS; ++s) {
-      const int k = sub + RS * s;
-      const int64_t row = r0 + k;
-      const bool lead = k == p;
+      const bool lead = (sub + RS * s) == p;
       const float sk = lead ? s1f : s2f;
       const float ck = lead ? rho - 1.0f : rho;
-      float t[8];
-      float tmin = INFINITY;
+      float tm = INFINITY;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        t[j] = fmaf(-ck, w[j], __fmul_rn(sk, x[s][j]));
-        tmin = fminf(tmin, t[j]);
+      for (int j = 0; j < 8; ++j) tm = fminf(tm, fmaf(-ck, w[j], __fmul_rn(sk, x[s][j])));
+      tmin[s] = row_reduce<LPR>(tm, OpMin());
+    }
+    if constexpr (TEAM > 1) {
+      if (lane == 0) {
+#pragma unroll
+        for (int s = 0; s < STEPS; ++s) xs_tm[warp][s] = tmin[s];
       }
-      const float z2 = row_reduce<LPR>(tmin, OpMin());
-      const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)o;
-      uint32_t c[8];
-      int rs2 = 0, rs1 = 0;
-      if (rv[s]) {
-        const uint4 w2 = philox_oct(q, 0u, key);
+      team_sync<TEAM>(team);
+      float mine = INFINITY;
+      if (lane < STEPS) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          c[j] = sr_code16(__fmul_rn(__fsub_rn(t[j], z2), 65536.0f), u16_of(w2, j), B2);
-          rs2 += (int)c[j];
-        }
-        if (a.c2) store_codes8(a.c2 + row * (int64_t)C + o * 8, c);
-        if (a.f2) store_carriers8(a.f2 + row * (int64_t)C + o * 8, c, (B2 + 1u) >> 1);
-        if (has_b1) {
-          const uint4 w1 = philox_oct(q, 1u, key);
+        for (int w2 = 0; w2 < TEAM; ++w2) mine = fminf(mine, xs_tm[team * TEAM + w2][lane]);
+      }
+#pragma unroll
+      for (int s = 0; s < STEPS; ++s) tmin[s] = __shfl_sync(0xffffffffu, mine, s);
+    }
+    // ---- outputs ----
+    if (sub == 0) {
+      float *wd = wsum + blk * (int64_t)C + col0;
+      *reinterpret_cast<float4 *>(wd) = make_float4(w[0], w[1], w[2], w[3]);
+      *reinterpret_cast<float4 *>(wd + 4) = make_float4(w[4], w[5], w[6], w[7]);
+    }
+    if (wi == 0 && o == 0) {
+#pragma unroll
+      for (int s = 0; s < STEPS; ++s) {
+        const int k = sub + RS * s;
+        if (!rv[s]) continue;
+        const float sk = k == p ? s1f : s2f;
+        a.inv2[r0 + k] = sk > 0.0f ? __fdiv_rn(1.0f, sk) : 0.0f;
+        a.zero2[r0 + k] = tmin[s];
+      }
+      if (sub == 0) {
+        bst[blk] = BhqBlock{__int_as_float(p), s1f, s2f, rho};
+        a.lead2[blk] = p;
+      }
+    }
+  }
+  // ---- range partials of the CTA (NaN marks a non-finite input) ----
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmn = fminf(gmn, __shfl_xor_sync(0xffffffffu, gmn, off));
+    gmx = fmaxf(gmx, __shfl_xor_sync(0xffffffffu, gmx, off));
+    nanacc += __shfl_xor_sync(0xffffffffu, nanacc, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmn, gmx);
+    redi[warp] = isnan(nanacc) ? 1 : 0;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int bad = 0;
+    for (int i = 0; i < (int)(blockDim.x >> 5); ++i) {
+      gmn = fminf(gmn, red[i].x);
+      gmx = fmaxf(gmx, red[i].y);
+      bad |= redi[i];
+    }
+    part[blockIdx.x] = bad ? make_float2(NAN, NAN) : make_float2(gmn, gmx);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Code pass of BHQ (the second pass over dH), fused with Q_b1 (App. E): per
+// entry t = s_k h_kj - c_k w_j (c_k = rho - 1 on the lead row, rho
+// elsewhere) as the statistics pass computed it, v = t - z'_k, stochastic
+// rounding of v (Q_b2) and of s (h - min H) (Q_b1), fp16 carriers (and
+// optional bytes), row sums of Q_b2 and column sums of the grad_W code set.
+// A warp takes chunks of kCodeRows rows; it walks the row's slabs of 8 LPR
+// columns one after another and, inside a slab, the chunk's rows 32 / LPR at
+// a time (lane: 8 columns of one row), so the loops stay rolled and rows
+// need no exchange between warps.
+// ---------------------------------------------------------------------------
+constexpr int kCodeRows = 32;
+
+template <typename T, int LPR>
+__global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
+                                                   const BhqBlock *__restrict__ bst,
+                                                   const float *__restrict__ wsum) {
+  constexpr int RS = 32 / LPR, SLAB = 8 * LPR;
+  __shared__ float2 red[8];
+  __shared__ int redi[8];
+  __shared__ int rs_s[8][2][kCodeRows];
+  extern __shared__ int csum_s[];  // C column sums of the grad_W code set
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int C = a.C, CO = C / 8, nb = a.block;
+  const int sub = lane / LPR, o = lane - sub * LPR;
+
+  // ---- global range (Q_b1 scale) from the statistics-pass partials ----
+  float gmin = INFINITY, gmax = -INFINITY;
+  int bad = 0;
+  for (int i = tid; i < a.npart; i += blockDim.x) {
+    const float2 p = a.part[i];
+    bad |= isnan(p.x);
+    gmin = fminf(gmin, p.x);
+    gmax = fmaxf(gmax, p.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    gmin = fminf(gmin, __shfl_xor_sync(0xffffffffu, gmin, off));
+    gmax = fmaxf(gmax, __shfl_xor_sync(0xffffffffu, gmax, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(gmin, gmax);
+    redi[warp] = bad;
+  }
+  for (int i = tid; i < C; i += blockDim.x) csum_s[i] = 0;
+  __syncthreads();
+  gmin = red[0].x;
+  gmax = red[0].y;
+  bad = redi[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w) {
+    gmin = fminf(gmin, red[w].x);
+    gmax = fmaxf(gmax, red[w].y);
+    bad |= redi[w];
+  }
+  if (bad) {
+    if (blockIdx.x == 0 && tid == 0) record_status(a.status, FQT_ENONFINITE);
+    return;
+  }
+  const uint32_t B2 = (1u << a.bits) - 1u;
+  const float fB2 = (float)B2;
+  const float s_g1 = affine_scale(gmin, gmax, 255u);
+  const bool has_b1 = a.c1 != nullptr || a.f1 != nullptr;
+  if (blockIdx.x == 0 && tid == 0 && has_b1) {
+    a.inv1[0] = __fdiv_rn(1.0f, s_g1);
+    a.zero1[0] = __fmul_rn(s_g1, gmin);
+  }
+  int32_t *const csum_g = has_b1 ? a.csum1 : a.csum2;
+  PhiloxKeys key;
+#pragma unroll
+  for (int i = 0; i < 20; ++i) key.k[i] = a.round_keys[i];
+  const __half2 bias2 = __half2half2(__int2half_rn(1024 + (int)((B2 + 1u) >> 1)));
+  const __half2 bias1 = __half2half2(__int2half_rn(1024 + 128));
+  const bool want_rs1 = has_b1 && a.rsum1 != nullptr;
+
+  const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;
+  const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t ch = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; ch < nchunks;
+       ch += wstride) {
+    const int64_t row0 = ch * kCodeRows;
+    const int rows = (int)min((int64_t)kCodeRows, a.N - row0);
+    rs_s[warp][0][lane] = 0;
+    rs_s[warp][1][lane] = 0;
+    __syncwarp();
+#pragma unroll 1
+    for (int c0 = 0; c0 < C; c0 += SLAB) {
+      const int col0 = c0 + o * 8;
+      uint32_t cs[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) cs[j] = 0u;
+      uint32_t cs_rows = 0;
+#pragma unroll 1
+      for (int rb = 0; rb < rows; rb += RS) {  // the same trip count in every lane
+        const int rr = rb + sub;
+        const bool valid = rr < rows;  // the LPR lanes of a row agree
+        uint32_t acc1 = 0u, acc2 = 0u;
+        if (valid) {
+          const int64_t row = row0 + rr;
+          const int64_t blk = row / nb;
+          const BhqBlock bs = bst[blk];
+          const bool lead = (int)(row - blk * nb) == __float_as_int(bs.p);
+          const float sk = lead ? bs.s1 : bs.s2;
+          const float ck = lead ? bs.rho - 1.0f : bs.rho;
+          const float zr = a.zero2[row];
+          float x[8], w[8];
+          load_oct(reinterpret_cast<const T *>(a.h) + row * C + col0, x);
+          load_oct(wsum + blk * (int64_t)C + col0, w);
+          const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)(col0 >> 3);
+          if (has_b1) {
+            const uint4 u1 = philox_oct(q, 1u, key);
+            uint32_t b[8];
+            acc1 = 0u - 8u * kSrBits;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float v = fminf(__fmul_rn(__fsub_rn(x[j], gmin), s_g1), 255.0f);
+              b[j] = sr_bits(v, sr_u(u1, j));
+              cs[j] += b[j];
+              acc1 += b[j];
+            }
+            ++cs_rows;
+            if (a.c1) store_codes_bits(a.c1 + row * (int64_t)C + col0, b);
+            if (a.f1) store_carriers_bits(a.f1 + row * (int64_t)C + col0, b, bias1);
+          }
+          const uint4 u2 = philox_oct(q, 0u, key);
+          uint32_t b[8];
+          acc2 = 0u - 8u * kSrBits;
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            const float v = __fmul_rn(__fsub_rn(x[s][j], gmin), s_g1_16);
-            c[j] = sr_code16(v, u16_of(w1, j), 255u);
-            rs1 += (int)c[j];
+            const float t = fmaf(-ck, w[j], __fmul_rn(sk, x[j]));
+            b[j] = sr_bits(fminf(__fsub_rn(t, zr), fB2), sr_u(u2, j));
+            acc2 += b[j];
+            if (!has_b1) cs[j] += b[j];
           }
-          if (a.c1) store_codes8(a.c1 + row * (int64_t)C + o * 8, c);
-          if (a.f1) store_carriers8(a.f1 + row * (int64_t)C + o * 8, c, 128u);
+          if (!has_b1) ++cs_rows;
+          if (a.c2) store_codes_bits(a.c2 + row * (int64_t)C + col0, b);
+          if (a.f2) store_carriers_bits(a.f2 + row * (int64_t)C + col0, b, bias2);
         }
+        if (want_rs1) {
+          const int r1 = row_reduce<LPR>((int)acc1, OpAdd());
+          if (o == 0 && valid) rs_s[warp][1][rr] += r1;
+        }
+        const int r2 = row_reduce<LPR>((int)acc2, OpAdd());
+        if (o == 0 && valid) rs_s[warp][0][rr] += r2;
+      }
+      // this slab's column sums: the lanes of one column add theirs
+      if (csum_g) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) cs[j] += (int)c[j];
-      }
-      rs2 = row_reduce<LPR>(rs2, OpAdd());
-      if (has_b1) rs1 = row_reduce<LPR>(rs1, OpAdd());
-      if (rv[s] && o == 0) {
-        if (a.rsum2) a.rsum2[row] = rs2;
-        if (has_b1 && a.rsum1) a.rsum1[row] = rs1;
-        a.inv2[row] = sk > 0.0f ? __fdiv_rn(1.0f, sk) : 0.0f;
-        a.zero2[row] = z2;
-      }
-      // the row's offset split 2^(b-1) + z' = m + d and R = sum_c (a + m);
-      // |z'| is a few times B sqrt(nb) here, so m and R fit int32 and m
-      // converts with the 1.5 2^23 FADD
-      const ff xo = two_sum((float)((B2 + 1u) >> 1), z2);
-      const float m = rintf(xo.h);
-      const ff d = fast_two_sum(__fsub_rn(xo.h, m), xo.l);
-      const int mi = (int)(__float_as_uint(__fadd_rn(m, 12582912.0f)) - 0x4B400000u);
-      const int R = rs2 - C * (int)((B2 + 1u) >> 1) + C * mi;
-      dv[s] = ff_round(d);
-      Rv[s] = R;
-      if (rv[s] && o == 0) {  // one lane per row adds the row's terms
-        sd = ff_add(sd, d);
-        sR += R;
+        for (int j = 0; j < 8; ++j) {
+          const int v = xor_reduce<LPR>((int)(cs[j] - cs_rows * kSrBits), OpAdd());
+          if (sub == 0 && v) atomicAdd(&csum_s[col0 + j], v);
+        }
       }
     }
-    if (want_off) {
-      // block sums of d (float-float) and R over the lanes that added them
-#pragma unroll
-      for (int off = LPR; off < 32; off <<= 1) {  // lanes o == 0 hold the rows' terms
-        const ff od = {__shfl_xor_sync(0xffffffffu, sd.h, off),
-                       __shfl_xor_sync(0xffffffffu, sd.l, off)};
-        sd = ff_add(sd, od);
-        sR += __shfl_xor_sync(0xffffffffu, sR, off);
-      }
-      float dp = 0.0f;
-      int Rp = 0;
-#pragma unroll
-      for (int s = 0; s < STEPS; ++s)
-        if (s == p / RS) {
-          dp = dv[s];
-          Rp = Rv[s];
-        }
-      dp = __shfl_sync(0xffffffffu, dp, (p % RS) * LPR);
-      Rp = __shfl_sync(0xffffffffu, Rp, (p % RS) * LPR);
-      if (nrows >= 2) {
-        const HhConst hcst = hh_const(nrows);
-        const ff rsd = ff_mul(hcst.rho, sd);
-        const ff rsR = ff_mul(hcst.rho, ff_from_i32s(sR));
-        const ff wd = ff_add(rsd, {-dp, 0.0f});
-        const ff wR = ff_add(rsR, ff_neg(ff_from_i32s(Rp)));
-#pragma unroll
-        for (int s = 0; s < STEPS; ++s) {
-          const int k = sub + RS * s;
-          if (!(rv[s] && o == 0)) continue;
-          float hzv, hrv;
-          if (k == p) {
-            hzv = ff_round(rsd);
-            hrv = ff_round(rsR);
-          } else {
-            hzv = ff_round(ff_add({dv[s], 0.0f}, ff_neg(ff_mul(hcst.kap, wd))));
-            hrv = ff_round(ff_add(ff_from_i32s(Rv[s]), ff_neg(ff_mul(hcst.kap, wR))));
-          }
-          a.hz[r0 + k] = hzv;
-          a.hr[r0 + k] = hrv;
-        }
-      } else {
-#pragma unroll
-        for (int s = 0; s < STEPS; ++s)
-          if (rv[s] && o == 0) {
-            a.hz[r0 + sub + RS * s] = dv[s];
-            a.hr[r0 + sub + RS * s] = ff_round(ff_from_i32s(Rv[s]));
-          }
-      }
+    __syncwarp();
+    if (lane < rows) {
+      if (a.rsum2) a.rsum2[row0 + lane] = rs_s[warp][0][lane];
+      if (want_rs1) a.rsum1[row0 + lane] = rs_s[warp][1][lane];
     }
-    if (o == 0 && sub == 0) a.lead2[blk] = p;
+    __syncwarp();
   }
-  // ---- column sums of the grad_W code set ----
   if (csum_g) {
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      int v = xor_reduce<LPR>(cs[j], OpAdd());
-      if (sub == 0 && v) atomicAdd(&csum_s[o * 8 + j], v);
-    }
     __syncthreads();
     for (int i = tid; i < C; i += blockDim.x)
       if (csum_s[i]) atomicAdd(&csum_g[i], csum_s[i]);
   }
 }
 
-// Launches k_bhq_warp when the shape fits it: BHQ with rows of 64, 128 or
-// 256 columns and blocks of (32 / LPR) STEPS rows, STEPS in {1, 2, 4, 8}.
-fqt_status launch_bhq_warp(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st) {
-  if (a.kind != KIND_BHQ || a.C % 8) return FQT_EUNSUPPORTED;
-  const int CO = a.C / 8;
-  if (CO != 8 && CO != 16 && CO != 32) return FQT_EUNSUPPORTED;
-  const int RS = 32 / CO;
-  if (a.block % RS) return FQT_EUNSUPPORTED;
-  const int steps = a.block / RS;
-  if (steps != 1 && steps != 2 && steps != 4 && steps != 8) return FQT_EUNSUPPORTED;
+template <typename T, int LPR, int STEPS, int TEAM>
+static cudaError_t launch_stats(const QuantArgs &a, BhqBlock *bst, float *wsum, float2 *part,
+                                int num_sms, int *grid_out, cudaStream_t st) {
+  auto kern = k_bhq_stats<T, LPR, STEPS, TEAM>;
+  int per_sm = 0;
+  const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, 0);
+  if (e != cudaSuccess) return e;
   const int64_t nblocks = (a.N + a.block - 1) / a.block;
-  int64_t grid = (nblocks + 7) / 8;
-  // persistent: the CTAs that fit at once (two per SM), each warp looping
-  const int64_t cap = (int64_t)num_sms * (steps >= 8 ? 1 : 2);
+  constexpr int TPC = 8 / TEAM;
+  int64_t grid = (nblocks + TPC - 1) / TPC;
+  int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);
+  if (cap > kMaxRangeCtas) cap = kMaxRangeCtas;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
+  *grid_out = (int)grid;
+  kern<<<(int)grid, 256, 0, st>>>(a, bst, wsum, part);
+  return cudaGetLastError();
+}
+
+template <typename T, int LPR>
+static cudaError_t launch_codes(const QuantArgs &a, const BhqBlock *bst, const float *wsum,
+                                int num_sms, cudaStream_t st) {
+  auto kern = k_bhq_codes<T, LPR>;
   const size_t smem = sizeof(int) * (size_t)a.C;
-#define FQT_BW(L, S)                                                                  \
-  if (CO == L && steps == S) {                                                        \
-    if (bf16)                                                                         \
-      k_bhq_warp<__nv_bfloat16, L, S><<<(int)grid, 256, smem, st>>>(a);               \
-    else                                                                              \
-      k_bhq_warp<float, L, S><<<(int)grid, 256, smem, st>>>(a);                       \
+  int per_sm = 0;
+  const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);
+  if (e != cudaSuccess) return e;
+  const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;
+  int64_t grid = (nchunks + 7) / 8;
+  const int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);
+  if (grid > cap) grid = cap;
+  if (grid < 1) grid = 1;
+  kern<<<(int)grid, 256, smem, st>>>(a, bst, wsum);
+  return cudaGetLastError();
+}
+
+// The two-pass BHQ quantizer takes fixed blocks of 4, 8 or 16 rows and rows
+// of 64, 128 or 256 t (t = 1, 2, 4, 8) columns; bf16 input with blocks of 16.
+bool bhq_pass_supported(int C, int block, bool bf16) {
+  if (block != 4 && block != 8 && block != 16) return false;
+  if (bf16 && block != 16) return false;
+  return C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048;
+}
+
+// Statistics pass, code pass and the grad_X offsets (k_bhq_offsets) of the
+// fixed-block BHQ quantizer with Q_b1.  `scratch` (bhq_pass_bytes) holds the
+// per-block records and column sums w between the passes; `part` receives
+// the statistics pass's range partials, which the code pass reduces.
+fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch,
+                             float2 *part, cudaStream_t st) {
+  if (a.kind != KIND_BHQ || !bhq_pass_supported(a.C, a.block, bf16)) return FQT_EUNSUPPORTED;
+  const int64_t nblocks = (a.N + a.block - 1) / a.block;
+  BhqBlock *bst = static_cast<BhqBlock *>(scratch);
+  float *wsum = reinterpret_cast<float *>(
+      (reinterpret_cast<uintptr_t>(bst + nblocks) + 255) & ~(uintptr_t)255);
+  const int C = a.C, nb = a.block;
+  int grid1 = 0;
+  cudaError_t e = cudaErrorInvalidValue;
+#define FQT_ST(TT, L, S, TM) e = launch_stats<TT, L, S, TM>(a, bst, wsum, part, num_sms, &grid1, st);
+  if (!bf16) {
+    if (C == 64) {
+      if (nb == 4) { FQT_ST(float, 8, 1, 1) } else if (nb == 8) { FQT_ST(float, 8, 2, 1) }
+      else { FQT_ST(float, 8, 4, 1) }
+    } else if (C == 128) {
+      if (nb == 4) { FQT_ST(float, 16, 2, 1) } else if (nb == 8) { FQT_ST(float, 16, 4, 1) }
+      else { FQT_ST(float, 16, 8, 1) }
+    } else {
+      const int team = C / 256;
+#define FQT_ST_T(S)                                                                  \
+  if (team == 1) { FQT_ST(float, 32, S, 1) } else if (team == 2) { FQT_ST(float, 32, S, 2) } \
+  else if (team == 4) { FQT_ST(float, 32, S, 4) } else { FQT_ST(float, 32, S, 8) }
+      if (nb == 4) { FQT_ST_T(4) } else if (nb == 8) { FQT_ST_T(8) } else { FQT_ST_T(16) }
+#undef FQT_ST_T
+    }
+  } else {
+    if (C == 64) { FQT_ST(__nv_bfloat16, 8, 4, 1) }
+    else if (C == 128) { FQT_ST(__nv_bfloat16, 16, 8, 1) }
+    else if (C == 256) { FQT_ST(__nv_bfloat16, 32, 16, 1) }
+    else if (C == 512) { FQT_ST(__nv_bfloat16, 32, 16, 2) }
+    else if (C == 1024) { FQT_ST(__nv_bfloat16, 32, 16, 4) }
+    else { FQT_ST(__nv_bfloat16, 32, 16, 8) }
   }
-  FQT_BW(8, 1)
-  FQT_BW(8, 2)
-  FQT_BW(8, 4)
-  FQT_BW(8, 8)
-  FQT_BW(16, 1)
-  FQT_BW(16, 2)
-  FQT_BW(16, 4)
-  FQT_BW(16, 8)
-  FQT_BW(32, 1)
-  FQT_BW(32, 2)
-  FQT_BW(32, 4)
-  FQT_BW(32, 8)
-#undef FQT_BW
-  return cuda_fail(cudaGetLastError(), "BHQ warp quantizer launch");
+#undef FQT_ST
+  if (e != cudaSuccess) return cuda_fail(e, "BHQ statistics pass launch");
+  QuantArgs a2 = a;
+  a2.part = part;
+  a2.npart = grid1;
+  const int lpr = C == 64 ? 8 : C == 128 ? 16 : 32;
+  if (!bf16) {
+    e = lpr == 8 ? launch_codes<float, 8>(a2, bst, wsum, num_sms, st)
+        : lpr == 16 ? launch_codes<float, 16>(a2, bst, wsum, num_sms, st)
+                    : launch_codes<float, 32>(a2, bst, wsum, num_sms, st);
+  } else {
+    e = lpr == 8 ? launch_codes<__nv_bfloat16, 8>(a2, bst, wsum, num_sms, st)
+        : lpr == 16 ? launch_codes<__nv_bfloat16, 16>(a2, bst, wsum, num_sms, st)
+                    : launch_codes<__nv_bfloat16, 32>(a2, bst, wsum, num_sms, st);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "BHQ code pass launch");
+  if (a.hz && a.hr) {
+    e = launch_bhq_offsets(a.zero2, a.rsum2, a.lead2, a.hz, a.hr, a.N, C, a.bits, a.block, st);
+    if (e != cudaSuccess) return cuda_fail(e, "BHQ offsets launch");
+  }
+  return FQT_OK;
 }
 
 // ---------------------------------------------------------------------------
