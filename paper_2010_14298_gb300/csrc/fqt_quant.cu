@@ -1223,24 +1223,39 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
 // elsewhere) as the statistics pass computed it, v = t - z'_k, stochastic
 // rounding of v (Q_b2) and of s (h - min H) (Q_b1), fp16 carriers (and
 // optional bytes), row sums of Q_b2 and column sums of the grad_W code set.
-// A warp takes chunks of kCodeRows rows; it walks the row's slabs of 8 LPR
-// columns one after another and, inside a slab, the chunk's rows 32 / LPR at
-// a time (lane: 8 columns of one row), so the loops stay rolled and rows
+// A lane owns two octs of a row, o and o + LPR of a slab of 16 LPR columns
+// (one coalesced 16 LPR x 4-byte access per oct); a warp takes chunks of
+// kCodeRows rows, walks the row's slabs one after another and, inside a
+// slab, the chunk's rows 32 / LPR at a time, issuing the loads of its next
+// row before it rounds the current one.  A block's w_j and scalars stay in
+// registers while the lane's rows belong to it.  Loops stay rolled and rows
 // need no exchange between warps.
 // ---------------------------------------------------------------------------
 constexpr int kCodeRows = 32;
 
+template <typename T>
+__device__ __forceinline__ void load_two_octs(const T *row, int c_a, int c_b, float (&x)[16]) {
+  float lo[8], hi[8];
+  load_oct(row + c_a, lo);
+  load_oct(row + c_b, hi);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    x[j] = lo[j];
+    x[8 + j] = hi[j];
+  }
+}
+
 template <typename T, int LPR>
 __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
                                                    const BhqBlock *__restrict__ bst,
-                                                   const float *__restrict__ wsum) {
-  constexpr int RS = 32 / LPR, SLAB = 8 * LPR;
+                                                   const float *__restrict__ wsum, int lg_nb) {
+  constexpr int RS = 32 / LPR, SLAB = 16 * LPR;
   __shared__ float2 red[8];
   __shared__ int redi[8];
   __shared__ int rs_s[8][2][kCodeRows];
   extern __shared__ int csum_s[];  // C column sums of the grad_W code set
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int C = a.C, CO = C / 8, nb = a.block;
+  const int C = a.C, CO = C / 8;
   const int sub = lane / LPR, o = lane - sub * LPR;
 
   // ---- global range (Q_b1 scale) from the statistics-pass partials ----
@@ -1291,6 +1306,8 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
   const __half2 bias2 = __half2half2(__int2half_rn(1024 + (int)((B2 + 1u) >> 1)));
   const __half2 bias1 = __half2half2(__int2half_rn(1024 + 128));
   const bool want_rs1 = has_b1 && a.rsum1 != nullptr;
+  const T *const h = reinterpret_cast<const T *>(a.h);
+  const int nbm = (1 << lg_nb) - 1;
 
   const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;
   const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
@@ -1303,56 +1320,100 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
     __syncwarp();
 #pragma unroll 1
     for (int c0 = 0; c0 < C; c0 += SLAB) {
-      const int col0 = c0 + o * 8;
-      uint32_t cs[8];
+      const int ca = c0 + o * 8, cb = ca + 8 * LPR;  // this lane's two octs
+      uint32_t cs[16];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) cs[j] = 0u;
+      for (int j = 0; j < 16; ++j) cs[j] = 0u;
       uint32_t cs_rows = 0;
+      int64_t cur_blk = -1;
+      float w[16];
+      float sk_l = 0.0f, sk_o = 0.0f, ck_l = 0.0f, ck_o = 0.0f;
+      int p_lead = -1;
+      // the first row's loads; every later row's are issued one row ahead
+      float xn[16];
+      float zn = 0.0f;
+      {
+        const int rr = sub;
+        if (rr < rows) {
+          load_two_octs(h + (row0 + rr) * C, ca, cb, xn);
+          zn = a.zero2[row0 + rr];
+        }
+      }
 #pragma unroll 1
       for (int rb = 0; rb < rows; rb += RS) {  // the same trip count in every lane
         const int rr = rb + sub;
         const bool valid = rr < rows;  // the LPR lanes of a row agree
+        float x[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) x[j] = xn[j];
+        const float zr = zn;
+        if (rr + RS < rows) {
+          load_two_octs(h + (row0 + rr + RS) * C, ca, cb, xn);
+          zn = a.zero2[row0 + rr + RS];
+        }
         uint32_t acc1 = 0u, acc2 = 0u;
         if (valid) {
           const int64_t row = row0 + rr;
-          const int64_t blk = row / nb;
-          const BhqBlock bs = bst[blk];
-          const bool lead = (int)(row - blk * nb) == __float_as_int(bs.p);
-          const float sk = lead ? bs.s1 : bs.s2;
-          const float ck = lead ? bs.rho - 1.0f : bs.rho;
-          const float zr = a.zero2[row];
-          float x[8], w[8];
-          load_oct(reinterpret_cast<const T *>(a.h) + row * C + col0, x);
-          load_oct(wsum + blk * (int64_t)C + col0, w);
-          const uint64_t q = (uint64_t)row * (uint64_t)CO + (uint64_t)(col0 >> 3);
+          const int64_t blk = row >> lg_nb;
+          if (blk != cur_blk) {  // a new block: its w_j and scalars
+            const BhqBlock bs = bst[blk];
+            p_lead = __float_as_int(bs.p);
+            sk_l = bs.s1;
+            sk_o = bs.s2;
+            ck_l = bs.rho - 1.0f;
+            ck_o = bs.rho;
+            load_two_octs(wsum + blk * (int64_t)C, ca, cb, w);
+            cur_blk = blk;
+          }
+          const bool lead = (int)(row & nbm) == p_lead;
+          const float sk = lead ? sk_l : sk_o;
+          const float ck = lead ? ck_l : ck_o;
+          const uint64_t qa = (uint64_t)row * (uint64_t)CO + (uint64_t)(ca >> 3);
+          const uint64_t qb = qa + (uint64_t)LPR;
           if (has_b1) {
-            const uint4 u1 = philox_oct(q, 1u, key);
-            uint32_t b[8];
-            acc1 = 0u - 8u * kSrBits;
+            const uint4 ua = philox_oct(qa, 1u, key), ub = philox_oct(qb, 1u, key);
+            uint32_t b[16];
+            acc1 = 0u - 16u * kSrBits;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+            for (int j = 0; j < 16; ++j) {
               const float v = fminf(__fmul_rn(__fsub_rn(x[j], gmin), s_g1), 255.0f);
-              b[j] = sr_bits(v, sr_u(u1, j));
+              b[j] = sr_bits(v, sr_u(j < 8 ? ua : ub, j & 7));
               cs[j] += b[j];
               acc1 += b[j];
             }
             ++cs_rows;
-            if (a.c1) store_codes_bits(a.c1 + row * (int64_t)C + col0, b);
-            if (a.f1) store_carriers_bits(a.f1 + row * (int64_t)C + col0, b, bias1);
+            uint32_t (&b0)[8] = *reinterpret_cast<uint32_t(*)[8]>(&b[0]);
+            uint32_t (&b1)[8] = *reinterpret_cast<uint32_t(*)[8]>(&b[8]);
+            if (a.c1) {
+              store_codes_bits(a.c1 + row * (int64_t)C + ca, b0);
+              store_codes_bits(a.c1 + row * (int64_t)C + cb, b1);
+            }
+            if (a.f1) {
+              store_carriers_bits(a.f1 + row * (int64_t)C + ca, b0, bias1);
+              store_carriers_bits(a.f1 + row * (int64_t)C + cb, b1, bias1);
+            }
           }
-          const uint4 u2 = philox_oct(q, 0u, key);
-          uint32_t b[8];
-          acc2 = 0u - 8u * kSrBits;
+          const uint4 ua = philox_oct(qa, 0u, key), ub = philox_oct(qb, 0u, key);
+          uint32_t b[16];
+          acc2 = 0u - 16u * kSrBits;
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
+          for (int j = 0; j < 16; ++j) {
             const float t = fmaf(-ck, w[j], __fmul_rn(sk, x[j]));
-            b[j] = sr_bits(fminf(__fsub_rn(t, zr), fB2), sr_u(u2, j));
+            b[j] = sr_bits(fminf(__fsub_rn(t, zr), fB2), sr_u(j < 8 ? ua : ub, j & 7));
             acc2 += b[j];
             if (!has_b1) cs[j] += b[j];
           }
           if (!has_b1) ++cs_rows;
-          if (a.c2) store_codes_bits(a.c2 + row * (int64_t)C + col0, b);
-          if (a.f2) store_carriers_bits(a.f2 + row * (int64_t)C + col0, b, bias2);
+          uint32_t (&b0)[8] = *reinterpret_cast<uint32_t(*)[8]>(&b[0]);
+          uint32_t (&b1)[8] = *reinterpret_cast<uint32_t(*)[8]>(&b[8]);
+          if (a.c2) {
+            store_codes_bits(a.c2 + row * (int64_t)C + ca, b0);
+            store_codes_bits(a.c2 + row * (int64_t)C + cb, b1);
+          }
+          if (a.f2) {
+            store_carriers_bits(a.f2 + row * (int64_t)C + ca, b0, bias2);
+            store_carriers_bits(a.f2 + row * (int64_t)C + cb, b1, bias2);
+          }
         }
         if (want_rs1) {
           const int r1 = row_reduce<LPR>((int)acc1, OpAdd());
@@ -1364,9 +1425,9 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
       // this slab's column sums: the lanes of one column add theirs
       if (csum_g) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 16; ++j) {
           const int v = xor_reduce<LPR>((int)(cs[j] - cs_rows * kSrBits), OpAdd());
-          if (sub == 0 && v) atomicAdd(&csum_s[col0 + j], v);
+          if (sub == 0 && v) atomicAdd(&csum_s[(j < 8 ? ca : cb) + (j & 7)], v);
         }
       }
     }
@@ -1406,6 +1467,8 @@ static cudaError_t launch_stats(const QuantArgs &a, BhqBlock *bst, float *wsum, 
 template <typename T, int LPR>
 static cudaError_t launch_codes(const QuantArgs &a, const BhqBlock *bst, const float *wsum,
                                 int num_sms, cudaStream_t st) {
+  int lg_nb = 0;
+  while ((1 << lg_nb) < a.block) ++lg_nb;
   auto kern = k_bhq_codes<T, LPR>;
   const size_t smem = sizeof(int) * (size_t)a.C;
   int per_sm = 0;
@@ -1416,7 +1479,7 @@ static cudaError_t launch_codes(const QuantArgs &a, const BhqBlock *bst, const f
   const int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  kern<<<(int)grid, 256, smem, st>>>(a, bst, wsum);
+  kern<<<(int)grid, 256, smem, st>>>(a, bst, wsum, lg_nb);
   return cudaGetLastError();
 }
 
@@ -1471,13 +1534,16 @@ fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch
   QuantArgs a2 = a;
   a2.part = part;
   a2.npart = grid1;
-  const int lpr = C == 64 ? 8 : C == 128 ? 16 : 32;
+  // lanes per row: a lane owns 16 columns (two octs) of a slab of 16 LPR
+  const int lpr = C == 64 ? 4 : C == 128 ? 8 : C == 256 ? 16 : 32;
   if (!bf16) {
-    e = lpr == 8 ? launch_codes<float, 8>(a2, bst, wsum, num_sms, st)
+    e = lpr == 4    ? launch_codes<float, 4>(a2, bst, wsum, num_sms, st)
+        : lpr == 8  ? launch_codes<float, 8>(a2, bst, wsum, num_sms, st)
         : lpr == 16 ? launch_codes<float, 16>(a2, bst, wsum, num_sms, st)
                     : launch_codes<float, 32>(a2, bst, wsum, num_sms, st);
   } else {
-    e = lpr == 8 ? launch_codes<__nv_bfloat16, 8>(a2, bst, wsum, num_sms, st)
+    e = lpr == 4    ? launch_codes<__nv_bfloat16, 4>(a2, bst, wsum, num_sms, st)
+        : lpr == 8  ? launch_codes<__nv_bfloat16, 8>(a2, bst, wsum, num_sms, st)
         : lpr == 16 ? launch_codes<__nv_bfloat16, 16>(a2, bst, wsum, num_sms, st)
                     : launch_codes<__nv_bfloat16, 32>(a2, bst, wsum, num_sms, st);
   }
