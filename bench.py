@@ -621,6 +621,31 @@ def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
         return out
 
     ex = {}
+    # dense tensor-core rates (burst, each kernel timed alone): the fp16 kind
+    # the contractions use, e4m3, and the legacy mma.sync IMMA path
+    wsp0 = fqt.Workspace(1, 16, 16, device=dev)
+    peaks = {}
+    for kind, name, iters in ((0, "tcgen05 kind::f16 (fp16 x fp16 -> fp32) TFLOP/s", 20000),
+                              (1, "tcgen05 kind::f8f6f4 (e4m3 x e4m3 -> fp32) TFLOP/s", 20000),
+                              (2, "mma.sync m16n8k32 u8 x s8 -> s32 TOPS", 4000)):
+        fqt.debug_mma_peak(kind, 50, wsp0)
+        torch.cuda.synchronize()
+        best = 0.0
+        for _ in range(3):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            ops = fqt.debug_mma_peak(kind, iters, wsp0)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            best = max(best, ops / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+        peaks[name] = best
+    peaks["tcgen05 kind::i8"] = "does not assemble for sm_103a (ptxas)"
+    props = torch.cuda.get_device_properties(dev)
+    peaks["sm_count"] = props.multi_processor_count
+    peaks["l2_bytes"] = getattr(props, "L2_cache_size", None)
+    peaks["device_status"] = fqt.sync_status(wsp0)
+    ex["mma_peaks"] = peaks
     # linear layer 128 x 256: launch-bound, reported as latency
     L1 = wl.config(0)[0]
     ex["linear-128x256"] = {

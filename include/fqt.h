@@ -297,6 +297,19 @@ FQT_API fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits
 FQT_API fqt_status fqt_debug_wait_timeout(void *workspace, size_t ws_bytes,
                                           uint64_t limit_ns, void *stream);
 
+/* Dense tensor-core rate kernels, the denominators of the contractions'
+ * rooflines: kind 0 tcgen05 kind::f16 (fp16 x fp16 -> fp32, the operand
+ * format of this library's contractions), kind 1 tcgen05 kind::f8f6f4 (e4m3
+ * x e4m3 -> fp32), kind 2 warp-level mma.sync m16n8k32 u8 x s8 -> s32.
+ * (tcgen05 kind::i8 does not assemble for sm_103a.)  Enqueues one launch on
+ * `stream` that runs `iters` rounds of back-to-back MMAs on zero operands
+ * on every SM and sets *ops_out (host memory) to the multiply-add
+ * operations it performs (2 per multiply-add); the caller times the launch.
+ * The workspace holds the status word (at least 256 bytes, 256-byte
+ * aligned).  Has no counterpart in the paper. */
+FQT_API fqt_status fqt_debug_mma_peak(int kind, int64_t iters, double *ops_out,
+                                      void *workspace, size_t ws_bytes, void *stream);
+
 /* Static description of a status code. */
 FQT_API const char *fqt_status_string(fqt_status status);
 

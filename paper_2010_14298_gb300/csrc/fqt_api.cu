@@ -414,6 +414,12 @@ fqt_status fqt_debug_wait_timeout(void *workspace, size_t ws_bytes, uint64_t lim
                             reinterpret_cast<cudaStream_t>(stream));
 }
 
+fqt_status fqt_debug_mma_peak(int kind, int64_t iters, double *ops_out, void *workspace,
+                              size_t ws_bytes, void *stream) {
+  return debug_mma_peak(kind, iters, ops_out, workspace, ws_bytes,
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
 const char *fqt_last_cuda_error(void) { return g_last_error; }
 
 const char *fqt_status_string(fqt_status status) {

@@ -3123,3 +3123,130 @@ fqt_status debug_wait_timeout(void *ws, size_t ws_bytes, uint64_t limit_ns,
 }
 
 }  // namespace fqt
+
+namespace fqt {
+
+// ---------------------------------------------------------------------------
+// Dense tensor-core rates of this GPU, the denominators of the contractions'
+// rooflines (kind 0: tcgen05 kind::f16, fp16 x fp16 -> fp32; kind 1: tcgen05
+// kind::f8f6f4, e4m3 x e4m3 -> fp32; kind 2: warp-level mma.sync m16n8k32
+// u8 x s8 -> s32).  tcgen05 kind::i8 does not assemble for sm_103a.  One CTA
+// per SM: one thread issues `iters` rounds of four back-to-back M128 N256
+// MMAs (K 16 each for f16, 32 for e4m3, i.e. one 128-byte row of operands)
+// into one TMEM accumulator, then waits (bounded) for them to drain.
+// Operands are zero: the rates do not depend on the values.
+// ---------------------------------------------------------------------------
+constexpr int kPeakN = 256;
+
+__device__ __forceinline__ void umma_f8(uint32_t tmem_d, uint64_t a_desc, uint64_t b_desc,
+                                        uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__global__ void __launch_bounds__(128, 1) k_peak_umma(int kind, int64_t iters, int *status) {
+  extern __shared__ __align__(1024) uint8_t peak_raw[];
+  uint8_t *ops = peak_raw + ((1024u - (smem_u32(peak_raw) & 1023u)) & 1023u);
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t tslot;
+  const int warp = threadIdx.x >> 5;
+  for (int i = threadIdx.x; i < (int)(kTileBytes + 2 * kTileBytes) / 16; i += blockDim.x)
+    reinterpret_cast<uint4 *>(ops)[i] = make_uint4(0u, 0u, 0u, 0u);
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tslot)),
+                 "r"((uint32_t)kPeakN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_proxy_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tslot;
+  if (threadIdx.x == 0) {
+    // A: 128 rows x 128 bytes, B: 256 rows x 128 bytes, K-major, 128-byte swizzle
+    const uint64_t da = sw128_desc(smem_u32(ops));
+    const uint64_t db = sw128_desc(smem_u32(ops + kTileBytes));
+    // D fp32; A, B fp16 (kind::f16) or e4m3 (kind::f8f6f4, format 0); K-major
+    const uint32_t idesc =
+        (1u << 4) | ((uint32_t)(kPeakN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+    for (int64_t it = 0; it < iters; ++it) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        if (kind == 0)
+          umma_f16(tmem, da + 2 * k, db + 2 * k, idesc, (it | k) ? 1u : 0u);
+        else
+          umma_f8(tmem, da + 2 * k, db + 2 * k, idesc, (it | k) ? 1u : 0u);
+      }
+    }
+    umma_commit(&bar);
+    mbar_wait(&bar, 0, status);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"((uint32_t)kPeakN)
+                 : "memory");
+  }
+}
+
+// mma.sync u8 x s8 -> s32 (m16n8k32): eight independent accumulators per warp
+__global__ void __launch_bounds__(256) k_peak_imma(int64_t iters, int *sink) {
+  const uint32_t lane = threadIdx.x & 31;
+  const uint32_t a0 = 0x01010101u * (lane & 7), a1 = a0 ^ 0x02020202u, a2 = a0 ^ 0x04040404u,
+                 a3 = a0 ^ 0x08080808u, b0 = 0x03030303u, b1 = 0x05050505u;
+  int acc[8][4];
+#pragma unroll
+  for (int c = 0; c < 8; ++c)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[c][i] = 0;
+  for (int64_t it = 0; it < iters; ++it) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+      asm volatile(
+          "mma.sync.aligned.m16n8k32.row.col.s32.u8.s8.s32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+          "{%8, %9}, {%0, %1, %2, %3};"
+          : "+r"(acc[c][0]), "+r"(acc[c][1]), "+r"(acc[c][2]), "+r"(acc[c][3])
+          : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  }
+  int s = 0;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) s += acc[c][0] + acc[c][1] + acc[c][2] + acc[c][3];
+  if (s == 0x7fffffff) *sink = s;  // keeps the accumulators live
+}
+
+fqt_status debug_mma_peak(int kind, int64_t iters, double *ops_out, void *ws, size_t ws_bytes,
+                          cudaStream_t st) {
+  if (kind < 0 || kind > 2 || iters <= 0 || iters > ((int64_t)1 << 32) || !ops_out)
+    return FQT_EINVAL;
+  if (!ws || ws_bytes < kHeaderBytes || ((uintptr_t)ws & 255)) return FQT_EWORKSPACE;
+  int *status = static_cast<int *>(ws);
+  const int nsm = device_sm_count();
+  if (kind <= 1) {
+    const size_t smem = 3 * kTileBytes + 1024;
+    cudaError_t e = cudaFuncSetAttribute(k_peak_umma, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "peak attribute");
+    k_peak_umma<<<nsm, 128, smem, st>>>(kind, iters, status);
+    const double k_per = kind == 0 ? 16.0 : 32.0;
+    *ops_out = 2.0 * BM * kPeakN * k_per * 4.0 * (double)iters * nsm;
+  } else {
+    const int ctas = nsm * 4;
+    k_peak_imma<<<ctas, 256, 0, st>>>(iters, status + 1);
+    *ops_out = 2.0 * 16 * 8 * 32 * 8.0 * (double)iters * ctas * 8;
+  }
+  return cuda_fail(cudaGetLastError(), "peak launch");
+}
+
+}  // namespace fqt

@@ -99,6 +99,8 @@ fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
                                 float *grad_W, cudaStream_t st);
 fqt_status fixed_scratch_status(int **out);
 fqt_status debug_wait_timeout(void *ws, size_t ws_bytes, uint64_t limit_ns, cudaStream_t st);
+fqt_status debug_mma_peak(int kind, int64_t iters, double *ops_out, void *ws, size_t ws_bytes,
+                          cudaStream_t st);
 fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H, void *ws,
                           size_t ws_bytes, cudaStream_t st);
 fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,

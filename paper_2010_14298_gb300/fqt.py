@@ -93,6 +93,9 @@ def load(build_if_missing: bool = True):
         lib.fqt_fixed_scratch_sync_status.restype = i32
         lib.fqt_debug_wait_timeout.argtypes = [P, sz, u64, P]
         lib.fqt_debug_wait_timeout.restype = i32
+        lib.fqt_debug_mma_peak.argtypes = [i32, i64, ctypes.POINTER(ctypes.c_double), P, sz,
+                                           P]
+        lib.fqt_debug_mma_peak.restype = i32
         lib.fqt_debug_int_gemm.argtypes = [P, i32, i32, P, i32, i32, i64, i64,
                                            i64, P, P, sz, P]
         lib.fqt_debug_int_gemm.restype = i32
@@ -463,6 +466,15 @@ def debug_wait_timeout(limit_ns: int, ws: Optional[Workspace] = None, stream=Non
                                     ws.nbytes if ws is not None else 0,
                                     ctypes.c_uint64(limit_ns), _stream(stream))
     _check(st, "fqt_debug_wait_timeout")
+
+
+def debug_mma_peak(kind: int, iters: int, ws: Workspace, stream=None) -> float:
+    """Enqueues the rate kernel of `kind` (0 tcgen05 f16, 1 tcgen05 e4m3,
+    2 mma.sync u8 x s8); returns the operations it performs."""
+    ops = ctypes.c_double(0.0)
+    _check(load().fqt_debug_mma_peak(kind, iters, ctypes.byref(ops), ws.ptr, ws.nbytes,
+                                     _stream(stream)), "fqt_debug_mma_peak")
+    return ops.value
 
 
 def status_string(code: int) -> str:
