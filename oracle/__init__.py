@@ -95,6 +95,8 @@ def _load():
         lib.orc_quant_bhq_groups.restype = i64
         lib.orc_dequant_groups_f64.argtypes = [P, i64, i64, P, i64, P, P, P]
         lib.orc_dequant_groups_f64.restype = None
+        lib.orc_col2im_nhwc.argtypes = [P, i64, i64, i64, i64, i32, i32, i32, i32, P]
+        lib.orc_col2im_nhwc.restype = None
         _lib = lib
         return lib
 
@@ -363,6 +365,69 @@ def grad_x(q_b2: dict, q_w: dict, codes_b2=None) -> np.ndarray:
 def grad_w(q_b1: dict, q_x: dict, codes_b1=None) -> np.ndarray:
     """grad_W = Q_b1(dH)^T X~ (C x D; the transpose of Eq. 6's D x C form)."""
     return matmul(dequant(q_b1, codes_b1), dequant(q_x), a_trans=True)
+
+
+# --------------------------------------------------------------------------
+# Per-image samples and col2im (a conv layer as a linear layer on im2col rows,
+# Sec. 2.1; a "sample" is one input's gradient, Sec. 4.1)
+# --------------------------------------------------------------------------
+def quantize_grad_samples(dH, rows_per_sample: int, kind: int, bits: int, block: int = 0,
+                          seed: int = 0, stream: int = STREAM_B2, want_v: bool = False) -> dict:
+    """Q_b2 with one sample per group of `rows_per_sample` consecutive rows of
+    dH (an image's H W output pixels of a conv layer): the quantizer of the
+    given kind applied to the (N / R) x (R C) matrix whose rows are the
+    images' whole gradients.  The flat index of every entry, and so its SR
+    uniform, is that of dH.  The dict is the quantizer's on that matrix
+    (codes, inv_s, zero, lead, v reshaped to N x C) with ``rows_per_sample``
+    set; ``inv_s_rows`` / ``zero_rows`` repeat the per-sample values for each
+    row (PTQ keeps its single entry)."""
+    h = _f32(dH)
+    n, c = h.shape
+    R = int(rows_per_sample)
+    if R < 1 or n % R:
+        raise OracleError("rows_per_sample must divide the rows")
+    q = quantize_grad(h.reshape(n // R, R * c), kind, bits, block, seed, stream, want_v)
+    q["codes"] = q["codes"].reshape(n, c)
+    if want_v:
+        q["v"] = q["v"].reshape(n, c)
+    q["rows_per_sample"] = R
+    if kind == PTQ:
+        q["inv_s_rows"], q["zero_rows"] = q["inv_s"], q["zero"]
+    else:
+        q["inv_s_rows"] = np.repeat(q["inv_s"], R)
+        q["zero_rows"] = np.repeat(q["zero"], R)
+    return q
+
+
+def dequant_samples(q: dict) -> np.ndarray:
+    """The value of a per-sample quantized dH (N x C): Eq. 9 on the
+    (N / R) x (R C) matrix of samples, read back as N x C."""
+    R = q["rows_per_sample"]
+    n, c = q["codes"].shape
+    view = dict(q)
+    view["codes"] = q["codes"].reshape(n // R, R * c)
+    return dequant(view).reshape(n, c)
+
+
+def col2im_nhwc(G, n: int, h: int, w: int, c: int, kh: int, kw: int, stride: int = 1,
+                pad: int = 0) -> np.ndarray:
+    """NHWC sum of an im2col-space gradient (the adjoint of im2col)."""
+    g = np.ascontiguousarray(G, dtype=np.float64)
+    oh = (h + 2 * pad - kh) // stride + 1
+    ow = (w + 2 * pad - kw) // stride + 1
+    if g.shape != (n * oh * ow, kh * kw * c):
+        raise OracleError("G has the wrong shape for this geometry")
+    out = np.zeros((n, h, w, c))
+    _load().orc_col2im_nhwc(_ptr(g), n, h, w, c, kh, kw, stride, pad, _ptr(out))
+    return out
+
+
+def grad_x_nhwc(q_b2: dict, q_w: dict, n: int, h: int, w: int, cin: int, k: int,
+                pad: int) -> np.ndarray:
+    """grad_X of a stride-1 k x k conv in NHWC: col2im of Q_b2(dH) W~ (Eq. 6),
+    Q_b2 per row, per sample (``rows_per_sample``) or per tensor."""
+    deq = dequant_samples(q_b2) if "rows_per_sample" in q_b2 else dequant(q_b2)
+    return col2im_nhwc(matmul(deq, dequant(q_w)), n, h, w, cin, k, k, 1, pad)
 
 
 def linear_backward(dH, X, W, kind: int, bits: int, block: int, seed: int,

@@ -666,3 +666,30 @@ void orc_matmul_f64(const double *A, int a_trans, const double *Bm, int64_t M,
       for (int64_t j = 0; j < N; ++j) out[i * N + j] += a * Bm[k * N + j];
     }
 }
+
+/* ------------------------------------------------------------------------ */
+/* col2im of an im2col-space gradient (the adjoint of im2col; a conv layer   */
+/* as a linear layer on im2col rows, Sec. 2.1): G has one row per output     */
+/* pixel (n, oy, ox) and columns (ky, kx, c); the result is NHWC,            */
+/* out[n, y, x, c] = sum of G[(n, oy, ox), (ky, kx, c)] over the output      */
+/* pixels and taps with y = oy stride + ky - pad, x = ox stride + kx - pad.  */
+/* ------------------------------------------------------------------------ */
+void orc_col2im_nhwc(const double *G, int64_t n, int64_t h, int64_t w, int64_t c, int kh,
+                     int kw, int stride, int pad, double *out) {
+  int64_t oh = (h + 2 * pad - kh) / stride + 1;
+  int64_t ow = (w + 2 * pad - kw) / stride + 1;
+  for (int64_t i = 0; i < n * h * w * c; ++i) out[i] = 0.0;
+  for (int64_t b = 0; b < n; ++b)
+    for (int64_t oy = 0; oy < oh; ++oy)
+      for (int64_t ox = 0; ox < ow; ++ox) {
+        const double *row = G + ((b * oh + oy) * ow + ox) * (int64_t)(kh * kw) * c;
+        for (int ky = 0; ky < kh; ++ky)
+          for (int kx = 0; kx < kw; ++kx) {
+            int64_t y = oy * stride + ky - pad, x = ox * stride + kx - pad;
+            if (y < 0 || y >= h || x < 0 || x >= w) continue; /* a padding entry */
+            const double *g = row + (int64_t)(ky * kw + kx) * c;
+            double *o = out + ((b * h + y) * w + x) * c;
+            for (int64_t ch = 0; ch < c; ++ch) o[ch] += g[ch];
+          }
+      }
+}

@@ -681,3 +681,95 @@ def test_shift_gradients_are_unbiased_exactly():
     assert np.abs(orc.matmul(e, Wt) - dH.astype(np.float64) @ Wt).max() <= 1e-4 * np.abs(dH @ Wt).max()
     assert np.abs(orc.matmul(e, Xt, a_trans=True) - dH.astype(np.float64).T @ Xt).max() <= \
         1e-4 * np.abs(dH.T @ Xt).max()
+
+
+# --------------------------------------------------------------------------
+# Per-image samples and col2im (Sec. 2.1 conv as a linear layer on im2col
+# rows; Sec. 4.1 a sample is one input's gradient)
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("n,h,w,c,k,stride,pad", [(2, 5, 6, 3, 3, 1, 1), (1, 7, 7, 4, 1, 1, 0),
+                                                  (2, 6, 5, 2, 3, 1, 0), (1, 9, 8, 3, 5, 1, 2),
+                                                  (2, 8, 8, 3, 3, 2, 1)])
+def test_col2im_is_the_adjoint_of_im2col(n, h, w, c, k, stride, pad):
+    """<col2im(G), x> = <G, im2col(x)> for every G and x, with the im2col of
+    the workload generator (an independent numpy implementation)."""
+    g = wl.rng(n * 100 + h * 10 + k)
+    x = g.standard_normal((n, h, w, c))
+    X = wl.im2col_nhwc(x, k, k, stride, pad)
+    G = g.standard_normal(X.shape)
+    lhs = float((orc.col2im_nhwc(G, n, h, w, c, k, k, stride, pad) * x).sum())
+    rhs = float((G * X).sum())
+    assert lhs == pytest.approx(rhs, rel=1e-12, abs=1e-12)
+
+
+def test_col2im_of_a_one_by_one_conv_is_the_identity():
+    g = wl.rng(77)
+    G = g.standard_normal((2 * 4 * 5, 3))
+    out = orc.col2im_nhwc(G, 2, 4, 5, 3, 1, 1, 1, 0)
+    assert np.array_equal(out.reshape(-1, 3), G)
+
+
+def test_grad_x_nhwc_is_the_transposed_convolution():
+    """The input gradient of a stride-1 conv by brute force: dX[n,y,x,ci] =
+    sum over taps and output channels of dY[n, y+pad-ky, x+pad-kx, co]
+    W[co, ky, kx, ci], against col2im of the dequantized product."""
+    g = wl.rng(91)
+    n, h, w, ci, co, k, pad = 2, 5, 4, 3, 4, 3, 1
+    dH = g.standard_normal((n * h * w, co)).astype(np.float32)
+    W = (0.3 * g.standard_normal((co, k * k * ci))).astype(np.float32)
+    q2 = orc.quantize_grad_samples(dH, h * w, orc.PSQ, 8, 0, seed=3)
+    qw = orc.quantize_fwd(W, 8)
+    got = orc.grad_x_nhwc(q2, qw, n, h, w, ci, k, pad)
+    dY = orc.dequant_samples(q2).reshape(n, h, w, co)
+    Wd = orc.dequant(qw).reshape(co, k, k, ci)
+    ref = np.zeros((n, h, w, ci))
+    for b in range(n):
+        for y in range(h):
+            for x in range(w):
+                for ky in range(k):
+                    for kx in range(k):
+                        oy, ox = y + pad - ky, x + pad - kx
+                        if 0 <= oy < h and 0 <= ox < w:
+                            ref[b, y, x] += dY[b, oy, ox] @ Wd[:, ky, kx]
+    assert np.abs(got - ref).max() <= 1e-12 * np.abs(ref).max()
+
+
+@pytest.mark.parametrize("kind,bits", [(orc.PSQ, 8), (orc.PSQ, 5), (orc.PTQ, 5)])
+def test_one_row_samples_are_the_row_quantizer(kind, bits):
+    g = wl.rng(5)
+    dH = wl.random_grad(g, 12, 16, outlier_frac=0.2)
+    a = orc.quantize_grad_samples(dH, 1, kind, bits, 0, seed=9)
+    b = orc.quantize_grad(dH, kind, bits, 0, seed=9)
+    assert np.array_equal(a["codes"], b["codes"])
+    assert np.array_equal(a["inv_s"], b["inv_s"]) and np.array_equal(a["zero"], b["zero"])
+
+
+def test_per_sample_scale_spans_the_whole_sample():
+    """PSQ with samples of R rows: one scale per sample, B / R(h_i) over all
+    R C entries of the sample (Sec. 4.1), shared by its rows."""
+    g = wl.rng(6)
+    R, n, c, bits = 6, 24, 8, 5
+    dH = wl.random_grad(g, n, c, sigma=1.5)
+    q = orc.quantize_grad_samples(dH, R, orc.PSQ, bits, 0, seed=2)
+    B = (1 << bits) - 1
+    for i in range(n // R):
+        blk = dH[i * R:(i + 1) * R].astype(np.float32)
+        rng_ = np.float32(blk.max()) - np.float32(blk.min())
+        s = np.float32(B) / rng_
+        assert q["inv_s"][i] == np.float32(1.0) / s
+        assert np.all(q["inv_s_rows"][i * R:(i + 1) * R] == q["inv_s"][i])
+        assert q["codes"][i * R:(i + 1) * R].min() == 0  # the sample's minimum maps to 0
+    assert q["codes"].max() <= B
+
+
+@pytest.mark.parametrize("kind,bits,block", [(orc.PSQ, 5, 0), (orc.PSQ, 8, 0),
+                                             (orc.BHQ, 5, 2)])
+def test_per_sample_quantizer_is_unbiased_exactly(kind, bits, block):
+    g = wl.rng(31 + bits)
+    R = 3
+    dH = wl.random_grad(g, 12, 4, sigma=2.0, outlier_frac=0.3)
+    q = orc.quantize_grad_samples(dH, R, kind, bits, block, seed=4, want_v=True)
+    m, _ = _moments(q["v"], (1 << bits) - 1)
+    e_deq = orc.dequant_samples(dict(q, codes=m))
+    scale = np.abs(dH).max()
+    assert np.abs(e_deq - dH).max() <= 2e-5 * scale
