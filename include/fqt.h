@@ -76,7 +76,9 @@ typedef struct fqt_qtensor {
   int32_t bits;      /* b in [2, 8] */
   int32_t kind;      /* fqt_kind */
   int32_t block;     /* BHQ rows per block (power of two, <= 128); else 0 */
-  int32_t reserved;
+  int32_t rows_per_sample; /* written by the gradient quantizers: rows of dH
+                        that form one sample (Sec. 4.1), 1 for fqt_quantize_grad,
+                        R for fqt_quantize_grad_samples; 0 elsewhere */
   uint8_t *codes;    /* rows x cols, row-major, values in [0, 2^b - 1] */
   float *inv_s;      /* PTQ: 1 entry; PSQ, BHQ: rows entries (1/s_i; BHQ rows
                         of a block whose other rows are all zero hold 0) */
@@ -196,6 +198,26 @@ FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
                              uint64_t seed, fqt_qtensor *q_b2,
                              fqt_qtensor *q_b1, void *workspace,
                              size_t ws_bytes, void *stream);
+
+/*
+ * Q_b2 with per-image samples (Sec. 4.1: a sample is one input's gradient,
+ * here `rows_per_sample` = R consecutive rows of dH, e.g. an image's H W
+ * output pixels of a conv layer lowered to im2col, Sec. 2.1) and Q_b1 as in
+ * fqt_quantize_grad.  PSQ: the scale and zero point of sample i come from
+ * all R C entries of its rows, s_i = B / R(h_i), z_i = min h_i; codes are
+ * SR(s_i (h - z_i)) with the uniforms of fqt_quantize_grad (the flat index
+ * of dH).  inv_s and zero hold one entry per ROW (the sample's value
+ * repeated), row_sum per row, so the result is an ordinary PSQ operand of
+ * fqt_linear_backward, and q_b2->rows_per_sample = R.  PTQ is the
+ * per-tensor quantizer.  BHQ returns FQT_EUNSUPPORTED (its reflection mixes
+ * samples at every pixel, which neither contraction's epilogue forms).
+ * Needs N % R == 0, C in {64, 128, 256, 512, 1024, 2048}, N / R <= 2^20.
+ */
+FQT_API fqt_status fqt_quantize_grad_samples(const void *dH, fqt_dtype dtype, int64_t N,
+                                             int64_t C, int64_t rows_per_sample,
+                                             fqt_kind kind, int bits, uint64_t seed,
+                                             fqt_qtensor *q_b2, fqt_qtensor *q_b1,
+                                             void *workspace, size_t ws_bytes, void *stream);
 
 /*
  * The two low-bit contractions of Eq. 6 with App. E's bifurcation:

@@ -163,7 +163,9 @@ size_t fqt_workspace_size(int64_t N, int64_t C, int64_t D) {
   const size_t grp = group_workspace_bytes(N);         // adaptive BHQ grouping
   const size_t list = group_list_bytes(N);               // its grad_X work lists
   const size_t bhq = bhq_pass_bytes(N, C);                // two-pass BHQ scratch
+  const size_t smp = sample_pass_bytes(N, C, 1);          // per-sample PSQ scratch
   if (grp > need) need = grp;
+  if (smp > need) need = smp;
   if (bhq > need) need = bhq;
   if (list > need) need = list;
   return kGemmOffset + need;
@@ -185,6 +187,85 @@ fqt_status fqt_quantize_weight(const void *W, fqt_dtype dtype, int64_t rows,
                                void *workspace, size_t ws_bytes, void *stream) {
   return quantize_forward(W, dtype, rows, cols, bits, out, workspace, ws_bytes,
                           stream);
+}
+
+fqt_status fqt_quantize_grad_samples(const void *dH, fqt_dtype dtype, int64_t N, int64_t C,
+                                     int64_t rows_per_sample, fqt_kind kind, int bits,
+                                     uint64_t seed, fqt_qtensor *q_b2, fqt_qtensor *q_b1,
+                                     void *workspace, size_t ws_bytes, void *stream) {
+  if (N < 0 || C <= 0 || C > (1 << 20) || bits < 2 || bits > 8 || rows_per_sample < 1)
+    return FQT_EINVAL;
+  if (!q_b2 || (N > 0 && N % rows_per_sample)) return FQT_EINVAL;
+  if (kind == FQT_PTQ) {  // one scale for the whole tensor: the per-tensor quantizer
+    const fqt_status s = fqt_quantize_grad(dH, dtype, N, C, kind, bits, 0, seed, q_b2, q_b1,
+                                           workspace, ws_bytes, stream);
+    if (s == FQT_OK) q_b2->rows_per_sample = (int32_t)rows_per_sample;
+    return s;
+  }
+  if (kind != FQT_PSQ) return kind == FQT_BHQ ? FQT_EUNSUPPORTED : FQT_EINVAL;
+  if (N > 0 && (!dH || (!q_b2->codes && !q_b2->codes_f16) || !q_b2->inv_s || !q_b2->zero))
+    return FQT_EINVAL;
+  if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
+  if (N > 0 && q_b1 && ((!q_b1->codes && !q_b1->codes_f16) || !q_b1->inv_s || !q_b1->zero))
+    return FQT_EINVAL;
+  if (!(C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048))
+    return FQT_EUNSUPPORTED;
+  if (N / rows_per_sample > ((int64_t)1 << 20) || rows_per_sample > (1 << 30))
+    return FQT_EUNSUPPORTED;
+  if (!aligned(dH, 16) || !aligned(q_b2->codes, 16) || !aligned(q_b2->codes_f16, 16) ||
+      (q_b1 && (!aligned(q_b1->codes, 16) || !aligned(q_b1->codes_f16, 16))))
+    return FQT_EINVAL;
+  fqt_status s =
+      check_ws(workspace, ws_bytes, kGemmOffset + sample_pass_bytes(N, C, rows_per_sample));
+  if (s != FQT_OK) return s;
+  q_b2->rows = N;
+  q_b2->cols = C;
+  q_b2->bits = bits;
+  q_b2->kind = FQT_PSQ;
+  q_b2->block = 0;
+  q_b2->rows_per_sample = (int32_t)rows_per_sample;
+  if (q_b1) {
+    q_b1->rows = N;
+    q_b1->cols = C;
+    q_b1->bits = 8;
+    q_b1->kind = FQT_PTQ;
+    q_b1->block = 0;
+    q_b1->rows_per_sample = 1;
+  }
+  if (N == 0) return FQT_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  char *w = static_cast<char *>(workspace);
+  QuantArgs a;
+  memset(&a, 0, sizeof(a));
+  a.h = dH;
+  a.N = N;
+  a.C = (int)C;
+  a.kind = FQT_PSQ;
+  a.bits = bits;
+  a.block = 1;
+  a.key0 = (uint32_t)seed;
+  a.key1 = (uint32_t)(seed >> 32);
+  for (int r = 0; r < 10; ++r) {  // Philox4x32-10 round keys (Weyl sequence)
+    a.round_keys[2 * r] = a.key0 + (uint32_t)r * 0x9E3779B9u;
+    a.round_keys[2 * r + 1] = a.key1 + (uint32_t)r * 0xBB67AE85u;
+  }
+  a.c2 = q_b2->codes;
+  a.f2 = q_b2->codes_f16;
+  a.inv2 = q_b2->inv_s;
+  a.zero2 = q_b2->zero;
+  a.rsum2 = q_b2->row_sum;
+  a.csum2 = q_b1 ? nullptr : q_b2->col_sum;
+  if (q_b1) {
+    a.c1 = q_b1->codes;
+    a.f1 = q_b1->codes_f16;
+    a.inv1 = q_b1->inv_s;
+    a.zero1 = q_b1->zero;
+    a.rsum1 = q_b1->row_sum;
+    a.csum1 = q_b1->col_sum;
+  }
+  a.status = reinterpret_cast<int *>(w);
+  return launch_sample_passes(a, dtype == FQT_BF16, rows_per_sample, device_sm_count(),
+                              w + kGemmOffset, reinterpret_cast<float2 *>(w + kRangeOffset), st);
 }
 
 fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
@@ -241,12 +322,14 @@ fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
   q_b2->bits = bits;
   q_b2->kind = kind;
   q_b2->block = block;
+  q_b2->rows_per_sample = 1;
   if (q_b1) {
     q_b1->rows = N;
     q_b1->cols = C;
     q_b1->bits = 8;
     q_b1->kind = FQT_PTQ;
     q_b1->block = 0;
+    q_b1->rows_per_sample = 1;
   }
   if (N == 0) return FQT_OK;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

@@ -70,6 +70,9 @@ bool bhq_pass_supported(int C, int block, bool bf16);
 size_t bhq_pass_bytes(int64_t N, int64_t C);
 fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch,
                              float2 *part, cudaStream_t st);
+size_t sample_pass_bytes(int64_t N, int64_t C, int64_t rows_per_sample);
+fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample, int num_sms,
+                                void *scratch, float2 *part, cudaStream_t st);
 fqt_status launch_shift(QuantArgs &a, bool bf16, int num_sms, cudaStream_t st);
 cudaError_t launch_bhq_offsets(const float *zero, const int32_t *rsum,
                                const int32_t *lead, float *hz, float *hr, int64_t N,

@@ -1245,10 +1245,15 @@ __device__ __forceinline__ void load_two_octs(const T *row, int c_a, int c_b, fl
   }
 }
 
-template <typename T, int LPR>
+// SAMPLES: the per-sample PSQ of fqt_quantize_grad_samples instead of BHQ:
+// v = s_i (h - z_i) with the scalars of sample i = row / rows_per_sample
+// (srec: s, z, inv_s, zero per sample), written per row as well.
+template <typename T, int LPR, bool SAMPLES = false>
 __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
                                                    const BhqBlock *__restrict__ bst,
-                                                   const float *__restrict__ wsum, int lg_nb) {
+                                                   const float *__restrict__ wsum, int lg_nb,
+                                                   const float4 *__restrict__ srec = nullptr,
+                                                   int rows_per_sample = 1) {
   constexpr int RS = 32 / LPR, SLAB = 16 * LPR;
   __shared__ float2 red[8];
   __shared__ int redi[8];
@@ -1336,7 +1341,7 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
         const int rr = sub;
         if (rr < rows) {
           load_two_octs(h + (row0 + rr) * C, ca, cb, xn);
-          zn = a.zero2[row0 + rr];
+          if (!SAMPLES) zn = a.zero2[row0 + rr];
         }
       }
 #pragma unroll 1
@@ -1349,21 +1354,33 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
         const float zr = zn;
         if (rr + RS < rows) {
           load_two_octs(h + (row0 + rr + RS) * C, ca, cb, xn);
-          zn = a.zero2[row0 + rr + RS];
+          if (!SAMPLES) zn = a.zero2[row0 + rr + RS];
         }
         uint32_t acc1 = 0u, acc2 = 0u;
         if (valid) {
           const int64_t row = row0 + rr;
-          const int64_t blk = row >> lg_nb;
-          if (blk != cur_blk) {  // a new block: its w_j and scalars
-            const BhqBlock bs = bst[blk];
-            p_lead = __float_as_int(bs.p);
-            sk_l = bs.s1;
-            sk_o = bs.s2;
-            ck_l = bs.rho - 1.0f;
-            ck_o = bs.rho;
-            load_two_octs(wsum + blk * (int64_t)C, ca, cb, w);
+          const int64_t blk = SAMPLES ? row / rows_per_sample : row >> lg_nb;
+          if (blk != cur_blk) {  // a new block (sample): its w_j and scalars
+            if constexpr (SAMPLES) {
+              const float4 sr = srec[blk];  // s, z, inv_s, zero of the sample
+              sk_l = sr.x;
+              ck_l = sr.y;
+              sk_o = sr.z;
+              ck_o = sr.w;
+            } else {
+              const BhqBlock bs = bst[blk];
+              p_lead = __float_as_int(bs.p);
+              sk_l = bs.s1;
+              sk_o = bs.s2;
+              ck_l = bs.rho - 1.0f;
+              ck_o = bs.rho;
+              load_two_octs(wsum + blk * (int64_t)C, ca, cb, w);
+            }
             cur_blk = blk;
+          }
+          if (SAMPLES && o == 0 && c0 == 0) {
+            a.inv2[row] = sk_o;
+            a.zero2[row] = ck_o;
           }
           const bool lead = (int)(row & nbm) == p_lead;
           const float sk = lead ? sk_l : sk_o;
@@ -1398,8 +1415,10 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
           acc2 = 0u - 16u * kSrBits;
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            const float t = fmaf(-ck, w[j], __fmul_rn(sk, x[j]));
-            b[j] = sr_bits(fminf(__fsub_rn(t, zr), fB2), sr_u(j < 8 ? ua : ub, j & 7));
+            // BHQ: t - z'; per-sample PSQ: s (h - z) with the sample's s, z (Sec. 4.1)
+            const float v = SAMPLES ? __fmul_rn(__fsub_rn(x[j], ck_l), sk_l)
+                                    : __fsub_rn(fmaf(-ck, w[j], __fmul_rn(sk, x[j])), zr);
+            b[j] = sr_bits(fminf(v, fB2), sr_u(j < 8 ? ua : ub, j & 7));
             acc2 += b[j];
             if (!has_b1) cs[j] += b[j];
           }
@@ -1479,8 +1498,178 @@ static cudaError_t launch_codes(const QuantArgs &a, const BhqBlock *bst, const f
   const int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  kern<<<(int)grid, 256, smem, st>>>(a, bst, wsum, lg_nb);
+  kern<<<(int)grid, 256, smem, st>>>(a, bst, wsum, lg_nb, nullptr, 1);
   return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Per-sample PSQ (fqt_quantize_grad_samples; Sec. 4.1 with a sample = R
+// consecutive rows of dH, an image's output pixels): k_sample_part takes the
+// (min, max) of chunks of kSampleChunk rows' worth of entries inside one
+// sample; k_sample_finish reduces each sample's chunks to s = B / R(h_i),
+// z = min h_i (affine_scale, as the row quantizer), 1 / s and s z, and leaves
+// per-CTA (min, max) of the whole tensor (the range of Q_b1).  The code pass
+// (k_bhq_codes, SAMPLES) then rounds and packs.
+// ---------------------------------------------------------------------------
+constexpr int kSampleChunkElems = 16384;
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_sample_part(const QuantArgs a, int64_t sample_elems,
+                                                     int chunks_per_sample, float2 *cpart) {
+  __shared__ float2 red[8];
+  __shared__ int redi[8];
+  const int64_t ch = blockIdx.x;
+  const int64_t smp = ch / chunks_per_sample;
+  const int64_t e0 = smp * sample_elems + (ch - smp * chunks_per_sample) * kSampleChunkElems;
+  const int64_t e1 = min(smp * sample_elems + sample_elems, e0 + kSampleChunkElems);
+  const T *h = reinterpret_cast<const T *>(a.h);
+  float mn = INFINITY, mx = -INFINITY, nanacc = 0.0f;
+  for (int64_t e = e0 + (int64_t)threadIdx.x * 8; e < e1; e += (int64_t)blockDim.x * 8) {
+    float x[8];
+    load_oct(h + e, x);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      mn = fminf(mn, x[j]);
+      mx = fmaxf(mx, x[j]);
+      nanacc = fmaf(x[j], 0.0f, nanacc);
+    }
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    nanacc += __shfl_xor_sync(0xffffffffu, nanacc, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(mn, mx);
+    redi[warp] = isnan(nanacc) ? 1 : 0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int bad = 0;
+    for (int i = 0; i < 8; ++i) {
+      mn = fminf(mn, red[i].x);
+      mx = fmaxf(mx, red[i].y);
+      bad |= redi[i];
+    }
+    cpart[ch] = bad ? make_float2(NAN, NAN) : make_float2(mn, mx);
+  }
+}
+
+__global__ void __launch_bounds__(256) k_sample_finish(const QuantArgs a, int64_t nsamples,
+                                                       int chunks_per_sample,
+                                                       const float2 *cpart, float4 *srec,
+                                                       float2 *part) {
+  __shared__ float2 red[8];
+  __shared__ int redi[8];
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const uint32_t B = (1u << a.bits) - 1u;
+  float mn = INFINITY, mx = -INFINITY;
+  int bad = 0;
+  if (i < nsamples) {
+    for (int k = 0; k < chunks_per_sample; ++k) {
+      const float2 p = cpart[i * chunks_per_sample + k];
+      bad |= isnan(p.x);
+      mn = fminf(mn, p.x);
+      mx = fmaxf(mx, p.y);
+    }
+    const float s = affine_scale(mn, mx, B);
+    srec[i] = make_float4(s, mn, __fdiv_rn(1.0f, s), __fmul_rn(s, mn));
+  }
+  // the CTA's (min, max) of the whole tensor, for Q_b1
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, off));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    bad |= __shfl_xor_sync(0xffffffffu, bad, off);
+  }
+  if (lane == 0) {
+    red[warp] = make_float2(mn, mx);
+    redi[warp] = bad;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < 8; ++w) {
+      mn = fminf(mn, red[w].x);
+      mx = fmaxf(mx, red[w].y);
+      bad |= redi[w];
+    }
+    mn = fminf(mn, red[0].x);
+    mx = fmaxf(mx, red[0].y);
+    bad |= redi[0];
+    part[blockIdx.x] = bad ? make_float2(NAN, NAN) : make_float2(mn, mx);
+  }
+  // the code pass accumulates column sums into these
+  for (int64_t k = i; k < a.C; k += (int64_t)gridDim.x * blockDim.x) {
+    if (a.csum1) a.csum1[k] = 0;
+    if (a.csum2) a.csum2[k] = 0;
+  }
+}
+
+// Workspace bytes of the per-sample quantizer: chunk partials and records.
+size_t sample_pass_bytes(int64_t N, int64_t C, int64_t rows_per_sample) {
+  if (rows_per_sample < 1) return 0;
+  const int64_t ns = N / rows_per_sample;
+  const int64_t cps = (rows_per_sample * C + kSampleChunkElems - 1) / kSampleChunkElems;
+  return (size_t)(ns * cps) * sizeof(float2) + (size_t)ns * sizeof(float4) + 512;
+}
+
+// The per-sample PSQ with Q_b1: rows of C in {64, 128, 256 t} columns
+// (t = 1, 2, 4, 8), N a multiple of rows_per_sample, at most 2^20 samples.
+fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample, int num_sms,
+                                void *scratch, float2 *part, cudaStream_t st) {
+  const int C = a.C;
+  if (!(C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048))
+    return FQT_EUNSUPPORTED;
+  const int64_t ns = a.N / rows_per_sample;
+  if (ns > ((int64_t)1 << 20)) return FQT_EUNSUPPORTED;
+  const int64_t se = rows_per_sample * C;
+  const int cps = (int)((se + kSampleChunkElems - 1) / kSampleChunkElems);
+  float2 *cpart = static_cast<float2 *>(scratch);
+  float4 *srec = reinterpret_cast<float4 *>(
+      (reinterpret_cast<uintptr_t>(cpart + ns * cps) + 255) & ~(uintptr_t)255);
+  if (bf16)
+    k_sample_part<__nv_bfloat16><<<(unsigned)(ns * cps), 256, 0, st>>>(a, se, cps, cpart);
+  else
+    k_sample_part<float><<<(unsigned)(ns * cps), 256, 0, st>>>(a, se, cps, cpart);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "sample statistics launch");
+  const int fin = (int)((ns + 255) / 256);
+  k_sample_finish<<<fin, 256, 0, st>>>(a, ns, cps, cpart, srec, part);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "sample scalars launch");
+  QuantArgs a2 = a;
+  a2.part = part;
+  a2.npart = fin;
+  const int lpr = C == 64 ? 4 : C == 128 ? 8 : C == 256 ? 16 : 32;
+  const int R = (int)rows_per_sample;
+#define FQT_SC(TT, L)                                                                        \
+  {                                                                                          \
+    auto kern = k_bhq_codes<TT, L, true>;                                                    \
+    const size_t smem = sizeof(int) * (size_t)C;                                             \
+    int per_sm = 0;                                                                          \
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);             \
+    if (e == cudaSuccess) {                                                                  \
+      const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;                             \
+      int64_t grid = (nchunks + 7) / 8;                                                      \
+      const int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);                     \
+      if (grid > cap) grid = cap;                                                            \
+      if (grid < 1) grid = 1;                                                                \
+      kern<<<(int)grid, 256, smem, st>>>(a2, nullptr, nullptr, 0, srec, R);                  \
+      e = cudaGetLastError();                                                                \
+    }                                                                                        \
+  }
+  if (!bf16) {
+    if (lpr == 4) FQT_SC(float, 4) else if (lpr == 8) FQT_SC(float, 8)
+    else if (lpr == 16) FQT_SC(float, 16) else FQT_SC(float, 32)
+  } else {
+    if (lpr == 4) FQT_SC(__nv_bfloat16, 4) else if (lpr == 8) FQT_SC(__nv_bfloat16, 8)
+    else if (lpr == 16) FQT_SC(__nv_bfloat16, 16) else FQT_SC(__nv_bfloat16, 32)
+  }
+#undef FQT_SC
+  return cuda_fail(e, "sample code pass launch");
 }
 
 // The two-pass BHQ quantizer takes fixed blocks of 4, 8 or 16 rows and rows

@@ -35,7 +35,7 @@ class FqtError(RuntimeError):
 class _QT(ctypes.Structure):
     _fields_ = [("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
                 ("bits", ctypes.c_int32), ("kind", ctypes.c_int32),
-                ("block", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("block", ctypes.c_int32), ("rows_per_sample", ctypes.c_int32),
                 ("codes", ctypes.c_void_p), ("inv_s", ctypes.c_void_p),
                 ("zero", ctypes.c_void_p), ("row_sum", ctypes.c_void_p),
                 ("col_sum", ctypes.c_void_p), ("lead", ctypes.c_void_p),
@@ -77,6 +77,9 @@ def load(build_if_missing: bool = True):
         lib.fqt_quantize_grad.argtypes = [P, i32, i64, i64, i32, i32, i32, u64,
                                           QP, QP, P, sz, P]
         lib.fqt_quantize_grad.restype = i32
+        lib.fqt_quantize_grad_samples.argtypes = [P, i32, i64, i64, i64, i32, i32, u64,
+                                                  QP, QP, P, sz, P]
+        lib.fqt_quantize_grad_samples.restype = i32
         lib.fqt_linear_backward.argtypes = [QP, QP, QP, QP, P, P, P, sz, P]
         lib.fqt_linear_backward.restype = i32
         lib.fqt_linear_forward.argtypes = [QP, QP, P, P, sz, P]
@@ -186,6 +189,7 @@ class QTensor:
     shift_col_sum: Optional[torch.Tensor] = None
     shift_scale: Optional[torch.Tensor] = None
     conv: Optional[tuple] = None   # implicit im2col operand: (n, h, w, c, kh, kw, pad, 0)
+    rows_per_sample: int = 1       # rows of dH per sample (quantize_grad_samples)
     logical: Optional[tuple] = None  # (rows, cols) of that im2col matrix
 
     @property
@@ -233,7 +237,7 @@ class QTensor:
     def c_struct(self) -> _QT:
         rows, cols = self.shape
         p = lambda t: t.data_ptr() if t is not None else None
-        return _QT(rows, cols, self.bits, self.kind, self.block, 0,
+        return _QT(rows, cols, self.bits, self.kind, self.block, self.rows_per_sample,
                    p(self.codes), self.inv_s.data_ptr(), self.zero.data_ptr(),
                    p(self.row_sum), p(self.col_sum), p(self.lead), p(self.codes16),
                    p(self.hz), p(self.hr), p(self.perm), p(self.gstart), p(self.gsize),
@@ -358,6 +362,35 @@ def quantize_grad(dH: torch.Tensor, kind: int, bits: int, block: int = 0,
                                ws.ptr, ws.nbytes, _stream(stream))
     _check(st, "fqt_quantize_grad")
     q_b2.kind, q_b2.bits, q_b2.block = kind, bits, block if kind == BHQ else 0
+    if with_b1:
+        q_b1.kind, q_b1.bits, q_b1.block = PTQ, 8, 0
+    return q_b2, (q_b1 if with_b1 else None)
+
+
+def quantize_grad_samples(dH: torch.Tensor, rows_per_sample: int, kind: int, bits: int,
+                          seed: int = 0, with_b1: bool = True, ws: Workspace = None,
+                          q_b2: QTensor = None, q_b1: QTensor = None, stream=None):
+    """(Q_b2, Q_b1) with one sample per `rows_per_sample` rows of dH (an
+    image's output pixels; Sec. 4.1): fqt_quantize_grad_samples."""
+    lib = load()
+    dH = dH.contiguous()
+    N, C = dH.shape
+    ws = ws or Workspace(N, C, 16, device=dH.device)
+    if q_b2 is None:
+        q_b2 = QTensor.empty(N, C, kind if kind != PTQ else PTQ, bits, 0, True,
+                             not with_b1, dH.device)
+    if with_b1 and q_b1 is None:
+        q_b1 = QTensor.empty(N, C, PTQ, 8, 0, False, True, dH.device)
+    s2 = q_b2.c_struct()
+    s1 = q_b1.c_struct() if with_b1 else None
+    st = lib.fqt_quantize_grad_samples(_ptr(dH), _dtype_code(dH), N, C, rows_per_sample, kind,
+                                       bits, ctypes.c_uint64(seed & (2 ** 64 - 1)),
+                                       ctypes.byref(s2),
+                                       ctypes.byref(s1) if s1 is not None else None,
+                                       ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "fqt_quantize_grad_samples")
+    q_b2.kind, q_b2.bits, q_b2.block = kind, bits, 0
+    q_b2.rows_per_sample = rows_per_sample
     if with_b1:
         q_b1.kind, q_b1.bits, q_b1.block = PTQ, 8, 0
     return q_b2, (q_b1 if with_b1 else None)

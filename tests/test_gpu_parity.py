@@ -907,6 +907,73 @@ def test_grad_x_several_chunks_and_tiles_per_cta(kind, bits):
     assert grad_rel_err(gx[rows], ref_x) <= GRAD_TOL
 
 
+# --------------------------------------------------------------------------
+# Per-image samples (Sec. 4.1: a sample is one input's gradient)
+# --------------------------------------------------------------------------
+SAMPLE_CASES = [  # rows N, C, rows per sample, bits, dtype
+    (2048, 64, 1024, 5, "f32"), (2048, 64, 1024, 8, "f32"), (3136 * 2, 256, 3136, 5, "f32"),
+    (196 * 4, 1024, 196, 5, "bf16"), (49 * 3, 2048, 49, 4, "f32"), (600, 128, 1, 5, "f32"),
+    (512, 512, 128, 8, "bf16")]
+
+
+@pytest.mark.parametrize("N,C,R,bits,dtype", SAMPLE_CASES)
+def test_per_sample_psq_matches_oracle(N, C, R, bits, dtype):
+    g = wl.rng(N + C + R)
+    dH = wl.random_grad(g, N, C, sigma=1.5, outlier_frac=0.05)
+    if dtype == "bf16":
+        dH = wl.to_bf16_values(dH)
+    q2, q1 = fqt.quantize_grad_samples(to_dev(dH, dtype), R, orc.PSQ, bits, seed=21)
+    torch.cuda.synchronize()
+    ref = orc.quantize_grad_samples(dH, R, orc.PSQ, bits, 0, seed=21)
+    h2 = q2.to_numpy()
+    assert np.array_equal(h2["codes"], ref["codes"])
+    assert np.array_equal(h2["inv_s"], ref["inv_s_rows"])
+    assert np.array_equal(h2["zero"], ref["zero_rows"])
+    assert np.array_equal(h2["row_sum"], h2["codes"].astype(np.int64).sum(1))
+    _check_b1(q1, dH, 21)
+    assert q2.c_struct().rows_per_sample == R
+
+
+def test_one_row_samples_equal_the_row_quantizer_on_the_gpu():
+    """rows_per_sample = 1 (the per-sample code pass) against quantize_grad's
+    PSQ (the staged row kernel): the same codes and metadata bit for bit."""
+    L = wl.config(1, batch=1)[0]
+    a2, a1 = fqt.quantize_grad_samples(to_dev(L.dH), 1, orc.PSQ, 5, seed=8)
+    b2, b1 = fqt.quantize_grad(to_dev(L.dH), orc.PSQ, 5, 0, 8)
+    for x, y in ((a2, b2), (a1, b1)):
+        hx, hy = x.to_numpy(), y.to_numpy()
+        for k in ("codes", "inv_s", "zero", "col_sum"):
+            if hx.get(k) is not None and hy.get(k) is not None:
+                assert np.array_equal(hx[k], hy[k]), k
+
+
+def test_per_sample_backward_matches_oracle():
+    """grad_X and grad_W of the ResNet-18 conv layer at batch 2 with per-image
+    PSQ-5 (1024 rows per image): the PSQ epilogue reads the repeated
+    per-row scalars."""
+    L = wl.config(1, batch=2)[0]
+    qx = fqt.quantize_act(to_dev(L.X), 8)
+    qw = fqt.quantize_weight(to_dev(L.W), 8)
+    q2, q1 = fqt.quantize_grad_samples(to_dev(L.dH), 1024, orc.PSQ, 5, seed=4)
+    gx, gw = fqt.linear_backward(q2, q1, qx, qw)
+    torch.cuda.synchronize()
+    ref = orc.quantize_grad_samples(L.dH, 1024, orc.PSQ, 5, 0, seed=4)
+    ref["codes"] = q2.to_numpy()["codes"]
+    rx = orc.matmul(orc.dequant_samples(ref), orc.dequant(qw.to_numpy()))
+    assert grad_rel_err(gx.cpu().numpy(), rx) <= GRAD_TOL
+    assert grad_rel_err(gw.cpu().numpy(), orc.grad_w(q1.to_numpy(), qx.to_numpy())) <= GRAD_TOL
+
+
+def test_per_sample_refusals():
+    dH = torch.zeros((100, 64), device="cuda")
+    with pytest.raises(fqt.FqtError) as e:
+        fqt.quantize_grad_samples(dH, 30, orc.PSQ, 5)  # 100 rows are not whole samples
+    assert e.value.status == 1
+    with pytest.raises(fqt.FqtError) as e:
+        fqt.quantize_grad_samples(dH, 10, orc.BHQ, 5)
+    assert e.value.status == 2
+
+
 def test_bhq_code_agreement_pooled():
     """The >= 99.99% BHQ code agreement over every case this module compared
     (cases below AGREE_MIN codes cannot show a 1e-4 rate on their own)."""
