@@ -243,6 +243,29 @@ FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,
                                size_t ws_bytes, void *stream);
 
 /*
+ * grad_X of a stride-1 k x k convolution directly in NHWC (n x h x w x cin,
+ * fp32): col2im of Q_b2(dH) W~ (Eq. 6 for a conv lowered to im2col rows,
+ * Sec. 2.1) fused into the contraction, computed as the transposed
+ * convolution dX[p] = sum over taps t of Q_b2(dH)[o(p, t)] W~[:, t, :]
+ * (o(p, t) the output pixel tap t of input pixel p reads; taps reading
+ * outside the image add nothing).  q_b2: the dH rows of the conv's output
+ * pixels (n h w x cout, row order (n, y, x)), PTQ (fqt_quantize_grad) or PSQ
+ * with one sample per image (fqt_quantize_grad_samples with rows_per_sample
+ * = h w): the scale must be the same for all pixels of an image so that it
+ * factors out of the sum over taps.  codes_f16, row_sum, inv_s, zero.
+ * qw: W~ from fqt_quantize_weight on the im2col weight cout x (k k cin)
+ * (columns (ky, kx, c_in)), codes_f16 and col_sum.  Needs k = 3, pad = 1,
+ * h, w >= 2, w <= 128, cin % 32 == 0, cout % 64 == 0 and one exact chunk
+ * (9 cout <= 2^(26 - b - bw)); else FQT_EUNSUPPORTED.  `workspace`: at least
+ * fqt_conv_grad_x_workspace_size(cin) bytes (status word and tables).
+ */
+FQT_API size_t fqt_conv_grad_x_workspace_size(int64_t cin);
+FQT_API fqt_status fqt_conv_grad_x_nhwc(const fqt_qtensor *q_b2, const fqt_qtensor *qw,
+                                        int64_t n, int64_t h, int64_t w, int64_t cin, int k,
+                                        int pad, float *grad_X, void *workspace,
+                                        size_t ws_bytes, void *stream);
+
+/*
  * The quantized forward of the layer (Sec. 2.1, Eq. 3): H = X~ W~^T, the
  * product of the dequantized 8-bit PTQ operands, N x C fp32 row-major.  The
  * integer product of the codes is exact (fp16 carriers on the tensor cores,

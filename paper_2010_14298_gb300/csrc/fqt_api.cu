@@ -503,6 +503,15 @@ fqt_status fqt_debug_mma_peak(int kind, int64_t iters, double *ops_out, void *wo
                         reinterpret_cast<cudaStream_t>(stream));
 }
 
+size_t fqt_conv_grad_x_workspace_size(int64_t cin) { return conv_grad_x_ws_bytes(cin); }
+
+fqt_status fqt_conv_grad_x_nhwc(const fqt_qtensor *q_b2, const fqt_qtensor *qw, int64_t n,
+                                int64_t h, int64_t w, int64_t cin, int k, int pad,
+                                float *grad_X, void *workspace, size_t ws_bytes, void *stream) {
+  return conv_grad_x_nhwc(q_b2, qw, n, h, w, cin, k, pad, grad_X, workspace, ws_bytes,
+                          reinterpret_cast<cudaStream_t>(stream));
+}
+
 const char *fqt_last_cuda_error(void) { return g_last_error; }
 
 const char *fqt_status_string(fqt_status status) {

@@ -3250,3 +3250,406 @@ fqt_status debug_mma_peak(int kind, int64_t iters, double *ops_out, void *ws, si
 }
 
 }  // namespace fqt
+
+namespace fqt {
+
+// ---------------------------------------------------------------------------
+// grad_X of a stride-1 k x k conv in NHWC, col2im fused (Sec. 2.1: a conv is a
+// linear layer on im2col rows; grad_X is summed back over the taps): the
+// transposed convolution dX[p, j] = sum over taps t and output channels c of
+// Q_b2(dH)[o(p, t), c] W~[c, t, j], o(p, t) the output pixel that tap t of
+// input pixel p reads (out of the image: no term).  It needs the scale of
+// Q_b2 to be the same for every output pixel of an image -- per tensor (PTQ)
+// or per image (fqt_quantize_grad_samples) -- so that it factors out of the
+// sum over taps.
+//
+// Contraction: M = C_in (tiles of 128), N = input pixels (a tile is r whole
+// image rows of one image, row j in a slot of `slot` >= W pixels starting on
+// a 1024-byte boundary), K = k^2 C_out in blocks of 64 (tap, 64 channels).
+// A = W~ read MN-major at column offset tap C_in; B = the dH carriers read by
+// one 4-D box (64 channels x W pixels x 1 row x 1 image) per image row at the
+// tap's shifted output row and column (TMA fills rows and columns outside the
+// image with zero carriers, which add nothing).  Exact integer products in
+// fp32 (one exact chunk).
+//
+// Dequantization.  With a, w the centred codes, the image's offset
+// 2^(b-1) + z' = m + d and y = 2^(bw-1) + z_w, for the set T(p) of taps of
+// p that read a pixel of the image:
+//   V_pj = I_pj + y R_p + d U_T(j),  I_pj = P_pj + m CW_T(j),
+//   R_p = sum_{t in T(p)} (row_sum[o(p, t)] - C 2^(b-1) + C m),
+//   CW_T(j) = sum_{t in T} sum_c w_ctj,  U_T(j) = CW_T(j) + |T| C y,
+// and dX = inv_sw inv_s V.  For k = 3, pad 1 the sets T are the nine border
+// classes of p (top / middle / bottom row times left / middle / right
+// column); the class tables CW, U are formed once per call.
+// ---------------------------------------------------------------------------
+constexpr int kCvStages = 4;
+constexpr int kCvThreads = 320;  // TMA, MMA, two sets of four epilogue warps
+constexpr int kCvClasses = 9;
+
+struct ConvXArgs {
+  int n, h, w, cin, cout, k, pad;
+  int slot, rows;          // pixel slots per image row in a tile, image rows per tile
+  int tiles_per_img, m_tiles;
+  int64_t n_items;
+  int kb_total, cbs;       // K blocks (taps x channel blocks), channel blocks per tap
+  int og, ow;              // 2^(b-1) of Q_b2, of W~
+  const float *inv_s, *zero;  // Q_b2: per row (per image constant) or one entry
+  int per_tensor;
+  const int32_t *row_sum;  // Q_b2 row sums (codes), one per output pixel
+  const float *inv_sw, *zero_w;
+  const float *cw_cls;     // [9][cin] CW_T(j)
+  const float *u_cls;      // [9][cin] U_T(j)
+  float *out;              // NHWC n h w cin
+  int *status;
+};
+
+__device__ __forceinline__ int conv_class(int y, int x, int h, int w) {
+  const int cy = y == 0 ? 0 : (y == h - 1 ? 2 : 1);
+  const int cx = x == 0 ? 0 : (x == w - 1 ? 2 : 1);
+  return cy * 3 + cx;
+}
+
+// Class tables: CW_T(j) and U_T(j) for the nine border classes of a 3 x 3
+// stride-1 pad-1 conv (T = the taps whose output pixel exists).
+__global__ void k_conv_classes(const int32_t *__restrict__ col_sum_w, int cin, int cout,
+                               int ow, const float *zero_w, float *cw_cls, float *u_cls) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= cin) return;
+  const ff y = two_sum((float)ow, *zero_w);
+  for (int cls = 0; cls < kCvClasses; ++cls) {
+    const int cy = cls / 3, cx = cls % 3;
+    long long cw = 0;
+    int taps = 0;
+    for (int ky = 0; ky < 3; ++ky)
+      for (int kx = 0; kx < 3; ++kx) {
+        // top row (cy 0): the tap ky = 2 reads output row -1; bottom: ky = 0
+        if ((cy == 0 && ky == 2) || (cy == 2 && ky == 0)) continue;
+        if ((cx == 0 && kx == 2) || (cx == 2 && kx == 0)) continue;
+        cw += (long long)col_sum_w[(ky * 3 + kx) * cin + j] - (long long)cout * ow;
+        ++taps;
+      }
+    cw_cls[cls * cin + j] = (float)cw;
+    // U = CW + |T| C y, rounded once from float-float
+    const ff tcy = ff_mul({(float)(taps * cout), 0.0f}, y);
+    u_cls[cls * cin + j] = ff_round(ff_add(ff_from_int(cw), tcy));
+  }
+}
+
+__device__ __forceinline__ void conv_decode(const ConvXArgs &g, int64_t it, int &m0, int &img,
+                                            int &y0) {
+  const int64_t mt = it % g.m_tiles, pt = it / g.m_tiles;
+  m0 = (int)mt * BM;
+  img = (int)(pt / g.tiles_per_img);
+  y0 = (int)(pt - (int64_t)img * g.tiles_per_img) * g.rows;
+}
+
+__global__ void __launch_bounds__(kCvThreads, 1)
+    k_gradx_nhwc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                 const ConvXArgs g) {
+  extern __shared__ __align__(1024) uint8_t cv_raw[];
+  uint8_t *smem = cv_raw + ((1024u - (smem_u32(cv_raw) & 1023u)) & 1023u);
+  uint8_t *ops = smem;  // kCvStages x (A 16 KB, B 16 KB)
+  float *pbp = reinterpret_cast<float *>(ops + (size_t)kCvStages * 2 * kTileBytes);  // [2][128]
+  int *pcls = reinterpret_cast<int *>(pbp + 2 * 128);                                 // [2][128]
+  float *pcw = reinterpret_cast<float *>(pcls + 2 * 128);                  // [2][9][128]
+  float *pu = pcw + 2 * kCvClasses * 128;                                  // [2][9][128]
+  uint64_t *bars = reinterpret_cast<uint64_t *>(pu + 2 * kCvClasses * 128);
+  uint64_t *full = bars, *empty = bars + kCvStages, *accf = empty + kCvStages,
+           *acce = accf + 2, *drain = acce + 2;
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(drain + 1);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kCvStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&accf[i], 1);
+      mbar_init(&acce[i], 4);  // the four warps of the set
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(256u)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t b_bytes = (uint32_t)g.rows * (uint32_t)g.w * 128u;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0;
+      for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
+        int m0, img, y0;
+        conv_decode(g, it, m0, img, y0);
+        bool ok = true;
+        for (int kb = 0; kb < g.kb_total; ++kb) {
+          const int t = kb / g.cbs, cb = kb - t * g.cbs;
+          const int ky = t / g.k, kx = t - ky * g.k;
+          if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) { ok = false; break; }
+          mbar_expect_tx(&full[s], (uint32_t)kTileBytes + b_bytes);
+          uint8_t *sa = ops + (size_t)(2 * s) * kTileBytes;
+          uint8_t *sb = sa + kTileBytes;
+          // A: W~ columns tap t, c_in m0 .. m0 + 127 (two 64-wide MN atoms), 64 output channels
+          tma_load_2d(sa, &tmA, m0 + t * g.cin, cb * 64, &full[s]);
+          tma_load_2d(sa + kTileBytes / 2, &tmA, m0 + 64 + t * g.cin, cb * 64, &full[s]);
+          // B: per image row of the tile, the carriers of output row y + pad - ky at columns
+          // x + pad - kx (x = 0 .. w - 1)
+          for (int j = 0; j < g.rows; ++j)
+            tma_load_4d(sb + (size_t)j * g.slot * 128, &tmB, cb * 64, g.pad - kx,
+                        y0 + j + g.pad - ky, img, &full[s]);
+          if (++s == kCvStages) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) { *abort_flag = 1; break; }
+      }
+      if (*abort_flag) {
+        sleep_ns(200000);  // copies in flight land before the CTA exits
+      } else {
+        for (int i = 0; i < kCvStages; ++i) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) break;
+          if (++s == kCvStages) { s = 0; ph ^= 1u; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // -------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      int s = 0;
+      uint32_t ph = 0, aph = 0;
+      const uint32_t idesc = make_idesc(true, false);  // A MN-major, B K-major
+      int64_t local = 0;
+      for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
+        const int buf = (int)(local & 1);
+        if (!mbar_wait(&acce[buf], ((aph >> buf) & 1u) ^ 1u, g.status)) { *abort_flag = 1; break; }
+        tc_fence_after();
+        const uint32_t dt = tmem + (uint32_t)(buf * BN);
+        bool ok = true;
+        for (int kb = 0; kb < g.kb_total; ++kb) {
+          if (!mbar_wait(&full[s], ph, g.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a_addr = smem_u32(ops + (size_t)(2 * s) * kTileBytes);
+          const uint64_t da = sw128_desc_mn(a_addr, (uint32_t)(kTileBytes / 2), 1024);
+          const uint64_t db = sw128_desc(a_addr + (uint32_t)kTileBytes);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            umma_f16(dt, da + (2048u >> 4) * k, db + 2 * k, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit(&empty[s]);
+          if (++s == kCvStages) { s = 0; ph ^= 1u; }
+        }
+        umma_commit(&accf[buf]);
+        aph ^= 1u << buf;
+        if (!ok) { *abort_flag = 1; break; }
+      }
+      umma_commit(drain);  // every MMA has completed before TMEM is released
+      mbar_wait(drain, 0, g.status);
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue
+    // set s owns accumulator s and the tiles local = s, s + 2, ...; warp q
+    // of the set reads TMEM lanes 32 q .. 32 q + 31 (output channels)
+    const int ew = warp - 2, set = ew >> 2, q = warp & 3;
+    const int st = (ew & 3) * 32 + lane;  // 0 .. 127 within the set
+    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(set * BN);
+    float *bp = pbp + set * 128;
+    int *cls_s = pcls + set * 128;
+    float *cw_s = pcw + set * kCvClasses * 128;
+    float *u_s = pu + set * kCvClasses * 128;
+    const float inv_sw = *g.inv_sw, zw = *g.zero_w;
+    const ff yy = two_sum((float)g.ow, zw);
+    const int C = g.cout;
+    bool dead = false;
+    int cur_m0 = -1;
+    int64_t local = set;
+    for (;; local += 2) {
+      const int64_t it = (int64_t)blockIdx.x + local * (int64_t)gridDim.x;
+      if (it >= g.n_items) break;  // the same trip count in the set's four warps
+      dead = dead || *abort_flag;
+      int m0, img, y0;
+      conv_decode(g, it, m0, img, y0);
+      // per-image scalars of Q_b2 (one scale per image or per tensor)
+      const int64_t prow = (int64_t)img * g.h * g.w;
+      const float inv = g.per_tensor ? g.inv_s[0] : g.inv_s[prow];
+      const float z = g.per_tensor ? g.zero[0] : g.zero[prow];
+      const float sc = __fmul_rn(inv_sw, inv);
+      const ff xo = two_sum((float)g.og, z);
+      const float m = rintf(xo.h);
+      const float dd = ff_round(fast_two_sum(__fsub_rn(xo.h, m), xo.l));
+      const float Ad = __fmul_rn(sc, dd);
+      // the pixel terms of this tile: thread st takes pixel slot st
+      {
+        const int jr = st / g.slot, x = st - jr * g.slot, y = y0 + jr;
+        const bool pv = !dead && x < g.w && jr < g.rows && y < g.h;
+        float B = 0.0f;
+        int cl = -1;
+        if (pv) {
+          cl = conv_class(y, x, g.h, g.w);
+          long long R = 0;
+          for (int ky = 0; ky < 3; ++ky)
+            for (int kx = 0; kx < 3; ++kx) {
+              const int oy = y + g.pad - ky, ox = x + g.pad - kx;
+              if (oy < 0 || oy >= g.h || ox < 0 || ox >= g.w) continue;
+              R += (long long)__ldg(g.row_sum + prow + (int64_t)oy * g.w + ox) -
+                   (long long)C * g.og + (long long)C * (long long)m;
+            }
+          const ff Rf = ff_from_int(R);
+          B = __fmul_rn(sc, ff_round(ff_mul(Rf, yy)));
+        }
+        bp[st] = B;
+        cls_s[st] = cl;
+        if (m0 != cur_m0) {  // the class tables of this tile's 128 channels
+          const int j = m0 + st;
+          for (int c = 0; c < kCvClasses; ++c) {
+            cw_s[c * 128 + st] = j < g.cin ? __ldg(g.cw_cls + c * g.cin + j) : 0.0f;
+            u_s[c * 128 + st] = j < g.cin ? __ldg(g.u_cls + c * g.cin + j) : 0.0f;
+          }
+        }
+      }
+      cur_m0 = m0;
+      asm volatile("bar.sync %0, 128;" ::"r"(1 + set) : "memory");
+      const int64_t n_tile = local >> 1;  // this set's earlier tiles
+      bool got = false;
+      if (!dead) got = mbar_wait(&accf[set], (uint32_t)(n_tile & 1), g.status);
+      got = __all_sync(0xffffffffu, got);
+      if (!got) {
+        if (!dead) *abort_flag = 1;
+        dead = true;
+      }
+      if (!dead) {
+        tc_fence_after();
+        const int jl = q * 32 + lane, j = m0 + jl;
+        const bool jv = j < g.cin;
+#pragma unroll 1
+        for (int b = 0; b < BN / 32; ++b) {
+          uint32_t r[32];
+          tmem_ld32_nw(lane_base + (uint32_t)(b * 32), r);
+          tmem_wait_ld(r);
+          if (b == BN / 32 - 1) {  // the accumulator has been read in full
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce[set]);
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int c = b * 32 + i;
+            const int cl = cls_s[c];  // warp-uniform
+            if (cl < 0 || !jv) continue;
+            const float cw = cw_s[cl * 128 + jl], u = u_s[cl * 128 + jl];
+            const float I = __fmaf_rn(m, cw, __uint_as_float(r[i]));
+            const float v = __fmaf_rn(sc, I, __fmaf_rn(Ad, u, bp[c]));
+            const int jr = c / g.slot, x = c - jr * g.slot;
+            __stcs(g.out + ((prow + (int64_t)(y0 + jr) * g.w + x) * g.cin + j), v);
+          }
+        }
+      }
+      asm volatile("bar.sync %0, 128;" ::"r"(1 + set) : "memory");
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256u)
+                 : "memory");
+  }
+}
+
+static bool make_map_f16_rows(CUtensorMap *m, const void *base, uint64_t n, uint64_t h,
+                              uint64_t w, uint64_t c) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {c, w, h, n};
+  cuuint64_t strides[3] = {c * 2, w * c * 2, h * w * c * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)w, 1, 1};  // 64 channels of one image row
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(base), dims, strides,
+            box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t conv_grad_x_ws_bytes(int64_t cin) {
+  return kGemmOffset + 2 * (size_t)kCvClasses * (size_t)(cin > 0 ? cin : 0) * sizeof(float) + 256;
+}
+
+fqt_status conv_grad_x_nhwc(const fqt_qtensor *q2, const fqt_qtensor *qw, int64_t n, int64_t h,
+                            int64_t w, int64_t cin, int k, int pad, float *out, void *ws,
+                            size_t ws_bytes, cudaStream_t st) {
+  if (!q2 || !qw || !out || n <= 0 || h <= 0 || w <= 0 || cin <= 0) return FQT_EINVAL;
+  if (!q2->codes_f16 || !q2->row_sum || !q2->inv_s || !q2->zero || !qw->codes_f16 ||
+      !qw->col_sum || !qw->inv_s || !qw->zero)
+    return FQT_EINVAL;
+  if (k != 3 || pad != 1 || h < 2 || w < 2 || w > 128) return FQT_EUNSUPPORTED;
+  const int64_t cout = q2->cols;
+  if (q2->rows != n * h * w || qw->rows != cout || qw->cols != 9 * cin) return FQT_EINVAL;
+  if (cout % 64 || cin % 32) return FQT_EUNSUPPORTED;
+  const bool per_tensor = q2->kind == FQT_PTQ;
+  if (!per_tensor && !(q2->kind == FQT_PSQ && q2->rows_per_sample == h * w))
+    return FQT_EUNSUPPORTED;  // the scale must be constant over every image's pixels
+  if (qw->kind != FQT_PTQ || q2->conv[0] || qw->conv[0]) return FQT_EUNSUPPORTED;
+  if (9 * cout > (int64_t)exact_chunk_blocks(q2->bits, qw->bits) * BK) return FQT_EUNSUPPORTED;
+  if (!aligned16(q2->codes_f16) || !aligned16(qw->codes_f16) || !aligned16(out))
+    return FQT_EINVAL;
+  if (!ws || ((uintptr_t)ws & 255) || ws_bytes < conv_grad_x_ws_bytes(cin))
+    return FQT_EWORKSPACE;
+  char *wb = static_cast<char *>(ws);
+  float *cw_cls = reinterpret_cast<float *>(wb + kGemmOffset);
+  float *u_cls = cw_cls + kCvClasses * cin;
+  k_conv_classes<<<(unsigned)((cin + 127) / 128), 128, 0, st>>>(
+      qw->col_sum, (int)cin, (int)cout, 1 << (qw->bits - 1), qw->zero, cw_cls, u_cls);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "class tables launch");
+  CUtensorMap ta, tb;
+  bool ok = make_map_f16(&ta, qw->codes_f16, (uint64_t)(9 * cin), (uint64_t)cout, 64, BK);
+  ok = ok && make_map_f16_rows(&tb, q2->codes_f16, (uint64_t)n, (uint64_t)h, (uint64_t)w,
+                               (uint64_t)cout);
+  if (!ok) return cuda_fail(cudaErrorInvalidValue, "tensor map encode");
+  ConvXArgs g;
+  memset(&g, 0, sizeof(g));
+  g.n = (int)n;
+  g.h = (int)h;
+  g.w = (int)w;
+  g.cin = (int)cin;
+  g.cout = (int)cout;
+  g.k = k;
+  g.pad = pad;
+  g.slot = (int)((w + 7) / 8 * 8);
+  g.rows = (int)min((int64_t)(128 / g.slot), h);
+  g.tiles_per_img = (int)((h + g.rows - 1) / g.rows);
+  g.m_tiles = (int)((cin + BM - 1) / BM);
+  g.n_items = n * g.tiles_per_img * (int64_t)g.m_tiles;
+  g.cbs = (int)(cout / 64);
+  g.kb_total = 9 * g.cbs;
+  g.og = 1 << (q2->bits - 1);
+  g.ow = 1 << (qw->bits - 1);
+  g.inv_s = q2->inv_s;
+  g.zero = q2->zero;
+  g.per_tensor = per_tensor ? 1 : 0;
+  g.row_sum = q2->row_sum;
+  g.inv_sw = qw->inv_s;
+  g.zero_w = qw->zero;
+  g.cw_cls = cw_cls;
+  g.u_cls = u_cls;
+  g.out = out;
+  g.status = reinterpret_cast<int *>(ws);
+  const size_t smem = 1024 + (size_t)kCvStages * 2 * kTileBytes +
+                      (size_t)(2 * 128 * 2 + 2 * 2 * kCvClasses * 128) * 4 + 16 * 8 + 16;
+  e = cudaFuncSetAttribute(k_gradx_nhwc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "conv grad_X shared-memory attribute");
+  const int nsm = device_sm_count();
+  const int64_t grid = g.n_items < nsm ? g.n_items : nsm;
+  k_gradx_nhwc<<<(int)grid, kCvThreads, smem, st>>>(ta, tb, g);
+  return cuda_fail(cudaGetLastError(), "conv grad_X launch");
+}
+
+}  // namespace fqt

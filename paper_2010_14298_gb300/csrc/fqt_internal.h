@@ -102,6 +102,10 @@ fqt_status grad_w_fixed_scratch(const fqt_qtensor *qa, const fqt_qtensor *qx,
                                 float *grad_W, cudaStream_t st);
 fqt_status fixed_scratch_status(int **out);
 fqt_status debug_wait_timeout(void *ws, size_t ws_bytes, uint64_t limit_ns, cudaStream_t st);
+size_t conv_grad_x_ws_bytes(int64_t cin);
+fqt_status conv_grad_x_nhwc(const fqt_qtensor *q2, const fqt_qtensor *qw, int64_t n, int64_t h,
+                            int64_t w, int64_t cin, int k, int pad, float *out, void *ws,
+                            size_t ws_bytes, cudaStream_t st);
 fqt_status debug_mma_peak(int kind, int64_t iters, double *ops_out, void *ws, size_t ws_bytes,
                           cudaStream_t st);
 fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H, void *ws,

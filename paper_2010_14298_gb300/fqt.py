@@ -80,6 +80,10 @@ def load(build_if_missing: bool = True):
         lib.fqt_quantize_grad_samples.argtypes = [P, i32, i64, i64, i64, i32, i32, u64,
                                                   QP, QP, P, sz, P]
         lib.fqt_quantize_grad_samples.restype = i32
+        lib.fqt_conv_grad_x_workspace_size.argtypes = [i64]
+        lib.fqt_conv_grad_x_workspace_size.restype = sz
+        lib.fqt_conv_grad_x_nhwc.argtypes = [QP, QP, i64, i64, i64, i64, i32, i32, P, P, sz, P]
+        lib.fqt_conv_grad_x_nhwc.restype = i32
         lib.fqt_linear_backward.argtypes = [QP, QP, QP, QP, P, P, P, sz, P]
         lib.fqt_linear_backward.restype = i32
         lib.fqt_linear_forward.argtypes = [QP, QP, P, P, sz, P]
@@ -444,6 +448,28 @@ def linear_backward(q_b2: QTensor, q_b1: Optional[QTensor], qx: QTensor,
                                  _stream(stream))
     _check(st, "fqt_linear_backward")
     return gx, gw
+
+
+def conv_grad_x_nhwc(q_b2: QTensor, qw: QTensor, n: int, h: int, w: int, cin: int,
+                     k: int = 3, pad: int = 1, ws: Workspace = None,
+                     out: torch.Tensor = None, stream=None) -> torch.Tensor:
+    """grad_X of a stride-1 conv in NHWC with col2im fused into the contraction
+    (fqt_conv_grad_x_nhwc); q_b2 PTQ or per-image PSQ (quantize_grad_samples
+    with rows_per_sample = h w)."""
+    lib = load()
+    dev = q_b2.inv_s.device
+    if out is None:
+        out = torch.empty((n, h, w, cin), dtype=torch.float32, device=dev)
+    need = int(lib.fqt_conv_grad_x_workspace_size(cin))
+    if ws is None or ws.nbytes < need:
+        ws = Workspace(1, 16, 16, device=dev)
+        ws.nbytes = need
+        ws.buf = torch.zeros(need, dtype=torch.uint8, device=dev)
+    s2, sw = q_b2.c_struct(), qw.c_struct()
+    st = lib.fqt_conv_grad_x_nhwc(ctypes.byref(s2), ctypes.byref(sw), n, h, w, cin, k, pad,
+                                  _ptr(out), ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "fqt_conv_grad_x_nhwc")
+    return out
 
 
 def grad_w_fixed_scratch(q_b1: QTensor, qx: QTensor, out: torch.Tensor = None,
