@@ -706,6 +706,33 @@ def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
                              "quantize_act_conv_ms": pi[0], "grad_w_ms": pi[1],
                              "explicit_ms": {"quantize_act": per_base[0], "grad_w": per_base[4]},
                              "device_status": fqt.sync_status(ws)}
+    # per-image samples (Sec. 4.1) and grad_X in NHWC with col2im fused: the
+    # same layer (batch 128, 32 x 32, 64 -> 64 channels), PSQ-5 with one
+    # sample per image
+    q2p = fqt.QTensor.empty(N, C, fqt.PSQ, 5, 0, True, False, dev, u8=False)
+    q1p = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+    nimg, hh, wimg, cin = L2.x_nhwc.shape
+    outn = torch.empty((nimg, hh, wimg, cin), dtype=torch.float32, device=dev)
+    wsc = fqt.Workspace(1, 16, 16, device=dev)
+    wsc.nbytes = int(fqt.load().fqt_conv_grad_x_workspace_size(cin))
+    wsc.buf = torch.zeros(wsc.nbytes, dtype=torch.uint8, device=dev)
+    ps_ = time_graphs([
+        lambda: fqt.quantize_grad_samples(dH, hh * wimg, fqt.PSQ, 5, 3, ws=ws, q_b2=q2p,
+                                          q_b1=q1p),
+        lambda: fqt.conv_grad_x_nhwc(q2p, base.qw, nimg, hh, wimg, cin, ws=wsc, out=outn),
+        lambda: fqt.linear_backward(q2p, q1p, base.qx, base.qw, grad_x=True, grad_w=False, ws=ws,
+                                    out_x=base.gx)])
+    nb_out = nimg * hh * wimg * cin * 4
+    by_nhwc = N * C + C * D + nb_out + N * 4 + D * 4
+    ex["per_image_samples_and_fused_col2im"] = {
+        "quantizer": "Q_b2 = PSQ-5 with one sample per image (rows_per_sample = 1024), Q_b1 PTQ-8",
+        "quantize_grad_samples_ms": ps_[0],
+        "grad_x_nhwc_ms": ps_[1],
+        "grad_x_nhwc_GBs": by_nhwc / (ps_[1] * 1e-3) / 1e9,
+        "grad_x_nhwc_frac_of_hbm": by_nhwc / (ps_[1] * 1e-3) / 1e9 / hbm_peak,
+        "grad_x_im2col_ms": ps_[2],
+        "output_bytes": {"nhwc": nb_out, "im2col": N * D * 4},
+        "device_status": max(fqt.sync_status(ws), fqt.sync_status(wsc))}
     qxr = fqt.quantize_act(X, 8, row_sum=True)
     qwr = fqt.quantize_weight(W, 8, row_sum=True)
     H = torch.empty((N, C), dtype=torch.float32, device=dev)
@@ -715,7 +742,7 @@ def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
                      "TOPS": 2 * N * C * D / (pf[0] * 1e-3) / 1e12,
                      "GBs": fb / (pf[0] * 1e-3) / 1e9,
                      "frac_of_hbm": fb / (pf[0] * 1e-3) / 1e9 / hbm_peak}
-    del dH, X, W, ws, base, qa, qa1, qs, xn, box, qxr, qwr, H
+    del dH, X, W, ws, base, qa, qa1, qs, xn, box, qxr, qwr, H, q2p, q1p, outn, wsc
     torch.cuda.empty_cache()
 
     # the paper's own overhead shape (Sec. 4.3): dH of a conv with N = 128,

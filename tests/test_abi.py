@@ -192,3 +192,39 @@ def test_fixed_scratch_and_wait_test_refusals_without_gpu():
     assert lib.fqt_debug_wait_timeout(ctypes.c_void_p(p.value + 16), 256, 1000, None) == 6
     assert lib.fqt_debug_wait_timeout(p, 128, 1000, None) == 6
     del raw
+
+
+def test_sample_and_nhwc_refusals_without_gpu():
+    """fqt_quantize_grad_samples and fqt_conv_grad_x_nhwc refuse bad requests
+    before any CUDA call: rows that are not whole samples, BHQ samples, a
+    5 x 5 kernel, per-row scales."""
+    from paper_2010_14298_gb300 import fqt
+    lib = fqt.load()
+    raw, p = _aligned()
+    q = fqt._QT()
+    for name in ("codes_f16", "inv_s", "zero", "row_sum", "col_sum"):
+        setattr(q, name, p.value)
+    PSQ, BHQ = 1, 2
+    assert lib.fqt_quantize_grad_samples(p, 0, 100, 64, 30, PSQ, 5, 0, ctypes.byref(q), None, p,
+                                         1 << 16, None) == 1
+    assert lib.fqt_quantize_grad_samples(p, 0, 100, 64, 10, BHQ, 5, 0, ctypes.byref(q), None, p,
+                                         1 << 16, None) == 2
+    assert lib.fqt_quantize_grad_samples(p, 0, 100, 72, 10, PSQ, 5, 0, ctypes.byref(q), None, p,
+                                         1 << 16, None) == 2
+    q2 = fqt._QT()
+    q2.rows, q2.cols, q2.bits, q2.kind, q2.rows_per_sample = 2 * 8 * 8, 64, 5, PSQ, 64
+    qw = fqt._QT()
+    qw.rows, qw.cols, qw.bits, qw.kind = 64, 9 * 32, 8, 0
+    for s in (q2, qw):
+        for name in ("codes_f16", "inv_s", "zero", "row_sum", "col_sum"):
+            setattr(s, name, p.value)
+    out = p
+    assert lib.fqt_conv_grad_x_nhwc(ctypes.byref(q2), ctypes.byref(qw), 2, 8, 8, 32, 5, 2, out, p,
+                                     1 << 16, None) == 2
+    q2.rows_per_sample = 1  # per-row scales do not factor out of the taps
+    assert lib.fqt_conv_grad_x_nhwc(ctypes.byref(q2), ctypes.byref(qw), 2, 8, 8, 32, 3, 1, out, p,
+                                     1 << 16, None) == 2
+    q2.rows_per_sample = 64
+    assert lib.fqt_conv_grad_x_nhwc(ctypes.byref(q2), ctypes.byref(qw), 2, 8, 8, 32, 3, 1, out, p,
+                                     64, None) == 6  # workspace too small
+    del raw
