@@ -282,12 +282,31 @@ __device__ __forceinline__ ff ff_mul(ff x, ff y) {
 }
 
 // An integer (|v| < 2^53) as float-float, exactly for |v| < 2^48.
+// Conversions to and from 64-bit integers run on the FP64 pipe, which is
+// narrow on this GPU; for |v| < 2^47 the value is split as a 2^24 + b with
+// 0 <= b < 2^24 and |a| < 2^23, both exact in fp32 after 32-bit conversions,
+// and joined error-free (|a 2^24| >= 2^24 > b when a != 0).
 __device__ __forceinline__ ff ff_from_int(long long v) {
+  if ((unsigned long long)(v + (1LL << 47)) < (1ULL << 48)) {
+    const float a = __int2float_rn((int)(v >> 24));
+    const float b = __int2float_rn((int)(v & 0xFFFFFF));
+    return fast_two_sum(__fmul_rn(a, 16777216.0f), b);
+  }
   const float h = __ll2float_rn(v);
   return {h, __ll2float_rn(v - (long long)h)};
 }
 
 __device__ __forceinline__ float ff_round(ff x) { return __fadd_rn(x.h, x.l); }
+
+// An int64 to fp32 rounded to nearest (the value of a 64-bit conversion),
+// for |v| < 2^47 without the FP64 pipe: v = a 2^24 + b with a and b exact in
+// fp32, and one fused multiply-add rounds a 2^24 + b once.
+__device__ __forceinline__ float ll_to_float(long long v) {
+  if ((unsigned long long)(v + (1LL << 47)) < (1ULL << 48))
+    return __fmaf_rn(__int2float_rn((int)(v >> 24)), 16777216.0f,
+                     __int2float_rn((int)(v & 0xFFFFFF)));
+  return __ll2float_rn(v);
+}
 
 // An int32 as float-float, exactly, with 32-bit conversions only.
 __device__ __forceinline__ ff ff_from_i32s(int v) {

@@ -41,12 +41,15 @@ constexpr int kPartialEpiWarps = 8;
 // per-tile parameter loader (warp 3 idles); the epilogue warps follow in
 // sets of four (one per TMEM lane quadrant) that take the tiles in turn.
 // The epilogue's arithmetic comes in three forms (FORM):
-//   0  int64 integer parts for every tile (several exact chunks, large C);
-//   1  the fp32 form for tiles whose row offsets allow it, int64 for the
+//   0  int32 integer parts (several exact chunks, or the fp32 form's offset
+//      bound below 0);
+//   1  the fp32 form for tiles whose row offsets allow it, int32 for the
 //      others, in the same epilogue (the fp32 form's offset bound is small);
-//   2  the fp32 form only: the rare tiles outside it are stored raw and
-//      finished by the CTA after its last tile (gradx_raw_fix).
-// FORM 2 has four sets: without the int64 path, warpgroup 0 can hand
+//   2  the fp32 form only.
+// In every form the rare tiles outside it (a row offset m beyond the int32
+// form's, or the fp32 form's in FORM 2) are stored raw and finished by the
+// CTA after its last tile (gradx_raw_fix).
+// FORM 2 has four sets: without the int32 path, warpgroup 0 can hand
 // registers to the epilogue warpgroups (setmaxnreg) and 104 per thread
 // suffice (96 for blocks of up to 16 rows, whose parameter loader keeps 80); tiles with a long reduction use three of the sets (g.sets), so
 // that the tensor cores fill a fourth accumulator while three are drained.
@@ -124,6 +127,7 @@ struct GemmArgs {
                                // group size of every stored row of Q_b2
   float raw_mmax;              // NB = 0: largest |m| of a row finished here
   float flt_mmax;              // largest |m| of a tile for the fp32 form
+  float i32_mmax;              // largest |m| of a tile for the int32 form
   const int32_t *col_sum_w;    // W~ column sums over C
   const float *inv_sw, *zero_w;
   float *out;                  // grad_X (N x M row-major) for MODE_GRADX
@@ -430,25 +434,45 @@ __device__ __forceinline__ BoxOut box_out(const GemmArgs &g, const Item &t, int 
 // an integer and a remainder, so I_k - beta loses nothing to the cancellation
 // of the reflection: every term left in fp32 is small or row-constant.
 //
-// Two forms of the integer part: F (fp32, every |I| below 2^24 / (2 +
-// sqrt(nb)): one exact chunk and |m_k| <= mmax, checked per tile) and
-// integer (int64 arithmetic, any size).
+// Two forms of the integer part, chosen per tile from the largest row offset
+// |m_k| of its rows:
+//   fp32   every |I| (2 + sqrt(nb)) below 2^24 (|I| below 2^24 without
+//          reflection): one exact chunk and |m_k| <= flt_mmax;
+//   int32  every |I| (2 + sqrt(nb)) below 2^31: |m_k| <= i32_mmax.  Every sum
+//          then fits in int32 (wrapping partial sums are harmless) and each
+//          result is one rounding of the exact integer.
+// A tile outside both keeps its exact products P (as int32 bit patterns
+// after several chunks) and the CTA finishes it after its last tile in int64
+// and float-float (gradx_raw_fix).  Conversions to and from 64-bit integers
+// run on the FP64 pipe, which is narrow on this GPU: the per-element path
+// uses none.
 // ---------------------------------------------------------------------------
-// beta = kappa (rho S - I_p) split as bi + bf (bi an integer) and the lead
-// value rho S, for a block of nact >= 2 rows.
+// fp32 integers of magnitude below 2^22 to int32 with one FADD: x + 1.5 2^23
+// holds x in its low mantissa bits.
+constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
+constexpr uint32_t kMagicBits = 0x4B400000u;
+
+__device__ __forceinline__ uint32_t magic_bits(float x) {
+  return __float_as_uint(__fadd_rn(x, kMagic));
+}
+
+__device__ __forceinline__ int magic_int(float x) { return (int)(magic_bits(x) - kMagicBits); }
+
+// beta = kappa (rho S - I_p) split as bi + bf (bi an integer, |bi| < 2^31 in
+// the int32 form) and the lead value rho S, for a block of nact >= 2 rows.
 struct BlockFix {
-  float bi, bf, lead;
-  long long bil;
+  float bf, lead;
+  int bi;
 };
 
-__device__ __forceinline__ BlockFix block_fix(const HhConst &c, long long S, long long Ip) {
+__device__ __forceinline__ BlockFix block_fix(const HhConst &c, long long S, int Ip) {
   const ff rS = ff_mul(c.rho, ff_from_int(S));
-  const ff w = ff_add(rS, ff_neg(ff_from_int(Ip)));
+  const ff w = ff_add(rS, ff_neg(ff_from_i32s(Ip)));
   const ff beta = ff_mul(c.kap, w);
   BlockFix f;
-  f.bi = rintf(beta.h);
-  f.bf = __fadd_rn(__fsub_rn(beta.h, f.bi), beta.l);
-  f.bil = (long long)f.bi;
+  const float bi = rintf(beta.h);
+  f.bi = __float2int_rn(bi);
+  f.bf = __fadd_rn(__fsub_rn(beta.h, bi), beta.l);
   f.lead = ff_round(rS);
   return f;
 }
@@ -458,71 +482,50 @@ __device__ __forceinline__ float dequant(const float4 &kq, float t, float U) {
   return __fmaf_rn(kq.x, t, __fmaf_rn(kq.y, U, kq.z));
 }
 
-// The integer parts I of 32 rows (one box) of this thread's column.
-//   F form: fp32 values, I = P + m CWc (one exact fma).
-//   integer form: int64, I = P + m CWc with P folded over chunks.
-template <bool F>
-struct Ints;
-
-template <>
-struct Ints<true> {
-  float v[32];
-  __device__ __forceinline__ long long ll(int i) const { return (long long)v[i]; }
-  __device__ __forceinline__ float f(int i) const { return v[i]; }
-  __device__ __forceinline__ float minus(int i, const BlockFix &b) const {
-    return __fsub_rn(__fsub_rn(v[i], b.bi), b.bf);
-  }
-};
-
-template <>
-struct Ints<false> {  // the int32 products; I = P + m CWc formed on use
+// The integer parts I = P + m CWc of 32 rows (one box) of this thread's
+// column in the int32 form.
+struct Ints {
   int v[32];
-  const float4 *kp;
-  long long cw;
-  __device__ __forceinline__ long long ll(int i) const {
-    return (long long)v[i] + (long long)kp[i].w * cw;
-  }
-  __device__ __forceinline__ float f(int i) const { return __ll2float_rn(ll(i)); }
+  __device__ __forceinline__ float f(int i) const { return __int2float_rn(v[i]); }
   __device__ __forceinline__ float minus(int i, const BlockFix &b) const {
-    return __fsub_rn(__ll2float_rn(ll(i) - b.bil), b.bf);
+    return __fsub_rn(__int2float_rn((int)((uint32_t)v[i] - (uint32_t)b.bi)), b.bf);
   }
 };
 
-// Loads the products of the 32 rows at TMEM column c0 and forms I.
-template <bool F>
-__device__ __forceinline__ void load_ints(uint32_t acc, uint32_t ints, bool multi, int c0,
-                                          const float4 *kp, float cwc, Ints<F> &I) {
-  uint32_t r[32];
+// The exact products P of one TMEM column group: the chunk's fp32 value plus
+// the int32 running sum of the earlier chunks.
+__device__ __forceinline__ void load_products(uint32_t acc, uint32_t ints, bool multi, int c0,
+                                              int (&P)[32]) {
+  uint32_t r[32], s[32];
   tmem_ld32_nw(acc + (uint32_t)c0, r);
-  if constexpr (F) {
-    tmem_wait_ld(r);
+  if (multi) tmem_ld32_nw(ints + (uint32_t)c0, s);
+  tmem_wait_ld(r);
+  if (multi) tmem_wait_ld(s);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) I.v[i] = __fmaf_rn(kp[c0 + i].w, cwc, __uint_as_float(r[i]));
-  } else {
-    uint32_t s[32];
-    if (multi) tmem_ld32_nw(ints + (uint32_t)c0, s);
-    tmem_wait_ld(r);
-    if (multi) tmem_wait_ld(s);
-    I.kp = kp + c0;
-    I.cw = (long long)cwc;
+  for (int i = 0; i < 32; ++i)
+    P[i] = (int)((uint32_t)__float2int_rn(__uint_as_float(r[i])) + (multi ? s[i] : 0u));
+}
+
+// Loads the products of the 32 rows at TMEM column c0 and forms I
+// (|m| <= i32_mmax and |CWc| <= C 2^(bw-1) are below 2^22).
+__device__ __forceinline__ void load_ints(uint32_t acc, uint32_t ints, bool multi, int c0,
+                                          const float4 *kp, float cwc, Ints &I) {
+  load_products(acc, ints, multi, c0, I.v);
+  const uint32_t cw = (uint32_t)magic_int(cwc);
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
-      I.v[i] = __float2int_rn(__uint_as_float(r[i])) + (multi ? (int)s[i] : 0);
-  }
+  for (int i = 0; i < 32; ++i)
+    I.v[i] = (int)((uint32_t)I.v[i] + (uint32_t)magic_int(kp[c0 + i].w) * cw);
 }
 
 // I of one row (TMEM column col) of this thread's column.
-template <bool F>
-__device__ __forceinline__ long long load_int1(uint32_t acc, uint32_t ints, bool multi,
-                                               int col, float m, float cwc) {
+__device__ __forceinline__ int load_int1(uint32_t acc, uint32_t ints, bool multi, int col,
+                                         float m, float cwc) {
   uint32_t v[2];
   v[0] = tmem_ld1_nw(acc + (uint32_t)col);
-  v[1] = (!F && multi) ? tmem_ld1_nw(ints + (uint32_t)col) : 0u;
+  v[1] = multi ? tmem_ld1_nw(ints + (uint32_t)col) : 0u;
   tmem_wait_ld(v);
-  if (F) return (long long)__fmaf_rn(m, cwc, __uint_as_float(v[0]));
-  long long P = __float2int_rn(__uint_as_float(v[0]));
-  if (multi) P += (int)v[1];
-  return P + (long long)m * (long long)cwc;
+  const uint32_t P = (uint32_t)__float2int_rn(__uint_as_float(v[0])) + v[1];
+  return (int)(P + (uint32_t)magic_int(m) * (uint32_t)magic_int(cwc));
 }
 
 // One box (32 rows r0 .. r0 + 31 of the tile) of blocks of NB <= 32 rows:
@@ -530,8 +533,8 @@ __device__ __forceinline__ long long load_int1(uint32_t acc, uint32_t ints, bool
 // lead products loaded per box: one per block of NB <= 32 rows
 __host__ __device__ constexpr int leads_per_box(int nb) { return nb > 1 && nb <= 32 ? 32 / nb : 1; }
 
-template <int NB, bool F>
-__device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip)[leads_per_box(NB)],
+template <int NB>
+__device__ __forceinline__ void box_small(const Ints &I, const int (&Ip)[leads_per_box(NB)],
                                           const HhConst &hc, const float4 *kp,
                                           const int *leads, int r0, int64_t row0,
                                           int64_t N, float U, const BoxOut &w) {
@@ -553,7 +556,7 @@ __device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip
     }
     long long S = 0;
 #pragma unroll
-    for (int l = 0; l < NBB; ++l) S += I.ll(b * NBB + l);
+    for (int l = 0; l < NBB; ++l) S += I.v[b * NBB + l];
     const BlockFix f = block_fix(nact == NBB ? hc : hh_const(nact), S, Ip[b]);
 #pragma unroll
     for (int l = 0; l < NBB; ++l) w.st(b * NBB + l, dequant(kp[kb0 + l], I.minus(b * NBB + l, f), U));
@@ -562,44 +565,47 @@ __device__ __forceinline__ void box_small(const Ints<F> &I, const long long (&Ip
   }
 }
 
-// The final chunk of one tile for this warp: groups of GW rows (a box, or
-// one block of NB > 32 rows spanning several boxes).
-template <int NB, bool F>
+// The final chunk of one tile for this warp in the int32 form: groups of GW
+// rows (a box, or one block of NB > 32 rows spanning several boxes).  raw: a
+// tile outside both forms, whose row terms are units (m = 0, so I = P): its
+// exact products P are stored as int32 bit patterns for gradx_raw_fix.
+template <int NB>
 __device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uint32_t acc,
                                            uint32_t ints, bool multi, const float4 *kp,
                                            const int *leads, const HhConst &hc, float cwc,
-                                           float U, uint64_t *acce_set, int q, int lane) {
+                                           float U, uint64_t *acce_set, int q, int lane,
+                                           bool raw) {
   constexpr int GW = NB > 32 ? NB : 32;
   constexpr int NPP = leads_per_box(NB);
 #pragma unroll 1
   for (int g0 = 0; g0 < BN; g0 += GW) {
     // blocks of more than 32 rows: their sums over all boxes first
-    long long S_big = 0, Ip_big = 0;
-    int p_big = 0;
+    long long S_big = 0;
+    int Ip_big = 0, p_big = 0;
     if (NB > 32) {
 #pragma unroll 1
       for (int bx = 0; bx < GW / 32; ++bx) {
-        Ints<F> I;
-        load_ints<F>(acc, ints, multi, g0 + bx * 32, kp, cwc, I);
+        Ints I;
+        load_ints(acc, ints, multi, g0 + bx * 32, kp, cwc, I);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) S_big += I.ll(i);
+        for (int i = 0; i < 32; ++i) S_big += I.v[i];
       }
       p_big = leads[g0 / (NB > 32 ? NB : 1)];
-      Ip_big = load_int1<F>(acc, ints, multi, g0 + p_big, kp[g0 + p_big].w, cwc);
+      Ip_big = load_int1(acc, ints, multi, g0 + p_big, kp[g0 + p_big].w, cwc);
     }
 #pragma unroll 1
     for (int bx = 0; bx < GW / 32; ++bx) {
       const int r0 = g0 + bx * 32;
       const BoxOut w = box_out(g, t, q, lane, r0);
-      Ints<F> I;
-      load_ints<F>(acc, ints, multi, r0, kp, cwc, I);
-      long long Ip[NPP];
+      Ints I;
+      load_ints(acc, ints, multi, r0, kp, cwc, I);
+      int Ip[NPP];
 #pragma unroll
       for (int b = 0; b < NPP; ++b) {
         Ip[b] = 0;
         if (NB > 1 && NB <= 32) {
           const int col = r0 + b * (32 / NPP) + leads[(r0 + b * (32 / NPP)) / (32 / NPP)];
-          Ip[b] = load_int1<F>(acc, ints, multi, col, kp[col].w, cwc);
+          Ip[b] = load_int1(acc, ints, multi, col, kp[col].w, cwc);
         }
       }
       if (r0 + 32 == BN) {  // the accumulator has been read in full
@@ -607,8 +613,12 @@ __device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uin
         __syncwarp();
         if (lane == 0) mbar_arrive(acce_set);
       }
+      if (raw) {
+        w.st32(reinterpret_cast<const float (&)[32]>(I.v));
+        continue;
+      }
       if constexpr (NB <= 32) {
-        box_small<NB, F>(I, Ip, hc, kp, leads, r0, t.n0 + r0, g.N, U, w);
+        box_small<NB>(I, Ip, hc, kp, leads, r0, t.n0 + r0, g.N, U, w);
       } else {
         const int64_t left = g.N - (t.n0 + g0);
         const int nact = left >= NB ? NB : (int)(left > 0 ? left : 0);
@@ -627,32 +637,13 @@ __device__ __forceinline__ void gradx_tile(const GemmArgs &g, const Item &t, uin
   }
 }
 
-// fp32 integers of magnitude below 2^22 to int32 with one FADD: x + 1.5 2^23
-// holds x in its low mantissa bits.  (Conversions to and from 64-bit
-// integers run on the FP64 pipe, which is slow on this GPU; the fp32 form
-// uses none per element.)
-constexpr float kMagic = 12582912.0f;  // 1.5 * 2^23
-constexpr uint32_t kMagicBits = 0x4B400000u;
-
-__device__ __forceinline__ uint32_t magic_bits(float x) {
-  return __float_as_uint(__fadd_rn(x, kMagic));
-}
-
-__device__ __forceinline__ int magic_int(float x) { return (int)(magic_bits(x) - kMagicBits); }
-
-// An int32 as float-float (exact).
-__device__ __forceinline__ ff ff_from_i32(int v) {
-  const float h = __int2float_rn(v);
-  return {h, __int2float_rn(v - __float2int_rz(h))};
-}
-
 struct BlockFixF {
   float bi, bf, lead;
 };
 
 __device__ __forceinline__ BlockFixF block_fix_f(const HhConst &c, int S, int Ip) {
-  const ff rS = ff_mul(c.rho, ff_from_i32(S));
-  const ff w = ff_add(rS, ff_neg(ff_from_i32(Ip)));
+  const ff rS = ff_mul(c.rho, ff_from_i32s(S));
+  const ff w = ff_add(rS, ff_neg(ff_from_i32s(Ip)));
   const ff beta = ff_mul(c.kap, w);
   BlockFixF f;
   f.bi = rintf(beta.h);
@@ -1044,18 +1035,22 @@ __device__ __forceinline__ void gradx_params(const GemmArgs &g, uint8_t *smem, u
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1)
       mabs = fmaxf(mabs, __shfl_xor_sync(0xffffffffu, mabs, off));
-    // fp32 form with fixed blocks: a tile with a row offset beyond it keeps
-    // the exact products P (unit row terms); its bit sends it to the CTA's
-    // final pass (gradx_raw_fix)
-    const bool raw = FORM == 2 && NB != 0 && !(mabs <= g.flt_mmax);
+    // a tile with a row offset beyond its forms (FORM 2: the fp32 form;
+    // otherwise the int32 form, which holds more) keeps the exact products P
+    // (unit row terms); its bit sends it to the CTA's final pass
+    // (gradx_raw_fix)
+    const bool raw = NB != 0 && !(mabs <= (FORM == 2 ? g.flt_mmax : g.i32_mmax));
     if (raw) {
 #pragma unroll
       for (int i = 0; i < BN / 32; ++i) kp[lane + 32 * i] = make_float4(1.0f, 0.0f, 0.0f, 0.0f);
       if (lane == 0 && local < kMaxLocalTiles) raw_mask[local >> 5] |= 1u << (local & 31);
     }
+    // 1: the fp32 form, 2: the int32 form, 0: raw
     if (lane == 0)
       *reinterpret_cast<int *>(P + kParFlag) =
-          NB == 0 || (FORM == 2 && !raw) || (FORM == 1 && mabs <= g.flt_mmax);
+          NB == 0 || (FORM == 2 && !raw) || (FORM == 1 && mabs <= g.flt_mmax) ? 1
+          : raw                                                             ? 0
+                                                                            : 2;
     __syncwarp();
     if (lane == 0) mbar_arrive(&pfull[s]);
     cur = nxt;
@@ -1098,7 +1093,7 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
     const int *leads = reinterpret_cast<const int *>(P + kParLeads);
     const int *msum = reinterpret_cast<const int *>(P + kParMsum);
     const int cs = reinterpret_cast<const int *>(P + kParCs)[q * 32 + lane];
-    const bool tile_f = FORM != 0 && *reinterpret_cast<const int *>(P + kParFlag) != 0;
+    const int tform = *reinterpret_cast<const int *>(P + kParFlag);  // 1 fp32, 2 int32, 0 raw
     const float cwc = (float)(cs - Cn * g.ow);
     const float U = __fmaf_rn((float)Cn, zw, (float)cs);
     for (int64_t c = 0; c < nchunks; ++c) {
@@ -1144,12 +1139,13 @@ __device__ __forceinline__ void gradx_epilogue(const GemmArgs &g, uint8_t *smem,
         if constexpr (FORM == 2) {
           // a tile outside the fp32 form has unit row terms (kq = (1, 0, 0, 0)):
           // the one-row epilogue stores its exact products P for gradx_raw_fix
-          gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane, !tile_f);
-        } else if (FORM == 1 && tile_f) {
+          gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane,
+                           tform != 1);
+        } else if (FORM == 1 && tform == 1) {
           gradx_tile_f<NB>(g, t, acc, kp, leads, msum, hc, cwc, U, &acce[buf], q, lane, false);
         } else {
-          gradx_tile<NB, false>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, &acce[buf], q,
-                                lane);
+          gradx_tile<NB>(g, t, acc, ints, multi, kp, leads, hc, cwc, U, &acce[buf], q, lane,
+                         tform == 0);
         }
       }
     }
@@ -1253,7 +1249,7 @@ __device__ __forceinline__ void partial_epilogue(const GemmArgs &g, uint8_t *rin
 // group fix-up, whose arithmetic it shares).
 template <int NB>
 __device__ __noinline__ void gradx_raw_fix(const GemmArgs &g, const uint32_t *raw_mask, int ew,
-                                           int nwarps, int lane);
+                                           int nwarps, int lane, bool p_bits);
 
 template <int MODE, int NB, int FORM>
 __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
@@ -1293,7 +1289,7 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (MODE == MODE_GRADX && FORM == 2 && NB != 0)
+  if (MODE == MODE_GRADX && NB != 0)
     for (int i = threadIdx.x; i < (int)(kRawMaskBytes / 4); i += blockDim.x)
       reinterpret_cast<uint32_t *>(smem + kOffRaw)[i] = 0u;
   if (warp == kWarpMma) {
@@ -1320,13 +1316,14 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
     if (MODE == MODE_GRADX) {
       gradx_epilogue<NB, FORM>(g, smem, ring, accf, acce, pfull, pempty, tmem, &tmOut,
                                abort_flag, warp, lane);
-      if constexpr (FORM == 2 && NB != 0) {
+      if constexpr (NB != 0) {
         // every epilogue warp arrives here once; then the tiles left raw
-        // (their products stored by this CTA) are finished
+        // (their products stored by this CTA: fp32 values in FORM 2, int32
+        // bit patterns otherwise) are finished
         asm volatile("bar.sync 1, %0;" ::"r"(32 * 4 * LY::sets) : "memory");
         if (!*abort_flag)
           gradx_raw_fix<NB>(g, reinterpret_cast<const uint32_t *>(smem + kOffRaw),
-                            warp - kGemmWarpEpi0, 4 * LY::sets, lane);
+                            warp - kGemmWarpEpi0, 4 * LY::sets, lane, FORM != 2);
       }
     }
     else if (warp < kGemmWarpEpi0 + kPartialEpiWarps)
@@ -1468,6 +1465,14 @@ __global__ void __launch_bounds__(kRedElems * kRedGroups) k_reduce(const ReduceA
   __shared__ long long acc[kRedGroups][kRedElems];
   const int64_t total = r.M * r.N;
   const int e = threadIdx.x % kRedElems, grp = threadIdx.x / kRedElems;
+  // per-tensor terms: z = -m + d with m an integer
+  const float za = r.out_i64 ? 0.0f : *r.zero_a, zb = r.out_i64 ? 0.0f : *r.zero_b;
+  const float sab = r.out_i64 ? 0.0f : (*r.inv_a) * (*r.inv_b);
+  const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
+  const float da = za + (float)ma, db = zb + (float)mb;
+  const int64_t ob = r.ob;
+  const int64_t code_pad = r.pad_a ? (int64_t)*r.code_zero - ob : 0;
+  const float kdd = ll_to_float(r.Kn) * da * db;
   for (int64_t base = (int64_t)blockIdx.x * kRedElems; base < total;
        base += (int64_t)gridDim.x * kRedElems) {
     const int64_t idx = base + e;
@@ -1492,19 +1497,15 @@ __global__ void __launch_bounds__(kRedElems * kRedGroups) k_reduce(const ReduceA
         r.out_i64[idx] = P;
       } else {
         const int64_t c = idx / r.N, d = idx - c * r.N;
-        const float za = *r.zero_a, zb = *r.zero_b;
-        const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
-        const float da = za + (float)ma, db = zb + (float)mb;
         const int64_t ca = r.cs_a[c], cb = r.cs_b[d];
-        const int64_t ob = r.ob;
-        if (r.pad_a) P += ((int64_t)*r.code_zero - ob) * r.pad_a[c * r.taps + d / r.cin];
+        if (r.pad_a) P += code_pad * r.pad_a[c * r.taps + d / r.cin];
         // I = sum (a - ma)(b - mb), exact, from the centred product P
         const int64_t I = P + (r.oa - ma) * (cb - r.Kn * ob) +
                           (ob - mb) * (ca - r.Kn * r.oa) +
                           r.Kn * (r.oa - ma) * (ob - mb);
-        const float V = (float)I + db * (float)(ca - r.Kn * ma) +
-                        da * (float)(cb - r.Kn * mb) + (float)r.Kn * da * db;
-        r.out_f32[idx] = (*r.inv_a) * (*r.inv_b) * V;
+        const float V = ll_to_float(I) + db * ll_to_float(ca - r.Kn * ma) +
+                        da * ll_to_float(cb - r.Kn * mb) + kdd;
+        r.out_f32[idx] = sab * V;
       }
     }
     __syncthreads();
@@ -1649,6 +1650,15 @@ typedef void (*GemmKernel)(CUtensorMap, CUtensorMap, CUtensorMap, GemmArgs);
 // has z' in [-(2^b - 1), 0], so |m| <= 2^(b-1): with mmax at least that, only
 // rows of one sign far from 0 leave the form, and form 2 finishes them in a
 // final pass; otherwise many tiles can, and form 1 keeps both paths.
+// The largest row offset |m| of the int32 form for a reduction over C with
+// codes of bw (W~) and b bits and blocks of nb rows: every |I| (2 + sqrt(nb))
+// below 2^31 with |I| <= C 2^(bw-1) (2^(b-1) + |m|); -1 when none.
+static float int32_form_mmax(int64_t C, int bw, int b, int nb) {
+  const double lim = nb <= 1 ? 2147483647.0 : 2147483647.0 / (2.0 + sqrt((double)nb));
+  const double m = floor(lim / ((double)C * (double)(1 << (bw - 1)))) - (double)(1 << (b - 1)) - 1.0;
+  return m >= 0.0 ? (float)m : -1.0f;
+}
+
 static int epilogue_form(bool flt, double mmax, int b) {
   if (!flt) return 0;
   return mmax >= (double)(1 << (b - 1)) ? 2 : 1;
@@ -1766,7 +1776,8 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   int64_t grid = g.n_items < nsm ? g.n_items : nsm;
   if (grid < 1) grid = 1;
   // the raw-tile bits of a CTA cover kMaxLocalTiles of its tiles
-  if (four && nb != 0 && (g.n_items + grid - 1) / grid > kMaxLocalTiles) return FQT_EUNSUPPORTED;
+  if (!partial && nb != 0 && (g.n_items + grid - 1) / grid > kMaxLocalTiles)
+    return FQT_EUNSUPPORTED;
   kern<<<(int)grid, threads, smem, st>>>(ta, tb, to, g);
   return cuda_fail(cudaGetLastError(), "gemm launch");
 }
@@ -2175,12 +2186,10 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
   if (!aligned16(qx->codes_f16) || !aligned16(qw->codes_f16) || !aligned16(H)) return FQT_EINVAL;
   const int nsm = device_sm_count();
   const SplitPlan p = plan_splits(C, Nr, D, qw->bits, qx->bits, nsm, false);
+  // no reflection: with P exact (one chunk) the fp32 form holds for all m
   const int64_t kc_terms = (int64_t)exact_chunk_blocks(qw->bits, qx->bits) * BK;
-  const double mmax = floor(16777216.0 / ((double)D * (double)(1 << (qw->bits - 1)))) -
-                      (double)(1 << (qx->bits - 1)) - 1.0;
-  const int64_t pmax = D << (qw->bits + qx->bits - 2);
-  const bool flt = D <= kc_terms && mmax >= 0.0;  // no block sums: |P| < 2^24 suffices
-  (void)pmax;
+  const double mmax = 1e30;
+  const bool flt = D <= kc_terms;
   GemmArgs g;
   memset(&g, 0, sizeof(g));
   g.status = reinterpret_cast<int *>(ws);
@@ -2194,6 +2203,7 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
   g.inv_sw = qw->inv_s;
   g.zero_w = qw->zero;
   g.flt_mmax = flt ? (float)mmax : -1.0f;
+  g.i32_mmax = int32_form_mmax(D, qw->bits, qx->bits, 1);
   return run_gemm(qw->codes_f16, 1, qw->bits, qx->codes_f16, 1, qx->bits, C, Nr, D, p, g, H,
                   MODE_GRADX, 1, epilogue_form(flt, mmax, qx->bits), st);
 }
@@ -2286,6 +2296,7 @@ struct FixArgs {
   // (PTQ) and the lead row of every block
   int nbk, per_tensor;
   const int32_t *lead;
+  int p_bits;  // the stored products are int32 bit patterns (else fp32 values)
   int *status;
 };
 
@@ -2356,7 +2367,10 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
   const int Cn = f.C;
   const bool refl = nb >= 2;
   // the fp32 form: |P| < 2^22 and |I| (2 + sqrt(nb)) < 2^24 for every row
-  bool fast = refl && f.small_p;
+  bool fast = refl && f.small_p && !f.p_bits;
+  auto pint = [&](float v) -> long long {
+    return f.p_bits ? (long long)__float_as_int(v) : (long long)__float2int_rn(v);
+  };
   if (fast) {
     const double lim = 16777216.0 / (2.0 + sqrt((double)nb));
     const double mmax = floor(lim / ((double)Cn * (double)(1 << (f.bw - 1)))) -
@@ -2419,7 +2433,7 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
       const float pv[4] = {P.x, P.y, P.z, P.w};
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
-        const long long I = (long long)__float2int_rn(pv[c]) + m * cwi[c];
+        const long long I = pint(pv[c]) + m * cwi[c];
         S[c] += I;
         if (r == lead) Ipl[c] = I;
       }
@@ -2442,7 +2456,7 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
       float o4[4];
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
-        const ff I = ff_from_int((long long)__float2int_rn(pv[c]) + m * cwi[c]);
+        const ff I = ff_from_int(pint(pv[c]) + m * cwi[c]);
         ff v = !refl ? I : (r == lead ? rS[c] : ff_add(I, ff_neg(beta[c])));
         v = ff_add(v, two_prod(t.hd, U[c]));
         v = ff_add(v, ff_mul({t.hR, 0.0f}, y));
@@ -2461,7 +2475,7 @@ __device__ __noinline__ void fix_group_general(const FixArgs &f, int64_t k0, int
 // float-float where the fp32 form is not exact).  NB = 1: one row per unit.
 template <int NB>
 __device__ __noinline__ void gradx_raw_fix(const GemmArgs &g, const uint32_t *raw_mask, int ew,
-                                           int nwarps, int lane) {
+                                           int nwarps, int lane, bool p_bits) {
   constexpr int NBD = NB > 1 ? NB : 1;
   constexpr int BPT = BN / NBD;  // units per tile
   int64_t n_local = (g.n_items - (int64_t)blockIdx.x + gridDim.x - 1) / gridDim.x;
@@ -2489,6 +2503,7 @@ __device__ __noinline__ void gradx_raw_fix(const GemmArgs &g, const uint32_t *ra
   f.zero_w = g.zero_w;
   f.col_sum_w = g.col_sum_w;
   f.small_p = g.small_p;
+  f.p_bits = p_bits;
   f.nbk = NB;
   f.per_tensor = g.kind == FQT_PTQ;
   f.lead = g.lead;
@@ -2812,10 +2827,14 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       // |P| < 2^22 and |I| (2 + sqrt(nb)) < 2^24 (|I| < 2^24 without
       // reflection) for every row offset |m| <= mmax, with
       // |I| <= C 2^(bw-1) (2^(b-1) + |m|)
+      // Without reflection (nb = 1) and with P exact (one chunk), fma(m,
+      // CWc, P) is the correctly rounded exact I for every row offset: the
+      // value the integer forms round to, so the fp32 form holds for all m.
       const int64_t kc_terms = (int64_t)exact_chunk_blocks(qw->bits, q_b2->bits) * BK;
       const double lim = nb <= 1 ? 16777216.0 : 16777216.0 / (2.0 + sqrt((double)nb));
-      const double mmax = floor(lim / ((double)C * (double)(1 << (qw->bits - 1)))) -
-                          (double)(1 << (q_b2->bits - 1)) - 1.0;
+      const double mmax = nb == 1 ? 1e30
+                                  : floor(lim / ((double)C * (double)(1 << (qw->bits - 1)))) -
+                                        (double)(1 << (q_b2->bits - 1)) - 1.0;
       const int64_t pmax = C << (qw->bits + q_b2->bits - 2);
       // the block sums of the reflection read |P| < 2^22 off the fp32 bits
       const bool flt = C <= kc_terms && mmax >= 0.0 && (nb <= 1 || pmax < ((int64_t)1 << 22));
@@ -2836,6 +2855,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       g.hz = q_b2->hz;
       g.hr = q_b2->hr;
       g.flt_mmax = flt ? (float)mmax : -1.0f;
+      g.i32_mmax = int32_form_mmax(C, qw->bits, q_b2->bits, nb);
       g.col_sum_w = qw->col_sum;
       g.inv_sw = qw->inv_s;
       g.zero_w = qw->zero;

@@ -314,6 +314,42 @@ def test_tiles_outside_the_fp32_form(kind, bits, block):
     assert grad_rel_err(gx, orc.grad_x(h2, hw)) <= GRAD_TOL
 
 
+@pytest.mark.parametrize("kind,bits,block,c,raw", [(orc.PSQ, 8, 0, 2048, True),
+                                                   (orc.PTQ, 8, 0, 3072, True),
+                                                   (orc.BHQ, 8, 16, 2048, True),
+                                                   (orc.BHQ, 5, 16, 2048, True),
+                                                   (orc.BHQ, 5, 128, 1024, False)])
+def test_tiles_outside_the_int32_form(kind, bits, block, c, raw):
+    """Long reductions (two or three exact chunks with 8-bit codes; one chunk
+    but no fp32 form with BHQ-5): the tile of a row whose offset m exceeds
+    the int32 form keeps its products P as int32 bit patterns and the CTA's
+    final pass finishes it in int64; a tile with a moderate offset stays in
+    the int32 form; the rest are ordinary.  Blocks of 128 rows spread a
+    row's offset over the block (every tile stays in the int32 form)."""
+    g = wl.rng(440 + bits + block + c // 1024)
+    n, d = 300, 208  # row tiles 0..127, 128..255, 256..299; ragged columns
+    dH = wl.random_grad(g, n, c, sigma=1.0)
+    if kind == orc.PTQ:
+        dH = (3000.0 + 1e-2 * g.standard_normal((n, c))).astype(np.float32)
+    else:
+        dH[10] = 5000.0 + 1e-2 * g.standard_normal(c)        # far beyond the int32 form
+        dH[140] = 6.0 + 0.5 * g.standard_normal(c)           # moderate offset
+        dH[299] = -3000.0 + 1e-2 * g.standard_normal(c)      # ragged last tile
+        dH = dH.astype(np.float32)
+    X = g.uniform(-1, 1, (n, d)).astype(np.float32)
+    W = (0.05 * g.standard_normal((c, d))).astype(np.float32)
+    L = wl.Layer("offsets-long", dH, X, W, "f32", [])
+    qx, qw, q2, q1, gx, gw = _backward(L, kind, bits, block)
+    h2, hw = q2.to_numpy(), qw.to_numpy()
+    m = np.rint(np.float32(2 ** (bits - 1)) + h2["zero"].astype(np.float32))
+    nb = max(block, 1)
+    lim = (2.0 ** 31 - 1) / (2.0 + np.sqrt(nb)) if nb > 1 else 2.0 ** 31 - 1
+    mmax32 = np.floor(lim / (c * 2.0 ** 7)) - 2 ** (bits - 1) - 1
+    assert (np.abs(m).max() > mmax32) == raw  # whether a tile leaves the int32 form
+    assert np.isfinite(gx).all()
+    assert grad_rel_err(gx, orc.grad_x(h2, hw)) <= GRAD_TOL
+
+
 def test_per_tensor_offset_sends_every_tile_to_the_tile_pass():
     """PTQ of an all-positive dH with a tiny range: one zero point for all
     rows, so every tile of grad_X -- and every tile of the forward for an X
