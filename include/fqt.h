@@ -211,7 +211,7 @@ FQT_API fqt_status fqt_quantize_grad(const void *dH, fqt_dtype dtype, int64_t N,
  * fqt_linear_backward, and q_b2->rows_per_sample = R.  PTQ is the
  * per-tensor quantizer.  BHQ returns FQT_EUNSUPPORTED (its reflection mixes
  * samples at every pixel, which neither contraction's epilogue forms).
- * Needs N % R == 0, C in {64, 128, 256, 512, 1024, 2048}, N / R <= 2^20.
+ * Needs N % R == 0, C in {64, 128, 256, 512, 1024, 2048, 4096}, N / R <= 2^20.
  */
 FQT_API fqt_status fqt_quantize_grad_samples(const void *dH, fqt_dtype dtype, int64_t N,
                                              int64_t C, int64_t rows_per_sample,

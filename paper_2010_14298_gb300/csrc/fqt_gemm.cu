@@ -1454,61 +1454,79 @@ struct ReduceArgs {
   int taps, cin;
   const int32_t *cs_a, *cs_b;  // column sums of Q_b1 codes (M) and X~ codes (N)
   const float *inv_a, *zero_a, *inv_b, *zero_b;
+  int vec;  // four outputs per thread (N % 4 == 0, 16-byte aligned buffers)
 };
 
-// A CTA sums 32 consecutive outputs over all splits: 8 groups of 32 threads
-// take every 8th split (loads of a group are one coalesced 128-byte row, four
-// in flight per thread), then the groups add up in shared memory.
-constexpr int kRedElems = 32, kRedGroups = 8;
+// A thread sums four consecutive outputs of one row over all splits (one
+// 16-byte load per split, coalesced across the warp, two splits in flight)
+// and dequantizes them (r.vec; else one output per thread).
+constexpr int kRedThreads = 256;
 
-__global__ void __launch_bounds__(kRedElems * kRedGroups) k_reduce(const ReduceArgs r) {
-  __shared__ long long acc[kRedGroups][kRedElems];
+__global__ void __launch_bounds__(kRedThreads) k_reduce(const ReduceArgs r) {
   const int64_t total = r.M * r.N;
-  const int e = threadIdx.x % kRedElems, grp = threadIdx.x / kRedElems;
+  const bool vec = r.vec != 0;
+  const int W = vec ? 4 : 1;
+  const int64_t units = vec ? total >> 2 : total;
   // per-tensor terms: z = -m + d with m an integer
-  const float za = r.out_i64 ? 0.0f : *r.zero_a, zb = r.out_i64 ? 0.0f : *r.zero_b;
-  const float sab = r.out_i64 ? 0.0f : (*r.inv_a) * (*r.inv_b);
+  const bool deq = r.out_i64 == nullptr;
+  const float za = deq ? *r.zero_a : 0.0f, zb = deq ? *r.zero_b : 0.0f;
+  const float sab = deq ? (*r.inv_a) * (*r.inv_b) : 0.0f;
   const int64_t ma = __float2int_rn(-za), mb = __float2int_rn(-zb);
   const float da = za + (float)ma, db = zb + (float)mb;
   const int64_t ob = r.ob;
   const int64_t code_pad = r.pad_a ? (int64_t)*r.code_zero - ob : 0;
   const float kdd = ll_to_float(r.Kn) * da * db;
-  for (int64_t base = (int64_t)blockIdx.x * kRedElems; base < total;
-       base += (int64_t)gridDim.x * kRedElems) {
-    const int64_t idx = base + e;
-    long long P0 = 0, P1 = 0, P2 = 0, P3 = 0;
-    if (idx < total) {
-      int sp = grp;
-      for (; sp + 3 * kRedGroups < r.splits; sp += 4 * kRedGroups) {
-        P0 += r.part[(int64_t)sp * total + idx];
-        P1 += r.part[(int64_t)(sp + kRedGroups) * total + idx];
-        P2 += r.part[(int64_t)(sp + 2 * kRedGroups) * total + idx];
-        P3 += r.part[(int64_t)(sp + 3 * kRedGroups) * total + idx];
+  // I = sum (a - ma)(b - mb) = P + ka cb + kb ca + k0, exact, from the
+  // centred product P (ca, cb the code column sums)
+  const int64_t ka = r.oa - ma, kb = ob - mb;
+  const int64_t k0 = r.Kn * ka * kb - ka * r.Kn * ob - kb * r.Kn * r.oa;
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < units;
+       u += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t idx = u * W;
+    long long P[4] = {0, 0, 0, 0};
+    if (vec) {
+      const int4 *src = reinterpret_cast<const int4 *>(r.part + idx);
+      const int64_t step = total >> 2;
+      int sp = 0;
+      for (; sp + 1 < r.splits; sp += 2) {
+        const int4 x = __ldcs(src + (int64_t)sp * step), y = __ldcs(src + (int64_t)(sp + 1) * step);
+        P[0] += (long long)x.x + y.x;
+        P[1] += (long long)x.y + y.y;
+        P[2] += (long long)x.z + y.z;
+        P[3] += (long long)x.w + y.w;
       }
-      for (; sp < r.splits; sp += kRedGroups) P0 += r.part[(int64_t)sp * total + idx];
-    }
-    acc[grp][e] = P0 + P1 + P2 + P3;
-    __syncthreads();
-    if (grp == 0 && idx < total) {
-      int64_t P = 0;
-#pragma unroll
-      for (int g2 = 0; g2 < kRedGroups; ++g2) P += acc[g2][e];
-      if (r.out_i64) {
-        r.out_i64[idx] = P;
-      } else {
-        const int64_t c = idx / r.N, d = idx - c * r.N;
-        const int64_t ca = r.cs_a[c], cb = r.cs_b[d];
-        if (r.pad_a) P += code_pad * r.pad_a[c * r.taps + d / r.cin];
-        // I = sum (a - ma)(b - mb), exact, from the centred product P
-        const int64_t I = P + (r.oa - ma) * (cb - r.Kn * ob) +
-                          (ob - mb) * (ca - r.Kn * r.oa) +
-                          r.Kn * (r.oa - ma) * (ob - mb);
-        const float V = ll_to_float(I) + db * ll_to_float(ca - r.Kn * ma) +
-                        da * ll_to_float(cb - r.Kn * mb) + kdd;
-        r.out_f32[idx] = sab * V;
+      if (sp < r.splits) {
+        const int4 x = __ldcs(src + (int64_t)sp * step);
+        P[0] += x.x;
+        P[1] += x.y;
+        P[2] += x.z;
+        P[3] += x.w;
       }
+    } else {
+      for (int sp = 0; sp < r.splits; ++sp) P[0] += __ldcs(r.part + (int64_t)sp * total + idx);
     }
-    __syncthreads();
+    if (!deq) {
+      for (int i = 0; i < W; ++i) r.out_i64[idx + i] = P[i];
+      continue;
+    }
+    const int64_t c = idx / r.N, d0 = idx - c * r.N;
+    const int64_t ca = r.cs_a[c];
+    // row term db (ca - Kn ma) of this thread's row
+    const float rt = db * ll_to_float(ca - r.Kn * ma);
+    const int64_t Ia = kb * ca + k0;
+    float o[4];
+    for (int i = 0; i < W; ++i) {
+      const int64_t d = d0 + i;
+      const int64_t cb = r.cs_b[d];
+      long long Pi = P[i];
+      if (r.pad_a) Pi += code_pad * r.pad_a[c * r.taps + d / r.cin];
+      const int64_t I = Pi + ka * cb + Ia;
+      o[i] = sab * (ll_to_float(I) + rt + da * ll_to_float(cb - r.Kn * mb) + kdd);
+    }
+    if (vec)
+      *reinterpret_cast<float4 *>(r.out_f32 + idx) = make_float4(o[0], o[1], o[2], o[3]);
+    else
+      r.out_f32[idx] = o[0];
   }
 }
 
@@ -1792,13 +1810,16 @@ __global__ void k_u8_to_f16(const uint8_t *__restrict__ src, uint16_t *dst,
   }
 }
 
-static void launch_reduce(const ReduceArgs &r, cudaStream_t st) {
+static void launch_reduce(ReduceArgs r, cudaStream_t st) {
   const int64_t total = r.M * r.N;
-  int64_t grid = (total + kRedElems - 1) / kRedElems;
-  const int64_t cap = (int64_t)device_sm_count() * 16;
+  auto a16 = [](const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
+  r.vec = (r.N & 3) == 0 && a16(r.part) && (r.out_i64 || a16(r.out_f32));
+  const int64_t units = r.vec ? total >> 2 : total;
+  int64_t grid = (units + kRedThreads - 1) / kRedThreads;
+  const int64_t cap = (int64_t)device_sm_count() * 8;
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
-  k_reduce<<<(int)grid, kRedElems * kRedGroups, 0, st>>>(r);
+  k_reduce<<<(int)grid, kRedThreads, 0, st>>>(r);
 }
 
 static bool aligned16(const void *p) {

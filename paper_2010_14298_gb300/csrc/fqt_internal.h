@@ -41,6 +41,9 @@ struct QuantArgs {
   float *sscale;
   const float2 *part;
   int npart;
+  // code pass of the two-pass quantizers: column parts per chunk of rows
+  // (> 1: the row sums are accumulated atomically, cleared by the first pass)
+  int code_split;
   int *status;
   // launch geometry
   int TW, OPT, RL, RPL, GT, G, nchunk, unit_rows, stage_bytes;

@@ -988,12 +988,15 @@ size_t bhq_pass_bytes(int64_t N, int64_t C) {
 // non-finite flag of the whole tensor (the range of Q_b1) and the clearing of
 // the column sums the code pass accumulates into.
 // ---------------------------------------------------------------------------
-template <typename T, int LPR, int STEPS, int TEAM>
+template <typename T, int LPR, int STEPS, int TEAM, int H>
 __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
     k_bhq_stats(const QuantArgs a, BhqBlock *__restrict__ bst, float *__restrict__ wsum,
                 float2 *__restrict__ part) {
   static_assert(TEAM == 1 || (LPR == 32 && STEPS <= kTeamRows), "team layout");
-  constexpr int RS = 32 / LPR, SLAB = 8 * LPR, C = SLAB * TEAM;
+  static_assert(H == 1 || TEAM == 8, "column halves only for a full team");
+  // H column parts of SLAB * TEAM columns each: a part is read, reduced and
+  // read again (from L2) after the block's scalars are known
+  constexpr int RS = 32 / LPR, SLAB = 8 * LPR, C = SLAB * TEAM * H;
   constexpr int TPC = 8 / TEAM;  // teams per CTA
   constexpr int XW = TEAM > 1 ? 8 : 1;
   __shared__ float2 xs_mm[XW][kTeamRows];
@@ -1004,9 +1007,9 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
   const int team = warp / TEAM, wi = warp - team * TEAM;
   const int nb = a.block;
   const int sub = lane / LPR, o = lane - sub * LPR;
-  const int col0 = (wi * LPR + o) * 8;
+  auto col_of = [&](int h) { return ((h * TEAM + wi) * LPR + o) * 8; };
   const float fB2 = (float)((1u << a.bits) - 1u);
-  // the code pass accumulates column sums into these
+  // the code pass accumulates column sums (and, split, row sums) into these
   {
     const int64_t g = (int64_t)blockIdx.x * blockDim.x + tid;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
@@ -1014,6 +1017,11 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
       if (a.csum1) a.csum1[i] = 0;
       if (a.csum2) a.csum2[i] = 0;
     }
+    if (a.code_split > 1)
+      for (int64_t i = g; i < a.N; i += stride) {
+        if (a.rsum1) a.rsum1[i] = 0;
+        if (a.rsum2) a.rsum2[i] = 0;
+      }
   }
   float gmn = INFINITY, gmx = -INFINITY, nanacc = 0.0f;
   const int64_t nblocks = (a.N + nb - 1) / nb;
@@ -1024,30 +1032,42 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
     float x[STEPS][8];
     bool rv[STEPS];
 #pragma unroll
-    for (int s = 0; s < STEPS; ++s) {
-      const int k = sub + RS * s;
-      rv[s] = k < nrows;
-      if (rv[s]) {
-        load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + col0, x[s]);
-      } else {
+    for (int s = 0; s < STEPS; ++s) rv[s] = sub + RS * s < nrows;
+    auto load_part = [&](int h) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) x[s][j] = 0.0f;
+      for (int s = 0; s < STEPS; ++s) {
+        const int k = sub + RS * s;
+        if (rv[s]) {
+          load_oct(reinterpret_cast<const T *>(a.h) + (r0 + k) * C + col_of(h), x[s]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) x[s][j] = 0.0f;
+        }
       }
-    }
+    };
     // ---- row statistics (and a NaN that any non-finite entry leaves) ----
     float rmin[STEPS], rmax[STEPS];
 #pragma unroll
     for (int s = 0; s < STEPS; ++s) {
-      float2 mm = make_float2(INFINITY, -INFINITY);
+      rmin[s] = INFINITY;
+      rmax[s] = -INFINITY;
+    }
+#pragma unroll 1
+    for (int h = 0; h < H; ++h) {
+      load_part(h);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        mm.x = fminf(mm.x, x[s][j]);
-        mm.y = fmaxf(mm.y, x[s][j]);
-        nanacc = fmaf(x[s][j], 0.0f, nanacc);
+      for (int s = 0; s < STEPS; ++s) {
+        float2 mm = make_float2(INFINITY, -INFINITY);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          mm.x = fminf(mm.x, x[s][j]);
+          mm.y = fmaxf(mm.y, x[s][j]);
+          nanacc = fmaf(x[s][j], 0.0f, nanacc);
+        }
+        mm = row_reduce<LPR>(mm, OpMinMax());
+        rmin[s] = fminf(rmin[s], mm.x);
+        rmax[s] = fmaxf(rmax[s], mm.y);
       }
-      mm = row_reduce<LPR>(mm, OpMinMax());
-      rmin[s] = mm.x;
-      rmax[s] = mm.y;
     }
     if constexpr (TEAM > 1) {
       if (lane == 0) {
@@ -1133,31 +1153,43 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
         kap = 1.0f / (1.0f - rho);
       }
     }
-    // w_j = sum_k e_k s_k h_kj over the block (lane: its 8 columns)
-    float w[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) w[j] = 0.0f;
-#pragma unroll
-    for (int s = 0; s < STEPS; ++s) {
-      const bool lead = (sub + RS * s) == p;
-      const float esk = __fmul_rn(kap * (lead ? rho - 1.0f : rho), lead ? s1f : s2f);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) w[j] = fmaf(esk, x[s][j], w[j]);
-    }
-#pragma unroll
-    for (int j = 0; j < 8; ++j) w[j] = xor_reduce<LPR>(w[j], OpAddF());
-    // ---- row minima of T; the code pass recomputes each t_kj with this
-    // same sequence of roundings, so z'_k is exactly its row minimum ----
     float tmin[STEPS];
 #pragma unroll
-    for (int s = 0; s < STEPS; ++s) {
-      const bool lead = (sub + RS * s) == p;
-      const float sk = lead ? s1f : s2f;
-      const float ck = lead ? rho - 1.0f : rho;
-      float tm = INFINITY;
+    for (int s = 0; s < STEPS; ++s) tmin[s] = INFINITY;
+    // the last part read is still in registers; the others are read again
+#pragma unroll 1
+    for (int h = H - 1; h >= 0; --h) {
+      if (h != H - 1) load_part(h);
+      // w_j = sum_k e_k s_k h_kj over the block (lane: its 8 columns)
+      float w[8];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) tm = fminf(tm, fmaf(-ck, w[j], __fmul_rn(sk, x[s][j])));
-      tmin[s] = row_reduce<LPR>(tm, OpMin());
+      for (int j = 0; j < 8; ++j) w[j] = 0.0f;
+#pragma unroll
+      for (int s = 0; s < STEPS; ++s) {
+        const bool lead = (sub + RS * s) == p;
+        const float esk = __fmul_rn(kap * (lead ? rho - 1.0f : rho), lead ? s1f : s2f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) w[j] = fmaf(esk, x[s][j], w[j]);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w[j] = xor_reduce<LPR>(w[j], OpAddF());
+      // ---- row minima of T; the code pass recomputes each t_kj with this
+      // same sequence of roundings, so z'_k is exactly its row minimum ----
+#pragma unroll
+      for (int s = 0; s < STEPS; ++s) {
+        const bool lead = (sub + RS * s) == p;
+        const float sk = lead ? s1f : s2f;
+        const float ck = lead ? rho - 1.0f : rho;
+        float tm = INFINITY;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) tm = fminf(tm, fmaf(-ck, w[j], __fmul_rn(sk, x[s][j])));
+        tmin[s] = fminf(tmin[s], row_reduce<LPR>(tm, OpMin()));
+      }
+      if (sub == 0) {
+        float *wd = wsum + blk * (int64_t)C + col_of(h);
+        *reinterpret_cast<float4 *>(wd) = make_float4(w[0], w[1], w[2], w[3]);
+        *reinterpret_cast<float4 *>(wd + 4) = make_float4(w[4], w[5], w[6], w[7]);
+      }
     }
     if constexpr (TEAM > 1) {
       if (lane == 0) {
@@ -1174,11 +1206,6 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
       for (int s = 0; s < STEPS; ++s) tmin[s] = __shfl_sync(0xffffffffu, mine, s);
     }
     // ---- outputs ----
-    if (sub == 0) {
-      float *wd = wsum + blk * (int64_t)C + col0;
-      *reinterpret_cast<float4 *>(wd) = make_float4(w[0], w[1], w[2], w[3]);
-      *reinterpret_cast<float4 *>(wd + 4) = make_float4(w[4], w[5], w[6], w[7]);
-    }
     if (wi == 0 && o == 0) {
 #pragma unroll
       for (int s = 0; s < STEPS; ++s) {
@@ -1224,12 +1251,13 @@ __global__ void __launch_bounds__(256, (STEPS >= 8 ? 1 : 2))
 // rounding of v (Q_b2) and of s (h - min H) (Q_b1), fp16 carriers (and
 // optional bytes), row sums of Q_b2 and column sums of the grad_W code set.
 // A lane owns two octs of a row, o and o + LPR of a slab of 16 LPR columns
-// (one coalesced 16 LPR x 4-byte access per oct); a warp takes chunks of
-// kCodeRows rows, walks the row's slabs one after another and, inside a
-// slab, the chunk's rows 32 / LPR at a time, issuing the loads of its next
-// row before it rounds the current one.  A block's w_j and scalars stay in
-// registers while the lane's rows belong to it.  Loops stay rolled and rows
-// need no exchange between warps.
+// (one coalesced 16 LPR x 4-byte access per oct); a warp takes units of
+// kCodeRows rows and 1 / code_split of the row's slabs, walks those slabs one
+// after another and, inside a slab, the unit's rows 32 / LPR at a time,
+// issuing the loads of its next row before it rounds the current one.  A
+// block's w_j and scalars stay in registers while the lane's rows belong to
+// it.  Loops stay rolled; a row's parts meet only in its row sums (atomic
+// when code_split > 1, so that wide rows of few chunks still fill the GPU).
 // ---------------------------------------------------------------------------
 constexpr int kCodeRows = 32;
 
@@ -1249,7 +1277,7 @@ __device__ __forceinline__ void load_two_octs(const T *row, int c_a, int c_b, fl
 // v = s_i (h - z_i) with the scalars of sample i = row / rows_per_sample
 // (srec: s, z, inv_s, zero per sample), written per row as well.
 template <typename T, int LPR, bool SAMPLES = false>
-__global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
+__global__ void __launch_bounds__(256, 2) k_bhq_codes(const QuantArgs a,
                                                    const BhqBlock *__restrict__ bst,
                                                    const float *__restrict__ wsum, int lg_nb,
                                                    const float4 *__restrict__ srec = nullptr,
@@ -1315,16 +1343,23 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
   const int nbm = (1 << lg_nb) - 1;
 
   const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;
+  // code_split: a power of two dividing C / SLAB
+  const int lg_split = a.code_split > 1 ? __ffs(a.code_split) - 1 : 0;
+  const int split = 1 << lg_split;
+  const int part_cols = C >> lg_split;
+  const int64_t nunits = nchunks << lg_split;
   const int64_t wstride = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t ch = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; ch < nchunks;
-       ch += wstride) {
+  for (int64_t u = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp; u < nunits;
+       u += wstride) {
+    const int64_t ch = u >> lg_split;
+    const int cpart = (int)u & (split - 1);
     const int64_t row0 = ch * kCodeRows;
     const int rows = (int)min((int64_t)kCodeRows, a.N - row0);
     rs_s[warp][0][lane] = 0;
     rs_s[warp][1][lane] = 0;
     __syncwarp();
 #pragma unroll 1
-    for (int c0 = 0; c0 < C; c0 += SLAB) {
+    for (int c0 = cpart * part_cols; c0 < (cpart + 1) * part_cols; c0 += SLAB) {
       const int ca = c0 + o * 8, cb = ca + 8 * LPR;  // this lane's two octs
       uint32_t cs[16];
 #pragma unroll
@@ -1452,8 +1487,13 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
     }
     __syncwarp();
     if (lane < rows) {
-      if (a.rsum2) a.rsum2[row0 + lane] = rs_s[warp][0][lane];
-      if (want_rs1) a.rsum1[row0 + lane] = rs_s[warp][1][lane];
+      if (split > 1) {
+        if (a.rsum2) atomicAdd(&a.rsum2[row0 + lane], rs_s[warp][0][lane]);
+        if (want_rs1) atomicAdd(&a.rsum1[row0 + lane], rs_s[warp][1][lane]);
+      } else {
+        if (a.rsum2) a.rsum2[row0 + lane] = rs_s[warp][0][lane];
+        if (want_rs1) a.rsum1[row0 + lane] = rs_s[warp][1][lane];
+      }
     }
     __syncwarp();
   }
@@ -1464,10 +1504,21 @@ __global__ void __launch_bounds__(256) k_bhq_codes(const QuantArgs a,
   }
 }
 
-template <typename T, int LPR, int STEPS, int TEAM>
+// Column parts per chunk of kCodeRows rows in the code pass: slabs of a row
+// are split until the (chunk, part) units reach about 64 per SM.
+static int code_split_of(int64_t N, int C, int lpr, int num_sms) {
+  const int nslab = C / (16 * lpr);
+  const int64_t nchunks = (N + kCodeRows - 1) / kCodeRows;
+  const int64_t target = (int64_t)num_sms * 64;
+  int split = 1;
+  while (split < nslab && nchunks * split < target) split *= 2;
+  return split;
+}
+
+template <typename T, int LPR, int STEPS, int TEAM, int H = 1>
 static cudaError_t launch_stats(const QuantArgs &a, BhqBlock *bst, float *wsum, float2 *part,
                                 int num_sms, int *grid_out, cudaStream_t st) {
-  auto kern = k_bhq_stats<T, LPR, STEPS, TEAM>;
+  auto kern = k_bhq_stats<T, LPR, STEPS, TEAM, H>;
   int per_sm = 0;
   const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, 0);
   if (e != cudaSuccess) return e;
@@ -1493,8 +1544,8 @@ static cudaError_t launch_codes(const QuantArgs &a, const BhqBlock *bst, const f
   int per_sm = 0;
   const cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);
   if (e != cudaSuccess) return e;
-  const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;
-  int64_t grid = (nchunks + 7) / 8;
+  const int64_t nunits = (a.N + kCodeRows - 1) / kCodeRows * (a.code_split > 1 ? a.code_split : 1);
+  int64_t grid = (nunits + 7) / 8;
   const int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);
   if (grid > cap) grid = cap;
   if (grid < 1) grid = 1;
@@ -1601,11 +1652,16 @@ __global__ void __launch_bounds__(256) k_sample_finish(const QuantArgs a, int64_
     bad |= redi[0];
     part[blockIdx.x] = bad ? make_float2(NAN, NAN) : make_float2(mn, mx);
   }
-  // the code pass accumulates column sums into these
+  // the code pass accumulates column sums (and, split, row sums) into these
   for (int64_t k = i; k < a.C; k += (int64_t)gridDim.x * blockDim.x) {
     if (a.csum1) a.csum1[k] = 0;
     if (a.csum2) a.csum2[k] = 0;
   }
+  if (a.code_split > 1)
+    for (int64_t k = i; k < a.N; k += (int64_t)gridDim.x * blockDim.x) {
+      if (a.rsum1) a.rsum1[k] = 0;
+      if (a.rsum2) a.rsum2[k] = 0;
+    }
 }
 
 // Workspace bytes of the per-sample quantizer: chunk partials and records.
@@ -1621,7 +1677,7 @@ size_t sample_pass_bytes(int64_t N, int64_t C, int64_t rows_per_sample) {
 fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample, int num_sms,
                                 void *scratch, float2 *part, cudaStream_t st) {
   const int C = a.C;
-  if (!(C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048))
+  if (!(C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048 || C == 4096))
     return FQT_EUNSUPPORTED;
   const int64_t ns = a.N / rows_per_sample;
   if (ns > ((int64_t)1 << 20)) return FQT_EUNSUPPORTED;
@@ -1630,6 +1686,8 @@ fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample
   float2 *cpart = static_cast<float2 *>(scratch);
   float4 *srec = reinterpret_cast<float4 *>(
       (reinterpret_cast<uintptr_t>(cpart + ns * cps) + 255) & ~(uintptr_t)255);
+  const int lpr = C == 64 ? 4 : C == 128 ? 8 : C == 256 ? 16 : 32;
+  a.code_split = code_split_of(a.N, C, lpr, num_sms);
   if (bf16)
     k_sample_part<__nv_bfloat16><<<(unsigned)(ns * cps), 256, 0, st>>>(a, se, cps, cpart);
   else
@@ -1643,7 +1701,6 @@ fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample
   QuantArgs a2 = a;
   a2.part = part;
   a2.npart = fin;
-  const int lpr = C == 64 ? 4 : C == 128 ? 8 : C == 256 ? 16 : 32;
   const int R = (int)rows_per_sample;
 #define FQT_SC(TT, L)                                                                        \
   {                                                                                          \
@@ -1652,8 +1709,8 @@ fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample
     int per_sm = 0;                                                                          \
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);             \
     if (e == cudaSuccess) {                                                                  \
-      const int64_t nchunks = (a.N + kCodeRows - 1) / kCodeRows;                             \
-      int64_t grid = (nchunks + 7) / 8;                                                      \
+      const int64_t nunits = (a.N + kCodeRows - 1) / kCodeRows * a2.code_split;              \
+      int64_t grid = (nunits + 7) / 8;                                                       \
       const int64_t cap = (int64_t)num_sms * (per_sm > 0 ? per_sm : 1);                     \
       if (grid > cap) grid = cap;                                                            \
       if (grid < 1) grid = 1;                                                                \
@@ -1673,11 +1730,11 @@ fqt_status launch_sample_passes(QuantArgs &a, bool bf16, int64_t rows_per_sample
 }
 
 // The two-pass BHQ quantizer takes fixed blocks of 4, 8 or 16 rows and rows
-// of 64, 128 or 256 t (t = 1, 2, 4, 8) columns; bf16 input with blocks of 16.
+// of 64, 128 or 256 t (t = 1, 2, 4, 8, 16) columns; bf16 input with blocks of 16.
 bool bhq_pass_supported(int C, int block, bool bf16) {
   if (block != 4 && block != 8 && block != 16) return false;
   if (bf16 && block != 16) return false;
-  return C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048;
+  return C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048 || C == 4096;
 }
 
 // Statistics pass, code pass and the grad_X offsets (k_bhq_offsets) of the
@@ -1692,9 +1749,15 @@ fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch
   float *wsum = reinterpret_cast<float *>(
       (reinterpret_cast<uintptr_t>(bst + nblocks) + 255) & ~(uintptr_t)255);
   const int C = a.C, nb = a.block;
+  // lanes per row of the code pass: a lane owns 16 columns (two octs) of a
+  // slab of 16 LPR
+  const int lpr = C == 64 ? 4 : C == 128 ? 8 : C == 256 ? 16 : 32;
+  a.code_split = code_split_of(a.N, C, lpr, num_sms);
   int grid1 = 0;
   cudaError_t e = cudaErrorInvalidValue;
 #define FQT_ST(TT, L, S, TM) e = launch_stats<TT, L, S, TM>(a, bst, wsum, part, num_sms, &grid1, st);
+  // C = 4096: a team of 8 warps over two column halves
+#define FQT_ST2(TT, L, S) e = launch_stats<TT, L, S, 8, 2>(a, bst, wsum, part, num_sms, &grid1, st);
   if (!bf16) {
     if (C == 64) {
       if (nb == 4) { FQT_ST(float, 8, 1, 1) } else if (nb == 8) { FQT_ST(float, 8, 2, 1) }
@@ -1706,7 +1769,8 @@ fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch
       const int team = C / 256;
 #define FQT_ST_T(S)                                                                  \
   if (team == 1) { FQT_ST(float, 32, S, 1) } else if (team == 2) { FQT_ST(float, 32, S, 2) } \
-  else if (team == 4) { FQT_ST(float, 32, S, 4) } else { FQT_ST(float, 32, S, 8) }
+  else if (team == 4) { FQT_ST(float, 32, S, 4) } else if (team == 8) { FQT_ST(float, 32, S, 8) } \
+  else { FQT_ST2(float, 32, S) }
       if (nb == 4) { FQT_ST_T(4) } else if (nb == 8) { FQT_ST_T(8) } else { FQT_ST_T(16) }
 #undef FQT_ST_T
     }
@@ -1716,15 +1780,15 @@ fqt_status launch_bhq_passes(QuantArgs &a, bool bf16, int num_sms, void *scratch
     else if (C == 256) { FQT_ST(__nv_bfloat16, 32, 16, 1) }
     else if (C == 512) { FQT_ST(__nv_bfloat16, 32, 16, 2) }
     else if (C == 1024) { FQT_ST(__nv_bfloat16, 32, 16, 4) }
-    else { FQT_ST(__nv_bfloat16, 32, 16, 8) }
+    else if (C == 2048) { FQT_ST(__nv_bfloat16, 32, 16, 8) }
+    else { FQT_ST2(__nv_bfloat16, 32, 16) }
   }
 #undef FQT_ST
+#undef FQT_ST2
   if (e != cudaSuccess) return cuda_fail(e, "BHQ statistics pass launch");
   QuantArgs a2 = a;
   a2.part = part;
   a2.npart = grid1;
-  // lanes per row: a lane owns 16 columns (two octs) of a slab of 16 LPR
-  const int lpr = C == 64 ? 4 : C == 128 ? 8 : C == 256 ? 16 : 32;
   if (!bf16) {
     e = lpr == 4    ? launch_codes<float, 4>(a2, bst, wsum, num_sms, st)
         : lpr == 8  ? launch_codes<float, 8>(a2, bst, wsum, num_sms, st)

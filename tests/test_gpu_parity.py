@@ -141,6 +141,31 @@ def test_quantize_grad_matches_oracle(cfg, small, kind, bits, block):
         _check_b1(q1, dH, seed)
 
 
+@pytest.mark.parametrize("C,block,dtype", [(4096, 16, "f32"), (4096, 4, "f32"),
+                                            (4096, 16, "bf16"), (2048, 8, "f32"),
+                                            (512, 16, "bf16"), (1024, 4, "f32")])
+def test_bhq_two_pass_widths_match_oracle(C, block, dtype):
+    """The two-pass BHQ quantizer at the widths of its statistics pass: one
+    warp per row group (C <= 128), a team of C / 256 warps (up to 2048), and
+    a team of 8 warps over two column halves (C = 4096, the FFN's hidden
+    width); ragged final block."""
+    g = wl.rng(C + block)
+    n = 37 * block + 3
+    dH = wl.random_grad(g, n, C, sigma=1.3)
+    if dtype == "bf16":
+        dH = torch.from_numpy(dH).to(torch.bfloat16).float().numpy()
+    seed = 4242
+    q2, q1 = fqt.quantize_grad(to_dev(dH, dtype), orc.BHQ, 5, block, seed)
+    ref = orc.quantize_grad(dH, orc.BHQ, 5, block, seed, orc.STREAM_B2, want_v=True)
+    h2 = q2.to_numpy()
+    assert np.array_equal(h2["lead"], ref["lead"])
+    _check_bhq_codes(h2["codes"], ref["codes"], ref["v"], seed)
+    assert np.allclose(h2["inv_s"], ref["inv_s"], rtol=1e-6, atol=0)
+    assert np.allclose(h2["zero"], ref["zero"], rtol=1e-5, atol=1e-4)
+    assert np.array_equal(h2["row_sum"], h2["codes"].astype(np.int64).sum(1))
+    _check_b1(q1, dH, seed)
+
+
 @pytest.mark.parametrize("kind,bits,block", [(orc.PTQ, 4, 0), (orc.PSQ, 8, 0),
                                              (orc.BHQ, 5, 16), (orc.BHQ, 5, 64)])
 def test_fp16_carriers_encode_the_codes(kind, bits, block):
@@ -949,7 +974,7 @@ def test_grad_x_several_chunks_and_tiles_per_cta(kind, bits):
 SAMPLE_CASES = [  # rows N, C, rows per sample, bits, dtype
     (2048, 64, 1024, 5, "f32"), (2048, 64, 1024, 8, "f32"), (3136 * 2, 256, 3136, 5, "f32"),
     (196 * 4, 1024, 196, 5, "bf16"), (49 * 3, 2048, 49, 4, "f32"), (600, 128, 1, 5, "f32"),
-    (512, 512, 128, 8, "bf16")]
+    (512, 512, 128, 8, "bf16"), (64 * 3, 4096, 64, 5, "bf16")]
 
 
 @pytest.mark.parametrize("N,C,R,bits,dtype", SAMPLE_CASES)
