@@ -208,7 +208,8 @@ fqt_status fqt_quantize_grad_samples(const void *dH, fqt_dtype dtype, int64_t N,
   if (dtype != FQT_F32 && dtype != FQT_BF16) return FQT_EINVAL;
   if (N > 0 && q_b1 && ((!q_b1->codes && !q_b1->codes_f16) || !q_b1->inv_s || !q_b1->zero))
     return FQT_EINVAL;
-  if (!(C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048))
+  if (!(C == 64 || C == 128 || C == 256 || C == 512 || C == 1024 || C == 2048 ||
+        C == 4096))
     return FQT_EUNSUPPORTED;
   if (N / rows_per_sample > ((int64_t)1 << 20) || rows_per_sample > (1 << 30))
     return FQT_EUNSUPPORTED;

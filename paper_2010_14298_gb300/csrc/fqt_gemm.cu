@@ -401,6 +401,19 @@ __device__ __forceinline__ Item decode_item(const GemmArgs &g, int64_t it) {
   return r;
 }
 
+// The items of one step of a CTA's schedule: item it, and with pairs the
+// CTA's next item it + gridDim.x when it exists.  Returns their count.
+__device__ __forceinline__ int group_items(const GemmArgs &g, int64_t it, bool pairs,
+                                           Item (&tt)[2]) {
+  tt[0] = decode_item(g, it);
+  tt[1] = tt[0];
+  if (pairs && it + (int64_t)gridDim.x < g.n_items) {
+    tt[1] = decode_item(g, it + (int64_t)gridDim.x);
+    return 2;
+  }
+  return 1;
+}
+
 __device__ __forceinline__ BoxOut box_out(const GemmArgs &g, const Item &t, int q, int lane,
                                           int r0) {
   BoxOut w;
@@ -1271,6 +1284,12 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
   // grad_X: one accumulator per item, served by 4 epilogue warps (one per
   // lane quadrant); partials: accumulators alternate per chunk, 8 warps each
   constexpr bool kPerItem = MODE == MODE_GRADX;
+  // grad_X with several exact chunks per tile (two accumulators, each tile on
+  // its own): the operand ring carries two tiles at a time, chunk by chunk,
+  // so that the fold of one tile's chunk overlaps the other tile's MMAs
+  // (FORM 2 runs one exact chunk per tile: never pairs)
+  const bool pairs = FORM != 2 && kPerItem && g.nacc == 2;
+  const int64_t gstep = (pairs ? 2 : 1) * (int64_t)gridDim.x;
   constexpr uint32_t kEpiArrivals = kPerItem ? 4u : (uint32_t)kPartialEpiWarps;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1336,28 +1355,64 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
     if (lane == 0) {
       int s = 0;
       uint32_t ph = 0;
-      for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
-        const Item t = decode_item(g, it);
-        for (int64_t kb = t.kb0; kb < t.kb1; ++kb) {
-          if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) { fail(); break; }
-          mbar_expect_tx(&full[s], (uint32_t)(2 * kTileBytes));
-          uint8_t *sa = ops + (size_t)(2 * s) * kTileBytes;
-          uint8_t *sb = sa + kTileBytes;
-          const int32_t kc = (int32_t)(kb * BK);
-          // K-major: one 64 x 128 box; MN-major: two 64 (MN) x 64 (K) boxes
-          if (g.a_kmajor) {
-            tma_load_2d(sa, &tmA, kc, (int32_t)t.m0, &full[s]);
-          } else {
-            tma_load_2d(sa, &tmA, (int32_t)t.m0, kc, &full[s]);
-            tma_load_2d(sa + kTileBytes / 2, &tmA, (int32_t)t.m0 + 64, kc, &full[s]);
+      if (pairs) {
+        bool ok = true;
+        for (int64_t it = blockIdx.x; ok && it < g.n_items && !*abort_flag; it += gstep) {
+          Item tt[2];
+          const int nu = group_items(g, it, pairs, tt);
+          const int64_t nch = (tt[0].kb1 - tt[0].kb0 + g.kc_blocks - 1) / g.kc_blocks;
+          for (int64_t c = 0; ok && c < nch; ++c) {
+            for (int u = 0; ok && u < nu; ++u) {
+              const Item &t = tt[u];
+              const int64_t c0 = t.kb0 + c * g.kc_blocks, c1 = min(t.kb1, c0 + g.kc_blocks);
+              for (int64_t kb = c0; kb < c1; ++kb) {
+                if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) { fail(); ok = false; break; }
+                mbar_expect_tx(&full[s], (uint32_t)(2 * kTileBytes));
+                uint8_t *sa = ops + (size_t)(2 * s) * kTileBytes;
+                uint8_t *sb = sa + kTileBytes;
+                const int32_t kc = (int32_t)(kb * BK);
+                // K-major: one 64 x 128 box; MN-major: two 64 (MN) x 64 (K) boxes
+                if (g.a_kmajor) {
+                  tma_load_2d(sa, &tmA, kc, (int32_t)t.m0, &full[s]);
+                } else {
+                  tma_load_2d(sa, &tmA, (int32_t)t.m0, kc, &full[s]);
+                  tma_load_2d(sa + kTileBytes / 2, &tmA, (int32_t)t.m0 + 64, kc, &full[s]);
+                }
+                if (g.b_kmajor) {
+                  tma_load_2d(sb, &tmB, kc, (int32_t)t.n0, &full[s]);
+                } else {
+                  tma_load_2d(sb, &tmB, (int32_t)t.n0, kc, &full[s]);
+                  tma_load_2d(sb + kTileBytes / 2, &tmB, (int32_t)t.n0 + 64, kc, &full[s]);
+                }
+                if (++s == nstages) { s = 0; ph ^= 1u; }
+              }
+            }
           }
-          if (g.b_kmajor) {
-            tma_load_2d(sb, &tmB, kc, (int32_t)t.n0, &full[s]);
-          } else {
-            tma_load_2d(sb, &tmB, (int32_t)t.n0, kc, &full[s]);
-            tma_load_2d(sb + kTileBytes / 2, &tmB, (int32_t)t.n0 + 64, kc, &full[s]);
+        }
+      } else {
+        for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
+          const Item t = decode_item(g, it);
+          for (int64_t kb = t.kb0; kb < t.kb1; ++kb) {
+            if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) { fail(); break; }
+            mbar_expect_tx(&full[s], (uint32_t)(2 * kTileBytes));
+            uint8_t *sa = ops + (size_t)(2 * s) * kTileBytes;
+            uint8_t *sb = sa + kTileBytes;
+            const int32_t kc = (int32_t)(kb * BK);
+            // K-major: one 64 x 128 box; MN-major: two 64 (MN) x 64 (K) boxes
+            if (g.a_kmajor) {
+              tma_load_2d(sa, &tmA, kc, (int32_t)t.m0, &full[s]);
+            } else {
+              tma_load_2d(sa, &tmA, (int32_t)t.m0, kc, &full[s]);
+              tma_load_2d(sa + kTileBytes / 2, &tmA, (int32_t)t.m0 + 64, kc, &full[s]);
+            }
+            if (g.b_kmajor) {
+              tma_load_2d(sb, &tmB, kc, (int32_t)t.n0, &full[s]);
+            } else {
+              tma_load_2d(sb, &tmB, (int32_t)t.n0, kc, &full[s]);
+              tma_load_2d(sb + kTileBytes / 2, &tmB, (int32_t)t.n0 + 64, kc, &full[s]);
+            }
+            if (++s == nstages) { s = 0; ph ^= 1u; }
           }
-          if (++s == nstages) { s = 0; ph ^= 1u; }
         }
       }
       // every issued load lands before the CTA exits: in normal operation
@@ -1384,34 +1439,78 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
       // swizzle row, two 8-row K atoms (2048 bytes) for MN-major
       const uint64_t a_step = g.a_kmajor ? 2u : (2048u >> 4);
       const uint64_t b_step = g.b_kmajor ? 2u : (2048u >> 4);
-      int64_t local = 0;
-      for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
-        const Item t = decode_item(g, it);
-        if (kPerItem) buf = (int)(local & (g.nacc - 1));
-        for (int64_t c0 = t.kb0; c0 < t.kb1 && !*abort_flag; c0 += g.kc_blocks) {
-          const int64_t c1 = min(t.kb1, c0 + g.kc_blocks);
-          if (!mbar_wait(&acce[buf], ((aph >> buf) & 1u) ^ 1u, g.status)) { fail(); break; }
-          tc_fence_after();
-          const uint32_t dt = tmem + (uint32_t)(buf * BN);
-          for (int64_t kb = c0; kb < c1; ++kb) {
-            if (!mbar_wait(&full[s], ph, g.status)) { fail(); break; }
-            tc_fence_after();
-            const uint32_t a_addr = smem_u32(ops + (size_t)(2 * s) * kTileBytes);
-            const uint32_t b_addr = a_addr + (uint32_t)kTileBytes;
-            const uint64_t da = g.a_kmajor ? sw128_desc(a_addr)
-                                           : sw128_desc_mn(a_addr, g.mn_lbo, g.mn_sbo);
-            const uint64_t db = g.b_kmajor ? sw128_desc(b_addr)
-                                           : sw128_desc_mn(b_addr, g.mn_lbo, g.mn_sbo);
-#pragma unroll
-            for (int k = 0; k < BK / 16; ++k)
-              umma_f16(dt, da + a_step * k, db + b_step * k, idesc,
-                       (kb > c0 || k > 0) ? 1u : 0u);
-            umma_commit(&empty[s]);
-            if (++s == nstages) { s = 0; ph ^= 1u; }
+      if (pairs) {
+        int64_t local = 0;
+        bool ok = true;
+        for (int64_t it = blockIdx.x; ok && it < g.n_items && !*abort_flag; it += gstep) {
+          Item tt[2];
+          const int nu = group_items(g, it, pairs, tt);
+          const int64_t nch = (tt[0].kb1 - tt[0].kb0 + g.kc_blocks - 1) / g.kc_blocks;
+          for (int64_t c = 0; ok && c < nch && !*abort_flag; ++c) {
+            for (int u = 0; ok && u < nu; ++u) {
+              const Item &t = tt[u];
+              if (kPerItem) buf = (int)((local + u) & (g.nacc - 1));
+              const int64_t c0 = t.kb0 + c * g.kc_blocks, c1 = min(t.kb1, c0 + g.kc_blocks);
+              if (!mbar_wait(&acce[buf], ((aph >> buf) & 1u) ^ 1u, g.status)) {
+                fail();
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint32_t dt = tmem + (uint32_t)(buf * BN);
+              for (int64_t kb = c0; kb < c1; ++kb) {
+                if (!mbar_wait(&full[s], ph, g.status)) { fail(); ok = false; break; }
+                tc_fence_after();
+                const uint32_t a_addr = smem_u32(ops + (size_t)(2 * s) * kTileBytes);
+                const uint32_t b_addr = a_addr + (uint32_t)kTileBytes;
+                const uint64_t da = g.a_kmajor ? sw128_desc(a_addr)
+                                               : sw128_desc_mn(a_addr, g.mn_lbo, g.mn_sbo);
+                const uint64_t db = g.b_kmajor ? sw128_desc(b_addr)
+                                               : sw128_desc_mn(b_addr, g.mn_lbo, g.mn_sbo);
+  #pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                  umma_f16(dt, da + a_step * k, db + b_step * k, idesc,
+                           (kb > c0 || k > 0) ? 1u : 0u);
+                umma_commit(&empty[s]);
+                if (++s == nstages) { s = 0; ph ^= 1u; }
+              }
+              umma_commit(&accf[buf]);
+              aph ^= 1u << buf;
+              if (!kPerItem) buf ^= 1;
+            }
           }
-          umma_commit(&accf[buf]);
-          aph ^= 1u << buf;
-          if (!kPerItem) buf ^= 1;
+          local += nu;
+        }
+      } else {
+        int64_t local = 0;
+        for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x, ++local) {
+          const Item t = decode_item(g, it);
+          if (kPerItem) buf = (int)(local & (g.nacc - 1));
+          for (int64_t c0 = t.kb0; c0 < t.kb1 && !*abort_flag; c0 += g.kc_blocks) {
+            const int64_t c1 = min(t.kb1, c0 + g.kc_blocks);
+            if (!mbar_wait(&acce[buf], ((aph >> buf) & 1u) ^ 1u, g.status)) { fail(); break; }
+            tc_fence_after();
+            const uint32_t dt = tmem + (uint32_t)(buf * BN);
+            for (int64_t kb = c0; kb < c1; ++kb) {
+              if (!mbar_wait(&full[s], ph, g.status)) { fail(); break; }
+              tc_fence_after();
+              const uint32_t a_addr = smem_u32(ops + (size_t)(2 * s) * kTileBytes);
+              const uint32_t b_addr = a_addr + (uint32_t)kTileBytes;
+              const uint64_t da = g.a_kmajor ? sw128_desc(a_addr)
+                                             : sw128_desc_mn(a_addr, g.mn_lbo, g.mn_sbo);
+              const uint64_t db = g.b_kmajor ? sw128_desc(b_addr)
+                                             : sw128_desc_mn(b_addr, g.mn_lbo, g.mn_sbo);
+  #pragma unroll
+              for (int k = 0; k < BK / 16; ++k)
+                umma_f16(dt, da + a_step * k, db + b_step * k, idesc,
+                         (kb > c0 || k > 0) ? 1u : 0u);
+              umma_commit(&empty[s]);
+              if (++s == nstages) { s = 0; ph ^= 1u; }
+            }
+            umma_commit(&accf[buf]);
+            aph ^= 1u << buf;
+            if (!kPerItem) buf ^= 1;
+          }
         }
       }
       // every MMA this thread issued has completed before TMEM is released
