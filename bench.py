@@ -251,17 +251,22 @@ class LayerState:
     """Device-resident operands, codes and outputs of one layer and its five
     C-ABI calls (Q_f, Q_theta, Q_b2 + Q_b1, grad_X, grad_W)."""
 
-    def __init__(self, fqt, dH, X, W, ws, kind=KIND, bits=BITS, block=BLOCK, seed=5):
+    def __init__(self, fqt, dH, X, W, ws, kind=KIND, bits=BITS, block=BLOCK, seed=5,
+                 byte_operands=False):
         dev = dH.device
         N, C = dH.shape
         D = X.shape[1]
         self.N, self.C, self.D = N, C, D
         self.dH, self.X, self.W = dH, X, W
         self.kind, self.bits, self.block, self.seed = kind, bits, block, seed
-        self.qx = fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+        # grad_W's operands X~ and Q_b1 as 1-byte codes (widened on chip by the
+        # contraction) or as fp16 carriers (the default: faster end to end, the
+        # widening binds the contraction)
+        b = byte_operands
+        self.qx = fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=b, f16=not b)
         self.qw = fqt.QTensor.empty(C, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
         self.q2 = fqt.QTensor.empty(N, C, kind, bits, block, True, False, dev, u8=False)
-        self.q1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
+        self.q1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=b, f16=not b)
         self.gx = torch_empty((N, D), dev)
         self.gw = torch_empty((C, D), dev)
         self.ws = ws
@@ -486,7 +491,7 @@ def e2e_sweep(fqt, layers, shapes, ops_step, args, dev, stream):
     dH, X and W are copied from pinned host memory and its grad_X and grad_W
     copied back, every step.  Layers are pipelined on three streams
     (host-to-device copies, the C-ABI calls, device-to-host copies) through
-    two device staging sets sized for the largest layer, so the copies of
+    three device staging sets sized for the largest layer, so the copies of
     neighbouring layers overlap each other and the calls."""
     import torch
     h_in, h_out = [], []
@@ -501,42 +506,44 @@ def e2e_sweep(fqt, layers, shapes, ops_step, args, dev, stream):
     except RuntimeError as exc:  # pinned host memory exhausted
         return {"value": None, "unit": "TOPS", "error": f"pinned host buffers: {exc}"[:200]}
     sz = {k: max(getattr(L, k).numel() for L in layers) for k in ("dH", "X", "W", "gx", "gw")}
+    NSET = 3
     sets = [{k: torch.empty(n, dtype=torch.float32, device=dev) for k, n in sz.items()}
-            for _ in range(2)]
+            for _ in range(NSET)]
     view = lambda s, k, t: s[k][:t.numel()].view(t.shape)
     s_in, s_cmp, s_out = (torch.cuda.Stream(dev) for _ in range(3))
-    done_cmp, done_out = [None, None], [None, None]
+    done_cmp, done_out = [None] * NSET, [None] * NSET
 
     def run(nsteps, seed0):
         g = 0
         for i in range(nsteps):
             for li, L in enumerate(layers):
-                s = sets[g & 1]
+                j = g % NSET
+                s = sets[j]
                 with torch.cuda.stream(s_in):
-                    if done_cmp[g & 1] is not None:  # the layer before has read the set
-                        s_in.wait_event(done_cmp[g & 1])
+                    if done_cmp[j] is not None:  # the set's last layer has read it
+                        s_in.wait_event(done_cmp[j])
                     for k, h in zip(("dH", "X", "W"), h_in[li]):
                         view(s, k, h).copy_(h, non_blocking=True)
                     ein = torch.cuda.Event()
                     ein.record(s_in)
                 with torch.cuda.stream(s_cmp):
                     s_cmp.wait_event(ein)
-                    if done_out[g & 1] is not None:  # its gradients have left
-                        s_cmp.wait_event(done_out[g & 1])
+                    if done_out[j] is not None:  # its gradients have left
+                        s_cmp.wait_event(done_out[j])
                     for f in L.calls(dH=view(s, "dH", L.dH), X=view(s, "X", L.X),
                                      W=view(s, "W", L.W), gx=view(s, "gx", L.gx),
                                      gw=view(s, "gw", L.gw), seed=seed0 + i):
                         f()
                     ec = torch.cuda.Event()
                     ec.record(s_cmp)
-                    done_cmp[g & 1] = ec
+                    done_cmp[j] = ec
                 with torch.cuda.stream(s_out):
                     s_out.wait_event(ec)
                     for k, h in zip(("gx", "gw"), h_out[li]):
                         h.copy_(view(s, k, h), non_blocking=True)
                     eo = torch.cuda.Event()
                     eo.record(s_out)
-                    done_out[g & 1] = eo
+                    done_out[j] = eo
                 g += 1
         for st_ in (s_in, s_cmp, s_out):
             stream.wait_stream(st_)
@@ -558,7 +565,7 @@ def e2e_sweep(fqt, layers, shapes, ops_step, args, dev, stream):
     del h_in, h_out, sets
     return {"value": ops_step / (ms * 1e-3) / 1e12, "unit": "TOPS", "ms_per_step": ms,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "schedule": "layers pipelined on three streams (H2D / C-ABI calls / D2H), two "
+            "schedule": "layers pipelined on three streams (H2D / C-ABI calls / D2H), three "
                         "device staging sets, pinned host buffers per layer, eager calls",
             "device_status": status}
 
@@ -668,7 +675,18 @@ def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
     dH, X, W = on_dev(L2)
     N, C, D = L2.N, L2.C, L2.D
     ws = fqt.Workspace(N, C, D, device=dev)
-    base = LayerState(fqt, dH, X, W, ws)
+    # carriers: the shift quantizer's and the implicit im2col's grad_W pair
+    # these operands with fp16 operands of their own
+    base = LayerState(fqt, dH, X, W, ws, byte_operands=False)
+    # grad_W's byte-operand path on the same layer (1-byte X~ and Q_b1)
+    byt = LayerState(fqt, dH, X, W, ws, byte_operands=True)
+    per_byt = time_graphs(byt.calls())
+    ex["byte_operands"] = {
+        "what": "X~ and Q_b1 written as 1-byte codes only; grad_W's split-K kernel widens "
+                "them to fp16 carriers on chip (bit-identical grad_W)",
+        "per_call_ms": dict(zip(CALLS, per_byt)),
+        "carriers_per_call_ms": dict(zip(CALLS, per_base)),
+        "device_status": fqt.sync_status(ws)}
     per_base = time_graphs(base.calls())
     qa = fqt.QTensor.empty(N, C, fqt.BHQ, BITS, 0, True, False, dev, u8=False)
     qa1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)

@@ -234,6 +234,11 @@ FQT_API fqt_status fqt_quantize_grad_samples(const void *dH, fqt_dtype dtype, in
  * q_b1->col_sum, qx->col_sum (grad_W).  q_b1 may be
  * NULL when q_b2 is PTQ with col_sum set, or FQT_SHIFT: grad_W then uses
  * q_b2 (for FQT_SHIFT its shift_f16, shift_col_sum and shift_scale).
+ * grad_W's two code sets may instead both be given as bytes only (codes set,
+ * codes_f16 NULL; not the shift quantizer's, not an implicit im2col X~): the
+ * split-K contraction then reads 1 byte per code and widens the codes to fp16
+ * on chip, with the same exact integer products (and so the same grad_W, bit
+ * for bit).  One set as bytes and the other as carriers is FQT_EINVAL.
  * C % 16 == 0 and D % 16 == 0.
  */
 FQT_API fqt_status fqt_linear_backward(const fqt_qtensor *q_b2,
@@ -324,6 +329,16 @@ FQT_API fqt_status fqt_sync_status(void *workspace, void *stream);
  * u8 codes.  The stored row pitch must be a multiple of 8 and N % 4 == 0.
  * The workspace must hold fqt_debug_workspace_size(M, N, K) bytes. */
 FQT_API size_t fqt_debug_workspace_size(int64_t M, int64_t N, int64_t K);
+
+/* The same exact contraction with both operands given as MN-major byte codes
+ * (A stored K x M, B stored K x N, 16-byte aligned, M % 16 == 0, N % 16 == 0),
+ * read as bytes and widened to fp16 carriers on chip: the path
+ * fqt_linear_backward's grad_W takes when both of its code sets are given as
+ * bytes only.  Workspace as for fqt_debug_int_gemm. */
+FQT_API fqt_status fqt_debug_int_gemm_u8(const uint8_t *A, int a_bits, const uint8_t *Bm,
+                                         int b_bits, int64_t M, int64_t N, int64_t K,
+                                         int64_t *out, void *workspace, size_t ws_bytes,
+                                         void *stream);
 
 FQT_API fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
                               const uint8_t *Bm, int b_kmajor, int b_bits,

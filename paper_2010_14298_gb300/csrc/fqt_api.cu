@@ -460,6 +460,13 @@ fqt_status fqt_debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
                         workspace, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
+fqt_status fqt_debug_int_gemm_u8(const uint8_t *A, int a_bits, const uint8_t *Bm, int b_bits,
+                                 int64_t M, int64_t N, int64_t K, int64_t *out,
+                                 void *workspace, size_t ws_bytes, void *stream) {
+  return debug_int_gemm_u8(A, a_bits, Bm, b_bits, M, N, K, out, workspace, ws_bytes,
+                           reinterpret_cast<cudaStream_t>(stream));
+}
+
 fqt_status fqt_sync_status(void *workspace, void *stream) {
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e = cudaStreamSynchronize(st);

@@ -87,7 +87,9 @@ constexpr size_t kOffPar = 0;
 constexpr size_t kOffBar = kOffPar + kParStages * kParBytes;
 // operand full / empty, accumulator full / empty (4 each), parameter full /
 // empty (4 each)
-constexpr size_t kNumBars = 2 * kMaxStages + 17;  // ... + the MMA drain barrier
+// ... + the MMA drain barrier + the byte-operand rings' barriers (carrier
+// stage widened, carrier stage consumed)
+constexpr size_t kNumBars = 4 * kMaxStages + 17;
 // grad_X in the fp32 form with fixed blocks: one bit per tile of this CTA
 // (in its order) for the tiles left raw, finished by the CTA at the end
 constexpr size_t kOffRaw = (kOffBar + kNumBars * 8 + 16 + 15) & ~(size_t)15;
@@ -95,8 +97,11 @@ constexpr size_t kRawMaskBytes = 4096;
 constexpr int64_t kMaxLocalTiles = (int64_t)kRawMaskBytes * 8;
 constexpr size_t kFixedBytes = (kOffRaw + kRawMaskBytes + 1023) & ~(size_t)1023;
 
-__host__ __device__ constexpr size_t gemm_smem_bytes(int stages, int ring) {
-  return kFixedBytes + (size_t)stages * 2 * kTileBytes +
+// Operand stages: `stages` of the A and B fp16 tiles (32 KB), and with byte
+// operands (split-K partials) `ustages` of their 8 KB byte tiles as TMA wrote
+// them (16 KB), a deeper ring of their own in front of the carrier ring.
+__host__ __device__ constexpr size_t gemm_smem_bytes(int stages, int ring, int ustages = 0) {
+  return kFixedBytes + (size_t)stages * 2 * kTileBytes + (size_t)ustages * kTileBytes +
          (size_t)kPartialEpiWarps * ring * kBoxBytes + 1024;  // + alignment slack
 }
 
@@ -134,6 +139,8 @@ struct GemmArgs {
   int sets;                    // grad_X epilogue sets in use (3 or 4)
   int bw, b2;                  // code bits of W~ and of Q_b2
   int small_p;                 // every |P| < 2^22 (block sums off the fp32 bits)
+  int u8;                      // MODE_PARTIAL: byte operands, widened on chip
+  int ustages;                 // ... through a ring of this many byte stages
   int *status;
 };
 
@@ -1258,6 +1265,108 @@ __device__ __forceinline__ void partial_epilogue(const GemmArgs &g, uint8_t *rin
   __syncwarp();
 }
 
+// ---------------------------------------------------------------------------
+// Byte operands of the split-K partials (both MN-major: K rows of 128 codes).
+// TMA lands each operand's 128 x 64 byte tile in the stage (128-byte rows,
+// 128-byte swizzle); kCvtWarps converter warps widen it into the fp16 carrier
+// tile the MMA reads (two 64-wide swizzle atoms, as the fp16 boxes would
+// land), code - 2^(b-1) exactly, rows past the end of the reduction as 0
+// (a zero byte would widen to -2^(b-1)), then fence the writes for the
+// tensor core and release the stage to the MMA issuer.
+// ---------------------------------------------------------------------------
+constexpr int kCvtWarps = 6;
+
+// Shared-memory offsets of a converter thread's chunks (at most 3 of the
+// 512 16-byte chunks of a 128 x 64 byte tile): the byte chunk, and the two
+// fp16 chunks it widens into.
+struct CvtSlots {
+  int n;
+  uint32_t src[3], dst0[3], dst1[3];
+  int row[3];
+};
+
+__device__ __forceinline__ CvtSlots cvt_slots(int t) {
+  CvtSlots o;
+  o.n = 0;
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    const int c = t + i * kCvtWarps * 32;
+    const int r = c >> 3, j = c & 7, cc = (j & 3) * 2;
+    const uint32_t base = (uint32_t)((j >> 2) * (kTileBytes / 2) + r * 128);
+    o.src[i] = (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4));
+    o.dst0[i] = base + (uint32_t)((cc ^ (r & 7)) << 4);
+    o.dst1[i] = base + (uint32_t)(((cc + 1) ^ (r & 7)) << 4);
+    o.row[i] = r;
+    if (c < 512) o.n = i + 1;
+  }
+  return o;
+}
+
+// codes 16j .. 16j + 15 of a row: fp16 chunks 2 (j mod 4) and 2 (j mod 4) + 1
+// of swizzle atom j / 4; rows from rows_valid on are 0
+__device__ __forceinline__ void widen_tile(const uint8_t *src, uint8_t *dst, int rows_valid,
+                                           __half2 bias, const CvtSlots &o) {
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    if (i >= o.n) break;
+    uint4 lo = make_uint4(0u, 0u, 0u, 0u), hi = lo;
+    if (o.row[i] < rows_valid) {
+      const uint4 v = *reinterpret_cast<const uint4 *>(src + o.src[i]);
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t h[8];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t a = __byte_perm(w[k], 0x6464u, 0x4140);
+        const uint32_t b = __byte_perm(w[k], 0x6464u, 0x4342);
+        __half2 x = __hsub2(*reinterpret_cast<const __half2 *>(&a), bias);
+        __half2 y = __hsub2(*reinterpret_cast<const __half2 *>(&b), bias);
+        h[2 * k] = *reinterpret_cast<uint32_t *>(&x);
+        h[2 * k + 1] = *reinterpret_cast<uint32_t *>(&y);
+      }
+      lo = make_uint4(h[0], h[1], h[2], h[3]);
+      hi = make_uint4(h[4], h[5], h[6], h[7]);
+    }
+    *reinterpret_cast<uint4 *>(dst + o.dst0[i]) = lo;
+    *reinterpret_cast<uint4 *>(dst + o.dst1[i]) = hi;
+  }
+}
+
+// Converter warp cw of kCvtWarps: byte stage su (ring of g.ustages) into
+// carrier stage sf (ring of g.stages), in the producer's K-block order.
+__device__ __noinline__ void partial_convert(const GemmArgs &g, uint8_t *ops, uint8_t *uops,
+                                             uint64_t *full, uint64_t *empty, uint64_t *cvt,
+                                             uint64_t *fempty, volatile int *abort_flag, int cw,
+                                             int lane) {
+  const CvtSlots slots = cvt_slots(cw * 32 + lane);
+  const __half2 bias_a = __half2half2(__int2half_rn(1024 + (1 << (g.bw - 1))));
+  const __half2 bias_b = __half2half2(__int2half_rn(1024 + (1 << (g.b2 - 1))));
+  int su = 0, sf = 0;
+  uint32_t phu = 0, phf = 0;
+  for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
+    const Item tt = decode_item(g, it);
+    for (int64_t kb = tt.kb0; kb < tt.kb1; ++kb) {
+      // the byte tiles have landed, and the MMA is done with the carrier stage
+      bool got = mbar_wait(&full[su], phu, g.status);
+      got = got && mbar_wait(&fempty[sf], phf ^ 1u, g.status);
+      if (!__all_sync(0xffffffffu, got)) { *abort_flag = 1; return; }
+      const uint8_t *us = uops + (size_t)su * kTileBytes;
+      uint8_t *fs = ops + (size_t)sf * 2 * kTileBytes;
+      const int64_t left = g.K - kb * BK;
+      const int rows_valid = left >= BK ? BK : (int)(left > 0 ? left : 0);
+      widen_tile(us, fs, rows_valid, bias_a, slots);
+      widen_tile(us + kTileBytes / 2, fs + kTileBytes, rows_valid, bias_b, slots);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&cvt[sf]);    // the carrier stage is ready for the MMA
+        mbar_arrive(&empty[su]);  // the byte stage is free for the next loads
+      }
+      if (++su == g.ustages) { su = 0; phu ^= 1u; }
+      if (++sf == g.stages) { sf = 0; phf ^= 1u; }
+    }
+  }
+}
+
 // The tiles of this CTA left raw by the fp32-form epilogue (defined with the
 // group fix-up, whose arithmetic it shares).
 template <int NB>
@@ -1274,11 +1383,17 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
   uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
   const int nstages = g.stages;
-  uint8_t *ops = smem + kFixedBytes;                                // operand stages
-  uint8_t *ring = ops + (size_t)nstages * 2 * kTileBytes;          // output boxes
+  const bool u8ops = MODE == MODE_PARTIAL && g.u8 != 0;
+  const int ustages = u8ops ? g.ustages : 0;
+  uint8_t *ops = smem + kFixedBytes;                                // carrier stages
+  uint8_t *uops = ops + (size_t)nstages * 2 * kTileBytes;          // byte stages
+  uint8_t *ring = uops + (size_t)ustages * kTileBytes;             // output boxes
   uint64_t *full = bars, *empty = bars + kMaxStages;
   uint64_t *accf = bars + 2 * kMaxStages, *acce = accf + 4;
   uint64_t *pfull = acce + 4, *pempty = pfull + 4, *drain = pempty + 4;
+  // byte operands: carrier stage widened (converters -> MMA), carrier stage
+  // consumed (MMA -> converters); full / empty then serve the byte ring
+  uint64_t *cvt = bars + 2 * kMaxStages + 17, *fempty = cvt + kMaxStages;
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kNumBars);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
   // grad_X: one accumulator per item, served by 4 epilogue warps (one per
@@ -1294,9 +1409,14 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int i = 0; i < nstages; ++i) {
+    const int nring = u8ops ? ustages : nstages;
+    for (int i = 0; i < nring; ++i) {
       mbar_init(&full[i], 1);
-      mbar_init(&empty[i], 1);
+      mbar_init(&empty[i], u8ops ? kCvtWarps : 1);
+    }
+    for (int i = 0; u8ops && i < nstages; ++i) {
+      mbar_init(&cvt[i], kCvtWarps);
+      mbar_init(&fempty[i], 1);
     }
     for (int i = 0; i < 4; ++i) {
       mbar_init(&accf[i], 1);
@@ -1347,6 +1467,9 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
     }
     else if (warp < kGemmWarpEpi0 + kPartialEpiWarps)
       partial_epilogue(g, ring, accf, acce, tmem, &tmOut, abort_flag, warp, lane);
+    else if (u8ops)  // the four warps after the partial epilogue
+      partial_convert(g, ops, uops, full, empty, cvt, fempty, abort_flag,
+                      2 + warp - (kGemmWarpEpi0 + kPartialEpiWarps), lane);
   } else {
   if constexpr (LY::regs_ctl > 0)
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(LY::regs_ctl));
@@ -1394,10 +1517,20 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
           const Item t = decode_item(g, it);
           for (int64_t kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) { fail(); break; }
-            mbar_expect_tx(&full[s], (uint32_t)(2 * kTileBytes));
+            const int32_t kc = (int32_t)(kb * BK);
+            if (u8ops) {
+              // byte operands (MN-major), into the byte ring: one 128 (MN) x
+              // 64 (K) byte box each
+              uint8_t *ua = uops + (size_t)s * kTileBytes;
+              mbar_expect_tx(&full[s], (uint32_t)kTileBytes);
+              tma_load_2d(ua, &tmA, (int32_t)t.m0, kc, &full[s]);
+              tma_load_2d(ua + kTileBytes / 2, &tmB, (int32_t)t.n0, kc, &full[s]);
+              if (++s == ustages) { s = 0; ph ^= 1u; }
+              continue;
+            }
             uint8_t *sa = ops + (size_t)(2 * s) * kTileBytes;
             uint8_t *sb = sa + kTileBytes;
-            const int32_t kc = (int32_t)(kb * BK);
+            mbar_expect_tx(&full[s], (uint32_t)(2 * kTileBytes));
             // K-major: one 64 x 128 box; MN-major: two 64 (MN) x 64 (K) boxes
             if (g.a_kmajor) {
               tma_load_2d(sa, &tmA, kc, (int32_t)t.m0, &full[s]);
@@ -1421,9 +1554,10 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
       if (*abort_flag) {
         sleep_ns(200000);
       } else {
-        for (int i = 0; i < nstages; ++i) {
+        const int pstages = u8ops ? ustages : nstages;
+        for (int i = 0; i < pstages; ++i) {
           if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) break;
-          if (++s == nstages) { s = 0; ph ^= 1u; }
+          if (++s == pstages) { s = 0; ph ^= 1u; }
         }
       }
     }
@@ -1492,7 +1626,9 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
             tc_fence_after();
             const uint32_t dt = tmem + (uint32_t)(buf * BN);
             for (int64_t kb = c0; kb < c1; ++kb) {
-              if (!mbar_wait(&full[s], ph, g.status)) { fail(); break; }
+              // byte operands: the carrier stage once the converter warps
+              // widened it
+              if (!mbar_wait(u8ops ? &cvt[s] : &full[s], ph, g.status)) { fail(); break; }
               tc_fence_after();
               const uint32_t a_addr = smem_u32(ops + (size_t)(2 * s) * kTileBytes);
               const uint32_t b_addr = a_addr + (uint32_t)kTileBytes;
@@ -1504,7 +1640,7 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
               for (int k = 0; k < BK / 16; ++k)
                 umma_f16(dt, da + a_step * k, db + b_step * k, idesc,
                          (kb > c0 || k > 0) ? 1u : 0u);
-              umma_commit(&empty[s]);
+              umma_commit(u8ops ? &fempty[s] : &empty[s]);
               if (++s == nstages) { s = 0; ph ^= 1u; }
             }
             umma_commit(&accf[buf]);
@@ -1520,6 +1656,9 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
     }
   } else if (warp == kGemmWarpPar) {
     if (MODE == MODE_GRADX) gradx_params<NB, FORM>(g, smem, pfull, pempty, abort_flag, lane);
+    else if (u8ops) partial_convert(g, ops, uops, full, empty, cvt, fempty, abort_flag, 0, lane);
+  } else if (MODE == MODE_PARTIAL && u8ops && warp == kGemmWarpPar + 1) {
+    partial_convert(g, ops, uops, full, empty, cvt, fempty, abort_flag, 1, lane);
   }
   }
 
@@ -1667,6 +1806,20 @@ static bool make_map_f16(CUtensorMap *m, const void *base, uint64_t inner,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map of MN-major byte codes stored as outer (K) rows of inner (MN)
+// bytes: 128 x 64 boxes (one 128-byte row per K row), 128-byte swizzle.
+static bool make_map_u8(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner};
+  cuuint32_t box[2] = {128, BK};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box,
+            es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Output tensor map: fp32 M x N (grad_X) or int32 splits x M x N
 // (partials), 32 x 32 boxes with 128-byte swizzle.
 static bool make_map_out(CUtensorMap *m, void *base, bool is_int, uint64_t cols,
@@ -1808,16 +1961,24 @@ static GemmKernel gemm_kernel(int mode, int nb, int form) {
 // M x K if a_kmajor, else K x M), B is the K x N operand (stored N x K if
 // b_kmajor, else K x N).  Partials: out is splits x M x N int32.  grad_X:
 // out is the N x M fp32 transpose (rows of dH x columns of W~).
-static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
-                           const uint16_t *Bm, int b_kmajor, int b_bits, int64_t M,
-                           int64_t N, int64_t K, const SplitPlan &p, GemmArgs &g,
-                           void *out, int mode, int nb, int form, cudaStream_t st) {
+static fqt_status run_gemm(const void *A, int a_kmajor, int a_bits, const void *Bm,
+                           int b_kmajor, int b_bits, int64_t M, int64_t N, int64_t K,
+                           const SplitPlan &p, GemmArgs &g, void *out, int mode, int nb,
+                           int form, cudaStream_t st) {
   const bool partial = mode == MODE_PARTIAL;
+  // byte operands (g.u8): split-K partials of MN-major operands only
+  if (g.u8 && (!partial || a_kmajor || b_kmajor)) return FQT_EUNSUPPORTED;
   CUtensorMap ta, tb;
-  bool ok = a_kmajor ? make_map_f16(&ta, A, (uint64_t)K, (uint64_t)M, BK, BM)
-                     : make_map_f16(&ta, A, (uint64_t)M, (uint64_t)K, 64, BK);
-  ok = ok && (b_kmajor ? make_map_f16(&tb, Bm, (uint64_t)K, (uint64_t)N, BK, BN)
-                       : make_map_f16(&tb, Bm, (uint64_t)N, (uint64_t)K, 64, BK));
+  bool ok;
+  if (g.u8) {
+    ok = make_map_u8(&ta, A, (uint64_t)M, (uint64_t)K) &&
+         make_map_u8(&tb, Bm, (uint64_t)N, (uint64_t)K);
+  } else {
+    ok = a_kmajor ? make_map_f16(&ta, A, (uint64_t)K, (uint64_t)M, BK, BM)
+                  : make_map_f16(&ta, A, (uint64_t)M, (uint64_t)K, 64, BK);
+    ok = ok && (b_kmajor ? make_map_f16(&tb, Bm, (uint64_t)K, (uint64_t)N, BK, BN)
+                         : make_map_f16(&tb, Bm, (uint64_t)N, (uint64_t)K, 64, BK));
+  }
   CUtensorMap to;
   ok = ok && (partial ? make_map_out(&to, out, true, (uint64_t)N, (uint64_t)M,
                                      (uint64_t)p.splits)
@@ -1847,7 +2008,9 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   g.small_p = (K << (a_bits + b_bits - 2)) < ((int64_t)1 << 22);
   // HBM-bound output tiles (grad_X): deep store ring; long reductions
   // (split-K partials): deep operand ring
-  g.stages = partial ? 5 : 2;
+  // byte operands: two carrier stages fed by a ring of six byte stages
+  g.stages = partial ? (g.u8 ? 2 : 5) : 2;
+  g.ustages = g.u8 ? 6 : 0;
   g.ring = partial ? 1 : 0;  // grad_X stores straight from registers
   // grad_X tiles with a long reduction (K of many blocks: a contraction that
   // is tensor-bound rather than bound by its output) keep more operand
@@ -1885,7 +2048,7 @@ static fqt_status run_gemm(const uint16_t *A, int a_kmajor, int a_bits,
   g.ks_blocks = p.ks_blocks;
   g.kb_total = p.kb_total;
   g.n_items = (int64_t)p.m_tiles * p.n_tiles * p.splits;
-  const size_t smem = gemm_smem_bytes(g.stages, g.ring);
+  const size_t smem = gemm_smem_bytes(g.stages, g.ring, g.ustages);
   const cudaError_t ea =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (ea != cudaSuccess) return cuda_fail(ea, "gemm shared-memory attribute");
@@ -1961,6 +2124,41 @@ fqt_status debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
   g.status = reinterpret_cast<int *>(ws);
   fqt_status s = run_gemm(a16, a_kmajor, a_bits, b16, b_kmajor, b_bits, M, N, K, p,
                           g, part, MODE_PARTIAL, 1, false, st);
+  if (s != FQT_OK) return s;
+  ReduceArgs r;
+  memset(&r, 0, sizeof(r));
+  r.part = part;
+  r.splits = p.splits;
+  r.M = M;
+  r.N = N;
+  r.out_i64 = out;
+  launch_reduce(r, st);
+  return cuda_fail(cudaGetLastError(), "split-K reduce launch");
+}
+
+// The same contraction with both operands MN-major byte codes (A stored
+// K x M, B stored K x N) read as bytes and widened on chip: the path grad_W
+// takes with byte operands.
+fqt_status debug_int_gemm_u8(const uint8_t *A, int a_bits, const uint8_t *Bm, int b_bits,
+                             int64_t M, int64_t N, int64_t K, int64_t *out, void *ws,
+                             size_t ws_bytes, cudaStream_t st) {
+  if (!A || !Bm || !out || M <= 0 || N <= 0 || K <= 0) return FQT_EINVAL;
+  if (a_bits < 2 || a_bits > 8 || b_bits < 2 || b_bits > 8) return FQT_EINVAL;
+  // TMA: byte rows of a multiple of 16 bytes, 16-byte aligned bases
+  if (M % 16 || N % 16) return FQT_EUNSUPPORTED;
+  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX) return FQT_EUNSUPPORTED;
+  if (!aligned16(A) || !aligned16(Bm)) return FQT_EINVAL;
+  const SplitPlan p = plan_splits(M, N, K, a_bits, b_bits, device_sm_count(), true);
+  const size_t part_bytes = round256((size_t)p.splits * (size_t)M * (size_t)N * 4);
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < kGemmOffset + part_bytes)
+    return FQT_EWORKSPACE;
+  int32_t *part = reinterpret_cast<int32_t *>(static_cast<char *>(ws) + kGemmOffset);
+  GemmArgs g;
+  memset(&g, 0, sizeof(g));
+  g.status = reinterpret_cast<int *>(ws);
+  g.u8 = 1;
+  fqt_status s = run_gemm(A, 0, a_bits, Bm, 0, b_bits, M, N, K, p, g, part, MODE_PARTIAL, 1,
+                          false, st);
   if (s != FQT_OK) return s;
   ReduceArgs r;
   memset(&r, 0, sizeof(r));
@@ -3034,13 +3232,19 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     const fqt_qtensor *qa = q_b1 ? q_b1 : q_b2;
     // the shift quantizer feeds grad_W itself: its codes on the common scale
     const bool shifted = qa && qa->kind == FQT_SHIFT;
-    if (!qa || !qx || !qx->codes_f16 || !qx->col_sum || !qx->inv_s || !qx->zero)
+    // byte operands: both code sets given as bytes only (no fp16 carriers);
+    // the split-K kernel widens them on chip
+    const bool bytes = qa && qx && !shifted && !qa->codes_f16 && !qx->codes_f16 && qa->codes &&
+                       qx->codes && qx->conv[0] == 0;
+    if (!qa || !qx || (!qx->codes_f16 && !bytes) || !qx->col_sum || !qx->inv_s || !qx->zero)
       return FQT_EINVAL;
     if (shifted ? (!qa->shift_f16 || !qa->shift_col_sum || !qa->shift_scale)
-                : (!qa->codes_f16 || !qa->col_sum || !qa->inv_s || !qa->zero))
+                : ((!qa->codes_f16 && !bytes) || !qa->col_sum || !qa->inv_s || !qa->zero))
       return FQT_EINVAL;
     if ((!shifted && qa->kind != FQT_PTQ) || qx->kind != FQT_PTQ) return FQT_EINVAL;
-    const uint16_t *A16 = shifted ? qa->shift_f16 : qa->codes_f16;
+    const void *A16 = bytes ? (const void *)qa->codes
+                            : shifted ? (const void *)qa->shift_f16 : (const void *)qa->codes_f16;
+    const void *X16 = bytes ? (const void *)qx->codes : (const void *)qx->codes_f16;
     // |shifted code| <= 16 (2^(b-1) - 1) < 2^(b+3): b + 4 bits of centred magnitude
     const int a_bits = shifted ? qa->bits + 4 : qa->bits;
     // an implicit im2col operand (its padding is corrected in the reduction)
@@ -3049,7 +3253,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     const int64_t Nr = qa->rows, C = qa->cols, D = qx->cols;
     if (qx->rows != Nr) return FQT_EINVAL;
     if (C % 16 || D % 16) return FQT_EUNSUPPORTED;
-    if (!aligned16(A16) || !aligned16(qx->codes_f16)) return FQT_EINVAL;
+    if (!aligned16(A16) || !aligned16(X16)) return FQT_EINVAL;
     if (conv) {
       const int32_t *g = qx->conv;
       const int64_t oh = (int64_t)g[1] + 2 * g[6] - g[4] + 1, ow = (int64_t)g[2] + 2 * g[6] - g[5] + 1;
@@ -3059,7 +3263,8 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
     }
     const SplitPlan p = plan_splits(C, D, Nr, a_bits, x_bits, nsm, true);
     const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, a_bits, x_bits, nsm) : WPlan{};
-    const bool w_ok = use_gradw(wp, nsm);
+    // byte operands take the split-K tile kernel, which widens them
+    const bool w_ok = use_gradw(wp, nsm) && !bytes;
     if (conv && Nr > 0 && !w_ok) return FQT_EUNSUPPORTED;  // the tile kernel reads plain matrices
     const int splits = w_ok ? wp.splits : p.splits;
     const size_t pbytes = (size_t)splits * (size_t)C * (size_t)D * 4;
@@ -3074,20 +3279,22 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       cudaError_t e = cudaMemsetAsync(pad_a, 0, (size_t)C * taps * 4, st);
       if (e != cudaSuccess) return cuda_fail(e, "padding sums clear");
       const int64_t warps = (int64_t)g[0] * taps;
-      k_conv_padsum<<<(int)((warps + 7) / 8), 256, 0, st>>>(A16, (int)C, g[0], g[1], g[2], g[5],
-                                                            g[6], oh, ow, taps, pad_a);
+      k_conv_padsum<<<(int)((warps + 7) / 8), 256, 0, st>>>(
+          static_cast<const uint16_t *>(A16), (int)C, g[0], g[1], g[2], g[5], g[6], oh, ow, taps,
+          pad_a);
       e = cudaGetLastError();
       if (e != cudaSuccess) return cuda_fail(e, "padding sums launch");
     }
     if (Nr > 0 && w_ok) {
-      fqt_status s = run_gradw(qx->codes_f16, A16, Nr, (int)C, (int)D, wp, part, status, st,
-                               conv ? qx->conv : nullptr);
+      fqt_status s = run_gradw(qx->codes_f16, static_cast<const uint16_t *>(A16), Nr, (int)C,
+                               (int)D, wp, part, status, st, conv ? qx->conv : nullptr);
       if (s != FQT_OK) return s;
     } else if (Nr > 0) {
       GemmArgs g;
       memset(&g, 0, sizeof(g));
       g.status = status;
-      fqt_status s = run_gemm(A16, 0, a_bits, qx->codes_f16, 0, qx->bits, C, D, Nr, p, g,
+      g.u8 = bytes ? 1 : 0;
+      fqt_status s = run_gemm(A16, 0, a_bits, X16, 0, qx->bits, C, D, Nr, p, g,
                               part, MODE_PARTIAL, 1, false, st);
       if (s != FQT_OK) return s;
     } else {

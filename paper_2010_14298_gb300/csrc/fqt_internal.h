@@ -121,5 +121,8 @@ fqt_status debug_int_gemm(const uint8_t *A, int a_kmajor, int a_bits,
                           const uint8_t *Bm, int b_kmajor, int b_bits, int64_t M,
                           int64_t N, int64_t K, int64_t *out, void *ws,
                           size_t ws_bytes, cudaStream_t st);
+fqt_status debug_int_gemm_u8(const uint8_t *A, int a_bits, const uint8_t *Bm, int b_bits,
+                             int64_t M, int64_t N, int64_t K, int64_t *out, void *ws,
+                             size_t ws_bytes, cudaStream_t st);
 
 }  // namespace fqt

@@ -106,6 +106,8 @@ def load(build_if_missing: bool = True):
         lib.fqt_debug_int_gemm.argtypes = [P, i32, i32, P, i32, i32, i64, i64,
                                            i64, P, P, sz, P]
         lib.fqt_debug_int_gemm.restype = i32
+        lib.fqt_debug_int_gemm_u8.argtypes = [P, i32, P, i32, i64, i64, i64, P, P, sz, P]
+        lib.fqt_debug_int_gemm_u8.restype = i32
         lib.fqt_status_string.argtypes = [i32]
         lib.fqt_status_string.restype = ctypes.c_char_p
         lib.fqt_last_cuda_error.argtypes = []
@@ -503,6 +505,23 @@ def debug_int_gemm(A: torch.Tensor, a_kmajor: bool, a_bits: int, B: torch.Tensor
                                 int(b_kmajor), b_bits, M, N, K, _ptr(out), ws.ptr,
                                 ws.nbytes, _stream(stream))
     _check(st, "fqt_debug_int_gemm")
+    return out
+
+
+def debug_int_gemm_u8(A: torch.Tensor, a_bits: int, B: torch.Tensor, b_bits: int, M: int,
+                      N: int, K: int, ws: Workspace = None, stream=None) -> torch.Tensor:
+    """debug_int_gemm with both operands MN-major bytes (A: K x M, B: K x N),
+    widened to fp16 carriers on chip (grad_W's byte-operand path)."""
+    lib = load()
+    out = torch.empty((M, N), dtype=torch.int64, device=A.device)
+    need = int(lib.fqt_debug_workspace_size(M, N, K))
+    if ws is None or ws.nbytes < need:
+        ws = Workspace(1, 16, 16, device=A.device)
+        ws.nbytes = need
+        ws.buf = torch.zeros(need, dtype=torch.uint8, device=A.device)
+    st = lib.fqt_debug_int_gemm_u8(_ptr(A), a_bits, _ptr(B), b_bits, M, N, K, _ptr(out),
+                                   ws.ptr, ws.nbytes, _stream(stream))
+    _check(st, "fqt_debug_int_gemm_u8")
     return out
 
 

@@ -70,6 +70,70 @@ def test_int_gemm_exact_at_extreme_magnitudes(K, fill):
     assert (got.cpu().numpy() == expect).all()
 
 
+U8_GEMM_CASES = [
+    # M, N, K, a_bits, b_bits: byte operands widened on chip (MN-major both)
+    (64, 576, 5000, 8, 8),     # grad_W shape, split-K, exact chunks, K tail of 8 rows
+    (128, 128, 64, 8, 8),
+    (256, 160, 1040, 8, 4),    # ragged N tile, K tail of 16
+    (48, 32, 16, 2, 8),        # one partial K block
+    (96, 208, 3000, 5, 8),     # ragged M and N tiles
+    (1024, 64, 777, 8, 8),
+]
+
+
+@pytest.mark.parametrize("M,N,K,ab,bb", U8_GEMM_CASES)
+def test_int_gemm_u8_operands_bit_exact(M, N, K, ab, bb):
+    """The split-K kernel reading byte codes and widening them on chip
+    (grad_W's byte-operand path): bit-exact against the oracle's integer
+    contraction, including K blocks past the end of the reduction (zero rows,
+    where a zero byte would widen to -2^(b-1))."""
+    g = wl.rng(M * 5 + N * 11 + K)
+    A = g.integers(0, 1 << ab, (K, M)).astype(np.uint8)   # K x M (MN-major)
+    B = g.integers(0, 1 << bb, (K, N)).astype(np.uint8)   # K x N (MN-major)
+    got = fqt.debug_int_gemm_u8(torch.from_numpy(A).cuda(), ab, torch.from_numpy(B).cuda(), bb,
+                                M, N, K)
+    ref = orc.int_gemm(A, 0, B, 0, M, N, K, 1 << (ab - 1), 1 << (bb - 1))
+    assert np.array_equal(got.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("K", [1024, 4096, 8192 + 64])
+@pytest.mark.parametrize("fill", [(255, 255), (0, 0), (0, 255)])
+def test_int_gemm_u8_exact_at_extreme_magnitudes(K, fill):
+    M, N = 128, 128
+    A = np.full((K, M), fill[0], dtype=np.uint8)
+    B = np.full((K, N), fill[1], dtype=np.uint8)
+    got = fqt.debug_int_gemm_u8(torch.from_numpy(A).cuda(), 8, torch.from_numpy(B).cuda(), 8,
+                                M, N, K)
+    expect = K * (int(fill[0]) - 128) * (int(fill[1]) - 128)
+    assert (got.cpu().numpy() == expect).all()
+
+
+@pytest.mark.parametrize("cfg", ["ffn-up", "conv"])
+def test_grad_w_byte_operands_equal_carriers(cfg):
+    """grad_W from byte-only code sets (Q_b1 and X~ without fp16 carriers)
+    equals grad_W from the carriers bit for bit: the same exact integer
+    partials, the same reduction."""
+    g = wl.rng(808)
+    if cfg == "ffn-up":
+        n, c, d = 4096, 1024, 512
+    else:
+        n, c, d = 20000, 64, 576
+    dH = wl.random_grad(g, n, c, sigma=1.0)
+    X = g.uniform(-1, 1, (n, d)).astype(np.float32)
+    dev = lambda a: to_dev(a, "f32")
+    qx_c = fqt.quantize_act(dev(X), 8)
+    q2, q1_c = fqt.quantize_grad(dev(dH), orc.BHQ, 5, 16, 17)
+    qx_b = fqt.QTensor.empty(n, d, orc.PTQ, 8, 0, False, True, "cuda", u8=True, f16=False)
+    fqt.quantize_act(dev(X), 8, out=qx_b)
+    q1_b = fqt.QTensor.empty(n, c, orc.PTQ, 8, 0, False, True, "cuda", u8=True, f16=False)
+    fqt.quantize_grad(dev(dH), orc.BHQ, 5, 16, 17, q_b2=q2, q_b1=q1_b)
+    _, gw_c = fqt.linear_backward(q2, q1_c, qx_c, None, grad_x=False, grad_w=True)
+    _, gw_b = fqt.linear_backward(q2, q1_b, qx_b, None, grad_x=False, grad_w=True)
+    torch.cuda.synchronize()
+    assert torch.equal(q1_b.codes, q1_c.codes) if q1_c.codes is not None else True
+    assert torch.equal(gw_b, gw_c)
+
+
 # --------------------------------------------------------------------------
 # Quantizers
 # --------------------------------------------------------------------------
