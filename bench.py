@@ -678,6 +678,7 @@ def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
     # carriers: the shift quantizer's and the implicit im2col's grad_W pair
     # these operands with fp16 operands of their own
     base = LayerState(fqt, dH, X, W, ws, byte_operands=False)
+    per_base = time_graphs(base.calls())
     # grad_W's byte-operand path on the same layer (1-byte X~ and Q_b1)
     byt = LayerState(fqt, dH, X, W, ws, byte_operands=True)
     per_byt = time_graphs(byt.calls())
@@ -687,7 +688,6 @@ def run_extras(args, fqt, wl, dev, stream, hbm_peak, bf16_peak):
         "per_call_ms": dict(zip(CALLS, per_byt)),
         "carriers_per_call_ms": dict(zip(CALLS, per_base)),
         "device_status": fqt.sync_status(ws)}
-    per_base = time_graphs(base.calls())
     qa = fqt.QTensor.empty(N, C, fqt.BHQ, BITS, 0, True, False, dev, u8=False)
     qa1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=False)
     pa = time_graphs([
