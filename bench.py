@@ -41,8 +41,8 @@ KIND, BITS, BLOCK = 2, 5, 16  # Q_b2 = BHQ-5, block 16
 SWEEP_BATCH = 256
 CALLS = ["quantize_act", "quantize_weight", "quantize_grad", "grad_x", "grad_w"]
 KERNELS = {"quantize_act": "k_range + k_fwd_codes", "quantize_weight": "k_range + k_fwd_codes",
-           "quantize_grad": "k_range + k_bhq_warp", "grad_x": "k_gemm",
-           "grad_w": "k_gradw (or split-K k_gemm) + k_reduce"}
+           "quantize_grad": "k_bhq_stats + k_bhq_codes + k_bhq_offsets", "grad_x": "k_gemm",
+           "grad_w": "split-K k_gemm + k_reduce"}
 
 
 def _peaks():
@@ -207,10 +207,14 @@ def alg_bytes(N: int, C: int, D: int, eb: int = 4, block: int = BLOCK) -> dict:
 
 
 def launches(C: int, kind: int = KIND, block: int = BLOCK) -> dict:
-    """Kernels each call launches (fixed by the library's dispatch)."""
-    warp_bhq = kind == KIND and block > 0 and C in (64, 128, 256)
+    """Kernels each call launches (fixed by the library's dispatch): Q_f and
+    Q_theta are a range pass and a code pass; the fixed-block BHQ quantizer on
+    the widths of its two-pass form is a statistics pass, a code pass and the
+    grad_X offsets, on other widths a range pass and one fused pass; grad_X
+    is one contraction, grad_W the split-K contraction and its reduction."""
+    two_pass = kind == KIND and block in (4, 8, 16) and C in (64, 128, 256, 512, 1024, 2048, 4096)
     return {"quantize_act": 2, "quantize_weight": 2,
-            "quantize_grad": 2 if (warp_bhq or kind != KIND) else 3,
+            "quantize_grad": 3 if two_pass else 2,
             "grad_x": 1, "grad_w": 2}
 
 
@@ -441,11 +445,13 @@ def run_gpu(args):
     roofline = {"bound": r["bound"], "achieved": r["achieved"], "peak": r["peak"],
                 "unit": r["unit"], "frac": r["frac"],
                 "traffic": _traffic_record("k_gemm", "resnet50-sweep-b256"),
+                "algorithmic_bytes": r.get("algorithmic_bytes"),
                 "kernel": "k_gemm", "call": dom, "peak_source": peak_src,
                 "launches": r["launches"],
-                "per_launch": ("algorithmic bytes (1 byte per code) and CUDA-event time summed "
-                               f"over the {r['launches']} {r['bound']}-bound grad_X launches of "
-                               "the step")}
+                "per_launch": ("algorithmic bytes (1 byte per code), DRAM traffic (ncu "
+                               "dram__bytes_read.sum + dram__bytes_write.sum) and CUDA-event "
+                               f"time summed over the {r['launches']} {r['bound']}-bound grad_X "
+                               "launches of the step")}
     slow = sorted(range(nl), key=lambda li: -per[li].sum())[:6]
     result = {
         "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
