@@ -7,9 +7,13 @@ im2col; 4.19 TOP of integer contractions):  for every layer
   Q_b2(dH) = BHQ 5-bit, block 16; Q_b1(dH) = 8-bit stochastic PTQ
   grad_X = Q_b2(dH) W~,  grad_W = Q_b1(dH)^T X~
 The reported value is quantized-backward throughput in TOPS: both
-contractions count 2 N C D integer ops each.  Every layer's inputs (34 GB of
-fp32 dH, X, W) are resident in HBM when timing starts; a step moves far more
-than the 129 MB L2, so no flush is needed between steps.
+contractions count 2 N C D integer ops each.  The stride-1 3 x 3 convolutions
+(13 of them) are lowered to their implicit im2col matrix: X stays the NHWC
+input, Q_f reads it once and grad_W reads the codes at each tap's offset (the
+codes, the contractions and the gradients are those of the explicit im2col
+matrix, bit for bit).  Every layer's inputs (fp32 dH, X, W) are resident in
+HBM when timing starts; a step moves far more than the 129 MB L2, so no flush
+is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
@@ -206,28 +210,51 @@ def alg_bytes(N: int, C: int, D: int, eb: int = 4, block: int = BLOCK) -> dict:
     }
 
 
-def launches(C: int, kind: int = KIND, block: int = BLOCK) -> dict:
+def launches(C: int, kind: int = KIND, block: int = BLOCK, implicit: bool = False) -> dict:
     """Kernels each call launches (fixed by the library's dispatch): Q_f and
     Q_theta are a range pass and a code pass; the fixed-block BHQ quantizer on
     the widths of its two-pass form is a statistics pass, a code pass and the
     grad_X offsets, on other widths a range pass and one fused pass; grad_X
-    is one contraction, grad_W the split-K contraction and its reduction."""
+    is one contraction, grad_W the split-K contraction and its reduction; an
+    implicit im2col X~ adds the column sums to Q_f and the padding sums to
+    grad_W."""
     two_pass = kind == KIND and block in (4, 8, 16) and C in (64, 128, 256, 512, 1024, 2048, 4096)
-    return {"quantize_act": 2, "quantize_weight": 2,
+    return {"quantize_act": 3 if implicit else 2, "quantize_weight": 2,
             "quantize_grad": 3 if two_pass else 2,
-            "grad_x": 1, "grad_w": 2}
+            "grad_x": 1, "grad_w": 3 if implicit else 2}
 
 
-def sweep_layer_tensors(sh, batch: int, seed: int, dev):
+def implicit_ok(sh) -> bool:
+    """A stride-1 3 x 3 conv whose grad_W reads the implicit im2col X~ (the
+    NHWC input, read once by Q_f) in blocks of whole output rows."""
+    ow = sh.hout
+    return (sh.k == 3 and sh.stride == 1 and sh.pad == 1 and sh.cin % 64 == 0 and
+            sh.D_pad == sh.D and (ow <= 64 or ow % 32 == 0))
+
+
+def sweep_layer_tensors(sh, batch: int, seed: int, dev, implicit: bool = False):
     """One layer of the sweep drawn on the device with torch's seeded
     generator: the recipe of workloads.resnet50_layer (input U[-1, 1] at the
     layer's input shape lowered by im2col, dH N(0, 1) rows scaled by
-    lognormal(0, 2), W N(0, 2 / D); D and C zero-padded to multiples of 16)."""
+    lognormal(0, 2), W N(0, 2 / D); D and C zero-padded to multiples of 16).
+    implicit: X is the NHWC input itself (its im2col matrix is the operand,
+    never formed)."""
     import torch
     import torch.nn.functional as F
     gen = torch.Generator(device=dev)
     gen.manual_seed(seed)
     Ns, Dp, Cp = sh.rows(batch), sh.D_pad, sh.C_pad
+    if implicit:
+        x = torch.rand((batch, sh.cin, sh.h, sh.h), generator=gen, device=dev) * 2.0 - 1.0
+        X = x.permute(0, 2, 3, 1).contiguous()
+        del x
+        dH = torch.zeros((Ns, Cp), dtype=torch.float32, device=dev)
+        dH[:, :sh.cout] = (torch.randn((Ns, sh.cout), generator=gen, device=dev)
+                           * torch.exp(2.0 * torch.randn((Ns, 1), generator=gen, device=dev)))
+        W = torch.zeros((Cp, Dp), dtype=torch.float32, device=dev)
+        W[:sh.cout, :sh.D] = (torch.randn((sh.cout, sh.D), generator=gen, device=dev)
+                              * float(np.sqrt(2.0 / sh.D)))
+        return dH, X, W
     X = torch.zeros((Ns, Dp), dtype=torch.float32, device=dev)
     # im2col in slices of the batch (the unfolded tensor of a whole layer can
     # exceed 2 GB)
@@ -259,7 +286,10 @@ class LayerState:
                  byte_operands=False):
         dev = dH.device
         N, C = dH.shape
-        D = X.shape[1]
+        # X: a matrix (N x D), or an NHWC conv input (n, h, w, c) read as its
+        # implicit im2col matrix (3 x 3 taps, pad 1)
+        self.implicit = X.dim() == 4
+        D = 9 * X.shape[3] if self.implicit else X.shape[1]
         self.N, self.C, self.D = N, C, D
         self.dH, self.X, self.W = dH, X, W
         self.kind, self.bits, self.block, self.seed = kind, bits, block, seed
@@ -267,7 +297,8 @@ class LayerState:
         # contraction) or as fp16 carriers (the default: faster end to end, the
         # widening binds the contraction)
         b = byte_operands
-        self.qx = fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=b, f16=not b)
+        self.qx = (fqt.quantize_act_conv(X, 3, 3, 1, 8, ws=ws) if self.implicit else
+                   fqt.QTensor.empty(N, D, fqt.PTQ, 8, 0, False, True, dev, u8=b, f16=not b))
         self.qw = fqt.QTensor.empty(C, D, fqt.PTQ, 8, 0, False, True, dev, u8=False)
         self.q2 = fqt.QTensor.empty(N, C, kind, bits, block, True, False, dev, u8=False)
         self.q1 = fqt.QTensor.empty(N, C, fqt.PTQ, 8, 0, False, True, dev, u8=b, f16=not b)
@@ -284,8 +315,10 @@ class LayerState:
         gx = self.gx if gx is None else gx
         gw = self.gw if gw is None else gw
         seed = self.seed if seed is None else seed
+        qa = ((lambda: f.quantize_act_conv(X, 3, 3, 1, 8, ws=ws, out=self.qx)) if self.implicit
+              else (lambda: f.quantize_act(X, 8, ws=ws, out=self.qx)))
         return [
-            lambda: f.quantize_act(X, 8, ws=ws, out=self.qx),
+            qa,
             lambda: f.quantize_weight(W, 8, ws=ws, out=self.qw),
             lambda: f.quantize_grad(dH, self.kind, self.bits, self.block, seed, ws=ws,
                                     q_b2=self.q2, q_b1=self.q1),
@@ -370,13 +403,18 @@ def run_gpu(args):
     ws = fqt.Workspace(big.rows(B), big.C_pad, big.D_pad, device=dev)  # calls run in order
     layers = []
     for li, sh in enumerate(shapes):
-        dH, X, W = sweep_layer_tensors(sh, B, rank_seed(rank, li), dev)
+        dH, X, W = sweep_layer_tensors(sh, B, rank_seed(rank, li), dev,
+                                       implicit=implicit_ok(sh))
         layers.append(LayerState(fqt, dH, X, W, ws))
     nl = len(layers)
     ops_layer = [4 * sh.rows(B) * sh.cout * sh.D for sh in shapes]
     ops_step = sum(ops_layer)
     byt = [alg_bytes(L.N, L.C, L.D) for L in layers]
-    nlaunch = sum(sum(launches(L.C).values()) for L in layers)
+    for L, b in zip(layers, byt):
+        if L.implicit:  # Q_f reads the NHWC input once and writes its codes
+            px = L.X.numel()
+            b["quantize_act"] = px * 4 + px + L.D * 4 + 8
+    nlaunch = sum(sum(launches(L.C, implicit=L.implicit).values()) for L in layers)
 
     for _ in range(args.warmup):
         for L in layers:
@@ -463,7 +501,12 @@ def run_gpu(args):
                    "quantizer": "Q_b2=BHQ-5 block16, Q_b1=PTQ-8 stochastic, X~/W~=PTQ-8",
                    "ops_per_step": ops_step,
                    "parallelism": f"replicas x{world} (independent batches)",
-                   "l2": "no flush: inputs larger than L2 (a step reads 34 GB of fp32 inputs)",
+                   "lowering": (f"{sum(L.implicit for L in layers)} stride-1 3x3 convs as "
+                                "implicit im2col (NHWC input read once), the rest as "
+                                "materialized im2col matrices"),
+                   "l2": ("no flush: inputs larger than L2 (a step reads "
+                          f"{sum(4 * (L.dH.numel() + L.X.numel() + L.W.numel()) for L in layers) / 1e9:.1f}"
+                          " GB of fp32 inputs)"),
                    "launch": "one CUDA graph per C-ABI call, events between calls",
                    "wall_s": t_wall},
         "roofline": roofline,

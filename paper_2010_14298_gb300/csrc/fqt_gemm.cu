@@ -141,6 +141,12 @@ struct GemmArgs {
   int small_p;                 // every |P| < 2^22 (block sums off the fp32 bits)
   int u8;                      // MODE_PARTIAL: byte operands, widened on chip
   int ustages;                 // ... through a ring of this many byte stages
+  // MODE_PARTIAL with an implicit im2col X~ (stride 1): K blocks of 64
+  // output-pixel slots = rpb output rows of pw slots (pw >= ow, the slots
+  // past ow zero); A (Q_b1) and B (the NHWC codes at each tap's offset) are
+  // read as 4-D boxes of (64 channels, pw, rpb, 1)
+  int conv, cpw, crpb, cybi, coh, cih, cin, ckw, cpad, cow, ciw;
+  int64_t cnimg;
   int *status;
 };
 
@@ -1531,6 +1537,29 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
             uint8_t *sa = ops + (size_t)(2 * s) * kTileBytes;
             uint8_t *sb = sa + kTileBytes;
             mbar_expect_tx(&full[s], (uint32_t)(2 * kTileBytes));
+            if (MODE == MODE_PARTIAL && g.conv) {
+              // implicit im2col: K block kb = output rows rpb yb .. of image
+              // img, slots 0 .. pw - 1 of each; Q_b1 rows at those pixels,
+              // X~ columns n0 .. n0 + 127 = (tap, 64 channels) pairs read at
+              // the tap's offset (outside the input: zeros, the padding)
+              const int img = (int)(kb / g.cybi);
+              const int oy0 = (int)(kb - (int64_t)img * g.cybi) * g.crpb;
+              tma_load_4d(sa, &tmA, (int32_t)t.m0, 0, oy0, img, &full[s]);
+              tma_load_4d(sa + kTileBytes / 2, &tmA, (int32_t)t.m0 + 64, 0, oy0, img, &full[s]);
+              for (int h = 0; h < 2; ++h) {
+                const int64_t d = t.n0 + 64 * h;
+                const int tap = (int)(d / g.cin), cg = (int)(d - (int64_t)tap * g.cin);
+                const int ky = tap / g.ckw, kx = tap - ky * g.ckw;
+                if (d < g.N)
+                  tma_load_4d(sb + h * (kTileBytes / 2), &tmB, cg, kx - g.cpad, oy0 + ky - g.cpad,
+                              img, &full[s]);
+                else  // past the last tap: a box outside the tensor (zeros)
+                  tma_load_4d(sb + h * (kTileBytes / 2), &tmB, 0, 0, g.cih + g.coh + 8, img,
+                              &full[s]);
+              }
+              if (++s == nstages) { s = 0; ph ^= 1u; }
+              continue;
+            }
             // K-major: one 64 x 128 box; MN-major: two 64 (MN) x 64 (K) boxes
             if (g.a_kmajor) {
               tma_load_2d(sa, &tmA, kc, (int32_t)t.m0, &full[s]);
@@ -1806,6 +1835,22 @@ static bool make_map_f16(CUtensorMap *m, const void *base, uint64_t inner,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 4-D map of NHWC-ordered fp16 carriers (c, w, h, n) with boxes of 64
+// channels x bw pixels x bh rows x 1 image, 128-byte swizzle: the image of a
+// (bw bh) x 64 MN-major operand tile (one 128-byte row per pixel).
+static bool make_map_f16_box4(CUtensorMap *m, const void *base, uint64_t n, uint64_t h,
+                              uint64_t w, uint64_t c, uint32_t bw, uint32_t bh) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {c, w, h, n};
+  cuuint64_t strides[3] = {c * 2, w * c * 2, h * w * c * 2};
+  cuuint32_t box[4] = {64, bw, bh, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void *>(base), dims, strides,
+            box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Tensor map of MN-major byte codes stored as outer (K) rows of inner (MN)
 // bytes: 128 x 64 boxes (one 128-byte row per K row), 128-byte swizzle.
 static bool make_map_u8(CUtensorMap *m, const void *base, uint64_t inner, uint64_t outer) {
@@ -1903,7 +1948,11 @@ size_t gemm_workspace_bytes(int64_t N, int64_t C, int64_t D) {
   int64_t splits = 0;
   for (int b = 2; b <= 12; ++b) {
     const WPlan w = gradw_plan(N, C, D, b, 8, nsm);
-    const int64_t sp = use_gradw(w, nsm) ? w.splits : plan_splits(C, D, N, b, 8, nsm, true).splits;
+    int64_t sp = use_gradw(w, nsm) ? w.splits : plan_splits(C, D, N, b, 8, nsm, true).splits;
+    // an implicit im2col operand pads each image's output rows to blocks of
+    // 64 slots: at most 2.4 N slots (ow = 9 in blocks of 4 rows of 16)
+    const int64_t sc = plan_splits(C, D, (N * 5 + 1) / 2, b, 8, nsm, true).splits;
+    if (sc > sp) sp = sc;
     if (sp > splits) splits = sp;
   }
   // + the padding table of an implicit im2col X~ (C x taps, taps <= D)
@@ -1973,6 +2022,14 @@ static fqt_status run_gemm(const void *A, int a_kmajor, int a_bits, const void *
   if (g.u8) {
     ok = make_map_u8(&ta, A, (uint64_t)M, (uint64_t)K) &&
          make_map_u8(&tb, Bm, (uint64_t)N, (uint64_t)K);
+  } else if (g.conv) {
+    // implicit im2col (split-K partials, both MN-major): Q_b1 as (C, ow, oh,
+    // n), the NHWC codes as (cin, iw, ih, n)
+    if (!partial || a_kmajor || b_kmajor) return FQT_EUNSUPPORTED;
+    ok = make_map_f16_box4(&ta, A, (uint64_t)g.cnimg, (uint64_t)g.coh, (uint64_t)g.cow,
+                           (uint64_t)M, (uint32_t)g.cpw, (uint32_t)g.crpb) &&
+         make_map_f16_box4(&tb, Bm, (uint64_t)g.cnimg, (uint64_t)g.cih, (uint64_t)g.ciw,
+                           (uint64_t)g.cin, (uint32_t)g.cpw, (uint32_t)g.crpb);
   } else {
     ok = a_kmajor ? make_map_f16(&ta, A, (uint64_t)K, (uint64_t)M, BK, BM)
                   : make_map_f16(&ta, A, (uint64_t)M, (uint64_t)K, 64, BK);
@@ -3259,16 +3316,44 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       const int64_t oh = (int64_t)g[1] + 2 * g[6] - g[4] + 1, ow = (int64_t)g[2] + 2 * g[6] - g[5] + 1;
       if (oh <= 0 || ow <= 0 || (int64_t)g[0] * oh * ow != Nr || (int64_t)g[4] * g[5] * g[3] != D)
         return FQT_EINVAL;
-      if (g[3] % 64 || ow % kWBK) return FQT_EUNSUPPORTED;
+      // 64-channel boxes; rows of up to 64 pixels (the tile kernel) or of a
+      // multiple of 32 (k_gradw)
+      if (g[3] % 64 || (ow > 64 && ow % kWBK)) return FQT_EUNSUPPORTED;
     }
-    const SplitPlan p = plan_splits(C, D, Nr, a_bits, x_bits, nsm, true);
+    // An implicit im2col operand with output rows of at most 64 pixels takes
+    // the split-K tile kernel too: K blocks of 64 slots are rpb = 64 / pw
+    // whole output rows of pw (the power of two >= ow) slots, the slots past
+    // ow and the rows past oh zero in Q_b1 (out of its bounds), so K runs over
+    // n ceil(oh / rpb) 64 slots.
+    int cpw = 0, crpb = 0, cybi = 0;
+    int64_t Kt = Nr;
+    if (conv) {
+      const int32_t *g = qx->conv;
+      const int ow = g[2] + 2 * g[6] - g[5] + 1, oh = g[1] + 2 * g[6] - g[4] + 1;
+      if (ow <= 64 && !bytes) {
+        cpw = 8;
+        while (cpw < ow) cpw *= 2;
+        crpb = 64 / cpw;
+        cybi = (oh + crpb - 1) / crpb;
+        Kt = (int64_t)g[0] * cybi * 64;
+        // the workspace holds the partials of at most 2.5 N slots (tiny
+        // images would pad far beyond)
+        if (2 * Kt > 5 * Nr) {
+          cpw = crpb = cybi = 0;
+          Kt = Nr;
+        }
+      }
+    }
+    const bool conv_tile = cpw > 0;
+    const SplitPlan p = plan_splits(C, D, Kt, a_bits, x_bits, nsm, true);
     const WPlan wp = Nr > 0 ? gradw_plan(Nr, C, D, a_bits, x_bits, nsm) : WPlan{};
-    // k_gradw serves the implicit im2col operand (4-D boxes of the NHWC
-    // codes); plain matrices take the split-K tile kernel, which measured
-    // faster wherever both apply (e.g. 66.7 against 110.8 us on a 200704 x
-    // 128 x 512 layer) and widens byte operands
-    const bool w_ok = use_gradw(wp, nsm) && conv;
-    if (conv && Nr > 0 && !w_ok) return FQT_EUNSUPPORTED;  // the tile kernel reads plain matrices
+    // k_gradw serves the implicit im2col operand with wider output rows (4-D
+    // boxes of 32 pixels of one row, ow % 32 == 0); plain matrices take the
+    // split-K tile kernel, which measured faster wherever both apply (e.g.
+    // 66.7 against 110.8 us on a 200704 x 128 x 512 layer) and widens byte
+    // operands
+    const bool w_ok = use_gradw(wp, nsm) && conv && !conv_tile;
+    if (conv && Nr > 0 && !w_ok && !conv_tile) return FQT_EUNSUPPORTED;
     const int splits = w_ok ? wp.splits : p.splits;
     const size_t pbytes = (size_t)splits * (size_t)C * (size_t)D * 4;
     const int taps = conv ? qx->conv[4] * qx->conv[5] : 0;
@@ -3297,7 +3382,22 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       memset(&g, 0, sizeof(g));
       g.status = status;
       g.u8 = bytes ? 1 : 0;
-      fqt_status s = run_gemm(A16, 0, a_bits, X16, 0, qx->bits, C, D, Nr, p, g,
+      if (conv_tile) {
+        const int32_t *cv = qx->conv;
+        g.conv = 1;
+        g.cpw = cpw;
+        g.crpb = crpb;
+        g.cybi = cybi;
+        g.cnimg = cv[0];
+        g.cih = cv[1];
+        g.ciw = cv[2];
+        g.cin = cv[3];
+        g.ckw = cv[5];
+        g.cpad = cv[6];
+        g.coh = cv[1] + 2 * cv[6] - cv[4] + 1;
+        g.cow = cv[2] + 2 * cv[6] - cv[5] + 1;
+      }
+      fqt_status s = run_gemm(A16, 0, a_bits, X16, 0, qx->bits, C, D, Kt, p, g,
                               part, MODE_PARTIAL, 1, false, st);
       if (s != FQT_OK) return s;
     } else {

@@ -882,6 +882,32 @@ def test_conv_grad_w_equals_the_explicit_path(batch):
     assert grad_rel_err(gwc[:, cols], ref) <= GRAD_TOL
 
 
+@pytest.mark.parametrize("n,h,w,cin,cout", [(2, 56, 56, 64, 64), (3, 28, 28, 128, 128),
+                                             (4, 14, 14, 64, 256), (5, 7, 7, 128, 64),
+                                             (2, 9, 11, 64, 128), (1, 64, 64, 64, 64),
+                                             (2, 12, 96, 64, 64)])
+def test_conv_grad_w_rows_in_blocks_equal_the_explicit_path(n, h, w, cin, cout):
+    """The implicit im2col X~ in the split-K tile kernel at the output-row
+    widths of ResNet-50's 3 x 3 layers (56, 28, 14, 7) and ragged ones: K
+    blocks of whole output rows padded to a power of two (64 / 32 / 16 / 8
+    slots, rows past oh and slots past ow zero), bit for bit the explicit
+    im2col grad_W; ow = 96 takes the one-range-per-CTA kernel."""
+    g = wl.rng(n * h * w + cin + cout)
+    x = g.uniform(-1, 1, (n, h, w, cin)).astype(np.float32)
+    xi = wl.im2col_nhwc(x, 3, 3, 1, 1)
+    N, D = xi.shape
+    dH = g.standard_normal((N, cout)).astype(np.float32)
+    dH[g.random(N) < 0.02] *= 50.0
+    q2, q1 = fqt.quantize_grad(to_dev(dH), orc.BHQ, 5, 16, seed=9)
+    ws = fqt.Workspace(N, cout, D)
+    qx = fqt.quantize_act(to_dev(xi), 8)
+    qc = fqt.quantize_act_conv(to_dev(x), 3, 3, 1, 8)
+    _, gw = fqt.linear_backward(q2, q1, qx, None, grad_x=False, ws=ws)
+    _, gwc = fqt.linear_backward(q2, q1, qc, None, grad_x=False, ws=ws)
+    assert fqt.sync_status(ws) == 0
+    assert torch.equal(gw, gwc)
+
+
 # --------------------------------------------------------------------------
 # Unbiasedness of the GPU quantizers over seeds (Sec. 3.3, 4.1-4.3; the
 # premise of Thm 1): the mean of the dequantized GPU codes is dH, with the
