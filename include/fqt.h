@@ -151,7 +151,7 @@ FQT_API fqt_status fqt_quantize_act(const void *X, fqt_dtype dtype, int64_t rows
  * be NULL.  c % 8 == 0, c <= 4096.  The workspace holds the status word and range
  * partials only (fqt_workspace_size(n h w, c, 16) bytes suffice).
  * fqt_linear_backward reads such an operand as qx for grad_W (stride 1,
- * c % 64 == 0, and ow <= 64 or ow % 32 == 0): rows of up to 64 output
+ * c % 64 == 0, pad <= 17, and ow <= 64 or ow % 32 == 0): rows of up to 64 output
  * pixels go to the split-K tile kernel in blocks of whole output rows,
  * wider rows to the one-range-per-CTA kernel.
  */

@@ -26,6 +26,7 @@
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math.h>
+#include <algorithm>
 #include <string.h>
 
 #include "fqt_common.cuh"
@@ -1521,6 +1522,23 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
       } else {
         for (int64_t it = blockIdx.x; it < g.n_items && !*abort_flag; it += gridDim.x) {
           const Item t = decode_item(g, it);
+          // implicit im2col: the item's two (tap, channel group) columns of
+          // X~ and its first block's (image, row group), then advanced per
+          // K block without divisions
+          int cimg = 0, cyb = 0, ccg[2] = {0, 0}, ckx[2] = {0, 0}, cky[2] = {0, 0};
+          bool cval[2] = {false, false};
+          if (MODE == MODE_PARTIAL && g.conv) {
+            cimg = (int)(t.kb0 / g.cybi);
+            cyb = (int)(t.kb0 - (int64_t)cimg * g.cybi);
+            for (int h = 0; h < 2; ++h) {
+              const int d = (int)t.n0 + 64 * h;
+              const int tap = d / g.cin;
+              ccg[h] = d - tap * g.cin;
+              cky[h] = tap / g.ckw;
+              ckx[h] = tap - cky[h] * g.ckw;
+              cval[h] = d < g.N;
+            }
+          }
           for (int64_t kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(&empty[s], ph ^ 1u, g.status)) { fail(); break; }
             const int32_t kc = (int32_t)(kb * BK);
@@ -1542,21 +1560,18 @@ __global__ void __launch_bounds__(GemmLayout<MODE, FORM, NB>::threads, 1)
               // img, slots 0 .. pw - 1 of each; Q_b1 rows at those pixels,
               // X~ columns n0 .. n0 + 127 = (tap, 64 channels) pairs read at
               // the tap's offset (outside the input: zeros, the padding)
-              const int img = (int)(kb / g.cybi);
-              const int oy0 = (int)(kb - (int64_t)img * g.cybi) * g.crpb;
-              tma_load_4d(sa, &tmA, (int32_t)t.m0, 0, oy0, img, &full[s]);
-              tma_load_4d(sa + kTileBytes / 2, &tmA, (int32_t)t.m0 + 64, 0, oy0, img, &full[s]);
+              const int oy0 = cyb * g.crpb;
+              tma_load_4d(sa, &tmA, (int32_t)t.m0, 0, oy0, cimg, &full[s]);
+              tma_load_4d(sa + kTileBytes / 2, &tmA, (int32_t)t.m0 + 64, 0, oy0, cimg, &full[s]);
               for (int h = 0; h < 2; ++h) {
-                const int64_t d = t.n0 + 64 * h;
-                const int tap = (int)(d / g.cin), cg = (int)(d - (int64_t)tap * g.cin);
-                const int ky = tap / g.ckw, kx = tap - ky * g.ckw;
-                if (d < g.N)
-                  tma_load_4d(sb + h * (kTileBytes / 2), &tmB, cg, kx - g.cpad, oy0 + ky - g.cpad,
-                              img, &full[s]);
+                if (cval[h])
+                  tma_load_4d(sb + h * (kTileBytes / 2), &tmB, ccg[h], ckx[h] - g.cpad,
+                              oy0 + cky[h] - g.cpad, cimg, &full[s]);
                 else  // past the last tap: a box outside the tensor (zeros)
-                  tma_load_4d(sb + h * (kTileBytes / 2), &tmB, 0, 0, g.cih + g.coh + 8, img,
+                  tma_load_4d(sb + h * (kTileBytes / 2), &tmB, 0, 0, g.cih + g.coh + 8, cimg,
                               &full[s]);
               }
+              if (++cyb == g.cybi) { cyb = 0; ++cimg; }
               if (++s == nstages) { s = 0; ph ^= 1u; }
               continue;
             }
@@ -2587,59 +2602,104 @@ fqt_status linear_forward(const fqt_qtensor *qx, const fqt_qtensor *qw, float *H
 // Implicit im2col X~ (stride 1): per tap (ky, kx), the sum over the output
 // pixels whose input pixel (oy + ky - pad, ox + kx - pad) lies in the padding
 // of the A operand's carriers (C per row), for the padding correction of
-// k_reduce.  One CTA per (tap, image) visits only that image's padding
-// pixels for the tap: whole rows above / below, then the left / right
-// columns of the other rows; threads over (channel, pixel lane).
+// k_reduce.  Only output pixels in the top / bottom pad rows or the left /
+// right pad columns can read padding, and whether they do depends only on
+// which of those rows and columns they sit in: (2 pad + 1)^2 classes (the
+// inside class never).  A CTA (a run of images, a group of channels) adds
+// each border pixel's carriers into its class in shared memory (16-byte
+// loads, four in flight per thread), then adds each tap's share, the classes
+// whose row or column reads padding, into the sums.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ int pad_class(int y, int p, int n) {
+  return y < p ? y : (y >= n - p ? 2 * p - (n - 1 - y) : p);
+}
+
+// the one output row (column) of border class r, or -1 for the inside class
+__device__ __forceinline__ int pad_class_row(int r, int p, int n) {
+  return r < p ? r : (r > p ? n - 1 - (2 * p - r) : -1);
+}
+
 __global__ void __launch_bounds__(256) k_conv_padsum(const uint16_t *__restrict__ A16, int C,
-                                                     int64_t nimg, int h, int w, int kw,
-                                                     int pad, int oh, int ow, int taps,
-                                                     int32_t *pad_a) {
-  // a warp per (tap, image); lane = a pair of channels; 8 pixels in flight
-  const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (wid >= nimg * taps) return;
-  const int tap = (int)(wid % taps);
-  const int64_t img = wid / taps;
-  const int ky = tap / kw, kx = tap - ky * kw;
-  const int top = min(oh, max(0, pad - ky)), bot = min(oh - top, max(0, oh - (h + pad - ky)));
-  const int left = min(ow, max(0, pad - kx)), right = min(ow - left, max(0, ow - (w + pad - kx)));
-  const int rows_out = top + bot, cols_out = left + right;
-  const int full_px = rows_out * ow;  // the pixel counts of one image fit int
-  const int count = full_px + (oh - rows_out) * cols_out;
-  for (int c2 = lane; c2 < C / 2; c2 += 32) {
-    int acc0 = 0, acc1 = 0;
-    for (int t0 = 0; t0 < count; t0 += 8) {
-      uint32_t v[8];
+                                                     int ch_group, int64_t nimg, int imgs_per_cta,
+                                                     int h, int w, int kw, int pad, int oh,
+                                                     int ow, int taps, int32_t *pad_a) {
+  extern __shared__ int cls_s[];  // classes x ch_group
+  const int cc = 2 * pad + 1, ncls = cc * cc;
+  const int64_t img0 = (int64_t)blockIdx.x * imgs_per_cta;
+  const int nim = (int)min((int64_t)imgs_per_cta, nimg - img0);
+  const int ch0 = (int)blockIdx.y * ch_group, nch = min(ch_group, C - ch0);
+  for (int i = threadIdx.x; i < ncls * ch_group; i += blockDim.x) cls_s[i] = 0;
+  __syncthreads();
+  const int top = min(pad, oh), nbot = oh - max(top, oh - pad), full_rows = top + nbot;
+  const int left = min(pad, ow), nright = ow - max(left, ow - pad), side = left + nright;
+  const int full_px = full_rows * ow;
+  const int npx = full_px + (oh - full_rows) * side;  // the pixel counts of one image fit int
+  const int octs = nch / 8, per_img = npx * octs, items = nim * per_img;
+  const uint16_t *base = A16 + (img0 * oh) * (int64_t)ow * C + ch0;
+  for (int i0 = threadIdx.x; i0 < items; i0 += 4 * blockDim.x) {
+    uint4 v[4];
+    int k[4], oc[4];
 #pragma unroll
-      for (int b = 0; b < 8; ++b) {
-        const int t = t0 + b;
-        v[b] = 0u;
-        if (t < count) {
-          int oy, ox;
-          if (t < full_px) {
-            const int r = t / ow;
-            oy = r < top ? r : oh - bot + (r - top);
-            ox = t - r * ow;
-          } else {
-            const int u = t - full_px, r = u / cols_out, cc = u - r * cols_out;
-            oy = top + r;
-            ox = cc < left ? cc : ow - right + (cc - left);
-          }
-          const int64_t pp = (img * oh + oy) * (int64_t)ow + ox;
-          v[b] = __ldg(reinterpret_cast<const uint32_t *>(A16 + pp * C) + c2);
+    for (int u = 0; u < 4; ++u) {
+      const int it = i0 + u * (int)blockDim.x;
+      k[u] = -1;
+      oc[u] = 0;
+      v[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (it < items) {
+        const int im = it / per_img, rem = it - im * per_img, t = rem / octs;
+        oc[u] = rem - t * octs;
+        int oy, ox;
+        if (t < full_px) {
+          const int r = t / ow;
+          oy = r < top ? r : oh - nbot + (r - top);
+          ox = t - r * ow;
+        } else {
+          const int q = t - full_px, r = q / side, cq = q - r * side;
+          oy = top + r;
+          ox = cq < left ? cq : ow - nright + (cq - left);
         }
-      }
-#pragma unroll
-      for (int b = 0; b < 8; ++b) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&v[b]));
-        acc0 += (int)f.x;
-        acc1 += (int)f.y;
+        k[u] = pad_class(oy, pad, oh) * cc + pad_class(ox, pad, ow);
+        v[u] = __ldg(reinterpret_cast<const uint4 *>(
+            base + (((int64_t)im * oh + oy) * ow + ox) * C + oc[u] * 8));
       }
     }
-    if (acc0) atomicAdd(&pad_a[(2 * c2) * taps + tap], acc0);
-    if (acc1) atomicAdd(&pad_a[(2 * c2 + 1) * taps + tap], acc1);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (k[u] < 0) continue;
+      const uint32_t wds[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&wds[q]));
+        int *dst = &cls_s[k[u] * ch_group + oc[u] * 8 + 2 * q];
+        if ((int)f.x) atomicAdd(dst, (int)f.x);
+        if ((int)f.y) atomicAdd(dst + 1, (int)f.y);
+      }
+    }
   }
+  __syncthreads();
+  for (int i = threadIdx.x; i < nch * taps; i += blockDim.x) {
+    const int ch = i / taps, tap = i - ch * taps, ky = tap / kw, kx = tap - ky * kw;
+    int v = 0;
+    for (int ry = 0; ry < cc; ++ry) {
+      const int yr = pad_class_row(ry, pad, oh);
+      const bool row_out = yr >= 0 && (yr + ky - pad < 0 || yr + ky - pad >= h);
+      for (int rx = 0; rx < cc; ++rx) {
+        const int xr = pad_class_row(rx, pad, ow);
+        const bool col_out = xr >= 0 && (xr + kx - pad < 0 || xr + kx - pad >= w);
+        if (row_out || col_out) v += cls_s[(ry * cc + rx) * ch_group + ch];
+      }
+    }
+    if (v) atomicAdd(&pad_a[(int64_t)(ch0 + ch) * taps + tap], v);
+  }
+}
+
+// Channels per CTA of k_conv_padsum: a multiple of 8 whose class sums fit
+// 40 KB of shared memory (0: the padding is too wide, pad > 17).
+static int padsum_group(int C, int pad) {
+  const int ncls = (2 * pad + 1) * (2 * pad + 1);
+  int grp = (40960 / (ncls * 4)) / 8 * 8;
+  if (grp < 8) return 0;
+  return grp < C ? grp : C;
 }
 
 // ---------------------------------------------------------------------------
@@ -3319,6 +3379,7 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       // 64-channel boxes; rows of up to 64 pixels (the tile kernel) or of a
       // multiple of 32 (k_gradw)
       if (g[3] % 64 || (ow > 64 && ow % kWBK)) return FQT_EUNSUPPORTED;
+      if (padsum_group((int)C, g[6]) == 0) return FQT_EUNSUPPORTED;
     }
     // An implicit im2col operand with output rows of at most 64 pixels takes
     // the split-K tile kernel too: K blocks of 64 slots are rpb = 64 / pw
@@ -3366,12 +3427,24 @@ fqt_status linear_backward(const fqt_qtensor *q_b2, const fqt_qtensor *q_b1,
       const int oh = g[1] + 2 * g[6] - g[4] + 1, ow = g[2] + 2 * g[6] - g[5] + 1;
       cudaError_t e = cudaMemsetAsync(pad_a, 0, (size_t)C * taps * 4, st);
       if (e != cudaSuccess) return cuda_fail(e, "padding sums clear");
-      const int64_t warps = (int64_t)g[0] * taps;
-      k_conv_padsum<<<(int)((warps + 7) / 8), 256, 0, st>>>(
-          static_cast<const uint16_t *>(A16), (int)C, g[0], g[1], g[2], g[5], g[6], oh, ow, taps,
-          pad_a);
-      e = cudaGetLastError();
-      if (e != cudaSuccess) return cuda_fail(e, "padding sums launch");
+      const int grp = padsum_group((int)C, g[6]);
+      if (g[6] > 0) {  // without padding no tap reads any
+        // about 16 loads per thread: runs of images whose border pixels
+        // (bounded by the pad rows and columns) fill a CTA
+        const int pd = g[6];
+        const int64_t border = (int64_t)std::min(oh, 2 * pd) * ow +
+                               (int64_t)std::max(0, oh - 2 * pd) * std::min(ow, 2 * pd);
+        const int64_t items = std::max<int64_t>(1, border * (grp / 8));
+        const int64_t per = std::max<int64_t>(1, (256 * 16) / items);
+        const int ipc = (int)std::min<int64_t>(per, g[0]);
+        const dim3 grid((unsigned)((g[0] + ipc - 1) / ipc), (unsigned)((C + grp - 1) / grp));
+        const int ncls = (2 * pd + 1) * (2 * pd + 1);
+        k_conv_padsum<<<grid, 256, sizeof(int) * (size_t)ncls * grp, st>>>(
+            static_cast<const uint16_t *>(A16), (int)C, grp, g[0], ipc, g[1], g[2], g[5], pd, oh,
+            ow, taps, pad_a);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_fail(e, "padding sums launch");
+      }
     }
     if (Nr > 0 && w_ok) {
       fqt_status s = run_gradw(qx->codes_f16, static_cast<const uint16_t *>(A16), Nr, (int)C,

@@ -21,6 +21,7 @@
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <math.h>
+#include <algorithm>
 
 #include "fqt_common.cuh"
 #include "fqt_internal.h"
@@ -2223,84 +2224,122 @@ __global__ void __launch_bounds__(256) k_conv_colsum(const uint16_t *__restrict_
   }
 }
 
-// The same sums in one pass for kernels of up to 9 taps: one CTA per image,
-// every input pixel's carriers added into the taps that read it (registers),
-// then shared memory, then the column sums.
-constexpr int kConvMaxTaps = 9;
-constexpr int kConvSlices = 4;
+// The same sums in one pass when the border classes fit shared memory.  Tap
+// (ky, kx) reads the input rows [max(0, ky - pad), min(h, ky - pad + oh));
+// for stride 1 every tap reads all rows but some of the top and bottom m =
+// kh - 1 - pad ones (columns alike, mw = kw - 1 - pad).  So each input pixel
+// falls in one of (2m + 1)(2mw + 1) classes: its row is one of the m top
+// rows, one of the m bottom rows or inside, its column likewise.  A CTA takes
+// a contiguous range of the n h w pixels (across rows and images: the column
+// sums run over all images), adds the inside pixels' carriers in registers
+// (most of them) and the border pixels' into shared memory by class, and
+// then adds each tap's share, the classes whose row and column the tap
+// reads, into the column sums.  Reads are 16 bytes per thread, eight in
+// flight.
+constexpr int kConvMaxClasses = 25;
+constexpr int kConvUnroll = 8;
+
+__device__ __forceinline__ int conv_class(int y, int m, int h) {
+  return y < m ? y : (y >= h - m ? 2 * m - (h - 1 - y) : m);
+}
+
+// the one input row (column) of border class r, or -1 for the inside class
+__device__ __forceinline__ int conv_class_row(int r, int m, int h) {
+  return r < m ? r : (r > m ? h - 1 - (2 * m - r) : -1);
+}
 
 __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict__ f16, int h,
                                                       int w, int c, int kh, int kw, int pad,
-                                                      int oh, int ow, int64_t nimg,
-                                                      int centre, int32_t *col_sum) {
-  extern __shared__ int acc_s[];  // taps x c
-  const int taps = kh * kw;
-  // CTA = (image, slice of kConvSlices input rows)
-  const int64_t img = blockIdx.x / kConvSlices;
-  const int slice = (int)(blockIdx.x % kConvSlices);
-  const int ys = (h * slice) / kConvSlices, ye = (h * (slice + 1)) / kConvSlices;
-  for (int i = threadIdx.x; i < taps * c; i += blockDim.x) acc_s[i] = 0;
+                                                      int oh, int ow, int64_t nimg, int centre,
+                                                      int64_t px_per_cta, int32_t *col_sum) {
+  extern __shared__ int cls_s[];  // classes x c
+  const int m = max(0, kh - 1 - pad), mw = max(0, kw - 1 - pad);
+  const int cc = 2 * mw + 1, ncls = (2 * m + 1) * cc, inner = m * cc + mw;
+  const int64_t npx = nimg * h * (int64_t)w;
+  const int64_t p0 = (int64_t)blockIdx.x * px_per_cta;
+  const int64_t p1 = min(npx, p0 + px_per_cta);
+  for (int i = threadIdx.x; i < ncls * c; i += blockDim.x) cls_s[i] = 0;
   __syncthreads();
-  int tky[kConvMaxTaps], tkx[kConvMaxTaps];
-#pragma unroll
-  for (int t = 0; t < kConvMaxTaps; ++t) {
-    tky[t] = t < taps ? t / kw : 0;
-    tkx[t] = t < taps ? t - (t / kw) * kw : 0;
-  }
   const int octs = c / 8;
   const int lanes = blockDim.x >= octs ? blockDim.x / octs : 1;
-  for (int oc = threadIdx.x % octs; oc < octs; oc += blockDim.x) {
-    const int pl = blockDim.x >= octs ? (int)threadIdx.x / octs : 0;
-    if (pl >= lanes) continue;
-    int a[kConvMaxTaps][8];
+  const int pl = blockDim.x >= octs ? (int)threadIdx.x / octs : 0;
+  for (int oc = threadIdx.x % octs; oc < octs && pl < lanes; oc += blockDim.x) {
+    int acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    int64_t p = p0 + pl;
+    int y = (int)((p / w) % h), x = (int)(p % w);
+    while (p < p1) {
+      uint4 v[kConvUnroll];
+      int py[kConvUnroll], px[kConvUnroll];
 #pragma unroll
-    for (int t = 0; t < kConvMaxTaps; ++t)
-#pragma unroll
-      for (int j = 0; j < 8; ++j) a[t][j] = 0;
-    for (int p = ys * w + pl; p < ye * w; p += lanes) {
-      const int y = p / w, x = p - y * w;
-      const uint4 v = __ldg(reinterpret_cast<const uint4 *>(
-          f16 + ((img * h + y) * (int64_t)w + x) * c + oc * 8));
-      const uint32_t wds[4] = {v.x, v.y, v.z, v.w};
-      int e[8];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&wds[q]));
-        e[2 * q] = (int)f.x;
-        e[2 * q + 1] = (int)f.y;
+      for (int u = 0; u < kConvUnroll; ++u) {
+        py[u] = y;
+        px[u] = x;
+        v[u] = make_uint4(0u, 0u, 0u, 0u);
+        if (p < p1)
+          v[u] = __ldg(reinterpret_cast<const uint4 *>(f16 + p * c + oc * 8));
+        else
+          py[u] = -1;
+        p += lanes;
+        x += lanes;
+        while (x >= w) {
+          x -= w;
+          if (++y == h) y = 0;
+        }
       }
 #pragma unroll
-      for (int t = 0; t < kConvMaxTaps; ++t) {
-        const int oy = y - tky[t] + pad, ox = x - tkx[t] + pad;
-        if (t < taps && oy >= 0 && oy < oh && ox >= 0 && ox < ow) {
+      for (int u = 0; u < kConvUnroll; ++u) {
+        if (py[u] < 0) continue;
+        const uint32_t wds[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+        int e[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j) a[t][j] += e[j];
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&wds[q]));
+          e[2 * q] = (int)f.x;
+          e[2 * q + 1] = (int)f.y;
+        }
+        const int k = conv_class(py[u], m, h) * cc + conv_class(px[u], mw, w);
+        if (k == inner) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) acc[j] += e[j];
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (e[j]) atomicAdd(&cls_s[k * c + oc * 8 + j], e[j]);
         }
       }
     }
     // lanes of a warp that share a channel oct add up by shuffles first
     const bool shfl_ok = octs <= 32 && (32 % octs) == 0;
 #pragma unroll
-    for (int t = 0; t < kConvMaxTaps; ++t)
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        int v = a[t][j];
-        if (shfl_ok) {
-          for (int off = octs; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-          if ((int)(threadIdx.x & 31) >= octs) v = 0;
-        }
-        if (t < taps && v) atomicAdd(&acc_s[t * c + oc * 8 + j], v);
+    for (int j = 0; j < 8; ++j) {
+      int v = acc[j];
+      if (shfl_ok) {
+        for (int off = octs; off < 32; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+        if ((int)(threadIdx.x & 31) >= octs) v = 0;
       }
+      if (v) atomicAdd(&cls_s[inner * c + oc * 8 + j], v);
+    }
   }
   __syncthreads();
+  const int taps = kh * kw;
   const int zc = col_sum[(int64_t)taps * c];
   const int64_t rows = nimg * oh * ow;
   for (int i = threadIdx.x; i < taps * c; i += blockDim.x) {
-    int v = acc_s[i];
-    if (img == 0 && slice == 0) {
-      const int t = i / c, ky = t / kw, kx = t - ky * kw;
-      const int ry = min(h, ky - pad + oh) - max(0, ky - pad);
-      const int rx = min(w, kx - pad + ow) - max(0, kx - pad);
+    const int t = i / c, ch = i - t * c, ky = t / kw, kx = t - ky * kw;
+    const int y0 = max(0, ky - pad), y1 = min(h, ky - pad + oh);
+    const int x0 = max(0, kx - pad), x1 = min(w, kx - pad + ow);
+    int v = 0;
+    for (int ry = 0; ry < 2 * m + 1; ++ry) {
+      const int yr = conv_class_row(ry, m, h);
+      if (yr >= 0 && (yr < y0 || yr >= y1)) continue;
+      for (int rx = 0; rx < cc; ++rx) {
+        const int xr = conv_class_row(rx, mw, w);
+        if (xr >= 0 && (xr < x0 || xr >= x1)) continue;
+        v += cls_s[(ry * cc + rx) * c + ch];
+      }
+    }
+    if (blockIdx.x == 0) {
+      const int ry = y1 - y0, rx = x1 - x0;
       const int64_t nvalid = nimg * (int64_t)(ry > 0 && rx > 0 ? ry * rx : 0);
       v += (int)(nvalid * centre + (rows - nvalid) * (int64_t)zc);
     }
@@ -2312,10 +2351,18 @@ fqt_status launch_conv_colsum(const uint16_t *f16, int64_t n, int h, int w, int 
                               int kw, int pad, int bits, int32_t *col_sum, cudaStream_t st) {
   const int oh = h + 2 * pad - kh + 1, ow = w + 2 * pad - kw + 1;
   if (n <= 0) return FQT_OK;
-  if (kh * kw <= kConvMaxTaps && (size_t)kh * kw * c * sizeof(int) <= 48 * 1024 &&
-      n * kConvSlices <= 0x7fffffff) {
-    k_conv_colsum1<<<(int)(n * kConvSlices), 256, sizeof(int) * (size_t)kh * kw * c, st>>>(
-        f16, h, w, c, kh, kw, pad, oh, ow, n, 1 << (bits - 1), col_sum);
+  const int m = std::max(0, kh - 1 - pad), mw = std::max(0, kw - 1 - pad);
+  const int ncls = (2 * m + 1) * (2 * mw + 1);
+  if (ncls <= kConvMaxClasses && h > 2 * m && w > 2 * mw &&
+      (size_t)ncls * c * sizeof(int) <= 48 * 1024) {
+    // about 32 loads of 16 bytes per thread, at most three CTAs per SM (each
+    // CTA adds taps x c sums into the column sums once)
+    const int64_t npx = n * h * (int64_t)w, octs = c / 8;
+    const int64_t want = (npx * octs + 256 * 32 - 1) / (256 * 32);
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(want, 3 * device_sm_count()));
+    const int64_t per = (npx + grid - 1) / grid;
+    k_conv_colsum1<<<(int)((npx + per - 1) / per), 256, sizeof(int) * (size_t)ncls * c, st>>>(
+        f16, h, w, c, kh, kw, pad, oh, ow, n, 1 << (bits - 1), per, col_sum);
     return cuda_fail(cudaGetLastError(), "conv column sums launch");
   }
   const int64_t grid = n * kh * kw;

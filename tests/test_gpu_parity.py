@@ -834,20 +834,26 @@ def _conv_codes_as_im2col(q, x_shape, kh, kw, pad):
     return cols.reshape(n * oh * ow, kh * kw * c), zc
 
 
-@pytest.mark.parametrize("n,h,w,c,pad,dtype", [(2, 32, 32, 64, 1, "f32"), (1, 32, 32, 128, 1, "bf16"),
-                                               (3, 8, 12, 16, 1, "f32"), (2, 9, 9, 64, 0, "f32")])
-def test_conv_quantizer_equals_the_im2col_quantizer(n, h, w, c, pad, dtype):
-    g = wl.rng(n * h + c + pad)
+@pytest.mark.parametrize("n,h,w,c,k,pad,dtype", [
+    (2, 32, 32, 64, 3, 1, "f32"), (1, 32, 32, 128, 3, 1, "bf16"), (3, 8, 12, 16, 3, 1, "f32"),
+    (2, 9, 9, 64, 3, 0, "f32"), (3, 7, 7, 512, 3, 1, "f32"), (2, 11, 10, 64, 5, 2, "f32"),
+    (2, 6, 7, 64, 3, 2, "f32"), (2, 5, 5, 32, 1, 0, "f32"), (1, 9, 9, 512, 3, 0, "f32")])
+def test_conv_quantizer_equals_the_im2col_quantizer(n, h, w, c, k, pad, dtype):
+    """Codes, scale and im2col column sums of the implicit Q_f against the
+    oracle's quantizer on the explicit im2col matrix; the kernel sizes and
+    paddings span the column sums' border classes (pad < k - 1, = k - 1,
+    > k - 1) and the per-tap fallback (9 x 9 classes of 512 channels)."""
+    g = wl.rng(n * h + c + pad + 7 * k)
     x = g.uniform(-1, 1, (n, h, w, c)).astype(np.float32)
     x[0, 0, 0, :4] = 3.0  # the range is not symmetric
     if dtype == "bf16":
         x = wl.to_bf16_values(x)
-    xi = wl.im2col_nhwc(x, 3, 3, 1, pad)
+    xi = wl.im2col_nhwc(x, k, k, 1, pad)
     ref = orc.quantize_fwd(xi, 8)
-    q = fqt.quantize_act_conv(to_dev(x, dtype), 3, 3, pad, 8)
+    q = fqt.quantize_act_conv(to_dev(x, dtype), k, k, pad, 8)
     torch.cuda.synchronize()
     assert q.shape == xi.shape
-    got, zc = _conv_codes_as_im2col(q, x.shape, 3, 3, pad)
+    got, zc = _conv_codes_as_im2col(q, x.shape, k, k, pad)
     assert np.array_equal(got, ref["codes"].astype(np.int64))
     assert np.array_equal(q.inv_s.cpu().numpy(), ref["inv_s"])
     assert np.array_equal(q.zero.cpu().numpy(), ref["zero"])
@@ -882,26 +888,28 @@ def test_conv_grad_w_equals_the_explicit_path(batch):
     assert grad_rel_err(gwc[:, cols], ref) <= GRAD_TOL
 
 
-@pytest.mark.parametrize("n,h,w,cin,cout", [(2, 56, 56, 64, 64), (3, 28, 28, 128, 128),
-                                             (4, 14, 14, 64, 256), (5, 7, 7, 128, 64),
-                                             (2, 9, 11, 64, 128), (1, 64, 64, 64, 64),
-                                             (2, 12, 96, 64, 64)])
-def test_conv_grad_w_rows_in_blocks_equal_the_explicit_path(n, h, w, cin, cout):
+@pytest.mark.parametrize("n,h,w,cin,cout,k,pad", [
+    (2, 56, 56, 64, 64, 3, 1), (3, 28, 28, 128, 128, 3, 1), (4, 14, 14, 64, 256, 3, 1),
+    (5, 7, 7, 128, 64, 3, 1), (2, 9, 11, 64, 128, 3, 1), (1, 64, 64, 64, 64, 3, 1),
+    (2, 12, 96, 64, 64, 3, 1), (2, 14, 13, 64, 64, 5, 2), (2, 10, 10, 64, 512, 3, 2),
+    (3, 9, 9, 64, 128, 1, 0), (2, 7, 7, 512, 512, 3, 1)])
+def test_conv_grad_w_rows_in_blocks_equal_the_explicit_path(n, h, w, cin, cout, k, pad):
     """The implicit im2col X~ in the split-K tile kernel at the output-row
     widths of ResNet-50's 3 x 3 layers (56, 28, 14, 7) and ragged ones: K
     blocks of whole output rows padded to a power of two (64 / 32 / 16 / 8
     slots, rows past oh and slots past ow zero), bit for bit the explicit
-    im2col grad_W; ow = 96 takes the one-range-per-CTA kernel."""
-    g = wl.rng(n * h * w + cin + cout)
+    im2col grad_W; ow = 96 takes the one-range-per-CTA kernel.  5 x 5 / pad 2,
+    pad 2 on 3 x 3 and 1 x 1 / pad 0 vary the padding correction's classes."""
+    g = wl.rng(n * h * w + cin + cout + 11 * k + pad)
     x = g.uniform(-1, 1, (n, h, w, cin)).astype(np.float32)
-    xi = wl.im2col_nhwc(x, 3, 3, 1, 1)
+    xi = wl.im2col_nhwc(x, k, k, 1, pad)
     N, D = xi.shape
     dH = g.standard_normal((N, cout)).astype(np.float32)
     dH[g.random(N) < 0.02] *= 50.0
     q2, q1 = fqt.quantize_grad(to_dev(dH), orc.BHQ, 5, 16, seed=9)
     ws = fqt.Workspace(N, cout, D)
     qx = fqt.quantize_act(to_dev(xi), 8)
-    qc = fqt.quantize_act_conv(to_dev(x), 3, 3, 1, 8)
+    qc = fqt.quantize_act_conv(to_dev(x), k, k, pad, 8)
     _, gw = fqt.linear_backward(q2, q1, qx, None, grad_x=False, ws=ws)
     _, gwc = fqt.linear_backward(q2, q1, qc, None, grad_x=False, ws=ws)
     assert fqt.sync_status(ws) == 0
