@@ -143,6 +143,19 @@ __device__ __forceinline__ void store_carriers8(uint16_t *dst, const uint32_t (&
   *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+// The other way, for sums of carriers: a word of two fp16 carriers v
+// (integers, |v| <= 512) as the two 16-bit lanes v + 512.  v + 1536 lies in
+// [1024, 2048), where fp16 steps by 1, so the packed addition is exact and
+// each half's bits are 0x6400 + v + 512.  kLaneAdds such words add up
+// without a carry between the lanes (64 x 1023 < 2^16).
+constexpr int kLaneAdds = 64;
+
+__device__ __forceinline__ uint32_t carrier_lanes(uint32_t wd) {
+  const __half2 bias = __half2half2(__ushort_as_half((unsigned short)0x6600u));
+  const __half2 s = __hadd2(*reinterpret_cast<const __half2 *>(&wd), bias);
+  return *reinterpret_cast<const uint32_t *>(&s) - 0x64006400u;
+}
+
 // ---------------------------------------------------------------------------
 // PTX wrappers: mbarrier, async-proxy fences, bulk / tensor copies.
 // ---------------------------------------------------------------------------

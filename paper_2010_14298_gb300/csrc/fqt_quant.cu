@@ -2234,10 +2234,10 @@ __global__ void __launch_bounds__(256) k_conv_colsum(const uint16_t *__restrict_
 // sums run over all images), adds the inside pixels' carriers in registers
 // (most of them) and the border pixels' into shared memory by class, and
 // then adds each tap's share, the classes whose row and column the tap
-// reads, into the column sums.  Reads are 16 bytes per thread, eight in
+// reads, into the column sums.  Reads are 16 bytes per thread, six in
 // flight.
 constexpr int kConvMaxClasses = 25;
-constexpr int kConvUnroll = 8;
+constexpr int kConvUnroll = 6;
 
 __device__ __forceinline__ int conv_class(int y, int m, int h) {
   return y < m ? y : (y >= h - m ? 2 * m - (h - 1 - y) : m);
@@ -2248,7 +2248,7 @@ __device__ __forceinline__ int conv_class_row(int r, int m, int h) {
   return r < m ? r : (r > m ? h - 1 - (2 * m - r) : -1);
 }
 
-__global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict__ f16, int h,
+__global__ void __launch_bounds__(256, 3) k_conv_colsum1(const uint16_t *__restrict__ f16, int h,
                                                       int w, int c, int kh, int kw, int pad,
                                                       int oh, int ow, int64_t nimg, int centre,
                                                       int64_t px_per_cta, int32_t *col_sum) {
@@ -2265,6 +2265,17 @@ __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict
   const int pl = blockDim.x >= octs ? (int)threadIdx.x / octs : 0;
   for (int oc = threadIdx.x % octs; oc < octs && pl < lanes; oc += blockDim.x) {
     int acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    uint32_t pk[4] = {0u, 0u, 0u, 0u};  // inside pixels, two lanes v + 512 a word
+    int npk = 0;
+    auto flush = [&]() {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        acc[2 * q] += (int)(pk[q] & 0xFFFFu) - 512 * npk;
+        acc[2 * q + 1] += (int)(pk[q] >> 16) - 512 * npk;
+        pk[q] = 0u;
+      }
+      npk = 0;
+    };
     int64_t p = p0 + pl;
     int y = (int)((p / w) % h), x = (int)(p % w);
     while (p < p1) {
@@ -2289,25 +2300,24 @@ __global__ void __launch_bounds__(256) k_conv_colsum1(const uint16_t *__restrict
 #pragma unroll
       for (int u = 0; u < kConvUnroll; ++u) {
         if (py[u] < 0) continue;
-        const uint32_t wds[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-        int e[8];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&wds[q]));
-          e[2 * q] = (int)f.x;
-          e[2 * q + 1] = (int)f.y;
-        }
+        const uint32_t t[4] = {carrier_lanes(v[u].x), carrier_lanes(v[u].y),
+                               carrier_lanes(v[u].z), carrier_lanes(v[u].w)};
         const int k = conv_class(py[u], m, h) * cc + conv_class(px[u], mw, w);
         if (k == inner) {
 #pragma unroll
-          for (int j = 0; j < 8; ++j) acc[j] += e[j];
+          for (int q = 0; q < 4; ++q) pk[q] += t[q];
+          if (++npk == kLaneAdds) flush();
         } else {
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (e[j]) atomicAdd(&cls_s[k * c + oc * 8 + j], e[j]);
+          for (int q = 0; q < 4; ++q) {
+            const int lo = (int)(t[q] & 0xFFFFu) - 512, hi = (int)(t[q] >> 16) - 512;
+            if (lo) atomicAdd(&cls_s[k * c + oc * 8 + 2 * q], lo);
+            if (hi) atomicAdd(&cls_s[k * c + oc * 8 + 2 * q + 1], hi);
+          }
         }
       }
     }
+    flush();
     // lanes of a warp that share a channel oct add up by shuffles first
     const bool shfl_ok = octs <= 32 && (32 % octs) == 0;
 #pragma unroll
