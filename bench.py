@@ -214,13 +214,13 @@ def launches(C: int, kind: int = KIND, block: int = BLOCK, implicit: bool = Fals
     """Kernels each call launches (fixed by the library's dispatch): Q_f and
     Q_theta are a range pass and a code pass; the fixed-block BHQ quantizer on
     the widths of its two-pass form is a statistics pass, a code pass and the
-    grad_X offsets, on other widths a range pass and one fused pass; grad_X
-    is one contraction, grad_W the split-K contraction and its reduction; an
+    grad_X offsets, on other widths a range pass, one fused pass and the
+    offsets (PTQ and PSQ: a range pass and one fused pass); grad_X is one
+    contraction, grad_W the split-K contraction and its reduction; an
     implicit im2col X~ adds the column sums to Q_f and the padding sums to
     grad_W."""
-    two_pass = kind == KIND and block in (4, 8, 16) and C in (64, 128, 256, 512, 1024, 2048, 4096)
     return {"quantize_act": 3 if implicit else 2, "quantize_weight": 2,
-            "quantize_grad": 3 if two_pass else 2,
+            "quantize_grad": 3 if kind == KIND else 2,
             "grad_x": 1, "grad_w": 3 if implicit else 2}
 
 
